@@ -1,0 +1,305 @@
+"""Plain CPU oracle for the OffQ W4A4 linear path (test infrastructure).
+
+This is test infrastructure, not the product. Only ``tests/``,
+``__graft_entry__.smoke()`` and the CPU-baseline leg of ``bench.py`` may import
+it. It shares no code with the CUDA path: it builds the Hadamard matrix
+explicitly, rotates with a dense float64 matmul, takes offsets as plain block
+means, and computes the integer GEMM exactly.
+
+Every function follows the paper (OffQ, arxiv 2606.07116) and cites the passage
+it implements. Where the paper is silent, it uses these readings:
+
+* Rounding of Eq. 1's round operator: round half to even (``numpy.rint``).
+* Residual quantizer: symmetric signed 4-bit with one scale per token,
+  s = max|R| / 7, codes clamped to [-7, 7] (the sign-magnitude 4-bit range),
+  s = 0 and all codes 0 for an all-zero residual row.
+* Offset of block b: the mean of the rotated block. For the Sylvester Hadamard
+  it equals the block's first channel divided by sqrt(g) (Sec. 3.2, Eq. 4-5).
+* Online rotation: the Sylvester Hadamard in natural order (first row all ones,
+  Sec. 3.2), applied block-diagonally with block size g (group-wise offsetting,
+  Sec. 3.2 "Group-Wise Offsetting"), normalised by 1/sqrt(g).
+* Weights: per-output-channel symmetric round-to-nearest (Sec. 4 settings; GPTQ
+  needs calibration data), after the same block rotation so that
+  W x = (W H)(H x) for the orthonormal, symmetric block Hadamard H.
+* Offset correction table: S[b, n] = s_w[n] * sum_{k in b} Qw[n, k], the
+  quantized weights' block row sums, so the epilogue reproduces W_hat @ X_hat
+  exactly (Sec. 3.2, Eq. 5: the offset is a constant added to every channel of
+  a block, so it leaves through the weight row sums).
+* Packing: two 4-bit sign-magnitude codes per byte, the even channel in the low
+  nibble; a code is (sign << 3) | |q|.
+
+Decisions that turn floating point into integers (the codes) are taken here in
+float64.
+"""
+
+from __future__ import annotations
+
+import math
+from typing import Dict, Optional
+
+import numpy as np
+
+QMAX = 7  # largest code magnitude of the symmetric 4-bit grid (Eq. 1 with b = 4, z absent)
+
+
+# ---------------------------------------------------------------------------
+# Hadamard matrix and the online rotation  (Sec. 3.2, Eq. 4)
+# ---------------------------------------------------------------------------
+
+def sylvester_hadamard(g: int) -> np.ndarray:
+    """Sylvester Hadamard H_g (int64, entries +-1), H_1 = [1], H_2m = [[H, H], [H, -H]].
+
+    The paper needs an orthogonal matrix with +-1 entries whose first row is all
+    ones (Sec. 3.2, "Offsetting Technique"); the Sylvester recursion gives one
+    for every power of two.
+    """
+    if g < 1 or (g & (g - 1)) != 0:
+        raise ValueError("g must be a power of two")
+    h = np.ones((1, 1), dtype=np.int64)
+    while h.shape[0] < g:
+        h = np.block([[h, h], [h, -h]])
+    return h
+
+
+def rotate_blocks(x: np.ndarray, g: int) -> np.ndarray:
+    """Y = X @ blockdiag(H_g, ..., H_g) / sqrt(g) for token rows X [T, K] (Eq. 4, group-wise).
+
+    Written as a dense float64 matmul per block of g channels: the definition,
+    not a butterfly.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    T, K = x.shape
+    if K % g != 0:
+        raise ValueError("g must divide K")
+    H = sylvester_hadamard(g).astype(np.float64)
+    y = np.empty_like(x)
+    for b in range(K // g):
+        sl = slice(b * g, (b + 1) * g)
+        y[:, sl] = x[:, sl] @ H / math.sqrt(g)
+    return y
+
+
+def block_offsets(y: np.ndarray, g: int) -> np.ndarray:
+    """o[t, b] = mean of Y[t, b*g:(b+1)*g]: the constant each block carries (Sec. 3.2, Eq. 5).
+
+    Each block sum is the correctly rounded sum (``math.fsum``), so the mean is
+    exact whenever it is representable.
+    """
+    y = np.asarray(y, dtype=np.float64)
+    T, K = y.shape
+    blocks = y.reshape(T * (K // g), g)
+    sums = np.fromiter((math.fsum(row) for row in blocks), dtype=np.float64, count=blocks.shape[0])
+    return (sums / g).reshape(T, K // g)
+
+
+def subtract_offsets(y: np.ndarray, o: np.ndarray, g: int) -> np.ndarray:
+    """Residual R = Y - o broadcast over each block (the part left after offsetting, Eq. 5)."""
+    T, K = y.shape
+    return (y.reshape(T, K // g, g) - o[:, :, None]).reshape(T, K)
+
+
+# ---------------------------------------------------------------------------
+# Uniform quantizer  (Sec. 3, Eq. 1)
+# ---------------------------------------------------------------------------
+
+def quantize_rows(r: np.ndarray):
+    """Symmetric per-row 4-bit quantization of Eq. 1 (no zero-point).
+
+    s[t] = max_k |r[t, k]| / 7;  q = clamp(round_half_even(r / s), -7, 7);
+    a row of zeros gets s = 0 and q = 0. Returns (q int64, s float64).
+    """
+    r = np.asarray(r, dtype=np.float64)
+    amax = np.max(np.abs(r), axis=1) if r.shape[1] > 0 else np.zeros(r.shape[0])
+    s = amax / QMAX
+    q = np.zeros(r.shape, dtype=np.int64)
+    nz = s > 0
+    q[nz] = np.clip(np.rint(r[nz] / s[nz, None]), -QMAX, QMAX).astype(np.int64)
+    return q, s
+
+
+def pack_codes(q: np.ndarray) -> np.ndarray:
+    """Pack signed codes [.., K] into bytes [.., K/2]: sign-magnitude nibbles, even channel low.
+
+    A nibble is (sign << 3) | |q| with sign = 1 for q < 0.
+    """
+    q = np.asarray(q, dtype=np.int64)
+    if q.shape[-1] % 2:
+        raise ValueError("K must be even")
+    if np.any(np.abs(q) > QMAX):
+        raise ValueError("code out of range")
+    nib = (np.abs(q) | np.where(q < 0, 8, 0)).astype(np.uint8)
+    return (nib[..., 0::2] | (nib[..., 1::2] << 4)).astype(np.uint8)
+
+
+def unpack_codes(packed: np.ndarray) -> np.ndarray:
+    """Inverse of :func:`pack_codes`: bytes [.., K/2] -> int64 codes [.., K]."""
+    p = np.asarray(packed, dtype=np.uint8)
+    lo = p & 0xF
+    hi = p >> 4
+    out = np.empty(p.shape[:-1] + (2 * p.shape[-1],), dtype=np.int64)
+    for dst, nib in ((out[..., 0::2], lo), (out[..., 1::2], hi)):
+        mag = (nib & 7).astype(np.int64)
+        dst[...] = np.where(nib & 8, -mag, mag)
+    return out
+
+
+# ---------------------------------------------------------------------------
+# Online activation path  (Sec. 3.2 offsetting + Sec. 3 Eq. 1)
+# ---------------------------------------------------------------------------
+
+def quantize_act(x: np.ndarray, g: int, rotate: bool = True, offset: bool = True) -> Dict[str, np.ndarray]:
+    """Rotate -> offset -> quantize -> pack one batch of token rows X [T, K].
+
+    Steps, in the paper's order:
+      1. Y = X H / sqrt(g) block-wise when ``rotate`` (Eq. 4); else Y = X.
+      2. o[t, b] = mean of block b of Y when ``offset`` (Eq. 5); else o = 0.
+      3. R = Y - o.
+      4. s[t] = max|R[t]| / 7, q = clamp(rne(R / s), -7, 7) (Eq. 1, symmetric).
+      5. Two codes per byte.
+
+    The product X H and its block means are formed before the 1/sqrt(g)
+    normalisation. For bf16/fp32 inputs of moderate range that keeps them exact
+    in float64, so a block holding only its leading (outlier) channel leaves a
+    residual of exactly zero, as the paper states (Eq. 5). R / s equals
+    7 R_u / max|R_u| for the unnormalised residual R_u = sqrt(g) R, so the codes
+    are taken from R_u directly.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    T, K = x.shape
+    if K % g != 0:
+        raise ValueError("g must divide K")
+    G = K // g
+    if rotate:
+        H = sylvester_hadamard(g).astype(np.float64)
+        yu = np.empty_like(x)
+        for b in range(G):
+            sl = slice(b * g, (b + 1) * g)
+            yu[:, sl] = x[:, sl] @ H
+        norm = math.sqrt(g)
+    else:
+        yu = x.copy()
+        norm = 1.0
+    ou = block_offsets(yu, g) if offset else np.zeros((T, G))
+    ru = subtract_offsets(yu, ou, g)
+    q, su = quantize_rows(ru)
+    return {"y": yu / norm, "offset": ou / norm, "residual": ru / norm, "q": q,
+            "scale": su / norm, "codes": pack_codes(q)}
+
+
+def dequantize_act(q: np.ndarray, s: np.ndarray, o: np.ndarray, g: int) -> np.ndarray:
+    """X_hat[t, k] = s[t] * q[t, k] + o[t, k // g]: what the 4-bit activation stands for."""
+    T, K = q.shape
+    xh = q.astype(np.float64) * s[:, None]
+    return (xh.reshape(T, K // g, g) + o[:, :, None]).reshape(T, K)
+
+
+# ---------------------------------------------------------------------------
+# Weights (offline)  (Sec. 3.3 Step 2 fusion of the rotation, Sec. 4 settings)
+# ---------------------------------------------------------------------------
+
+def prepare_weight(w: np.ndarray, g: int, rotate: bool = True) -> Dict[str, np.ndarray]:
+    """Per-output-channel symmetric 4-bit weights for y = W x with W [N, K].
+
+    W_eff = W blockdiag(H_g) / sqrt(g) when the input takes the online rotation
+    (Sec. 3.3 Step 2 (4): the inverse rotation is fused into the weight, and the
+    block Hadamard is symmetric and orthonormal); s_w[n] = max|W_eff[n]| / 7;
+    Qw = clamp(rne(W_eff / s_w), -7, 7); S[b, n] = s_w[n] * sum_{k in block b} Qw[n, k].
+    """
+    w = np.asarray(w, dtype=np.float64)
+    N, K = w.shape
+    # Same rotate-then-quantize steps as the activations, with no offset.
+    res = quantize_act(w, g, rotate=rotate, offset=False)
+    w_eff, qw, sw = res["y"], res["q"], res["scale"]
+    G = K // g
+    rowsum = qw.reshape(N, G, g).sum(axis=2)          # int64 [N, G]
+    S = (rowsum.astype(np.float64) * sw[:, None]).T    # float64 [G, N]
+    return {"w_eff": w_eff, "q": qw, "scale": sw, "offsum": S, "rowsum": rowsum.T,
+            "codes": pack_codes(qw)}
+
+
+# ---------------------------------------------------------------------------
+# W4A4 GEMM and epilogue
+# ---------------------------------------------------------------------------
+
+def int_gemm(qa: np.ndarray, qw: np.ndarray) -> np.ndarray:
+    """acc[t, n] = sum_k qa[t, k] * qw[n, k] exactly, as int64.
+
+    A float64 BLAS product on integer-valued arrays is exact here: every partial
+    sum is an integer of magnitude <= 49 * K < 2**53.
+    """
+    qa = np.asarray(qa, dtype=np.int64)
+    qw = np.asarray(qw, dtype=np.int64)
+    if 49 * qa.shape[1] >= 2 ** 53:
+        raise ValueError("K too large for an exact float64 product")
+    acc = qa.astype(np.float64) @ qw.astype(np.float64).T
+    return np.rint(acc).astype(np.int64)
+
+
+def int_gemm_loops(qa: np.ndarray, qw: np.ndarray) -> np.ndarray:
+    """Triple-loop int64 GEMM for tiny shapes (a cross-check of :func:`int_gemm`)."""
+    T, K = qa.shape
+    N = qw.shape[0]
+    acc = np.zeros((T, N), dtype=np.int64)
+    for t in range(T):
+        for n in range(N):
+            a = 0
+            for k in range(K):
+                a += int(qa[t, k]) * int(qw[n, k])
+            acc[t, n] = a
+    return acc
+
+
+def epilogue(acc: np.ndarray, s_a: np.ndarray, o: np.ndarray, s_w: np.ndarray,
+             S: np.ndarray) -> np.ndarray:
+    """y[t, n] = s_a[t] * s_w[n] * acc[t, n] + sum_b o[t, b] * S[b, n], in float64.
+
+    The second term is the offset's rank-G correction: each block's constant
+    offset meets the block row sums of the dequantized weights.
+    """
+    return (np.asarray(s_a, np.float64)[:, None] * np.asarray(s_w, np.float64)[None, :]
+            * np.asarray(acc, np.float64)
+            + np.asarray(o, np.float64) @ np.asarray(S, np.float64))
+
+
+def w4a4_linear(qa: np.ndarray, s_a: np.ndarray, o: np.ndarray, qw: np.ndarray,
+                s_w: np.ndarray, S: np.ndarray) -> Dict[str, np.ndarray]:
+    """Integer GEMM of the codes plus the dequant + offset epilogue."""
+    acc = int_gemm(qa, qw)
+    return {"acc": acc, "y": epilogue(acc, s_a, o, s_w, S)}
+
+
+def linear_reference(x: np.ndarray, w: np.ndarray) -> np.ndarray:
+    """Unquantized y = X W^T in float64 (for the quality report, not parity)."""
+    return np.asarray(x, np.float64) @ np.asarray(w, np.float64).T
+
+
+# ---------------------------------------------------------------------------
+# KV-cache 4-bit quantization  (Sec. 3.3 Step 2 (2)-(3): per-head H3, KV group = head dim)
+# ---------------------------------------------------------------------------
+
+def kv4_quantize(kv: np.ndarray, rotate: bool = True, offset: bool = True) -> Dict[str, np.ndarray]:
+    """Per-(token, head) rotate/offset/quantize of KV vectors [T, H, hd] with g = hd.
+
+    The head is one block: the per-head online Hadamard H3 of the keys
+    (Sec. 3.3 Step 2 (3)), one offset and one scale per (token, head).
+    """
+    kv = np.asarray(kv, dtype=np.float64)
+    T, H, hd = kv.shape
+    res = quantize_act(kv.reshape(T * H, hd), hd, rotate=rotate, offset=offset)
+    return {"q": res["q"].reshape(T, H, hd), "scale": res["scale"].reshape(T, H),
+            "offset": res["offset"].reshape(T, H), "codes": res["codes"].reshape(T, H, hd // 2),
+            "residual": res["residual"].reshape(T, H, hd)}
+
+
+# ---------------------------------------------------------------------------
+# Storage accounting  (Sec. 3.4 "Efficiency of Per-Group Activation Quantization")
+# ---------------------------------------------------------------------------
+
+def effective_bits(group: int, code_bits: int = 4, param_bits: int = 16, n_params: int = 2) -> float:
+    """Bits per activation when each group of ``group`` codes stores ``n_params`` parameters."""
+    return (code_bits * group + param_bits * n_params) / group
+
+
+def effective_bits_per_token_offset(K: int, g: int, code_bits: int = 4, param_bits: int = 32) -> float:
+    """Bits per activation of this path's layout: one scale per token and one offset per block."""
+    return (code_bits * K + param_bits * (1 + K // g)) / K

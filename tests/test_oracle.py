@@ -1,0 +1,319 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix.
+
+Each test would fail under a plausible slip in the oracle: a wrong Hadamard
+ordering or normalisation, a dropped or mis-indexed offset term, a wrong
+rounding mode or scale, a transposed GEMM operand, or a wrong nibble layout.
+"""
+
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import scipy.linalg
+
+import oracle as O
+import workloads as W
+
+
+def _load(golden_dir, name):
+    with open(os.path.join(golden_dir, name)) as f:
+        return json.load(f)
+
+
+# --------------------------------------------------------------------------
+# Hadamard (Sec. 3.2): +-1 entries, orthogonal, first row all ones.
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("g", [1, 2, 4, 8, 32, 128, 512, 2048])
+def test_hadamard_structure(g):
+    H = O.sylvester_hadamard(g)
+    assert H.shape == (g, g)
+    assert set(np.unique(H)) <= {-1, 1}
+    assert np.all(H[0] == 1)
+    np.testing.assert_array_equal(H @ H.T, g * np.eye(g, dtype=np.int64))
+    # Every row but the first sums to zero: the reason the offset is x_1 / sqrt(g).
+    np.testing.assert_array_equal(H[1:].sum(axis=1), 0)
+
+
+@pytest.mark.parametrize("g", [2, 16, 256, 1024])
+def test_hadamard_matches_library(g):
+    # scipy builds the Sylvester matrix independently.
+    np.testing.assert_array_equal(O.sylvester_hadamard(g), scipy.linalg.hadamard(g))
+
+
+def test_hadamard_h4_golden(golden_dir):
+    d = _load(golden_dir, "hadamard_h4.json")
+    np.testing.assert_array_equal(O.sylvester_hadamard(4), np.array(d["H4"]))
+
+
+def test_rotation_against_butterfly():
+    """The dense-matmul rotation equals an independent fast butterfly transform."""
+    rng = np.random.default_rng(3)
+    g, T = 64, 5
+    x = rng.standard_normal((T, 3 * g))
+
+    def fwht(v):
+        v = v.copy()
+        h = 1
+        while h < len(v):
+            for i in range(0, len(v), 2 * h):
+                a = v[i:i + h].copy()
+                b = v[i + h:i + 2 * h].copy()
+                v[i:i + h] = a + b
+                v[i + h:i + 2 * h] = a - b
+            h *= 2
+        return v
+
+    y = O.rotate_blocks(x, g)
+    for t in range(T):
+        for b in range(3):
+            blk = x[t, b * g:(b + 1) * g]
+            np.testing.assert_allclose(y[t, b * g:(b + 1) * g], fwht(blk) / math.sqrt(g),
+                                       rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("g", [2, 8, 128, 1024])
+def test_rotation_is_orthonormal(g):
+    rng = np.random.default_rng(g)
+    x = rng.standard_normal((4, 2 * g))
+    y = O.rotate_blocks(x, g)
+    # Parseval per block: a wrong normalisation (1/g, none) changes the norm.
+    for b in range(2):
+        sl = slice(b * g, (b + 1) * g)
+        np.testing.assert_allclose(np.linalg.norm(y[:, sl], axis=1),
+                                   np.linalg.norm(x[:, sl], axis=1), rtol=1e-12)
+    # Applying it twice is the identity (H/sqrt(g) is symmetric and orthogonal).
+    np.testing.assert_allclose(O.rotate_blocks(y, g), x, rtol=0, atol=1e-11)
+
+
+# --------------------------------------------------------------------------
+# Offsetting (Sec. 3.2, Eq. 4-5).
+# --------------------------------------------------------------------------
+
+def test_eq5_worked_example(golden_dir):
+    d = _load(golden_dir, "eq5_two_channel.json")
+    for c in d["cases"]:
+        x = np.array([c["x"]])
+        y = O.rotate_blocks(x, 2)
+        np.testing.assert_allclose(y[0], c["y"], rtol=1e-15, atol=1e-15)
+        res = O.quantize_act(x, 2, rotate=True, offset=True)
+        np.testing.assert_allclose(res["offset"][0, 0], c["offset"], rtol=1e-15, atol=1e-15)
+        np.testing.assert_allclose(res["residual"][0], c["residual"], rtol=1e-15, atol=1e-15)
+
+
+@pytest.mark.parametrize("g", [2, 4, 32, 256, 1024])
+def test_offset_is_first_channel_over_sqrt_g(g):
+    """The block mean of X H / sqrt(g) is x_1 / sqrt(g) (Sec. 3.2)."""
+    rng = np.random.default_rng(11 + g)
+    G = 3
+    x = rng.standard_normal((6, G * g)) * 3.0
+    res = O.quantize_act(x, g, rotate=True, offset=True)
+    expect = x[:, ::g] / math.sqrt(g)
+    np.testing.assert_allclose(res["offset"], expect, rtol=1e-12, atol=1e-12)
+    # The residual of every block sums to zero.
+    np.testing.assert_allclose(res["residual"].reshape(6, G, g).sum(axis=2), 0.0, atol=1e-10)
+
+
+def test_outlier_only_row_leaves_zero_residual():
+    g = 128
+    x = np.zeros((2, 2 * g))
+    x[0, 0] = 300.0
+    x[0, g] = -20.5
+    x[1, 0] = 1e-3
+    res = O.quantize_act(x, g, rotate=True, offset=True)
+    assert np.all(res["residual"] == 0.0)
+    assert np.all(res["q"] == 0) and np.all(res["scale"] == 0.0)
+    np.testing.assert_allclose(res["offset"][0], [300.0 / math.sqrt(g), -20.5 / math.sqrt(g)], rtol=1e-15)
+
+
+def test_unit_channel_gives_hadamard_row_codes():
+    """x = e_j (j >= 1) rotates to H[j]/sqrt(g): offset 0, all codes +-7 in H's sign pattern."""
+    g = 64
+    H = O.sylvester_hadamard(g)
+    for j in (1, 5, 63):
+        x = np.zeros((1, g))
+        x[0, j] = 1.0
+        res = O.quantize_act(x, g, rotate=True, offset=True)
+        assert res["offset"][0, 0] == 0.0
+        np.testing.assert_array_equal(res["q"][0], 7 * H[j])
+        np.testing.assert_allclose(res["scale"][0], 1.0 / (7.0 * math.sqrt(g)), rtol=1e-15)
+
+
+def test_offset_without_rotation_is_block_mean():
+    x = np.array([[1.0, 2.0, 3.0, 6.0, -1.0, -1.0, -1.0, -1.0]])
+    res = O.quantize_act(x, 4, rotate=False, offset=True)
+    np.testing.assert_array_equal(res["offset"], [[3.0, -1.0]])
+    np.testing.assert_array_equal(res["residual"], [[-2.0, -1.0, 0.0, 3.0, 0.0, 0.0, 0.0, 0.0]])
+    # Residual max is 3 -> scale 3/7; codes rne(r * 7/3).
+    np.testing.assert_array_equal(res["q"], [[-5, -2, 0, 7, 0, 0, 0, 0]])
+
+
+def test_offsetting_reduces_quantization_error():
+    """Statistical property the method rests on (Sec. 3.2): with a concentrated
+    outlier channel, offsetting lowers the 4-bit reconstruction error."""
+    g = 512
+    x = W.activations(64, g, seed=5, n_out=1, mult=100.0)
+    with_off = O.quantize_act(x, g, rotate=True, offset=True)
+    no_off = O.quantize_act(x, g, rotate=True, offset=False)
+    y = with_off["y"]
+
+    def mse(res):
+        xh = O.dequantize_act(res["q"], res["scale"], res["offset"], g)
+        return np.mean((xh - y) ** 2)
+
+    assert mse(with_off) < 0.5 * mse(no_off)
+
+
+# --------------------------------------------------------------------------
+# Quantizer (Eq. 1, symmetric; readings: rne, s = max/7, [-7, 7]).
+# --------------------------------------------------------------------------
+
+def test_rtn_textbook_rows(golden_dir):
+    d = _load(golden_dir, "rtn_textbook.json")
+    for row in d["rows"]:
+        x = np.array([row["x"]])
+        res = O.quantize_act(x, 8, rotate=False, offset=False)
+        np.testing.assert_array_equal(res["q"][0], row["q"])
+        np.testing.assert_allclose(res["scale"][0], row["scale"], rtol=1e-15)
+        assert np.all(res["offset"] == 0.0)
+
+
+def test_quantization_error_bound():
+    rng = np.random.default_rng(21)
+    x = rng.standard_normal((32, 256)) * rng.uniform(0.1, 10, size=(32, 1))
+    for rotate in (False, True):
+        for offset in (False, True):
+            res = O.quantize_act(x, 64, rotate=rotate, offset=offset)
+            err = np.abs(res["residual"] - res["scale"][:, None] * res["q"])
+            assert np.all(err <= res["scale"][:, None] / 2 * (1 + 1e-12))
+            # The largest residual of each row lands on the grid's end.
+            assert np.all(np.max(np.abs(res["q"]), axis=1) == 7)
+
+
+def test_brute_force_eight_channels():
+    """At D = 8, each code is the grid point nearest to R/s, ties to the even code."""
+    rng = np.random.default_rng(8)
+    grid = np.arange(-7, 8)
+    for trial in range(200):
+        x = rng.standard_normal((1, 8)) * rng.uniform(0.01, 100)
+        if trial % 4 == 0:
+            x[0, 0] += 50.0
+        rotate = trial % 2 == 0
+        res = O.quantize_act(x, 8, rotate=rotate, offset=True)
+        r, s = res["residual"][0], res["scale"][0]
+        for k in range(8):
+            d = np.abs(r[k] / s - grid)
+            best = grid[d <= d.min() + 1e-12]
+            expect = best[0] if len(best) == 1 else best[best % 2 == 0][0]
+            assert res["q"][0, k] == expect
+
+
+def test_pack_layout_golden(golden_dir):
+    d = _load(golden_dir, "pack_layout.json")
+    packed = O.pack_codes(np.array([d["codes"]]))
+    np.testing.assert_array_equal(packed[0], d["bytes"])
+    np.testing.assert_array_equal(O.unpack_codes(packed)[0], d["codes"])
+
+
+def test_pack_roundtrip_all_codes():
+    q = np.array(np.meshgrid(np.arange(-7, 8), np.arange(-7, 8))).reshape(2, -1).T.reshape(1, -1)
+    np.testing.assert_array_equal(O.unpack_codes(O.pack_codes(q)), q)
+    with pytest.raises(ValueError):
+        O.pack_codes(np.array([[8, 0]]))
+
+
+# --------------------------------------------------------------------------
+# Weights, GEMM and epilogue.
+# --------------------------------------------------------------------------
+
+def test_weight_rotation_cancels():
+    """(X H)(W H)^T = X W^T for the symmetric orthonormal block Hadamard."""
+    rng = np.random.default_rng(4)
+    g, K, N = 32, 96, 7
+    x = rng.standard_normal((5, K))
+    w = rng.standard_normal((N, K))
+    y = O.rotate_blocks(x, g)
+    wp = O.prepare_weight(w, g, rotate=True)
+    np.testing.assert_allclose(y @ wp["w_eff"].T, x @ w.T, rtol=1e-11, atol=1e-11)
+
+
+def test_weight_table_is_block_rowsum():
+    rng = np.random.default_rng(6)
+    g, K, N = 16, 64, 9
+    w = rng.standard_normal((N, K))
+    wp = O.prepare_weight(w, g, rotate=True)
+    q = O.unpack_codes(wp["codes"])
+    np.testing.assert_array_equal(q, wp["q"])
+    for b in range(K // g):
+        for n in range(N):
+            assert wp["offsum"][b, n] == pytest.approx(wp["scale"][n] * q[n, b * g:(b + 1) * g].sum(), rel=1e-15)
+
+
+def test_int_gemm_loops_match_blas():
+    rng = np.random.default_rng(9)
+    qa = rng.integers(-7, 8, size=(5, 40))
+    qw = rng.integers(-7, 8, size=(6, 40))
+    np.testing.assert_array_equal(O.int_gemm(qa, qw), O.int_gemm_loops(qa, qw))
+    # Not transposed: a row of ones against a one-hot weight picks one column sum.
+    e = np.zeros((1, 40), dtype=np.int64)
+    e[0, 3] = 1
+    np.testing.assert_array_equal(O.int_gemm(qa, e)[:, 0], qa[:, 3])
+
+
+def test_int_gemm_exact_at_largest_k():
+    K = 28672
+    qa = np.full((2, K), 7)
+    qw = np.full((3, K), -7)
+    qw[1] = 7
+    acc = O.int_gemm(qa, qw)
+    assert acc[0, 0] == -49 * K and acc[0, 1] == 49 * K
+
+
+def test_offset_identity_unquantized():
+    """W x = W (x - o 1) + o W 1 per block, in float64 before any rounding."""
+    rng = np.random.default_rng(10)
+    g, G, N = 32, 3, 11
+    x = rng.standard_normal((4, g * G)) * 5
+    w = rng.standard_normal((N, g * G))
+    o = rng.standard_normal((4, G)) * 20
+    ob = np.repeat(o, g, axis=1)
+    lhs = x @ w.T
+    rhs = (x - ob) @ w.T + o @ w.reshape(N, G, g).sum(axis=2).T
+    np.testing.assert_allclose(lhs, rhs, rtol=1e-12, atol=1e-10)
+
+
+@pytest.mark.parametrize("rotate", [False, True])
+def test_epilogue_equals_dequantized_product(rotate):
+    """s_a s_w acc + o S equals X_hat W_hat^T computed from the dequantized matrices."""
+    g, G, N, T = 64, 3, 13, 7
+    x = W.activations(T, g * G, seed=12, n_out=2, mult=40.0)
+    w = W.weights(N, g * G, seed=13)
+    a = O.quantize_act(x, g, rotate=rotate, offset=True)
+    wp = O.prepare_weight(w, g, rotate=rotate)
+    out = O.w4a4_linear(a["q"], a["scale"], a["offset"], wp["q"], wp["scale"], wp["offsum"])
+    xh = O.dequantize_act(a["q"], a["scale"], a["offset"], g)
+    wh = wp["q"] * wp["scale"][:, None]
+    np.testing.assert_allclose(out["y"], xh @ wh.T, rtol=1e-12, atol=1e-12 * np.abs(out["y"]).max())
+    # And it approximates the unquantized layer.
+    ref = O.linear_reference(x, w)
+    assert np.linalg.norm(out["y"] - ref) < 0.3 * np.linalg.norm(ref)
+
+
+def test_kv4_is_per_head_block():
+    kv = W.kv_heads(3, 4, 128, seed=2)
+    res = O.kv4_quantize(kv)
+    for t in range(3):
+        for h in range(4):
+            one = O.quantize_act(kv[t, h][None, :], 128)
+            np.testing.assert_array_equal(res["q"][t, h], one["q"][0])
+            assert res["scale"][t, h] == one["scale"][0]
+            assert res["offset"][t, h] == one["offset"][0, 0]
+
+
+def test_storage_bits_golden(golden_dir):
+    d = _load(golden_dir, "storage_bits.json")
+    assert O.effective_bits(d["group"], d["code_bits"], d["param_bits"], d["n_params"]) == d["bits"]
+    # This path: one fp32 scale per token + one fp32 offset per block.
+    assert O.effective_bits_per_token_offset(4096, 4096) == pytest.approx(4 + 64 / 4096)
