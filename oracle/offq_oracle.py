@@ -25,8 +25,9 @@ it implements. Where the paper is silent, it uses these readings:
   quantized weights' block row sums, so the epilogue reproduces W_hat @ X_hat
   exactly (Sec. 3.2, Eq. 5: the offset is a constant added to every channel of
   a block, so it leaves through the weight row sums).
-* Packing: two 4-bit sign-magnitude codes per byte, the even channel in the low
-  nibble; a code is (sign << 3) | |q|.
+* Packing of activation codes: Eq. 1's unsigned form with zero-point 8 (nibble
+  q + 8), two per byte, even channel low. Weight codes: sign-magnitude nibbles
+  interleaved per 8 channels (layout in :func:`pack_weight_codes`).
 
 Decisions that turn floating point into integers (the codes) are taken here in
 float64.
@@ -117,30 +118,64 @@ def quantize_rows(r: np.ndarray):
     return q, s
 
 
-def pack_codes(q: np.ndarray) -> np.ndarray:
-    """Pack signed codes [.., K] into bytes [.., K/2]: sign-magnitude nibbles, even channel low.
+def pack_act_codes(q: np.ndarray) -> np.ndarray:
+    """Activation codes [.., K] -> bytes [.., K/2] in Eq. 1's unsigned form.
 
-    A nibble is (sign << 3) | |q| with sign = 1 for q < 0.
+    Eq. 1 stores x_q = round(x / s) + z in [0, 2^b - 1]; with b = 4 and the
+    zero-point z = 8 a symmetric code q in [-7, 7] becomes the nibble q + 8.
+    Two nibbles per byte, the even channel in the low nibble.
     """
     q = np.asarray(q, dtype=np.int64)
     if q.shape[-1] % 2:
         raise ValueError("K must be even")
     if np.any(np.abs(q) > QMAX):
         raise ValueError("code out of range")
-    nib = (np.abs(q) | np.where(q < 0, 8, 0)).astype(np.uint8)
-    return (nib[..., 0::2] | (nib[..., 1::2] << 4)).astype(np.uint8)
+    u = (q + 8).astype(np.uint8)
+    return (u[..., 0::2] | (u[..., 1::2] << 4)).astype(np.uint8)
 
 
-def unpack_codes(packed: np.ndarray) -> np.ndarray:
-    """Inverse of :func:`pack_codes`: bytes [.., K/2] -> int64 codes [.., K]."""
-    p = np.asarray(packed, dtype=np.uint8)
-    lo = p & 0xF
-    hi = p >> 4
+def unpack_act_codes(packed: np.ndarray) -> np.ndarray:
+    """Inverse of :func:`pack_act_codes`."""
+    p = np.asarray(packed, dtype=np.uint8).astype(np.int64)
     out = np.empty(p.shape[:-1] + (2 * p.shape[-1],), dtype=np.int64)
-    for dst, nib in ((out[..., 0::2], lo), (out[..., 1::2], hi)):
-        mag = (nib & 7).astype(np.int64)
-        dst[...] = np.where(nib & 8, -mag, mag)
+    out[..., 0::2] = (p & 0xF) - 8
+    out[..., 1::2] = (p >> 4) - 8
     return out
+
+
+def pack_weight_codes(q: np.ndarray) -> np.ndarray:
+    """Weight codes [.., K] -> bytes [.., K/2], sign-magnitude, interleaved by 8.
+
+    Each group of 8 channels c0..c7 occupies 4 bytes B0..B3 with
+    Bj bits 0-2 = |q(c_2j)|, bit 7 = sign(q(c_2j)), bits 4-6 = |q(c_2j+1)|,
+    bit 3 = sign(q(c_(2j-1) mod 8)); sign = 1 for a negative code.
+    """
+    q = np.asarray(q, dtype=np.int64)
+    if q.shape[-1] % 8:
+        raise ValueError("K must be a multiple of 8")
+    if np.any(np.abs(q) > QMAX):
+        raise ValueError("code out of range")
+    lead = q.shape[:-1]
+    g8 = q.reshape(lead + (q.shape[-1] // 8, 8))
+    mag = np.abs(g8)
+    neg = (g8 < 0).astype(np.int64)
+    out = np.zeros(lead + (q.shape[-1] // 8, 4), dtype=np.int64)
+    for j in range(4):
+        out[..., j] = (mag[..., 2 * j] | (neg[..., 2 * j] << 7) | (mag[..., 2 * j + 1] << 4)
+                       | (neg[..., (2 * j - 1) % 8] << 3))
+    return out.reshape(lead + (q.shape[-1] // 2,)).astype(np.uint8)
+
+
+def unpack_weight_codes(packed: np.ndarray) -> np.ndarray:
+    """Inverse of :func:`pack_weight_codes`."""
+    p = np.asarray(packed, dtype=np.uint8).astype(np.int64)
+    lead = p.shape[:-1]
+    b = p.reshape(lead + (p.shape[-1] // 4, 4))
+    q = np.zeros(lead + (p.shape[-1] // 4, 8), dtype=np.int64)
+    for j in range(4):
+        q[..., 2 * j] = np.where((b[..., j] >> 7) & 1, -1, 1) * (b[..., j] & 7)
+        q[..., 2 * j + 1] = ((b[..., j] >> 4) & 7) * np.where((b[..., (j + 1) % 4] >> 3) & 1, -1, 1)
+    return q.reshape(lead + (2 * p.shape[-1],))
 
 
 # ---------------------------------------------------------------------------
@@ -183,7 +218,7 @@ def quantize_act(x: np.ndarray, g: int, rotate: bool = True, offset: bool = True
     ru = subtract_offsets(yu, ou, g)
     q, su = quantize_rows(ru)
     return {"y": yu / norm, "offset": ou / norm, "residual": ru / norm, "q": q,
-            "scale": su / norm, "codes": pack_codes(q)}
+            "scale": su / norm, "codes": pack_act_codes(q)}
 
 
 def dequantize_act(q: np.ndarray, s: np.ndarray, o: np.ndarray, g: int) -> np.ndarray:
@@ -214,7 +249,7 @@ def prepare_weight(w: np.ndarray, g: int, rotate: bool = True) -> Dict[str, np.n
     rowsum = qw.reshape(N, G, g).sum(axis=2)          # int64 [N, G]
     S = (rowsum.astype(np.float64) * sw[:, None]).T    # float64 [G, N]
     return {"w_eff": w_eff, "q": qw, "scale": sw, "offsum": S, "rowsum": rowsum.T,
-            "codes": pack_codes(qw)}
+            "codes": pack_weight_codes(qw)}
 
 
 # ---------------------------------------------------------------------------

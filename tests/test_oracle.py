@@ -212,16 +212,22 @@ def test_brute_force_eight_channels():
 
 def test_pack_layout_golden(golden_dir):
     d = _load(golden_dir, "pack_layout.json")
-    packed = O.pack_codes(np.array([d["codes"]]))
-    np.testing.assert_array_equal(packed[0], d["bytes"])
-    np.testing.assert_array_equal(O.unpack_codes(packed)[0], d["codes"])
+    codes = np.array([d["codes"]])
+    np.testing.assert_array_equal(O.pack_act_codes(codes)[0], d["act_bytes"])
+    np.testing.assert_array_equal(O.unpack_act_codes(np.array([d["act_bytes"]]))[0], d["codes"])
+    np.testing.assert_array_equal(O.pack_weight_codes(codes)[0], d["weight_bytes"])
+    np.testing.assert_array_equal(O.unpack_weight_codes(np.array([d["weight_bytes"]]))[0], d["codes"])
 
 
 def test_pack_roundtrip_all_codes():
-    q = np.array(np.meshgrid(np.arange(-7, 8), np.arange(-7, 8))).reshape(2, -1).T.reshape(1, -1)
-    np.testing.assert_array_equal(O.unpack_codes(O.pack_codes(q)), q)
+    rng = np.random.default_rng(1)
+    q = rng.integers(-7, 8, size=(3, 256))
+    np.testing.assert_array_equal(O.unpack_act_codes(O.pack_act_codes(q)), q)
+    np.testing.assert_array_equal(O.unpack_weight_codes(O.pack_weight_codes(q)), q)
     with pytest.raises(ValueError):
-        O.pack_codes(np.array([[8, 0]]))
+        O.pack_act_codes(np.array([[8, 0]]))
+    with pytest.raises(ValueError):
+        O.pack_weight_codes(np.array([[-8, 0, 0, 0, 0, 0, 0, 0]]))
 
 
 # --------------------------------------------------------------------------
@@ -244,7 +250,7 @@ def test_weight_table_is_block_rowsum():
     g, K, N = 16, 64, 9
     w = rng.standard_normal((N, K))
     wp = O.prepare_weight(w, g, rotate=True)
-    q = O.unpack_codes(wp["codes"])
+    q = O.unpack_weight_codes(wp["codes"])
     np.testing.assert_array_equal(q, wp["q"])
     for b in range(K // g):
         for n in range(N):
