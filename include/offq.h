@@ -1,0 +1,200 @@
+/*
+ * offq.h -- C ABI of the OffQ W4A4 linear hot path on GB300 (sm_103a).
+ *
+ * OffQ (arxiv 2606.07116) makes 4-bit weight/activation/KV quantization work
+ * by rotating each activation row with a Hadamard matrix whose first row is all
+ * ones, so the concentrated outlier channel turns into a constant offset shared
+ * by a whole block of channels (Sec. 3.2, Eq. 4-5), and quantizing what is left
+ * on a uniform 4-bit grid (Sec. 3, Eq. 1). This library runs the online part of
+ * that method:
+ *
+ *   offq_quantize_act   token rows -> block Hadamard -> offsets -> 4-bit codes
+ *   offq_w4a4_linear    4-bit x 4-bit GEMM + dequant + offset epilogue
+ *   offq_kv4_quantize   per-(token, head) version of the quantizer (KV cache)
+ *   offq_prepare_weight offline: rotated, per-channel 4-bit weights + tables
+ *
+ * Conventions shared by every call
+ *   - Pointers named as device buffers are device pointers allocated and owned
+ *     by the caller. The library never allocates, frees, or synchronizes the
+ *     stream (offq_get_device_status is the one call that synchronizes).
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *   - Arguments are checked on the host before anything is launched. A bad
+ *     shape or flag returns OFFQ_ERR_INVALID_ARG or OFFQ_ERR_UNSUPPORTED; a
+ *     pointer or leading dimension that breaks the alignment rule of the call
+ *     returns OFFQ_ERR_MISALIGNED; a failed launch returns OFFQ_ERR_CUDA.
+ *     Nothing is written when a call returns an error.
+ *   - Errors that only the device can see (a bounded wait that ran out inside
+ *     a kernel) are recorded in a device status word; offq_get_device_status
+ *     reads and clears it.
+ *   - NaN or Inf inputs: results are unspecified (no checks on the hot path).
+ *   - Calls are thread-safe; the only state is a per-process cache of TMA
+ *     descriptors guarded by a mutex, and the device status word.
+ *
+ * Block size g. The online rotation is block-diagonal with g x g Sylvester
+ * Hadamard blocks (group-wise offsetting, Sec. 3.2); each block of g channels
+ * of a row gets one offset. g is a power of two in [32, 8192] and divides K.
+ * The scale is one per token row across all blocks.
+ *
+ * Code formats (the paper fixes the 4-bit uniform grid, not a bit layout):
+ *   Activation codes: Eq. 1's unsigned form with zero-point 8. A residual
+ *     quantized to q in [-7, 7] is stored as the nibble u = q + 8 (1..15). Two
+ *     nibbles per byte, the even channel in the low nibble; row t occupies
+ *     bytes [t*K/2, (t+1)*K/2).
+ *   Weight codes: per-output-channel signed q in [-7, 7], sign-magnitude,
+ *     interleaved per group of 8 channels c0..c7 held in 4 bytes B0..B3:
+ *       Bj bits 0-2 = |q(c_2j)|, bit 7 = sign(q(c_2j)),
+ *       Bj bits 4-6 = |q(c_2j+1)|, bit 3 = sign(q(c_(2j-1) mod 8)).
+ *     (This lets the GEMM widen 8 codes to fp8 tensor-core operands with one
+ *     rotate and two masks.) Row n occupies bytes [n*K/2, (n+1)*K/2).
+ */
+#ifndef OFFQ_H
+#define OFFQ_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define OFFQ_ABI_VERSION 1
+
+typedef enum {
+  OFFQ_OK = 0,
+  OFFQ_ERR_INVALID_ARG = -1,  /* shape, flag or NULL pointer not allowed   */
+  OFFQ_ERR_UNSUPPORTED = -2,  /* valid request this build does not handle  */
+  OFFQ_ERR_MISALIGNED = -3,   /* pointer / leading dimension alignment     */
+  OFFQ_ERR_CUDA = -4,         /* a CUDA runtime call failed                */
+  OFFQ_ERR_TIMEOUT = -5       /* a device-side bounded wait ran out        */
+} offq_status;
+
+/* Element types of floating-point buffers. */
+enum { OFFQ_F32 = 0, OFFQ_BF16 = 1, OFFQ_F16 = 2 };
+
+/* Flags of the quantizers. */
+enum {
+  OFFQ_ROTATE = 1, /* apply the online block Hadamard H/sqrt(g) (Eq. 4)       */
+  OFFQ_OFFSET = 2  /* subtract each block's mean as its offset (Eq. 5)        */
+};
+
+/*
+ * offq_quantize_act -- online activation quantizer (paper Sec. 3.2 Eq. 4-5,
+ * Sec. 3 Eq. 1; the online rotation H4 of Sec. 3.3 Step 2 (4)).
+ *
+ * For each token row x (K channels) and each block b of g channels:
+ *   y = x_b H_g / sqrt(g)          if OFFQ_ROTATE (else y = x_b)
+ *   o[b] = mean(y)                 if OFFQ_OFFSET (else 0); with the rotation
+ *                                  this equals x_b[0] / sqrt(g)
+ *   r = y - o[b]
+ * then over the whole row: s = max|r| / 7 (0 for an all-zero residual),
+ * q = clamp(round_half_even(r / s), -7, 7), stored as u = q + 8.
+ *
+ *   x       device, [T][ldx] elements of x_dtype (OFFQ_F32/BF16/F16), row-major;
+ *           16-byte aligned, ldx * sizeof(elem) a multiple of 16, ldx >= K.
+ *   T       token rows, >= 0 (T = 0 launches nothing).
+ *   K       channels, a multiple of g and of 32, K <= 32768.
+ *   g       block size, power of two in [32, 8192].
+ *   flags   OR of OFFQ_ROTATE, OFFQ_OFFSET.
+ *   codes   device, [T][K/2] bytes (activation code format), 16-byte aligned.
+ *   scale   device, [T] float32.
+ *   offset  device, [T][K/g] float32; required with OFFQ_OFFSET; when given
+ *           without OFFQ_OFFSET it is filled with zeros; may be NULL otherwise.
+ */
+int offq_quantize_act(const void* x, int x_dtype, int64_t T, int64_t K, int64_t ldx,
+                      int32_t g, int32_t flags,
+                      uint8_t* codes, float* scale, float* offset, void* stream);
+
+/*
+ * offq_w4a4_linear -- W4A4 GEMM with fused dequant and offset epilogue
+ * ("all matrix multiplications in uniform 4-bit execution", Sec. 1; the
+ * offset leaves a block as a constant, Eq. 5, so it meets the weight block
+ * row sums).
+ *
+ *   y[t][n] = s_a[t] * s_w[n] * sum_k q_a[t][k] q_w[n][k]
+ *           + s_w[n] * sum_b o[t][b] * R[b][n]
+ *
+ * accumulated exactly in integers (the tensor cores see both codes as exact
+ * fp8 values; every partial sum is an integer below 2^24), dequantized in fp32
+ * and rounded once to the output type.
+ *
+ *   a_codes   device, [T][K/2] activation codes (offq_quantize_act), 16-B aligned.
+ *   a_scale   device, [T] float32.
+ *   a_offset  device, [T][K/g] float32, or NULL for all-zero offsets.
+ *   T, N, K   tokens, output channels, input channels; T >= 0, N >= 1,
+ *             K a multiple of g and of 32, K <= 65536.
+ *   g         block size used when the codes were made (power of two, 32..8192).
+ *   w_codes   device, [N][K/2] weight codes (offq_prepare_weight), 16-B aligned.
+ *   w_scale   device, [N] float32.
+ *   w_offsum  device, [K/g][N] float32: R[b][n] = sum_{k in block b} q_w[n][k],
+ *             the integer block row sums of the weight codes (exact in fp32).
+ *   out       device, [T][ldo] of out_dtype (OFFQ_F32/BF16/F16), ldo >= N,
+ *             16-byte aligned with ldo * sizeof(out) a multiple of 16.
+ *   acc_debug device, [T][N] int32 or NULL. When given, also receives the
+ *             integer the tensor cores accumulate, sum_k (q_a + 8) * q_w
+ *             (equal to the true dot product plus 8 * sum_k q_w[n][k]).
+ */
+int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, const float* a_offset,
+                     int64_t T, int64_t N, int64_t K, int32_t g,
+                     const uint8_t* w_codes, const float* w_scale, const float* w_offsum,
+                     void* out, int out_dtype, int64_t ldo, int32_t* acc_debug, void* stream);
+
+/*
+ * offq_kv4_quantize -- KV-cache quantizer: offq_quantize_act applied to every
+ * (token, head) vector with g = head_dim, i.e. the per-head online Hadamard H3
+ * of the keys (Sec. 3.3 Step 2 (3)) with one offset and one scale per head
+ * (the KV quantization group equals the head dimension, Sec. 4.2).
+ *
+ *   kv        device, element (t, h, d) at kv[t*ld_token + h*head_dim + d];
+ *             16-byte aligned, ld_token * sizeof(elem) a multiple of 16,
+ *             ld_token >= H * head_dim.
+ *   T, H      tokens (>= 0) and heads (>= 1).
+ *   head_dim  power of two in [32, 8192].
+ *   flags     OR of OFFQ_ROTATE, OFFQ_OFFSET (V vectors, rotated offline by
+ *             R2, may pass OFFQ_OFFSET alone).
+ *   codes     device, [T][H][head_dim/2] activation code format, 16-B aligned.
+ *   scale     device, [T][H] float32.
+ *   offset    device, [T][H] float32 (same rules as offq_quantize_act).
+ */
+int offq_kv4_quantize(const void* kv, int dtype, int64_t T, int32_t H, int32_t head_dim,
+                      int64_t ld_token, int32_t flags,
+                      uint8_t* codes, float* scale, float* offset, void* stream);
+
+/*
+ * offq_prepare_weight -- offline weight preparation (not on the timed path).
+ * The inverse of the online rotation is fused into the weight (Sec. 3.3
+ * Step 2 (4): W x = (W H)(H x) for the symmetric orthonormal block Hadamard),
+ * then each output channel is quantized symmetrically (per-channel symmetric
+ * weights, Sec. 4 "Implementation and Settings"; round-to-nearest stands in
+ * for GPTQ, which needs calibration data):
+ *   W_eff = W blockdiag(H_g)/sqrt(g) if rotate else W
+ *   s_w[n] = max|W_eff[n]| / 7,  q_w = clamp(rne(W_eff / s_w), -7, 7)
+ *   R[b][n] = sum_{k in block b} q_w[n][k]   (integers, stored as float32)
+ *
+ *   w         device, [N][K] of dtype, row-major, 16-byte aligned.
+ *   N, K, g   as in offq_w4a4_linear.
+ *   rotate    nonzero to fuse the block Hadamard.
+ *   w_codes   device, [N][K/2] weight code format, 16-B aligned.
+ *   w_scale   device, [N] float32.
+ *   w_offsum  device, [K/g][N] float32.
+ */
+int offq_prepare_weight(const void* w, int dtype, int64_t N, int64_t K, int32_t g, int32_t rotate,
+                        uint8_t* w_codes, float* w_scale, float* w_offsum, void* stream);
+
+/*
+ * offq_get_device_status -- synchronizes `stream`, returns the device status
+ * word of the current device (OFFQ_OK, or OFFQ_ERR_TIMEOUT when a kernel's
+ * bounded wait ran out since the last call) and clears it. Returns
+ * OFFQ_ERR_CUDA if the synchronization itself fails.
+ */
+int offq_get_device_status(void* stream);
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char* offq_status_string(int status);
+
+/* OFFQ_ABI_VERSION of the loaded library. */
+int offq_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* OFFQ_H */

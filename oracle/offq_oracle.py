@@ -21,10 +21,11 @@ it implements. Where the paper is silent, it uses these readings:
 * Weights: per-output-channel symmetric round-to-nearest (Sec. 4 settings; GPTQ
   needs calibration data), after the same block rotation so that
   W x = (W H)(H x) for the orthonormal, symmetric block Hadamard H.
-* Offset correction table: S[b, n] = s_w[n] * sum_{k in b} Qw[n, k], the
-  quantized weights' block row sums, so the epilogue reproduces W_hat @ X_hat
-  exactly (Sec. 3.2, Eq. 5: the offset is a constant added to every channel of
-  a block, so it leaves through the weight row sums).
+* Offset correction table: R[b, n] = sum_{k in b} Qw[n, k], the quantized
+  weights' integer block row sums, so the epilogue
+  y = s_a s_w acc + s_w sum_b o_b R[b, n] reproduces W_hat @ X_hat exactly
+  (Sec. 3.2, Eq. 5: the offset is a constant added to every channel of a
+  block, so it leaves through the weight row sums).
 * Packing of activation codes: Eq. 1's unsigned form with zero-point 8 (nibble
   q + 8), two per byte, even channel low. Weight codes: sign-magnitude nibbles
   interleaved per 8 channels (layout in :func:`pack_weight_codes`).
@@ -238,7 +239,7 @@ def prepare_weight(w: np.ndarray, g: int, rotate: bool = True) -> Dict[str, np.n
     W_eff = W blockdiag(H_g) / sqrt(g) when the input takes the online rotation
     (Sec. 3.3 Step 2 (4): the inverse rotation is fused into the weight, and the
     block Hadamard is symmetric and orthonormal); s_w[n] = max|W_eff[n]| / 7;
-    Qw = clamp(rne(W_eff / s_w), -7, 7); S[b, n] = s_w[n] * sum_{k in block b} Qw[n, k].
+    Qw = clamp(rne(W_eff / s_w), -7, 7); R[b, n] = sum_{k in block b} Qw[n, k] (integers).
     """
     w = np.asarray(w, dtype=np.float64)
     N, K = w.shape
@@ -246,10 +247,9 @@ def prepare_weight(w: np.ndarray, g: int, rotate: bool = True) -> Dict[str, np.n
     res = quantize_act(w, g, rotate=rotate, offset=False)
     w_eff, qw, sw = res["y"], res["q"], res["scale"]
     G = K // g
-    rowsum = qw.reshape(N, G, g).sum(axis=2)          # int64 [N, G]
-    S = (rowsum.astype(np.float64) * sw[:, None]).T    # float64 [G, N]
-    return {"w_eff": w_eff, "q": qw, "scale": sw, "offsum": S, "rowsum": rowsum.T,
-            "codes": pack_weight_codes(qw)}
+    rowsum = qw.reshape(N, G, g).sum(axis=2).T        # int64 [G, N]
+    return {"w_eff": w_eff, "q": qw, "scale": sw, "offsum": rowsum.astype(np.float64),
+            "rowsum": rowsum, "codes": pack_weight_codes(qw)}
 
 
 # ---------------------------------------------------------------------------
@@ -285,22 +285,22 @@ def int_gemm_loops(qa: np.ndarray, qw: np.ndarray) -> np.ndarray:
 
 
 def epilogue(acc: np.ndarray, s_a: np.ndarray, o: np.ndarray, s_w: np.ndarray,
-             S: np.ndarray) -> np.ndarray:
-    """y[t, n] = s_a[t] * s_w[n] * acc[t, n] + sum_b o[t, b] * S[b, n], in float64.
+             R: np.ndarray) -> np.ndarray:
+    """y[t, n] = s_a[t] s_w[n] acc[t, n] + s_w[n] sum_b o[t, b] R[b, n], in float64.
 
     The second term is the offset's rank-G correction: each block's constant
     offset meets the block row sums of the dequantized weights.
     """
-    return (np.asarray(s_a, np.float64)[:, None] * np.asarray(s_w, np.float64)[None, :]
-            * np.asarray(acc, np.float64)
-            + np.asarray(o, np.float64) @ np.asarray(S, np.float64))
+    s_w = np.asarray(s_w, np.float64)[None, :]
+    return (np.asarray(s_a, np.float64)[:, None] * s_w * np.asarray(acc, np.float64)
+            + s_w * (np.asarray(o, np.float64) @ np.asarray(R, np.float64)))
 
 
 def w4a4_linear(qa: np.ndarray, s_a: np.ndarray, o: np.ndarray, qw: np.ndarray,
-                s_w: np.ndarray, S: np.ndarray) -> Dict[str, np.ndarray]:
+                s_w: np.ndarray, R: np.ndarray) -> Dict[str, np.ndarray]:
     """Integer GEMM of the codes plus the dequant + offset epilogue."""
     acc = int_gemm(qa, qw)
-    return {"acc": acc, "y": epilogue(acc, s_a, o, s_w, S)}
+    return {"acc": acc, "y": epilogue(acc, s_a, o, s_w, R)}
 
 
 def linear_reference(x: np.ndarray, w: np.ndarray) -> np.ndarray:
