@@ -36,6 +36,7 @@ float64.
 
 from __future__ import annotations
 
+import functools
 import math
 from typing import Dict, Optional
 
@@ -48,6 +49,22 @@ QMAX = 7  # largest code magnitude of the symmetric 4-bit grid (Eq. 1 with b = 4
 # Hadamard matrix and the online rotation  (Sec. 3.2, Eq. 4)
 # ---------------------------------------------------------------------------
 
+@functools.lru_cache(maxsize=4)
+def _sylvester_cached(g: int) -> np.ndarray:
+    h = np.ones((1, 1), dtype=np.int64)
+    while h.shape[0] < g:
+        h = np.block([[h, h], [h, -h]])
+    h.setflags(write=False)
+    return h
+
+
+@functools.lru_cache(maxsize=4)
+def _hadamard_f64(g: int) -> np.ndarray:
+    h = _sylvester_cached(g).astype(np.float64)
+    h.setflags(write=False)
+    return h
+
+
 def sylvester_hadamard(g: int) -> np.ndarray:
     """Sylvester Hadamard H_g (int64, entries +-1), H_1 = [1], H_2m = [[H, H], [H, -H]].
 
@@ -57,10 +74,7 @@ def sylvester_hadamard(g: int) -> np.ndarray:
     """
     if g < 1 or (g & (g - 1)) != 0:
         raise ValueError("g must be a power of two")
-    h = np.ones((1, 1), dtype=np.int64)
-    while h.shape[0] < g:
-        h = np.block([[h, h], [h, -h]])
-    return h
+    return _sylvester_cached(g).copy()
 
 
 def rotate_blocks(x: np.ndarray, g: int) -> np.ndarray:
@@ -73,7 +87,7 @@ def rotate_blocks(x: np.ndarray, g: int) -> np.ndarray:
     T, K = x.shape
     if K % g != 0:
         raise ValueError("g must divide K")
-    H = sylvester_hadamard(g).astype(np.float64)
+    H = _hadamard_f64(g)  # the Sylvester matrix of sylvester_hadamard, as float64
     y = np.empty_like(x)
     for b in range(K // g):
         sl = slice(b * g, (b + 1) * g)
@@ -206,7 +220,7 @@ def quantize_act(x: np.ndarray, g: int, rotate: bool = True, offset: bool = True
         raise ValueError("g must divide K")
     G = K // g
     if rotate:
-        H = sylvester_hadamard(g).astype(np.float64)
+        H = _hadamard_f64(g)  # the Sylvester matrix of sylvester_hadamard, as float64
         yu = np.empty_like(x)
         for b in range(G):
             sl = slice(b * g, (b + 1) * g)

@@ -1,0 +1,38 @@
+// Host-side helpers shared by the OffQ translation units (not part of the ABI).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "offq.h"
+
+namespace offq {
+
+// Device address of the status word of the current device (set up once per
+// device). Returns nullptr if the runtime call failed.
+int* device_status_ptr();
+
+inline bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+inline bool is_pow2(int64_t v) { return v > 0 && (v & (v - 1)) == 0; }
+
+inline int elem_bytes(int dtype) {
+  switch (dtype) {
+    case OFFQ_F32: return 4;
+    case OFFQ_BF16: return 2;
+    case OFFQ_F16: return 2;
+    default: return 0;
+  }
+}
+
+inline int launch_status() {
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? OFFQ_OK : OFFQ_ERR_CUDA;
+}
+
+// Largest input dimension the row quantizer stages in shared memory.
+constexpr int64_t kMaxQuantK = 32768;
+// Largest K of the GEMM: every partial sum stays an integer below 2^24.
+constexpr int64_t kMaxGemmK = 65536;
+
+}  // namespace offq

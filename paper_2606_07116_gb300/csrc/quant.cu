@@ -1,0 +1,503 @@
+// Row quantizers of the OffQ path: the online activation quantizer
+// (offq_quantize_act), the KV-cache quantizer (offq_kv4_quantize) and the
+// offline weight preparation (offq_prepare_weight).
+//
+// Per row and per block of g channels (paper Sec. 3.2, Eq. 4-5; Sec. 3 Eq. 1):
+//   y = x H_g / sqrt(g),  o = mean(y) = x[0] / sqrt(g),  r = y - o,
+//   s = max|r| / 7 over the row,  q = rne(r / s),  stored as q + 8.
+//
+// With the rotation on, the kernel uses that the first row of the Sylvester
+// Hadamard is all ones: zeroing x[0] before the transform yields the
+// unnormalised residual sqrt(g) * r directly, and the offset is x[0]/sqrt(g).
+// The 1/sqrt(g) factor cancels in r / s, so it is applied only to the stored
+// scale and offset.
+//
+// Kernel layout (per g = 2^L): a thread owns E = 2^ceil((L+1)/2) elements of a
+// block and TPB = g / E threads share a block. Pass 1 loads 16-byte vectors
+// (coalesced across the block's threads) and runs the butterflies of every
+// index bit it holds in registers; one transpose through shared memory then
+// gives each thread the remaining index bits (plus the lowest one or two, so
+// neighbouring channels stay together for packing) and pass 2 finishes the
+// transform. The Hadamard is a Kronecker product of 2x2 stages, so the stages
+// may run in any order.
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include <algorithm>
+#include <cmath>
+
+#include "offq.h"
+#include "offq_device.cuh"
+#include "offq_host.h"
+
+namespace {
+
+using namespace offq;
+
+struct QuantArgs {
+  const void* x;
+  int64_t ld_t;     // elements between consecutive tokens
+  int64_t ld_h;     // elements between consecutive heads (0 when H == 1)
+  int64_t rows;     // tokens * heads
+  int H;            // heads per token (1 for activations)
+  int K;            // channels per row
+  int G;            // blocks per row
+  int flags;
+  uint8_t* codes;   // [rows][K/2]
+  float* scale;     // [rows]
+  float* offset;    // [rows][G] or nullptr
+  float inv_sqrt_g; // 1/sqrt(g) with the rotation, else 1
+  float scale_mul;  // inv_sqrt_g / 7
+  int tpr;          // threads per row (a power of two <= 32 or a multiple of 32)
+  int rows_per_cta;
+};
+
+template <int L>
+struct Geo {
+  static constexpr int kLogE = (L + 2) / 2;
+  static constexpr int kE = 1 << kLogE;       // elements per thread
+  static constexpr int kP = L - kLogE;        // log2 threads per block
+  static constexpr int kTPB = 1 << kP;        // threads per block
+  static constexpr int kQ = kLogE - kP;       // low index bits kept in pass 2 (1 or 2)
+  static constexpr int kNC = kE / 8;          // 8-element chunks per thread in pass 1
+  static constexpr int kMaxThreads = kLogE >= 7 ? 256 : (kLogE == 6 ? 512 : 1024);
+  static_assert(kQ >= 1 && kQ <= 2, "pass-2 layout keeps one or two low bits");
+  static_assert(kP >= 2, "swizzle assumes at least four threads per block");
+};
+
+// ---------------------------------------------------------------------------
+// Loads of one 8-element chunk (16 bytes of bf16/f16, 32 bytes of f32).
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint4 ldg_nc_v4(const void* p) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
+__device__ __forceinline__ void bf16x2_to_f32(uint32_t w, float& lo, float& hi) {
+  lo = __uint_as_float(w << 16);
+  hi = __uint_as_float(w & 0xFFFF0000u);
+}
+
+__device__ __forceinline__ void f16x2_to_f32(uint32_t w, float& lo, float& hi) {
+  __half2 h;
+  *reinterpret_cast<uint32_t*>(&h) = w;
+  const float2 f = __half22float2(h);
+  lo = f.x;
+  hi = f.y;
+}
+
+__device__ __forceinline__ void load_chunk8(const __nv_bfloat16* p, float* v) {
+  const uint4 w = ldg_nc_v4(p);
+  bf16x2_to_f32(w.x, v[0], v[1]);
+  bf16x2_to_f32(w.y, v[2], v[3]);
+  bf16x2_to_f32(w.z, v[4], v[5]);
+  bf16x2_to_f32(w.w, v[6], v[7]);
+}
+
+__device__ __forceinline__ void load_chunk8(const __half* p, float* v) {
+  const uint4 w = ldg_nc_v4(p);
+  f16x2_to_f32(w.x, v[0], v[1]);
+  f16x2_to_f32(w.y, v[2], v[3]);
+  f16x2_to_f32(w.z, v[4], v[5]);
+  f16x2_to_f32(w.w, v[6], v[7]);
+}
+
+__device__ __forceinline__ void load_chunk8(const float* p, float* v) {
+  const uint4 a = ldg_nc_v4(p);
+  const uint4 b = ldg_nc_v4(p + 4);
+  v[0] = __uint_as_float(a.x); v[1] = __uint_as_float(a.y);
+  v[2] = __uint_as_float(a.z); v[3] = __uint_as_float(a.w);
+  v[4] = __uint_as_float(b.x); v[5] = __uint_as_float(b.y);
+  v[6] = __uint_as_float(b.z); v[7] = __uint_as_float(b.w);
+}
+
+// ---------------------------------------------------------------------------
+// In-register fast Walsh-Hadamard stages (Sylvester order: (a, b) -> (a+b, a-b)
+// for the pair of indices that differ in one bit, the lower index first).
+// ---------------------------------------------------------------------------
+template <int E, int BIT>
+__device__ __forceinline__ void fwht_stage(float (&v)[E]) {
+  constexpr int m = 1 << BIT;
+  if constexpr (BIT == 0) {
+#pragma unroll
+    for (int r = 0; r < E; r += 4) butterfly2(v[r], v[r + 2], v[r + 1], v[r + 3]);
+  } else {
+#pragma unroll
+    for (int r = 0; r < E; r += 2) {
+      if ((r & m) == 0) butterfly2(v[r], v[r + 1], v[r + m], v[r + m + 1]);
+    }
+  }
+}
+
+template <int E, int LO, int HI>
+__device__ __forceinline__ void fwht_bits(float (&v)[E]) {
+  if constexpr (LO < HI) {
+    fwht_stage<E, LO>(v);
+    fwht_bits<E, LO + 1, HI>(v);
+  }
+}
+
+// Swizzle of the row's fp32 transpose buffer: flips bits 2-4 of the element
+// index with higher bits so that both the pass-1 stores and the pass-2 loads of
+// a warp spread over the 32 banks. Bits >= 5 are untouched, so it is a bijection.
+template <int P>
+__device__ __forceinline__ int swz(int idx) {
+  return idx ^ (((idx >> 5) & 1) << 2) ^ (((idx >> (3 + P)) & 3) << 3);
+}
+
+// Reduction over aligned groups of W consecutive threads (W a power of two up
+// to 32, or a multiple of 32). All threads of the CTA must call it.
+template <bool kMax>
+__device__ __forceinline__ float group_reduce(float v, int W, float* scratch) {
+  const int lane = threadIdx.x & 31;
+  const int wl = W < 32 ? W : 32;
+  for (int o = wl >> 1; o > 0; o >>= 1) {
+    const float u = __shfl_xor_sync(0xFFFFFFFFu, v, o);
+    v = kMax ? fmaxf(v, u) : v + u;
+  }
+  if (W > 32) {
+    const int warp = threadIdx.x >> 5;
+    if (lane == 0) scratch[warp] = v;
+    __syncthreads();
+    const int nw = W >> 5;
+    const int first = (warp / nw) * nw;
+    float acc = kMax ? 0.f : 0.f;
+    for (int i = 0; i < nw; ++i) {
+      const float u = scratch[first + i];
+      acc = kMax ? fmaxf(acc, u) : acc + u;
+    }
+    v = acc;
+    __syncthreads();
+  }
+  return v;
+}
+
+// Round-to-nearest-even of x*inv as the integer held in the low mantissa bits
+// of fma(x, inv, 1.5 * 2^23 + 8) (the classic magic-number rounding: the
+// addend puts the result's ulp at 1). For |x*inv| <= 7 the low nibble is
+// rne(x*inv) + 8, the activation code.
+constexpr float kMagic8 = 12582920.0f;
+
+template <int L, typename Tin>
+__global__ void __launch_bounds__(Geo<L>::kMaxThreads) quantize_rows_kernel(const QuantArgs a) {
+  using GG = Geo<L>;
+  constexpr int E = GG::kE, P = GG::kP, TPB = GG::kTPB, Q = GG::kQ, NC = GG::kNC, LOGE = GG::kLogE;
+  constexpr int g = 1 << L;
+
+  extern __shared__ __align__(16) uint8_t smem[];
+  const bool rotate = (a.flags & OFFQ_ROTATE) != 0;
+  const bool offs = (a.flags & OFFQ_OFFSET) != 0;
+  const int R = a.rows_per_cta;
+  const int K = a.K;
+  float* buf = reinterpret_cast<float*>(smem);                                  // [R][K] fp32 (rotate)
+  uint8_t* cbuf = smem + (rotate ? static_cast<size_t>(R) * K * 4 : 0);         // [R][K/2] codes (rotate)
+  float* red = reinterpret_cast<float*>(cbuf + (rotate ? static_cast<size_t>(R) * (K / 2) : 0));
+
+  const int tid = threadIdx.x;
+  const int lrow = tid / a.tpr;
+  const int j = tid - lrow * a.tpr;
+  const int64_t row = static_cast<int64_t>(blockIdx.x) * R + lrow;
+  const bool row_ok = row < a.rows;
+  const bool active = row_ok && (j < a.G * TPB);
+  const int b = j / TPB;
+  const int t1 = j % TPB;
+
+  float v[E];
+  if (active) {
+    const int64_t t = row / a.H;
+    const int64_t h = row - t * a.H;
+    const Tin* p = static_cast<const Tin*>(a.x) + t * a.ld_t + h * a.ld_h + static_cast<int64_t>(b) * g + 8 * t1;
+#pragma unroll
+    for (int i = 0; i < NC; ++i) load_chunk8(p + i * 8 * TPB, &v[8 * i]);
+  } else {
+#pragma unroll
+    for (int r = 0; r < E; ++r) v[r] = 0.f;
+  }
+
+  float off = 0.f;
+  if (rotate) {
+    // Offset = x[block start] / sqrt(g); removing it first leaves the residual.
+    if (offs && t1 == 0) {
+      off = v[0];
+      v[0] = 0.f;
+    }
+    fwht_bits<E, 0, LOGE>(v);  // index bits {0,1,2} and {3+P, .., L-1}
+    float* rb = buf + static_cast<size_t>(lrow) * K + static_cast<size_t>(b) * g;
+    if (active) {
+#pragma unroll
+      for (int i = 0; i < NC; ++i) {
+        const int e0 = 8 * t1 + 8 * TPB * i;
+        *reinterpret_cast<float4*>(rb + swz<P>(e0)) = make_float4(v[8 * i], v[8 * i + 1], v[8 * i + 2], v[8 * i + 3]);
+        *reinterpret_cast<float4*>(rb + swz<P>(e0 + 4)) =
+            make_float4(v[8 * i + 4], v[8 * i + 5], v[8 * i + 6], v[8 * i + 7]);
+      }
+    }
+    __syncthreads();
+    if (active) {
+#pragma unroll
+      for (int hi = 0; hi < (1 << P); ++hi) {
+        const int e = ((t1 & ((1 << (3 - Q)) - 1)) << Q) | (hi << 3) | ((t1 >> (3 - Q)) << (3 + P));
+        if constexpr (Q == 2) {
+          const float4 f = *reinterpret_cast<const float4*>(rb + swz<P>(e));
+          v[4 * hi] = f.x; v[4 * hi + 1] = f.y; v[4 * hi + 2] = f.z; v[4 * hi + 3] = f.w;
+        } else {
+          const float2 f = *reinterpret_cast<const float2*>(rb + swz<P>(e));
+          v[2 * hi] = f.x; v[2 * hi + 1] = f.y;
+        }
+      }
+    }
+    fwht_bits<E, Q, LOGE>(v);  // index bits {3, .., 3+P-1}
+  } else if (offs) {
+    float s = 0.f;
+#pragma unroll
+    for (int r = 0; r < E; ++r) s += v[r];
+    s = group_reduce<false>(s, TPB, red);
+    off = s * (1.0f / static_cast<float>(g));
+#pragma unroll
+    for (int r = 0; r < E; ++r) v[r] -= off;
+  }
+
+  // Per-row absmax of the residual.
+  float m = 0.f;
+#pragma unroll
+  for (int r = 0; r < E; ++r) m = fmaxf(m, fabsf(v[r]));
+  m = group_reduce<true>(m, a.tpr, red);
+  const float inv = m > 0.f ? __fdiv_rn(7.0f, m) : 0.f;
+
+#pragma unroll
+  for (int r = 0; r < E; r += 2) fma2(v[r], v[r + 1], inv, kMagic8);
+
+  if (rotate) {
+    if (active) {
+      uint8_t* crow = cbuf + static_cast<size_t>(lrow) * (K / 2) + static_cast<size_t>(b) * (g / 2);
+#pragma unroll
+      for (int hi = 0; hi < (1 << P); ++hi) {
+        const int e = ((t1 & ((1 << (3 - Q)) - 1)) << Q) | (hi << 3) | ((t1 >> (3 - Q)) << (3 + P));
+        if constexpr (Q == 2) {
+          const uint32_t u0 = __float_as_uint(v[4 * hi]) & 0xFu, u1 = __float_as_uint(v[4 * hi + 1]) & 0xFu;
+          const uint32_t u2 = __float_as_uint(v[4 * hi + 2]) & 0xFu, u3 = __float_as_uint(v[4 * hi + 3]) & 0xFu;
+          *reinterpret_cast<uint16_t*>(crow + e / 2) =
+              static_cast<uint16_t>(u0 | (u1 << 4) | (u2 << 8) | (u3 << 12));
+        } else {
+          const uint32_t u0 = __float_as_uint(v[2 * hi]) & 0xFu, u1 = __float_as_uint(v[2 * hi + 1]) & 0xFu;
+          crow[e / 2] = static_cast<uint8_t>(u0 | (u1 << 4));
+        }
+      }
+    }
+    __syncthreads();
+    const int64_t row0 = static_cast<int64_t>(blockIdx.x) * R;
+    const int nrows = static_cast<int>(a.rows - row0 < R ? a.rows - row0 : R);
+    const int cpr = K / 32;  // 16-byte chunks of codes per row
+    for (int c = tid; c < nrows * cpr; c += blockDim.x) {
+      const int rr = c / cpr, cc = c - rr * cpr;
+      const uint4 w = *reinterpret_cast<const uint4*>(cbuf + static_cast<size_t>(rr) * (K / 2) + cc * 16);
+      *reinterpret_cast<uint4*>(a.codes + (row0 + rr) * (K / 2) + cc * 16) = w;
+    }
+  } else if (active) {
+    uint8_t* crow = a.codes + row * (K / 2) + static_cast<int64_t>(b) * (g / 2);
+#pragma unroll
+    for (int i = 0; i < NC; ++i) {
+      uint32_t w = 0;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) w |= (__float_as_uint(v[8 * i + e]) & 0xFu) << (4 * e);
+      *reinterpret_cast<uint32_t*>(crow + 4 * t1 + 4 * TPB * i) = w;
+    }
+  }
+
+  if (row_ok && j == 0) a.scale[row] = m * a.scale_mul;
+  if (active && t1 == 0 && a.offset != nullptr) {
+    a.offset[row * a.G + b] = offs ? (rotate ? off * a.inv_sqrt_g : off) : 0.f;
+  }
+}
+
+template <int L, typename Tin>
+int launch_quant(QuantArgs a, cudaStream_t stream) {
+  using GG = Geo<L>;
+  const int raw = a.G * GG::kTPB;
+  int tpr = 1;
+  if (raw <= 32) {
+    while (tpr < raw) tpr <<= 1;
+  } else {
+    tpr = (raw + 31) / 32 * 32;
+  }
+  if (tpr > GG::kMaxThreads) return OFFQ_ERR_UNSUPPORTED;
+  const bool rotate = (a.flags & OFFQ_ROTATE) != 0;
+  const size_t row_smem = rotate ? static_cast<size_t>(a.K) * 4 + a.K / 2 : 0;
+  int R = std::max(1, std::min(GG::kMaxThreads, 256) / tpr);
+  while (R > 1 && static_cast<size_t>(R) * row_smem > 64 * 1024) --R;
+  a.tpr = tpr;
+  a.rows_per_cta = R;
+  const size_t smem = static_cast<size_t>(R) * row_smem + 32 * sizeof(float);
+  auto kern = quantize_rows_kernel<L, Tin>;
+  if (smem > 48 * 1024) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
+        cudaSuccess)
+      return OFFQ_ERR_CUDA;
+  }
+  const int64_t grid = (a.rows + R - 1) / R;
+  if (grid > 0x7FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
+  kern<<<static_cast<unsigned>(grid), R * tpr, smem, stream>>>(a);
+  return launch_status();
+}
+
+template <typename Tin>
+int dispatch_g(const QuantArgs& a, int g, cudaStream_t s) {
+  switch (g) {
+    case 32: return launch_quant<5, Tin>(a, s);
+    case 64: return launch_quant<6, Tin>(a, s);
+    case 128: return launch_quant<7, Tin>(a, s);
+    case 256: return launch_quant<8, Tin>(a, s);
+    case 512: return launch_quant<9, Tin>(a, s);
+    case 1024: return launch_quant<10, Tin>(a, s);
+    case 2048: return launch_quant<11, Tin>(a, s);
+    case 4096: return launch_quant<12, Tin>(a, s);
+    case 8192: return launch_quant<13, Tin>(a, s);
+    default: return OFFQ_ERR_UNSUPPORTED;
+  }
+}
+
+int run_quant(QuantArgs a, int dtype, int g, cudaStream_t s) {
+  const double isg = (a.flags & OFFQ_ROTATE) ? 1.0 / std::sqrt(static_cast<double>(g)) : 1.0;
+  a.inv_sqrt_g = static_cast<float>(isg);
+  a.scale_mul = static_cast<float>(isg / 7.0);
+  switch (dtype) {
+    case OFFQ_BF16: return dispatch_g<__nv_bfloat16>(a, g, s);
+    case OFFQ_F16: return dispatch_g<__half>(a, g, s);
+    case OFFQ_F32: return dispatch_g<float>(a, g, s);
+    default: return OFFQ_ERR_INVALID_ARG;
+  }
+}
+
+// K and g rules shared by the row quantizers.
+int check_row_shape(int64_t K, int32_t g) {
+  if (!is_pow2(g) || g < 32 || g > 8192) return OFFQ_ERR_INVALID_ARG;
+  if (K <= 0 || K % g != 0 || K % 32 != 0) return OFFQ_ERR_INVALID_ARG;
+  if (K > kMaxQuantK || K > 128 * static_cast<int64_t>(g)) return OFFQ_ERR_UNSUPPORTED;
+  return OFFQ_OK;
+}
+
+// Offline: activation-format codes (q + 8) -> weight format, in place, plus the
+// integer block row sums R[b][n]. One thread per (row, block).
+__global__ void weight_repack_kernel(uint8_t* __restrict__ codes, float* __restrict__ rowsum, int64_t N, int K,
+                                     int g) {
+  const int G = K / g;
+  const int64_t id = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (id >= N * G) return;
+  const int64_t n = id / G;
+  const int b = static_cast<int>(id - n * G);
+  uint32_t* w = reinterpret_cast<uint32_t*>(codes + n * (K / 2) + static_cast<int64_t>(b) * (g / 2));
+  int sum = 0;
+  for (int i = 0; i < g / 8; ++i) {
+    const uint32_t u = w[i];
+    uint32_t mag[8], neg[8];
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      const int q = static_cast<int>((u >> (4 * c)) & 0xFu) - 8;
+      sum += q;
+      mag[c] = static_cast<uint32_t>(q < 0 ? -q : q);
+      neg[c] = q < 0 ? 1u : 0u;
+    }
+    uint32_t out = 0;
+#pragma unroll
+    for (int jj = 0; jj < 4; ++jj) {
+      const uint32_t byte = mag[2 * jj] | (neg[2 * jj] << 7) | (mag[2 * jj + 1] << 4) | (neg[(2 * jj + 7) & 7] << 3);
+      out |= byte << (8 * jj);
+    }
+    w[i] = out;
+  }
+  rowsum[static_cast<int64_t>(b) * N + n] = static_cast<float>(sum);
+}
+
+}  // namespace
+
+extern "C" int offq_quantize_act(const void* x, int x_dtype, int64_t T, int64_t K, int64_t ldx, int32_t g,
+                                 int32_t flags, uint8_t* codes, float* scale, float* offset, void* stream) {
+  const int eb = elem_bytes(x_dtype);
+  if (eb == 0 || T < 0 || (flags & ~(OFFQ_ROTATE | OFFQ_OFFSET)) != 0) return OFFQ_ERR_INVALID_ARG;
+  const int st = check_row_shape(K, g);
+  if (st != OFFQ_OK) return st;
+  if (ldx < K) return OFFQ_ERR_INVALID_ARG;
+  if (T == 0) return OFFQ_OK;
+  if (x == nullptr || codes == nullptr || scale == nullptr) return OFFQ_ERR_INVALID_ARG;
+  if ((flags & OFFQ_OFFSET) && offset == nullptr) return OFFQ_ERR_INVALID_ARG;
+  if (!aligned(x, 16) || (ldx * eb) % 16 != 0 || !aligned(codes, 16) || !aligned(scale, 4) ||
+      (offset != nullptr && !aligned(offset, 4)))
+    return OFFQ_ERR_MISALIGNED;
+  QuantArgs a{};
+  a.x = x;
+  a.ld_t = ldx;
+  a.ld_h = 0;
+  a.rows = T;
+  a.H = 1;
+  a.K = static_cast<int>(K);
+  a.G = static_cast<int>(K / g);
+  a.flags = flags;
+  a.codes = codes;
+  a.scale = scale;
+  a.offset = offset;
+  return run_quant(a, x_dtype, g, static_cast<cudaStream_t>(stream));
+}
+
+extern "C" int offq_kv4_quantize(const void* kv, int dtype, int64_t T, int32_t H, int32_t head_dim,
+                                 int64_t ld_token, int32_t flags, uint8_t* codes, float* scale, float* offset,
+                                 void* stream) {
+  const int eb = elem_bytes(dtype);
+  if (eb == 0 || T < 0 || H < 1 || (flags & ~(OFFQ_ROTATE | OFFQ_OFFSET)) != 0) return OFFQ_ERR_INVALID_ARG;
+  const int st = check_row_shape(head_dim, head_dim);
+  if (st != OFFQ_OK) return st;
+  if (ld_token < static_cast<int64_t>(H) * head_dim) return OFFQ_ERR_INVALID_ARG;
+  if (T == 0) return OFFQ_OK;
+  if (kv == nullptr || codes == nullptr || scale == nullptr) return OFFQ_ERR_INVALID_ARG;
+  if ((flags & OFFQ_OFFSET) && offset == nullptr) return OFFQ_ERR_INVALID_ARG;
+  if (!aligned(kv, 16) || (ld_token * eb) % 16 != 0 || !aligned(codes, 16) || !aligned(scale, 4) ||
+      (offset != nullptr && !aligned(offset, 4)))
+    return OFFQ_ERR_MISALIGNED;
+  QuantArgs a{};
+  a.x = kv;
+  a.ld_t = ld_token;
+  a.ld_h = head_dim;
+  a.rows = T * H;
+  a.H = H;
+  a.K = head_dim;
+  a.G = 1;
+  a.flags = flags;
+  a.codes = codes;
+  a.scale = scale;
+  a.offset = offset;
+  return run_quant(a, dtype, head_dim, static_cast<cudaStream_t>(stream));
+}
+
+extern "C" int offq_prepare_weight(const void* w, int dtype, int64_t N, int64_t K, int32_t g, int32_t rotate,
+                                   uint8_t* w_codes, float* w_scale, float* w_offsum, void* stream) {
+  const int eb = elem_bytes(dtype);
+  if (eb == 0 || N < 1) return OFFQ_ERR_INVALID_ARG;
+  const int st = check_row_shape(K, g);
+  if (st != OFFQ_OK) return st;
+  if (w == nullptr || w_codes == nullptr || w_scale == nullptr || w_offsum == nullptr) return OFFQ_ERR_INVALID_ARG;
+  if (!aligned(w, 16) || (K * eb) % 16 != 0 || !aligned(w_codes, 16) || !aligned(w_scale, 4) ||
+      !aligned(w_offsum, 4))
+    return OFFQ_ERR_MISALIGNED;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  QuantArgs a{};
+  a.x = w;
+  a.ld_t = K;
+  a.ld_h = 0;
+  a.rows = N;
+  a.H = 1;
+  a.K = static_cast<int>(K);
+  a.G = static_cast<int>(K / g);
+  a.flags = rotate ? OFFQ_ROTATE : 0;
+  a.codes = w_codes;
+  a.scale = w_scale;
+  a.offset = nullptr;
+  int rc = run_quant(a, dtype, g, s);
+  if (rc != OFFQ_OK) return rc;
+  const int64_t units = N * (K / g);
+  const int threads = 256;
+  weight_repack_kernel<<<static_cast<unsigned>((units + threads - 1) / threads), threads, 0, s>>>(
+      w_codes, w_offsum, N, static_cast<int>(K), g);
+  return launch_status();
+}

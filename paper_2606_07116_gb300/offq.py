@@ -1,0 +1,217 @@
+"""Python binding of liboffq.so (the OffQ W4A4 linear path on GB300).
+
+The functions named ``offq_*`` mirror the C ABI in ``include/offq.h`` one to
+one: they take torch CUDA tensors, pass their device pointers, sizes and the
+current CUDA stream to the library, and raise :class:`OffqError` on a non-zero
+status. All computation happens in the library's kernels; torch supplies device
+memory and streams only. The helpers without the prefix (``quantize_act``,
+``w4a4_linear``, ...) allocate the outputs with torch and call the same entry
+points.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+from typing import Optional, Tuple
+
+import torch
+
+from . import build as _build
+
+OFFQ_OK = 0
+OFFQ_ERR_INVALID_ARG = -1
+OFFQ_ERR_UNSUPPORTED = -2
+OFFQ_ERR_MISALIGNED = -3
+OFFQ_ERR_CUDA = -4
+OFFQ_ERR_TIMEOUT = -5
+
+OFFQ_F32, OFFQ_BF16, OFFQ_F16 = 0, 1, 2
+OFFQ_ROTATE, OFFQ_OFFSET = 1, 2
+
+_DTYPE_CODE = {torch.float32: OFFQ_F32, torch.bfloat16: OFFQ_BF16, torch.float16: OFFQ_F16}
+_CODE_DTYPE = {v: k for k, v in _DTYPE_CODE.items()}
+
+_c_vp = ctypes.c_void_p
+_c_i64 = ctypes.c_int64
+_c_i32 = ctypes.c_int32
+_c_int = ctypes.c_int
+
+_SIGNATURES = {
+    "offq_quantize_act": (_c_int, [_c_vp, _c_int, _c_i64, _c_i64, _c_i64, _c_i32, _c_i32, _c_vp, _c_vp, _c_vp, _c_vp]),
+    "offq_w4a4_linear": (_c_int, [_c_vp, _c_vp, _c_vp, _c_i64, _c_i64, _c_i64, _c_i32, _c_vp, _c_vp, _c_vp, _c_vp,
+                                  _c_int, _c_i64, _c_vp, _c_vp]),
+    "offq_kv4_quantize": (_c_int, [_c_vp, _c_int, _c_i64, _c_i32, _c_i32, _c_i64, _c_i32, _c_vp, _c_vp, _c_vp, _c_vp]),
+    "offq_prepare_weight": (_c_int, [_c_vp, _c_int, _c_i64, _c_i64, _c_i32, _c_i32, _c_vp, _c_vp, _c_vp, _c_vp]),
+    "offq_get_device_status": (_c_int, [_c_vp]),
+    "offq_status_string": (ctypes.c_char_p, [_c_int]),
+    "offq_abi_version": (_c_int, []),
+}
+
+_lib = None
+
+
+class OffqError(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        self.status = status
+        super().__init__(f"{fn} failed: {status_string(status)} ({status})")
+
+
+def library_path() -> str:
+    return _build.LIB_PATH
+
+
+def load_library(path: Optional[str] = None) -> ctypes.CDLL:
+    """Loads liboffq.so (raises if it was not built: there is no fallback)."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    p = path or library_path()
+    if not os.path.exists(p):
+        raise RuntimeError(f"liboffq.so not found at {p}; build it with "
+                           "paper_2606_07116_gb300.build.build() (no CPU fallback exists)")
+    lib = ctypes.CDLL(p)
+    for name, (res, args) in _SIGNATURES.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    if path is None:
+        _lib = lib
+    return lib
+
+
+def declared_symbols(header: Optional[str] = None):
+    """Names of the functions include/offq.h declares."""
+    header = header or os.path.join(_build.INCLUDE, "offq.h")
+    with open(header) as f:
+        text = f.read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(offq_[a-z0-9_]+)\s*\(", text)))
+
+
+def status_string(status: int) -> str:
+    return load_library().offq_status_string(status).decode()
+
+
+def abi_version() -> int:
+    return load_library().offq_abi_version()
+
+
+def _check(fn: str, rc: int):
+    if rc != OFFQ_OK:
+        raise OffqError(fn, rc)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("tensors passed to liboffq must live on a CUDA device")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    if isinstance(stream, torch.cuda.Stream):
+        return ctypes.c_void_p(stream.cuda_stream)
+    return ctypes.c_void_p(int(stream))
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype not in _DTYPE_CODE:
+        raise ValueError(f"unsupported dtype {t.dtype}")
+    return _DTYPE_CODE[t.dtype]
+
+
+# ---------------------------------------------------------------------------
+# One-to-one wrappers of the C ABI.
+# ---------------------------------------------------------------------------
+
+def offq_quantize_act(x: torch.Tensor, T: int, K: int, ldx: int, g: int, flags: int,
+                      codes: torch.Tensor, scale: torch.Tensor, offset: Optional[torch.Tensor],
+                      stream=None) -> None:
+    _check("offq_quantize_act", load_library().offq_quantize_act(
+        _ptr(x), _dtype_code(x), T, K, ldx, g, flags, _ptr(codes), _ptr(scale), _ptr(offset), _stream(stream)))
+
+
+def offq_w4a4_linear(a_codes: torch.Tensor, a_scale: torch.Tensor, a_offset: Optional[torch.Tensor],
+                     T: int, N: int, K: int, g: int, w_codes: torch.Tensor, w_scale: torch.Tensor,
+                     w_offsum: torch.Tensor, out: torch.Tensor, ldo: int,
+                     acc_debug: Optional[torch.Tensor] = None, stream=None) -> None:
+    _check("offq_w4a4_linear", load_library().offq_w4a4_linear(
+        _ptr(a_codes), _ptr(a_scale), _ptr(a_offset), T, N, K, g, _ptr(w_codes), _ptr(w_scale),
+        _ptr(w_offsum), _ptr(out), _dtype_code(out), ldo, _ptr(acc_debug), _stream(stream)))
+
+
+def offq_kv4_quantize(kv: torch.Tensor, T: int, H: int, head_dim: int, ld_token: int, flags: int,
+                      codes: torch.Tensor, scale: torch.Tensor, offset: Optional[torch.Tensor],
+                      stream=None) -> None:
+    _check("offq_kv4_quantize", load_library().offq_kv4_quantize(
+        _ptr(kv), _dtype_code(kv), T, H, head_dim, ld_token, flags, _ptr(codes), _ptr(scale), _ptr(offset),
+        _stream(stream)))
+
+
+def offq_prepare_weight(w: torch.Tensor, N: int, K: int, g: int, rotate: bool, w_codes: torch.Tensor,
+                        w_scale: torch.Tensor, w_offsum: torch.Tensor, stream=None) -> None:
+    _check("offq_prepare_weight", load_library().offq_prepare_weight(
+        _ptr(w), _dtype_code(w), N, K, g, 1 if rotate else 0, _ptr(w_codes), _ptr(w_scale), _ptr(w_offsum),
+        _stream(stream)))
+
+
+def offq_get_device_status(stream=None) -> int:
+    return load_library().offq_get_device_status(_stream(stream))
+
+
+# ---------------------------------------------------------------------------
+# Allocating helpers (torch allocates; the entry points above compute).
+# ---------------------------------------------------------------------------
+
+def quantize_act(x: torch.Tensor, g: int, rotate: bool = True, offset: bool = True,
+                 stream=None) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    T, K = x.shape
+    codes = torch.empty((T, K // 2), dtype=torch.uint8, device=x.device)
+    scale = torch.empty((T,), dtype=torch.float32, device=x.device)
+    off = torch.empty((T, K // g), dtype=torch.float32, device=x.device)
+    flags = (OFFQ_ROTATE if rotate else 0) | (OFFQ_OFFSET if offset else 0)
+    offq_quantize_act(x, T, K, x.stride(0), g, flags, codes, scale, off, stream)
+    return codes, scale, off
+
+
+def kv4_quantize(kv: torch.Tensor, rotate: bool = True, offset: bool = True,
+                 stream=None) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    T, H, hd = kv.shape
+    if kv.stride(2) != 1 or kv.stride(1) != hd:
+        raise ValueError("heads of a token must be contiguous")
+    codes = torch.empty((T, H, hd // 2), dtype=torch.uint8, device=kv.device)
+    scale = torch.empty((T, H), dtype=torch.float32, device=kv.device)
+    off = torch.empty((T, H), dtype=torch.float32, device=kv.device)
+    flags = (OFFQ_ROTATE if rotate else 0) | (OFFQ_OFFSET if offset else 0)
+    offq_kv4_quantize(kv, T, H, hd, kv.stride(0), flags, codes, scale, off, stream)
+    return codes, scale, off
+
+
+def prepare_weight(w: torch.Tensor, g: int, rotate: bool = True,
+                   stream=None) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    N, K = w.shape
+    w = w.contiguous()
+    codes = torch.empty((N, K // 2), dtype=torch.uint8, device=w.device)
+    scale = torch.empty((N,), dtype=torch.float32, device=w.device)
+    rowsum = torch.empty((K // g, N), dtype=torch.float32, device=w.device)
+    offq_prepare_weight(w, N, K, g, rotate, codes, scale, rowsum, stream)
+    return codes, scale, rowsum
+
+
+def w4a4_linear(a_codes: torch.Tensor, a_scale: torch.Tensor, a_offset: Optional[torch.Tensor],
+                w_codes: torch.Tensor, w_scale: torch.Tensor, w_offsum: torch.Tensor, g: int,
+                out_dtype: torch.dtype = torch.bfloat16, out: Optional[torch.Tensor] = None,
+                acc_debug: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    T = a_codes.shape[0]
+    K = a_codes.shape[1] * 2
+    N = w_codes.shape[0]
+    if out is None:
+        out = torch.empty((T, N), dtype=out_dtype, device=a_codes.device)
+    offq_w4a4_linear(a_codes, a_scale, a_offset, T, N, K, g, w_codes, w_scale, w_offsum, out, out.stride(0),
+                     acc_debug, stream)
+    return out

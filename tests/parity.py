@@ -1,0 +1,114 @@
+"""Comparison helpers for the GPU-vs-oracle parity tests.
+
+Tolerances follow from the arithmetic of the kernels (fp32, unit roundoff
+u = 2^-24), never from observed differences:
+
+* Codes. The kernel decides each code in fp32 and the oracle in float64, so a
+  code may differ only where the oracle's r/s lies within the fp32 error of a
+  rounding tie; mismatches must be +-1, within TIE_WINDOW code units of a
+  half-integer, and at most 1e-4 of all codes (the stated bound).
+* Scales and offsets. The kernel's transform is a radix-2 tree of L = log2(g)
+  fp32 additions per output, so each rotated value carries an absolute error of
+  at most L u sum|x| over its block; the scale inherits that relative to max|r|.
+* GEMM outputs. Integer accumulators are exact. The epilogue is a chain of G+2
+  fp32 multiply-adds whose error is bounded by (G + 4) u times the sum of the
+  magnitudes of its terms; a bf16 / fp16 result adds half an ulp of its own
+  format (relative 2^-8 / 2^-11).
+"""
+
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+U32 = 2.0 ** -24
+TIE_WINDOW = 1e-3
+MAX_MISMATCH_FRACTION = 1e-4
+
+
+def check_codes(q_gpu: np.ndarray, q_ref: np.ndarray, r_ref: np.ndarray, s_ref: np.ndarray, what: str = "codes"):
+    """q_* int codes [rows, K]; r_ref residual [rows, K]; s_ref scale [rows] (oracle, float64)."""
+    q_gpu = np.asarray(q_gpu, dtype=np.int64)
+    q_ref = np.asarray(q_ref, dtype=np.int64)
+    assert q_gpu.shape == q_ref.shape, (q_gpu.shape, q_ref.shape)
+    diff = q_gpu - q_ref
+    mism = diff != 0
+    n = int(mism.sum())
+    if n == 0:
+        return 0
+    assert np.all(np.abs(diff) <= 1), f"{what}: a code differs by more than 1"
+    s = np.broadcast_to(np.asarray(s_ref, np.float64).reshape(-1, *([1] * (q_ref.ndim - 1))), q_ref.shape)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        z = np.where(s > 0, np.asarray(r_ref, np.float64) / s, 0.0)
+    zm = np.abs(z[mism])
+    dist = np.abs(zm - np.floor(zm) - 0.5)
+    assert np.all(dist < TIE_WINDOW), f"{what}: mismatch away from a rounding tie (min dist {dist.max():.3g})"
+    frac = n / q_ref.size
+    assert frac <= MAX_MISMATCH_FRACTION, f"{what}: {n} codes differ ({frac:.2e} > {MAX_MISMATCH_FRACTION})"
+    return n
+
+
+def rotation_abs_error(x: np.ndarray, g: int, rotate: bool) -> np.ndarray:
+    """Per-row bound on the absolute fp32 error of an unnormalised rotated value."""
+    x = np.abs(np.asarray(x, np.float64))
+    T, K = x.shape
+    blk = x.reshape(T, K // g, g).sum(axis=2).max(axis=1)
+    L = int(math.log2(g)) if rotate else 0
+    return (L + 2) * U32 * blk
+
+
+def check_scales(s_gpu, s_ref, x, g, rotate, what="scale"):
+    s_gpu = np.asarray(s_gpu, np.float64)
+    s_ref = np.asarray(s_ref, np.float64)
+    norm = math.sqrt(g) if rotate else 1.0
+    err_u = rotation_abs_error(x, g, rotate)          # on the unnormalised residual
+    tol = err_u / (7.0 * norm) + 4 * U32 * np.abs(s_ref)
+    bad = np.abs(s_gpu - s_ref) > tol
+    assert not np.any(bad), f"{what}: {bad.sum()} rows out of tolerance; worst " \
+                            f"{np.max(np.abs(s_gpu - s_ref) / np.maximum(tol, 1e-300)):.3g}x"
+
+
+def check_offsets(o_gpu, o_ref, x, g, rotate, what="offset"):
+    o_gpu = np.asarray(o_gpu, np.float64)
+    o_ref = np.asarray(o_ref, np.float64)
+    x = np.abs(np.asarray(x, np.float64))
+    T, K = x.shape
+    if rotate:
+        tol = 4 * U32 * np.abs(o_ref)   # x[0] * fl(1/sqrt(g)): two roundings
+    else:
+        tol = (int(math.log2(g)) + 2) * U32 * x.reshape(T, K // g, g).sum(axis=2) / g + 2 * U32 * np.abs(o_ref)
+    bad = np.abs(o_gpu - o_ref) > tol
+    assert not np.any(bad), f"{what}: {bad.sum()} offsets out of tolerance"
+
+
+def epilogue_terms(acc_raw, s_a, o, s_w, R):
+    """Magnitudes the fp32 epilogue adds up (float64), for its error bound."""
+    s_a = np.asarray(s_a, np.float64)
+    s_w = np.abs(np.asarray(s_w, np.float64))
+    o = np.asarray(o, np.float64)
+    o_shift = np.abs(o - 8.0 * s_a[:, None])
+    return s_w[None, :] * (np.abs(s_a[:, None] * np.asarray(acc_raw, np.float64)) + o_shift @ np.abs(R))
+
+
+def check_outputs(y_gpu, y_ref, terms, G, out_dtype: str, what="y"):
+    y_gpu = np.asarray(y_gpu, np.float64)
+    y_ref = np.asarray(y_ref, np.float64)
+    tol = (G + 4) * U32 * terms + 1e-30
+    if out_dtype == "bf16":
+        tol = tol + 2.0 ** -8 * np.abs(y_ref)
+    elif out_dtype == "f16":
+        tol = tol + 2.0 ** -11 * np.abs(y_ref) + 2.0 ** -25
+    err = np.abs(y_gpu - y_ref)
+    bad = err > tol
+    assert not np.any(bad), f"{what}: {bad.sum()} of {bad.size} outputs out of tolerance; worst " \
+                            f"{np.max(err / tol):.3g}x the bound"
+    return float(np.max(err / np.maximum(np.abs(y_ref), 1e-2 * np.sqrt(np.mean(y_ref ** 2)) + 1e-30)))
+
+
+def max_rel_err_floored(y_gpu, y_ref):
+    """max |y - y_ref| / max(|y_ref|, 1e-2 rms(y_ref)) (elementwise relative error with a floor)."""
+    y_gpu = np.asarray(y_gpu, np.float64)
+    y_ref = np.asarray(y_ref, np.float64)
+    floor = 1e-2 * np.sqrt(np.mean(y_ref ** 2)) + 1e-30
+    return float(np.max(np.abs(y_gpu - y_ref) / np.maximum(np.abs(y_ref), floor)))

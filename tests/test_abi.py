@@ -1,0 +1,101 @@
+"""The C-ABI library loads, exports every symbol include/offq.h declares, and
+rejects bad arguments on the host (no GPU needed: no call here reaches a
+CUDA runtime function)."""
+
+import ctypes
+
+import pytest
+
+from paper_2606_07116_gb300 import build as B
+from paper_2606_07116_gb300 import offq as Q
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return Q.load_library()
+
+
+def test_exports_every_declared_symbol(lib):
+    declared = Q.declared_symbols()
+    assert {"offq_quantize_act", "offq_w4a4_linear", "offq_kv4_quantize", "offq_prepare_weight",
+            "offq_get_device_status", "offq_status_string", "offq_abi_version"} <= set(declared)
+    for name in declared:
+        assert hasattr(lib, name), name
+
+
+def test_status_strings_and_version(lib):
+    assert Q.abi_version() == 1
+    for code, name in [(0, "OFFQ_OK"), (-1, "OFFQ_ERR_INVALID_ARG"), (-2, "OFFQ_ERR_UNSUPPORTED"),
+                       (-3, "OFFQ_ERR_MISALIGNED"), (-4, "OFFQ_ERR_CUDA"), (-5, "OFFQ_ERR_TIMEOUT")]:
+        assert Q.status_string(code) == name
+    assert Q.status_string(12345) == "OFFQ_UNKNOWN_STATUS"
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    with pytest.raises(RuntimeError):
+        Q.load_library(str(tmp_path / "nope.so"))
+
+
+P = ctypes.c_void_p
+A16 = P(0x10000)      # a 16-byte aligned (never dereferenced) address
+A8 = P(0x10008)       # only 8-byte aligned
+
+
+def quant(lib, x=A16, dt=Q.OFFQ_BF16, T=4, K=1024, ldx=1024, g=256, flags=3, codes=A16, scale=A16, off=A16):
+    return lib.offq_quantize_act(x, dt, T, K, ldx, g, flags, codes, scale, off, None)
+
+
+def test_quantize_argument_checks(lib):
+    assert quant(lib, g=33) == Q.OFFQ_ERR_INVALID_ARG          # g not a power of two
+    assert quant(lib, g=16) == Q.OFFQ_ERR_INVALID_ARG          # g below 32
+    assert quant(lib, g=16384, K=16384) == Q.OFFQ_ERR_INVALID_ARG
+    assert quant(lib, K=1000) == Q.OFFQ_ERR_INVALID_ARG        # g does not divide K
+    assert quant(lib, K=0) == Q.OFFQ_ERR_INVALID_ARG
+    assert quant(lib, K=65536, ldx=65536) == Q.OFFQ_ERR_UNSUPPORTED
+    assert quant(lib, g=32, K=8192, ldx=8192) == Q.OFFQ_ERR_UNSUPPORTED  # K > 128 g
+    assert quant(lib, ldx=1000) == Q.OFFQ_ERR_INVALID_ARG      # ldx < K
+    assert quant(lib, dt=7) == Q.OFFQ_ERR_INVALID_ARG
+    assert quant(lib, flags=4) == Q.OFFQ_ERR_INVALID_ARG
+    assert quant(lib, T=-1) == Q.OFFQ_ERR_INVALID_ARG
+    assert quant(lib, x=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert quant(lib, off=None) == Q.OFFQ_ERR_INVALID_ARG      # OFFSET needs an offset buffer
+    assert quant(lib, x=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert quant(lib, codes=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert quant(lib, ldx=1028) == Q.OFFQ_ERR_MISALIGNED       # row pitch not a multiple of 16 bytes
+    assert quant(lib, T=0) == Q.OFFQ_OK                        # nothing to do, nothing launched
+    assert quant(lib, T=0, x=None, codes=None) == Q.OFFQ_OK
+
+
+def gemm(lib, a=A16, sa=A16, oa=A16, T=8, N=64, K=1024, g=256, w=A16, sw=A16, R=A16, out=A16, dt=Q.OFFQ_BF16,
+         ldo=64, dbg=None):
+    return lib.offq_w4a4_linear(a, sa, oa, T, N, K, g, w, sw, R, out, dt, ldo, dbg, None)
+
+
+def test_gemm_argument_checks(lib):
+    assert gemm(lib, g=100) == Q.OFFQ_ERR_INVALID_ARG
+    assert gemm(lib, K=1000) == Q.OFFQ_ERR_INVALID_ARG
+    assert gemm(lib, N=0) == Q.OFFQ_ERR_INVALID_ARG
+    assert gemm(lib, ldo=32) == Q.OFFQ_ERR_INVALID_ARG
+    assert gemm(lib, dt=9) == Q.OFFQ_ERR_INVALID_ARG
+    assert gemm(lib, K=131072, g=4096) == Q.OFFQ_ERR_UNSUPPORTED
+    assert gemm(lib, K=32768, g=32) == Q.OFFQ_ERR_UNSUPPORTED   # more offset blocks than the epilogue stages
+    assert gemm(lib, w=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert gemm(lib, a=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert gemm(lib, out=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert gemm(lib, ldo=65) == Q.OFFQ_ERR_MISALIGNED
+    assert gemm(lib, T=0) == Q.OFFQ_OK
+
+
+def test_kv_and_weight_argument_checks(lib):
+    kv = lib.offq_kv4_quantize
+    assert kv(A16, Q.OFFQ_BF16, 4, 0, 128, 128, 3, A16, A16, A16, None) == Q.OFFQ_ERR_INVALID_ARG    # H = 0
+    assert kv(A16, Q.OFFQ_BF16, 4, 8, 96, 768, 3, A16, A16, A16, None) == Q.OFFQ_ERR_INVALID_ARG     # head_dim
+    assert kv(A16, Q.OFFQ_BF16, 4, 8, 128, 512, 3, A16, A16, A16, None) == Q.OFFQ_ERR_INVALID_ARG    # ld_token
+    assert kv(A8, Q.OFFQ_BF16, 4, 8, 128, 1024, 3, A16, A16, A16, None) == Q.OFFQ_ERR_MISALIGNED
+    assert kv(A16, Q.OFFQ_BF16, 0, 8, 128, 1024, 3, A16, A16, A16, None) == Q.OFFQ_OK
+    pw = lib.offq_prepare_weight
+    assert pw(A16, Q.OFFQ_F32, 0, 1024, 256, 1, A16, A16, A16, None) == Q.OFFQ_ERR_INVALID_ARG      # N = 0
+    assert pw(A16, Q.OFFQ_F32, 8, 1000, 256, 1, A16, A16, A16, None) == Q.OFFQ_ERR_INVALID_ARG
+    assert pw(A16, Q.OFFQ_F32, 8, 1024, 256, 1, A16, A16, None, None) == Q.OFFQ_ERR_INVALID_ARG
+    assert pw(A8, Q.OFFQ_F32, 8, 1024, 256, 1, A16, A16, A16, None) == Q.OFFQ_ERR_MISALIGNED

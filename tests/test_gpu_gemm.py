@@ -1,0 +1,167 @@
+"""GPU parity of the W4A4 GEMM (offq_w4a4_linear) against the oracle.
+
+Integer accumulators must match bit for bit given identical codes; outputs
+must lie within the fp32 epilogue bound (plus half an ulp of bf16/fp16) of the
+oracle's float64 dequantized result from the same codes, scales and offsets."""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import workloads as W
+from paper_2606_07116_gb300 import build as B
+from paper_2606_07116_gb300 import offq as Q
+from parity import check_outputs, epilogue_terms, max_rel_err_floored
+
+pytestmark = pytest.mark.gpu
+
+OUT_DT = {"f32": torch.float32, "bf16": torch.bfloat16, "f16": torch.float16}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    B.build()
+    Q.load_library()
+
+
+def _run_gemm(a_codes, a_scale, a_off, w_codes, w_scale, rowsum, g, out_dt, ldo=None, T=None, N=None):
+    T = a_codes.shape[0] if T is None else T
+    N = w_codes.shape[0] if N is None else N
+    ldo = N if ldo is None else ldo
+    out = torch.full((T, ldo), float("nan"), dtype=OUT_DT[out_dt], device="cuda")
+    acc = torch.zeros((T, N), dtype=torch.int32, device="cuda")
+    K = a_codes.shape[1] * 2
+    Q.offq_w4a4_linear(a_codes, a_scale, a_off, T, N, K, g, w_codes, w_scale, rowsum, out, ldo, acc)
+    torch.cuda.synchronize()
+    assert Q.offq_get_device_status() == Q.OFFQ_OK
+    return out[:, :N].float().cpu().numpy().astype(np.float64), acc.cpu().numpy()
+
+
+def _check_layer(T, K, N, g, out_dt, rotate=True, seed=0, ldo=None, rows=None, n_out=2, mult=50.0,
+                 dist="normal"):
+    x = W.activations(T, K, seed=seed, dist=dist, n_out=n_out, mult=mult)
+    w = W.weights(N, K, seed=seed + 1)
+    xh = torch.from_numpy(x).to(torch.bfloat16)
+    a_codes, a_scale, a_off = Q.quantize_act(xh.cuda(), g, rotate=rotate, offset=True)
+    w_codes, w_scale, rowsum = Q.prepare_weight(torch.from_numpy(w).cuda(), g, rotate=rotate)
+    y, acc = _run_gemm(a_codes, a_scale, a_off, w_codes, w_scale, rowsum, g, out_dt, ldo=ldo)
+    sel = np.arange(T) if rows is None else rows
+    qa = O.unpack_act_codes(a_codes.cpu().numpy()[sel])
+    qw = O.unpack_weight_codes(w_codes.cpu().numpy())
+    sa = a_scale.cpu().numpy().astype(np.float64)[sel]
+    oa = a_off.cpu().numpy().astype(np.float64)[sel]
+    sw = w_scale.cpu().numpy().astype(np.float64)
+    R = rowsum.cpu().numpy().astype(np.float64)
+    # The accumulator the tensor cores hold: sum_k (q_a + 8) q_w, exact.
+    acc_ref = O.int_gemm(qa + 8, qw)
+    np.testing.assert_array_equal(acc[sel], acc_ref)
+    y_ref = O.epilogue(O.int_gemm(qa, qw), sa, oa, sw, R)
+    terms = epilogue_terms(acc_ref, sa, oa, sw, R)
+    check_outputs(y[sel], y_ref, terms, K // g, out_dt)
+    return y[sel], y_ref, x[sel], w
+
+
+@pytest.mark.parametrize("out_dt", ["f32", "bf16", "f16"])
+def test_toy_layer(out_dt):
+    wl = W.WORKLOADS["toy"]
+    T, K = wl.T, 512
+    x = W.layer_inputs(wl, wl.layers[0])
+    w = W.weights(512, K)
+    a_codes, a_scale, a_off = Q.quantize_act(torch.from_numpy(x).cuda(), 512)
+    w_codes, w_scale, rowsum = Q.prepare_weight(torch.from_numpy(w).cuda(), 512)
+    y, acc = _run_gemm(a_codes, a_scale, a_off, w_codes, w_scale, rowsum, 512, out_dt)
+    qa = O.unpack_act_codes(a_codes.cpu().numpy())
+    qw = O.unpack_weight_codes(w_codes.cpu().numpy())
+    np.testing.assert_array_equal(acc, O.int_gemm(qa + 8, qw))
+    sa, oa = a_scale.cpu().numpy().astype(np.float64), a_off.cpu().numpy().astype(np.float64)
+    sw, R = w_scale.cpu().numpy().astype(np.float64), rowsum.cpu().numpy().astype(np.float64)
+    y_ref = O.epilogue(O.int_gemm(qa, qw), sa, oa, sw, R)
+    check_outputs(y, y_ref, epilogue_terms(O.int_gemm(qa + 8, qw), sa, oa, sw, R), 1, out_dt)
+    if out_dt == "f16":
+        assert max_rel_err_floored(y, y_ref) <= 2e-3
+    # Quality sanity against the unquantized layer (not parity).
+    ref = O.linear_reference(x, w)
+    assert np.linalg.norm(y - ref) < 0.25 * np.linalg.norm(ref)
+
+
+def test_oracle_codes_through_gemm():
+    """Codes, scales and offsets made by the oracle go through the GPU GEMM."""
+    T, K, N, g = 45, 1024, 320, 256
+    x = W.activations(T, K, seed=31, n_out=2, mult=60.0)
+    w = W.weights(N, K, seed=32)
+    xa = torch.from_numpy(x).to(torch.bfloat16).to(torch.float64).numpy()
+    a = O.quantize_act(xa, g)
+    wp = O.prepare_weight(w.astype(np.float64), g)
+    dev = lambda arr, dt: torch.from_numpy(np.ascontiguousarray(arr)).to(dt).cuda()
+    y, acc = _run_gemm(dev(a["codes"], torch.uint8), dev(a["scale"], torch.float32),
+                       dev(a["offset"], torch.float32), dev(wp["codes"], torch.uint8),
+                       dev(wp["scale"], torch.float32), dev(wp["offsum"], torch.float32), g, "f32")
+    np.testing.assert_array_equal(acc, O.int_gemm(a["q"] + 8, wp["q"]))
+    sa = a["scale"].astype(np.float32).astype(np.float64)
+    oa = a["offset"].astype(np.float32).astype(np.float64)
+    sw = wp["scale"].astype(np.float32).astype(np.float64)
+    y_ref = O.epilogue(O.int_gemm(a["q"], wp["q"]), sa, oa, sw, wp["offsum"])
+    check_outputs(y, y_ref, epilogue_terms(O.int_gemm(a["q"] + 8, wp["q"]), sa, oa, sw, wp["offsum"]), K // g, "f32")
+
+
+@pytest.mark.parametrize("T,K,N,g,out_dt,ldo", [
+    (33, 1024, 300, 256, "bf16", 304),     # ragged T and N, padded output rows
+    (130, 11008, 264, 256, "bf16", None),  # 43 offset blocks
+    (64, 14336, 512, 1024, "f16", None),   # 14 offset blocks
+    (3, 4096, 1000, 4096, "f32", 1000),
+    (1, 4096, 11008, 4096, "bf16", None),  # one decode token
+    (200, 4096, 4096, 4096, "bf16", None),
+    (129, 2048, 257, 2048, "f32", 260),
+])
+def test_layers(T, K, N, g, out_dt, ldo):
+    _check_layer(T, K, N, g, out_dt, ldo=ldo, seed=T + K)
+
+
+def test_no_rotation_site():
+    """q/k/v/gate/up sites: codes made without the online rotation."""
+    _check_layer(64, 4096, 768, 4096, "bf16", rotate=False, seed=5)
+
+
+def test_null_offset_means_zero():
+    T, K, N, g = 16, 512, 256, 512
+    x = W.activations(T, K, seed=41)
+    a_codes, a_scale, _ = Q.quantize_act(torch.from_numpy(x).cuda(), g, rotate=True, offset=False)
+    w_codes, w_scale, rowsum = Q.prepare_weight(torch.from_numpy(W.weights(N, K, seed=42)).cuda(), g)
+    y, acc = _run_gemm(a_codes, a_scale, None, w_codes, w_scale, rowsum, g, "f32")
+    qa = O.unpack_act_codes(a_codes.cpu().numpy())
+    qw = O.unpack_weight_codes(w_codes.cpu().numpy())
+    sa, sw = a_scale.cpu().numpy().astype(np.float64), w_scale.cpu().numpy().astype(np.float64)
+    R = rowsum.cpu().numpy().astype(np.float64)
+    zero = np.zeros((T, 1))
+    y_ref = O.epilogue(O.int_gemm(qa, qw), sa, zero, sw, R)
+    check_outputs(y, y_ref, epilogue_terms(acc, sa, zero, sw, R), 1, "f32")
+
+
+def test_accumulator_exact_at_largest_k():
+    """K = 28672 with every code at +-7: the extreme integer sums stay exact."""
+    T, N, K, g = 8, 256, 28672, 1024
+    qa = np.full((T, K), 7, dtype=np.int64)
+    qa[1::2] = -7
+    qw = np.full((N, K), 7, dtype=np.int64)
+    qw[::3] = -7
+    dev = lambda arr, dt: torch.from_numpy(np.ascontiguousarray(arr)).to(dt).cuda()
+    sa = np.ones(T, dtype=np.float32)
+    sw = np.ones(N, dtype=np.float32)
+    R = qw.reshape(N, K // g, g).sum(axis=2).T.astype(np.float32)
+    y, acc = _run_gemm(dev(O.pack_act_codes(qa), torch.uint8), dev(sa, torch.float32), None,
+                       dev(O.pack_weight_codes(qw), torch.uint8), dev(sw, torch.float32), dev(R, torch.float32),
+                       g, "f32")
+    np.testing.assert_array_equal(acc, O.int_gemm(qa + 8, qw))
+    np.testing.assert_array_equal(y, O.int_gemm(qa, qw).astype(np.float64))
+
+
+def test_full_llama2_7b_gate_sampled():
+    """Full 2048 x 4096 -> 11008 launch, checked on 128 sampled token rows."""
+    rows = W.unit_index_sample(2048, 128, seed=4)
+    _check_layer(2048, 4096, 11008, 4096, "bf16", rows=rows, n_out=4, mult=100.0)
+
+
+def test_full_llama2_7b_down_sampled():
+    rows = W.unit_index_sample(2048, 64, seed=5)
+    _check_layer(2048, 11008, 4096, 256, "bf16", rows=rows, n_out=4, mult=100.0)

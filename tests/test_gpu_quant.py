@@ -1,0 +1,199 @@
+"""GPU parity of the row quantizers (offq_quantize_act, offq_kv4_quantize,
+offq_prepare_weight) against the float64 oracle, on seeded synthetic inputs."""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import workloads as W
+from paper_2606_07116_gb300 import build as B
+from paper_2606_07116_gb300 import offq as Q
+from parity import check_codes, check_offsets, check_scales
+
+pytestmark = pytest.mark.gpu
+
+TORCH_DT = {"bf16": torch.bfloat16, "f16": torch.float16, "f32": torch.float32}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    B.build()
+    Q.load_library()
+
+
+def _host(x32: np.ndarray, dt: str) -> torch.Tensor:
+    """The input as the kernel sees it, made on the CPU (RNE cast)."""
+    return torch.from_numpy(np.ascontiguousarray(x32)).to(TORCH_DT[dt])
+
+
+def _quant_and_check(x_host: torch.Tensor, g: int, rotate: bool, offset: bool, rows=None, ldx=None):
+    T, K = x_host.shape
+    if ldx is None:
+        xd = x_host.cuda()
+    else:
+        buf = torch.zeros((T, ldx), dtype=x_host.dtype)
+        buf[:, :K] = x_host
+        xd = buf.cuda()[:, :K]
+    codes, scale, off = Q.quantize_act(xd, g, rotate=rotate, offset=offset)
+    torch.cuda.synchronize()
+    assert Q.offq_get_device_status() == Q.OFFQ_OK
+    x64 = x_host.to(torch.float64).numpy()
+    sel = np.arange(T) if rows is None else rows
+    ref = O.quantize_act(x64[sel], g, rotate=rotate, offset=offset)
+    q_gpu = O.unpack_act_codes(codes.cpu().numpy()[sel])
+    nmis = check_codes(q_gpu, ref["q"], ref["residual"], ref["scale"])
+    check_scales(scale.cpu().numpy()[sel], ref["scale"], x64[sel], g, rotate)
+    o = off.cpu().numpy()[sel]
+    if offset:
+        check_offsets(o, ref["offset"], x64[sel], g, rotate)
+    else:
+        assert np.all(o == 0.0)
+    return nmis
+
+
+@pytest.mark.parametrize("g", [32, 64, 128, 256, 512, 1024, 2048, 4096, 8192])
+@pytest.mark.parametrize("G", [1, 3])
+def test_quantize_every_block_size(g, G):
+    T = 37
+    x = W.activations(T, g * G, seed=100 + g + G, n_out=2, mult=50.0)
+    _quant_and_check(_host(x, "bf16"), g, True, True)
+
+
+@pytest.mark.parametrize("dt", ["bf16", "f16", "f32"])
+@pytest.mark.parametrize("rotate,offset", [(True, True), (True, False), (False, True), (False, False)])
+def test_quantize_flags_and_dtypes(dt, rotate, offset):
+    x = W.activations(29, 512, seed=7, n_out=2, mult=30.0)
+    _quant_and_check(_host(x, dt), 256, rotate, offset)
+
+
+@pytest.mark.parametrize("T,K,g,dist", [
+    (16, 512, 512, "normal"),          # toy layer (fp32 in the workload; bf16 here)
+    (64, 11008, 256, "normal"),        # down-proj input, 43 blocks
+    (48, 14336, 1024, "student_t3"),   # Llama-3-8B down-proj input, 14 blocks
+    (8, 28672, 1024, "normal"),        # Llama-2-70B down-proj input, 28 blocks
+    (40, 8192, 8192, "normal"),        # Llama-2-70B hidden
+])
+def test_quantize_workload_shapes(T, K, g, dist):
+    x = W.activations(T, K, seed=11, dist=dist, n_out=4, mult=100.0)
+    _quant_and_check(_host(x, "bf16"), g, True, True)
+
+
+def test_quantize_toy_fp32():
+    w = W.WORKLOADS["toy"]
+    x = W.layer_inputs(w, w.layers[0])
+    _quant_and_check(_host(x, "f32"), 512, True, True)
+
+
+def test_quantize_full_llama2_7b_sampled():
+    """Full 2048 x 4096 bf16 launch, checked on 256 sampled rows."""
+    x = W.activations(2048, 4096, seed=0, n_out=4, mult=100.0)
+    rows = W.unit_index_sample(2048, 256, seed=3)
+    _quant_and_check(_host(x, "bf16"), 4096, True, True, rows=rows)
+
+
+def test_quantize_strided_rows():
+    x = W.activations(21, 1024, seed=12, n_out=1, mult=20.0)
+    _quant_and_check(_host(x, "bf16"), 1024, True, True, ldx=1024 + 64)
+
+
+def test_quantize_degenerate_rows():
+    g, G = 256, 2
+    x = W.activations(6, g * G, seed=13)
+    x[0] = 0.0                                   # all-zero row: scale 0, codes 0
+    x[1] = 0.0
+    x[1, 0], x[1, g] = 123.0, -7.5               # only the block-leading channels: zero residual
+    x[2, :] = 0.0
+    x[2, 5] = 1.0                                # one unit channel
+    xh = _host(x, "f32")
+    codes, scale, off = Q.quantize_act(xh.cuda(), g)
+    torch.cuda.synchronize()
+    q = O.unpack_act_codes(codes.cpu().numpy())
+    assert np.all(q[0] == 0) and scale[0].item() == 0.0 and np.all(off[0].cpu().numpy() == 0.0)
+    assert np.all(q[1] == 0) and scale[1].item() == 0.0
+    np.testing.assert_allclose(off[1].cpu().numpy(), [123.0 / math.sqrt(g), -7.5 / math.sqrt(g)], rtol=3e-7)
+    H = O.sylvester_hadamard(g)
+    np.testing.assert_array_equal(q[2, :g], 7 * H[5])   # x = e_5 rotates to H[5] / sqrt(g)
+    np.testing.assert_array_equal(q[2, g:], 0)
+    _quant_and_check(xh, g, True, True)
+
+
+def test_quantize_exact_ties_round_half_even():
+    """Without rotation and offset, scale 1 and half-integer inputs: ties resolve to even, bit-exact."""
+    row = np.array([7.0, -7.0, 0.5, 1.5, 2.5, 3.5, -0.5, -1.5, -2.5, -3.5, 4.5, -4.5, 5.5, 6.5, -5.5, -6.5]
+                   * 2, dtype=np.float32)
+    x = np.tile(row, (5, 2))
+    codes, scale, _ = Q.quantize_act(torch.from_numpy(x).cuda(), 32, rotate=False, offset=False)
+    torch.cuda.synchronize()
+    q = O.unpack_act_codes(codes.cpu().numpy())
+    ref = O.quantize_act(x.astype(np.float64), 32, rotate=False, offset=False)
+    np.testing.assert_array_equal(q, ref["q"])
+    np.testing.assert_array_equal(scale.cpu().numpy(), 1.0)
+    assert list(q[0, :16]) == [7, -7, 0, 2, 2, 4, 0, -2, -2, -4, 4, -4, 6, 6, -6, -6]
+
+
+def test_quantize_single_token():
+    x = W.activations(1, 4096, seed=14, n_out=4, mult=100.0)
+    _quant_and_check(_host(x, "bf16"), 4096, True, True)
+
+
+# --------------------------------------------------------------------------
+# KV4
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("T,H", [(1, 32), (5, 32), (64, 32), (33, 8)])
+@pytest.mark.parametrize("flags", [3, 2])
+def test_kv4_against_oracle(T, H, flags):
+    hd = 128
+    kv = W.kv_heads(T, H, hd, seed=2 + T)
+    kvh = _host(kv.reshape(T, H * hd), "bf16").reshape(T, H, hd)
+    rotate = bool(flags & 1)
+    codes, scale, off = Q.kv4_quantize(kvh.cuda(), rotate=rotate, offset=True)
+    torch.cuda.synchronize()
+    ref = O.kv4_quantize(kvh.to(torch.float64).numpy(), rotate=rotate, offset=True)
+    q = O.unpack_act_codes(codes.cpu().numpy())
+    check_codes(q.reshape(T * H, hd), ref["q"].reshape(T * H, hd), ref["residual"].reshape(T * H, hd),
+                ref["scale"].reshape(T * H))
+    x64 = kvh.to(torch.float64).numpy().reshape(T * H, hd)
+    check_scales(scale.cpu().numpy().reshape(-1), ref["scale"].reshape(-1), x64, hd, rotate)
+    check_offsets(off.cpu().numpy().reshape(-1, 1), ref["offset"].reshape(-1, 1), x64, hd, rotate)
+
+
+def test_kv4_padded_token_stride():
+    T, H, hd = 7, 8, 128
+    kv = W.kv_heads(T, H, hd, seed=9)
+    host = _host(kv.reshape(T, H * hd), "bf16")
+    buf = torch.zeros((T, H * hd + 256), dtype=torch.bfloat16)
+    buf[:, :H * hd] = host
+    dev = buf.cuda()
+    codes = torch.empty((T, H, hd // 2), dtype=torch.uint8, device="cuda")
+    scale = torch.empty((T, H), dtype=torch.float32, device="cuda")
+    off = torch.empty((T, H), dtype=torch.float32, device="cuda")
+    Q.offq_kv4_quantize(dev, T, H, hd, H * hd + 256, Q.OFFQ_ROTATE | Q.OFFQ_OFFSET, codes, scale, off)
+    torch.cuda.synchronize()
+    ref = O.kv4_quantize(host.to(torch.float64).numpy().reshape(T, H, hd))
+    q = O.unpack_act_codes(codes.cpu().numpy()).reshape(T * H, hd)
+    check_codes(q, ref["q"].reshape(T * H, hd), ref["residual"].reshape(T * H, hd), ref["scale"].reshape(-1))
+
+
+# --------------------------------------------------------------------------
+# Weight preparation (offline)
+# --------------------------------------------------------------------------
+
+@pytest.mark.parametrize("N,K,g,rotate", [(300, 1024, 256, True), (64, 512, 512, False), (40, 11008, 256, True),
+                                          (24, 14336, 1024, True)])
+def test_prepare_weight(N, K, g, rotate):
+    w = W.weights(N, K, seed=21)
+    wh = torch.from_numpy(w)
+    codes, scale, rowsum = Q.prepare_weight(wh.cuda(), g, rotate=rotate)
+    torch.cuda.synchronize()
+    ref = O.prepare_weight(w.astype(np.float64), g, rotate=rotate)
+    qg = O.unpack_weight_codes(codes.cpu().numpy())
+    # Reuse the activation-path checks: weights are rows quantized without offset.
+    ra = O.quantize_act(w.astype(np.float64), g, rotate=rotate, offset=False)
+    check_codes(qg, ref["q"], ra["residual"], ra["scale"], what="weight codes")
+    check_scales(scale.cpu().numpy(), ref["scale"], w.astype(np.float64), g, rotate, what="weight scale")
+    # Row sums are exact integers of the GPU's own codes.
+    np.testing.assert_array_equal(rowsum.cpu().numpy(), qg.reshape(N, K // g, g).sum(axis=2).T)
