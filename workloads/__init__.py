@@ -153,13 +153,14 @@ class Workload:
 
 def _llama_layers(hidden: int, inter: int, kv_dim: int) -> Tuple[Linear, ...]:
     # q/k/v/gate/up inputs arrive already in the offset basis (their rotation
-    # is fused into the weights offline); o-proj and down-proj inputs take the
-    # online Hadamard.
+    # is fused into the weights offline), as does the o-proj input (per-head
+    # rotation fused into W_V / W_O); the down-proj input takes the online
+    # group-wise Hadamard H4.
     return (
         Linear("q", hidden, hidden, False),
         Linear("k", hidden, kv_dim, False),
         Linear("v", hidden, kv_dim, False),
-        Linear("o", hidden, hidden, True),
+        Linear("o", hidden, hidden, False),
         Linear("gate", hidden, inter, False),
         Linear("up", hidden, inter, False),
         Linear("down", inter, hidden, True),
