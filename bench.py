@@ -1,0 +1,532 @@
+#!/usr/bin/env python3
+"""Benchmark of the OffQ W4A4 linear path on GB300.
+
+One step = one pass of the whole hot path over one batch of synthetic input of
+the workload: the activation quantizer (online block Hadamard where the site
+has one, offsets, 4-bit codes) on every layer input, the seven W4A4 GEMMs with
+the fused dequant + offset epilogue (q, k, v, o, gate, up, down), and the KV4
+quantizer on the K and V projections. Weights are prepared once, offline.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl reference]
+
+Prints one JSON line (rank 0). ``value`` is the whole-job W4A4 linear
+throughput in TOPS (2*T*N*K integer multiply-adds per layer) with inputs
+resident in HBM; ``e2e`` is the same metric through the public API with the
+inputs copied from pinned host memory and the final output read back inside
+the timed region. ``--impl reference`` times the CPU oracle instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import platform
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import workloads as W  # noqa: E402
+
+METRIC = "W4A4 OffQ linear TOPS (% dense INT8 peak); act-quant GB/s (% of HBM BW)"
+UNIT = "TOPS"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+FP8_PER_BF16 = 2.0   # nominal dense fp8 / bf16 tensor ratio (4.5 / 2.25 PFLOP/s)
+L2_FLUSH_BYTES = 512 << 20
+
+
+def _env_int(name, default):
+    try:
+        return int(os.environ.get(name, default))
+    except ValueError:
+        return default
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return {"hbm_gbs": float(d["hbm_gbs"]), "bf16_tflops": float(d["bf16_tflops"]),
+                "bf16_tflops_sustained": float(d.get("bf16_tflops_sustained", d["bf16_tflops"])),
+                "source": "measured"}
+    except (OSError, KeyError, ValueError):
+        return dict(FALLBACK_PEAKS, source="fallback")
+
+
+def workload_by_name(name: str) -> W.Workload:
+    if name in W.WORKLOADS:
+        return W.WORKLOADS[name]
+    if name.startswith("decode_t"):
+        return W.decode_workload(int(name[len("decode_t"):]))
+    raise SystemExit(f"unknown workload {name}")
+
+
+def gemm_ops(w: W.Workload, T: int) -> float:
+    return float(sum(2.0 * T * l.N * l.K for l in w.layers))
+
+
+def sites(w: W.Workload):
+    """Distinct layer inputs: (site name, K, rotate, [layers fed])."""
+    out = []
+    seen = {}
+    for l in w.layers:
+        key = {"q": "attn_in", "k": "attn_in", "v": "attn_in", "o": "attn_out", "gate": "mlp_in",
+               "up": "mlp_in", "down": "down_in"}.get(l.name, l.name)
+        if key not in seen:
+            seen[key] = len(out)
+            out.append([key, l.K, l.rotate, []])
+        out[seen[key]][3].append(l)
+    return out
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.dev = device_index
+        self.proc = None
+        self.lines = []
+        self.error = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "50",
+                 "-i", str(self.dev)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.first = threading.Event()
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+            # nvidia-smi needs a moment to start; its first sample predates the timed region.
+            self.first.wait(timeout=5.0)
+            self.lines = []
+        except OSError as e:
+            self.error = str(e)
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+            self.first.set()
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.thread.join(timeout=5)
+
+    def summary(self):
+        if self.error or not self.lines:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0,
+                    "note": self.error or "no nvidia-smi samples"}
+        sm, smax, power, reasons = [], [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+                power.append(float(parts[3]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm), "power_w_max": max(power)}
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+
+class GpuStep:
+    """Device buffers of one layer step and the library calls that make the step."""
+
+    def __init__(self, w: W.Workload, T: int, device, seed_base: int = 0):
+        import torch
+        from paper_2606_07116_gb300 import offq as Q
+        self.torch, self.Q, self.w, self.T, self.device = torch, Q, w, T, device
+        dt = torch.bfloat16 if w.x_dtype == "bf16" else torch.float32
+        self.sites = []
+        for i, (name, K, rotate, layers) in enumerate(sites(w)):
+            x = W.activations(T, K, seed=seed_base + 10 + i, dist=w.dist, n_out=w.n_out, mult=w.mult)
+            host = torch.from_numpy(x).to(dt).pin_memory()
+            dev = host.to(device)
+            g = W.block_for(K)
+            codes = torch.empty((T, K // 2), dtype=torch.uint8, device=device)
+            scale = torch.empty((T,), dtype=torch.float32, device=device)
+            off = torch.empty((T, K // g), dtype=torch.float32, device=device)
+            flags = (Q.OFFQ_ROTATE if rotate else 0) | Q.OFFQ_OFFSET
+            gemms = []
+            for l in layers:
+                wt = torch.from_numpy(W.weights(l.N, l.K, seed=seed_base + 100 + len(self.sites) * 10 + len(gemms)))
+                wc, ws, wr = Q.prepare_weight(wt.to(device), g, rotate=l.rotate)
+                out = torch.empty((T, l.N), dtype=torch.bfloat16, device=device)
+                gemms.append({"layer": l, "codes": wc, "scale": ws, "rowsum": wr, "out": out})
+            self.sites.append({"name": name, "K": K, "g": g, "flags": flags, "host": host, "dev": dev,
+                               "codes": codes, "scale": scale, "off": off, "gemms": gemms,
+                               "in_bytes": dev.element_size()})
+        self.kv = []
+        if w.kv_heads:
+            H, hd = w.kv_heads, w.head_dim
+            for site in self.sites:
+                for gm in site["gemms"]:
+                    if gm["layer"].name in ("k", "v"):
+                        rot = gm["layer"].name == "k"    # K takes the per-head online Hadamard H3
+                        flags = (Q.OFFQ_ROTATE if rot else 0) | Q.OFFQ_OFFSET
+                        self.kv.append({"src": gm["out"], "H": H, "hd": hd, "flags": flags,
+                                        "codes": torch.empty((T, H, hd // 2), dtype=torch.uint8, device=device),
+                                        "scale": torch.empty((T, H), dtype=torch.float32, device=device),
+                                        "off": torch.empty((T, H), dtype=torch.float32, device=device)})
+        last = self.sites[-1]["gemms"][-1]["out"]
+        self.result = last
+        self.result_host = torch.empty(last.shape, dtype=last.dtype).pin_memory()
+        torch.cuda.synchronize(device)
+
+    def launches_per_step(self):
+        return len(self.sites) + sum(len(s["gemms"]) for s in self.sites) + len(self.kv)
+
+    def quant_bytes(self):
+        T = self.T
+        return sum(T * s["K"] * s["in_bytes"] + T * s["K"] // 2 + 4 * T + 4 * T * (s["K"] // s["g"])
+                   for s in self.sites)
+
+    def kv_bytes(self):
+        T = self.T
+        return sum(T * k["H"] * k["hd"] * 2 + T * k["H"] * (k["hd"] // 2) + 8 * T * k["H"] for k in self.kv)
+
+    def run(self, stream, timers=None, h2d=False, d2h=False):
+        Q, torch = self.Q, self.torch
+        T = self.T
+
+        def rec(kind):
+            if timers is None:
+                return None
+            e = torch.cuda.Event(enable_timing=True)
+            e.record(stream)
+            timers.setdefault(kind, []).append(e)
+            return e
+
+        kv_done = False
+        for s in self.sites:
+            if h2d:
+                s["dev"].copy_(s["host"], non_blocking=True)
+            rec("quant")
+            Q.offq_quantize_act(s["dev"], T, s["K"], s["dev"].stride(0), s["g"], s["flags"], s["codes"],
+                                s["scale"], s["off"], stream)
+            rec("quant")
+            for gm in s["gemms"]:
+                l = gm["layer"]
+                rec("gemm")
+                Q.offq_w4a4_linear(s["codes"], s["scale"], s["off"], T, l.N, l.K, s["g"], gm["codes"],
+                                   gm["scale"], gm["rowsum"], gm["out"], gm["out"].stride(0), None, stream)
+                rec("gemm")
+            if not kv_done and any(g["layer"].name == "v" for g in s["gemms"]):
+                for k in self.kv:
+                    rec("kv4")
+                    Q.offq_kv4_quantize(k["src"], T, k["H"], k["hd"], k["src"].stride(0), k["flags"], k["codes"],
+                                        k["scale"], k["off"], stream)
+                    rec("kv4")
+                kv_done = True
+        if d2h:
+            self.result_host.copy_(self.result, non_blocking=True)
+
+
+def _pair_times(events):
+    return [events[i].elapsed_time(events[i + 1]) for i in range(0, len(events), 2)]
+
+
+def load_traffic_record():
+    path = os.path.join(ROOT, "profiles", "gemm_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    src = os.path.join(ROOT, "paper_2606_07116_gb300", "csrc", "gemm.cu")
+    with open(src, "rb") as f:
+        digest = hashlib.sha256(f.read()).hexdigest()
+    if rec.get("gemm_cu_sha256") != digest:
+        return None
+    return rec
+
+
+def run_gpu(args, rank, world, local_rank):
+    import torch
+    import __graft_entry__ as G
+    G.build()
+    from paper_2606_07116_gb300 import offq as Q
+
+    device = torch.device("cuda", local_rank)
+    torch.cuda.set_device(device)
+    w = workload_by_name(args.workload)
+    T = w.T
+    step = GpuStep(w, T, device, seed_base=rank * 1000)
+    stream = torch.cuda.current_stream(device)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
+
+    dist = None
+    if world > 1:
+        import torch.distributed as dist_mod
+        dist = dist_mod
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        step.run(stream)
+    torch.cuda.synchronize(device)
+    st = Q.offq_get_device_status(stream)
+    if st != Q.OFFQ_OK:
+        raise RuntimeError(f"device status after warm-up: {Q.status_string(st)}")
+
+    # ---- timed region: K steps, inputs resident, L2 flushed between steps ----
+    timers = {}
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    barrier()
+    torch.cuda.synchronize(device)
+    with ClockSampler(device.index if device.index is not None else 0) as clk:
+        wall0 = time.perf_counter()
+        for i in range(args.steps):
+            flush.zero_()
+            starts[i].record(stream)
+            step.run(stream, timers=timers)
+            ends[i].record(stream)
+        torch.cuda.synchronize(device)
+        wall1 = time.perf_counter()
+    barrier()
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    dev_ms = sum(step_ms)
+    gemm_ms = sum(_pair_times(timers["gemm"]))
+    quant_ms = sum(_pair_times(timers["quant"]))
+    kv_ms = sum(_pair_times(timers.get("kv4", []))) if timers.get("kv4") else 0.0
+    n_gemm = len(timers["gemm"]) // 2
+    st = Q.offq_get_device_status(stream)
+    if st != Q.OFFQ_OK:
+        raise RuntimeError(f"device status after the timed region: {Q.status_string(st)}")
+
+    # ---- end to end through the public API: pinned H2D inputs, D2H result ----
+    e2e_steps = max(1, args.steps)
+    barrier()
+    torch.cuda.synchronize(device)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        step.run(stream, h2d=True, d2h=True)
+    e1.record(stream)
+    torch.cuda.synchronize(device)
+    barrier()
+    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+
+    ms_per_step = dev_ms / args.steps
+    if dist is not None:
+        t = torch.tensor([ms_per_step, e2e_ms], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_per_step, e2e_ms = float(t[0]), float(t[1])
+    ops = gemm_ops(w, T)
+    value = ops * world / (ms_per_step * 1e-3) / 1e12
+    e2e_value = ops * world / (e2e_ms * 1e-3) / 1e12
+
+    peaks = load_peaks()
+    fp8_peak = peaks["bf16_tflops_sustained"] * FP8_PER_BF16
+    gemm_tflops = ops * args.steps / (gemm_ms * 1e-3) / 1e12
+    quant_gbs = step.quant_bytes() * args.steps / (quant_ms * 1e-3) / 1e9
+    kv_gbs = step.kv_bytes() * args.steps / (kv_ms * 1e-3) / 1e9 if kv_ms > 0 else None
+    traffic = load_traffic_record()
+    if rank != 0:
+        return None
+    line = {
+        "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int4",
+        "data": "synthetic (seeded Llama-shaped activations with outlier channels, N(0,0.02) weights)",
+        "config": {"workload": w.name, "description": w.description, "tokens": T,
+                   "layers": [f"{l.name}:{l.K}->{l.N}" for l in w.layers],
+                   "kv4_heads": w.kv_heads, "block_sizes": {str(s['K']): s['g'] for s in step.sites},
+                   "out_dtype": "bf16", "l2": "flushed (512 MiB write) between timed steps",
+                   "parallelism": f"dp{world} (token batches, no collective in the data path)"},
+        "roofline": {"bound": "tensor", "kernel": "w4a4_gemm_kernel (tcgen05.mma kind::f8f6f4)",
+                     "achieved": round(gemm_tflops, 2), "peak": round(fp8_peak, 1), "unit": "TFLOP/s",
+                     "frac": round(gemm_tflops / fp8_peak, 4),
+                     "peak_source": f"{peaks['source']}: bf16 sustained {peaks['bf16_tflops_sustained']} "
+                                    f"x nominal fp8/bf16 ratio {FP8_PER_BF16}",
+                     "traffic": traffic["bytes_per_launch"] if traffic else None,
+                     "traffic_note": traffic.get("note") if traffic else "no ncu record for this gemm.cu",
+                     "gemm_ms_per_step": round(gemm_ms / args.steps, 4)},
+        "act_quant": {"value": round(quant_gbs, 1), "unit": "GB/s", "peak": peaks["hbm_gbs"],
+                      "frac": round(quant_gbs / peaks["hbm_gbs"], 4),
+                      "ms_per_step": round(quant_ms / args.steps, 4), "bytes_per_step": step.quant_bytes()},
+        "kv4": {"value": round(kv_gbs, 1) if kv_gbs else None, "unit": "GB/s",
+                "ms_per_step": round(kv_ms / args.steps, 4), "bytes_per_step": step.kv_bytes()},
+        "e2e": {"value": round(e2e_value, 3), "unit": UNIT,
+                "h2d_bytes_per_step": int(sum(s["host"].numel() * s["host"].element_size() for s in step.sites)),
+                "d2h_bytes_per_step": int(step.result.numel() * step.result.element_size()),
+                "ms_per_step": round(e2e_ms, 4)},
+        "gpu_launches": step.launches_per_step() * args.steps,
+        "gemm_launches": n_gemm,
+        "wall_s_timed_region": round(wall1 - wall0, 4),
+        "clocks": clk.summary(),
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
+    return line
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle (baseline leg and the reference arm)
+# ---------------------------------------------------------------------------
+
+class OracleStep:
+    """The same step computed by the float64 oracle on a sample of tokens."""
+
+    def __init__(self, w: W.Workload, T_full: int):
+        import oracle as O
+        self.O, self.w = O, w
+        dt = w.x_dtype
+        self.inputs = []
+        self.weights = []
+        for i, (name, K, rotate, layers) in enumerate(sites(w)):
+            x = W.activations(T_full, K, seed=10 + i, dist=w.dist, n_out=w.n_out, mult=w.mult)
+            if dt == "bf16":
+                x = W.bf16_to_f64(W.to_bf16(x))
+            g = W.block_for(K)
+            wl = []
+            for j, l in enumerate(layers):
+                wp = O.prepare_weight(W.weights(l.N, l.K, seed=100 + i * 10 + j).astype(np.float64), g,
+                                      rotate=l.rotate)
+                wl.append((l, wp))
+            self.inputs.append((name, K, g, rotate, x.astype(np.float64)))
+            self.weights.append(wl)
+
+    def run(self, rows: np.ndarray):
+        O = self.O
+        outs = {}
+        for (name, K, g, rotate, x), wl in zip(self.inputs, self.weights):
+            a = O.quantize_act(x[rows], g, rotate=rotate, offset=True)
+            for l, wp in wl:
+                y = O.w4a4_linear(a["q"], a["scale"], a["offset"], wp["q"], wp["scale"], wp["offsum"])["y"]
+                outs[l.name] = y
+        if self.w.kv_heads:
+            H, hd = self.w.kv_heads, self.w.head_dim
+            for nm, rot in (("k", True), ("v", False)):
+                if nm in outs:
+                    O.kv4_quantize(outs[nm].reshape(len(rows), H, hd), rotate=rot, offset=True)
+        return outs
+
+
+def _cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(w: W.Workload, budget_s: float = 15.0):
+    ostep = OracleStep(w, w.T)
+    rows = W.unit_index_sample(w.T, 8, seed=1)
+    t0 = time.perf_counter()
+    ostep.run(rows)
+    per_tok = (time.perf_counter() - t0) / len(rows)
+    n = int(max(8, min(w.T, budget_s / max(per_tok, 1e-9))))
+    rows = W.unit_index_sample(w.T, n, seed=2)
+    t0 = time.perf_counter()
+    ostep.run(rows)
+    dt = time.perf_counter() - t0
+    value = gemm_ops(w, len(rows)) / dt / 1e12
+    return {"value": value, "unit": UNIT, "cores": _cores(), "kind": "oracle",
+            "sample": f"{len(rows)} of {w.T} tokens through every layer (float64 oracle: explicit Hadamard, "
+                      f"exact integer GEMM via float64 BLAS, float64 epilogue, KV4), {dt:.1f} s",
+            "cpu": platform.processor() or platform.machine()}
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return None
+    w = workload_by_name(args.workload)
+    ostep = OracleStep(w, w.T)
+    probe = W.unit_index_sample(w.T, 4, seed=1)
+    t0 = time.perf_counter()
+    ostep.run(probe)
+    per_tok = (time.perf_counter() - t0) / len(probe)
+    per_step_budget = max(1.0, args.ref_budget / max(1, args.steps + args.warmup))
+    n = int(max(4, min(w.T, per_step_budget / max(per_tok, 1e-9))))
+    rows = W.unit_index_sample(w.T, n, seed=2)
+    for _ in range(args.warmup):
+        ostep.run(rows)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        ostep.run(rows)
+    dt = (time.perf_counter() - t0) / args.steps
+    value = gemm_ops(w, n) / dt / 1e12
+    sample = f"{n} of {w.T} tokens per step through every layer and KV4 (float64 oracle)"
+    return {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "description": w.description, "tokens_per_step": n},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": _cores(), "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--workload", default="llama2_7b")
+    ap.add_argument("--impl", default="offq", choices=["offq", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
+    ap.add_argument("--ref-budget", type=float, default=120.0, help="seconds of oracle work for --impl reference")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        raise SystemExit("--warmup must be at least 3")
+
+    world = _env_int("WORLD_SIZE", 1)
+    rank = _env_int("RANK", 0)
+    local_rank = _env_int("LOCAL_RANK", 0)
+    if args.impl == "reference":
+        line = run_reference(args, rank, world)
+    else:
+        if world > 1:
+            import torch
+            import torch.distributed as dist
+            torch.cuda.set_device(local_rank)
+            dist.init_process_group("nccl")
+        line = run_gpu(args, rank, world, local_rank)
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+    if line is not None and rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()
