@@ -13,12 +13,15 @@
 // "+8" is removed in the epilogue with the weight block row sums R, together
 // with the offsets: sum_b 8 s_a R[b][n] = 8 s_a sum_k q_w[n][k].
 //
-// CTA tile 128 (tokens) x 256 (channels), k-tile 128 codes. Warp roles:
-//   warp 0     TMA producer: packed int4 tiles of A and B into a 4-stage ring
-//   warp 1     TMEM allocation and the single-thread MMA issuer
-//   warps 2-5  widen packed codes to E4M3 tiles in the 128-byte-swizzled
-//              K-major layout of the MMA (2-stage ring), then run the epilogue
-//              from TMEM (each warp owns one 32-lane quarter of the accumulator)
+// Persistent CTAs (one per SM), tile 128 (tokens) x 256 (channels), k-tile 128
+// codes. Warp roles:
+//   warp 0       TMA producer: packed int4 tiles of A and B into a 4-stage ring
+//   warp 1       TMEM allocation and the single-thread MMA issuer
+//   warps 2-9    widen packed codes to E4M3 tiles in the 128-byte-swizzled
+//                K-major layout of the MMA (2-stage ring)
+//   warps 10-13  epilogue from TMEM (each warp owns one 32-lane quarter of the
+//                accumulator); two accumulator buffers (2 x 256 columns) let the
+//                epilogue of a tile overlap the main loop of the next
 // Every wait is bounded; a wait that runs out aborts the CTA and records
 // OFFQ_ERR_TIMEOUT in the device status word.
 #include <cuda.h>
@@ -40,9 +43,16 @@ constexpr int BN = 256;
 constexpr int BK = 128;  // codes per k-tile (128 fp8 bytes = one swizzle row)
 constexpr int kPackStages = 4;
 constexpr int kF8Stages = 2;
-constexpr int kThreads = 192;
-constexpr int kConvThreads = 128;
-constexpr int kMaxEpilogueG = 96;
+constexpr int kConvWarps = 8;
+constexpr int kEpiWarps = 4;
+constexpr int kConvThreads = kConvWarps * 32;
+constexpr int kEpiThreads = kEpiWarps * 32;
+constexpr int kFirstConvWarp = 2;
+constexpr int kFirstEpiWarp = kFirstConvWarp + kConvWarps;
+constexpr int kThreads = (kFirstEpiWarp + kEpiWarps) * 32;
+constexpr int kAccCols = BN;          // fp32 accumulator columns per buffer
+constexpr int kTmemCols = 2 * kAccCols;  // double-buffered accumulator
+constexpr int kMaxEpilogueG = 2048;
 
 constexpr int kAPack = BM * BK / 2;  // 8 KB
 constexpr int kBPack = BN * BK / 2;  // 16 KB
@@ -54,13 +64,13 @@ constexpr int kOffF8B = kOffF8A + kF8Stages * kAF8;
 constexpr int kOffPackA = kOffF8B + kF8Stages * kBF8;
 constexpr int kOffPackB = kOffPackA + kPackStages * kAPack;
 constexpr int kOffBars = kOffPackB + kPackStages * kBPack;
-constexpr int kNumBars = 2 * kPackStages + 2 * kF8Stages + 1;
+constexpr int kNumBars = 2 * kPackStages + 2 * kF8Stages + 4;
 constexpr int kOffMisc = kOffBars + kNumBars * 8;
 constexpr int kSmemBytes = kOffMisc + 64 + 1024;  // + alignment slack for the 1024-byte base
 
 static_assert(kOffPackA % 1024 == 0 && kOffF8B % 1024 == 0, "MMA tiles need 1024-byte alignment");
-static_assert(kMaxEpilogueG * BN * 4 <= kF8Stages * (kAF8 + kBF8), "R tile must fit the fp8 region");
-static_assert(BM * (kMaxEpilogueG + 1) * 4 + BN * 4 <= kPackStages * (kAPack + kBPack), "O tile must fit");
+static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+static_assert(BM * 4 % kConvThreads == 0 && BN * 4 % kConvThreads == 0, "even converter split");
 
 constexpr uint32_t kIdesc = idesc_e4m3_f32(BM, BN);
 
@@ -74,6 +84,7 @@ struct GemmParams {
   int32_t* acc_debug;
   int* status;
   int T, N, K, G, out_dtype;
+  int m_tiles, n_tiles;
 };
 
 __device__ __forceinline__ bool mbar_wait_teardown(uint32_t bar, uint32_t parity) {
@@ -110,25 +121,23 @@ __device__ __forceinline__ uint4 lds128(uint32_t addr) {
   return r;
 }
 
-__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
-
-template <int OUT>
+template <int OUT, int CW>
 __device__ __forceinline__ void store_out(void* out, int64_t off, const float* y, int nvalid) {
   if (OUT == OFFQ_F32) {
     float* o = static_cast<float*>(out) + off;
-    if (nvalid == 32) {
+    if (nvalid == CW) {
 #pragma unroll
-      for (int i = 0; i < 8; ++i)
+      for (int i = 0; i < CW / 4; ++i)
         *reinterpret_cast<float4*>(o + 4 * i) = make_float4(y[4 * i], y[4 * i + 1], y[4 * i + 2], y[4 * i + 3]);
     } else {
 #pragma unroll
-      for (int i = 0; i < 32; ++i)
+      for (int i = 0; i < CW; ++i)
         if (i < nvalid) o[i] = y[i];
     }
   } else {
-    uint32_t p[16];
+    uint32_t p[CW / 2];
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
+    for (int i = 0; i < CW / 2; ++i) {
       if (OUT == OFFQ_BF16) {
         const __nv_bfloat162 h = __floats2bfloat162_rn(y[2 * i], y[2 * i + 1]);
         p[i] = *reinterpret_cast<const uint32_t*>(&h);
@@ -138,18 +147,22 @@ __device__ __forceinline__ void store_out(void* out, int64_t off, const float* y
       }
     }
     uint16_t* o = static_cast<uint16_t*>(out) + off;
-    if (nvalid == 32) {
+    if (nvalid == CW) {
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
+      for (int i = 0; i < CW / 8; ++i)
         *reinterpret_cast<uint4*>(o + 8 * i) = make_uint4(p[4 * i], p[4 * i + 1], p[4 * i + 2], p[4 * i + 3]);
     } else {
 #pragma unroll
-      for (int i = 0; i < 32; ++i)
+      for (int i = 0; i < CW; ++i)
         if (i < nvalid) o[i] = static_cast<uint16_t>(p[i >> 1] >> (16 * (i & 1)));
     }
   }
 }
 
+// Persistent kernel: CTA b processes tiles b, b + gridDim.x, ... (tile index =
+// m_tile * n_tiles + n_tile). The k-tile pipeline counters run across tiles, and
+// the accumulator alternates between two TMEM buffers so the epilogue of one tile
+// overlaps the main loop of the next.
 template <int OUT>
 __global__ void __launch_bounds__(kThreads, 1)
     w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
@@ -161,16 +174,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int n0 = blockIdx.x * BN;
-  const int m0 = blockIdx.y * BM;
   const int nk = (p.K + BK - 1) / BK;
+  const int num_tiles = p.m_tiles * p.n_tiles;
 
   const uint32_t bar0 = base + kOffBars;
   auto full_pack = [&](int s) { return bar0 + 8u * s; };
   auto empty_pack = [&](int s) { return bar0 + 8u * (kPackStages + s); };
   auto full_f8 = [&](int s) { return bar0 + 8u * (2 * kPackStages + s); };
   auto empty_f8 = [&](int s) { return bar0 + 8u * (2 * kPackStages + kF8Stages + s); };
-  const uint32_t accum_full = bar0 + 8u * (2 * kPackStages + 2 * kF8Stages);
+  auto acc_full = [&](int b) { return bar0 + 8u * (2 * kPackStages + 2 * kF8Stages + b); };
+  auto acc_empty = [&](int b) { return bar0 + 8u * (2 * kPackStages + 2 * kF8Stages + 2 + b); };
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffMisc);
   volatile int* abort = reinterpret_cast<volatile int*>(smem + kOffMisc + 16);
 
@@ -183,14 +196,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(full_f8(s), kConvThreads);
       mbar_init(empty_f8(s), 1);
     }
-    mbar_init(accum_full, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(acc_full(b), 1);
+      mbar_init(acc_empty(b), kEpiThreads);
+    }
     *abort = 0;
     mbar_fence_init();
     tma_prefetch_desc(&tmap_a);
     tma_prefetch_desc(&tmap_b);
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), BN);
+    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -198,163 +214,208 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  int issued = 0;  // producer: k-tiles whose TMA loads were issued
+  int issued = 0;     // producer: k-tiles whose TMA loads were issued (global count)
+  int mma_tiles = 0;  // MMA issuer: tiles whose accumulation was committed
 
   if (warp == 0) {
+    // ---------------- TMA producer ----------------
     if (lane == 0) {
-      for (int kt = 0; kt < nk; ++kt) {
-        const int s = kt % kPackStages;
-        const uint32_t ph = (kt / kPackStages) & 1;
-        if (!mbar_wait(empty_pack(s), ph ^ 1, abort)) break;
-        mbar_arrive_expect_tx(full_pack(s), kAPack + kBPack);
-        tma_load_2d(base + kOffPackA + s * kAPack, &tmap_a, full_pack(s), kt * (BK / 2), m0);
-        tma_load_2d(base + kOffPackB + s * kBPack, &tmap_b, full_pack(s), kt * (BK / 2), n0);
-        issued = kt + 1;
+      int g = 0;
+      for (int tile = blockIdx.x; tile < num_tiles && !*abort; tile += gridDim.x) {
+        const int m0 = (tile / p.n_tiles) * BM;
+        const int n0 = (tile % p.n_tiles) * BN;
+        for (int kt = 0; kt < nk; ++kt, ++g) {
+          const int s = g % kPackStages;
+          const uint32_t ph = (g / kPackStages) & 1;
+          if (!mbar_wait(empty_pack(s), ph ^ 1, abort)) break;
+          mbar_arrive_expect_tx(full_pack(s), kAPack + kBPack);
+          tma_load_2d(base + kOffPackA + s * kAPack, &tmap_a, full_pack(s), kt * (BK / 2), m0);
+          tma_load_2d(base + kOffPackB + s * kBPack, &tmap_b, full_pack(s), kt * (BK / 2), n0);
+          issued = g + 1;
+        }
       }
     }
   } else if (warp == 1) {
+    // ---------------- MMA issuer ----------------
     if (lane == 0) {
-      for (int kt = 0; kt < nk; ++kt) {
-        const int s = kt % kF8Stages;
-        const uint32_t ph = (kt / kF8Stages) & 1;
-        if (!mbar_wait(full_f8(s), ph, abort)) break;
+      int g = 0, lt = 0;
+      for (int tile = blockIdx.x; tile < num_tiles && !*abort; tile += gridDim.x, ++lt) {
+        const int ab = lt & 1;
+        if (!mbar_wait(acc_empty(ab), ((lt >> 1) & 1) ^ 1, abort)) break;
         tc_fence_after();
-        const uint32_t a_addr = base + kOffF8A + s * kAF8;
-        const uint32_t b_addr = base + kOffF8B + s * kBF8;
+        const uint32_t acc = tmem + ab * kAccCols;
+        bool ok = true;
+        for (int kt = 0; kt < nk; ++kt, ++g) {
+          const int s = g % kF8Stages;
+          const uint32_t ph = (g / kF8Stages) & 1;
+          if (!mbar_wait(full_f8(s), ph, abort)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_addr = base + kOffF8A + s * kAF8;
+          const uint32_t b_addr = base + kOffF8B + s * kBF8;
 #pragma unroll
-        for (int kk = 0; kk < BK / 32; ++kk) {
-          mma_f8f6f4(tmem, smem_desc_sw128(a_addr + 32 * kk), smem_desc_sw128(b_addr + 32 * kk), kIdesc,
-                     (kt | kk) != 0 ? 1u : 0u);
+          for (int kk = 0; kk < BK / 32; ++kk) {
+            mma_f8f6f4(acc, smem_desc_sw128(a_addr + 32 * kk), smem_desc_sw128(b_addr + 32 * kk), kIdesc,
+                       (kt | kk) != 0 ? 1u : 0u);
+          }
+          mma_commit(empty_f8(s));
         }
-        mma_commit(empty_f8(s));
+        mma_commit(acc_full(ab));
+        mma_tiles = lt + 1;
+        if (!ok) break;
       }
-      mma_commit(accum_full);
+    }
+  } else if (warp < kFirstEpiWarp) {
+    // ---------------- widen packed codes to E4M3 operand tiles ----------------
+    const int ct = threadIdx.x - kFirstConvWarp * 32;
+    int g = 0;
+    for (int tile = blockIdx.x; tile < num_tiles && !*abort; tile += gridDim.x) {
+      for (int kt = 0; kt < nk; ++kt, ++g) {
+        const int ps = g % kPackStages;
+        const uint32_t pph = (g / kPackStages) & 1;
+        const int fs = g % kF8Stages;
+        const uint32_t fph = (g / kF8Stages) & 1;
+        if (!mbar_wait(full_pack(ps), pph, abort)) break;
+        if (!mbar_wait(empty_f8(fs), fph ^ 1, abort)) break;
+        const uint32_t pa = base + kOffPackA + ps * kAPack;
+        const uint32_t pb = base + kOffPackB + ps * kBPack;
+        const uint32_t fa = base + kOffF8A + fs * kAF8;
+        const uint32_t fb = base + kOffF8B + fs * kBF8;
+#pragma unroll
+        for (int it = 0; it < BM * 4 / kConvThreads; ++it) {
+          const int i = ct + it * kConvThreads;
+          const int r = i >> 2, j = i & 3;
+          const uint4 w = lds128(pa + i * 16);
+          uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
+          widen_act(w.x, a0, a1);
+          widen_act(w.y, a2, a3);
+          widen_act(w.z, b0, b1);
+          widen_act(w.w, b2, b3);
+          sts128(fa + r * 128 + (((2 * j) ^ (r & 7)) << 4), a0, a1, a2, a3);
+          sts128(fa + r * 128 + (((2 * j + 1) ^ (r & 7)) << 4), b0, b1, b2, b3);
+        }
+#pragma unroll
+        for (int it = 0; it < BN * 4 / kConvThreads; ++it) {
+          const int i = ct + it * kConvThreads;
+          const int r = i >> 2, j = i & 3;
+          const uint4 w = lds128(pb + i * 16);
+          uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
+          widen_weight(w.x, a0, a1);
+          widen_weight(w.y, a2, a3);
+          widen_weight(w.z, b0, b1);
+          widen_weight(w.w, b2, b3);
+          sts128(fb + r * 128 + (((2 * j) ^ (r & 7)) << 4), a0, a1, a2, a3);
+          sts128(fb + r * 128 + (((2 * j + 1) ^ (r & 7)) << 4), b0, b1, b2, b3);
+        }
+        fence_proxy_async_smem();
+        mbar_arrive(empty_pack(ps));
+        mbar_arrive(full_f8(fs));
+      }
     }
   } else {
-    // ---------------- widen packed codes to E4M3 operand tiles ----------------
-    const int ct = threadIdx.x - 64;
-    for (int kt = 0; kt < nk; ++kt) {
-      const int ps = kt % kPackStages;
-      const uint32_t pph = (kt / kPackStages) & 1;
-      const int fs = kt % kF8Stages;
-      const uint32_t fph = (kt / kF8Stages) & 1;
-      if (!mbar_wait(full_pack(ps), pph, abort)) break;
-      if (!mbar_wait(empty_f8(fs), fph ^ 1, abort)) break;
-      const uint32_t pa = base + kOffPackA + ps * kAPack;
-      const uint32_t pb = base + kOffPackB + ps * kBPack;
-      const uint32_t fa = base + kOffF8A + fs * kAF8;
-      const uint32_t fb = base + kOffF8B + fs * kBF8;
-#pragma unroll
-      for (int i = ct; i < BM * 4; i += kConvThreads) {
-        const int r = i >> 2, j = i & 3;
-        const uint4 w = lds128(pa + r * 64 + j * 16);
-        uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
-        widen_act(w.x, a0, a1);
-        widen_act(w.y, a2, a3);
-        widen_act(w.z, b0, b1);
-        widen_act(w.w, b2, b3);
-        sts128(fa + r * 128 + (((2 * j) ^ (r & 7)) << 4), a0, a1, a2, a3);
-        sts128(fa + r * 128 + (((2 * j + 1) ^ (r & 7)) << 4), b0, b1, b2, b3);
-      }
-#pragma unroll
-      for (int i = ct; i < BN * 4; i += kConvThreads) {
-        const int r = i >> 2, j = i & 3;
-        const uint4 w = lds128(pb + r * 64 + j * 16);
-        uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
-        widen_weight(w.x, a0, a1);
-        widen_weight(w.y, a2, a3);
-        widen_weight(w.z, b0, b1);
-        widen_weight(w.w, b2, b3);
-        sts128(fb + r * 128 + (((2 * j) ^ (r & 7)) << 4), a0, a1, a2, a3);
-        sts128(fb + r * 128 + (((2 * j + 1) ^ (r & 7)) << 4), b0, b1, b2, b3);
-      }
-      fence_proxy_async_smem();
-      mbar_arrive(empty_pack(ps));
-      mbar_arrive(full_f8(fs));
-    }
-
     // ---------------- epilogue ----------------
-    const bool ok = mbar_wait(accum_full, 0, abort);
-    tc_fence_after();
-    const int G = p.G;
-    const int Gp = G | 1;  // odd row stride: conflict-free per-lane reads
-    float* Rs = reinterpret_cast<float*>(smem + kOffF8A);    // [G][BN]
-    float* Os = reinterpret_cast<float*>(smem + kOffPackA);  // [BM][Gp]
-    float* Ws = Os + BM * Gp;                                // [BN]
-    if (ok) {
-      for (int i = ct; i < G * BN; i += kConvThreads) {
-        const int b = i / BN, jn = i - b * BN;
-        const int n = n0 + jn;
-        Rs[i] = n < p.N ? p.rowsum[static_cast<int64_t>(b) * p.N + n] : 0.f;
-      }
-      for (int i = ct; i < BM * G; i += kConvThreads) {
-        const int r = i / G, b = i - r * G;
-        const int t = m0 + r;
-        float v = 0.f;
-        if (t < p.T) {
-          const float o = p.a_offset != nullptr ? p.a_offset[static_cast<int64_t>(t) * G + b] : 0.f;
-          v = o - 8.0f * p.a_scale[t];
-        }
-        Os[r * Gp + b] = v;
-      }
-      for (int i = ct; i < BN; i += kConvThreads) Ws[i] = n0 + i < p.N ? p.w_scale[n0 + i] : 0.f;
-    }
-    epi_bar();
-    const int quarter = warp & 3;
+    const int quarter = warp & 3;  // TMEM lanes this warp may read
     const int rl = quarter * 32 + lane;
-    const int t = m0 + rl;
-    const float sa = (ok && t < p.T) ? p.a_scale[t] : 0.f;
-    if (ok) {
-      for (int c = 0; c < BN / 32; ++c) {
-        uint32_t acc[32];
-        tmem_ld_32cols(tmem + (static_cast<uint32_t>(quarter * 32) << 16) + c * 32, acc);
+    const int G = p.G;
+    int lt = 0;
+    for (int tile = blockIdx.x; tile < num_tiles && !*abort; tile += gridDim.x, ++lt) {
+      const int ab = lt & 1;
+      const int m0 = (tile / p.n_tiles) * BM;
+      const int n0 = (tile % p.n_tiles) * BN;
+      if (!mbar_wait(acc_full(ab), (lt >> 1) & 1, abort)) break;
+      tc_fence_after();
+      const int t = m0 + rl;
+      const bool row_ok = t < p.T;
+      const float sa = row_ok ? __ldg(p.a_scale + t) : 0.f;
+      const float* orow = p.a_offset != nullptr && row_ok ? p.a_offset + static_cast<int64_t>(t) * G : nullptr;
+      const float o0 = (orow != nullptr ? __ldg(orow) : 0.f) - 8.0f * sa;
+      const uint32_t acc_tm = tmem + ab * kAccCols + (static_cast<uint32_t>(quarter * 32) << 16);
+      constexpr int CW = 16;  // accumulator columns per TMEM load
+      for (int c = 0; c < BN / CW; ++c) {
+        uint32_t acc[CW];
+        tmem_ld_16cols(acc_tm + c * CW, acc);
         tmem_ld_wait();
-        const int nb = n0 + c * 32;
-        if (t >= p.T || nb >= p.N) continue;
-        float y[32];
+        const int nb = n0 + c * CW;
+        if (!row_ok || nb >= p.N) continue;
+        const int nvalid = p.N - nb < CW ? p.N - nb : CW;
+        float y[CW];
+        if (nvalid == CW) {
+          const float4* r4 = reinterpret_cast<const float4*>(p.rowsum + nb);
 #pragma unroll
-        for (int jj = 0; jj < 32; ++jj) y[jj] = 0.f;
-        for (int b = 0; b < G; ++b) {
-          const float ob = Os[rl * Gp + b];
-          const float4* rr = reinterpret_cast<const float4*>(Rs + b * BN + c * 32);
+          for (int q4 = 0; q4 < CW / 4; ++q4) {
+            const float4 rv = __ldg(r4 + q4);
+            y[4 * q4] = o0 * rv.x; y[4 * q4 + 1] = o0 * rv.y; y[4 * q4 + 2] = o0 * rv.z; y[4 * q4 + 3] = o0 * rv.w;
+          }
+          for (int b = 1; b < G; ++b) {
+            const float ob = __ldg(orow + b) - 8.0f * sa;
+            const float4* rb4 = reinterpret_cast<const float4*>(p.rowsum + static_cast<int64_t>(b) * p.N + nb);
 #pragma unroll
-          for (int q4 = 0; q4 < 8; ++q4) {
-            const float4 w = rr[q4];
-            y[4 * q4] = fmaf(ob, w.x, y[4 * q4]);
-            y[4 * q4 + 1] = fmaf(ob, w.y, y[4 * q4 + 1]);
-            y[4 * q4 + 2] = fmaf(ob, w.z, y[4 * q4 + 2]);
-            y[4 * q4 + 3] = fmaf(ob, w.w, y[4 * q4 + 3]);
+            for (int q4 = 0; q4 < CW / 4; ++q4) {
+              const float4 rv = __ldg(rb4 + q4);
+              y[4 * q4] = fmaf(ob, rv.x, y[4 * q4]);
+              y[4 * q4 + 1] = fmaf(ob, rv.y, y[4 * q4 + 1]);
+              y[4 * q4 + 2] = fmaf(ob, rv.z, y[4 * q4 + 2]);
+              y[4 * q4 + 3] = fmaf(ob, rv.w, y[4 * q4 + 3]);
+            }
+          }
+          const float4* w4 = reinterpret_cast<const float4*>(p.w_scale + nb);
+#pragma unroll
+          for (int q4 = 0; q4 < CW / 4; ++q4) {
+            const float4 wv = __ldg(w4 + q4);
+            const float sw4[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const int jj = 4 * q4 + e;
+              const float accf = __uint_as_float(acc[jj]) * 262144.0f;  // exact: * 2^18
+              y[jj] = sw4[e] * fmaf(sa, accf, y[jj]);
+            }
+          }
+        } else {
+#pragma unroll
+          for (int jj = 0; jj < CW; ++jj) y[jj] = jj < nvalid ? o0 * __ldg(p.rowsum + nb + jj) : 0.f;
+          for (int b = 1; b < G; ++b) {
+            const float ob = __ldg(orow + b) - 8.0f * sa;
+            const float* rb = p.rowsum + static_cast<int64_t>(b) * p.N + nb;
+#pragma unroll
+            for (int jj = 0; jj < CW; ++jj)
+              if (jj < nvalid) y[jj] = fmaf(ob, __ldg(rb + jj), y[jj]);
+          }
+#pragma unroll
+          for (int jj = 0; jj < CW; ++jj) {
+            const float accf = __uint_as_float(acc[jj]) * 262144.0f;
+            y[jj] = jj < nvalid ? __ldg(p.w_scale + nb + jj) * fmaf(sa, accf, y[jj]) : 0.f;
           }
         }
-        const int nvalid = p.N - nb < 32 ? p.N - nb : 32;
-#pragma unroll
-        for (int jj = 0; jj < 32; ++jj) {
-          const float accf = __uint_as_float(acc[jj]) * 262144.0f;  // exact: * 2^18
-          y[jj] = Ws[c * 32 + jj] * fmaf(sa, accf, y[jj]);
-        }
-        store_out<OUT>(p.out, static_cast<int64_t>(t) * p.ldo + nb, y, nvalid);
+        store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, y, nvalid);
         if (p.acc_debug != nullptr) {
           int32_t* d = p.acc_debug + static_cast<int64_t>(t) * p.N + nb;
 #pragma unroll
-          for (int jj = 0; jj < 32; ++jj)
+          for (int jj = 0; jj < CW; ++jj)
             if (jj < nvalid) d[jj] = __float2int_rn(__uint_as_float(acc[jj]) * 262144.0f);
         }
       }
+      tc_fence_before();
+      mbar_arrive(acc_empty(ab));
     }
   }
 
   // ---------------- teardown ----------------
   if (*abort && warp == 0 && lane == 0) {
     // Let TMA copies still in flight land before the CTA's shared memory goes away.
-    for (int kt = issued - kPackStages < 0 ? 0 : issued - kPackStages; kt < issued; ++kt)
-      mbar_wait_teardown(full_pack(kt % kPackStages), (kt / kPackStages) & 1);
+    for (int g = issued - kPackStages < 0 ? 0 : issued - kPackStages; g < issued; ++g)
+      mbar_wait_teardown(full_pack(g % kPackStages), (g / kPackStages) & 1);
   }
-  if (*abort && warp == 1 && lane == 0) mbar_wait_teardown(accum_full, 0);
+  if (*abort && warp == 1 && lane == 0 && mma_tiles > 0) {
+    const int lt = mma_tiles - 1;
+    mbar_wait_teardown(acc_full(lt & 1), (lt >> 1) & 1);
+  }
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, BN);
+    tmem_dealloc(tmem, kTmemCols);
   }
   if (threadIdx.x == 0 && *abort && p.status != nullptr) atomicExch(p.status, kErrTimeout);
 }
@@ -390,6 +451,18 @@ bool make_code_map(CUtensorMap* m, const void* ptr, int64_t rows, int64_t row_by
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+int num_sms() {
+  static int sms[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (sms[dev] == 0) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    sms[dev] = v;
+  }
+  return sms[dev];
+}
+
 template <int OUT>
 int launch_gemm(const CUtensorMap& ma, const CUtensorMap& mb, const GemmParams& p, cudaStream_t s) {
   auto kern = w4a4_gemm_kernel<OUT>;
@@ -399,7 +472,10 @@ int launch_gemm(const CUtensorMap& ma, const CUtensorMap& mb, const GemmParams& 
     attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
   });
   if (attr_err != cudaSuccess) return OFFQ_ERR_CUDA;
-  const dim3 grid((p.N + BN - 1) / BN, (p.T + BM - 1) / BM);
+  const int sms = num_sms();
+  if (sms <= 0) return OFFQ_ERR_CUDA;
+  const int tiles = p.m_tiles * p.n_tiles;
+  const int grid = tiles < sms ? tiles : sms;
   kern<<<grid, kThreads, kSmemBytes, s>>>(ma, mb, p);
   return launch_status();
 }
@@ -441,6 +517,8 @@ extern "C" int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, co
   p.K = static_cast<int>(K);
   p.G = static_cast<int>(K / g);
   p.out_dtype = out_dtype;
+  p.m_tiles = static_cast<int>((T + BM - 1) / BM);
+  p.n_tiles = static_cast<int>((N + BN - 1) / BN);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   switch (out_dtype) {
     case OFFQ_F32: return launch_gemm<OFFQ_F32>(ma, mb, p, s);

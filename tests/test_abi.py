@@ -79,7 +79,6 @@ def test_gemm_argument_checks(lib):
     assert gemm(lib, ldo=32) == Q.OFFQ_ERR_INVALID_ARG
     assert gemm(lib, dt=9) == Q.OFFQ_ERR_INVALID_ARG
     assert gemm(lib, K=131072, g=4096) == Q.OFFQ_ERR_UNSUPPORTED
-    assert gemm(lib, K=32768, g=32) == Q.OFFQ_ERR_UNSUPPORTED   # more offset blocks than the epilogue stages
     assert gemm(lib, w=None) == Q.OFFQ_ERR_INVALID_ARG
     assert gemm(lib, a=A8) == Q.OFFQ_ERR_MISALIGNED
     assert gemm(lib, out=A8) == Q.OFFQ_ERR_MISALIGNED

@@ -113,6 +113,8 @@ def test_oracle_codes_through_gemm():
     (1, 4096, 11008, 4096, "bf16", None),  # one decode token
     (200, 4096, 4096, 4096, "bf16", None),
     (129, 2048, 257, 2048, "f32", 260),
+    (40, 4096, 512, 32, "f32", None),      # 128 offset blocks of 32 channels
+    (300, 1024, 800, 128, "bf16", None),   # the paper's group size, 8 blocks; several tiles per CTA
 ])
 def test_layers(T, K, N, g, out_dt, ldo):
     _check_layer(T, K, N, g, out_dt, ldo=ldo, seed=T + K)
