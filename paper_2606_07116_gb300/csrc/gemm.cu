@@ -85,6 +85,7 @@ struct GemmParams {
   int* status;
   int T, N, K, G, out_dtype;
   int m_tiles, n_tiles;
+  int vec_ok;  // rowsum and w_scale rows are 16-byte aligned (float4 loads allowed)
 };
 
 __device__ __forceinline__ bool mbar_wait_teardown(uint32_t bar, uint32_t parity) {
@@ -329,8 +330,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int t = m0 + rl;
       const bool row_ok = t < p.T;
       const float sa = row_ok ? __ldg(p.a_scale + t) : 0.f;
-      const float* orow = p.a_offset != nullptr && row_ok ? p.a_offset + static_cast<int64_t>(t) * G : nullptr;
-      const float o0 = (orow != nullptr ? __ldg(orow) : 0.f) - 8.0f * sa;
+      const bool has_off = p.a_offset != nullptr && row_ok;
+      const float* orow = has_off ? p.a_offset + static_cast<int64_t>(t) * G : p.a_scale;
+      const float o0 = (has_off ? __ldg(orow) : 0.f) - 8.0f * sa;
       const uint32_t acc_tm = tmem + ab * kAccCols + (static_cast<uint32_t>(quarter * 32) << 16);
       constexpr int CW = 16;  // accumulator columns per TMEM load
       for (int c = 0; c < BN / CW; ++c) {
@@ -341,7 +343,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!row_ok || nb >= p.N) continue;
         const int nvalid = p.N - nb < CW ? p.N - nb : CW;
         float y[CW];
-        if (nvalid == CW) {
+        if (nvalid == CW && p.vec_ok) {
           const float4* r4 = reinterpret_cast<const float4*>(p.rowsum + nb);
 #pragma unroll
           for (int q4 = 0; q4 < CW / 4; ++q4) {
@@ -349,7 +351,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             y[4 * q4] = o0 * rv.x; y[4 * q4 + 1] = o0 * rv.y; y[4 * q4 + 2] = o0 * rv.z; y[4 * q4 + 3] = o0 * rv.w;
           }
           for (int b = 1; b < G; ++b) {
-            const float ob = __ldg(orow + b) - 8.0f * sa;
+            const float ob = (has_off ? __ldg(orow + b) : 0.f) - 8.0f * sa;
             const float4* rb4 = reinterpret_cast<const float4*>(p.rowsum + static_cast<int64_t>(b) * p.N + nb);
 #pragma unroll
             for (int q4 = 0; q4 < CW / 4; ++q4) {
@@ -376,7 +378,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int jj = 0; jj < CW; ++jj) y[jj] = jj < nvalid ? o0 * __ldg(p.rowsum + nb + jj) : 0.f;
           for (int b = 1; b < G; ++b) {
-            const float ob = __ldg(orow + b) - 8.0f * sa;
+            const float ob = (has_off ? __ldg(orow + b) : 0.f) - 8.0f * sa;
             const float* rb = p.rowsum + static_cast<int64_t>(b) * p.N + nb;
 #pragma unroll
             for (int jj = 0; jj < CW; ++jj)
@@ -518,6 +520,7 @@ extern "C" int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, co
   p.G = static_cast<int>(K / g);
   p.out_dtype = out_dtype;
   p.m_tiles = static_cast<int>((T + BM - 1) / BM);
+  p.vec_ok = aligned(w_offsum, 16) && aligned(w_scale, 16) && (N % 4 == 0);
   p.n_tiles = static_cast<int>((N + BN - 1) / BN);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   switch (out_dtype) {

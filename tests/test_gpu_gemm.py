@@ -115,6 +115,7 @@ def test_oracle_codes_through_gemm():
     (129, 2048, 257, 2048, "f32", 260),
     (40, 4096, 512, 32, "f32", None),      # 128 offset blocks of 32 channels
     (300, 1024, 800, 128, "bf16", None),   # the paper's group size, 8 blocks; several tiles per CTA
+    (50, 1024, 258, 256, "bf16", 264),     # N % 4 != 0 with 4 offset blocks (scalar epilogue loads)
 ])
 def test_layers(T, K, N, g, out_dt, ldo):
     _check_layer(T, K, N, g, out_dt, ldo=ldo, seed=T + K)
