@@ -177,7 +177,7 @@ class GpuStep:
             host = torch.from_numpy(x).to(dt).pin_memory()
             dev = host.to(device)
             g = W.block_for(K)
-            codes = torch.empty((T, K // 2), dtype=torch.uint8, device=device)
+            codes = torch.empty((Q.padded_rows(T), K // 2), dtype=torch.uint8, device=device)
             scale = torch.empty((T,), dtype=torch.float32, device=device)
             off = torch.empty((T, K // g), dtype=torch.float32, device=device)
             flags = (Q.OFFQ_ROTATE if rotate else 0) | Q.OFFQ_OFFSET

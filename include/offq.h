@@ -38,14 +38,20 @@
  * Code formats (the paper fixes the 4-bit uniform grid, not a bit layout):
  *   Activation codes: Eq. 1's unsigned form with zero-point 8. A residual
  *     quantized to q in [-7, 7] is stored as the nibble u = q + 8 (1..15). Two
- *     nibbles per byte, the even channel in the low nibble; row t occupies
- *     bytes [t*K/2, (t+1)*K/2).
+ *     nibbles per byte, the even channel in the low nibble, so row t is a
+ *     string of K/2 bytes.
  *   Weight codes: per-output-channel signed q in [-7, 7], sign-magnitude,
  *     interleaved per group of 8 channels c0..c7 held in 4 bytes B0..B3:
  *       Bj bits 0-2 = |q(c_2j)|, bit 7 = sign(q(c_2j)),
  *       Bj bits 4-6 = |q(c_2j+1)|, bit 3 = sign(q(c_(2j-1) mod 8)).
  *     (This lets the GEMM widen 8 codes to fp8 tensor-core operands with one
- *     rotate and two masks.) Row n occupies bytes [n*K/2, (n+1)*K/2).
+ *     rotate and two masks.) Row n is a string of K/2 bytes.
+ *   Tiled operand layout (activation and weight codes): rows are grouped by
+ *     32 and split into 16-byte chunks of 32 codes; byte j of row r is stored
+ *     at ((r / 32) * (K / 32) + j / 16) * 512 + (r % 32) * 16 + j % 16. A
+ *     buffer of R rows therefore holds ceil(R/32)*32 rows (offq_act_codes_bytes,
+ *     offq_weight_codes_bytes). The GEMM's warps then load 32 rows x 16 bytes
+ *     as 512 contiguous bytes. KV-cache codes stay row-major.
  */
 #ifndef OFFQ_H
 #define OFFQ_H
@@ -94,7 +100,9 @@ enum {
  *   K       channels, a multiple of g and of 32, K <= 32768.
  *   g       block size, power of two in [32, 8192].
  *   flags   OR of OFFQ_ROTATE, OFFQ_OFFSET.
- *   codes   device, [T][K/2] bytes (activation code format), 16-byte aligned.
+ *   codes   device, offq_act_codes_bytes(T, K) bytes, activation code format in
+ *           the tiled operand layout, 16-byte aligned (rows beyond T in the
+ *           last 32-row group are left as they are).
  *   scale   device, [T] float32.
  *   offset  device, [T][K/g] float32; required with OFFQ_OFFSET; when given
  *           without OFFQ_OFFSET it is filled with zeros; may be NULL otherwise.
@@ -116,13 +124,13 @@ int offq_quantize_act(const void* x, int x_dtype, int64_t T, int64_t K, int64_t 
  * fp8 values; every partial sum is an integer below 2^24), dequantized in fp32
  * and rounded once to the output type.
  *
- *   a_codes   device, [T][K/2] activation codes (offq_quantize_act), 16-B aligned.
+ *   a_codes   device, tiled activation codes of T rows (offq_quantize_act), 16-B aligned.
  *   a_scale   device, [T] float32.
  *   a_offset  device, [T][K/g] float32, or NULL for all-zero offsets.
  *   T, N, K   tokens, output channels, input channels; T >= 0, N >= 1,
  *             K a multiple of g and of 32, K <= 65536.
  *   g         block size used when the codes were made (power of two, 32..8192).
- *   w_codes   device, [N][K/2] weight codes (offq_prepare_weight), 16-B aligned.
+ *   w_codes   device, tiled weight codes of N rows (offq_prepare_weight), 16-B aligned.
  *   w_scale   device, [N] float32.
  *   w_offsum  device, [K/g][N] float32: R[b][n] = sum_{k in block b} q_w[n][k],
  *             the integer block row sums of the weight codes (exact in fp32).
@@ -172,12 +180,20 @@ int offq_kv4_quantize(const void* kv, int dtype, int64_t T, int32_t H, int32_t h
  *   w         device, [N][K] of dtype, row-major, 16-byte aligned.
  *   N, K, g   as in offq_w4a4_linear.
  *   rotate    nonzero to fuse the block Hadamard.
- *   w_codes   device, [N][K/2] weight code format, 16-B aligned.
+ *   w_codes   device, offq_weight_codes_bytes(N, K) bytes, weight code format in
+ *             the tiled operand layout (padding rows set to zero), 16-B aligned.
  *   w_scale   device, [N] float32.
  *   w_offsum  device, [K/g][N] float32.
  */
 int offq_prepare_weight(const void* w, int dtype, int64_t N, int64_t K, int32_t g, int32_t rotate,
                         uint8_t* w_codes, float* w_scale, float* w_offsum, void* stream);
+
+/* Bytes of a tiled activation-code buffer for T rows of K codes (-1 if K is
+ * not a positive multiple of 32 or T < 0): ceil(T/32) * 32 * K / 2. */
+int64_t offq_act_codes_bytes(int64_t T, int64_t K);
+
+/* Bytes of a tiled weight-code buffer for N rows of K codes (-1 on bad sizes). */
+int64_t offq_weight_codes_bytes(int64_t N, int64_t K);
 
 /*
  * offq_get_device_status -- synchronizes `stream`, returns the device status

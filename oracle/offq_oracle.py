@@ -193,6 +193,37 @@ def unpack_weight_codes(packed: np.ndarray) -> np.ndarray:
     return q.reshape(lead + (2 * p.shape[-1],))
 
 
+TILE_ROWS = 32   # rows per tile of the GEMM operand layout
+TILE_CODES = 32  # codes (16 bytes) per row of a tile
+
+
+def tile_codes(packed: np.ndarray) -> np.ndarray:
+    """Row-major packed codes [R, K/2] -> the tiled byte order of the GEMM operands.
+
+    Rows are padded with zero bytes to a multiple of 32. The result is the
+    array [ceil(R/32), K/32, 32, 16] flattened: tile (rb, c) of 512 bytes holds
+    the 16-byte chunk c (codes 32c .. 32c+31) of rows 32 rb .. 32 rb + 31, one
+    row after the other. Byte (r, j) of the row-major input lands at
+    ((r // 32) * (K // 32) + j // 16) * 512 + (r % 32) * 16 + j % 16.
+    """
+    p = np.asarray(packed, dtype=np.uint8)
+    R, KB = p.shape
+    if KB % 16:
+        raise ValueError("K must be a multiple of 32")
+    Rp = -(-R // TILE_ROWS) * TILE_ROWS
+    q = np.zeros((Rp, KB), dtype=np.uint8)
+    q[:R] = p
+    return q.reshape(Rp // TILE_ROWS, TILE_ROWS, KB // 16, 16).transpose(0, 2, 1, 3).reshape(-1).copy()
+
+
+def untile_codes(tiled: np.ndarray, R: int, K: int) -> np.ndarray:
+    """Inverse of :func:`tile_codes`: the first R rows as row-major [R, K/2]."""
+    t = np.asarray(tiled, dtype=np.uint8).reshape(-1)
+    Rp = -(-R // TILE_ROWS) * TILE_ROWS
+    KB = K // 2
+    return t[:Rp * KB].reshape(Rp // TILE_ROWS, KB // 16, TILE_ROWS, 16).transpose(0, 2, 1, 3).reshape(Rp, KB)[:R].copy()
+
+
 # ---------------------------------------------------------------------------
 # Online activation path  (Sec. 3.2 offsetting + Sec. 3 Eq. 1)
 # ---------------------------------------------------------------------------

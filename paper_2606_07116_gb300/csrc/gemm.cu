@@ -13,15 +13,26 @@
 // "+8" is removed in the epilogue with the weight block row sums R, together
 // with the offsets: sum_b 8 s_a R[b][n] = 8 s_a sum_k q_w[n][k].
 //
-// Persistent CTAs (one per SM), tile 128 (tokens) x 256 (channels), k-tile 128
-// codes. Warp roles:
-//   warp 0       TMA producer: packed int4 tiles of A and B into a 4-stage ring
-//   warp 1       TMEM allocation and the single-thread MMA issuer
-//   warps 2-9    widen packed codes to E4M3 tiles in the 128-byte-swizzled
-//                K-major layout of the MMA (2-stage ring)
-//   warps 10-13  epilogue from TMEM (each warp owns one 32-lane quarter of the
-//                accumulator); two accumulator buffers (2 x 256 columns) let the
-//                epilogue of a tile overlap the main loop of the next
+// Design. Widening 4-bit codes to fp8 operands costs shared-memory bandwidth,
+// which the tensor core's operand reads share. So:
+//  * two SMs form a pair (cluster of 2, tcgen05 cta_group::2) computing a
+//    256 x 256 tile; each SM holds 128 rows of A and half (128 rows) of B, and
+//    the pair's MMA reads each half of B once for both SMs;
+//  * A never touches shared memory: converter warps load its packed codes with
+//    coalesced 16-byte loads, widen them in registers and write the E4M3
+//    operand straight into tensor memory (tcgen05.st), where the MMA reads it;
+//  * B is loaded the same way, widened, and stored once into the 128-byte-
+//    swizzled K-major shared-memory layout the MMA reads;
+//  * both code matrices use a 32-row tiled layout, so each 16-byte load of a
+//    warp covers 512 contiguous bytes and lane i receives row i.
+// Per SM and 128-code k-tile this moves 16 KB of shared memory for the MMA's B
+// reads and 16 KB of B stores, against 512 cycles of MMA work.
+//
+// Warp roles per CTA (17 warps):
+//   warp 0       TMEM allocation; in the leader CTA, lane 0 issues the MMAs
+//   warps 1-4    A converters (one per 32-lane quarter of TMEM)
+//   warps 5-8    B converters (32 rows each)
+//   warps 9-16   epilogue (two per TMEM quarter, 128 columns each)
 // Every wait is bounded; a wait that runs out aborts the CTA and records
 // OFFQ_ERR_TIMEOUT in the device status word.
 #include <cuda.h>
@@ -38,43 +49,35 @@ namespace {
 
 using namespace offq;
 
-constexpr int BM = 128;
-constexpr int BN = 256;
-constexpr int BK = 128;  // codes per k-tile (128 fp8 bytes = one swizzle row)
-constexpr int kPackStages = 4;
-constexpr int kF8Stages = 2;
-constexpr int kConvWarps = 8;
-constexpr int kEpiWarps = 4;
-constexpr int kConvThreads = kConvWarps * 32;
-constexpr int kEpiThreads = kEpiWarps * 32;
-constexpr int kFirstConvWarp = 2;
-constexpr int kFirstEpiWarp = kFirstConvWarp + kConvWarps;
-constexpr int kThreads = (kFirstEpiWarp + kEpiWarps) * 32;
-constexpr int kAccCols = BN;          // fp32 accumulator columns per buffer
-constexpr int kTmemCols = 2 * kAccCols;  // double-buffered accumulator
-constexpr int kMaxEpilogueG = 2048;
+constexpr int BM = 128;            // rows of A per CTA (256 per pair)
+constexpr int BN = 256;            // output channels per pair tile (128 rows of B per CTA)
+constexpr int BNH = BN / 2;        // rows of B held by one CTA
+constexpr int BK = 128;            // codes per k-tile
+constexpr int kChunksPerKt = BK / 32;  // 16-byte packed chunks per row per k-tile
+constexpr int kStages = 4;
+constexpr int kAWarps = 4, kBWarps = 4, kEpiWarps = 8;
+constexpr int kFirstA = 1, kFirstB = kFirstA + kAWarps, kFirstEpi = kFirstB + kBWarps;
+constexpr int kThreads = (kFirstEpi + kEpiWarps) * 32;
+constexpr int kConvThreadsPerCta = (kAWarps + kBWarps) * 32;
+constexpr int kEpiThreadsPerCta = kEpiWarps * 32;
+constexpr int kAccCols = BN;       // fp32 accumulator columns (TMEM lanes = rows)
+constexpr int kACol0 = kAccCols;   // A operand stages live in TMEM after the accumulator
+constexpr int kAColsPerStage = BK / 4;  // 4 E4M3 values per 32-bit column
+constexpr int kTmemCols = 512;
+static_assert(kACol0 + kStages * kAColsPerStage <= kTmemCols, "TMEM budget");
 
-constexpr int kAPack = BM * BK / 2;  // 8 KB
-constexpr int kBPack = BN * BK / 2;  // 16 KB
-constexpr int kAF8 = BM * BK;        // 16 KB
-constexpr int kBF8 = BN * BK;        // 32 KB
-
-constexpr int kOffF8A = 0;
-constexpr int kOffF8B = kOffF8A + kF8Stages * kAF8;
-constexpr int kOffPackA = kOffF8B + kF8Stages * kBF8;
-constexpr int kOffPackB = kOffPackA + kPackStages * kAPack;
-constexpr int kOffBars = kOffPackB + kPackStages * kBPack;
-constexpr int kNumBars = 2 * kPackStages + 2 * kF8Stages + 4;
+constexpr int kBStage = BNH * BK;  // 16 KB of E4M3 per stage
+constexpr int kOffB = 0;
+constexpr int kOffBars = kOffB + kStages * kBStage;
+constexpr int kNumBars = 2 * kStages + 2;
 constexpr int kOffMisc = kOffBars + kNumBars * 8;
-constexpr int kSmemBytes = kOffMisc + 64 + 1024;  // + alignment slack for the 1024-byte base
+constexpr int kSmemBytes = kOffMisc + 64 + 1024;  // + slack to align the base to 1024
 
-static_assert(kOffPackA % 1024 == 0 && kOffF8B % 1024 == 0, "MMA tiles need 1024-byte alignment");
-static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
-static_assert(BM * 4 % kConvThreads == 0 && BN * 4 % kConvThreads == 0, "even converter split");
-
-constexpr uint32_t kIdesc = idesc_e4m3_f32(BM, BN);
+constexpr uint32_t kIdesc = idesc_e4m3_f32(2 * BM, BN);  // pair MMA: M = 256, N = 256
 
 struct GemmParams {
+  const uint8_t* a_codes;  // tiled [ceil(T/32)*32][K/2]
+  const uint8_t* w_codes;  // tiled [ceil(N/32)*32][K/2]
   const float* a_scale;
   const float* a_offset;  // [T][G] or nullptr
   const float* w_scale;
@@ -83,17 +86,133 @@ struct GemmParams {
   int64_t ldo;
   int32_t* acc_debug;
   int* status;
-  int T, N, K, G, out_dtype;
-  int m_tiles, n_tiles;
-  int vec_ok;  // rowsum and w_scale rows are 16-byte aligned (float4 loads allowed)
+  int T, N, K, G;
+  int m_pairs, n_tiles;    // pair tiles: m_pairs x n_tiles
+  int t_blocks, n_blocks;  // 32-row tiles present in the code buffers
+  int kchunks;             // K / 32
+  int vec_ok;              // rowsum and w_scale rows are 16-byte aligned
 };
 
-__device__ __forceinline__ bool mbar_wait_teardown(uint32_t bar, uint32_t parity) {
+// ---------------------------------------------------------------------------
+// Cluster / pair helpers
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Address of the same shared-memory offset in the leader CTA (rank 0).
+__device__ __forceinline__ uint32_t leader_addr(uint32_t local) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(0u));
+  return r;
+}
+
+__device__ __forceinline__ void arrive_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+__device__ __forceinline__ bool try_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n"
+      ".reg .pred p;\n"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+      "selp.u32 %0, 1, 0, p;\n"
+      "}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ bool wait_cluster(uint32_t bar, uint32_t parity, volatile int* abort) {
+  if (try_wait_cluster(bar, parity)) return true;
   const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity)) {
+  while (true) {
+    if (try_wait_cluster(bar, parity)) return true;
+    if (*abort) return false;
+    if (clock64() - t0 > kWaitCycles) {
+      *abort = 1;
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ bool wait_teardown(uint32_t bar, uint32_t parity) {
+  const long long t0 = clock64();
+  while (!try_wait_cluster(bar, parity)) {
     if (clock64() - t0 > kWaitCycles) return false;
   }
   return true;
+}
+
+__device__ __forceinline__ void tmem_alloc2(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_relinquish2() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc2(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+// D[tmem] (+)= A[tmem] * B[smem]^T over the CTA pair, E4M3 operands, fp32 accumulate.
+__device__ __forceinline__ void mma2_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                        uint32_t accumulate) {
+  asm volatile(
+      "{\n"
+      ".reg .pred p;\n"
+      "setp.ne.b32 p, %4, 0;\n"
+      "tcgen05.mma.cta_group::2.kind::f8f6f4 [%0], [%1], %2, %3, p;\n"
+      "}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrives on the barrier at this offset in both CTAs of the pair once every
+// MMA issued so far by this thread is done.
+__device__ __forceinline__ void mma2_commit_both(uint32_t bar) {
+  const uint16_t mask = 0x3;
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+          bar),
+      "h"(mask)
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_32cols(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+      "{%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+      "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]),
+      "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]),
+      "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+__device__ __forceinline__ uint4 ldg_stream(const uint8_t* p) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
+__device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
 }
 
 // Eight activation codes (u = q + 8 nibbles) -> eight E4M3 bytes, ordered
@@ -109,17 +228,6 @@ __device__ __forceinline__ void widen_act(uint32_t w, uint32_t& lo, uint32_t& hi
 __device__ __forceinline__ void widen_weight(uint32_t w, uint32_t& lo, uint32_t& hi) {
   lo = w & 0x87878787u;
   hi = __funnelshift_r(w, w, 4) & 0x87878787u;
-}
-
-__device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
-  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
-}
-
-__device__ __forceinline__ uint4 lds128(uint32_t addr) {
-  uint4 r;
-  asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "r"(addr)
-               : "memory");
-  return r;
 }
 
 template <int OUT, int CW>
@@ -160,14 +268,34 @@ __device__ __forceinline__ void store_out(void* out, int64_t off, const float* y
   }
 }
 
-// Persistent kernel: CTA b processes tiles b, b + gridDim.x, ... (tile index =
-// m_tile * n_tiles + n_tile). The k-tile pipeline counters run across tiles, and
-// the accumulator alternates between two TMEM buffers so the epilogue of one tile
-// overlaps the main loop of the next.
+// Loads the four 16-byte chunks of k-tile kt of one row of a tiled code matrix
+// (zeros where the row block or the chunk does not exist).
+__device__ __forceinline__ void load_kt(const uint8_t* codes, int rb, int rb_count, int kchunks, int kt, int lane,
+                                        uint4 (&v)[kChunksPerKt]) {
+#pragma unroll
+  for (int j = 0; j < kChunksPerKt; ++j) {
+    const int c = kt * kChunksPerKt + j;
+    if (rb < rb_count && c < kchunks)
+      v[j] = ldg_stream(codes + (static_cast<int64_t>(rb) * kchunks + c) * 512 + lane * 16);
+    else
+      v[j] = make_uint4(0u, 0u, 0u, 0u);
+  }
+}
+
+// Row block (of 32 rows) of this CTA's A rows / B rows for a pair tile.
+__device__ __forceinline__ int a_block(const GemmParams& p, int tile, uint32_t rank, int quarter) {
+  return ((tile / p.n_tiles) * 2 * BM + static_cast<int>(rank) * BM + quarter * 32) >> 5;
+}
+
+__device__ __forceinline__ int b_block(const GemmParams& p, int tile, uint32_t rank, int wb) {
+  return ((tile % p.n_tiles) * BN + static_cast<int>(rank) * BNH + wb * 32) >> 5;
+}
+
+// Persistent pair kernel: cluster c processes pair tiles c, c + clusters, ...
+// (pair tile index = m_pair * n_tiles + n_tile). The k-tile counter g runs
+// across tiles so the stage ring never drains between tiles.
 template <int OUT>
-__global__ void __launch_bounds__(kThreads, 1)
-    w4a4_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
-                     const GemmParams p) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_gemm_kernel(const GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -175,167 +303,166 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const int cluster = blockIdx.x >> 1;
+  const int clusters = gridDim.x >> 1;
   const int nk = (p.K + BK - 1) / BK;
-  const int num_tiles = p.m_tiles * p.n_tiles;
+  const int num_tiles = p.m_pairs * p.n_tiles;
 
   const uint32_t bar0 = base + kOffBars;
-  auto full_pack = [&](int s) { return bar0 + 8u * s; };
-  auto empty_pack = [&](int s) { return bar0 + 8u * (kPackStages + s); };
-  auto full_f8 = [&](int s) { return bar0 + 8u * (2 * kPackStages + s); };
-  auto empty_f8 = [&](int s) { return bar0 + 8u * (2 * kPackStages + kF8Stages + s); };
-  auto acc_full = [&](int b) { return bar0 + 8u * (2 * kPackStages + 2 * kF8Stages + b); };
-  auto acc_empty = [&](int b) { return bar0 + 8u * (2 * kPackStages + 2 * kF8Stages + 2 + b); };
+  auto full = [&](int s) { return bar0 + 8u * s; };                // leader: operands of stage s ready
+  auto empty = [&](int s) { return bar0 + 8u * (kStages + s); };   // both: stage s consumed
+  const uint32_t acc_full = bar0 + 8u * (2 * kStages);             // both: accumulator complete
+  const uint32_t acc_empty = bar0 + 8u * (2 * kStages + 1);        // leader: accumulator drained
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kOffMisc);
   volatile int* abort = reinterpret_cast<volatile int*>(smem + kOffMisc + 16);
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kPackStages; ++s) {
-      mbar_init(full_pack(s), 1);
-      mbar_init(empty_pack(s), kConvThreads);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(full(s), 2 * kConvThreadsPerCta);
+      mbar_init(empty(s), 1);
     }
-    for (int s = 0; s < kF8Stages; ++s) {
-      mbar_init(full_f8(s), kConvThreads);
-      mbar_init(empty_f8(s), 1);
-    }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(acc_full(b), 1);
-      mbar_init(acc_empty(b), kEpiThreads);
-    }
+    mbar_init(acc_full, 1);
+    mbar_init(acc_empty, 2 * kEpiThreadsPerCta);
     *abort = 0;
     mbar_fence_init();
-    tma_prefetch_desc(&tmap_a);
-    tma_prefetch_desc(&tmap_b);
   }
-  if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
-    tmem_relinquish();
+  if (warp == 0) {
+    tmem_alloc2(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish2();
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();  // barriers initialised and TMEM allocated in both CTAs
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-
-  int issued = 0;     // producer: k-tiles whose TMA loads were issued (global count)
-  int mma_tiles = 0;  // MMA issuer: tiles whose accumulation was committed
+  int mma_tiles = 0;
 
   if (warp == 0) {
-    // ---------------- TMA producer ----------------
-    if (lane == 0) {
-      int g = 0;
-      for (int tile = blockIdx.x; tile < num_tiles && !*abort; tile += gridDim.x) {
-        const int m0 = (tile / p.n_tiles) * BM;
-        const int n0 = (tile % p.n_tiles) * BN;
-        for (int kt = 0; kt < nk; ++kt, ++g) {
-          const int s = g % kPackStages;
-          const uint32_t ph = (g / kPackStages) & 1;
-          if (!mbar_wait(empty_pack(s), ph ^ 1, abort)) break;
-          mbar_arrive_expect_tx(full_pack(s), kAPack + kBPack);
-          tma_load_2d(base + kOffPackA + s * kAPack, &tmap_a, full_pack(s), kt * (BK / 2), m0);
-          tma_load_2d(base + kOffPackB + s * kBPack, &tmap_b, full_pack(s), kt * (BK / 2), n0);
-          issued = g + 1;
-        }
-      }
-    }
-  } else if (warp == 1) {
-    // ---------------- MMA issuer ----------------
-    if (lane == 0) {
+    // ---------------- MMA issuer (leader CTA) ----------------
+    if (rank == 0 && lane == 0) {
       int g = 0, lt = 0;
-      for (int tile = blockIdx.x; tile < num_tiles && !*abort; tile += gridDim.x, ++lt) {
-        const int ab = lt & 1;
-        if (!mbar_wait(acc_empty(ab), ((lt >> 1) & 1) ^ 1, abort)) break;
+      for (int tile = cluster; tile < num_tiles && !*abort; tile += clusters, ++lt) {
+        if (!wait_cluster(acc_empty, (lt & 1) ^ 1, abort)) break;
         tc_fence_after();
-        const uint32_t acc = tmem + ab * kAccCols;
         bool ok = true;
         for (int kt = 0; kt < nk; ++kt, ++g) {
-          const int s = g % kF8Stages;
-          const uint32_t ph = (g / kF8Stages) & 1;
-          if (!mbar_wait(full_f8(s), ph, abort)) {
+          const int s = g % kStages;
+          if (!wait_cluster(full(s), (g / kStages) & 1, abort)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t a_addr = base + kOffF8A + s * kAF8;
-          const uint32_t b_addr = base + kOffF8B + s * kBF8;
+          const uint32_t b_addr = base + kOffB + s * kBStage;
 #pragma unroll
           for (int kk = 0; kk < BK / 32; ++kk) {
-            mma_f8f6f4(acc, smem_desc_sw128(a_addr + 32 * kk), smem_desc_sw128(b_addr + 32 * kk), kIdesc,
-                       (kt | kk) != 0 ? 1u : 0u);
+            mma2_ts(tmem, tmem + kACol0 + s * kAColsPerStage + 8 * kk, smem_desc_sw128(b_addr + 32 * kk), kIdesc,
+                    (kt | kk) != 0 ? 1u : 0u);
           }
-          mma_commit(empty_f8(s));
+          mma2_commit_both(empty(s));
         }
-        mma_commit(acc_full(ab));
+        mma2_commit_both(acc_full);
         mma_tiles = lt + 1;
         if (!ok) break;
       }
     }
-  } else if (warp < kFirstEpiWarp) {
-    // ---------------- widen packed codes to E4M3 operand tiles ----------------
-    const int ct = threadIdx.x - kFirstConvWarp * 32;
-    int g = 0;
-    for (int tile = blockIdx.x; tile < num_tiles && !*abort; tile += gridDim.x) {
-      for (int kt = 0; kt < nk; ++kt, ++g) {
-        const int ps = g % kPackStages;
-        const uint32_t pph = (g / kPackStages) & 1;
-        const int fs = g % kF8Stages;
-        const uint32_t fph = (g / kF8Stages) & 1;
-        if (!mbar_wait(full_pack(ps), pph, abort)) break;
-        if (!mbar_wait(empty_f8(fs), fph ^ 1, abort)) break;
-        const uint32_t pa = base + kOffPackA + ps * kAPack;
-        const uint32_t pb = base + kOffPackB + ps * kBPack;
-        const uint32_t fa = base + kOffF8A + fs * kAF8;
-        const uint32_t fb = base + kOffF8B + fs * kBF8;
+  } else if (warp < kFirstB) {
+    // ---------------- A converters: packed codes -> E4M3 in TMEM ----------------
+    const int quarter = warp & 3;
+    const uint32_t tm_lane = static_cast<uint32_t>(quarter * 32) << 16;
+    const uint32_t full_l = leader_addr(full(0));
+    int g = 0, tile = cluster, kt = 0;
+    uint4 nxt[kChunksPerKt];
+    if (tile < num_tiles) load_kt(p.a_codes, a_block(p, tile, rank, quarter), p.t_blocks, p.kchunks, 0, lane, nxt);
+    while (tile < num_tiles && !*abort) {
+      uint4 cur[kChunksPerKt];
 #pragma unroll
-        for (int it = 0; it < BM * 4 / kConvThreads; ++it) {
-          const int i = ct + it * kConvThreads;
-          const int r = i >> 2, j = i & 3;
-          const uint4 w = lds128(pa + i * 16);
-          uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
-          widen_act(w.x, a0, a1);
-          widen_act(w.y, a2, a3);
-          widen_act(w.z, b0, b1);
-          widen_act(w.w, b2, b3);
-          sts128(fa + r * 128 + (((2 * j) ^ (r & 7)) << 4), a0, a1, a2, a3);
-          sts128(fa + r * 128 + (((2 * j + 1) ^ (r & 7)) << 4), b0, b1, b2, b3);
-        }
-#pragma unroll
-        for (int it = 0; it < BN * 4 / kConvThreads; ++it) {
-          const int i = ct + it * kConvThreads;
-          const int r = i >> 2, j = i & 3;
-          const uint4 w = lds128(pb + i * 16);
-          uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
-          widen_weight(w.x, a0, a1);
-          widen_weight(w.y, a2, a3);
-          widen_weight(w.z, b0, b1);
-          widen_weight(w.w, b2, b3);
-          sts128(fb + r * 128 + (((2 * j) ^ (r & 7)) << 4), a0, a1, a2, a3);
-          sts128(fb + r * 128 + (((2 * j + 1) ^ (r & 7)) << 4), b0, b1, b2, b3);
-        }
-        fence_proxy_async_smem();
-        mbar_arrive(empty_pack(ps));
-        mbar_arrive(full_f8(fs));
+      for (int j = 0; j < kChunksPerKt; ++j) cur[j] = nxt[j];
+      // Issue the next k-tile's loads (possibly of the next tile) before waiting.
+      int ntile = tile, nkt = kt + 1;
+      if (nkt == nk) {
+        nkt = 0;
+        ntile += clusters;
       }
+      if (ntile < num_tiles)
+        load_kt(p.a_codes, a_block(p, ntile, rank, quarter), p.t_blocks, p.kchunks, nkt, lane, nxt);
+      const int s = g % kStages;
+      if (!wait_cluster(empty(s), ((g / kStages) & 1) ^ 1, abort)) break;
+      tc_fence_after();
+      uint32_t f8[32];
+#pragma unroll
+      for (int j = 0; j < kChunksPerKt; ++j) {
+        widen_act(cur[j].x, f8[8 * j + 0], f8[8 * j + 1]);
+        widen_act(cur[j].y, f8[8 * j + 2], f8[8 * j + 3]);
+        widen_act(cur[j].z, f8[8 * j + 4], f8[8 * j + 5]);
+        widen_act(cur[j].w, f8[8 * j + 6], f8[8 * j + 7]);
+      }
+      tmem_st_32cols(tmem + tm_lane + kACol0 + s * kAColsPerStage, f8);
+      tmem_st_wait();
+      tc_fence_before();
+      arrive_cluster(full_l + 8u * s);
+      ++g;
+      tile = ntile;
+      kt = nkt;
+    }
+  } else if (warp < kFirstEpi) {
+    // ---------------- B converters: packed codes -> E4M3 in shared memory ----------------
+    const int wb = warp - kFirstB;  // 32-row group of this CTA's half of B
+    const int r = wb * 32 + lane;   // row within the stage tile
+    const uint32_t full_l = leader_addr(full(0));
+    int g = 0, tile = cluster, kt = 0;
+    uint4 nxt[kChunksPerKt];
+    if (tile < num_tiles) load_kt(p.w_codes, b_block(p, tile, rank, wb), p.n_blocks, p.kchunks, 0, lane, nxt);
+    while (tile < num_tiles && !*abort) {
+      uint4 cur[kChunksPerKt];
+#pragma unroll
+      for (int j = 0; j < kChunksPerKt; ++j) cur[j] = nxt[j];
+      int ntile = tile, nkt = kt + 1;
+      if (nkt == nk) {
+        nkt = 0;
+        ntile += clusters;
+      }
+      if (ntile < num_tiles)
+        load_kt(p.w_codes, b_block(p, ntile, rank, wb), p.n_blocks, p.kchunks, nkt, lane, nxt);
+      const int s = g % kStages;
+      if (!wait_cluster(empty(s), ((g / kStages) & 1) ^ 1, abort)) break;
+      const uint32_t st = base + kOffB + s * kBStage + r * 128;
+#pragma unroll
+      for (int j = 0; j < kChunksPerKt; ++j) {
+        uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
+        widen_weight(cur[j].x, a0, a1);
+        widen_weight(cur[j].y, a2, a3);
+        widen_weight(cur[j].z, b0, b1);
+        widen_weight(cur[j].w, b2, b3);
+        sts128(st + (((2 * j) ^ (r & 7)) << 4), a0, a1, a2, a3);
+        sts128(st + (((2 * j + 1) ^ (r & 7)) << 4), b0, b1, b2, b3);
+      }
+      fence_proxy_async_smem();
+      arrive_cluster(full_l + 8u * s);
+      ++g;
+      tile = ntile;
+      kt = nkt;
     }
   } else {
     // ---------------- epilogue ----------------
-    const int quarter = warp & 3;  // TMEM lanes this warp may read
-    const int rl = quarter * 32 + lane;
+    const int quarter = warp & 3;              // TMEM lanes this warp may read
+    const int half = (warp - kFirstEpi) / 4;   // which 128 accumulator columns
     const int G = p.G;
+    const uint32_t acc_empty_l = leader_addr(acc_empty);
     int lt = 0;
-    for (int tile = blockIdx.x; tile < num_tiles && !*abort; tile += gridDim.x, ++lt) {
-      const int ab = lt & 1;
-      const int m0 = (tile / p.n_tiles) * BM;
-      const int n0 = (tile % p.n_tiles) * BN;
-      if (!mbar_wait(acc_full(ab), (lt >> 1) & 1, abort)) break;
+    for (int tile = cluster; tile < num_tiles && !*abort; tile += clusters, ++lt) {
+      const int m0 = (tile / p.n_tiles) * 2 * BM + static_cast<int>(rank) * BM;
+      const int n0 = (tile % p.n_tiles) * BN + half * (BN / 2);
+      if (!wait_cluster(acc_full, lt & 1, abort)) break;
       tc_fence_after();
-      const int t = m0 + rl;
+      const int t = m0 + quarter * 32 + lane;
       const bool row_ok = t < p.T;
       const float sa = row_ok ? __ldg(p.a_scale + t) : 0.f;
       const bool has_off = p.a_offset != nullptr && row_ok;
       const float* orow = has_off ? p.a_offset + static_cast<int64_t>(t) * G : p.a_scale;
       const float o0 = (has_off ? __ldg(orow) : 0.f) - 8.0f * sa;
-      const uint32_t acc_tm = tmem + ab * kAccCols + (static_cast<uint32_t>(quarter * 32) << 16);
+      const uint32_t acc_tm = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + half * (BN / 2);
       constexpr int CW = 16;  // accumulator columns per TMEM load
-      for (int c = 0; c < BN / CW; ++c) {
+      for (int c = 0; c < (BN / 2) / CW; ++c) {
         uint32_t acc[CW];
         tmem_ld_16cols(acc_tm + c * CW, acc);
         tmem_ld_wait();
@@ -399,58 +526,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       tc_fence_before();
-      mbar_arrive(acc_empty(ab));
+      arrive_cluster(acc_empty_l);
     }
   }
 
   // ---------------- teardown ----------------
-  if (*abort && warp == 0 && lane == 0) {
-    // Let TMA copies still in flight land before the CTA's shared memory goes away.
-    for (int g = issued - kPackStages < 0 ? 0 : issued - kPackStages; g < issued; ++g)
-      mbar_wait_teardown(full_pack(g % kPackStages), (g / kPackStages) & 1);
-  }
-  if (*abort && warp == 1 && lane == 0 && mma_tiles > 0) {
-    const int lt = mma_tiles - 1;
-    mbar_wait_teardown(acc_full(lt & 1), (lt >> 1) & 1);
+  if (*abort && warp == 0 && lane == 0 && rank == 0 && mma_tiles > 0) {
+    // Let the MMAs already issued finish before tensor memory is released.
+    wait_teardown(acc_full, (mma_tiles - 1) & 1);
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 1) {
+  cluster_sync();  // the pair's MMAs read both CTAs' memory: leave together
+  if (warp == 0) {
     tc_fence_after();
-    tmem_dealloc(tmem, kTmemCols);
+    tmem_dealloc2(tmem, kTmemCols);
   }
   if (threadIdx.x == 0 && *abort && p.status != nullptr) atomicExch(p.status, kErrTimeout);
-}
-
-using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn encode_fn() {
-  static EncodeTiledFn fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* ptr = nullptr;
-    cudaDriverEntryPointQueryResult q{};
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-            cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiledFn>(ptr);
-  });
-  return fn;
-}
-
-// 2-D map over a [rows][row_bytes] byte matrix, box = 64 bytes x box_rows.
-bool make_code_map(CUtensorMap* m, const void* ptr, int64_t rows, int64_t row_bytes, int box_rows) {
-  EncodeTiledFn fn = encode_fn();
-  if (fn == nullptr) return false;
-  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(row_bytes), static_cast<cuuint64_t>(rows)};
-  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(row_bytes)};
-  const cuuint32_t box[2] = {BK / 2, static_cast<cuuint32_t>(box_rows)};
-  const cuuint32_t estr[2] = {1, 1};
-  return fn(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(ptr), dims, strides, box, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 int num_sms() {
@@ -466,7 +558,7 @@ int num_sms() {
 }
 
 template <int OUT>
-int launch_gemm(const CUtensorMap& ma, const CUtensorMap& mb, const GemmParams& p, cudaStream_t s) {
+int launch_gemm(const GemmParams& p, cudaStream_t s) {
   auto kern = w4a4_gemm_kernel<OUT>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
@@ -475,10 +567,10 @@ int launch_gemm(const CUtensorMap& ma, const CUtensorMap& mb, const GemmParams& 
   });
   if (attr_err != cudaSuccess) return OFFQ_ERR_CUDA;
   const int sms = num_sms();
-  if (sms <= 0) return OFFQ_ERR_CUDA;
-  const int tiles = p.m_tiles * p.n_tiles;
-  const int grid = tiles < sms ? tiles : sms;
-  kern<<<grid, kThreads, kSmemBytes, s>>>(ma, mb, p);
+  if (sms < 2) return OFFQ_ERR_CUDA;
+  const int tiles = p.m_pairs * p.n_tiles;
+  const int clusters = tiles < sms / 2 ? tiles : sms / 2;
+  kern<<<2 * clusters, kThreads, kSmemBytes, s>>>(p);
   return launch_status();
 }
 
@@ -491,8 +583,7 @@ extern "C" int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, co
   const int ob = elem_bytes(out_dtype);
   if (ob == 0 || T < 0 || N < 1 || !is_pow2(g) || g < 32 || g > 8192) return OFFQ_ERR_INVALID_ARG;
   if (K <= 0 || K % g != 0 || K % 32 != 0 || ldo < N) return OFFQ_ERR_INVALID_ARG;
-  if (K > kMaxGemmK || T > 0x7FFFFFFF / 2 || N > 0x7FFFFFFF / 2) return OFFQ_ERR_UNSUPPORTED;
-  if (K / g > kMaxEpilogueG) return OFFQ_ERR_UNSUPPORTED;
+  if (K > kMaxGemmK || T > 0x3FFFFFFF || N > 0x3FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
   if (T == 0) return OFFQ_OK;
   if (a_codes == nullptr || a_scale == nullptr || w_codes == nullptr || w_scale == nullptr || w_offsum == nullptr ||
       out == nullptr)
@@ -502,10 +593,9 @@ extern "C" int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, co
       (a_offset != nullptr && !aligned(a_offset, 4)) || (acc_debug != nullptr && !aligned(acc_debug, 4)))
     return OFFQ_ERR_MISALIGNED;
 
-  CUtensorMap ma, mb;
-  if (!make_code_map(&ma, a_codes, T, K / 2, BM) || !make_code_map(&mb, w_codes, N, K / 2, BN))
-    return OFFQ_ERR_CUDA;
   GemmParams p{};
+  p.a_codes = a_codes;
+  p.w_codes = w_codes;
   p.a_scale = a_scale;
   p.a_offset = a_offset;
   p.w_scale = w_scale;
@@ -518,15 +608,17 @@ extern "C" int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, co
   p.N = static_cast<int>(N);
   p.K = static_cast<int>(K);
   p.G = static_cast<int>(K / g);
-  p.out_dtype = out_dtype;
-  p.m_tiles = static_cast<int>((T + BM - 1) / BM);
-  p.vec_ok = aligned(w_offsum, 16) && aligned(w_scale, 16) && (N % 4 == 0);
+  p.m_pairs = static_cast<int>((T + 2 * BM - 1) / (2 * BM));
   p.n_tiles = static_cast<int>((N + BN - 1) / BN);
+  p.t_blocks = static_cast<int>((T + 31) / 32);
+  p.n_blocks = static_cast<int>((N + 31) / 32);
+  p.kchunks = static_cast<int>(K / 32);
+  p.vec_ok = aligned(w_offsum, 16) && aligned(w_scale, 16) && (N % 4 == 0);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   switch (out_dtype) {
-    case OFFQ_F32: return launch_gemm<OFFQ_F32>(ma, mb, p, s);
-    case OFFQ_BF16: return launch_gemm<OFFQ_BF16>(ma, mb, p, s);
-    case OFFQ_F16: return launch_gemm<OFFQ_F16>(ma, mb, p, s);
+    case OFFQ_F32: return launch_gemm<OFFQ_F32>(p, s);
+    case OFFQ_BF16: return launch_gemm<OFFQ_BF16>(p, s);
+    case OFFQ_F16: return launch_gemm<OFFQ_F16>(p, s);
     default: return OFFQ_ERR_INVALID_ARG;
   }
 }

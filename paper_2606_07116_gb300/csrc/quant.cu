@@ -50,6 +50,7 @@ struct QuantArgs {
   float scale_mul;  // inv_sqrt_g / 7
   int tpr;          // threads per row (a power of two <= 32 or a multiple of 32)
   int rows_per_cta;
+  int tiled;        // codes in the 32-row tiled operand layout (else row-major)
 };
 
 template <int L>
@@ -193,8 +194,8 @@ __global__ void __launch_bounds__(Geo<L>::kMaxThreads) quantize_rows_kernel(cons
   const int R = a.rows_per_cta;
   const int K = a.K;
   float* buf = reinterpret_cast<float*>(smem);                                  // [R][K] fp32 (rotate)
-  uint8_t* cbuf = smem + (rotate ? static_cast<size_t>(R) * K * 4 : 0);         // [R][K/2] codes (rotate)
-  float* red = reinterpret_cast<float*>(cbuf + (rotate ? static_cast<size_t>(R) * (K / 2) : 0));
+  uint8_t* cbuf = smem + (rotate ? static_cast<size_t>(R) * K * 4 : 0);         // [R][K/2] codes
+  float* red = reinterpret_cast<float*>(cbuf + static_cast<size_t>(R) * (K / 2));
 
   const int tid = threadIdx.x;
   const int lrow = tid / a.tpr;
@@ -270,9 +271,9 @@ __global__ void __launch_bounds__(Geo<L>::kMaxThreads) quantize_rows_kernel(cons
 #pragma unroll
   for (int r = 0; r < E; r += 2) fma2(v[r], v[r + 1], inv, kMagic8);
 
-  if (rotate) {
-    if (active) {
-      uint8_t* crow = cbuf + static_cast<size_t>(lrow) * (K / 2) + static_cast<size_t>(b) * (g / 2);
+  uint8_t* crow = cbuf + static_cast<size_t>(lrow) * (K / 2) + static_cast<size_t>(b) * (g / 2);
+  if (active) {
+    if (rotate) {
 #pragma unroll
       for (int hi = 0; hi < (1 << P); ++hi) {
         const int e = ((t1 & ((1 << (3 - Q)) - 1)) << Q) | (hi << 3) | ((t1 >> (3 - Q)) << (3 + P));
@@ -286,24 +287,30 @@ __global__ void __launch_bounds__(Geo<L>::kMaxThreads) quantize_rows_kernel(cons
           crow[e / 2] = static_cast<uint8_t>(u0 | (u1 << 4));
         }
       }
+    } else {
+#pragma unroll
+      for (int i = 0; i < NC; ++i) {
+        uint32_t w = 0;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) w |= (__float_as_uint(v[8 * i + e]) & 0xFu) << (4 * e);
+        *reinterpret_cast<uint32_t*>(crow + 4 * t1 + 4 * TPB * i) = w;
+      }
     }
-    __syncthreads();
+  }
+  __syncthreads();
+  {
+    // Codes leave in 16-byte chunks, rows fastest so that neighbouring rows of
+    // the tiled layout (16 bytes apart) are written by neighbouring threads.
     const int64_t row0 = static_cast<int64_t>(blockIdx.x) * R;
     const int nrows = static_cast<int>(a.rows - row0 < R ? a.rows - row0 : R);
     const int cpr = K / 32;  // 16-byte chunks of codes per row
     for (int c = tid; c < nrows * cpr; c += blockDim.x) {
-      const int rr = c / cpr, cc = c - rr * cpr;
+      const int cc = c / nrows, rr = c - cc * nrows;
+      const int64_t t = row0 + rr;
       const uint4 w = *reinterpret_cast<const uint4*>(cbuf + static_cast<size_t>(rr) * (K / 2) + cc * 16);
-      *reinterpret_cast<uint4*>(a.codes + (row0 + rr) * (K / 2) + cc * 16) = w;
-    }
-  } else if (active) {
-    uint8_t* crow = a.codes + row * (K / 2) + static_cast<int64_t>(b) * (g / 2);
-#pragma unroll
-    for (int i = 0; i < NC; ++i) {
-      uint32_t w = 0;
-#pragma unroll
-      for (int e = 0; e < 8; ++e) w |= (__float_as_uint(v[8 * i + e]) & 0xFu) << (4 * e);
-      *reinterpret_cast<uint32_t*>(crow + 4 * t1 + 4 * TPB * i) = w;
+      uint8_t* dst = a.tiled ? a.codes + ((t >> 5) * cpr + cc) * 512 + (t & 31) * 16
+                             : a.codes + t * (K / 2) + cc * 16;
+      *reinterpret_cast<uint4*>(dst) = w;
     }
   }
 
@@ -325,7 +332,7 @@ int launch_quant(QuantArgs a, cudaStream_t stream) {
   }
   if (tpr > GG::kMaxThreads) return OFFQ_ERR_UNSUPPORTED;
   const bool rotate = (a.flags & OFFQ_ROTATE) != 0;
-  const size_t row_smem = rotate ? static_cast<size_t>(a.K) * 4 + a.K / 2 : 0;
+  const size_t row_smem = (rotate ? static_cast<size_t>(a.K) * 4 : 0) + a.K / 2;
   int R = std::max(1, std::min(GG::kMaxThreads, 256) / tpr);
   while (R > 1 && static_cast<size_t>(R) * row_smem > 64 * 1024) --R;
   a.tpr = tpr;
@@ -380,18 +387,26 @@ int check_row_shape(int64_t K, int32_t g) {
 }
 
 // Offline: activation-format codes (q + 8) -> weight format, in place, plus the
-// integer block row sums R[b][n]. One thread per (row, block).
-__global__ void weight_repack_kernel(uint8_t* __restrict__ codes, float* __restrict__ rowsum, int64_t N, int K,
-                                     int g) {
+// integer block row sums R[b][n]; the padding rows of the last 32-row tile are
+// zeroed. Codes are in the tiled operand layout. One thread per (row, block).
+__global__ void weight_repack_kernel(uint8_t* __restrict__ codes, float* __restrict__ rowsum, int64_t N,
+                                     int64_t N_pad, int K, int g) {
   const int G = K / g;
   const int64_t id = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (id >= N * G) return;
+  if (id >= N_pad * G) return;
   const int64_t n = id / G;
   const int b = static_cast<int>(id - n * G);
-  uint32_t* w = reinterpret_cast<uint32_t*>(codes + n * (K / 2) + static_cast<int64_t>(b) * (g / 2));
+  const int64_t cpr = K / 32;
+  uint8_t* tile_row = codes + (n >> 5) * cpr * 512 + (n & 31) * 16;
   int sum = 0;
   for (int i = 0; i < g / 8; ++i) {
-    const uint32_t u = w[i];
+    const int64_t bo = static_cast<int64_t>(b) * (g / 2) + 4 * i;  // byte of the row-major row
+    uint32_t* w = reinterpret_cast<uint32_t*>(tile_row + (bo >> 4) * 512 + (bo & 15));
+    if (n >= N) {
+      *w = 0u;
+      continue;
+    }
+    const uint32_t u = *w;
     uint32_t mag[8], neg[8];
 #pragma unroll
     for (int c = 0; c < 8; ++c) {
@@ -406,9 +421,9 @@ __global__ void weight_repack_kernel(uint8_t* __restrict__ codes, float* __restr
       const uint32_t byte = mag[2 * jj] | (neg[2 * jj] << 7) | (mag[2 * jj + 1] << 4) | (neg[(2 * jj + 7) & 7] << 3);
       out |= byte << (8 * jj);
     }
-    w[i] = out;
+    *w = out;
   }
-  rowsum[static_cast<int64_t>(b) * N + n] = static_cast<float>(sum);
+  if (n < N) rowsum[static_cast<int64_t>(b) * N + n] = static_cast<float>(sum);
 }
 
 }  // namespace
@@ -438,6 +453,7 @@ extern "C" int offq_quantize_act(const void* x, int x_dtype, int64_t T, int64_t 
   a.codes = codes;
   a.scale = scale;
   a.offset = offset;
+  a.tiled = 1;
   return run_quant(a, x_dtype, g, static_cast<cudaStream_t>(stream));
 }
 
@@ -467,6 +483,7 @@ extern "C" int offq_kv4_quantize(const void* kv, int dtype, int64_t T, int32_t H
   a.codes = codes;
   a.scale = scale;
   a.offset = offset;
+  a.tiled = 0;
   return run_quant(a, dtype, head_dim, static_cast<cudaStream_t>(stream));
 }
 
@@ -493,11 +510,23 @@ extern "C" int offq_prepare_weight(const void* w, int dtype, int64_t N, int64_t 
   a.codes = w_codes;
   a.scale = w_scale;
   a.offset = nullptr;
+  a.tiled = 1;
   int rc = run_quant(a, dtype, g, s);
   if (rc != OFFQ_OK) return rc;
-  const int64_t units = N * (K / g);
+  const int64_t n_pad = (N + 31) / 32 * 32;
+  const int64_t units = n_pad * (K / g);
   const int threads = 256;
   weight_repack_kernel<<<static_cast<unsigned>((units + threads - 1) / threads), threads, 0, s>>>(
-      w_codes, w_offsum, N, static_cast<int>(K), g);
+      w_codes, w_offsum, N, n_pad, static_cast<int>(K), g);
   return launch_status();
+}
+
+extern "C" int64_t offq_act_codes_bytes(int64_t T, int64_t K) {
+  if (T < 0 || K <= 0 || K % 32 != 0) return -1;
+  return (T + 31) / 32 * 32 * (K / 2);
+}
+
+extern "C" int64_t offq_weight_codes_bytes(int64_t N, int64_t K) {
+  if (N < 1 || K <= 0 || K % 32 != 0) return -1;
+  return (N + 31) / 32 * 32 * (K / 2);
 }

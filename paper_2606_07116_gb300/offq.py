@@ -6,7 +6,8 @@ current CUDA stream to the library, and raise :class:`OffqError` on a non-zero
 status. All computation happens in the library's kernels; torch supplies device
 memory and streams only. The helpers without the prefix (``quantize_act``,
 ``w4a4_linear``, ...) allocate the outputs with torch and call the same entry
-points.
+points. Activation and weight code buffers are [ceil(R/32)*32, K/2] uint8
+tensors holding the tiled operand layout of include/offq.h.
 """
 
 from __future__ import annotations
@@ -47,6 +48,8 @@ _SIGNATURES = {
     "offq_get_device_status": (_c_int, [_c_vp]),
     "offq_status_string": (ctypes.c_char_p, [_c_int]),
     "offq_abi_version": (_c_int, []),
+    "offq_act_codes_bytes": (_c_i64, [_c_i64, _c_i64]),
+    "offq_weight_codes_bytes": (_c_i64, [_c_i64, _c_i64]),
 }
 
 _lib = None
@@ -164,6 +167,19 @@ def offq_get_device_status(stream=None) -> int:
     return load_library().offq_get_device_status(_stream(stream))
 
 
+def offq_act_codes_bytes(T: int, K: int) -> int:
+    return load_library().offq_act_codes_bytes(T, K)
+
+
+def offq_weight_codes_bytes(N: int, K: int) -> int:
+    return load_library().offq_weight_codes_bytes(N, K)
+
+
+def padded_rows(R: int) -> int:
+    """Rows a tiled code buffer holds for R rows (a multiple of 32)."""
+    return (R + 31) // 32 * 32
+
+
 # ---------------------------------------------------------------------------
 # Allocating helpers (torch allocates; the entry points above compute).
 # ---------------------------------------------------------------------------
@@ -171,7 +187,7 @@ def offq_get_device_status(stream=None) -> int:
 def quantize_act(x: torch.Tensor, g: int, rotate: bool = True, offset: bool = True,
                  stream=None) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
     T, K = x.shape
-    codes = torch.empty((T, K // 2), dtype=torch.uint8, device=x.device)
+    codes = torch.empty((padded_rows(T), K // 2), dtype=torch.uint8, device=x.device)
     scale = torch.empty((T,), dtype=torch.float32, device=x.device)
     off = torch.empty((T, K // g), dtype=torch.float32, device=x.device)
     flags = (OFFQ_ROTATE if rotate else 0) | (OFFQ_OFFSET if offset else 0)
@@ -196,7 +212,7 @@ def prepare_weight(w: torch.Tensor, g: int, rotate: bool = True,
                    stream=None) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
     N, K = w.shape
     w = w.contiguous()
-    codes = torch.empty((N, K // 2), dtype=torch.uint8, device=w.device)
+    codes = torch.empty((padded_rows(N), K // 2), dtype=torch.uint8, device=w.device)
     scale = torch.empty((N,), dtype=torch.float32, device=w.device)
     rowsum = torch.empty((K // g, N), dtype=torch.float32, device=w.device)
     offq_prepare_weight(w, N, K, g, rotate, codes, scale, rowsum, stream)
@@ -207,9 +223,9 @@ def w4a4_linear(a_codes: torch.Tensor, a_scale: torch.Tensor, a_offset: Optional
                 w_codes: torch.Tensor, w_scale: torch.Tensor, w_offsum: torch.Tensor, g: int,
                 out_dtype: torch.dtype = torch.bfloat16, out: Optional[torch.Tensor] = None,
                 acc_debug: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
-    T = a_codes.shape[0]
+    T = a_scale.shape[0]
     K = a_codes.shape[1] * 2
-    N = w_codes.shape[0]
+    N = w_scale.shape[0]
     if out is None:
         out = torch.empty((T, N), dtype=out_dtype, device=a_codes.device)
     offq_w4a4_linear(a_codes, a_scale, a_offset, T, N, K, g, w_codes, w_scale, w_offsum, out, out.stride(0),

@@ -112,3 +112,17 @@ def max_rel_err_floored(y_gpu, y_ref):
     y_ref = np.asarray(y_ref, np.float64)
     floor = 1e-2 * np.sqrt(np.mean(y_ref ** 2)) + 1e-30
     return float(np.max(np.abs(y_gpu - y_ref) / np.maximum(np.abs(y_ref), floor)))
+
+
+def act_q(codes, T: int, K: int) -> np.ndarray:
+    """Integer codes [T, K] from a tiled activation-code buffer (decoded by the oracle)."""
+    import oracle as O
+    arr = codes.cpu().numpy() if hasattr(codes, "cpu") else np.asarray(codes)
+    return O.unpack_act_codes(O.untile_codes(arr, T, K))
+
+
+def weight_q(codes, N: int, K: int) -> np.ndarray:
+    """Integer codes [N, K] from a tiled weight-code buffer (decoded by the oracle)."""
+    import oracle as O
+    arr = codes.cpu().numpy() if hasattr(codes, "cpu") else np.asarray(codes)
+    return O.unpack_weight_codes(O.untile_codes(arr, N, K))

@@ -98,3 +98,14 @@ def test_kv_and_weight_argument_checks(lib):
     assert pw(A16, Q.OFFQ_F32, 8, 1000, 256, 1, A16, A16, A16, None) == Q.OFFQ_ERR_INVALID_ARG
     assert pw(A16, Q.OFFQ_F32, 8, 1024, 256, 1, A16, A16, None, None) == Q.OFFQ_ERR_INVALID_ARG
     assert pw(A8, Q.OFFQ_F32, 8, 1024, 256, 1, A16, A16, A16, None) == Q.OFFQ_ERR_MISALIGNED
+
+
+def test_code_buffer_sizes(lib):
+    assert Q.offq_act_codes_bytes(1, 4096) == 32 * 2048
+    assert Q.offq_act_codes_bytes(64, 4096) == 64 * 2048
+    assert Q.offq_act_codes_bytes(65, 64) == 96 * 32
+    assert Q.offq_act_codes_bytes(0, 64) == 0
+    assert Q.offq_act_codes_bytes(4, 48) == -1
+    assert Q.offq_weight_codes_bytes(11008, 4096) == 11008 * 2048
+    assert Q.offq_weight_codes_bytes(300, 1024) == 320 * 512
+    assert Q.offq_weight_codes_bytes(0, 1024) == -1

@@ -12,7 +12,7 @@ import oracle as O
 import workloads as W
 from paper_2606_07116_gb300 import build as B
 from paper_2606_07116_gb300 import offq as Q
-from parity import check_outputs, epilogue_terms, max_rel_err_floored
+from parity import act_q, check_outputs, epilogue_terms, max_rel_err_floored, weight_q
 
 pytestmark = pytest.mark.gpu
 
@@ -26,8 +26,8 @@ def _lib():
 
 
 def _run_gemm(a_codes, a_scale, a_off, w_codes, w_scale, rowsum, g, out_dt, ldo=None, T=None, N=None):
-    T = a_codes.shape[0] if T is None else T
-    N = w_codes.shape[0] if N is None else N
+    T = a_scale.shape[0] if T is None else T
+    N = w_scale.shape[0] if N is None else N
     ldo = N if ldo is None else ldo
     out = torch.full((T, ldo), float("nan"), dtype=OUT_DT[out_dt], device="cuda")
     acc = torch.zeros((T, N), dtype=torch.int32, device="cuda")
@@ -47,8 +47,8 @@ def _check_layer(T, K, N, g, out_dt, rotate=True, seed=0, ldo=None, rows=None, n
     w_codes, w_scale, rowsum = Q.prepare_weight(torch.from_numpy(w).cuda(), g, rotate=rotate)
     y, acc = _run_gemm(a_codes, a_scale, a_off, w_codes, w_scale, rowsum, g, out_dt, ldo=ldo)
     sel = np.arange(T) if rows is None else rows
-    qa = O.unpack_act_codes(a_codes.cpu().numpy()[sel])
-    qw = O.unpack_weight_codes(w_codes.cpu().numpy())
+    qa = act_q(a_codes, T, K)[sel]
+    qw = weight_q(w_codes, N, K)
     sa = a_scale.cpu().numpy().astype(np.float64)[sel]
     oa = a_off.cpu().numpy().astype(np.float64)[sel]
     sw = w_scale.cpu().numpy().astype(np.float64)
@@ -71,8 +71,8 @@ def test_toy_layer(out_dt):
     a_codes, a_scale, a_off = Q.quantize_act(torch.from_numpy(x).cuda(), 512)
     w_codes, w_scale, rowsum = Q.prepare_weight(torch.from_numpy(w).cuda(), 512)
     y, acc = _run_gemm(a_codes, a_scale, a_off, w_codes, w_scale, rowsum, 512, out_dt)
-    qa = O.unpack_act_codes(a_codes.cpu().numpy())
-    qw = O.unpack_weight_codes(w_codes.cpu().numpy())
+    qa = act_q(a_codes, T, K)
+    qw = weight_q(w_codes, 512, K)
     np.testing.assert_array_equal(acc, O.int_gemm(qa + 8, qw))
     sa, oa = a_scale.cpu().numpy().astype(np.float64), a_off.cpu().numpy().astype(np.float64)
     sw, R = w_scale.cpu().numpy().astype(np.float64), rowsum.cpu().numpy().astype(np.float64)
@@ -94,8 +94,8 @@ def test_oracle_codes_through_gemm():
     a = O.quantize_act(xa, g)
     wp = O.prepare_weight(w.astype(np.float64), g)
     dev = lambda arr, dt: torch.from_numpy(np.ascontiguousarray(arr)).to(dt).cuda()
-    y, acc = _run_gemm(dev(a["codes"], torch.uint8), dev(a["scale"], torch.float32),
-                       dev(a["offset"], torch.float32), dev(wp["codes"], torch.uint8),
+    y, acc = _run_gemm(dev(O.tile_codes(a["codes"]), torch.uint8), dev(a["scale"], torch.float32),
+                       dev(a["offset"], torch.float32), dev(O.tile_codes(wp["codes"]), torch.uint8),
                        dev(wp["scale"], torch.float32), dev(wp["offsum"], torch.float32), g, "f32")
     np.testing.assert_array_equal(acc, O.int_gemm(a["q"] + 8, wp["q"]))
     sa = a["scale"].astype(np.float32).astype(np.float64)
@@ -132,8 +132,8 @@ def test_null_offset_means_zero():
     a_codes, a_scale, _ = Q.quantize_act(torch.from_numpy(x).cuda(), g, rotate=True, offset=False)
     w_codes, w_scale, rowsum = Q.prepare_weight(torch.from_numpy(W.weights(N, K, seed=42)).cuda(), g)
     y, acc = _run_gemm(a_codes, a_scale, None, w_codes, w_scale, rowsum, g, "f32")
-    qa = O.unpack_act_codes(a_codes.cpu().numpy())
-    qw = O.unpack_weight_codes(w_codes.cpu().numpy())
+    qa = act_q(a_codes, T, K)
+    qw = weight_q(w_codes, N, K)
     sa, sw = a_scale.cpu().numpy().astype(np.float64), w_scale.cpu().numpy().astype(np.float64)
     R = rowsum.cpu().numpy().astype(np.float64)
     zero = np.zeros((T, 1))
@@ -152,8 +152,9 @@ def test_accumulator_exact_at_largest_k():
     sa = np.ones(T, dtype=np.float32)
     sw = np.ones(N, dtype=np.float32)
     R = qw.reshape(N, K // g, g).sum(axis=2).T.astype(np.float32)
-    y, acc = _run_gemm(dev(O.pack_act_codes(qa), torch.uint8), dev(sa, torch.float32), None,
-                       dev(O.pack_weight_codes(qw), torch.uint8), dev(sw, torch.float32), dev(R, torch.float32),
+    y, acc = _run_gemm(dev(O.tile_codes(O.pack_act_codes(qa)), torch.uint8), dev(sa, torch.float32), None,
+                       dev(O.tile_codes(O.pack_weight_codes(qw)), torch.uint8), dev(sw, torch.float32),
+                       dev(R, torch.float32),
                        g, "f32")
     np.testing.assert_array_equal(acc, O.int_gemm(qa + 8, qw))
     np.testing.assert_array_equal(y, O.int_gemm(qa, qw).astype(np.float64))

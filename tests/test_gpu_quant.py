@@ -11,7 +11,7 @@ import oracle as O
 import workloads as W
 from paper_2606_07116_gb300 import build as B
 from paper_2606_07116_gb300 import offq as Q
-from parity import check_codes, check_offsets, check_scales
+from parity import act_q, check_codes, check_offsets, check_scales, weight_q
 
 pytestmark = pytest.mark.gpu
 
@@ -43,7 +43,7 @@ def _quant_and_check(x_host: torch.Tensor, g: int, rotate: bool, offset: bool, r
     x64 = x_host.to(torch.float64).numpy()
     sel = np.arange(T) if rows is None else rows
     ref = O.quantize_act(x64[sel], g, rotate=rotate, offset=offset)
-    q_gpu = O.unpack_act_codes(codes.cpu().numpy()[sel])
+    q_gpu = act_q(codes, T, K)[sel]
     nmis = check_codes(q_gpu, ref["q"], ref["residual"], ref["scale"])
     check_scales(scale.cpu().numpy()[sel], ref["scale"], x64[sel], g, rotate)
     o = off.cpu().numpy()[sel]
@@ -110,7 +110,7 @@ def test_quantize_degenerate_rows():
     xh = _host(x, "f32")
     codes, scale, off = Q.quantize_act(xh.cuda(), g)
     torch.cuda.synchronize()
-    q = O.unpack_act_codes(codes.cpu().numpy())
+    q = act_q(codes, 6, g * G)
     assert np.all(q[0] == 0) and scale[0].item() == 0.0 and np.all(off[0].cpu().numpy() == 0.0)
     assert np.all(q[1] == 0) and scale[1].item() == 0.0
     np.testing.assert_allclose(off[1].cpu().numpy(), [123.0 / math.sqrt(g), -7.5 / math.sqrt(g)], rtol=3e-7)
@@ -127,7 +127,7 @@ def test_quantize_exact_ties_round_half_even():
     x = np.tile(row, (5, 2))
     codes, scale, _ = Q.quantize_act(torch.from_numpy(x).cuda(), 32, rotate=False, offset=False)
     torch.cuda.synchronize()
-    q = O.unpack_act_codes(codes.cpu().numpy())
+    q = act_q(codes, x.shape[0], x.shape[1])
     ref = O.quantize_act(x.astype(np.float64), 32, rotate=False, offset=False)
     np.testing.assert_array_equal(q, ref["q"])
     np.testing.assert_array_equal(scale.cpu().numpy(), 1.0)
@@ -190,7 +190,11 @@ def test_prepare_weight(N, K, g, rotate):
     codes, scale, rowsum = Q.prepare_weight(wh.cuda(), g, rotate=rotate)
     torch.cuda.synchronize()
     ref = O.prepare_weight(w.astype(np.float64), g, rotate=rotate)
-    qg = O.unpack_weight_codes(codes.cpu().numpy())
+    qg = weight_q(codes, N, K)
+    # Padding rows of the last 32-row tile are zero bytes.
+    full = codes.cpu().numpy()
+    tail = O.untile_codes(full, full.shape[0], K)[N:]
+    assert np.all(tail == 0)
     # Reuse the activation-path checks: weights are rows quantized without offset.
     ra = O.quantize_act(w.astype(np.float64), g, rotate=rotate, offset=False)
     check_codes(qg, ref["q"], ra["residual"], ra["scale"], what="weight codes")

@@ -230,6 +230,24 @@ def test_pack_roundtrip_all_codes():
         O.pack_weight_codes(np.array([[-8, 0, 0, 0, 0, 0, 0, 0]]))
 
 
+def test_tiled_layout_positions():
+    """Hand-worked positions of the tiled operand layout (R = 33 rows, K = 64 codes)."""
+    R, K = 33, 64
+    p = np.zeros((R, K // 2), dtype=np.uint8)
+    p[0, 0] = 1      # row 0, byte 0   -> tile (0, 0), row 0      -> 0
+    p[1, 3] = 2      # row 1, byte 3   -> tile (0, 0), row 1      -> 16 + 3 = 19
+    p[2, 17] = 3     # row 2, byte 17  -> tile (0, 1), row 2      -> 512 + 32 + 1 = 545
+    p[31, 31] = 4    # row 31, byte 31 -> tile (0, 1), row 31     -> 512 + 496 + 15 = 1023
+    p[32, 16] = 5    # row 32, byte 16 -> tile (1, 1), row 0      -> 3 * 512 = 1536
+    t = O.tile_codes(p)
+    assert t.size == 64 * 32                      # rows padded to 64
+    expect = {0: 1, 19: 2, 545: 3, 1023: 4, 1536: 5}
+    for pos, val in expect.items():
+        assert t[pos] == val
+    assert np.count_nonzero(t) == len(expect)
+    np.testing.assert_array_equal(O.untile_codes(t, R, K), p)
+
+
 # --------------------------------------------------------------------------
 # Weights, GEMM and epilogue.
 # --------------------------------------------------------------------------
