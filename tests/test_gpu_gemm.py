@@ -94,8 +94,8 @@ def test_oracle_codes_through_gemm():
     a = O.quantize_act(xa, g)
     wp = O.prepare_weight(w.astype(np.float64), g)
     dev = lambda arr, dt: torch.from_numpy(np.ascontiguousarray(arr)).to(dt).cuda()
-    y, acc = _run_gemm(dev(O.tile_codes(a["codes"]), torch.uint8), dev(a["scale"], torch.float32),
-                       dev(a["offset"], torch.float32), dev(O.tile_codes(wp["codes"]), torch.uint8),
+    y, acc = _run_gemm(dev(O.tile_codes(a["codes"]).reshape(-1, K // 2), torch.uint8), dev(a["scale"], torch.float32),
+                       dev(a["offset"], torch.float32), dev(O.tile_codes(wp["codes"]).reshape(-1, K // 2), torch.uint8),
                        dev(wp["scale"], torch.float32), dev(wp["offsum"], torch.float32), g, "f32")
     np.testing.assert_array_equal(acc, O.int_gemm(a["q"] + 8, wp["q"]))
     sa = a["scale"].astype(np.float32).astype(np.float64)
@@ -152,8 +152,9 @@ def test_accumulator_exact_at_largest_k():
     sa = np.ones(T, dtype=np.float32)
     sw = np.ones(N, dtype=np.float32)
     R = qw.reshape(N, K // g, g).sum(axis=2).T.astype(np.float32)
-    y, acc = _run_gemm(dev(O.tile_codes(O.pack_act_codes(qa)), torch.uint8), dev(sa, torch.float32), None,
-                       dev(O.tile_codes(O.pack_weight_codes(qw)), torch.uint8), dev(sw, torch.float32),
+    y, acc = _run_gemm(dev(O.tile_codes(O.pack_act_codes(qa)).reshape(-1, K // 2), torch.uint8),
+                       dev(sa, torch.float32), None,
+                       dev(O.tile_codes(O.pack_weight_codes(qw)).reshape(-1, K // 2), torch.uint8), dev(sw, torch.float32),
                        dev(R, torch.float32),
                        g, "f32")
     np.testing.assert_array_equal(acc, O.int_gemm(qa + 8, qw))
