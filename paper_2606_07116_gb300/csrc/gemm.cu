@@ -58,8 +58,9 @@ constexpr int kStages = 4;
 constexpr int kAWarps = 4, kBWarps = 4, kEpiWarps = 8;
 constexpr int kFirstA = 1, kFirstB = kFirstA + kAWarps, kFirstEpi = kFirstB + kBWarps;
 constexpr int kThreads = (kFirstEpi + kEpiWarps) * 32;
-constexpr int kConvThreadsPerCta = (kAWarps + kBWarps) * 32;
-constexpr int kEpiThreadsPerCta = kEpiWarps * 32;
+constexpr int kConvWarpsPerCta = kAWarps + kBWarps;  // one barrier arrival per warp
+constexpr int kPrefetch = 3;                         // k-tiles of loads in flight per converter thread
+constexpr int kMaxStageG = 64;                       // offset blocks staged in shared memory
 constexpr int kAccCols = BN;       // fp32 accumulator columns (TMEM lanes = rows)
 constexpr int kACol0 = kAccCols;   // A operand stages live in TMEM after the accumulator
 constexpr int kAColsPerStage = BK / 4;  // 4 E4M3 values per 32-bit column
@@ -68,10 +69,18 @@ static_assert(kACol0 + kStages * kAColsPerStage <= kTmemCols, "TMEM budget");
 
 constexpr int kBStage = BNH * BK;  // 16 KB of E4M3 per stage
 constexpr int kOffB = 0;
-constexpr int kOffBars = kOffB + kStages * kBStage;
+// Epilogue constants of one tile: row sums R[b][256 columns], channel scales,
+// and per row o[t][b] - 8 s_a[t] (odd row pitch: conflict-free per-lane reads).
+constexpr int kStageGp = kMaxStageG + 1;
+constexpr int kOffR = kOffB + kStages * kBStage;
+constexpr int kOffW = kOffR + kMaxStageG * BN * 4;
+constexpr int kOffO = kOffW + BN * 4;
+constexpr int kOffSa = kOffO + BM * kStageGp * 4;
+constexpr int kOffBars = kOffSa + BM * 4;
 constexpr int kNumBars = 2 * kStages + 2;
 constexpr int kOffMisc = kOffBars + kNumBars * 8;
 constexpr int kSmemBytes = kOffMisc + 64 + 1024;  // + slack to align the base to 1024
+static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 
 constexpr uint32_t kIdesc = idesc_e4m3_f32(2 * BM, BN);  // pair MMA: M = 256, N = 256
 
@@ -201,6 +210,11 @@ __device__ __forceinline__ void tmem_st_32cols(uint32_t taddr, const uint32_t (&
       : "memory");
 }
 
+// Named barrier among the epilogue warps only.
+__device__ __forceinline__ void epi_sync() {
+  asm volatile("bar.sync 1, %0;" ::"r"(kEpiWarps * 32) : "memory");
+}
+
 __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
 __device__ __forceinline__ uint4 ldg_stream(const uint8_t* p) {
@@ -319,11 +333,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(full(s), 2 * kConvThreadsPerCta);
+      mbar_init(full(s), 2 * kConvWarpsPerCta);
       mbar_init(empty(s), 1);
     }
     mbar_init(acc_full, 1);
-    mbar_init(acc_empty, 2 * kEpiThreadsPerCta);
+    mbar_init(acc_empty, 2 * kEpiWarps);
     *abort = 0;
     mbar_fence_init();
   }
@@ -365,146 +379,193 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
         if (!ok) break;
       }
     }
-  } else if (warp < kFirstB) {
-    // ---------------- A converters: packed codes -> E4M3 in TMEM ----------------
-    const int quarter = warp & 3;
-    const uint32_t tm_lane = static_cast<uint32_t>(quarter * 32) << 16;
-    const uint32_t full_l = leader_addr(full(0));
-    int g = 0, tile = cluster, kt = 0;
-    uint4 nxt[kChunksPerKt];
-    if (tile < num_tiles) load_kt(p.a_codes, a_block(p, tile, rank, quarter), p.t_blocks, p.kchunks, 0, lane, nxt);
-    while (tile < num_tiles && !*abort) {
-      uint4 cur[kChunksPerKt];
-#pragma unroll
-      for (int j = 0; j < kChunksPerKt; ++j) cur[j] = nxt[j];
-      // Issue the next k-tile's loads (possibly of the next tile) before waiting.
-      int ntile = tile, nkt = kt + 1;
-      if (nkt == nk) {
-        nkt = 0;
-        ntile += clusters;
-      }
-      if (ntile < num_tiles)
-        load_kt(p.a_codes, a_block(p, ntile, rank, quarter), p.t_blocks, p.kchunks, nkt, lane, nxt);
-      const int s = g % kStages;
-      if (!wait_cluster(empty(s), ((g / kStages) & 1) ^ 1, abort)) break;
-      tc_fence_after();
-      uint32_t f8[32];
-#pragma unroll
-      for (int j = 0; j < kChunksPerKt; ++j) {
-        widen_act(cur[j].x, f8[8 * j + 0], f8[8 * j + 1]);
-        widen_act(cur[j].y, f8[8 * j + 2], f8[8 * j + 3]);
-        widen_act(cur[j].z, f8[8 * j + 4], f8[8 * j + 5]);
-        widen_act(cur[j].w, f8[8 * j + 6], f8[8 * j + 7]);
-      }
-      tmem_st_32cols(tmem + tm_lane + kACol0 + s * kAColsPerStage, f8);
-      tmem_st_wait();
-      tc_fence_before();
-      arrive_cluster(full_l + 8u * s);
-      ++g;
-      tile = ntile;
-      kt = nkt;
-    }
   } else if (warp < kFirstEpi) {
-    // ---------------- B converters: packed codes -> E4M3 in shared memory ----------------
-    const int wb = warp - kFirstB;  // 32-row group of this CTA's half of B
-    const int r = wb * 32 + lane;   // row within the stage tile
+    // ---------------- converters: packed codes -> E4M3 operands ----------------
+    // A warps write 32 TMEM lanes (their quarter); B warps write 32 rows of the
+    // shared-memory stage. Each thread keeps kPrefetch k-tiles of loads in
+    // flight in a register ring.
+    const bool is_a = warp < kFirstB;
+    const int quarter = warp & 3;
+    const int wb = warp - kFirstB;
     const uint32_t full_l = leader_addr(full(0));
-    int g = 0, tile = cluster, kt = 0;
-    uint4 nxt[kChunksPerKt];
-    if (tile < num_tiles) load_kt(p.w_codes, b_block(p, tile, rank, wb), p.n_blocks, p.kchunks, 0, lane, nxt);
-    while (tile < num_tiles && !*abort) {
-      uint4 cur[kChunksPerKt];
-#pragma unroll
-      for (int j = 0; j < kChunksPerKt; ++j) cur[j] = nxt[j];
-      int ntile = tile, nkt = kt + 1;
-      if (nkt == nk) {
-        nkt = 0;
-        ntile += clusters;
+    const uint8_t* codes = is_a ? p.a_codes : p.w_codes;
+    const int rb_count = is_a ? p.t_blocks : p.n_blocks;
+    auto block_of = [&](int tile) { return is_a ? a_block(p, tile, rank, quarter) : b_block(p, tile, rank, wb); };
+    uint4 ring[kPrefetch][kChunksPerKt];
+    int ld_tile = cluster, ld_kt = 0;  // next k-tile to load
+    auto advance = [&](int& tile, int& kt) {
+      if (++kt == nk) {
+        kt = 0;
+        tile += clusters;
       }
-      if (ntile < num_tiles)
-        load_kt(p.w_codes, b_block(p, ntile, rank, wb), p.n_blocks, p.kchunks, nkt, lane, nxt);
-      const int s = g % kStages;
-      if (!wait_cluster(empty(s), ((g / kStages) & 1) ^ 1, abort)) break;
-      const uint32_t st = base + kOffB + s * kBStage + r * 128;
+    };
 #pragma unroll
-      for (int j = 0; j < kChunksPerKt; ++j) {
-        uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
-        widen_weight(cur[j].x, a0, a1);
-        widen_weight(cur[j].y, a2, a3);
-        widen_weight(cur[j].z, b0, b1);
-        widen_weight(cur[j].w, b2, b3);
-        sts128(st + (((2 * j) ^ (r & 7)) << 4), a0, a1, a2, a3);
-        sts128(st + (((2 * j + 1) ^ (r & 7)) << 4), b0, b1, b2, b3);
+    for (int i = 0; i < kPrefetch; ++i) {
+      if (ld_tile < num_tiles) load_kt(codes, block_of(ld_tile), rb_count, p.kchunks, ld_kt, lane, ring[i]);
+      advance(ld_tile, ld_kt);
+    }
+    int tile = cluster, kt = 0, g = 0;
+    bool run = tile < num_tiles;
+    while (run) {
+#pragma unroll
+      for (int slot = 0; slot < kPrefetch; ++slot) {
+        if (!run) break;
+        const int s = g % kStages;
+        // Warp-uniform outcome, so the __syncwarp below is reached by all lanes.
+        if (!__all_sync(0xFFFFFFFFu, wait_cluster(empty(s), ((g / kStages) & 1) ^ 1, abort))) {
+          run = false;
+          break;
+        }
+        if (is_a) {
+          tc_fence_after();
+          uint32_t f8[32];
+#pragma unroll
+          for (int j = 0; j < kChunksPerKt; ++j) {
+            widen_act(ring[slot][j].x, f8[8 * j + 0], f8[8 * j + 1]);
+            widen_act(ring[slot][j].y, f8[8 * j + 2], f8[8 * j + 3]);
+            widen_act(ring[slot][j].z, f8[8 * j + 4], f8[8 * j + 5]);
+            widen_act(ring[slot][j].w, f8[8 * j + 6], f8[8 * j + 7]);
+          }
+          tmem_st_32cols(tmem + (static_cast<uint32_t>(quarter * 32) << 16) + kACol0 + s * kAColsPerStage, f8);
+          tmem_st_wait();
+          tc_fence_before();
+        } else {
+          const int r = wb * 32 + lane;
+          const uint32_t st = base + kOffB + s * kBStage + r * 128;
+#pragma unroll
+          for (int j = 0; j < kChunksPerKt; ++j) {
+            uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
+            widen_weight(ring[slot][j].x, a0, a1);
+            widen_weight(ring[slot][j].y, a2, a3);
+            widen_weight(ring[slot][j].z, b0, b1);
+            widen_weight(ring[slot][j].w, b2, b3);
+            sts128(st + (((2 * j) ^ (r & 7)) << 4), a0, a1, a2, a3);
+            sts128(st + (((2 * j + 1) ^ (r & 7)) << 4), b0, b1, b2, b3);
+          }
+          fence_proxy_async_smem();
+        }
+        __syncwarp();
+        if (lane == 0) arrive_cluster(full_l + 8u * s);
+        // Refill this slot kPrefetch k-tiles ahead.
+        if (ld_tile < num_tiles) load_kt(codes, block_of(ld_tile), rb_count, p.kchunks, ld_kt, lane, ring[slot]);
+        advance(ld_tile, ld_kt);
+        advance(tile, kt);
+        ++g;
+        run = __all_sync(0xFFFFFFFFu, tile < num_tiles && !*abort);
       }
-      fence_proxy_async_smem();
-      arrive_cluster(full_l + 8u * s);
-      ++g;
-      tile = ntile;
-      kt = nkt;
     }
   } else {
     // ---------------- epilogue ----------------
     const int quarter = warp & 3;              // TMEM lanes this warp may read
     const int half = (warp - kFirstEpi) / 4;   // which 128 accumulator columns
+    const int et = threadIdx.x - kFirstEpi * 32;
     const int G = p.G;
+    const bool staged = G <= kMaxStageG;
+    float* Rs = reinterpret_cast<float*>(smem + kOffR);
+    float* Ws = reinterpret_cast<float*>(smem + kOffW);
+    float* Os = reinterpret_cast<float*>(smem + kOffO);
+    float* Sa = reinterpret_cast<float*>(smem + kOffSa);
     const uint32_t acc_empty_l = leader_addr(acc_empty);
+    // Loop exit decided only from a flag the epilogue warps write before their
+    // own barrier, so all eight warps leave together (bar.sync has no timeout).
+    volatile int* epi_stop = reinterpret_cast<volatile int*>(smem + kOffMisc + 32);
+    if (et == 0) *epi_stop = 0;
+    epi_sync();
     int lt = 0;
-    for (int tile = cluster; tile < num_tiles && !*abort; tile += clusters, ++lt) {
+    for (int tile = cluster; tile < num_tiles; tile += clusters, ++lt) {
       const int m0 = (tile / p.n_tiles) * 2 * BM + static_cast<int>(rank) * BM;
-      const int n0 = (tile % p.n_tiles) * BN + half * (BN / 2);
-      if (!wait_cluster(acc_full, lt & 1, abort)) break;
+      const int nt0 = (tile % p.n_tiles) * BN;
+      // Stage this tile's constants while the main loop runs.
+      if (staged) {
+        for (int i = et; i < G * BN; i += kEpiWarps * 32) {
+          const int b = i / BN, j = i - b * BN, n = nt0 + j;
+          Rs[i] = n < p.N ? __ldg(p.rowsum + static_cast<int64_t>(b) * p.N + n) : 0.f;
+        }
+        for (int i = et; i < BN; i += kEpiWarps * 32) Ws[i] = nt0 + i < p.N ? __ldg(p.w_scale + nt0 + i) : 0.f;
+        for (int i = et; i < BM; i += kEpiWarps * 32) Sa[i] = m0 + i < p.T ? __ldg(p.a_scale + m0 + i) : 0.f;
+        for (int i = et; i < BM * G; i += kEpiWarps * 32) {
+          const int r = i / G, b = i - r * G, t = m0 + r;
+          float v = 0.f;
+          if (t < p.T) {
+            const float o = p.a_offset != nullptr ? __ldg(p.a_offset + static_cast<int64_t>(t) * G + b) : 0.f;
+            v = o - 8.0f * __ldg(p.a_scale + t);
+          }
+          Os[r * kStageGp + b] = v;
+        }
+      }
+      epi_sync();
+      const bool ok = __all_sync(0xFFFFFFFFu, wait_cluster(acc_full, lt & 1, abort));
+      if (!ok && lane == 0) *epi_stop = 1;
       tc_fence_after();
-      const int t = m0 + quarter * 32 + lane;
+      const int rl = quarter * 32 + lane;
+      const int t = m0 + rl;
       const bool row_ok = t < p.T;
-      const float sa = row_ok ? __ldg(p.a_scale + t) : 0.f;
-      const bool has_off = p.a_offset != nullptr && row_ok;
-      const float* orow = has_off ? p.a_offset + static_cast<int64_t>(t) * G : p.a_scale;
-      const float o0 = (has_off ? __ldg(orow) : 0.f) - 8.0f * sa;
+      const int n0 = nt0 + half * (BN / 2);
       const uint32_t acc_tm = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + half * (BN / 2);
       constexpr int CW = 16;  // accumulator columns per TMEM load
-      for (int c = 0; c < (BN / 2) / CW; ++c) {
-        uint32_t acc[CW];
-        tmem_ld_16cols(acc_tm + c * CW, acc);
-        tmem_ld_wait();
-        const int nb = n0 + c * CW;
-        if (!row_ok || nb >= p.N) continue;
-        const int nvalid = p.N - nb < CW ? p.N - nb : CW;
-        float y[CW];
-        if (nvalid == CW && p.vec_ok) {
-          const float4* r4 = reinterpret_cast<const float4*>(p.rowsum + nb);
-#pragma unroll
-          for (int q4 = 0; q4 < CW / 4; ++q4) {
-            const float4 rv = __ldg(r4 + q4);
-            y[4 * q4] = o0 * rv.x; y[4 * q4 + 1] = o0 * rv.y; y[4 * q4 + 2] = o0 * rv.z; y[4 * q4 + 3] = o0 * rv.w;
-          }
-          for (int b = 1; b < G; ++b) {
-            const float ob = (has_off ? __ldg(orow + b) : 0.f) - 8.0f * sa;
-            const float4* rb4 = reinterpret_cast<const float4*>(p.rowsum + static_cast<int64_t>(b) * p.N + nb);
+      if (!ok) {
+        // Aborted: nothing to drain.
+      } else if (staged) {
+        const float sa = Sa[rl];
+        for (int c = 0; c < (BN / 2) / CW; ++c) {
+          uint32_t acc[CW];
+          tmem_ld_16cols(acc_tm + c * CW, acc);
+          tmem_ld_wait();
+          const int nb = n0 + c * CW;
+          const int jc = half * (BN / 2) + c * CW;  // column within the staged tile
+          if (!row_ok || nb >= p.N) continue;
+          const int nvalid = p.N - nb < CW ? p.N - nb : CW;
+          float y[CW];
+          {
+            const float ob = Os[rl * kStageGp];
+            const float4* r4 = reinterpret_cast<const float4*>(Rs + jc);
 #pragma unroll
             for (int q4 = 0; q4 < CW / 4; ++q4) {
-              const float4 rv = __ldg(rb4 + q4);
+              const float4 rv = r4[q4];
+              y[4 * q4] = ob * rv.x; y[4 * q4 + 1] = ob * rv.y; y[4 * q4 + 2] = ob * rv.z; y[4 * q4 + 3] = ob * rv.w;
+            }
+          }
+          for (int b = 1; b < G; ++b) {
+            const float ob = Os[rl * kStageGp + b];
+            const float4* r4 = reinterpret_cast<const float4*>(Rs + b * BN + jc);
+#pragma unroll
+            for (int q4 = 0; q4 < CW / 4; ++q4) {
+              const float4 rv = r4[q4];
               y[4 * q4] = fmaf(ob, rv.x, y[4 * q4]);
               y[4 * q4 + 1] = fmaf(ob, rv.y, y[4 * q4 + 1]);
               y[4 * q4 + 2] = fmaf(ob, rv.z, y[4 * q4 + 2]);
               y[4 * q4 + 3] = fmaf(ob, rv.w, y[4 * q4 + 3]);
             }
           }
-          const float4* w4 = reinterpret_cast<const float4*>(p.w_scale + nb);
 #pragma unroll
-          for (int q4 = 0; q4 < CW / 4; ++q4) {
-            const float4 wv = __ldg(w4 + q4);
-            const float sw4[4] = {wv.x, wv.y, wv.z, wv.w};
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const int jj = 4 * q4 + e;
-              const float accf = __uint_as_float(acc[jj]) * 262144.0f;  // exact: * 2^18
-              y[jj] = sw4[e] * fmaf(sa, accf, y[jj]);
-            }
+          for (int jj = 0; jj < CW; ++jj) {
+            const float accf = __uint_as_float(acc[jj]) * 262144.0f;  // exact: * 2^18
+            y[jj] = Ws[jc + jj] * fmaf(sa, accf, y[jj]);
           }
-        } else {
+          store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, y, nvalid);
+          if (p.acc_debug != nullptr) {
+            int32_t* d = p.acc_debug + static_cast<int64_t>(t) * p.N + nb;
 #pragma unroll
-          for (int jj = 0; jj < CW; ++jj) y[jj] = jj < nvalid ? o0 * __ldg(p.rowsum + nb + jj) : 0.f;
-          for (int b = 1; b < G; ++b) {
+            for (int jj = 0; jj < CW; ++jj)
+              if (jj < nvalid) d[jj] = __float2int_rn(__uint_as_float(acc[jj]) * 262144.0f);
+          }
+        }
+      } else {
+        // More offset blocks than the staging area holds: read the constants directly.
+        const float sa = row_ok ? __ldg(p.a_scale + t) : 0.f;
+        const bool has_off = p.a_offset != nullptr && row_ok;
+        const float* orow = has_off ? p.a_offset + static_cast<int64_t>(t) * G : p.a_scale;
+        for (int c = 0; c < (BN / 2) / CW; ++c) {
+          uint32_t acc[CW];
+          tmem_ld_16cols(acc_tm + c * CW, acc);
+          tmem_ld_wait();
+          const int nb = n0 + c * CW;
+          if (!row_ok || nb >= p.N) continue;
+          const int nvalid = p.N - nb < CW ? p.N - nb : CW;
+          float y[CW];
+#pragma unroll
+          for (int jj = 0; jj < CW; ++jj) y[jj] = 0.f;
+          for (int b = 0; b < G; ++b) {
             const float ob = (has_off ? __ldg(orow + b) : 0.f) - 8.0f * sa;
             const float* rb = p.rowsum + static_cast<int64_t>(b) * p.N + nb;
 #pragma unroll
@@ -516,17 +577,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
             const float accf = __uint_as_float(acc[jj]) * 262144.0f;
             y[jj] = jj < nvalid ? __ldg(p.w_scale + nb + jj) * fmaf(sa, accf, y[jj]) : 0.f;
           }
-        }
-        store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, y, nvalid);
-        if (p.acc_debug != nullptr) {
-          int32_t* d = p.acc_debug + static_cast<int64_t>(t) * p.N + nb;
+          store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, y, nvalid);
+          if (p.acc_debug != nullptr) {
+            int32_t* d = p.acc_debug + static_cast<int64_t>(t) * p.N + nb;
 #pragma unroll
-          for (int jj = 0; jj < CW; ++jj)
-            if (jj < nvalid) d[jj] = __float2int_rn(__uint_as_float(acc[jj]) * 262144.0f);
+            for (int jj = 0; jj < CW; ++jj)
+              if (jj < nvalid) d[jj] = __float2int_rn(__uint_as_float(acc[jj]) * 262144.0f);
+          }
         }
       }
       tc_fence_before();
-      arrive_cluster(acc_empty_l);
+      __syncwarp();
+      if (ok && lane == 0) arrive_cluster(acc_empty_l);
+      epi_sync();  // the staged constants are reused for the next tile
+      if (*epi_stop) break;
     }
   }
 
