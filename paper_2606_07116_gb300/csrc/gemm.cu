@@ -28,11 +28,11 @@
 // Per SM and 128-code k-tile this moves 16 KB of shared memory for the MMA's B
 // reads and 16 KB of B stores, against 512 cycles of MMA work.
 //
-// Warp roles per CTA (17 warps):
+// Warp roles per CTA (21 warps):
 //   warp 0       TMEM allocation; in the leader CTA, lane 0 issues the MMAs
-//   warps 1-4    A converters (one per 32-lane quarter of TMEM)
-//   warps 5-8    B converters (32 rows each)
-//   warps 9-16   epilogue (two per TMEM quarter, 128 columns each)
+//   warps 1-8    A converters: two per 32-lane quarter of TMEM, alternating k-tiles
+//   warps 9-16   B converters: two per 32-row group, alternating k-tiles
+//   warps 17-20  epilogue (one per TMEM quarter, all 256 columns)
 // Every wait is bounded; a wait that runs out aborts the CTA and records
 // OFFQ_ERR_TIMEOUT in the device status word.
 #include <cuda.h>
@@ -54,12 +54,21 @@ constexpr int BN = 256;            // output channels per pair tile (128 rows of
 constexpr int BNH = BN / 2;        // rows of B held by one CTA
 constexpr int BK = 128;            // codes per k-tile
 constexpr int kChunksPerKt = BK / 32;  // 16-byte packed chunks per row per k-tile
-constexpr int kStages = 4;
-constexpr int kAWarps = 4, kBWarps = 4, kEpiWarps = 8;
+constexpr int kStages = 6;
+constexpr int kSplit = 2;  // converter warps per 32-row group (they take turns by k-tile)
+constexpr int kAWarps = 4 * kSplit, kBWarps = 4 * kSplit, kEpiWarps = 4;
+// Arrivals on the leader's barriers use the default (CTA-scope) release. Each
+// producing thread has already completed its own writes for the consumer (the
+// MMA reads them through the async proxy): fence.proxy.async after shared-memory
+// stores, tcgen05.wait::st after tensor-memory stores, tcgen05.wait::ld before
+// releasing the accumulator. A cluster-scope release would add a fence that
+// also waits for the converters' prefetch loads still in flight.
+constexpr bool kArriveClusterScope = false;
+constexpr int kEpiCols = BN / (kEpiWarps / 4);  // accumulator columns per epilogue warp
 constexpr int kFirstA = 1, kFirstB = kFirstA + kAWarps, kFirstEpi = kFirstB + kBWarps;
 constexpr int kThreads = (kFirstEpi + kEpiWarps) * 32;
-constexpr int kConvWarpsPerCta = kAWarps + kBWarps;  // one barrier arrival per warp
-constexpr int kPrefetch = 3;                         // k-tiles of loads in flight per converter thread
+constexpr int kConvWarpsPerCta = (kAWarps + kBWarps) / kSplit;  // one arrival per 32-row group and stage
+constexpr int kPrefetch = 2;                         // k-tiles of loads in flight per converter thread
 constexpr int kMaxStageG = 64;                       // offset blocks staged in shared memory
 constexpr int kAccCols = BN;       // fp32 accumulator columns (TMEM lanes = rows)
 constexpr int kACol0 = kAccCols;   // A operand stages live in TMEM after the accumulator
@@ -123,7 +132,10 @@ __device__ __forceinline__ uint32_t leader_addr(uint32_t local) {
 }
 
 __device__ __forceinline__ void arrive_cluster(uint32_t cluster_addr) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+  if constexpr (kArriveClusterScope)
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+  else
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 
 __device__ __forceinline__ bool try_wait_cluster(uint32_t bar, uint32_t parity) {
@@ -386,25 +398,34 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
     // flight in a register ring.
     const bool is_a = warp < kFirstB;
     const int quarter = warp & 3;
-    const int wb = warp - kFirstB;
+    const int wb = (warp - kFirstB) & 3;
+    const int part = is_a ? (warp - kFirstA) >> 2 : (warp - kFirstB) >> 2;  // k-tiles g == part mod kSplit
     const uint32_t full_l = leader_addr(full(0));
     const uint8_t* codes = is_a ? p.a_codes : p.w_codes;
     const int rb_count = is_a ? p.t_blocks : p.n_blocks;
     auto block_of = [&](int tile) { return is_a ? a_block(p, tile, rank, quarter) : b_block(p, tile, rank, wb); };
     uint4 ring[kPrefetch][kChunksPerKt];
     int ld_tile = cluster, ld_kt = 0;  // next k-tile to load
-    auto advance = [&](int& tile, int& kt) {
+    auto advance1 = [&](int& tile, int& kt) {
       if (++kt == nk) {
         kt = 0;
         tile += clusters;
       }
     };
+    auto advance = [&](int& tile, int& kt) {
+#pragma unroll
+      for (int i = 0; i < kSplit; ++i) advance1(tile, kt);
+    };
+#pragma unroll
+    for (int i = 0; i < kSplit; ++i)
+      if (i < part) advance1(ld_tile, ld_kt);
+    const int start_tile = ld_tile, start_kt = ld_kt;
 #pragma unroll
     for (int i = 0; i < kPrefetch; ++i) {
       if (ld_tile < num_tiles) load_kt(codes, block_of(ld_tile), rb_count, p.kchunks, ld_kt, lane, ring[i]);
       advance(ld_tile, ld_kt);
     }
-    int tile = cluster, kt = 0, g = 0;
+    int tile = start_tile, kt = start_kt, g = part;
     bool run = tile < num_tiles;
     while (run) {
 #pragma unroll
@@ -450,14 +471,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
         if (ld_tile < num_tiles) load_kt(codes, block_of(ld_tile), rb_count, p.kchunks, ld_kt, lane, ring[slot]);
         advance(ld_tile, ld_kt);
         advance(tile, kt);
-        ++g;
+        g += kSplit;
         run = __all_sync(0xFFFFFFFFu, tile < num_tiles && !*abort);
       }
     }
   } else {
     // ---------------- epilogue ----------------
     const int quarter = warp & 3;              // TMEM lanes this warp may read
-    const int half = (warp - kFirstEpi) / 4;   // which 128 accumulator columns
+    const int half = (warp - kFirstEpi) / 4;   // which kEpiCols accumulator columns
     const int et = threadIdx.x - kFirstEpi * 32;
     const int G = p.G;
     const bool staged = G <= kMaxStageG;
@@ -500,19 +521,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
       const int rl = quarter * 32 + lane;
       const int t = m0 + rl;
       const bool row_ok = t < p.T;
-      const int n0 = nt0 + half * (BN / 2);
-      const uint32_t acc_tm = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + half * (BN / 2);
+      const int n0 = nt0 + half * kEpiCols;
+      const uint32_t acc_tm = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + half * kEpiCols;
       constexpr int CW = 16;  // accumulator columns per TMEM load
       if (!ok) {
         // Aborted: nothing to drain.
       } else if (staged) {
         const float sa = Sa[rl];
-        for (int c = 0; c < (BN / 2) / CW; ++c) {
+        for (int c = 0; c < kEpiCols / CW; ++c) {
           uint32_t acc[CW];
           tmem_ld_16cols(acc_tm + c * CW, acc);
           tmem_ld_wait();
           const int nb = n0 + c * CW;
-          const int jc = half * (BN / 2) + c * CW;  // column within the staged tile
+          const int jc = half * kEpiCols + c * CW;  // column within the staged tile
           if (!row_ok || nb >= p.N) continue;
           const int nvalid = p.N - nb < CW ? p.N - nb : CW;
           float y[CW];
@@ -555,7 +576,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
         const float sa = row_ok ? __ldg(p.a_scale + t) : 0.f;
         const bool has_off = p.a_offset != nullptr && row_ok;
         const float* orow = has_off ? p.a_offset + static_cast<int64_t>(t) * G : p.a_scale;
-        for (int c = 0; c < (BN / 2) / CW; ++c) {
+        for (int c = 0; c < kEpiCols / CW; ++c) {
           uint32_t acc[CW];
           tmem_ld_16cols(acc_tm + c * CW, acc);
           tmem_ld_wait();
