@@ -320,6 +320,69 @@ __global__ void __launch_bounds__(Geo<L>::kMaxThreads) quantize_rows_kernel(cons
   }
 }
 
+// Rows without the rotation whose offset block is the whole row (g == K): one
+// warp per row, two passes over the row. Pass 1 takes sum, min and max; the
+// second pass re-reads the row (now in L2) and quantizes. Since rounding is
+// monotonic, max_k |fl(x_k - o)| = max(fl(max x - o), fl(o - min x)), so pass 1
+// already yields the row's residual absmax.
+template <typename Tin>
+__global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantArgs a) {
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int64_t row = static_cast<int64_t>(blockIdx.x) * 8 + warp;
+  if (row >= a.rows) return;
+  const bool offs = (a.flags & OFFQ_OFFSET) != 0;
+  const int K = a.K;
+  const int nch = K / 8;  // 8-element chunks per row
+  const int64_t t = row / a.H;
+  const int64_t h = row - t * a.H;
+  const Tin* xr = static_cast<const Tin*>(a.x) + t * a.ld_t + h * a.ld_h;
+
+  float sum = 0.f, mn = 3.402823466e38f, mx = -3.402823466e38f;
+  for (int c = lane; c < nch; c += 32) {
+    float v[8];
+    load_chunk8(xr + 8 * c, v);
+    float s4[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      s4[e] = v[2 * e] + v[2 * e + 1];
+      mn = fminf(mn, fminf(v[2 * e], v[2 * e + 1]));
+      mx = fmaxf(mx, fmaxf(v[2 * e], v[2 * e + 1]));
+    }
+    sum += (s4[0] + s4[1]) + (s4[2] + s4[3]);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+    mn = fminf(mn, __shfl_xor_sync(0xFFFFFFFFu, mn, o));
+    mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
+  }
+  const float off = offs ? sum * (1.0f / static_cast<float>(K)) : 0.f;  // K is a power of two
+  const float m = fmaxf(fmaxf(mx - off, off - mn), 0.f);
+  const float inv = m > 0.f ? __fdiv_rn(7.0f, m) : 0.f;
+
+  const int cpr = K / 32;
+  uint8_t* tile_row = a.tiled ? a.codes + (row >> 5) * cpr * 512 + (row & 31) * 16 : a.codes + row * (K / 2);
+  for (int c = lane; c < nch; c += 32) {
+    float v[8];
+    load_chunk8(xr + 8 * c, v);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] -= off;
+#pragma unroll
+    for (int e = 0; e < 8; e += 2) fma2(v[e], v[e + 1], inv, kMagic8);
+    uint32_t w = 0;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) w |= (__float_as_uint(v[e]) & 0xFu) << (4 * e);
+    const int bo = 4 * c;  // byte of the row-major row
+    uint8_t* dst = a.tiled ? tile_row + (bo >> 4) * 512 + (bo & 15) : tile_row + bo;
+    *reinterpret_cast<uint32_t*>(dst) = w;
+  }
+  if (lane == 0) {
+    a.scale[row] = m * a.scale_mul;
+    if (a.offset != nullptr) a.offset[row] = off;
+  }
+}
+
 template <int L, typename Tin>
 int launch_quant(QuantArgs a, cudaStream_t stream) {
   using GG = Geo<L>;
@@ -351,7 +414,16 @@ int launch_quant(QuantArgs a, cudaStream_t stream) {
 }
 
 template <typename Tin>
+int launch_stream(const QuantArgs& a, cudaStream_t stream) {
+  const int64_t grid = (a.rows + 7) / 8;
+  if (grid > 0x7FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
+  quantize_rows_stream_kernel<Tin><<<static_cast<unsigned>(grid), 256, 0, stream>>>(a);
+  return launch_status();
+}
+
+template <typename Tin>
 int dispatch_g(const QuantArgs& a, int g, cudaStream_t s) {
+  if ((a.flags & OFFQ_ROTATE) == 0 && a.G == 1) return launch_stream<Tin>(a, s);
   switch (g) {
     case 32: return launch_quant<5, Tin>(a, s);
     case 64: return launch_quant<6, Tin>(a, s);
