@@ -25,6 +25,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <type_traits>
 
 #include "offq.h"
 #include "offq_device.cuh"
@@ -236,7 +237,12 @@ __global__ void __launch_bounds__(Geo<L>::kMaxThreads) quantize_rows_kernel(cons
             make_float4(v[8 * i + 4], v[8 * i + 5], v[8 * i + 6], v[8 * i + 7]);
       }
     }
-    __syncthreads();
+    // A block's TPB threads share one warp (TPB <= 32) except for g = 8192.
+    if constexpr (TPB <= 32) {
+      __syncwarp();
+    } else {
+      __syncthreads();
+    }
     if (active) {
 #pragma unroll
       for (int hi = 0; hi < (1 << P); ++hi) {
@@ -297,19 +303,20 @@ __global__ void __launch_bounds__(Geo<L>::kMaxThreads) quantize_rows_kernel(cons
       }
     }
   }
-  __syncthreads();
-  {
-    // Codes leave in 16-byte chunks, rows fastest so that neighbouring rows of
-    // the tiled layout (16 bytes apart) are written by neighbouring threads.
-    const int64_t row0 = static_cast<int64_t>(blockIdx.x) * R;
-    const int nrows = static_cast<int>(a.rows - row0 < R ? a.rows - row0 : R);
-    const int cpr = K / 32;  // 16-byte chunks of codes per row
-    for (int c = tid; c < nrows * cpr; c += blockDim.x) {
-      const int cc = c / nrows, rr = c - cc * nrows;
-      const int64_t t = row0 + rr;
-      const uint4 w = *reinterpret_cast<const uint4*>(cbuf + static_cast<size_t>(rr) * (K / 2) + cc * 16);
-      uint8_t* dst = a.tiled ? a.codes + ((t >> 5) * cpr + cc) * 512 + (t & 31) * 16
-                             : a.codes + t * (K / 2) + cc * 16;
+  // Each block's TPB threads write the block's g/2 code bytes as 16-byte chunks.
+  if constexpr (TPB <= 32) {
+    __syncwarp();
+  } else {
+    __syncthreads();
+  }
+  if (active) {
+    const int cpr = K / 32;       // 16-byte chunks per row
+    const int cpb = g / 32;       // 16-byte chunks per block
+    for (int c = t1; c < cpb; c += TPB) {
+      const int cc = b * cpb + c;
+      const uint4 w = *reinterpret_cast<const uint4*>(crow + c * 16);
+      uint8_t* dst = a.tiled ? a.codes + ((row >> 5) * cpr + cc) * 512 + (row & 31) * 16
+                             : a.codes + row * (K / 2) + cc * 16;
       *reinterpret_cast<uint4*>(dst) = w;
     }
   }
@@ -321,11 +328,39 @@ __global__ void __launch_bounds__(Geo<L>::kMaxThreads) quantize_rows_kernel(cons
 }
 
 // Rows without the rotation whose offset block is the whole row (g == K): one
-// warp per row, two passes over the row. Pass 1 takes sum, min and max; the
-// second pass re-reads the row (now in L2) and quantizes. Since rounding is
-// monotonic, max_k |fl(x_k - o)| = max(fl(max x - o), fl(o - min x)), so pass 1
+// warp per row. Each lane issues the loads of up to CB 8-element chunks at once
+// and keeps them (raw) in registers, so a row of up to 256*CB elements costs one
+// trip to memory; longer rows are read twice in batches of CB chunks (the
+// second time from L2). Since rounding is monotonic,
+// max_k |fl(x_k - o)| = max(fl(max x - o), fl(o - min x)), so the first sweep
 // already yields the row's residual absmax.
 template <typename Tin>
+struct RawChunk {
+  static constexpr int kWords = sizeof(Tin) == 4 ? 8 : 4;  // 32-bit words per 8-element chunk
+  uint32_t w[kWords];
+  __device__ __forceinline__ void load(const Tin* p) {
+    const uint4 a = ldg_nc_v4(p);
+    w[0] = a.x; w[1] = a.y; w[2] = a.z; w[3] = a.w;
+    if constexpr (kWords == 8) {
+      const uint4 b = ldg_nc_v4(p + 4);
+      w[4] = b.x; w[5] = b.y; w[6] = b.z; w[7] = b.w;
+    }
+  }
+  __device__ __forceinline__ void unpack(float (&v)[8]) const {
+    if constexpr (kWords == 8) {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) v[e] = __uint_as_float(w[e]);
+    } else if constexpr (std::is_same<Tin, __half>::value) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) f16x2_to_f32(w[e], v[2 * e], v[2 * e + 1]);
+    } else {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) bf16x2_to_f32(w[e], v[2 * e], v[2 * e + 1]);
+    }
+  }
+};
+
+template <typename Tin, int CB>
 __global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantArgs a) {
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -337,19 +372,32 @@ __global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantAr
   const int64_t t = row / a.H;
   const int64_t h = row - t * a.H;
   const Tin* xr = static_cast<const Tin*>(a.x) + t * a.ld_t + h * a.ld_h;
+  const bool resident = nch <= 32 * CB;
 
+  RawChunk<Tin> raw[CB];
   float sum = 0.f, mn = 3.402823466e38f, mx = -3.402823466e38f;
-  for (int c = lane; c < nch; c += 32) {
-    float v[8];
-    load_chunk8(xr + 8 * c, v);
-    float s4[4];
+  for (int c0 = 0; c0 < nch; c0 += 32 * CB) {
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      s4[e] = v[2 * e] + v[2 * e + 1];
-      mn = fminf(mn, fminf(v[2 * e], v[2 * e + 1]));
-      mx = fmaxf(mx, fmaxf(v[2 * e], v[2 * e + 1]));
+    for (int i = 0; i < CB; ++i) {
+      const int c = c0 + lane + 32 * i;
+      if (c < nch) raw[i].load(xr + 8 * c);
     }
-    sum += (s4[0] + s4[1]) + (s4[2] + s4[3]);
+#pragma unroll
+    for (int i = 0; i < CB; ++i) {
+      const int c = c0 + lane + 32 * i;
+      if (c < nch) {
+        float v[8];
+        raw[i].unpack(v);
+        float s4[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          s4[e] = v[2 * e] + v[2 * e + 1];
+          mn = fminf(mn, fminf(v[2 * e], v[2 * e + 1]));
+          mx = fmaxf(mx, fmaxf(v[2 * e], v[2 * e + 1]));
+        }
+        sum += (s4[0] + s4[1]) + (s4[2] + s4[3]);
+      }
+    }
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -363,19 +411,32 @@ __global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantAr
 
   const int cpr = K / 32;
   uint8_t* tile_row = a.tiled ? a.codes + (row >> 5) * cpr * 512 + (row & 31) * 16 : a.codes + row * (K / 2);
-  for (int c = lane; c < nch; c += 32) {
-    float v[8];
-    load_chunk8(xr + 8 * c, v);
+  for (int c0 = 0; c0 < nch; c0 += 32 * CB) {
+    if (!resident) {
 #pragma unroll
-    for (int e = 0; e < 8; ++e) v[e] -= off;
+      for (int i = 0; i < CB; ++i) {
+        const int c = c0 + lane + 32 * i;
+        if (c < nch) raw[i].load(xr + 8 * c);
+      }
+    }
 #pragma unroll
-    for (int e = 0; e < 8; e += 2) fma2(v[e], v[e + 1], inv, kMagic8);
-    uint32_t w = 0;
+    for (int i = 0; i < CB; ++i) {
+      const int c = c0 + lane + 32 * i;
+      if (c < nch) {
+        float v[8];
+        raw[i].unpack(v);
 #pragma unroll
-    for (int e = 0; e < 8; ++e) w |= (__float_as_uint(v[e]) & 0xFu) << (4 * e);
-    const int bo = 4 * c;  // byte of the row-major row
-    uint8_t* dst = a.tiled ? tile_row + (bo >> 4) * 512 + (bo & 15) : tile_row + bo;
-    *reinterpret_cast<uint32_t*>(dst) = w;
+        for (int e = 0; e < 8; ++e) v[e] -= off;
+#pragma unroll
+        for (int e = 0; e < 8; e += 2) fma2(v[e], v[e + 1], inv, kMagic8);
+        uint32_t w = 0;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) w |= (__float_as_uint(v[e]) & 0xFu) << (4 * e);
+        const int bo = 4 * c;  // byte of the row-major row
+        uint8_t* dst = a.tiled ? tile_row + (bo >> 4) * 512 + (bo & 15) : tile_row + bo;
+        *reinterpret_cast<uint32_t*>(dst) = w;
+      }
+    }
   }
   if (lane == 0) {
     a.scale[row] = m * a.scale_mul;
@@ -417,7 +478,9 @@ template <typename Tin>
 int launch_stream(const QuantArgs& a, cudaStream_t stream) {
   const int64_t grid = (a.rows + 7) / 8;
   if (grid > 0x7FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
-  quantize_rows_stream_kernel<Tin><<<static_cast<unsigned>(grid), 256, 0, stream>>>(a);
+  // Up to 16 chunks (64 registers of bf16) per lane stay resident.
+  constexpr int CB = sizeof(Tin) == 4 ? 8 : 16;
+  quantize_rows_stream_kernel<Tin, CB><<<static_cast<unsigned>(grid), 256, 0, stream>>>(a);
   return launch_status();
 }
 
