@@ -12,14 +12,23 @@
 // The 1/sqrt(g) factor cancels in r / s, so it is applied only to the stored
 // scale and offset.
 //
-// Kernel layout (per g = 2^L): a thread owns E = 2^ceil((L+1)/2) elements of a
-// block and TPB = g / E threads share a block. Pass 1 loads 16-byte vectors
-// (coalesced across the block's threads) and runs the butterflies of every
-// index bit it holds in registers; one transpose through shared memory then
-// gives each thread the remaining index bits (plus the lowest one or two, so
-// neighbouring channels stay together for packing) and pass 2 finishes the
-// transform. The Hadamard is a Kronecker product of 2x2 stages, so the stages
-// may run in any order.
+// Kernel layouts (per g = 2^L; the Hadamard is a Kronecker product of 2x2
+// stages, so the stages may run in any order):
+//  * g <= 512 (quantize_rows_kernel): a thread owns E = 2^ceil((L+3)/2)
+//    elements and TPB = g / E threads share a block. Pass 1 loads 16-byte
+//    vectors (8 channels, coalesced across the block's threads) and runs the
+//    stages of every index bit it holds except bit 0; one swizzled transpose
+//    through shared memory gives each thread E contiguous channels, pass 2 runs
+//    the stages of bit 0 and of the bits that were spread over threads, and the
+//    thread packs its E codes into whole 16-byte chunks of the code buffer.
+//    Packed fp32x2 instructions take register pairs that differ in index bit 0,
+//    so the bit-0 stage alone runs on scalar adds.
+//  * g >= 1024 (quantize_rows_wide_kernel): E = 2^ceil((L+1)/2) elements per
+//    thread, the same two passes with pass 2 keeping the lowest one or two
+//    index bits, and codes staged in shared memory before the 16-byte writes.
+//  * No rotation and one block of g >= 1024 per row
+//    (quantize_rows_stream_kernel): a warp per row, offset and absmax from one
+//    sweep, codes from a second.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -55,7 +64,7 @@ struct QuantArgs {
 };
 
 template <int L>
-struct Geo {
+struct WideGeo {
   static constexpr int kLogE = (L + 2) / 2;
   static constexpr int kE = 1 << kLogE;       // elements per thread
   static constexpr int kP = L - kLogE;        // log2 threads per block
@@ -183,9 +192,214 @@ __device__ __forceinline__ float group_reduce(float v, int W, float* scratch) {
 // rne(x*inv) + 8, the activation code.
 constexpr float kMagic8 = 12582920.0f;
 
+// The bit pattern of such a rounded value is 0x4B400000 | (q + 8): bits 4-21
+// are zero, so (u1 << 4) + u0 has the byte of two codes in its low 8 bits.
+// pack_codes8 returns the 32-bit code word of channels c0..c7 (code of
+// channel 2k in the low nibble of byte k, channel 2k+1 in the high nibble).
+__device__ __forceinline__ uint32_t pack_codes8(uint32_t u0, uint32_t u1, uint32_t u2, uint32_t u3, uint32_t u4,
+                                                uint32_t u5, uint32_t u6, uint32_t u7) {
+  const uint32_t b0 = (u1 << 4) + u0, b1 = (u3 << 4) + u2, b2 = (u5 << 4) + u4, b3 = (u7 << 4) + u6;
+  return __byte_perm(__byte_perm(b0, b1, 0x0040), __byte_perm(b2, b3, 0x0040), 0x5410);
+}
+
+// Packed subtraction {a0 - c, a1 - c}.
+__device__ __forceinline__ void sub2(float& a0, float& a1, float c) {
+  const uint64_t A = pack2(a0, a1);
+  const uint64_t C = pack2(c, c);
+  uint64_t R;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(R) : "l"(A), "l"(C));
+  unpack2(R, a0, a1);
+}
+
+// Butterflies between registers r and r + 2^M (M >= 1) of every pair with bit M
+// of r clear, two per packed instruction: the pair (v[r], v[r+1]) against
+// (v[r+2^M], v[r+2^M+1]).
+template <int E, int M>
+__device__ __forceinline__ void fwht_reg_stage(float (&v)[E]) {
+  static_assert(M >= 1, "register bit 0 pairs the packed lanes");
+  constexpr int d = 1 << M;
+#pragma unroll
+  for (int r = 0; r < E; r += 2) {
+    if ((r & d) == 0) butterfly2(v[r], v[r + 1], v[r + d], v[r + d + 1]);
+  }
+}
+
+template <int E, int LO, int HI>
+__device__ __forceinline__ void fwht_reg_stages(float (&v)[E]) {
+  if constexpr (LO < HI) {
+    fwht_reg_stage<E, LO>(v);
+    fwht_reg_stages<E, LO + 1, HI>(v);
+  }
+}
+
+// Pairwise sum of N values (a balanced tree of depth log2 N).
+template <int N>
+__device__ __forceinline__ float tree_sum(const float* v) {
+  if constexpr (N == 1) {
+    return v[0];
+  } else {
+    return tree_sum<N / 2>(v) + tree_sum<N / 2>(v + N / 2);
+  }
+}
+
+// Geometry of quantize_rows_kernel (g = 2^L <= 512). E >= 2^(3+P) puts a
+// thread's in-block position (pass-1 index bits 3..3+P-1) below the bits it
+// holds in registers, so a pass-2 thread owns E contiguous channels.
+template <int L>
+struct NarrowGeo {
+  static constexpr int kLogE = (L + 4) / 2;   // ceil((L + 3) / 2)
+  static constexpr int kE = 1 << kLogE;       // elements per thread
+  static constexpr int kP = L - kLogE;        // log2 threads per block
+  static constexpr int kTPB = 1 << kP;
+  static constexpr int kNC = kE / 8;          // 8-channel loads per thread
+  static constexpr int kMaxThreads = 512;     // 128 blocks of g = 256 or 64 of g = 512
+  static_assert(3 + kP <= kLogE && kP >= 1 && kE >= 16, "narrow geometry");
+};
+
+// Transpose swizzle of quantize_rows_kernel (float index within the CTA's
+// buffer): bits 3-4 take the two lowest pass-2 thread bits, bit 2 the parity of
+// the block and of bit 5. Only bits >= 5 feed bits 2-4, so it is a bijection;
+// for g = 128 and 256 every quarter-warp of the pass-1 stores and of the
+// pass-2 loads hits eight distinct 16-byte bank groups, for g = 64 and 512 at
+// most two lanes share one. g = 32 keeps the plain layout.
+template <int L, int LOGE>
+__device__ __forceinline__ int swz_narrow(int idx) {
+  if constexpr (L == 5) {
+    return idx;
+  } else {
+    return idx ^ (((idx >> LOGE) & 3) << 3) ^ ((((idx >> L) ^ (idx >> 5)) & 1) << 2);
+  }
+}
+
 template <int L, typename Tin>
-__global__ void __launch_bounds__(Geo<L>::kMaxThreads) quantize_rows_kernel(const QuantArgs a) {
-  using GG = Geo<L>;
+__global__ void __launch_bounds__(NarrowGeo<L>::kMaxThreads) quantize_rows_kernel(const QuantArgs a) {
+  using GG = NarrowGeo<L>;
+  constexpr int E = GG::kE, P = GG::kP, TPB = GG::kTPB, NC = GG::kNC, LOGE = GG::kLogE;
+  constexpr int g = 1 << L;
+
+  extern __shared__ __align__(16) uint8_t smem[];
+  float* red = reinterpret_cast<float*>(smem);          // 32 floats for group_reduce
+  float* buf = reinterpret_cast<float*>(smem + 128);    // [rows_per_cta][K] fp32 transpose
+  const bool rotate = (a.flags & OFFQ_ROTATE) != 0;
+  const bool offs = (a.flags & OFFQ_OFFSET) != 0;
+  const int K = a.K;
+
+  const int tid = threadIdx.x;
+  const int lrow = tid / a.tpr;
+  const int j = tid - lrow * a.tpr;
+  const int64_t row = static_cast<int64_t>(blockIdx.x) * a.rows_per_cta + lrow;
+  const bool row_ok = row < a.rows;
+  const bool active = row_ok && (j < a.G * TPB);
+  const int b = j >> P;
+  const int t = j & (TPB - 1);
+
+  // Pass 1: register 8i + c holds channel 8t + 8 TPB i + c of block b.
+  float v[E];
+  if (active) {
+    const int64_t tok = row / a.H;
+    const int64_t h = row - tok * a.H;
+    const Tin* p = static_cast<const Tin*>(a.x) + tok * a.ld_t + h * a.ld_h + static_cast<int64_t>(b) * g + 8 * t;
+#pragma unroll
+    for (int i = 0; i < NC; ++i) load_chunk8(p + i * 8 * TPB, &v[8 * i]);
+  } else {
+#pragma unroll
+    for (int r = 0; r < E; ++r) v[r] = 0.f;
+  }
+
+  float off = 0.f;
+  if (rotate) {
+    // Offset = x[block start] / sqrt(g); removing it first leaves the residual.
+    if (offs && t == 0) {
+      off = v[0];
+      v[0] = 0.f;
+    }
+    fwht_reg_stages<E, 1, LOGE>(v);   // channel bits 1, 2 and 3+P .. L-1
+  } else if (offs) {
+    // Block mean by a pairwise tree (depth log2(E) in the thread, P across threads).
+    off = group_reduce<false>(tree_sum<E>(v), TPB, red) * (1.0f / static_cast<float>(g));
+  }
+
+  const int base = lrow * K + b * g;
+  if (active) {
+#pragma unroll
+    for (int i = 0; i < NC; ++i) {
+      const int e0 = base + 8 * t + 8 * TPB * i;
+      *reinterpret_cast<float4*>(buf + swz_narrow<L, LOGE>(e0)) =
+          make_float4(v[8 * i], v[8 * i + 1], v[8 * i + 2], v[8 * i + 3]);
+      *reinterpret_cast<float4*>(buf + swz_narrow<L, LOGE>(e0 + 4)) =
+          make_float4(v[8 * i + 4], v[8 * i + 5], v[8 * i + 6], v[8 * i + 7]);
+    }
+  }
+  __syncwarp();  // a block's TPB <= 8 threads share one warp
+  // Pass 2: register r holds channel E t + r of block b.
+  if (active) {
+#pragma unroll
+    for (int m = 0; m < E / 4; ++m) {
+      const float4 f = *reinterpret_cast<const float4*>(buf + swz_narrow<L, LOGE>(base + E * t + 4 * m));
+      v[4 * m] = f.x;
+      v[4 * m + 1] = f.y;
+      v[4 * m + 2] = f.z;
+      v[4 * m + 3] = f.w;
+    }
+  }
+  if (rotate) {
+#pragma unroll
+    for (int r = 0; r < E; r += 2) {   // channel bit 0
+      const float x0 = v[r], x1 = v[r + 1];
+      v[r] = x0 + x1;
+      v[r + 1] = x0 - x1;
+    }
+    fwht_reg_stages<E, 3, 3 + P>(v);   // channel bits 3 .. 3+P-1
+  } else if (offs) {
+#pragma unroll
+    for (int r = 0; r < E; r += 2) sub2(v[r], v[r + 1], off);
+  }
+
+  // Per-row absmax of the residual.
+  float mx[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int r = 0; r < E; ++r) mx[r & 3] = fmaxf(mx[r & 3], fabsf(v[r]));
+  float m = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+  m = group_reduce<true>(m, a.tpr, red);
+  const float inv = m > 0.f ? __fdiv_rn(7.0f, m) : 0.f;
+
+#pragma unroll
+  for (int r = 0; r < E; r += 2) fma2(v[r], v[r + 1], inv, kMagic8);
+
+  if (active) {
+    uint32_t wd[E / 8];
+#pragma unroll
+    for (int w = 0; w < E / 8; ++w) {
+      const float* q = &v[8 * w];
+      wd[w] = pack_codes8(__float_as_uint(q[0]), __float_as_uint(q[1]), __float_as_uint(q[2]),
+                          __float_as_uint(q[3]), __float_as_uint(q[4]), __float_as_uint(q[5]),
+                          __float_as_uint(q[6]), __float_as_uint(q[7]));
+    }
+    const int es = b * g + E * t;              // first channel of the thread's run
+    const int cpr = K / 32;                    // 16-byte chunks per row
+    uint8_t* rdst = a.tiled ? a.codes + (row >> 5) * cpr * 512 + (row & 31) * 16
+                            : a.codes + row * (K / 2);
+    const int cstride = a.tiled ? 512 : 16;    // bytes between consecutive chunks of a row
+    if constexpr (E >= 32) {
+#pragma unroll
+      for (int q = 0; q < E / 32; ++q) {
+        *reinterpret_cast<uint4*>(rdst + ((es >> 5) + q) * cstride) =
+            make_uint4(wd[4 * q], wd[4 * q + 1], wd[4 * q + 2], wd[4 * q + 3]);
+      }
+    } else {
+      *reinterpret_cast<uint2*>(rdst + (es >> 5) * cstride + (es & 31) / 2) = make_uint2(wd[0], wd[1]);
+    }
+  }
+
+  if (row_ok && j == 0) a.scale[row] = m * a.scale_mul;
+  if (active && t == 0 && a.offset != nullptr) {
+    a.offset[row * a.G + b] = offs ? (rotate ? off * a.inv_sqrt_g : off) : 0.f;
+  }
+}
+
+template <int L, typename Tin>
+__global__ void __launch_bounds__(WideGeo<L>::kMaxThreads) quantize_rows_wide_kernel(const QuantArgs a) {
+  using GG = WideGeo<L>;
   constexpr int E = GG::kE, P = GG::kP, TPB = GG::kTPB, Q = GG::kQ, NC = GG::kNC, LOGE = GG::kLogE;
   constexpr int g = 1 << L;
 
@@ -360,6 +574,65 @@ struct RawChunk {
   }
 };
 
+// Running min and max over raw input words: packed bf16x2 / f16x2 (exact) for
+// the 16-bit types, one fp32 value per word for fp32.
+template <typename Tin>
+struct RowMinMax {
+  uint32_t lo, hi;
+  __device__ __forceinline__ RowMinMax() {
+    if constexpr (std::is_same<Tin, __half>::value) {
+      lo = 0x7BFF7BFFu;  // +65504 twice
+      hi = 0xFBFFFBFFu;
+    } else {
+      lo = 0x7F7F7F7Fu;  // largest finite bf16 twice
+      hi = 0xFF7FFF7Fu;
+    }
+  }
+  __device__ __forceinline__ void add_word(uint32_t w) {
+    if constexpr (std::is_same<Tin, __half>::value) {
+      asm("min.f16x2 %0, %0, %1;" : "+r"(lo) : "r"(w));
+      asm("max.f16x2 %0, %0, %1;" : "+r"(hi) : "r"(w));
+    } else {
+      asm("min.bf16x2 %0, %0, %1;" : "+r"(lo) : "r"(w));
+      asm("max.bf16x2 %0, %0, %1;" : "+r"(hi) : "r"(w));
+    }
+  }
+  __device__ __forceinline__ void result(float& mn, float& mx) const {
+    float a, b, c, d;
+    if constexpr (std::is_same<Tin, __half>::value) {
+      f16x2_to_f32(lo, a, b);
+      f16x2_to_f32(hi, c, d);
+    } else {
+      bf16x2_to_f32(lo, a, b);
+      bf16x2_to_f32(hi, c, d);
+    }
+    mn = fminf(a, b);
+    mx = fmaxf(c, d);
+  }
+};
+
+template <>
+struct RowMinMax<float> {
+  float mn = 3.402823466e38f, mx = -3.402823466e38f;
+  __device__ __forceinline__ void add_word(uint32_t w) {
+    mn = fminf(mn, __uint_as_float(w));
+    mx = fmaxf(mx, __uint_as_float(w));
+  }
+  __device__ __forceinline__ void result(float& a, float& b) const {
+    a = mn;
+    b = mx;
+  }
+};
+
+// Packed accumulation {a0 + b0, a1 + b1}.
+__device__ __forceinline__ void add2(float& a0, float& a1, float b0, float b1) {
+  const uint64_t A = pack2(a0, a1);
+  const uint64_t B = pack2(b0, b1);
+  uint64_t R;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(R) : "l"(A), "l"(B));
+  unpack2(R, a0, a1);
+}
+
 template <typename Tin, int CB>
 __global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantArgs a) {
   const int warp = threadIdx.x >> 5;
@@ -375,7 +648,8 @@ __global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantAr
   const bool resident = nch <= 32 * CB;
 
   RawChunk<Tin> raw[CB];
-  float sum = 0.f, mn = 3.402823466e38f, mx = -3.402823466e38f;
+  RowMinMax<Tin> mm;
+  float s0 = 0.f, s1 = 0.f;
   for (int c0 = 0; c0 < nch; c0 += 32 * CB) {
 #pragma unroll
     for (int i = 0; i < CB; ++i) {
@@ -386,19 +660,19 @@ __global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantAr
     for (int i = 0; i < CB; ++i) {
       const int c = c0 + lane + 32 * i;
       if (c < nch) {
+#pragma unroll
+        for (int e = 0; e < RawChunk<Tin>::kWords; ++e) mm.add_word(raw[i].w[e]);
         float v[8];
         raw[i].unpack(v);
-        float s4[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          s4[e] = v[2 * e] + v[2 * e + 1];
-          mn = fminf(mn, fminf(v[2 * e], v[2 * e + 1]));
-          mx = fmaxf(mx, fmaxf(v[2 * e], v[2 * e + 1]));
-        }
-        sum += (s4[0] + s4[1]) + (s4[2] + s4[3]);
+        add2(v[0], v[1], v[2], v[3]);
+        add2(v[4], v[5], v[6], v[7]);
+        add2(v[0], v[1], v[4], v[5]);
+        add2(s0, s1, v[0], v[1]);
       }
     }
   }
+  float sum = s0 + s1, mn, mx;
+  mm.result(mn, mx);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
@@ -426,12 +700,13 @@ __global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantAr
         float v[8];
         raw[i].unpack(v);
 #pragma unroll
-        for (int e = 0; e < 8; ++e) v[e] -= off;
-#pragma unroll
-        for (int e = 0; e < 8; e += 2) fma2(v[e], v[e + 1], inv, kMagic8);
-        uint32_t w = 0;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) w |= (__float_as_uint(v[e]) & 0xFu) << (4 * e);
+        for (int e = 0; e < 8; e += 2) {
+          sub2(v[e], v[e + 1], off);
+          fma2(v[e], v[e + 1], inv, kMagic8);
+        }
+        const uint32_t w = pack_codes8(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]),
+                                       __float_as_uint(v[3]), __float_as_uint(v[4]), __float_as_uint(v[5]),
+                                       __float_as_uint(v[6]), __float_as_uint(v[7]));
         const int bo = 4 * c;  // byte of the row-major row
         uint8_t* dst = a.tiled ? tile_row + (bo >> 4) * 512 + (bo & 15) : tile_row + bo;
         *reinterpret_cast<uint32_t*>(dst) = w;
@@ -444,9 +719,55 @@ __global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantAr
   }
 }
 
+// Asks for the largest shared-memory carveout for a kernel, once per device,
+// so that the CTAs' shared memory does not cap residency below the register
+// limit.
+template <typename F>
+int prefer_max_shared(F* kern) {
+  static unsigned long long done = 0;  // bit d: set on device d
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return OFFQ_ERR_CUDA;
+  if (dev < 64 && (__atomic_load_n(&done, __ATOMIC_ACQUIRE) >> dev) & 1ull) return OFFQ_OK;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared) !=
+      cudaSuccess)
+    return OFFQ_ERR_CUDA;
+  if (dev < 64) __atomic_fetch_or(&done, 1ull << dev, __ATOMIC_ACQ_REL);
+  return OFFQ_OK;
+}
+
 template <int L, typename Tin>
-int launch_quant(QuantArgs a, cudaStream_t stream) {
-  using GG = Geo<L>;
+int launch_narrow(QuantArgs a, cudaStream_t stream) {
+  using GG = NarrowGeo<L>;
+  const int raw = a.G * GG::kTPB;
+  int tpr = 1;
+  if (raw <= 32) {
+    while (tpr < raw) tpr <<= 1;
+  } else {
+    tpr = (raw + 31) / 32 * 32;
+  }
+  if (tpr > GG::kMaxThreads) return OFFQ_ERR_UNSUPPORTED;
+  const size_t row_smem = static_cast<size_t>(a.K) * 4;
+  int R = std::max(1, 256 / tpr);
+  while (R > 1 && static_cast<size_t>(R) * row_smem > 64 * 1024) --R;
+  a.tpr = tpr;
+  a.rows_per_cta = R;
+  const size_t smem = 128 + static_cast<size_t>(R) * row_smem;
+  auto kern = quantize_rows_kernel<L, Tin>;
+  if (prefer_max_shared(kern) != OFFQ_OK) return OFFQ_ERR_CUDA;
+  if (smem > 48 * 1024) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
+        cudaSuccess)
+      return OFFQ_ERR_CUDA;
+  }
+  const int64_t grid = (a.rows + R - 1) / R;
+  if (grid > 0x7FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
+  kern<<<static_cast<unsigned>(grid), R * tpr, smem, stream>>>(a);
+  return launch_status();
+}
+
+template <int L, typename Tin>
+int launch_wide(QuantArgs a, cudaStream_t stream) {
+  using GG = WideGeo<L>;
   const int raw = a.G * GG::kTPB;
   int tpr = 1;
   if (raw <= 32) {
@@ -462,7 +783,7 @@ int launch_quant(QuantArgs a, cudaStream_t stream) {
   a.tpr = tpr;
   a.rows_per_cta = R;
   const size_t smem = static_cast<size_t>(R) * row_smem + 32 * sizeof(float);
-  auto kern = quantize_rows_kernel<L, Tin>;
+  auto kern = quantize_rows_wide_kernel<L, Tin>;
   if (smem > 48 * 1024) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
         cudaSuccess)
@@ -486,17 +807,17 @@ int launch_stream(const QuantArgs& a, cudaStream_t stream) {
 
 template <typename Tin>
 int dispatch_g(const QuantArgs& a, int g, cudaStream_t s) {
-  if ((a.flags & OFFQ_ROTATE) == 0 && a.G == 1) return launch_stream<Tin>(a, s);
+  if ((a.flags & OFFQ_ROTATE) == 0 && a.G == 1 && g >= 1024) return launch_stream<Tin>(a, s);
   switch (g) {
-    case 32: return launch_quant<5, Tin>(a, s);
-    case 64: return launch_quant<6, Tin>(a, s);
-    case 128: return launch_quant<7, Tin>(a, s);
-    case 256: return launch_quant<8, Tin>(a, s);
-    case 512: return launch_quant<9, Tin>(a, s);
-    case 1024: return launch_quant<10, Tin>(a, s);
-    case 2048: return launch_quant<11, Tin>(a, s);
-    case 4096: return launch_quant<12, Tin>(a, s);
-    case 8192: return launch_quant<13, Tin>(a, s);
+    case 32: return launch_narrow<5, Tin>(a, s);
+    case 64: return launch_narrow<6, Tin>(a, s);
+    case 128: return launch_narrow<7, Tin>(a, s);
+    case 256: return launch_narrow<8, Tin>(a, s);
+    case 512: return launch_narrow<9, Tin>(a, s);
+    case 1024: return launch_wide<10, Tin>(a, s);
+    case 2048: return launch_wide<11, Tin>(a, s);
+    case 4096: return launch_wide<12, Tin>(a, s);
+    case 8192: return launch_wide<13, Tin>(a, s);
     default: return OFFQ_ERR_UNSUPPORTED;
   }
 }

@@ -81,6 +81,15 @@ def test_quantize_workload_shapes(T, K, g, dist):
     _quant_and_check(_host(x, "bf16"), g, True, True)
 
 
+@pytest.mark.parametrize("K,dt", [(1024, "bf16"), (4096, "bf16"), (4096, "f16"), (4096, "f32"), (8192, "bf16")])
+@pytest.mark.parametrize("offset", [True, False])
+def test_quantize_whole_row_block_without_rotation(K, dt, offset):
+    """One offset block per row and no rotation (the q/k/v, o and gate/up sites); 45 rows leave a
+    ragged last CTA, and K = 8192 bf16 / 4096 fp32 rows take the two-sweep path."""
+    x = W.activations(45, K, seed=31 + K, n_out=4, mult=100.0)
+    _quant_and_check(_host(x, dt), K, False, offset)
+
+
 def test_quantize_toy_fp32():
     w = W.WORKLOADS["toy"]
     x = W.layer_inputs(w, w.layers[0])
