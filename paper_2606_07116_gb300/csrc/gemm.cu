@@ -68,7 +68,11 @@ constexpr int kEpiCols = BN / (kEpiWarps / 4);  // accumulator columns per epilo
 constexpr int kFirstA = 1, kFirstB = kFirstA + kAWarps, kFirstEpi = kFirstB + kBWarps;
 constexpr int kThreads = (kFirstEpi + kEpiWarps) * 32;
 constexpr int kConvWarpsPerCta = (kAWarps + kBWarps) / kSplit;  // one arrival per 32-row group and stage
-constexpr int kPrefetch = 2;                         // k-tiles of loads in flight per converter thread
+// k-tiles of loads in flight per converter thread. With one, a warp's loads
+// are issued right after its barrier arrival and have its next turn (two k-tiles
+// later) to land, and no load is outstanding when the arrival's release orders
+// the warp's earlier memory operations.
+constexpr int kPrefetch = 1;
 constexpr int kMaxStageG = 64;                       // offset blocks staged in shared memory
 constexpr int kAccCols = BN;       // fp32 accumulator columns (TMEM lanes = rows)
 constexpr int kACol0 = kAccCols;   // A operand stages live in TMEM after the accumulator
