@@ -27,8 +27,9 @@
  *     a kernel) are recorded in a device status word; offq_get_device_status
  *     reads and clears it.
  *   - NaN or Inf inputs: results are unspecified (no checks on the hot path).
- *   - Calls are thread-safe; the only state is a per-process cache of TMA
- *     descriptors guarded by a mutex, and the device status word.
+ *   - Calls are thread-safe. The only state is set on first use per device
+ *     (kernel attributes, the SM count, the status word's address) and the
+ *     device status word itself.
  *
  * Block size g. The online rotation is block-diagonal with g x g Sylvester
  * Hadamard blocks (group-wise offsetting, Sec. 3.2); each block of g channels
