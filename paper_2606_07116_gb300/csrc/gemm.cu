@@ -365,6 +365,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
   cluster_sync();  // barriers initialised and TMEM allocated in both CTAs
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // Setup above touches no global memory; from here on, the inputs of the
+  // previous kernel in the stream must be complete.
+  griddep_wait();
+  griddep_launch_dependents();
   int mma_tiles = 0;
 
   if (warp == 0) {
@@ -659,8 +663,7 @@ int launch_gemm(const GemmParams& p, cudaStream_t s) {
   if (sms < 2) return OFFQ_ERR_CUDA;
   const int tiles = p.m_pairs * p.n_tiles;
   const int clusters = tiles < sms / 2 ? tiles : sms / 2;
-  kern<<<2 * clusters, kThreads, kSmemBytes, s>>>(p);
-  return launch_status();
+  return launch_pdl(kern, dim3(2 * clusters), dim3(kThreads), kSmemBytes, s, p);
 }
 
 }  // namespace

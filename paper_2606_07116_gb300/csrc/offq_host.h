@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cstdint>
+#include <utility>
 #include <cuda_runtime.h>
 
 #include "offq.h"
@@ -28,6 +29,26 @@ inline int elem_bytes(int dtype) {
 inline int launch_status() {
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? OFFQ_OK : OFFQ_ERR_CUDA;
+}
+
+// Launches kern<<<grid, block, smem, stream>>>(args...) with programmatic
+// stream serialization: the kernel may be scheduled while the previous kernel
+// in the stream finishes, and waits for it (griddepcontrol.wait) before its
+// first global-memory access. Returns the launch's status.
+template <typename... KArgs, typename... Args>
+inline int launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                      Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...) == cudaSuccess ? OFFQ_OK : OFFQ_ERR_CUDA;
 }
 
 // Largest input dimension the row quantizer stages in shared memory.

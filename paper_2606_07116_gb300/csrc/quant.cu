@@ -276,6 +276,8 @@ __global__ void __launch_bounds__(NarrowGeo<L>::kMaxThreads) quantize_rows_kerne
   using GG = NarrowGeo<L>;
   constexpr int E = GG::kE, P = GG::kP, TPB = GG::kTPB, NC = GG::kNC, LOGE = GG::kLogE;
   constexpr int g = 1 << L;
+  griddep_wait();
+  griddep_launch_dependents();
 
   extern __shared__ __align__(16) uint8_t smem[];
   float* red = reinterpret_cast<float*>(smem);          // 32 floats for group_reduce
@@ -402,6 +404,8 @@ __global__ void __launch_bounds__(WideGeo<L>::kMaxThreads) quantize_rows_wide_ke
   using GG = WideGeo<L>;
   constexpr int E = GG::kE, P = GG::kP, TPB = GG::kTPB, Q = GG::kQ, NC = GG::kNC, LOGE = GG::kLogE;
   constexpr int g = 1 << L;
+  griddep_wait();
+  griddep_launch_dependents();
 
   extern __shared__ __align__(16) uint8_t smem[];
   const bool rotate = (a.flags & OFFQ_ROTATE) != 0;
@@ -635,6 +639,8 @@ __device__ __forceinline__ void add2(float& a0, float& a1, float b0, float b1) {
 
 template <typename Tin, int CB>
 __global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantArgs a) {
+  griddep_wait();
+  griddep_launch_dependents();
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int64_t row = static_cast<int64_t>(blockIdx.x) * 8 + warp;
@@ -761,8 +767,7 @@ int launch_narrow(QuantArgs a, cudaStream_t stream) {
   }
   const int64_t grid = (a.rows + R - 1) / R;
   if (grid > 0x7FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
-  kern<<<static_cast<unsigned>(grid), R * tpr, smem, stream>>>(a);
-  return launch_status();
+  return launch_pdl(kern, dim3(static_cast<unsigned>(grid)), dim3(R * tpr), smem, stream, a);
 }
 
 template <int L, typename Tin>
@@ -791,8 +796,7 @@ int launch_wide(QuantArgs a, cudaStream_t stream) {
   }
   const int64_t grid = (a.rows + R - 1) / R;
   if (grid > 0x7FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
-  kern<<<static_cast<unsigned>(grid), R * tpr, smem, stream>>>(a);
-  return launch_status();
+  return launch_pdl(kern, dim3(static_cast<unsigned>(grid)), dim3(R * tpr), smem, stream, a);
 }
 
 template <typename Tin>
@@ -801,8 +805,7 @@ int launch_stream(const QuantArgs& a, cudaStream_t stream) {
   if (grid > 0x7FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
   // Up to 16 chunks (64 registers of bf16) per lane stay resident.
   constexpr int CB = sizeof(Tin) == 4 ? 8 : 16;
-  quantize_rows_stream_kernel<Tin, CB><<<static_cast<unsigned>(grid), 256, 0, stream>>>(a);
-  return launch_status();
+  return launch_pdl(quantize_rows_stream_kernel<Tin, CB>, dim3(static_cast<unsigned>(grid)), dim3(256), 0, stream, a);
 }
 
 template <typename Tin>
@@ -847,6 +850,8 @@ int check_row_shape(int64_t K, int32_t g) {
 // zeroed. Codes are in the tiled operand layout. One thread per (row, block).
 __global__ void weight_repack_kernel(uint8_t* __restrict__ codes, float* __restrict__ rowsum, int64_t N,
                                      int64_t N_pad, int K, int g) {
+  griddep_wait();
+  griddep_launch_dependents();
   const int G = K / g;
   const int64_t id = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (id >= N_pad * G) return;
@@ -972,9 +977,8 @@ extern "C" int offq_prepare_weight(const void* w, int dtype, int64_t N, int64_t 
   const int64_t n_pad = (N + 31) / 32 * 32;
   const int64_t units = n_pad * (K / g);
   const int threads = 256;
-  weight_repack_kernel<<<static_cast<unsigned>((units + threads - 1) / threads), threads, 0, s>>>(
-      w_codes, w_offsum, N, n_pad, static_cast<int>(K), g);
-  return launch_status();
+  return launch_pdl(weight_repack_kernel, dim3(static_cast<unsigned>((units + threads - 1) / threads)),
+                    dim3(threads), 0, s, w_codes, w_offsum, N, n_pad, static_cast<int>(K), g);
 }
 
 extern "C" int64_t offq_act_codes_bytes(int64_t T, int64_t K) {
