@@ -197,6 +197,7 @@ class GpuStep:
             x = W.activations(T, K, seed=seed_base + 10 + i, dist=w.dist, n_out=w.n_out, mult=w.mult)
             host = torch.from_numpy(x).to(dt).pin_memory()
             dev = host.to(device)
+            dev_alt = host.to(device)  # end-to-end steps alternate between two input buffers
             g = W.block_for(K)
             codes = torch.empty((Q.padded_rows(T), K // 2), dtype=torch.uint8, device=device)
             scale = torch.empty((T,), dtype=torch.float32, device=device)
@@ -209,6 +210,7 @@ class GpuStep:
                 out = torch.empty((T, l.N), dtype=torch.bfloat16, device=device)
                 gemms.append({"layer": l, "codes": wc, "scale": ws, "rowsum": wr, "out": out})
             self.sites.append({"name": name, "K": K, "g": g, "flags": flags, "host": host, "dev": dev,
+                               "dev_alt": dev_alt, "consumed": [None, None],
                                "codes": codes, "scale": scale, "off": off, "gemms": gemms,
                                "in_bytes": dev.element_size()})
         self.kv = []
@@ -226,6 +228,8 @@ class GpuStep:
         last = self.sites[-1]["gemms"][-1]["out"]
         self.result = last
         self.result_host = torch.empty(last.shape, dtype=last.dtype).pin_memory()
+        self.copy_stream = torch.cuda.Stream(device)
+        self.parity = 0
         torch.cuda.synchronize(device)
 
     def launches_per_step(self):
@@ -253,13 +257,34 @@ class GpuStep:
             return e
 
         kv_done = False
+        ready = {}
+        if h2d:
+            # All of the step's inputs are on the host at its start: copy them on a
+            # side stream, each into the buffer its last use has finished reading.
+            par = self.parity
+            for s in self.sites:
+                dst = s["dev_alt"] if par else s["dev"]
+                if s["consumed"][par] is not None:
+                    self.copy_stream.wait_event(s["consumed"][par])
+                with torch.cuda.stream(self.copy_stream):
+                    dst.copy_(s["host"], non_blocking=True)
+                    ev = torch.cuda.Event()
+                    ev.record(self.copy_stream)
+                ready[s["name"]] = (dst, ev)
+            self.parity ^= 1
         for s in self.sites:
+            x = s["dev"]
             if h2d:
-                s["dev"].copy_(s["host"], non_blocking=True)
+                x, ev = ready[s["name"]]
+                stream.wait_event(ev)
             rec("quant")
-            Q.offq_quantize_act(s["dev"], T, s["K"], s["dev"].stride(0), s["g"], s["flags"], s["codes"],
+            Q.offq_quantize_act(x, T, s["K"], x.stride(0), s["g"], s["flags"], s["codes"],
                                 s["scale"], s["off"], stream)
             rec("quant")
+            if h2d:
+                done = torch.cuda.Event()
+                done.record(stream)
+                s["consumed"][par] = done
             for gm in s["gemms"]:
                 l = gm["layer"]
                 rec("gemm")
@@ -334,7 +359,8 @@ def run_gpu(args, rank, world, local_rank):
         raise RuntimeError(f"device status after warm-up: {Q.status_string(st)}")
 
     # ---- timed region: K steps, inputs resident, L2 flushed between steps ----
-    timers = {}
+    # Events bracket whole steps only: an event recorded between two launches
+    # would keep the second from being scheduled during the first one's tail.
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     barrier()
@@ -344,17 +370,24 @@ def run_gpu(args, rank, world, local_rank):
         for i in range(args.steps):
             flush_l2()
             starts[i].record(stream)
-            step.run(stream, timers=timers)
+            step.run(stream)
             ends[i].record(stream)
         torch.cuda.synchronize(device)
         wall1 = time.perf_counter()
     barrier()
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     dev_ms = sum(step_ms)
-    gemm_ms = sum(_pair_times(timers["gemm"]))
-    quant_ms = sum(_pair_times(timers["quant"]))
-    kv_ms = sum(_pair_times(timers.get("kv4", []))) if timers.get("kv4") else 0.0
-    n_gemm = len(timers["gemm"]) // 2
+
+    # ---- per-kernel durations: the same steps again, an event pair around every call ----
+    timers = {}
+    kb = max(1, min(args.steps, 50))
+    for _ in range(kb):
+        flush_l2()
+        step.run(stream, timers=timers)
+    torch.cuda.synchronize(device)
+    gemm_ms = sum(_pair_times(timers["gemm"])) * args.steps / kb
+    quant_ms = sum(_pair_times(timers["quant"])) * args.steps / kb
+    kv_ms = sum(_pair_times(timers.get("kv4", []))) * args.steps / kb if timers.get("kv4") else 0.0
     st = Q.offq_get_device_status(stream)
     if st != Q.OFFQ_OK:
         raise RuntimeError(f"device status after the timed region: {Q.status_string(st)}")
@@ -366,6 +399,7 @@ def run_gpu(args, rank, world, local_rank):
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
+    step.copy_stream.wait_event(e0)  # no copy starts before the timed region does
     for _ in range(e2e_steps):
         step.run(stream, h2d=True, d2h=True)
     e1.record(stream)
@@ -415,7 +449,7 @@ def run_gpu(args, rank, world, local_rank):
                 "d2h_bytes_per_step": int(step.result.numel() * step.result.element_size()),
                 "ms_per_step": round(e2e_ms, 4)},
         "gpu_launches": step.launches_per_step() * args.steps,
-        "gemm_launches": n_gemm,
+        "kernel_timing": f"per-launch durations from {kb} more flushed steps with an event pair around every call",
         "wall_s_timed_region": round(wall1 - wall0, 4),
         "clocks": clk.summary(),
     }
