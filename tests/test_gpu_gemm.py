@@ -170,3 +170,21 @@ def test_full_llama2_7b_gate_sampled():
 def test_full_llama2_7b_down_sampled():
     rows = W.unit_index_sample(2048, 64, seed=5)
     _check_layer(2048, 11008, 4096, 256, "bf16", rows=rows, n_out=4, mult=100.0)
+
+
+@pytest.mark.parametrize("T", [8, 32, 64])
+def test_decode_sweep(T):
+    """Decode batches of the Llama-2-7B up-projection shape (4096 -> 11008)."""
+    _check_layer(T, 4096, 11008, 4096, "bf16", seed=60 + T, n_out=4, mult=100.0)
+
+
+def test_llama3_8b_mlp_down_sampled():
+    """4096 tokens x 14336 -> 4096 with 14 offset blocks of 1024, Student-t(3) inputs, 3 outliers."""
+    rows = W.unit_index_sample(4096, 48, seed=6)
+    _check_layer(4096, 14336, 4096, 1024, "bf16", rows=rows, n_out=3, mult=100.0, dist="student_t3")
+
+
+def test_llama2_70b_down_shape_sampled():
+    """K = 28672 in 28 offset blocks of 1024, 6 outliers at 200x (1024 tokens, 1024 outputs)."""
+    rows = W.unit_index_sample(1024, 64, seed=7)
+    _check_layer(1024, 28672, 1024, 1024, "bf16", rows=rows, n_out=6, mult=200.0)
