@@ -324,7 +324,10 @@ __device__ __forceinline__ int b_block(const GemmParams& p, int tile, uint32_t r
 // Persistent pair kernel: cluster c processes pair tiles c, c + clusters, ...
 // (pair tile index = m_pair * n_tiles + n_tile). The k-tile counter g runs
 // across tiles so the stage ring never drains between tiles.
-template <int OUT>
+// kOneBlock: the offsets span the whole row (G == 1). Layers with several
+// offset blocks run a separate instantiation, so the register allocation of
+// the common one-block kernel does not carry the G-term epilogue loop.
+template <int OUT, bool kOneBlock>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_gemm_kernel(const GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
@@ -488,8 +491,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
     const int quarter = warp & 3;              // TMEM lanes this warp may read
     const int half = (warp - kFirstEpi) / 4;   // which kEpiCols accumulator columns
     const int et = threadIdx.x - kFirstEpi * 32;
-    const int G = p.G;
-    const bool staged = G <= kMaxStageG;
+    const int G = kOneBlock ? 1 : p.G;
+    const bool staged = kOneBlock || G <= kMaxStageG;
     float* Rs = reinterpret_cast<float*>(smem + kOffR);
     float* Ws = reinterpret_cast<float*>(smem + kOffW);
     float* Os = reinterpret_cast<float*>(smem + kOffO);
@@ -534,7 +537,60 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
       constexpr int CW = 16;  // accumulator columns per TMEM load
       if (!ok) {
         // Aborted: nothing to drain.
-      } else if (staged) {
+      } else if (!kOneBlock && staged) {
+        // Several offset blocks: the correction of 32 columns at a time (32
+        // independent FMA chains per block), then the accumulator in two halves.
+        const float sa = Sa[rl];
+        const float* orow = Os + rl * kStageGp;
+        for (int c2 = 0; c2 < kEpiCols / 32; ++c2) {
+          const int jc = half * kEpiCols + c2 * 32;  // column within the staged tile
+          float y[32];
+          {
+            const float ob = orow[0];
+            const float4* r4 = reinterpret_cast<const float4*>(Rs + jc);
+#pragma unroll
+            for (int q4 = 0; q4 < 8; ++q4) {
+              const float4 rv = r4[q4];
+              y[4 * q4] = ob * rv.x; y[4 * q4 + 1] = ob * rv.y; y[4 * q4 + 2] = ob * rv.z; y[4 * q4 + 3] = ob * rv.w;
+            }
+          }
+#pragma unroll 2
+          for (int b = 1; b < G; ++b) {
+            const float ob = orow[b];
+            const float4* r4 = reinterpret_cast<const float4*>(Rs + b * BN + jc);
+#pragma unroll
+            for (int q4 = 0; q4 < 8; ++q4) {
+              const float4 rv = r4[q4];
+              y[4 * q4] = fmaf(ob, rv.x, y[4 * q4]);
+              y[4 * q4 + 1] = fmaf(ob, rv.y, y[4 * q4 + 1]);
+              y[4 * q4 + 2] = fmaf(ob, rv.z, y[4 * q4 + 2]);
+              y[4 * q4 + 3] = fmaf(ob, rv.w, y[4 * q4 + 3]);
+            }
+          }
+#pragma unroll
+          for (int hh = 0; hh < 2; ++hh) {
+            uint32_t acc[CW];
+            tmem_ld_16cols(acc_tm + c2 * 32 + hh * CW, acc);
+            tmem_ld_wait();
+            const int nb = n0 + c2 * 32 + hh * CW;
+            if (!row_ok || nb >= p.N) continue;
+            const int nvalid = p.N - nb < CW ? p.N - nb : CW;
+            float z[CW];
+#pragma unroll
+            for (int jj = 0; jj < CW; ++jj) {
+              const float accf = __uint_as_float(acc[jj]) * 262144.0f;  // exact: * 2^18
+              z[jj] = Ws[jc + hh * CW + jj] * fmaf(sa, accf, y[hh * CW + jj]);
+            }
+            store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, z, nvalid);
+            if (p.acc_debug != nullptr) {
+              int32_t* d = p.acc_debug + static_cast<int64_t>(t) * p.N + nb;
+#pragma unroll
+              for (int jj = 0; jj < CW; ++jj)
+                if (jj < nvalid) d[jj] = __float2int_rn(__uint_as_float(acc[jj]) * 262144.0f);
+            }
+          }
+        }
+      } else if (kOneBlock) {
         const float sa = Sa[rl];
         for (int c = 0; c < kEpiCols / CW; ++c) {
           uint32_t acc[CW];
@@ -650,9 +706,9 @@ int num_sms() {
   return sms[dev];
 }
 
-template <int OUT>
+template <int OUT, bool kOneBlock>
 int launch_gemm(const GemmParams& p, cudaStream_t s) {
-  auto kern = w4a4_gemm_kernel<OUT>;
+  auto kern = w4a4_gemm_kernel<OUT, kOneBlock>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [&] {
@@ -708,9 +764,9 @@ extern "C" int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, co
   p.vec_ok = aligned(w_offsum, 16) && aligned(w_scale, 16) && (N % 4 == 0);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   switch (out_dtype) {
-    case OFFQ_F32: return launch_gemm<OFFQ_F32>(p, s);
-    case OFFQ_BF16: return launch_gemm<OFFQ_BF16>(p, s);
-    case OFFQ_F16: return launch_gemm<OFFQ_F16>(p, s);
+    case OFFQ_F32: return p.G == 1 ? launch_gemm<OFFQ_F32, true>(p, s) : launch_gemm<OFFQ_F32, false>(p, s);
+    case OFFQ_BF16: return p.G == 1 ? launch_gemm<OFFQ_BF16, true>(p, s) : launch_gemm<OFFQ_BF16, false>(p, s);
+    case OFFQ_F16: return p.G == 1 ? launch_gemm<OFFQ_F16, true>(p, s) : launch_gemm<OFFQ_F16, false>(p, s);
     default: return OFFQ_ERR_INVALID_ARG;
   }
 }
