@@ -81,19 +81,31 @@ constexpr int kTmemCols = 512;
 static_assert(kACol0 + kStages * kAColsPerStage <= kTmemCols, "TMEM budget");
 
 constexpr int kBStage = BNH * BK;  // 16 KB of E4M3 per stage
-constexpr int kOffB = 0;
-// Epilogue constants of one tile: row sums R[b][256 columns], channel scales,
-// and per row o[t][b] - 8 s_a[t] (odd row pitch: conflict-free per-lane reads).
-constexpr int kStageGp = kMaxStageG + 1;
-constexpr int kOffR = kOffB + kStages * kBStage;
-constexpr int kOffW = kOffR + kMaxStageG * BN * 4;
-constexpr int kOffO = kOffW + BN * 4;
-constexpr int kOffSa = kOffO + BM * kStageGp * 4;
-constexpr int kOffBars = kOffSa + BM * 4;
 constexpr int kNumBars = 2 * kStages + 2;
-constexpr int kOffMisc = kOffBars + kNumBars * 8;
-constexpr int kSmemBytes = kOffMisc + 64 + 1024;  // + slack to align the base to 1024
-static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
+// Output rows staged by the one-block epilogue (16-bit outputs): pitch padded
+// by 16 bytes, so the 32 rows a warp writes at once fall in distinct bank groups.
+constexpr int kOutPitch = BN * 2 + 16;
+
+// Shared memory of one instantiation: B stages; the tile's epilogue constants
+// (row sums R[b][256 columns], channel scales, per row o[t][b] - 8 s_a[t] with
+// an odd pitch for conflict-free per-lane reads, s_a); for one offset block the
+// staged output rows; barriers.
+template <bool kOneBlock>
+struct Smem {
+  static constexpr int kMaxG = kOneBlock ? 1 : kMaxStageG;
+  static constexpr int kGp = kOneBlock ? 1 : kMaxStageG + 1;
+  static constexpr int kOffB = 0;
+  static constexpr int kOffR = kOffB + kStages * kBStage;
+  static constexpr int kOffW = kOffR + kMaxG * BN * 4;
+  static constexpr int kOffO = kOffW + BN * 4;
+  static constexpr int kOffSa = kOffO + BM * kGp * 4;
+  static constexpr int kOffOut = kOffSa + BM * 4;
+  static constexpr int kOffBars = kOffOut + (kOneBlock ? BM * kOutPitch : 0);
+  static constexpr int kOffMisc = kOffBars + kNumBars * 8;
+  static constexpr int kBytes = kOffMisc + 64 + 1024;  // + slack to align the base to 1024
+  static_assert(kBytes <= 227 * 1024, "shared memory budget");
+  static_assert(kOffOut % 16 == 0, "bulk copies need 16-byte aligned rows");
+};
 
 constexpr uint32_t kIdesc = idesc_e4m3_f32(2 * BM, BN);  // pair MMA: M = 256, N = 256
 
@@ -113,6 +125,7 @@ struct GemmParams {
   int t_blocks, n_blocks;  // 32-row tiles present in the code buffers
   int kchunks;             // K / 32
   int vec_ok;              // rowsum and w_scale rows are 16-byte aligned
+  int async_out;           // 16-bit output and N % 8 == 0: one-block rows leave by bulk copy
 };
 
 // ---------------------------------------------------------------------------
@@ -241,6 +254,17 @@ __device__ __forceinline__ uint4 ldg_stream(const uint8_t* p) {
   return r;
 }
 
+// Bulk copy shared -> global (async proxy), tracked per thread in bulk groups.
+__device__ __forceinline__ void bulk_store(void* gdst, uint32_t ssrc, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(gdst), "r"(ssrc), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// This thread's bulk copies have read their shared-memory source.
+__device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// This thread's bulk copies are complete.
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
 __device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
 }
@@ -330,6 +354,9 @@ __device__ __forceinline__ int b_block(const GemmParams& p, int tile, uint32_t r
 template <int OUT, bool kOneBlock>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_gemm_kernel(const GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
+  using SL = Smem<kOneBlock>;
+  constexpr int kOffB = SL::kOffB, kOffR = SL::kOffR, kOffW = SL::kOffW, kOffO = SL::kOffO, kOffSa = SL::kOffSa;
+  constexpr int kOffBars = SL::kOffBars, kOffMisc = SL::kOffMisc, kStageGp = SL::kGp;
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* smem = smem_raw + (base - raw);
@@ -591,49 +618,70 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
           }
         }
       } else if (kOneBlock) {
-        const float sa = Sa[rl];
-        for (int c = 0; c < kEpiCols / CW; ++c) {
-          uint32_t acc[CW];
-          tmem_ld_16cols(acc_tm + c * CW, acc);
-          tmem_ld_wait();
-          const int nb = n0 + c * CW;
-          const int jc = half * kEpiCols + c * CW;  // column within the staged tile
-          if (!row_ok || nb >= p.N) continue;
-          const int nvalid = p.N - nb < CW ? p.N - nb : CW;
-          float y[CW];
-          {
-            const float ob = Os[rl * kStageGp];
+        // Packed fp32 pairs; each lane rounds as y = s_w * fma(s_a, acc * 2^18, o R)
+        // does (s_a * 2^18 and its product with acc are exact). 16-bit rows go to
+        // shared memory and leave by one bulk copy per row once the accumulator is
+        // read, so the tile's output write overlaps the next tile's MMAs.
+        const float sa2 = Sa[rl] * 262144.0f;
+        const float ob = Os[rl * kStageGp];
+        const uint64_t SA2 = pack2(sa2, sa2), OB = pack2(ob, ob);
+        const bool async_out = OUT != OFFQ_F32 && p.async_out != 0;
+        const uint32_t orow_s = base + SL::kOffOut + rl * kOutPitch;
+        if (async_out) bulk_wait_read_all();  // this row's previous copy has read the buffer
+        for (int c = 0; c < kEpiCols / CW; c += 2) {
+          uint32_t acc2[2 * CW];
+          tmem_ld_32cols_waited(acc_tm + c * CW, acc2);
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const uint32_t* acc = &acc2[h * CW];
+            const int nb = n0 + (c + h) * CW;
+            const int jc = half * kEpiCols + (c + h) * CW;
+            if (!row_ok || nb >= p.N) continue;
+            const int nvalid = p.N - nb < CW ? p.N - nb : CW;
             const float4* r4 = reinterpret_cast<const float4*>(Rs + jc);
+            const float4* w4 = reinterpret_cast<const float4*>(Ws + jc);
+            float y[CW];
 #pragma unroll
             for (int q4 = 0; q4 < CW / 4; ++q4) {
-              const float4 rv = r4[q4];
-              y[4 * q4] = ob * rv.x; y[4 * q4 + 1] = ob * rv.y; y[4 * q4 + 2] = ob * rv.z; y[4 * q4 + 3] = ob * rv.w;
+              const float4 rv = r4[q4], wv = w4[q4];
+              const uint64_t A0 = pack2(__uint_as_float(acc[4 * q4]), __uint_as_float(acc[4 * q4 + 1]));
+              const uint64_t A1 = pack2(__uint_as_float(acc[4 * q4 + 2]), __uint_as_float(acc[4 * q4 + 3]));
+              unpack2(mul2v(pack2(wv.x, wv.y), fma2v(SA2, A0, mul2v(OB, pack2(rv.x, rv.y)))), y[4 * q4],
+                      y[4 * q4 + 1]);
+              unpack2(mul2v(pack2(wv.z, wv.w), fma2v(SA2, A1, mul2v(OB, pack2(rv.z, rv.w)))), y[4 * q4 + 2],
+                      y[4 * q4 + 3]);
+            }
+            if (async_out) {
+              uint32_t hv[CW / 2];
+#pragma unroll
+              for (int i = 0; i < CW / 2; ++i) {
+                if (OUT == OFFQ_BF16) {
+                  const __nv_bfloat162 v = __floats2bfloat162_rn(y[2 * i], y[2 * i + 1]);
+                  hv[i] = *reinterpret_cast<const uint32_t*>(&v);
+                } else {
+                  const __half2 v = __floats2half2_rn(y[2 * i], y[2 * i + 1]);
+                  hv[i] = *reinterpret_cast<const uint32_t*>(&v);
+                }
+              }
+              sts128(orow_s + (c + h) * CW * 2, hv[0], hv[1], hv[2], hv[3]);
+              sts128(orow_s + (c + h) * CW * 2 + 16, hv[4], hv[5], hv[6], hv[7]);
+            } else {
+              store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, y, nvalid);
+            }
+            if (p.acc_debug != nullptr) {
+              int32_t* d = p.acc_debug + static_cast<int64_t>(t) * p.N + nb;
+#pragma unroll
+              for (int jj = 0; jj < CW; ++jj)
+                if (jj < nvalid) d[jj] = __float2int_rn(__uint_as_float(acc[jj]) * 262144.0f);
             }
           }
-          for (int b = 1; b < G; ++b) {
-            const float ob = Os[rl * kStageGp + b];
-            const float4* r4 = reinterpret_cast<const float4*>(Rs + b * BN + jc);
-#pragma unroll
-            for (int q4 = 0; q4 < CW / 4; ++q4) {
-              const float4 rv = r4[q4];
-              y[4 * q4] = fmaf(ob, rv.x, y[4 * q4]);
-              y[4 * q4 + 1] = fmaf(ob, rv.y, y[4 * q4 + 1]);
-              y[4 * q4 + 2] = fmaf(ob, rv.z, y[4 * q4 + 2]);
-              y[4 * q4 + 3] = fmaf(ob, rv.w, y[4 * q4 + 3]);
-            }
-          }
-#pragma unroll
-          for (int jj = 0; jj < CW; ++jj) {
-            const float accf = __uint_as_float(acc[jj]) * 262144.0f;  // exact: * 2^18
-            y[jj] = Ws[jc + jj] * fmaf(sa, accf, y[jj]);
-          }
-          store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, y, nvalid);
-          if (p.acc_debug != nullptr) {
-            int32_t* d = p.acc_debug + static_cast<int64_t>(t) * p.N + nb;
-#pragma unroll
-            for (int jj = 0; jj < CW; ++jj)
-              if (jj < nvalid) d[jj] = __float2int_rn(__uint_as_float(acc[jj]) * 262144.0f);
-          }
+        }
+        if (async_out && row_ok && n0 < p.N) {
+          const int ncols = p.N - n0 < kEpiCols ? p.N - n0 : kEpiCols;
+          fence_proxy_async_smem();  // the row's shared stores, visible to the bulk copy
+          bulk_store(static_cast<uint16_t*>(p.out) + static_cast<int64_t>(t) * p.ldo + n0, orow_s,
+                     static_cast<uint32_t>(ncols) * 2);
+          bulk_commit();
         }
       } else {
         // More offset blocks than the staging area holds: read the constants directly.
@@ -677,6 +725,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
       epi_sync();  // the staged constants are reused for the next tile
       if (*epi_stop) break;
     }
+    if (kOneBlock) bulk_wait_all();  // output rows in flight are written before the CTA ends
   }
 
   // ---------------- teardown ----------------
@@ -709,6 +758,7 @@ int num_sms() {
 template <int OUT, bool kOneBlock>
 int launch_gemm(const GemmParams& p, cudaStream_t s) {
   auto kern = w4a4_gemm_kernel<OUT, kOneBlock>;
+  constexpr int kSmemBytes = Smem<kOneBlock>::kBytes;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [&] {
@@ -762,6 +812,7 @@ extern "C" int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, co
   p.n_blocks = static_cast<int>((N + 31) / 32);
   p.kchunks = static_cast<int>(K / 32);
   p.vec_ok = aligned(w_offsum, 16) && aligned(w_scale, 16) && (N % 4 == 0);
+  p.async_out = out_dtype != OFFQ_F32 && N % 8 == 0;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   switch (out_dtype) {
     case OFFQ_F32: return p.G == 1 ? launch_gemm<OFFQ_F32, true>(p, s) : launch_gemm<OFFQ_F32, false>(p, s);
