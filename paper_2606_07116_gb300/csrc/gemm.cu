@@ -324,13 +324,14 @@ __device__ __forceinline__ void store_out(void* out, int64_t off, const float* y
 
 // Loads the four 16-byte chunks of k-tile kt of one row of a tiled code matrix
 // (zeros where the row block or the chunk does not exist).
-__device__ __forceinline__ void load_kt(const uint8_t* codes, int rb, int rb_count, int kchunks, int kt, int lane,
-                                        uint4 (&v)[kChunksPerKt]) {
+// blk: this lane's first byte of the row block (nullptr if the block does not
+// exist); the block's chunk c starts 512 * c bytes further.
+__device__ __forceinline__ void load_kt(const uint8_t* blk, int kchunks, int kt, uint4 (&v)[kChunksPerKt]) {
 #pragma unroll
   for (int j = 0; j < kChunksPerKt; ++j) {
     const int c = kt * kChunksPerKt + j;
-    if (rb < rb_count && c < kchunks)
-      v[j] = ldg_stream(codes + (static_cast<int64_t>(rb) * kchunks + c) * 512 + lane * 16);
+    if (blk != nullptr && c < kchunks)
+      v[j] = ldg_stream(blk + c * 512);
     else
       v[j] = make_uint4(0u, 0u, 0u, 0u);
   }
@@ -441,7 +442,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
     const uint32_t full_l = leader_addr(full(0));
     const uint8_t* codes = is_a ? p.a_codes : p.w_codes;
     const int rb_count = is_a ? p.t_blocks : p.n_blocks;
-    auto block_of = [&](int tile) { return is_a ? a_block(p, tile, rank, quarter) : b_block(p, tile, rank, wb); };
+    // This lane's first byte of the row block a tile needs (nullptr: the block
+    // lies past the buffer's rows). Computed once per tile, not per load.
+    auto block_ptr = [&](int tile) -> const uint8_t* {
+      const int rb = is_a ? a_block(p, tile, rank, quarter) : b_block(p, tile, rank, wb);
+      return rb < rb_count ? codes + static_cast<int64_t>(rb) * p.kchunks * 512 + lane * 16 : nullptr;
+    };
     uint4 ring[kPrefetch][kChunksPerKt];
     int ld_tile = cluster, ld_kt = 0;  // next k-tile to load
     auto advance1 = [&](int& tile, int& kt) {
@@ -460,10 +466,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
     const int start_tile = ld_tile, start_kt = ld_kt;
 #pragma unroll
     for (int i = 0; i < kPrefetch; ++i) {
-      if (ld_tile < num_tiles) load_kt(codes, block_of(ld_tile), rb_count, p.kchunks, ld_kt, lane, ring[i]);
+      if (ld_tile < num_tiles) load_kt(block_ptr(ld_tile), p.kchunks, ld_kt, ring[i]);
       advance(ld_tile, ld_kt);
     }
     int tile = start_tile, kt = start_kt, g = part;
+    int blk_tile = ld_tile;  // the tile whose row block blk points into
+    const uint8_t* blk = ld_tile < num_tiles ? block_ptr(ld_tile) : nullptr;
     bool run = tile < num_tiles;
     while (run) {
 #pragma unroll
@@ -506,7 +514,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
         __syncwarp();
         if (lane == 0) arrive_cluster(full_l + 8u * s);
         // Refill this slot kPrefetch k-tiles ahead.
-        if (ld_tile < num_tiles) load_kt(codes, block_of(ld_tile), rb_count, p.kchunks, ld_kt, lane, ring[slot]);
+        if (ld_tile < num_tiles) {
+          if (ld_tile != blk_tile) {
+            blk_tile = ld_tile;
+            blk = block_ptr(ld_tile);
+          }
+          load_kt(blk, p.kchunks, ld_kt, ring[slot]);
+        }
         advance(ld_tile, ld_kt);
         advance(tile, kt);
         g += kSplit;
