@@ -67,6 +67,7 @@ constexpr bool kArriveClusterScope = false;
 constexpr int kEpiCols = BN / (kEpiWarps / 4);  // accumulator columns per epilogue warp
 constexpr int kFirstA = 1, kFirstB = kFirstA + kAWarps, kFirstEpi = kFirstB + kBWarps;
 constexpr int kThreads = (kFirstEpi + kEpiWarps) * 32;
+static_assert(kSplit <= kStages, "a converter's next stage is at most one ring turn ahead");
 constexpr int kConvWarpsPerCta = (kAWarps + kBWarps) / kSplit;  // one arrival per 32-row group and stage
 // k-tiles of loads in flight per converter thread. With one, a warp's loads
 // are issued right after its barrier arrival and have its next turn (two k-tiles
@@ -405,14 +406,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
   if (warp == 0) {
     // ---------------- MMA issuer (leader CTA) ----------------
     if (rank == 0 && lane == 0) {
-      int g = 0, lt = 0;
+      int s = 0, phase = 0, lt = 0;  // stage and phase parity of the next k-tile
       for (int tile = cluster; tile < num_tiles && !*abort; tile += clusters, ++lt) {
         if (!wait_cluster(acc_empty, (lt & 1) ^ 1, abort)) break;
         tc_fence_after();
         bool ok = true;
-        for (int kt = 0; kt < nk; ++kt, ++g) {
-          const int s = g % kStages;
-          if (!wait_cluster(full(s), (g / kStages) & 1, abort)) {
+        for (int kt = 0; kt < nk; ++kt) {
+          if (!wait_cluster(full(s), phase, abort)) {
             ok = false;
             break;
           }
@@ -424,6 +424,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
                     (kt | kk) != 0 ? 1u : 0u);
           }
           mma2_commit_both(empty(s));
+          if (++s == kStages) {
+            s = 0;
+            phase ^= 1;
+          }
         }
         mma2_commit_both(acc_full);
         mma_tiles = lt + 1;
@@ -469,7 +473,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
       if (ld_tile < num_tiles) load_kt(block_ptr(ld_tile), p.kchunks, ld_kt, ring[i]);
       advance(ld_tile, ld_kt);
     }
-    int tile = start_tile, kt = start_kt, g = part;
+    int tile = start_tile, kt = start_kt;
+    int s = part, phase = 0;  // stage and phase parity of this warp's k-tile g (g == part mod kSplit)
     int blk_tile = ld_tile;  // the tile whose row block blk points into
     const uint8_t* blk = ld_tile < num_tiles ? block_ptr(ld_tile) : nullptr;
     bool run = tile < num_tiles;
@@ -477,9 +482,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
 #pragma unroll
       for (int slot = 0; slot < kPrefetch; ++slot) {
         if (!run) break;
-        const int s = g % kStages;
-        // Warp-uniform outcome, so the __syncwarp below is reached by all lanes.
-        if (!__all_sync(0xFFFFFFFFu, wait_cluster(empty(s), ((g / kStages) & 1) ^ 1, abort))) {
+        // Warp-uniform outcome, so the __syncwarp below is reached by all lanes. After
+        // an abort no stage frees up again, so this wait is where a converter stops.
+        if (!__all_sync(0xFFFFFFFFu, wait_cluster(empty(s), phase ^ 1, abort))) {
           run = false;
           break;
         }
@@ -523,8 +528,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
         }
         advance(ld_tile, ld_kt);
         advance(tile, kt);
-        g += kSplit;
-        run = __all_sync(0xFFFFFFFFu, tile < num_tiles && !*abort);
+        s += kSplit;
+        if (s >= kStages) {
+          s -= kStages;
+          phase ^= 1;
+        }
+        run = tile < num_tiles;  // warp-uniform
       }
     }
   } else {
