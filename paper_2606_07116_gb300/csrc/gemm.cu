@@ -54,9 +54,26 @@ constexpr int BN = 256;            // output channels per pair tile (128 rows of
 constexpr int BNH = BN / 2;        // rows of B held by one CTA
 constexpr int BK = 128;            // codes per k-tile
 constexpr int kChunksPerKt = BK / 32;  // 16-byte packed chunks per row per k-tile
-constexpr int kStages = 6;
-constexpr int kSplit = 2;  // converter warps per 32-row group (they take turns by k-tile)
-constexpr int kAWarps = 4 * kSplit, kBWarps = 4 * kSplit, kEpiWarps = 4;
+// Warp roles of one instantiation. kSplitA / kSplitB converter warps serve each
+// 32-row group of A / B, taking turns by k-tile; kEpiWarps drain the
+// accumulator (one or two per 32-lane TMEM quarter). 21 warps put 6 on one SM
+// sub-partition: 80 registers per thread. (Trading B converters for epilogue
+// warps in the several-block kernel left one B warp per group too slow.)
+template <bool kOneBlock>
+struct Roles {
+  // Stages of the operand ring. Several offset blocks take 4, so 128 TMEM columns
+  // stay free for half of the precomputed offset correction.
+  static constexpr int kStages = kOneBlock ? 6 : 4;
+  static constexpr int kSplitA = 2;
+  static constexpr int kSplitB = 2;
+  static constexpr int kAWarps = 4 * kSplitA, kBWarps = 4 * kSplitB;
+  static constexpr int kEpiWarps = 4;
+  static constexpr int kEpiCols = BN / (kEpiWarps / 4);  // accumulator columns per epilogue warp
+  static constexpr int kFirstA = 1, kFirstB = kFirstA + kAWarps, kFirstEpi = kFirstB + kBWarps;
+  static constexpr int kThreads = (kFirstEpi + kEpiWarps) * 32;
+  static_assert(kSplitA <= kStages && kSplitB <= kStages, "a converter's next stage is at most one ring turn ahead");
+};
+constexpr int kConvWarpsPerCta = 8;  // arrivals per stage and CTA: one per 32-row group of A and of B
 // Arrivals on the leader's barriers use the default (CTA-scope) release. Each
 // producing thread has already completed its own writes for the consumer (the
 // MMA reads them through the async proxy): fence.proxy.async after shared-memory
@@ -64,25 +81,26 @@ constexpr int kAWarps = 4 * kSplit, kBWarps = 4 * kSplit, kEpiWarps = 4;
 // releasing the accumulator. A cluster-scope release would add a fence that
 // also waits for the converters' prefetch loads still in flight.
 constexpr bool kArriveClusterScope = false;
-constexpr int kEpiCols = BN / (kEpiWarps / 4);  // accumulator columns per epilogue warp
-constexpr int kFirstA = 1, kFirstB = kFirstA + kAWarps, kFirstEpi = kFirstB + kBWarps;
-constexpr int kThreads = (kFirstEpi + kEpiWarps) * 32;
-static_assert(kSplit <= kStages, "a converter's next stage is at most one ring turn ahead");
-constexpr int kConvWarpsPerCta = (kAWarps + kBWarps) / kSplit;  // one arrival per 32-row group and stage
 // k-tiles of loads in flight per converter thread. With one, a warp's loads
 // are issued right after its barrier arrival and have its next turn (two k-tiles
 // later) to land, and no load is outstanding when the arrival's release orders
 // the warp's earlier memory operations.
 constexpr int kPrefetch = 1;
-constexpr int kMaxStageG = 64;                       // offset blocks staged in shared memory
+constexpr int kMaxStageG = 48;                       // offset blocks staged in shared memory
 constexpr int kAccCols = BN;       // fp32 accumulator columns (TMEM lanes = rows)
 constexpr int kACol0 = kAccCols;   // A operand stages live in TMEM after the accumulator
 constexpr int kAColsPerStage = BK / 4;  // 4 E4M3 values per 32-bit column
 constexpr int kTmemCols = 512;
-static_assert(kACol0 + kStages * kAColsPerStage <= kTmemCols, "TMEM budget");
+static_assert(kACol0 + Roles<true>::kStages * kAColsPerStage <= kTmemCols, "TMEM budget");
+// Several offset blocks: the correction sum_b (o_b - 8 s_a) R[b][n] of a tile is
+// computed while its MMAs run; accumulator columns 0..127 keep theirs in TMEM
+// after the A stages, columns 128..255 in shared memory.
+constexpr int kCorrCol0 = kACol0 + Roles<false>::kStages * kAColsPerStage;
+constexpr int kCorrTmemCols = 128;
+static_assert(kCorrCol0 + kCorrTmemCols <= kTmemCols, "TMEM budget with the correction");
+constexpr int kCorrPitch = (BN - kCorrTmemCols) * 4 + 16;  // bytes per row of the shared half, padded
 
 constexpr int kBStage = BNH * BK;  // 16 KB of E4M3 per stage
-constexpr int kNumBars = 2 * kStages + 2;
 // Output rows staged by the one-block epilogue (16-bit outputs): pitch padded
 // by 16 bytes, so the 32 rows a warp writes at once fall in distinct bank groups.
 constexpr int kOutPitch = BN * 2 + 16;
@@ -93,6 +111,8 @@ constexpr int kOutPitch = BN * 2 + 16;
 // staged output rows; barriers.
 template <bool kOneBlock>
 struct Smem {
+  static constexpr int kStages = Roles<kOneBlock>::kStages;
+  static constexpr int kNumBars = 2 * kStages + 2;
   static constexpr int kMaxG = kOneBlock ? 1 : kMaxStageG;
   static constexpr int kGp = kOneBlock ? 1 : kMaxStageG + 1;
   static constexpr int kOffB = 0;
@@ -100,8 +120,8 @@ struct Smem {
   static constexpr int kOffW = kOffR + kMaxG * BN * 4;
   static constexpr int kOffO = kOffW + BN * 4;
   static constexpr int kOffSa = kOffO + BM * kGp * 4;
-  static constexpr int kOffOut = kOffSa + BM * 4;
-  static constexpr int kOffBars = kOffOut + (kOneBlock ? BM * kOutPitch : 0);
+  static constexpr int kOffOut = kOffSa + BM * 4;  // one block: staged output rows; several: the correction half
+  static constexpr int kOffBars = kOffOut + (kOneBlock ? BM * kOutPitch : BM * kCorrPitch);
   static constexpr int kOffMisc = kOffBars + kNumBars * 8;
   static constexpr int kBytes = kOffMisc + 64 + 1024;  // + slack to align the base to 1024
   static_assert(kBytes <= 227 * 1024, "shared memory budget");
@@ -241,6 +261,7 @@ __device__ __forceinline__ void tmem_st_32cols(uint32_t taddr, const uint32_t (&
 }
 
 // Named barrier among the epilogue warps only.
+template <int kEpiWarps>
 __device__ __forceinline__ void epi_sync() {
   asm volatile("bar.sync 1, %0;" ::"r"(kEpiWarps * 32) : "memory");
 }
@@ -265,6 +286,12 @@ __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.comm
 __device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 // This thread's bulk copies are complete.
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+  uint4 r;
+  asm volatile("ld.shared.v4.b32 {%0,%1,%2,%3}, [%4];" : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "r"(addr) : "memory");
+  return r;
+}
 
 __device__ __forceinline__ void sts128(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
@@ -354,9 +381,14 @@ __device__ __forceinline__ int b_block(const GemmParams& p, int tile, uint32_t r
 // offset blocks run a separate instantiation, so the register allocation of
 // the common one-block kernel does not carry the G-term epilogue loop.
 template <int OUT, bool kOneBlock>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_gemm_kernel(const GemmParams p) {
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kThreads, 1)
+    w4a4_gemm_kernel(const GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
   using SL = Smem<kOneBlock>;
+  using RL = Roles<kOneBlock>;
+  constexpr int kStages = RL::kStages;
+  constexpr int kFirstA = RL::kFirstA, kFirstB = RL::kFirstB, kFirstEpi = RL::kFirstEpi;
+  constexpr int kEpiWarps = RL::kEpiWarps, kEpiCols = RL::kEpiCols;
   constexpr int kOffB = SL::kOffB, kOffR = SL::kOffR, kOffW = SL::kOffW, kOffO = SL::kOffO, kOffSa = SL::kOffSa;
   constexpr int kOffBars = SL::kOffBars, kOffMisc = SL::kOffMisc, kStageGp = SL::kGp;
   const uint32_t raw = smem_u32(smem_raw);
@@ -442,7 +474,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
     const bool is_a = warp < kFirstB;
     const int quarter = warp & 3;
     const int wb = (warp - kFirstB) & 3;
-    const int part = is_a ? (warp - kFirstA) >> 2 : (warp - kFirstB) >> 2;  // k-tiles g == part mod kSplit
+    const int part = is_a ? (warp - kFirstA) >> 2 : (warp - kFirstB) >> 2;  // k-tiles g == part mod split
+    static_assert(RL::kSplitA == RL::kSplitB, "one k-tile stride for both converter kinds");
+    constexpr int split = RL::kSplitA;
     const uint32_t full_l = leader_addr(full(0));
     const uint8_t* codes = is_a ? p.a_codes : p.w_codes;
     const int rb_count = is_a ? p.t_blocks : p.n_blocks;
@@ -462,10 +496,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
     };
     auto advance = [&](int& tile, int& kt) {
 #pragma unroll
-      for (int i = 0; i < kSplit; ++i) advance1(tile, kt);
+      for (int i = 0; i < split; ++i) advance1(tile, kt);
     };
 #pragma unroll
-    for (int i = 0; i < kSplit; ++i)
+    for (int i = 0; i < split; ++i)
       if (i < part) advance1(ld_tile, ld_kt);
     const int start_tile = ld_tile, start_kt = ld_kt;
 #pragma unroll
@@ -474,7 +508,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
       advance(ld_tile, ld_kt);
     }
     int tile = start_tile, kt = start_kt;
-    int s = part, phase = 0;  // stage and phase parity of this warp's k-tile g (g == part mod kSplit)
+    int s = part, phase = 0;  // stage and phase parity of this warp's k-tile g (g == part mod split)
     int blk_tile = ld_tile;  // the tile whose row block blk points into
     const uint8_t* blk = ld_tile < num_tiles ? block_ptr(ld_tile) : nullptr;
     bool run = tile < num_tiles;
@@ -528,7 +562,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
         }
         advance(ld_tile, ld_kt);
         advance(tile, kt);
-        s += kSplit;
+        s += split;
         if (s >= kStages) {
           s -= kStages;
           phase ^= 1;
@@ -552,7 +586,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
     // own barrier, so all eight warps leave together (bar.sync has no timeout).
     volatile int* epi_stop = reinterpret_cast<volatile int*>(smem + kOffMisc + 32);
     if (et == 0) *epi_stop = 0;
-    epi_sync();
+    epi_sync<kEpiWarps>();
     int lt = 0;
     for (int tile = cluster; tile < num_tiles; tile += clusters, ++lt) {
       const int m0 = (tile / p.n_tiles) * 2 * BM + static_cast<int>(rank) * BM;
@@ -575,7 +609,56 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
           Os[r * kStageGp + b] = v;
         }
       }
-      epi_sync();
+      epi_sync<kEpiWarps>();
+      if constexpr (!kOneBlock) {
+        if (staged) {
+          // While this tile's MMAs run: its offset correction, per element the same
+          // chain as at the tile end (block 0 multiplied, then FMAs in block order).
+          constexpr int CW = 16;
+          const int rl = quarter * 32 + lane;
+          const float* orow = Os + rl * kStageGp;
+          const uint32_t corr_tm = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + kCorrCol0;
+          const uint32_t corr_s = base + SL::kOffOut + rl * kCorrPitch;
+          for (int c = 0; c < kEpiCols / CW; ++c) {
+            const int jc = half * kEpiCols + c * CW;  // column within the tile
+            float y[CW];
+            {
+              const float ob = orow[0];
+              const float4* r4 = reinterpret_cast<const float4*>(Rs + jc);
+#pragma unroll
+              for (int q4 = 0; q4 < CW / 4; ++q4) {
+                const float4 rv = r4[q4];
+                y[4 * q4] = ob * rv.x; y[4 * q4 + 1] = ob * rv.y; y[4 * q4 + 2] = ob * rv.z; y[4 * q4 + 3] = ob * rv.w;
+              }
+            }
+            for (int b = 1; b < G; ++b) {
+              const float ob = orow[b];
+              const float4* r4 = reinterpret_cast<const float4*>(Rs + b * BN + jc);
+#pragma unroll
+              for (int q4 = 0; q4 < CW / 4; ++q4) {
+                const float4 rv = r4[q4];
+                y[4 * q4] = fmaf(ob, rv.x, y[4 * q4]);
+                y[4 * q4 + 1] = fmaf(ob, rv.y, y[4 * q4 + 1]);
+                y[4 * q4 + 2] = fmaf(ob, rv.z, y[4 * q4 + 2]);
+                y[4 * q4 + 3] = fmaf(ob, rv.w, y[4 * q4 + 3]);
+              }
+            }
+            if (jc < kCorrTmemCols) {
+              uint32_t u[CW];
+#pragma unroll
+              for (int jj = 0; jj < CW; ++jj) u[jj] = __float_as_uint(y[jj]);
+              tmem_st_16cols(corr_tm + jc, u);
+            } else {
+              const uint32_t a = corr_s + (jc - kCorrTmemCols) * 4;
+#pragma unroll
+              for (int q4 = 0; q4 < CW / 4; ++q4)
+                sts128(a + 16 * q4, __float_as_uint(y[4 * q4]), __float_as_uint(y[4 * q4 + 1]),
+                       __float_as_uint(y[4 * q4 + 2]), __float_as_uint(y[4 * q4 + 3]));
+            }
+          }
+          tmem_st_wait();
+        }
+      }
       const bool ok = __all_sync(0xFFFFFFFFu, wait_cluster(acc_full, lt & 1, abort));
       if (!ok && lane == 0) *epi_stop = 1;
       tc_fence_after();
@@ -588,56 +671,39 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
       if (!ok) {
         // Aborted: nothing to drain.
       } else if (!kOneBlock && staged) {
-        // Several offset blocks: the correction of 32 columns at a time (32
-        // independent FMA chains per block), then the accumulator in two halves.
+        // Several offset blocks: the correction was computed during the main loop.
         const float sa = Sa[rl];
-        const float* orow = Os + rl * kStageGp;
-        for (int c2 = 0; c2 < kEpiCols / 32; ++c2) {
-          const int jc = half * kEpiCols + c2 * 32;  // column within the staged tile
-          float y[32];
-          {
-            const float ob = orow[0];
-            const float4* r4 = reinterpret_cast<const float4*>(Rs + jc);
+        const uint32_t corr_tm = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + kCorrCol0;
+        const uint32_t corr_s = base + SL::kOffOut + rl * kCorrPitch;
+        for (int c = 0; c < kEpiCols / CW; ++c) {
+          const int jc = half * kEpiCols + c * CW;  // column within the tile
+          uint32_t acc[CW], cr[CW];
+          tmem_ld_16cols(acc_tm + c * CW, acc);
+          if (jc < kCorrTmemCols) tmem_ld_16cols(corr_tm + jc, cr);
+          tmem_ld_wait();
+          const int nb = n0 + c * CW;
+          if (!row_ok || nb >= p.N) continue;
+          if (jc >= kCorrTmemCols) {
+            const uint32_t a = corr_s + (jc - kCorrTmemCols) * 4;
 #pragma unroll
-            for (int q4 = 0; q4 < 8; ++q4) {
-              const float4 rv = r4[q4];
-              y[4 * q4] = ob * rv.x; y[4 * q4 + 1] = ob * rv.y; y[4 * q4 + 2] = ob * rv.z; y[4 * q4 + 3] = ob * rv.w;
+            for (int q4 = 0; q4 < CW / 4; ++q4) {
+              const uint4 v = lds128(a + 16 * q4);
+              cr[4 * q4] = v.x; cr[4 * q4 + 1] = v.y; cr[4 * q4 + 2] = v.z; cr[4 * q4 + 3] = v.w;
             }
           }
-#pragma unroll 2
-          for (int b = 1; b < G; ++b) {
-            const float ob = orow[b];
-            const float4* r4 = reinterpret_cast<const float4*>(Rs + b * BN + jc);
+          const int nvalid = p.N - nb < CW ? p.N - nb : CW;
+          float z[CW];
 #pragma unroll
-            for (int q4 = 0; q4 < 8; ++q4) {
-              const float4 rv = r4[q4];
-              y[4 * q4] = fmaf(ob, rv.x, y[4 * q4]);
-              y[4 * q4 + 1] = fmaf(ob, rv.y, y[4 * q4 + 1]);
-              y[4 * q4 + 2] = fmaf(ob, rv.z, y[4 * q4 + 2]);
-              y[4 * q4 + 3] = fmaf(ob, rv.w, y[4 * q4 + 3]);
-            }
+          for (int jj = 0; jj < CW; ++jj) {
+            const float accf = __uint_as_float(acc[jj]) * 262144.0f;  // exact: * 2^18
+            z[jj] = Ws[jc + jj] * fmaf(sa, accf, __uint_as_float(cr[jj]));
           }
+          store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, z, nvalid);
+          if (p.acc_debug != nullptr) {
+            int32_t* d = p.acc_debug + static_cast<int64_t>(t) * p.N + nb;
 #pragma unroll
-          for (int hh = 0; hh < 2; ++hh) {
-            uint32_t acc[CW];
-            tmem_ld_16cols(acc_tm + c2 * 32 + hh * CW, acc);
-            tmem_ld_wait();
-            const int nb = n0 + c2 * 32 + hh * CW;
-            if (!row_ok || nb >= p.N) continue;
-            const int nvalid = p.N - nb < CW ? p.N - nb : CW;
-            float z[CW];
-#pragma unroll
-            for (int jj = 0; jj < CW; ++jj) {
-              const float accf = __uint_as_float(acc[jj]) * 262144.0f;  // exact: * 2^18
-              z[jj] = Ws[jc + hh * CW + jj] * fmaf(sa, accf, y[hh * CW + jj]);
-            }
-            store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, z, nvalid);
-            if (p.acc_debug != nullptr) {
-              int32_t* d = p.acc_debug + static_cast<int64_t>(t) * p.N + nb;
-#pragma unroll
-              for (int jj = 0; jj < CW; ++jj)
-                if (jj < nvalid) d[jj] = __float2int_rn(__uint_as_float(acc[jj]) * 262144.0f);
-            }
+            for (int jj = 0; jj < CW; ++jj)
+              if (jj < nvalid) d[jj] = __float2int_rn(__uint_as_float(acc[jj]) * 262144.0f);
           }
         }
       } else if (kOneBlock) {
@@ -745,7 +811,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1) w4a4_ge
       tc_fence_before();
       __syncwarp();
       if (ok && lane == 0) arrive_cluster(acc_empty_l);
-      epi_sync();  // the staged constants are reused for the next tile
+      epi_sync<kEpiWarps>();  // the staged constants are reused for the next tile
       if (*epi_stop) break;
     }
     if (kOneBlock) bulk_wait_all();  // output rows in flight are written before the CTA ends
@@ -781,6 +847,7 @@ int num_sms() {
 template <int OUT, bool kOneBlock>
 int launch_gemm(const GemmParams& p, cudaStream_t s) {
   auto kern = w4a4_gemm_kernel<OUT, kOneBlock>;
+  constexpr int kThreads = Roles<kOneBlock>::kThreads;
   constexpr int kSmemBytes = Smem<kOneBlock>::kBytes;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
