@@ -29,6 +29,8 @@ it implements. Where the paper is silent, it uses these readings:
 * Packing of activation codes: Eq. 1's unsigned form with zero-point 8 (nibble
   q + 8), two per byte, even channel low. Weight codes: sign-magnitude nibbles
   interleaved per 8 channels (layout in :func:`pack_weight_codes`).
+* The per-group asymmetric activation path (the paper's evaluated setting)
+  has its own readings, listed with :func:`quantize_groups_asym`.
 
 Decisions that turn floating point into integers (the codes) are taken here in
 float64.
@@ -369,6 +371,129 @@ def kv4_quantize(kv: np.ndarray, rotate: bool = True, offset: bool = True) -> Di
     return {"q": res["q"].reshape(T, H, hd), "scale": res["scale"].reshape(T, H),
             "offset": res["offset"].reshape(T, H), "codes": res["codes"].reshape(T, H, hd // 2),
             "residual": res["residual"].reshape(T, H, hd)}
+
+
+# ---------------------------------------------------------------------------
+# Per-group asymmetric activations  (Sec. 3 Eq. 1 with its zero-point; Sec. 3.2
+# footnote at Eq. 5; Sec. 4 settings: groups of 128 activations)
+# ---------------------------------------------------------------------------
+#
+# The paper's evaluated activation quantizer. Eq. 1 with the zero-point z is
+# applied to every group of GROUP consecutive channels of a (rotated) token
+# row. After the Hadamard rotation the outlier is a constant offset over a
+# whole block (Eq. 5); a zero-point absorbs it because the grid need not hold
+# 0 (Sec. 3.2 footnote), so this path keeps no explicit offset. Readings:
+#
+# * s = (max - min) / 15 over the group (the 2^b - 1 steps of Eq. 1's range
+#   [0, 2^b - 1] span the group's range); z = -rne(min / s), any integer
+#   (0 need not lie in the range); q = clamp(rne(y / s) + z, 0, 15).
+# * A constant group (max == min) gets s = 0, z = 0 and q = 0.
+# * Storage: s and z in float32 (z integer-valued); the paper's 16-bit storage
+#   (Sec. 3.4) is an accounting choice left out here.
+# * Codes: the unsigned 4-bit q is the nibble itself, two per byte, even
+#   channel low (the layout of :func:`pack_act_codes`).
+# * Weights: the per-channel symmetric codes of :func:`prepare_weight` (Sec. 4
+#   settings), with integer row sums per activation group.
+
+GROUP = 128  # activation group size of the evaluated setting (Sec. 4)
+UMAX = 15    # largest code of Eq. 1's unsigned grid for b = 4
+
+
+def quantize_groups_asym(y: np.ndarray, group: int):
+    """Eq. 1 with a zero-point for every group of ``group`` channels of each row.
+
+    Returns q (int64 [T, K], in [0, 15]), s (float64 [T, K/group]) and z
+    (float64, integer-valued, [T, K/group]).
+    """
+    y = np.asarray(y, dtype=np.float64)
+    T, K = y.shape
+    if K % group != 0:
+        raise ValueError("group must divide K")
+    yg = y.reshape(T, K // group, group)
+    mn, mx = yg.min(axis=2), yg.max(axis=2)
+    s = (mx - mn) / UMAX
+    z = np.zeros_like(s)
+    q = np.zeros(yg.shape, dtype=np.int64)
+    nz = s > 0
+    z[nz] = -np.rint(mn[nz] / s[nz])
+    q[nz] = np.clip(np.rint(yg[nz] / s[nz][:, None]) + z[nz][:, None], 0, UMAX).astype(np.int64)
+    return q.reshape(T, K), s, z
+
+
+def pack_unsigned_codes(q: np.ndarray) -> np.ndarray:
+    """Unsigned codes in [0, 15] -> nibbles, two per byte, even channel low."""
+    q = np.asarray(q, dtype=np.int64)
+    if np.any((q < 0) | (q > UMAX)):
+        raise ValueError("code out of range")
+    if q.shape[-1] % 2:
+        raise ValueError("K must be even")
+    u = q.astype(np.uint8)
+    return (u[..., 0::2] | (u[..., 1::2] << 4)).astype(np.uint8)
+
+
+def quantize_act_group(x: np.ndarray, g: int, group: int = GROUP, rotate: bool = True) -> Dict[str, np.ndarray]:
+    """Rotate -> per-group asymmetric quantize -> pack one batch of token rows X [T, K].
+
+    Steps, in the paper's order:
+      1. Y = X H / sqrt(g) block-wise when ``rotate`` (Eq. 4); else Y = X.
+      2. Per group of ``group`` channels: s, z, q of Eq. 1 (readings above).
+      3. Two codes per byte.
+
+    As in :func:`quantize_act`, the codes are taken from the unnormalised
+    product X H (y / s is the same ratio), so the decisions see no 1/sqrt(g)
+    rounding.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    T, K = x.shape
+    if K % g != 0 or K % group != 0:
+        raise ValueError("g and group must divide K")
+    if rotate:
+        H = _hadamard_f64(g)
+        yu = np.empty_like(x)
+        for b in range(K // g):
+            sl = slice(b * g, (b + 1) * g)
+            yu[:, sl] = x[:, sl] @ H
+        norm = math.sqrt(g)
+    else:
+        yu = x.copy()
+        norm = 1.0
+    q, su, z = quantize_groups_asym(yu, group)
+    return {"y": yu / norm, "q": q, "scale": su / norm, "zero": z, "codes": pack_unsigned_codes(q)}
+
+
+def dequantize_act_group(q: np.ndarray, s: np.ndarray, z: np.ndarray, group: int) -> np.ndarray:
+    """X_hat[t, k] = s[t, k // group] * (q[t, k] - z[t, k // group]) (Eq. 1 inverted)."""
+    T, K = q.shape
+    qg = np.asarray(q, np.float64).reshape(T, K // group, group)
+    return (np.asarray(s, np.float64)[:, :, None] * (qg - np.asarray(z, np.float64)[:, :, None])).reshape(T, K)
+
+
+def weight_group_sums(qw: np.ndarray, group: int) -> np.ndarray:
+    """R[j, n] = sum_{k in group j} Qw[n, k]: integer row sums per activation group."""
+    qw = np.asarray(qw, dtype=np.int64)
+    N, K = qw.shape
+    return qw.reshape(N, K // group, group).sum(axis=2).T
+
+
+def w4a4_linear_group(q: np.ndarray, s: np.ndarray, z: np.ndarray, qw: np.ndarray, s_w: np.ndarray,
+                      R: np.ndarray, group: int) -> Dict[str, np.ndarray]:
+    """y[t, n] = s_w[n] sum_j s[t, j] (P_j[t, n] - z[t, j] R[j, n]), in float64.
+
+    P_j = sum_{k in group j} q[t, k] Qw[n, k] is each group's exact integer
+    product; subtracting z R removes the zero-point (Eq. 1 inverted), and the
+    per-group scale leaves the sum over groups as floating point.
+    """
+    q = np.asarray(q, np.int64)
+    qw = np.asarray(qw, np.int64)
+    T, K = q.shape
+    G = K // group
+    P = np.stack([int_gemm(q[:, j * group:(j + 1) * group], qw[:, j * group:(j + 1) * group]) for j in range(G)])
+    s = np.asarray(s, np.float64)
+    z = np.asarray(z, np.float64)
+    acc = np.zeros((T, qw.shape[0]))
+    for j in range(G):
+        acc += s[:, j, None] * (P[j].astype(np.float64) - z[:, j, None] * np.asarray(R, np.float64)[j][None, :])
+    return {"P": P, "y": np.asarray(s_w, np.float64)[None, :] * acc}
 
 
 # ---------------------------------------------------------------------------

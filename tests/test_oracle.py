@@ -341,3 +341,136 @@ def test_storage_bits_golden(golden_dir):
     assert O.effective_bits(d["group"], d["code_bits"], d["param_bits"], d["n_params"]) == d["bits"]
     # This path: one fp32 scale per token + one fp32 offset per block.
     assert O.effective_bits_per_token_offset(4096, 4096) == pytest.approx(4 + 64 / 4096)
+
+
+# --------------------------------------------------------------------------
+# Per-group asymmetric activations (Eq. 1 with z; Sec. 3.2 footnote; Sec. 4:
+# groups of 128). Readings: s = (max - min) / 15, z = -rne(min / s),
+# q = clamp(rne(y / s) + z, 0, 15); a constant group has s = z = q = 0.
+# --------------------------------------------------------------------------
+
+def test_group_affine_grid_is_exact():
+    """A group whose values sit on s0 * (j - z0), j covering 0..15, comes back
+    exactly: s = s0, z = z0, q = j (powers of two keep every division exact)."""
+    rng = np.random.default_rng(40)
+    for trial in range(50):
+        group = 16 * int(rng.integers(1, 5))
+        s0 = 2.0 ** int(rng.integers(-6, 4))
+        z0 = int(rng.integers(-40, 40))
+        j = rng.integers(0, 16, size=group)
+        j[rng.integers(0, group)] = 0
+        j[(rng.integers(1, group) + 3) % group] = 15
+        if j.min() != 0 or j.max() != 15:
+            j[0], j[1] = 0, 15
+        y = s0 * (j - z0).astype(np.float64)
+        q, s, z = O.quantize_groups_asym(y[None, :], group)
+        assert s[0, 0] == s0 and z[0, 0] == z0
+        np.testing.assert_array_equal(q[0], j)
+        np.testing.assert_array_equal(O.dequantize_act_group(q, s, z, group)[0], y)
+
+
+def test_group_eq5_two_channel_example(golden_dir):
+    """Eq. 5's two-channel token: after H/sqrt(2) the outlier x1 is a common
+    offset, so with one group of 2 the step is 2|x2| / (15 sqrt 2) whatever x1
+    is, and the two channels take the ends of the grid."""
+    d = _load(golden_dir, "eq5_two_channel.json")
+    for case in d["cases"]:
+        x = np.array([case["x"]], dtype=np.float64)
+        res = O.quantize_act_group(x, 2, group=2, rotate=True)
+        x2 = case["x"][1]
+        np.testing.assert_allclose(res["y"][0], case["y"], rtol=1e-14)
+        np.testing.assert_allclose(res["scale"][0, 0], 2 * abs(x2) / (15 * math.sqrt(2)), rtol=1e-12)
+        # x2 = 0 leaves a constant group: s = z = q = 0 (the reading).
+        expect = [15, 0] if x2 > 0 else [0, 15] if x2 < 0 else [0, 0]
+        np.testing.assert_array_equal(res["q"][0], expect)
+
+
+def test_group_rotation_absorbs_outlier():
+    """A channel-0 outlier adds the same constant to every rotated channel of
+    its block (Eq. 5): the group scales do not move, unlike the symmetric
+    per-token scale, and the reconstruction stays within s / 2."""
+    rng = np.random.default_rng(41)
+    K, group = 512, 128
+    base = rng.standard_normal((16, K))
+    spiked = base.copy()
+    spiked[:, 0] += rng.uniform(400, 2000, size=16)
+    a = O.quantize_act_group(base, K, group, rotate=True)
+    b = O.quantize_act_group(spiked, K, group, rotate=True)
+    np.testing.assert_allclose(b["scale"], a["scale"], rtol=1e-9)
+    err = np.abs(O.dequantize_act_group(b["q"], b["scale"], b["zero"], group) - b["y"])
+    assert np.all(err <= np.repeat(b["scale"], group, axis=1) * (0.5 + 1e-9))
+    sym = O.quantize_act(spiked, K, rotate=True, offset=False)
+    assert np.all(sym["scale"] > 5 * b["scale"].max(axis=1))
+
+
+def test_group_error_bound_and_ends():
+    rng = np.random.default_rng(42)
+    x = rng.standard_normal((32, 512)) * rng.uniform(0.01, 30, size=(32, 1)) + rng.uniform(-5, 5, size=(32, 1))
+    for rotate in (False, True):
+        res = O.quantize_act_group(x, 256, 128, rotate=rotate)
+        q, s, z = res["q"], res["scale"], res["zero"]
+        sg = np.repeat(s, 128, axis=1)
+        err = np.abs(O.dequantize_act_group(q, s, z, 128) - res["y"])
+        clamped = (q == 15) & (np.rint(res["y"] / sg) + np.repeat(z, 128, axis=1) > 15)
+        assert np.all(err[~clamped] <= sg[~clamped] * (0.5 + 1e-9))
+        assert np.all(err <= sg * (1 + 1e-9))
+        yg = res["y"].reshape(32, 4, 128)
+        qg = q.reshape(32, 4, 128)
+        # The group minimum always lands on code 0; the maximum on 15 (14 only
+        # when both ends sit on rounding ties of opposite parity).
+        at_min = np.take_along_axis(qg, yg.argmin(axis=2)[..., None], axis=2)
+        at_max = np.take_along_axis(qg, yg.argmax(axis=2)[..., None], axis=2)
+        assert np.all(at_min == 0) and np.all(at_max >= 14)
+
+
+def test_group_brute_force_small_groups():
+    """Group of 4: each code is the index of the nearest point of the grid
+    s (j - z), j = 0..15, ties to an even j - z."""
+    rng = np.random.default_rng(43)
+    j = np.arange(16)
+    for trial in range(300):
+        y = rng.standard_normal((1, 4)) * rng.uniform(0.01, 50) + rng.uniform(-20, 20)
+        q, s, z = O.quantize_groups_asym(y, 4)
+        for k in range(4):
+            d = np.abs(y[0, k] - s[0, 0] * (j - z[0, 0]))
+            best = j[d <= d.min() + 1e-12 * s[0, 0]]
+            expect = best[0] if len(best) == 1 else best[(best - int(z[0, 0])) % 2 == 0][0]
+            assert q[0, k] == expect
+
+
+def test_group_constant_and_zero_groups():
+    y = np.zeros((2, 256))
+    y[1, 128:] = 3.25
+    q, s, z = O.quantize_groups_asym(y, 128)
+    assert np.all(s == 0) and np.all(z == 0) and np.all(q == 0)
+
+
+def test_group_pack_roundtrip():
+    rng = np.random.default_rng(44)
+    q = rng.integers(0, 16, size=(3, 64))
+    packed = O.pack_unsigned_codes(q)
+    assert packed[0, 0] == (q[0, 0] | (q[0, 1] << 4))
+    np.testing.assert_array_equal(O.unpack_act_codes(packed) + 8, q)
+
+
+@pytest.mark.parametrize("rotate", [False, True])
+def test_group_gemm_equals_dequantized_product(rotate):
+    """s_w sum_j s_j (P_j - z_j R_j) is the product of the dequantized
+    activations and weights, formed here by a plain float64 matmul."""
+    rng = np.random.default_rng(45)
+    T, K, N, g = 9, 512, 24, 256
+    x = W.activations(T, K, seed=46, n_out=2, mult=80.0)
+    w = rng.standard_normal((N, K)) * 0.02
+    a = O.quantize_act_group(x, g, 128, rotate=rotate)
+    wp = O.prepare_weight(w, g, rotate=rotate)
+    R = O.weight_group_sums(wp["q"], 128)
+    res = O.w4a4_linear_group(a["q"], a["scale"], a["zero"], wp["q"], wp["scale"], R, 128)
+    xh = O.dequantize_act_group(a["q"], a["scale"], a["zero"], 128)
+    wh = wp["q"] * wp["scale"][:, None]
+    ref = xh @ wh.T
+    np.testing.assert_allclose(res["y"], ref, rtol=1e-11, atol=1e-12 * np.abs(ref).max())
+    # Each group's integer product, by the triple loop on a corner.
+    np.testing.assert_array_equal(res["P"][1][:3, :4], O.int_gemm_loops(a["q"][:3, 128:256], wp["q"][:4, 128:256]))
+    # And the group layer approximates the unquantized one.
+    y32 = O.linear_reference(x, w)
+    assert np.linalg.norm(res["y"] - y32) < 0.3 * np.linalg.norm(y32)
