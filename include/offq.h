@@ -13,6 +13,12 @@
  *   offq_kv4_quantize   per-(token, head) version of the quantizer (KV cache)
  *   offq_prepare_weight offline: rotated, per-channel 4-bit weights + tables
  *
+ * and the paper's evaluated per-group asymmetric variant of the first two:
+ *
+ *   offq_quantize_act_group  rotation -> groups of 128 with zero-points -> codes
+ *   offq_weight_group_sums   offline: weight row sums per activation group
+ *   offq_w4a4_linear_group   GEMM with per-group scales and zero-points
+ *
  * Conventions shared by every call
  *   - Pointers named as device buffers are device pointers allocated and owned
  *     by the caller. The library never allocates, frees, or synchronizes the
@@ -188,6 +194,78 @@ int offq_kv4_quantize(const void* kv, int dtype, int64_t T, int32_t H, int32_t h
  */
 int offq_prepare_weight(const void* w, int dtype, int64_t N, int64_t K, int32_t g, int32_t rotate,
                         uint8_t* w_codes, float* w_scale, float* w_offsum, void* stream);
+
+/*
+ * Per-group asymmetric path -- the paper's evaluated activation setting
+ * (Sec. 4 "Implementation and Settings": activations quantized per group of
+ * 128 channels, asymmetrically; Sec. 3 Eq. 1 with its zero-point z). After
+ * the Hadamard rotation the outlier is a constant offset over a block
+ * (Eq. 5), which each group's zero-point absorbs (Sec. 3.2 footnote: the grid
+ * need not hold 0), so this path stores no explicit offset.
+ *
+ * offq_quantize_act_group -- for each token row x (K channels):
+ *   y = x_b H_g / sqrt(g) per block b of g channels   if OFFQ_ROTATE (else y = x)
+ * then for each group j of `group` channels of y:
+ *   s[j] = (max - min) / 15,  z[j] = -round_half_even(min / s[j])  (any integer),
+ *   u = clamp(round_half_even(y / s[j]) + z[j], 0, 15);
+ * a constant group gets s = z = u = 0. y ~ s (u - z).
+ *
+ *   x       device, [T][ldx] elements of x_dtype, row-major; 16-byte aligned,
+ *           ldx * sizeof(elem) a multiple of 16, ldx >= K.
+ *   T       token rows, >= 0 (T = 0 launches nothing).
+ *   K       channels, a multiple of `group` (and of g with the rotation),
+ *           K <= 65536.
+ *   g       rotation block (power of two in [32, 8192]; this build rotates
+ *           blocks of at most 512 and returns OFFQ_ERR_UNSUPPORTED above);
+ *           ignored without OFFQ_ROTATE.
+ *   group   channels per quantization group; this build supports 128
+ *           (OFFQ_ERR_UNSUPPORTED for other positive values).
+ *   flags   0 or OFFQ_ROTATE.
+ *   codes   device, offq_act_codes_bytes(T, K) bytes: u as the nibble, two per
+ *           byte (even channel low), in the tiled operand layout, 16-B aligned
+ *           (rows beyond T in the last 32-row group are left as they are).
+ *   scale   device, [T][K/group] float32.
+ *   zero    device, [T][K/group] float32 (integer-valued).
+ */
+int offq_quantize_act_group(const void* x, int x_dtype, int64_t T, int64_t K, int64_t ldx,
+                            int32_t g, int32_t group, int32_t flags,
+                            uint8_t* codes, float* scale, float* zero, void* stream);
+
+/*
+ * offq_weight_group_sums -- offline: R[j][n] = sum_{k in group j} q_w[n][k],
+ * the integer row sums of prepared weight codes (offq_prepare_weight) over
+ * each activation group, stored as float32. They carry the zero-point term
+ * of the per-group GEMM.
+ *
+ *   w_codes     device, tiled weight codes of N rows (offq_prepare_weight), 16-B aligned.
+ *   N, K        output and input channels (K a multiple of 32 and of group).
+ *   group       power of two >= 32 dividing K.
+ *   w_groupsum  device, [K/group][N] float32.
+ */
+int offq_weight_group_sums(const uint8_t* w_codes, int64_t N, int64_t K, int32_t group,
+                           float* w_groupsum, void* stream);
+
+/*
+ * offq_w4a4_linear_group -- W4A4 GEMM of the per-group path:
+ *   y[t][n] = s_w[n] * sum_j s[t][j] * (P_j[t][n] - z[t][j] * R[j][n]),
+ *   P_j[t][n] = sum_{k in group j} u[t][k] * q_w[n][k]   (exact integers),
+ * i.e. y = X_hat W_hat^T with X_hat = s (u - z) and W_hat = s_w q_w. Each
+ * group's product is exact on the tensor cores; the per-group scaling and the
+ * zero-point term are fp32 multiply-adds in group order, rounded once to the
+ * output type.
+ *
+ *   a_codes, a_scale, a_zero  from offq_quantize_act_group (T rows, K channels).
+ *   T, N, K     T >= 0, N >= 1, K a multiple of group, K <= 65536.
+ *   group       128 in this build (OFFQ_ERR_UNSUPPORTED otherwise).
+ *   w_codes, w_scale          from offq_prepare_weight (any rotation block).
+ *   w_groupsum  from offq_weight_group_sums with the same group.
+ *   out         device, [T][ldo] of out_dtype, ldo >= N, 16-byte aligned with
+ *               ldo * sizeof(out) a multiple of 16.
+ */
+int offq_w4a4_linear_group(const uint8_t* a_codes, const float* a_scale, const float* a_zero,
+                           int64_t T, int64_t N, int64_t K, int32_t group,
+                           const uint8_t* w_codes, const float* w_scale, const float* w_groupsum,
+                           void* out, int out_dtype, int64_t ldo, void* stream);
 
 /* Bytes of a tiled activation-code buffer for T rows of K codes (-1 if K is
  * not a positive multiple of 32 or T < 0): ceil(T/32) * 32 * K / 2. */

@@ -1,0 +1,452 @@
+// W4A4 GEMM with per-group activation scales and zero-points
+// (offq_w4a4_linear_group): the paper's evaluated activation setting, groups
+// of 128 channels quantized asymmetrically (Sec. 3 Eq. 1 with its zero-point,
+// Sec. 4 settings), against per-channel symmetric 4-bit weights.
+//
+//   y[t][n] = s_w[n] * sum_j s[t][j] * (P_j[t][n] - z[t][j] * R[j][n])
+//   P_j[t][n] = sum_{k in group j} u[t][k] * q_w[n][k]
+//
+// u in [0, 15] is the stored code (Eq. 1's x_q), q_w in [-7, 7], and R[j][n]
+// the integer row sum of the weight codes over group j. Both codes widen to
+// exact E4M3 operands (bytes 0x00..0x0F are 0..15 * 2^-9), so P_j, an integer
+// times 2^-18 below 2^24 * 2^-18, is exact in the fp32 accumulator.
+//
+// One 128-code k-tile is one group, so the per-(token, group) scale cannot sit
+// in the operands: the pair MMA (M 256, N 128) writes each group's P_j into one
+// of two TMEM partial buffers, and four scaler warps fold it into a running
+// fp32 sum,
+//   d = fma(-z, R, P)   (exact while |z R| < 2^24),   S = fma(s, d, S),
+// (on the accumulator's P * 2^-18, with -z * 2^-18 and s * 2^18),
+// while the MMA fills the other buffer. After a tile's last group the scalers
+// multiply by s_w and store y, rounding once to the output type.
+//
+// TMEM (512 columns per CTA): P0 [0, 128), P1 [128, 256), running sum
+// [256, 384), 4 A stages of 32 columns [384, 512). The N = 128 pair tile is
+// what lets the running sum and both partials fit next to the A stages.
+//
+// Warp roles per CTA (17 warps):
+//   warp 0       TMEM allocation; in the leader CTA, lane 0 issues the MMAs
+//   warps 1-8    A converters: two per 32-lane TMEM quarter, alternating k-tiles
+//   warps 9-12   B converters: two per 32-row group (64 rows of B per CTA)
+//   warps 13-16  scalers and epilogue, one per TMEM quarter (128 columns)
+// Every wait is bounded; a wait that runs out aborts the CTA and records
+// OFFQ_ERR_TIMEOUT in the device status word.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include <mutex>
+
+#include "offq.h"
+#include "offq_device.cuh"
+#include "offq_host.h"
+#include "pair_common.cuh"
+
+namespace {
+
+using namespace offq;
+
+constexpr int GBM = 128;         // rows of A per CTA (256 per pair)
+constexpr int GBN = 128;         // output channels per pair tile
+constexpr int GBNH = GBN / 2;    // rows of B held by one CTA
+constexpr int GBK = 128;         // codes per k-tile = one activation group
+constexpr int kGroup = GBK;
+constexpr int kGChunks = GBK / 32;  // 16-byte packed chunks per row per k-tile
+constexpr int kGStages = 4;
+constexpr int kGSplit = 2;          // converter warps per row group, alternating k-tiles
+constexpr int kGAWarps = 4 * kGSplit;
+constexpr int kGBWarps = (GBNH / 32) * kGSplit;
+constexpr int kGScWarps = 4;
+constexpr int kGFirstA = 1, kGFirstB = kGFirstA + kGAWarps, kGFirstSc = kGFirstB + kGBWarps;
+constexpr int kGThreads = (kGFirstSc + kGScWarps) * 32;
+constexpr int kGArrivals = 4 + GBNH / 32;  // per stage and CTA: one per A quarter and per B row group
+constexpr int kPCol0 = 0;                  // two partial buffers of GBN columns
+constexpr int kSCol0 = 2 * GBN;            // running sum
+constexpr int kGACol0 = 3 * GBN;           // A stages
+constexpr int kGAColsPerStage = GBK / 4;
+constexpr int kGTmemCols = 512;
+static_assert(kGACol0 + kGStages * kGAColsPerStage <= kGTmemCols, "TMEM budget");
+constexpr int kGBStage = GBNH * GBK;  // 8 KB of E4M3 per stage
+constexpr uint32_t kGIdesc = idesc_e4m3_f32(2 * GBM, GBN);  // pair MMA: M = 256, N = 128
+
+// Shared memory: B stages, barriers (full/empty per stage, partial full/empty
+// per buffer), misc. The request is padded so that one CTA holds an SM: the
+// pair allocates all 512 TMEM columns.
+constexpr int kGOffBars = kGStages * kGBStage;
+constexpr int kGNumBars = 2 * kGStages + 4;
+constexpr int kGOffMisc = kGOffBars + kGNumBars * 8;
+constexpr int kGUsed = kGOffMisc + 64 + 1024;
+constexpr int kGBytes = kGUsed < 120 * 1024 ? 120 * 1024 : kGUsed;
+
+struct GroupParams {
+  const uint8_t* a_codes;  // tiled [ceil(T/32)*32][K/2], unsigned codes
+  const uint8_t* w_codes;  // tiled [ceil(N/32)*32][K/2]
+  const float* a_scale;    // [T][Gq]
+  const float* a_zero;     // [T][Gq]
+  const float* w_scale;    // [N]
+  const float* gsum;       // [Gq][N]
+  void* out;
+  int64_t ldo;
+  int* status;
+  int T, N, K, Gq;
+  int m_pairs, n_tiles;
+  int t_blocks, n_blocks;
+  int kchunks;  // K / 32
+  int vec;      // N % 4 == 0 and gsum, w_scale 16-byte aligned
+};
+
+__device__ __forceinline__ void load_group_kt(const uint8_t* blk, int kchunks, int kt, uint4 (&v)[kGChunks]) {
+#pragma unroll
+  for (int j = 0; j < kGChunks; ++j) {
+    const int c = kt * kGChunks + j;
+    if (blk != nullptr && c < kchunks)
+      v[j] = ldg_stream(blk + c * 512);
+    else
+      v[j] = make_uint4(0u, 0u, 0u, 0u);
+  }
+}
+
+// Four consecutive entries of a [.][N] float row from column n (zeros past N).
+__device__ __forceinline__ float4 ldg_cols4(const float* row, int n, int N, bool vec) {
+  if (vec) return n < N ? __ldg(reinterpret_cast<const float4*>(row + n)) : make_float4(0.f, 0.f, 0.f, 0.f);
+  float4 r;
+  r.x = n < N ? __ldg(row + n) : 0.f;
+  r.y = n + 1 < N ? __ldg(row + n + 1) : 0.f;
+  r.z = n + 2 < N ? __ldg(row + n + 2) : 0.f;
+  r.w = n + 3 < N ? __ldg(row + n + 3) : 0.f;
+  return r;
+}
+
+// Persistent pair kernel over pair tiles (m_pair * n_tiles + n_tile), cluster c
+// taking tiles c, c + clusters, ... The global k-tile counter j runs across
+// tiles: operand stage j mod 4, partial buffer j mod 2.
+template <int OUT>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGThreads, 1)
+    w4a4_group_gemm_kernel(const GroupParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (base - raw);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const int cluster = blockIdx.x >> 1;
+  const int clusters = gridDim.x >> 1;
+  const int nk = p.Gq;
+  const int num_tiles = p.m_pairs * p.n_tiles;
+
+  const uint32_t bar0 = base + kGOffBars;
+  auto full = [&](int s) { return bar0 + 8u * s; };                  // leader: operands of stage s ready
+  auto empty = [&](int s) { return bar0 + 8u * (kGStages + s); };    // both: stage s consumed
+  auto pfull = [&](int b) { return bar0 + 8u * (2 * kGStages + b); };      // both: partial b written
+  auto pempty = [&](int b) { return bar0 + 8u * (2 * kGStages + 2 + b); }; // leader: partial b read
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kGOffMisc);
+  volatile int* abort = reinterpret_cast<volatile int*>(smem + kGOffMisc + 16);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kGStages; ++s) {
+      mbar_init(full(s), 2 * kGArrivals);
+      mbar_init(empty(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(pfull(b), 1);
+      mbar_init(pempty(b), 2 * kGScWarps);
+    }
+    *abort = 0;
+    mbar_fence_init();
+  }
+  if (warp == 0) {
+    tmem_alloc2(smem_u32(tmem_slot), kGTmemCols);
+    tmem_relinquish2();
+  }
+  tc_fence_before();
+  cluster_sync();  // barriers initialised and TMEM allocated in both CTAs
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  griddep_wait();
+  griddep_launch_dependents();
+  uint32_t mma_groups = 0;
+
+  if (warp == 0) {
+    // ---------------- MMA issuer (leader CTA) ----------------
+    if (rank == 0 && lane == 0) {
+      int s = 0, phase = 0;
+      uint32_t j = 0;
+      for (int tile = cluster; tile < num_tiles && !*abort; tile += clusters) {
+        bool ok = true;
+        for (int kt = 0; kt < nk; ++kt, ++j) {
+          const uint32_t b = j & 1u, use = j >> 1;
+          if (!wait_cluster(pempty(b), (use & 1u) ^ 1u, abort) || !wait_cluster(full(s), phase, abort)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t b_addr = base + s * kGBStage;
+#pragma unroll
+          for (int kk = 0; kk < GBK / 32; ++kk)
+            mma2_ts(tmem + kPCol0 + b * GBN, tmem + kGACol0 + s * kGAColsPerStage + 8 * kk,
+                    smem_desc_sw128(b_addr + 32 * kk), kGIdesc, kk != 0 ? 1u : 0u);
+          mma2_commit_both(empty(s));
+          mma2_commit_both(pfull(b));
+          mma_groups = j + 1;
+          if (++s == kGStages) {
+            s = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+      }
+    }
+  } else if (warp < kGFirstSc) {
+    // ---------------- converters: packed codes -> E4M3 operands ----------------
+    const bool is_a = warp < kGFirstB;
+    const int quarter = warp & 3;
+    const int wb = (warp - kGFirstB) & 1;
+    const int part = is_a ? (warp - kGFirstA) >> 2 : (warp - kGFirstB) >> 1;  // k-tiles g == part mod 2
+    const uint32_t full_l = leader_addr(full(0));
+    const uint8_t* codes = is_a ? p.a_codes : p.w_codes;
+    const int rb_count = is_a ? p.t_blocks : p.n_blocks;
+    auto block_ptr = [&](int tile) -> const uint8_t* {
+      const int rb = is_a ? ((tile / p.n_tiles) * 2 * GBM + static_cast<int>(rank) * GBM + quarter * 32) >> 5
+                          : ((tile % p.n_tiles) * GBN + static_cast<int>(rank) * GBNH + wb * 32) >> 5;
+      return rb < rb_count ? codes + static_cast<int64_t>(rb) * p.kchunks * 512 + lane * 16 : nullptr;
+    };
+    auto advance1 = [&](int& tile, int& kt) {
+      if (++kt == nk) {
+        kt = 0;
+        tile += clusters;
+      }
+    };
+    int ld_tile = cluster, ld_kt = 0;
+    if (part) advance1(ld_tile, ld_kt);
+    int tile = ld_tile, kt = ld_kt;
+    uint4 ring[kGChunks];
+    int blk_tile = ld_tile;
+    const uint8_t* blk = ld_tile < num_tiles ? block_ptr(ld_tile) : nullptr;
+    if (ld_tile < num_tiles) load_group_kt(blk, p.kchunks, ld_kt, ring);
+    advance1(ld_tile, ld_kt);
+    advance1(ld_tile, ld_kt);
+    int s = part, phase = 0;
+    while (tile < num_tiles) {
+      if (!__all_sync(0xFFFFFFFFu, wait_cluster(empty(s), phase ^ 1, abort))) break;
+      if (is_a) {
+        tc_fence_after();
+        uint32_t f8[32];
+#pragma unroll
+        for (int c = 0; c < kGChunks; ++c) {
+          widen_act(ring[c].x, f8[8 * c + 0], f8[8 * c + 1]);
+          widen_act(ring[c].y, f8[8 * c + 2], f8[8 * c + 3]);
+          widen_act(ring[c].z, f8[8 * c + 4], f8[8 * c + 5]);
+          widen_act(ring[c].w, f8[8 * c + 6], f8[8 * c + 7]);
+        }
+        tmem_st_32cols(tmem + (static_cast<uint32_t>(quarter * 32) << 16) + kGACol0 + s * kGAColsPerStage, f8);
+        tmem_st_wait();
+        tc_fence_before();
+      } else {
+        const int r = wb * 32 + lane;
+        const uint32_t st = base + s * kGBStage + r * 128;
+#pragma unroll
+        for (int c = 0; c < kGChunks; ++c) {
+          uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
+          widen_weight(ring[c].x, a0, a1);
+          widen_weight(ring[c].y, a2, a3);
+          widen_weight(ring[c].z, b0, b1);
+          widen_weight(ring[c].w, b2, b3);
+          sts128(st + (((2 * c) ^ (r & 7)) << 4), a0, a1, a2, a3);
+          sts128(st + (((2 * c + 1) ^ (r & 7)) << 4), b0, b1, b2, b3);
+        }
+        fence_proxy_async_smem();
+      }
+      __syncwarp();
+      if (lane == 0) arrive_cluster(full_l + 8u * s);
+      if (ld_tile < num_tiles) {
+        if (ld_tile != blk_tile) {
+          blk_tile = ld_tile;
+          blk = block_ptr(ld_tile);
+        }
+        load_group_kt(blk, p.kchunks, ld_kt, ring);
+      }
+      advance1(ld_tile, ld_kt);
+      advance1(ld_tile, ld_kt);
+      advance1(tile, kt);
+      advance1(tile, kt);
+      s += kGSplit;
+      if (s >= kGStages) {
+        s -= kGStages;
+        phase ^= 1;
+      }
+    }
+  } else {
+    // ---------------- scalers and epilogue ----------------
+    const int quarter = warp & 3;
+    const int rl = quarter * 32 + lane;  // TMEM lane = row within the CTA
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+    const uint32_t pempty_l = leader_addr(pempty(0));
+    const bool vec = p.vec != 0;
+    uint32_t j = 0;
+    bool ok = true;
+    for (int tile = cluster; tile < num_tiles && ok; tile += clusters) {
+      const int t = (tile / p.n_tiles) * 2 * GBM + static_cast<int>(rank) * GBM + rl;
+      const int n0 = (tile % p.n_tiles) * GBN;
+      const bool row_ok = t < p.T;
+      const float* srow = p.a_scale + static_cast<int64_t>(row_ok ? t : 0) * p.Gq;
+      const float* zrow = p.a_zero + static_cast<int64_t>(row_ok ? t : 0) * p.Gq;
+      for (int kt = 0; kt < nk; ++kt, ++j) {
+        const uint32_t b = j & 1u, use = j >> 1;
+        // The accumulator holds P * 2^-18 (each E4M3 operand carries 2^-9):
+        // d' = P 2^-18 - z R 2^-18 and s 2^18 d' = s (P - z R), all exact scalings.
+        const float sg = row_ok ? __ldg(srow + kt) * 262144.0f : 0.f;
+        const float nz = row_ok ? __ldg(zrow + kt) * -3.814697265625e-06f : 0.f;
+        ok = __all_sync(0xFFFFFFFFu, wait_cluster(pfull(b), use & 1u, abort));
+        if (!ok) break;
+        tc_fence_after();
+        const float* rrow = p.gsum + static_cast<int64_t>(kt) * p.N;
+        const bool last = kt == nk - 1;
+        const uint64_t SG = pack2(sg, sg), NZ = pack2(nz, nz);
+#pragma unroll 1
+        for (int c = 0; c < GBN / 32; ++c) {
+          uint32_t pv[32], sv[32];
+          tmem_ld_32cols(lane_base + kPCol0 + b * GBN + c * 32, pv);
+          if (kt > 0) tmem_ld_32cols(lane_base + kSCol0 + c * 32, sv);
+          tmem_ld_wait();
+          if (c == GBN / 32 - 1) {
+            // The partial is in registers: its buffer may take the group after next.
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) arrive_cluster(pempty_l + 8u * b);
+          }
+          const int nc = n0 + c * 32;
+#pragma unroll
+          for (int q4 = 0; q4 < 8; ++q4) {
+            const float4 r = ldg_cols4(rrow, nc + 4 * q4, p.N, vec);
+            const uint64_t d0 = fma2v(NZ, pack2(r.x, r.y), pack2(__uint_as_float(pv[4 * q4]), __uint_as_float(pv[4 * q4 + 1])));
+            const uint64_t d1 =
+                fma2v(NZ, pack2(r.z, r.w), pack2(__uint_as_float(pv[4 * q4 + 2]), __uint_as_float(pv[4 * q4 + 3])));
+            uint64_t a0, a1;
+            if (kt == 0) {
+              a0 = mul2v(SG, d0);
+              a1 = mul2v(SG, d1);
+            } else {
+              a0 = fma2v(SG, d0, pack2(__uint_as_float(sv[4 * q4]), __uint_as_float(sv[4 * q4 + 1])));
+              a1 = fma2v(SG, d1, pack2(__uint_as_float(sv[4 * q4 + 2]), __uint_as_float(sv[4 * q4 + 3])));
+            }
+            float f0, f1, f2, f3;
+            unpack2(a0, f0, f1);
+            unpack2(a1, f2, f3);
+            sv[4 * q4] = __float_as_uint(f0);
+            sv[4 * q4 + 1] = __float_as_uint(f1);
+            sv[4 * q4 + 2] = __float_as_uint(f2);
+            sv[4 * q4 + 3] = __float_as_uint(f3);
+          }
+          if (!last) {
+            tmem_st_32cols(lane_base + kSCol0 + c * 32, sv);
+          } else if (row_ok && nc < p.N) {
+            float y[32];
+#pragma unroll
+            for (int q4 = 0; q4 < 8; ++q4) {
+              const float4 w = ldg_cols4(p.w_scale, nc + 4 * q4, p.N, vec);
+              y[4 * q4] = w.x * __uint_as_float(sv[4 * q4]);
+              y[4 * q4 + 1] = w.y * __uint_as_float(sv[4 * q4 + 1]);
+              y[4 * q4 + 2] = w.z * __uint_as_float(sv[4 * q4 + 2]);
+              y[4 * q4 + 3] = w.w * __uint_as_float(sv[4 * q4 + 3]);
+            }
+            const int nvalid = p.N - nc < 32 ? p.N - nc : 32;
+            store_out<OUT, 32>(p.out, static_cast<int64_t>(t) * p.ldo + nc, y, nvalid);
+          }
+        }
+        if (!last) tmem_st_wait();  // the running sum is in TMEM before the next group reads it
+      }
+    }
+  }
+
+  // ---------------- teardown ----------------
+  if (*abort && warp == 0 && lane == 0 && rank == 0 && mma_groups > 0) {
+    // Let the MMAs already issued finish before tensor memory is released.
+    const uint32_t last = mma_groups - 1;
+    wait_teardown(pfull(last & 1u), (last >> 1) & 1u);
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc2(tmem, kGTmemCols);
+  }
+  if (threadIdx.x == 0 && *abort && p.status != nullptr) atomicExch(p.status, kErrTimeout);
+}
+
+int group_num_sms() {
+  static int sms[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (sms[dev] == 0) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    sms[dev] = v;
+  }
+  return sms[dev];
+}
+
+template <int OUT>
+int launch_group_gemm(const GroupParams& p, cudaStream_t s) {
+  auto kern = w4a4_group_gemm_kernel<OUT>;
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [&] {
+    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kGBytes);
+  });
+  if (attr_err != cudaSuccess) return OFFQ_ERR_CUDA;
+  const int sms = group_num_sms();
+  if (sms < 2) return OFFQ_ERR_CUDA;
+  const int tiles = p.m_pairs * p.n_tiles;
+  const int clusters = tiles < sms / 2 ? tiles : sms / 2;
+  return launch_pdl(kern, dim3(2 * clusters), dim3(kGThreads), kGBytes, s, p);
+}
+
+}  // namespace
+
+extern "C" int offq_w4a4_linear_group(const uint8_t* a_codes, const float* a_scale, const float* a_zero, int64_t T,
+                                      int64_t N, int64_t K, int32_t group, const uint8_t* w_codes,
+                                      const float* w_scale, const float* w_groupsum, void* out, int out_dtype,
+                                      int64_t ldo, void* stream) {
+  const int ob = elem_bytes(out_dtype);
+  if (ob == 0 || T < 0 || N < 1 || K <= 0 || ldo < N) return OFFQ_ERR_INVALID_ARG;
+  if (group != kGroup) return group > 0 ? OFFQ_ERR_UNSUPPORTED : OFFQ_ERR_INVALID_ARG;
+  if (K % kGroup != 0) return OFFQ_ERR_INVALID_ARG;
+  if (K > kMaxGemmK || T > 0x3FFFFFFF || N > 0x3FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
+  if (T == 0) return OFFQ_OK;
+  if (a_codes == nullptr || a_scale == nullptr || a_zero == nullptr || w_codes == nullptr || w_scale == nullptr ||
+      w_groupsum == nullptr || out == nullptr)
+    return OFFQ_ERR_INVALID_ARG;
+  if (!aligned(a_codes, 16) || !aligned(w_codes, 16) || !aligned(out, 16) || (ldo * ob) % 16 != 0 ||
+      !aligned(a_scale, 4) || !aligned(a_zero, 4) || !aligned(w_scale, 4) || !aligned(w_groupsum, 4))
+    return OFFQ_ERR_MISALIGNED;
+  GroupParams p{};
+  p.a_codes = a_codes;
+  p.w_codes = w_codes;
+  p.a_scale = a_scale;
+  p.a_zero = a_zero;
+  p.w_scale = w_scale;
+  p.gsum = w_groupsum;
+  p.out = out;
+  p.ldo = ldo;
+  p.status = device_status_ptr();
+  p.T = static_cast<int>(T);
+  p.N = static_cast<int>(N);
+  p.K = static_cast<int>(K);
+  p.Gq = static_cast<int>(K / kGroup);
+  p.m_pairs = static_cast<int>((T + 2 * GBM - 1) / (2 * GBM));
+  p.n_tiles = static_cast<int>((N + GBN - 1) / GBN);
+  p.t_blocks = static_cast<int>((T + 31) / 32);
+  p.n_blocks = static_cast<int>((N + 31) / 32);
+  p.kchunks = static_cast<int>(K / 32);
+  p.vec = N % 4 == 0 && aligned(w_groupsum, 16) && aligned(w_scale, 16);
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  switch (out_dtype) {
+    case OFFQ_F32: return launch_group_gemm<OFFQ_F32>(p, s);
+    case OFFQ_BF16: return launch_group_gemm<OFFQ_BF16>(p, s);
+    case OFFQ_F16: return launch_group_gemm<OFFQ_F16>(p, s);
+    default: return OFFQ_ERR_INVALID_ARG;
+  }
+}

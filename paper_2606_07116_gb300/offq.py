@@ -50,6 +50,11 @@ _SIGNATURES = {
     "offq_abi_version": (_c_int, []),
     "offq_act_codes_bytes": (_c_i64, [_c_i64, _c_i64]),
     "offq_weight_codes_bytes": (_c_i64, [_c_i64, _c_i64]),
+    "offq_quantize_act_group": (_c_int, [_c_vp, _c_int, _c_i64, _c_i64, _c_i64, _c_i32, _c_i32, _c_i32, _c_vp, _c_vp,
+                                         _c_vp, _c_vp]),
+    "offq_weight_group_sums": (_c_int, [_c_vp, _c_i64, _c_i64, _c_i32, _c_vp, _c_vp]),
+    "offq_w4a4_linear_group": (_c_int, [_c_vp, _c_vp, _c_vp, _c_i64, _c_i64, _c_i64, _c_i32, _c_vp, _c_vp, _c_vp,
+                                        _c_vp, _c_int, _c_i64, _c_vp]),
 }
 
 _lib = None
@@ -163,6 +168,26 @@ def offq_prepare_weight(w: torch.Tensor, N: int, K: int, g: int, rotate: bool, w
         _stream(stream)))
 
 
+def offq_quantize_act_group(x: torch.Tensor, T: int, K: int, ldx: int, g: int, group: int, flags: int,
+                            codes: torch.Tensor, scale: torch.Tensor, zero: torch.Tensor, stream=None) -> None:
+    _check("offq_quantize_act_group", load_library().offq_quantize_act_group(
+        _ptr(x), _dtype_code(x), T, K, ldx, g, group, flags, _ptr(codes), _ptr(scale), _ptr(zero), _stream(stream)))
+
+
+def offq_weight_group_sums(w_codes: torch.Tensor, N: int, K: int, group: int, w_groupsum: torch.Tensor,
+                           stream=None) -> None:
+    _check("offq_weight_group_sums", load_library().offq_weight_group_sums(
+        _ptr(w_codes), N, K, group, _ptr(w_groupsum), _stream(stream)))
+
+
+def offq_w4a4_linear_group(a_codes: torch.Tensor, a_scale: torch.Tensor, a_zero: torch.Tensor, T: int, N: int,
+                           K: int, group: int, w_codes: torch.Tensor, w_scale: torch.Tensor,
+                           w_groupsum: torch.Tensor, out: torch.Tensor, ldo: int, stream=None) -> None:
+    _check("offq_w4a4_linear_group", load_library().offq_w4a4_linear_group(
+        _ptr(a_codes), _ptr(a_scale), _ptr(a_zero), T, N, K, group, _ptr(w_codes), _ptr(w_scale),
+        _ptr(w_groupsum), _ptr(out), _dtype_code(out), ldo, _stream(stream)))
+
+
 def offq_get_device_status(stream=None) -> int:
     return load_library().offq_get_device_status(_stream(stream))
 
@@ -230,4 +255,40 @@ def w4a4_linear(a_codes: torch.Tensor, a_scale: torch.Tensor, a_offset: Optional
         out = torch.empty((T, N), dtype=out_dtype, device=a_codes.device)
     offq_w4a4_linear(a_codes, a_scale, a_offset, T, N, K, g, w_codes, w_scale, w_offsum, out, out.stride(0),
                      acc_debug, stream)
+    return out
+
+
+GROUP = 128  # activation group size of the per-group path (the paper's evaluated setting)
+
+
+def quantize_act_group(x: torch.Tensor, g: int, group: int = GROUP, rotate: bool = True,
+                       stream=None) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    """Per-group asymmetric codes, scales and zero-points of token rows x [T, K]."""
+    T, K = x.shape
+    codes = torch.empty((padded_rows(T), K // 2), dtype=torch.uint8, device=x.device)
+    scale = torch.empty((T, K // group), dtype=torch.float32, device=x.device)
+    zero = torch.empty((T, K // group), dtype=torch.float32, device=x.device)
+    offq_quantize_act_group(x, T, K, x.stride(0), g, group, OFFQ_ROTATE if rotate else 0, codes, scale, zero,
+                            stream)
+    return codes, scale, zero
+
+
+def weight_group_sums(w_codes: torch.Tensor, N: int, K: int, group: int = GROUP, stream=None) -> torch.Tensor:
+    """Integer row sums of the weight codes per activation group, [K/group, N] float32."""
+    sums = torch.empty((K // group, N), dtype=torch.float32, device=w_codes.device)
+    offq_weight_group_sums(w_codes, N, K, group, sums, stream)
+    return sums
+
+
+def w4a4_linear_group(a_codes: torch.Tensor, a_scale: torch.Tensor, a_zero: torch.Tensor,
+                      w_codes: torch.Tensor, w_scale: torch.Tensor, w_groupsum: torch.Tensor,
+                      group: int = GROUP, out_dtype: torch.dtype = torch.bfloat16,
+                      out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    T = a_scale.shape[0]
+    K = a_codes.shape[1] * 2
+    N = w_scale.shape[0]
+    if out is None:
+        out = torch.empty((T, N), dtype=out_dtype, device=a_codes.device)
+    offq_w4a4_linear_group(a_codes, a_scale, a_zero, T, N, K, group, w_codes, w_scale, w_groupsum, out,
+                           out.stride(0), stream)
     return out

@@ -131,3 +131,55 @@ def weight_q(codes, N: int, K: int) -> np.ndarray:
     import oracle as O
     arr = codes.cpu().numpy() if hasattr(codes, "cpu") else np.asarray(codes)
     return O.unpack_weight_codes(O.untile_codes(arr, N, K))
+
+
+def check_group_quant(q_gpu, s_gpu, z_gpu, ref, x, g, rotate, group=128, what="group"):
+    """Per-group asymmetric quantizer (GPU, fp32 decisions) against the oracle.
+
+    q_gpu [T, K] codes in [0, 15]; s_gpu, z_gpu [T, K/group]; ref the oracle's
+    quantize_act_group result on the same input.
+    * Scales: the group range comes from rotated values each off by at most
+      the rotation bound, so s differs by at most 2/15 of it (over sqrt(g))
+      plus a few roundings.
+    * Zero-points: equal, except +-1 where the oracle's min/s lies within
+      TIE_WINDOW of a half-integer.
+    * Codes, compared as q - z (what dequantizes): equal, except +-1 where
+      y/s lies within TIE_WINDOW of a half-integer, or at the grid's ends of a
+      group whose zero-point took the other side of a tie; at most
+      MAX_MISMATCH_FRACTION of all codes.
+    """
+    q_gpu = np.asarray(q_gpu, np.int64)
+    s_gpu = np.asarray(s_gpu, np.float64)
+    z_gpu = np.asarray(z_gpu, np.float64)
+    s_ref, z_ref, q_ref, y = ref["scale"], ref["zero"], ref["q"], ref["y"]
+    T, K = q_ref.shape
+    Gq = K // group
+    norm = math.sqrt(g) if rotate else 1.0
+    err_u = rotation_abs_error(x, g, rotate)[:, None]
+    tol_s = 2.0 * err_u / (15.0 * norm) + 4 * U32 * np.abs(s_ref)
+    bad = np.abs(s_gpu - s_ref) > tol_s
+    assert not np.any(bad), f"{what}: {bad.sum()} scales out of tolerance"
+    yg = y.reshape(T, Gq, group)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        t_min = np.where(s_ref > 0, yg.min(axis=2) / s_ref, 0.0)
+        ratio = np.where(np.repeat(s_ref, group, axis=1) > 0, y / np.repeat(s_ref, group, axis=1), 0.0)
+    near = lambda v: np.abs(np.abs(v) - np.floor(np.abs(v)) - 0.5) < TIE_WINDOW
+    zd = z_gpu != z_ref
+    assert np.all(np.abs(z_gpu - z_ref)[zd] <= 1) and np.all(near(t_min[zd])), f"{what}: zero-point off a tie"
+    d = (q_gpu - np.repeat(z_gpu, group, axis=1).astype(np.int64)) - (q_ref - np.repeat(z_ref, group, axis=1).astype(np.int64))
+    mism = d != 0
+    if mism.any():
+        assert np.all(np.abs(d[mism]) <= 1), f"{what}: a code differs by more than 1"
+        at_end = (q_gpu == 0) | (q_gpu == 15) | (q_ref == 0) | (q_ref == 15)
+        allowed = near(ratio) | (np.repeat(zd, group, axis=1) & at_end)
+        assert np.all(allowed[mism]), f"{what}: code mismatch away from a rounding tie"
+        assert mism.sum() <= max(1, MAX_MISMATCH_FRACTION * mism.size), f"{what}: {mism.sum()} codes differ"
+    return int(mism.sum())
+
+
+def group_terms(P, s, z, R, s_w):
+    """Magnitudes the per-group fp32 chain adds up: s_w sum_j |s_j| (|P_j| + |z_j R_j|)."""
+    acc = np.zeros(P.shape[1:])
+    for j in range(P.shape[0]):
+        acc += np.abs(s[:, j, None]) * (np.abs(P[j]) + np.abs(z[:, j, None] * R[j][None, :]))
+    return np.abs(np.asarray(s_w, np.float64))[None, :] * acc

@@ -109,3 +109,37 @@ def test_code_buffer_sizes(lib):
     assert Q.offq_weight_codes_bytes(11008, 4096) == 11008 * 2048
     assert Q.offq_weight_codes_bytes(300, 1024) == 320 * 512
     assert Q.offq_weight_codes_bytes(0, 1024) == -1
+
+
+def test_group_path_argument_checks(lib):
+    qg = lambda x=A16, dt=Q.OFFQ_BF16, T=4, K=1024, ldx=1024, g=256, group=128, flags=1, c=A16, s=A16, z=A16: \
+        lib.offq_quantize_act_group(x, dt, T, K, ldx, g, group, flags, c, s, z, None)
+    assert qg(group=64) == Q.OFFQ_ERR_UNSUPPORTED          # this build quantizes groups of 128
+    assert qg(group=0) == Q.OFFQ_ERR_INVALID_ARG
+    assert qg(K=1000, ldx=1000) == Q.OFFQ_ERR_INVALID_ARG  # group does not divide K
+    assert qg(g=100) == Q.OFFQ_ERR_INVALID_ARG             # rotation block not a power of two
+    assert qg(g=1024) == Q.OFFQ_ERR_UNSUPPORTED            # rotation blocks above 512
+    assert qg(flags=2) == Q.OFFQ_ERR_INVALID_ARG           # no explicit offset on this path
+    assert qg(ldx=1000) == Q.OFFQ_ERR_INVALID_ARG
+    assert qg(z=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert qg(x=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert qg(ldx=1028) == Q.OFFQ_ERR_MISALIGNED
+    assert qg(T=0) == Q.OFFQ_OK
+    ws = lambda w=A16, N=64, K=1024, group=128, out=A16: lib.offq_weight_group_sums(w, N, K, group, out, None)
+    assert ws(group=100) == Q.OFFQ_ERR_INVALID_ARG
+    assert ws(K=1000) == Q.OFFQ_ERR_INVALID_ARG
+    assert ws(N=0) == Q.OFFQ_ERR_INVALID_ARG
+    assert ws(out=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert ws(w=A8) == Q.OFFQ_ERR_MISALIGNED
+    lg = lambda a=A16, sa=A16, za=A16, T=8, N=64, K=1024, group=128, w=A16, sw=A16, R=A16, out=A16, \
+        dt=Q.OFFQ_BF16, ldo=64: lib.offq_w4a4_linear_group(a, sa, za, T, N, K, group, w, sw, R, out, dt, ldo, None)
+    assert lg(group=256) == Q.OFFQ_ERR_UNSUPPORTED
+    assert lg(K=1000) == Q.OFFQ_ERR_INVALID_ARG
+    assert lg(N=0) == Q.OFFQ_ERR_INVALID_ARG
+    assert lg(ldo=32) == Q.OFFQ_ERR_INVALID_ARG
+    assert lg(dt=9) == Q.OFFQ_ERR_INVALID_ARG
+    assert lg(K=131072) == Q.OFFQ_ERR_UNSUPPORTED
+    assert lg(za=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert lg(a=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert lg(ldo=65) == Q.OFFQ_ERR_MISALIGNED
+    assert lg(T=0) == Q.OFFQ_OK
