@@ -13,22 +13,24 @@
 //
 // One 128-code k-tile is one group, so the per-(token, group) scale cannot sit
 // in the operands: the pair MMA (M 256, N 128) writes each group's P_j into one
-// of two TMEM partial buffers, and four scaler warps fold it into a running
-// fp32 sum,
+// of two TMEM partial buffers, and eight scaler warps fold it into a running
+// fp32 sum held in their registers,
 //   d = fma(-z, R, P)   (exact while |z R| < 2^24),   S = fma(s, d, S),
 // (on the accumulator's P * 2^-18, with -z * 2^-18 and s * 2^18),
 // while the MMA fills the other buffer. After a tile's last group the scalers
 // multiply by s_w and store y, rounding once to the output type.
 //
-// TMEM (512 columns per CTA): P0 [0, 128), P1 [128, 256), running sum
-// [256, 384), 4 A stages of 32 columns [384, 512). The N = 128 pair tile is
-// what lets the running sum and both partials fit next to the A stages.
+// TMEM (512 columns per CTA): P0 [0, 128), P1 [128, 256), 6 A stages of 32
+// columns [256, 448). The N = 128 pair tile keeps both partials next to the
+// A stages, and each scaler thread's 64 running sums in its registers.
 //
-// Warp roles per CTA (17 warps):
+// Warp roles per CTA (15 warps, so up to 128 registers per thread):
 //   warp 0       TMEM allocation; in the leader CTA, lane 0 issues the MMAs
-//   warps 1-8    A converters: two per 32-lane TMEM quarter, alternating k-tiles
-//   warps 9-12   B converters: two per 32-row group (64 rows of B per CTA)
-//   warps 13-16  scalers and epilogue, one per TMEM quarter (128 columns)
+//   warps 1-4    A converters: one per 32-lane TMEM quarter, every k-tile
+//   warps 5-6    B converters: one per 32-row group (64 rows of B per CTA)
+//   warps 7-14   scalers and epilogue, two per TMEM quarter (64 columns each);
+//                they prefetch the row sums R and s_w into shared memory
+//                two groups ahead (cp.async)
 // Every wait is bounded; a wait that runs out aborts the CTA and records
 // OFFQ_ERR_TIMEOUT in the device status word.
 #include <cuda.h>
@@ -52,27 +54,37 @@ constexpr int GBNH = GBN / 2;    // rows of B held by one CTA
 constexpr int GBK = 128;         // codes per k-tile = one activation group
 constexpr int kGroup = GBK;
 constexpr int kGChunks = GBK / 32;  // 16-byte packed chunks per row per k-tile
-constexpr int kGStages = 4;
-constexpr int kGSplit = 2;          // converter warps per row group, alternating k-tiles
-constexpr int kGAWarps = 4 * kGSplit;
-constexpr int kGBWarps = (GBNH / 32) * kGSplit;
-constexpr int kGScWarps = 4;
+constexpr int kGStages = 6;
+constexpr int kGRing = 3;           // k-tiles of loads in flight per converter thread
+constexpr int kGAWarps = 4;         // one per 32-lane TMEM quarter, every k-tile
+constexpr int kGBWarps = GBNH / 32; // one per 32-row group of B
+constexpr int kGScWarps = 8;            // two per TMEM quarter
+constexpr int kGScCols = GBN / (kGScWarps / 4);  // columns per scaler warp
 constexpr int kGFirstA = 1, kGFirstB = kGFirstA + kGAWarps, kGFirstSc = kGFirstB + kGBWarps;
 constexpr int kGThreads = (kGFirstSc + kGScWarps) * 32;
 constexpr int kGArrivals = 4 + GBNH / 32;  // per stage and CTA: one per A quarter and per B row group
 constexpr int kPCol0 = 0;                  // two partial buffers of GBN columns
-constexpr int kSCol0 = 2 * GBN;            // running sum
-constexpr int kGACol0 = 3 * GBN;           // A stages
+constexpr int kGACol0 = 2 * GBN;           // A stages
 constexpr int kGAColsPerStage = GBK / 4;
 constexpr int kGTmemCols = 512;
 static_assert(kGACol0 + kGStages * kGAColsPerStage <= kGTmemCols, "TMEM budget");
 constexpr int kGBStage = GBNH * GBK;  // 8 KB of E4M3 per stage
 constexpr uint32_t kGIdesc = idesc_e4m3_f32(2 * GBM, GBN);  // pair MMA: M = 256, N = 128
 
-// Shared memory: B stages, barriers (full/empty per stage, partial full/empty
-// per buffer), misc. The request is padded so that one CTA holds an SM: the
-// pair allocates all 512 TMEM columns.
-constexpr int kGOffBars = kGStages * kGBStage;
+// Each scaler warp prefetches, two groups ahead, its columns of the row sums
+// R[j] into a ring of kRSlots rows, and each tile's s_w into a ring of kWSlots
+// rows (three, so that with one group per tile the copy two tiles ahead does
+// not land on the row in use).
+constexpr int kRSlots = 3;
+constexpr int kWSlots = 3;
+constexpr int kScRowBytes = kGScCols * 4;
+constexpr int kScBytes = (kRSlots + kWSlots) * kScRowBytes;  // per scaler warp
+
+// Shared memory: B stages, the scalers' rows, barriers (full/empty per stage,
+// partial full/empty per buffer), misc. The request is padded so that one CTA
+// holds an SM: the pair allocates all 512 TMEM columns.
+constexpr int kGOffSc = kGStages * kGBStage;
+constexpr int kGOffBars = kGOffSc + kGScWarps * kScBytes;
 constexpr int kGNumBars = 2 * kGStages + 4;
 constexpr int kGOffMisc = kGOffBars + kGNumBars * 8;
 constexpr int kGUsed = kGOffMisc + 64 + 1024;
@@ -92,7 +104,6 @@ struct GroupParams {
   int m_pairs, n_tiles;
   int t_blocks, n_blocks;
   int kchunks;  // K / 32
-  int vec;      // N % 4 == 0 and gsum, w_scale 16-byte aligned
 };
 
 __device__ __forceinline__ void load_group_kt(const uint8_t* blk, int kchunks, int kt, uint4 (&v)[kGChunks]) {
@@ -106,20 +117,30 @@ __device__ __forceinline__ void load_group_kt(const uint8_t* blk, int kchunks, i
   }
 }
 
-// Four consecutive entries of a [.][N] float row from column n (zeros past N).
-__device__ __forceinline__ float4 ldg_cols4(const float* row, int n, int N, bool vec) {
-  if (vec) return n < N ? __ldg(reinterpret_cast<const float4*>(row + n)) : make_float4(0.f, 0.f, 0.f, 0.f);
-  float4 r;
-  r.x = n < N ? __ldg(row + n) : 0.f;
-  r.y = n + 1 < N ? __ldg(row + n + 1) : 0.f;
-  r.z = n + 2 < N ? __ldg(row + n + 2) : 0.f;
-  r.w = n + 3 < N ? __ldg(row + n + 3) : 0.f;
-  return r;
+__device__ __forceinline__ void cp_async4(uint32_t dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit_group() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait_groups() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Copies row[n0 .. n0 + kGScCols) (entries past N skipped) into shared memory
+// at dst: lanes 0-15 four entries each.
+__device__ __forceinline__ void copy_cols(uint32_t dst, const float* row, int n0, int N, int lane) {
+  if (lane < kGScCols / 4) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int n = n0 + 4 * lane + i;
+      if (n < N) cp_async4(dst + (4 * lane + i) * 4, row + n);
+    }
+  }
 }
 
 // Persistent pair kernel over pair tiles (m_pair * n_tiles + n_tile), cluster c
 // taking tiles c, c + clusters, ... The global k-tile counter j runs across
-// tiles: operand stage j mod 4, partial buffer j mod 2.
+// tiles: operand stage j mod 6, partial buffer j mod 2.
 template <int OUT>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGThreads, 1)
     w4a4_group_gemm_kernel(const GroupParams p) {
@@ -200,10 +221,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGThreads, 1)
     }
   } else if (warp < kGFirstSc) {
     // ---------------- converters: packed codes -> E4M3 operands ----------------
+    // One warp per 32-row group converts every k-tile, with kGRing k-tiles of
+    // loads in flight (a register ring), which covers the load latency over
+    // three MMA k-tiles.
     const bool is_a = warp < kGFirstB;
     const int quarter = warp & 3;
-    const int wb = (warp - kGFirstB) & 1;
-    const int part = is_a ? (warp - kGFirstA) >> 2 : (warp - kGFirstB) >> 1;  // k-tiles g == part mod 2
+    const int wb = warp - kGFirstB;
     const uint32_t full_l = leader_addr(full(0));
     const uint8_t* codes = is_a ? p.a_codes : p.w_codes;
     const int rb_count = is_a ? p.t_blocks : p.n_blocks;
@@ -212,152 +235,199 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGThreads, 1)
                           : ((tile % p.n_tiles) * GBN + static_cast<int>(rank) * GBNH + wb * 32) >> 5;
       return rb < rb_count ? codes + static_cast<int64_t>(rb) * p.kchunks * 512 + lane * 16 : nullptr;
     };
-    auto advance1 = [&](int& tile, int& kt) {
+    auto advance = [&](int& tile, int& kt) {
       if (++kt == nk) {
         kt = 0;
         tile += clusters;
       }
     };
+    uint4 ring[kGRing][kGChunks];
     int ld_tile = cluster, ld_kt = 0;
-    if (part) advance1(ld_tile, ld_kt);
-    int tile = ld_tile, kt = ld_kt;
-    uint4 ring[kGChunks];
     int blk_tile = ld_tile;
-    const uint8_t* blk = ld_tile < num_tiles ? block_ptr(ld_tile) : nullptr;
-    if (ld_tile < num_tiles) load_group_kt(blk, p.kchunks, ld_kt, ring);
-    advance1(ld_tile, ld_kt);
-    advance1(ld_tile, ld_kt);
-    int s = part, phase = 0;
-    while (tile < num_tiles) {
-      if (!__all_sync(0xFFFFFFFFu, wait_cluster(empty(s), phase ^ 1, abort))) break;
-      if (is_a) {
-        tc_fence_after();
-        uint32_t f8[32];
+    const uint8_t* blk = block_ptr(ld_tile);
 #pragma unroll
-        for (int c = 0; c < kGChunks; ++c) {
-          widen_act(ring[c].x, f8[8 * c + 0], f8[8 * c + 1]);
-          widen_act(ring[c].y, f8[8 * c + 2], f8[8 * c + 3]);
-          widen_act(ring[c].z, f8[8 * c + 4], f8[8 * c + 5]);
-          widen_act(ring[c].w, f8[8 * c + 6], f8[8 * c + 7]);
-        }
-        tmem_st_32cols(tmem + (static_cast<uint32_t>(quarter * 32) << 16) + kGACol0 + s * kGAColsPerStage, f8);
-        tmem_st_wait();
-        tc_fence_before();
-      } else {
-        const int r = wb * 32 + lane;
-        const uint32_t st = base + s * kGBStage + r * 128;
-#pragma unroll
-        for (int c = 0; c < kGChunks; ++c) {
-          uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
-          widen_weight(ring[c].x, a0, a1);
-          widen_weight(ring[c].y, a2, a3);
-          widen_weight(ring[c].z, b0, b1);
-          widen_weight(ring[c].w, b2, b3);
-          sts128(st + (((2 * c) ^ (r & 7)) << 4), a0, a1, a2, a3);
-          sts128(st + (((2 * c + 1) ^ (r & 7)) << 4), b0, b1, b2, b3);
-        }
-        fence_proxy_async_smem();
-      }
-      __syncwarp();
-      if (lane == 0) arrive_cluster(full_l + 8u * s);
+    for (int r = 0; r < kGRing; ++r) {
       if (ld_tile < num_tiles) {
         if (ld_tile != blk_tile) {
           blk_tile = ld_tile;
           blk = block_ptr(ld_tile);
         }
-        load_group_kt(blk, p.kchunks, ld_kt, ring);
+        load_group_kt(blk, p.kchunks, ld_kt, ring[r]);
       }
-      advance1(ld_tile, ld_kt);
-      advance1(ld_tile, ld_kt);
-      advance1(tile, kt);
-      advance1(tile, kt);
-      s += kGSplit;
-      if (s >= kGStages) {
-        s -= kGStages;
-        phase ^= 1;
+      advance(ld_tile, ld_kt);
+    }
+    int tile = cluster, kt = 0, s = 0, phase = 0;
+    bool run = true;
+    while (run) {
+#pragma unroll
+      for (int r = 0; r < kGRing; ++r) {
+        if (tile >= num_tiles) {
+          run = false;
+          break;
+        }
+        if (!__all_sync(0xFFFFFFFFu, wait_cluster(empty(s), phase ^ 1, abort))) {
+          run = false;
+          break;
+        }
+        if (is_a) {
+          tc_fence_after();
+          uint32_t f8[32];
+#pragma unroll
+          for (int c = 0; c < kGChunks; ++c) {
+            widen_act(ring[r][c].x, f8[8 * c + 0], f8[8 * c + 1]);
+            widen_act(ring[r][c].y, f8[8 * c + 2], f8[8 * c + 3]);
+            widen_act(ring[r][c].z, f8[8 * c + 4], f8[8 * c + 5]);
+            widen_act(ring[r][c].w, f8[8 * c + 6], f8[8 * c + 7]);
+          }
+          tmem_st_32cols(tmem + (static_cast<uint32_t>(quarter * 32) << 16) + kGACol0 + s * kGAColsPerStage, f8);
+          tmem_st_wait();
+          tc_fence_before();
+        } else {
+          const int rr = wb * 32 + lane;
+          const uint32_t st = base + s * kGBStage + rr * 128;
+#pragma unroll
+          for (int c = 0; c < kGChunks; ++c) {
+            uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
+            widen_weight(ring[r][c].x, a0, a1);
+            widen_weight(ring[r][c].y, a2, a3);
+            widen_weight(ring[r][c].z, b0, b1);
+            widen_weight(ring[r][c].w, b2, b3);
+            sts128(st + (((2 * c) ^ (rr & 7)) << 4), a0, a1, a2, a3);
+            sts128(st + (((2 * c + 1) ^ (rr & 7)) << 4), b0, b1, b2, b3);
+          }
+          fence_proxy_async_smem();
+        }
+        __syncwarp();
+        if (lane == 0) arrive_cluster(full_l + 8u * s);
+        // Refill this ring slot kGRing k-tiles ahead.
+        if (ld_tile < num_tiles) {
+          if (ld_tile != blk_tile) {
+            blk_tile = ld_tile;
+            blk = block_ptr(ld_tile);
+          }
+          load_group_kt(blk, p.kchunks, ld_kt, ring[r]);
+        }
+        advance(ld_tile, ld_kt);
+        advance(tile, kt);
+        if (++s == kGStages) {
+          s = 0;
+          phase ^= 1;
+        }
       }
     }
   } else {
     // ---------------- scalers and epilogue ----------------
+    const int sw = warp - kGFirstSc;
     const int quarter = warp & 3;
-    const int rl = quarter * 32 + lane;  // TMEM lane = row within the CTA
-    const uint32_t lane_base = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+    const int c0 = (sw >> 2) * kGScCols;  // this warp's first column of the tile
+    const int rl = quarter * 32 + lane;   // TMEM lane = row within the CTA
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + c0;
     const uint32_t pempty_l = leader_addr(pempty(0));
-    const bool vec = p.vec != 0;
+    const uint32_t rbuf = base + kGOffSc + sw * kScBytes;  // kRSlots rows of R, then kWSlots rows of s_w
+    const uint32_t wbuf = rbuf + kRSlots * kScRowBytes;
+    // Prefetch position: two groups ahead of the one being scaled.
+    int pf_tile = cluster, pf_kt = 0, pf_slot = 0, pf_wslot = 0;
+    auto prefetch = [&]() {
+      if (pf_tile < num_tiles) {
+        const int n0 = (pf_tile % p.n_tiles) * GBN + c0;
+        copy_cols(rbuf + pf_slot * kScRowBytes, p.gsum + static_cast<int64_t>(pf_kt) * p.N, n0, p.N, lane);
+        if (pf_kt == 0) copy_cols(wbuf + pf_wslot * kScRowBytes, p.w_scale, n0, p.N, lane);
+      }
+      cp_async_commit_group();
+      if (++pf_slot == kRSlots) pf_slot = 0;
+      if (++pf_kt == nk) {
+        pf_kt = 0;
+        pf_tile += clusters;
+        if (++pf_wslot == kWSlots) pf_wslot = 0;
+      }
+    };
+    prefetch();
+    prefetch();
     uint32_t j = 0;
+    int slot = 0, wslot = 0;
     bool ok = true;
-    for (int tile = cluster; tile < num_tiles && ok; tile += clusters) {
+    for (int tile = cluster; tile < num_tiles && ok; tile += clusters, wslot = wslot + 1 == kWSlots ? 0 : wslot + 1) {
       const int t = (tile / p.n_tiles) * 2 * GBM + static_cast<int>(rank) * GBM + rl;
-      const int n0 = (tile % p.n_tiles) * GBN;
+      const int n0 = (tile % p.n_tiles) * GBN + c0;
       const bool row_ok = t < p.T;
       const float* srow = p.a_scale + static_cast<int64_t>(row_ok ? t : 0) * p.Gq;
       const float* zrow = p.a_zero + static_cast<int64_t>(row_ok ? t : 0) * p.Gq;
+      float S[kGScCols];  // running sum of this row's columns c0 .. c0 + kGScCols of the tile
+      // This row's scale and zero-point of the group being scaled, loaded one group ahead.
+      float s_next = row_ok ? __ldg(srow) : 0.f, z_next = row_ok ? __ldg(zrow) : 0.f;
       for (int kt = 0; kt < nk; ++kt, ++j) {
         const uint32_t b = j & 1u, use = j >> 1;
+        const bool last = kt == nk - 1;
         // The accumulator holds P * 2^-18 (each E4M3 operand carries 2^-9):
         // d' = P 2^-18 - z R 2^-18 and s 2^18 d' = s (P - z R), all exact scalings.
-        const float sg = row_ok ? __ldg(srow + kt) * 262144.0f : 0.f;
-        const float nz = row_ok ? __ldg(zrow + kt) * -3.814697265625e-06f : 0.f;
+        const float sg = s_next * 262144.0f;
+        const float nz = z_next * -3.814697265625e-06f;
+        if (row_ok && kt + 1 < nk) {
+          s_next = __ldg(srow + kt + 1);
+          z_next = __ldg(zrow + kt + 1);
+        }
+        __syncwarp();  // every lane is done with the ring slot the next copy overwrites
+        prefetch();
+        if (last)
+          cp_async_wait_groups<0>();  // this tile's s_w as well
+        else
+          cp_async_wait_groups<2>();  // R of this group has landed (own copies)
+        __syncwarp();                 // ... and the other lanes' copies are visible
         ok = __all_sync(0xFFFFFFFFu, wait_cluster(pfull(b), use & 1u, abort));
         if (!ok) break;
         tc_fence_after();
-        const float* rrow = p.gsum + static_cast<int64_t>(kt) * p.N;
-        const bool last = kt == nk - 1;
+        const uint32_t rrow = rbuf + slot * kScRowBytes;
+        const uint32_t wrow = wbuf + wslot * kScRowBytes;
         const uint64_t SG = pack2(sg, sg), NZ = pack2(nz, nz);
-#pragma unroll 1
-        for (int c = 0; c < GBN / 32; ++c) {
-          uint32_t pv[32], sv[32];
+#pragma unroll
+        for (int c = 0; c < kGScCols / 32; ++c) {
+          uint32_t pv[32];
           tmem_ld_32cols(lane_base + kPCol0 + b * GBN + c * 32, pv);
-          if (kt > 0) tmem_ld_32cols(lane_base + kSCol0 + c * 32, sv);
           tmem_ld_wait();
-          if (c == GBN / 32 - 1) {
+          if (c == kGScCols / 32 - 1) {
             // The partial is in registers: its buffer may take the group after next.
             tc_fence_before();
             __syncwarp();
             if (lane == 0) arrive_cluster(pempty_l + 8u * b);
           }
-          const int nc = n0 + c * 32;
 #pragma unroll
           for (int q4 = 0; q4 < 8; ++q4) {
-            const float4 r = ldg_cols4(rrow, nc + 4 * q4, p.N, vec);
-            const uint64_t d0 = fma2v(NZ, pack2(r.x, r.y), pack2(__uint_as_float(pv[4 * q4]), __uint_as_float(pv[4 * q4 + 1])));
-            const uint64_t d1 =
-                fma2v(NZ, pack2(r.z, r.w), pack2(__uint_as_float(pv[4 * q4 + 2]), __uint_as_float(pv[4 * q4 + 3])));
+            const uint4 rv = lds128(rrow + (c * 32 + 4 * q4) * 4);
+            const uint64_t d0 = fma2v(NZ, pack2(__uint_as_float(rv.x), __uint_as_float(rv.y)),
+                                      pack2(__uint_as_float(pv[4 * q4]), __uint_as_float(pv[4 * q4 + 1])));
+            const uint64_t d1 = fma2v(NZ, pack2(__uint_as_float(rv.z), __uint_as_float(rv.w)),
+                                      pack2(__uint_as_float(pv[4 * q4 + 2]), __uint_as_float(pv[4 * q4 + 3])));
+            float* S4 = &S[c * 32 + 4 * q4];
             uint64_t a0, a1;
             if (kt == 0) {
               a0 = mul2v(SG, d0);
               a1 = mul2v(SG, d1);
             } else {
-              a0 = fma2v(SG, d0, pack2(__uint_as_float(sv[4 * q4]), __uint_as_float(sv[4 * q4 + 1])));
-              a1 = fma2v(SG, d1, pack2(__uint_as_float(sv[4 * q4 + 2]), __uint_as_float(sv[4 * q4 + 3])));
+              a0 = fma2v(SG, d0, pack2(S4[0], S4[1]));
+              a1 = fma2v(SG, d1, pack2(S4[2], S4[3]));
             }
-            float f0, f1, f2, f3;
-            unpack2(a0, f0, f1);
-            unpack2(a1, f2, f3);
-            sv[4 * q4] = __float_as_uint(f0);
-            sv[4 * q4 + 1] = __float_as_uint(f1);
-            sv[4 * q4 + 2] = __float_as_uint(f2);
-            sv[4 * q4 + 3] = __float_as_uint(f3);
+            unpack2(a0, S4[0], S4[1]);
+            unpack2(a1, S4[2], S4[3]);
           }
-          if (!last) {
-            tmem_st_32cols(lane_base + kSCol0 + c * 32, sv);
-          } else if (row_ok && nc < p.N) {
+          const int nc = n0 + c * 32;
+          if (last && row_ok && nc < p.N) {
             float y[32];
 #pragma unroll
             for (int q4 = 0; q4 < 8; ++q4) {
-              const float4 w = ldg_cols4(p.w_scale, nc + 4 * q4, p.N, vec);
-              y[4 * q4] = w.x * __uint_as_float(sv[4 * q4]);
-              y[4 * q4 + 1] = w.y * __uint_as_float(sv[4 * q4 + 1]);
-              y[4 * q4 + 2] = w.z * __uint_as_float(sv[4 * q4 + 2]);
-              y[4 * q4 + 3] = w.w * __uint_as_float(sv[4 * q4 + 3]);
+              const uint4 wv = lds128(wrow + (c * 32 + 4 * q4) * 4);
+              y[4 * q4] = __uint_as_float(wv.x) * S[c * 32 + 4 * q4];
+              y[4 * q4 + 1] = __uint_as_float(wv.y) * S[c * 32 + 4 * q4 + 1];
+              y[4 * q4 + 2] = __uint_as_float(wv.z) * S[c * 32 + 4 * q4 + 2];
+              y[4 * q4 + 3] = __uint_as_float(wv.w) * S[c * 32 + 4 * q4 + 3];
             }
             const int nvalid = p.N - nc < 32 ? p.N - nc : 32;
             store_out<OUT, 32>(p.out, static_cast<int64_t>(t) * p.ldo + nc, y, nvalid);
           }
         }
-        if (!last) tmem_st_wait();  // the running sum is in TMEM before the next group reads it
+        if (++slot == kRSlots) slot = 0;
       }
     }
+    cp_async_wait_groups<0>();  // no copy into shared memory outlives the CTA
   }
 
   // ---------------- teardown ----------------
@@ -441,7 +511,6 @@ extern "C" int offq_w4a4_linear_group(const uint8_t* a_codes, const float* a_sca
   p.t_blocks = static_cast<int>((T + 31) / 32);
   p.n_blocks = static_cast<int>((N + 31) / 32);
   p.kchunks = static_cast<int>(K / 32);
-  p.vec = N % 4 == 0 && aligned(w_groupsum, 16) && aligned(w_scale, 16);
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   switch (out_dtype) {
     case OFFQ_F32: return launch_group_gemm<OFFQ_F32>(p, s);

@@ -130,6 +130,13 @@ def test_group_gemm_ragged(out_dt, rotate):
     _check_group_layer(300, 512, 200, 512, out_dt, rotate, seed=70)
 
 
+@pytest.mark.parametrize("K", [128, 256])
+def test_group_gemm_one_and_two_groups(K):
+    """K = 128 (one group per tile: the prefetch runs two tiles ahead) and
+    K = 256, over more tiles than clusters."""
+    _check_group_layer(600, K, 2000, K, "bf16", False, seed=80)
+
+
 def test_group_gemm_leading_dimension():
     _check_group_layer(40, 1024, 96, 256, "bf16", True, seed=71, ldo=136)
 
