@@ -302,6 +302,99 @@ class GpuStep:
             self.result_host.copy_(self.result, non_blocking=True)
 
 
+class GroupStep:
+    """The same layers through the per-group asymmetric path (the paper's
+    evaluated activation setting: groups of 128 with zero-points): per site the
+    group quantizer (with the site's rotation), then its layers' group GEMMs."""
+
+    def __init__(self, w: W.Workload, T: int, device, seed_base: int = 0):
+        import torch
+        from paper_2606_07116_gb300 import offq as Q
+        self.torch, self.Q, self.T = torch, Q, T
+        dt = torch.bfloat16 if w.x_dtype == "bf16" else torch.float32
+        self.sites = []
+        for i, (name, K, rotate, layers) in enumerate(sites(w)):
+            x = torch.from_numpy(W.activations(T, K, seed=seed_base + 10 + i, dist=w.dist, n_out=w.n_out,
+                                               mult=w.mult)).to(dt).to(device)
+            g = W.block_for(K)
+            G = K // Q.GROUP
+            gemms = []
+            for l in layers:
+                wt = torch.from_numpy(W.weights(l.N, l.K, seed=seed_base + 100 + len(self.sites) * 10 + len(gemms)))
+                wc, ws, _ = Q.prepare_weight(wt.to(device), g, rotate=l.rotate)
+                gemms.append({"layer": l, "codes": wc, "scale": ws, "gsum": Q.weight_group_sums(wc, l.N, l.K),
+                              "out": torch.empty((T, l.N), dtype=torch.bfloat16, device=device)})
+            self.sites.append({"K": K, "g": g, "flags": Q.OFFQ_ROTATE if rotate else 0, "x": x,
+                               "codes": torch.empty((Q.padded_rows(T), K // 2), dtype=torch.uint8, device=device),
+                               "scale": torch.empty((T, G), dtype=torch.float32, device=device),
+                               "zero": torch.empty((T, G), dtype=torch.float32, device=device),
+                               "gemms": gemms})
+        torch.cuda.synchronize(device)
+
+    def launches_per_step(self):
+        return len(self.sites) + sum(len(s["gemms"]) for s in self.sites)
+
+    def quant_bytes(self):
+        T = self.T
+        return sum(T * s["K"] * s["x"].element_size() + T * s["K"] // 2 + 8 * T * (s["K"] // self.Q.GROUP)
+                   for s in self.sites)
+
+    def run(self, stream, timers=None):
+        Q, torch, T = self.Q, self.torch, self.T
+
+        def rec(kind):
+            if timers is not None:
+                e = torch.cuda.Event(enable_timing=True)
+                e.record(stream)
+                timers.setdefault(kind, []).append(e)
+
+        for s in self.sites:
+            rec("quant")
+            Q.offq_quantize_act_group(s["x"], T, s["K"], s["x"].stride(0), s["g"], Q.GROUP, s["flags"],
+                                      s["codes"], s["scale"], s["zero"], stream)
+            rec("quant")
+            for gm in s["gemms"]:
+                l = gm["layer"]
+                rec("gemm")
+                Q.offq_w4a4_linear_group(s["codes"], s["scale"], s["zero"], T, l.N, l.K, Q.GROUP, gm["codes"],
+                                         gm["scale"], gm["gsum"], gm["out"], gm["out"].stride(0), stream)
+                rec("gemm")
+
+
+def time_group_path(w, T, device, args, rank, flush_l2, barrier, stream, fp8_peak, peaks):
+    """Step time and per-kernel rates of the per-group path (same protocol as the main step)."""
+    import torch
+    from paper_2606_07116_gb300 import offq as Q
+    gstep = GroupStep(w, T, device, seed_base=rank_seed_base(rank))
+    for _ in range(args.warmup):
+        flush_l2()
+        gstep.run(stream)
+    steps = args.steps
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    barrier()
+    torch.cuda.synchronize(device)
+    for i in range(steps):
+        flush_l2()
+        starts[i].record(stream)
+        gstep.run(stream)
+        ends[i].record(stream)
+    torch.cuda.synchronize(device)
+    dev_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends))
+    timers = {}
+    kb = max(1, min(steps, 50))
+    for _ in range(kb):
+        flush_l2()
+        gstep.run(stream, timers=timers)
+    torch.cuda.synchronize(device)
+    st = Q.offq_get_device_status(stream)
+    if st != Q.OFFQ_OK:
+        raise RuntimeError(f"device status after the group path: {Q.status_string(st)}")
+    gemm_ms = sum(_pair_times(timers["gemm"])) / kb
+    quant_ms = sum(_pair_times(timers["quant"])) / kb
+    return gstep, dev_ms / steps, gemm_ms, quant_ms
+
+
 def _pair_times(events):
     return [events[i].elapsed_time(events[i + 1]) for i in range(0, len(events), 2)]
 
@@ -414,6 +507,26 @@ def run_gpu(args, rank, world, local_rank):
 
     peaks = load_peaks()
     fp8_peak = peaks["bf16_tflops_sustained"] * FP8_PER_BF16
+    group = None
+    if not args.no_group:
+        gstep, g_ms, g_gemm_ms, g_quant_ms = time_group_path(w, T, device, args, rank, flush_l2, barrier, stream,
+                                                             fp8_peak, peaks)
+        (g_ms,) = reduce_over_ranks([g_ms], dist, device)
+        g_gemm_tflops = ops / (g_gemm_ms * 1e-3) / 1e12
+        g_quant_gbs = gstep.quant_bytes() / (g_quant_ms * 1e-3) / 1e9
+        group = {
+            "what": "the paper's evaluated activation setting on the same layers: per-group (128) asymmetric "
+                    "activations with zero-points (offq_quantize_act_group + offq_w4a4_linear_group), no KV4",
+            "value": round(job_tops(ops, world, g_ms), 3), "unit": UNIT, "ms_per_step": round(g_ms, 4),
+            "roofline": {"bound": "tensor", "kernel": "w4a4_group_gemm_kernel (tcgen05.mma kind::f8f6f4, "
+                                                      "per-group scaling in the scaler warps)",
+                         "achieved": round(g_gemm_tflops, 2), "peak": round(fp8_peak, 1), "unit": "TFLOP/s",
+                         "frac": round(g_gemm_tflops / fp8_peak, 4), "gemm_ms_per_step": round(g_gemm_ms, 4)},
+            "act_quant": {"value": round(g_quant_gbs, 1), "unit": "GB/s", "peak": peaks["hbm_gbs"],
+                          "frac": round(g_quant_gbs / peaks["hbm_gbs"], 4), "ms_per_step": round(g_quant_ms, 4),
+                          "bytes_per_step": gstep.quant_bytes()},
+            "gpu_launches": gstep.launches_per_step() * args.steps,
+        }
     gemm_tflops = ops * args.steps / (gemm_ms * 1e-3) / 1e12
     quant_gbs = step.quant_bytes() * args.steps / (quant_ms * 1e-3) / 1e9
     kv_gbs = step.kv_bytes() * args.steps / (kv_ms * 1e-3) / 1e9 if kv_ms > 0 else None
@@ -453,6 +566,8 @@ def run_gpu(args, rank, world, local_rank):
         "wall_s_timed_region": round(wall1 - wall0, 4),
         "clocks": clk.summary(),
     }
+    if group is not None:
+        line["group_asym"] = group
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
     return line
@@ -561,6 +676,7 @@ def main():
     ap.add_argument("--workload", default="llama2_7b")
     ap.add_argument("--impl", default="offq", choices=["offq", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-group", action="store_true", help="skip the per-group asymmetric path's timing")
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--ref-budget", type=float, default=120.0, help="seconds of oracle work for --impl reference")
     args = ap.parse_args()
