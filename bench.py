@@ -406,12 +406,18 @@ def load_traffic_record():
             rec = json.load(f)
     except (OSError, ValueError):
         return None
-    src = os.path.join(ROOT, "paper_2606_07116_gb300", "csrc", "gemm.cu")
-    with open(src, "rb") as f:
-        digest = hashlib.sha256(f.read()).hexdigest()
-    if rec.get("gemm_cu_sha256") != digest:
+    if rec.get("gemm_src_sha256") != gemm_source_digest():
         return None
     return rec
+
+
+def gemm_source_digest() -> str:
+    """sha256 over the per-token GEMM's sources (gemm.cu, then pair_common.cuh)."""
+    h = hashlib.sha256()
+    for name in ("gemm.cu", "pair_common.cuh"):
+        with open(os.path.join(ROOT, "paper_2606_07116_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
 
 
 def run_gpu(args, rank, world, local_rank):
