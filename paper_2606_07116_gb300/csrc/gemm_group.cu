@@ -117,6 +117,11 @@ __device__ __forceinline__ void load_group_kt(const uint8_t* blk, int kchunks, i
   }
 }
 
+// Two 64-bit shared-memory words (four floats as two packed pairs).
+__device__ __forceinline__ void lds_2x64(uint32_t addr, uint64_t& a, uint64_t& b) {
+  asm volatile("ld.shared.v2.b64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "r"(addr) : "memory");
+}
+
 __device__ __forceinline__ void cp_async4(uint32_t dst, const void* src) {
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(dst), "l"(src) : "memory");
 }
@@ -352,7 +357,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGThreads, 1)
       const bool row_ok = t < p.T;
       const float* srow = p.a_scale + static_cast<int64_t>(row_ok ? t : 0) * p.Gq;
       const float* zrow = p.a_zero + static_cast<int64_t>(row_ok ? t : 0) * p.Gq;
-      float S[kGScCols];  // running sum of this row's columns c0 .. c0 + kGScCols of the tile
+      uint64_t S2[kGScCols / 2];  // running sums of this row's columns c0 .. c0 + kGScCols, packed in pairs
       // This row's scale and zero-point of the group being scaled, loaded one group ahead.
       float s_next = row_ok ? __ldg(srow) : 0.f, z_next = row_ok ? __ldg(zrow) : 0.f;
       for (int kt = 0; kt < nk; ++kt, ++j) {
@@ -392,33 +397,29 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGThreads, 1)
           }
 #pragma unroll
           for (int q4 = 0; q4 < 8; ++q4) {
-            const uint4 rv = lds128(rrow + (c * 32 + 4 * q4) * 4);
-            const uint64_t d0 = fma2v(NZ, pack2(__uint_as_float(rv.x), __uint_as_float(rv.y)),
-                                      pack2(__uint_as_float(pv[4 * q4]), __uint_as_float(pv[4 * q4 + 1])));
-            const uint64_t d1 = fma2v(NZ, pack2(__uint_as_float(rv.z), __uint_as_float(rv.w)),
-                                      pack2(__uint_as_float(pv[4 * q4 + 2]), __uint_as_float(pv[4 * q4 + 3])));
-            float* S4 = &S[c * 32 + 4 * q4];
-            uint64_t a0, a1;
+            uint64_t r01, r23;
+            lds_2x64(rrow + (c * 32 + 4 * q4) * 4, r01, r23);
+            const uint64_t d0 = fma2v(NZ, r01, pack2(__uint_as_float(pv[4 * q4]), __uint_as_float(pv[4 * q4 + 1])));
+            const uint64_t d1 = fma2v(NZ, r23, pack2(__uint_as_float(pv[4 * q4 + 2]), __uint_as_float(pv[4 * q4 + 3])));
+            uint64_t& a0 = S2[c * 16 + 2 * q4];
+            uint64_t& a1 = S2[c * 16 + 2 * q4 + 1];
             if (kt == 0) {
               a0 = mul2v(SG, d0);
               a1 = mul2v(SG, d1);
             } else {
-              a0 = fma2v(SG, d0, pack2(S4[0], S4[1]));
-              a1 = fma2v(SG, d1, pack2(S4[2], S4[3]));
+              a0 = fma2v(SG, d0, a0);
+              a1 = fma2v(SG, d1, a1);
             }
-            unpack2(a0, S4[0], S4[1]);
-            unpack2(a1, S4[2], S4[3]);
           }
           const int nc = n0 + c * 32;
           if (last && row_ok && nc < p.N) {
             float y[32];
 #pragma unroll
             for (int q4 = 0; q4 < 8; ++q4) {
-              const uint4 wv = lds128(wrow + (c * 32 + 4 * q4) * 4);
-              y[4 * q4] = __uint_as_float(wv.x) * S[c * 32 + 4 * q4];
-              y[4 * q4 + 1] = __uint_as_float(wv.y) * S[c * 32 + 4 * q4 + 1];
-              y[4 * q4 + 2] = __uint_as_float(wv.z) * S[c * 32 + 4 * q4 + 2];
-              y[4 * q4 + 3] = __uint_as_float(wv.w) * S[c * 32 + 4 * q4 + 3];
+              uint64_t w01, w23;
+              lds_2x64(wrow + (c * 32 + 4 * q4) * 4, w01, w23);
+              unpack2(mul2v(w01, S2[c * 16 + 2 * q4]), y[4 * q4], y[4 * q4 + 1]);
+              unpack2(mul2v(w23, S2[c * 16 + 2 * q4 + 1]), y[4 * q4 + 2], y[4 * q4 + 3]);
             }
             const int nvalid = p.N - nc < 32 ? p.N - nc : 32;
             store_out<OUT, 32>(p.out, static_cast<int64_t>(t) * p.ldo + nc, y, nvalid);
