@@ -374,6 +374,84 @@ def kv4_quantize(kv: np.ndarray, rotate: bool = True, offset: bool = True) -> Di
 
 
 # ---------------------------------------------------------------------------
+# Key cache with a dense per-head rotation  (Sec. 3.3 Step 2 (3): U3 P3 H3)
+# ---------------------------------------------------------------------------
+#
+# With bias-induced outliers in the keys, the per-head online Hadamard H3 is
+# replaced by M = U3 P3 H3: a per-head top-1 PCA rotation U3, a permutation
+# P3 and H3 (Sec. 3.3 Step 1 (2), Step 2 (3)). It is applied to the
+# RoPE-encoded outputs of W_Q and W_K, so Q K^T is unchanged (M orthonormal),
+# and the key cache is quantized per (token, head) as before: M's last factor
+# has an all-ones first row, so the concentrated outlier leaves as the head's
+# constant offset (Eq. 5).
+
+
+def rotate_heads(x: np.ndarray, rot: np.ndarray) -> np.ndarray:
+    """y[t, h, :] = x[t, h, :] @ rot[h] for x [T, H, hd] and rot [H, hd, hd], float64."""
+    x = np.asarray(x, np.float64)
+    rot = np.asarray(rot, np.float64)
+    return np.einsum("thi,hij->thj", x, rot)
+
+
+def kv4_quantize_dense(kv: np.ndarray, rot: np.ndarray, offset: bool = True) -> Dict[str, np.ndarray]:
+    """Per-(token, head) 4-bit keys after the dense rotation: offset = mean of the
+    rotated head (Eq. 5), symmetric scale max|r| / 7, q = clamp(rne(r / s), -7, 7)."""
+    y = rotate_heads(kv, rot)
+    T, H, hd = y.shape
+    flat = y.reshape(T * H, hd)
+    o = np.array([math.fsum(r) / hd for r in flat]) if offset else np.zeros(T * H)
+    r = flat - o[:, None]
+    q, s = quantize_rows(r)
+    return {"y": y, "q": q.reshape(T, H, hd), "scale": s.reshape(T, H), "offset": o.reshape(T, H),
+            "residual": r.reshape(T, H, hd), "codes": pack_act_codes(q).reshape(T, H, hd // 2)}
+
+
+def householder_to_first(v: np.ndarray) -> np.ndarray:
+    """Symmetric orthonormal U with U e_1 = v / |v| (a reflection): a row vector k
+    rotated as k U carries k . v / |v| in channel 0, the role of U3's top-1 PCA
+    direction (Sec. 3.3 Step 1 (2))."""
+    v = np.asarray(v, np.float64)
+    v = v / np.linalg.norm(v)
+    e = np.zeros_like(v)
+    e[0] = 1.0
+    w = v - e
+    nw = np.dot(w, w)
+    if nw < 1e-30:
+        return np.eye(len(v))
+    return np.eye(len(v)) - 2.0 * np.outer(w, w) / nw
+
+
+def top1_pca_direction(x: np.ndarray) -> np.ndarray:
+    """Leading right singular vector of the (uncentred) rows of x: the top-1 PCA
+    direction of Sec. 3.3 Step 1, sign fixed so its largest entry is positive."""
+    _, _, vt = np.linalg.svd(np.asarray(x, np.float64), full_matrices=False)
+    v = vt[0]
+    return v if v[np.argmax(np.abs(v))] > 0 else -v
+
+
+def key_rotation(keys: np.ndarray, perm: Optional[np.ndarray] = None) -> np.ndarray:
+    """Per-head M = U3 P3 H3 from key samples [T, H, hd]: U3 the reflection taking
+    channel 0 to the head's top-1 PCA direction, P3 the permutation ``perm``
+    (new channel c takes old channel perm[c]; identity by default), H3 the
+    normalised Sylvester Hadamard. Returns [H, hd, hd].
+
+    P3 keeps channel 0 first: the concentrated channel must stay block-leading
+    to meet the Hadamard's all-ones first row and leave as the offset (Eq. 5,
+    group-wise offsetting of Sec. 3.2)."""
+    keys = np.asarray(keys, np.float64)
+    T, H, hd = keys.shape
+    if perm is not None and perm[0] != 0:
+        raise ValueError("P3 must keep the concentrated channel 0 first")
+    Hs = _hadamard_f64(hd) / math.sqrt(hd)
+    P = np.eye(hd)[:, perm] if perm is not None else np.eye(hd)
+    out = np.empty((H, hd, hd))
+    for h in range(H):
+        U = householder_to_first(top1_pca_direction(keys[:, h, :]))
+        out[h] = U @ P @ Hs
+    return out
+
+
+# ---------------------------------------------------------------------------
 # Per-group asymmetric activations  (Sec. 3 Eq. 1 with its zero-point; Sec. 3.2
 # footnote at Eq. 5; Sec. 4 settings: groups of 128 activations)
 # ---------------------------------------------------------------------------

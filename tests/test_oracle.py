@@ -491,3 +491,91 @@ def test_group_fp32_decisions_differ_only_at_ties():
     mism = (d != 0) & (dz == 0)
     near = np.abs(np.abs(t) - np.floor(np.abs(t)) - 0.5) < 1e-3
     assert np.all(np.abs(d) <= 1) and np.all(near[mism])
+
+
+# --------------------------------------------------------------------------
+# Key cache with a dense per-head rotation M = U3 P3 H3 (Sec. 3.3 Step 2 (3)).
+# --------------------------------------------------------------------------
+
+def _keys_with_outlier(T=96, H=2, hd=128, seed=50, mag=(20.0, 60.0)):
+    rng = np.random.default_rng(seed)
+    k = rng.standard_normal((T, H, hd))
+    dirs = rng.standard_normal((H, hd))
+    dirs /= np.linalg.norm(dirs, axis=1, keepdims=True)
+    a = rng.uniform(*mag, size=(T, H))
+    return k + a[:, :, None] * dirs[None], dirs, a
+
+
+def test_householder_and_pca_direction():
+    rng = np.random.default_rng(51)
+    v = rng.standard_normal(128)
+    U = O.householder_to_first(v)
+    np.testing.assert_allclose(U, U.T, atol=1e-15)
+    np.testing.assert_allclose(U @ U, np.eye(128), atol=1e-13)
+    np.testing.assert_allclose(U[:, 0], v / np.linalg.norm(v), atol=1e-14)
+    # Rank-one data plus tiny noise: the top-1 direction is the generating one.
+    t = rng.uniform(1, 2, size=200)
+    x = np.outer(t, v) + 1e-6 * rng.standard_normal((200, 128))
+    np.testing.assert_allclose(O.top1_pca_direction(x), v / np.linalg.norm(v) * np.sign(v[np.argmax(np.abs(v))]),
+                               atol=1e-6)
+
+
+def test_key_rotation_is_orthonormal_and_keeps_scores():
+    k, _, _ = _keys_with_outlier()
+    q = np.random.default_rng(52).standard_normal(k.shape)
+    perm = np.concatenate([[0], 1 + np.random.default_rng(53).permutation(127)])
+    M = O.key_rotation(k, perm)
+    for h in range(M.shape[0]):
+        np.testing.assert_allclose(M[h] @ M[h].T, np.eye(128), atol=1e-13)
+    qr, kr = O.rotate_heads(q, M), O.rotate_heads(k, M)
+    for h in range(M.shape[0]):
+        np.testing.assert_allclose(qr[:, h] @ kr[:, h].T, q[:, h] @ k[:, h].T, rtol=1e-11, atol=1e-9)
+
+
+def test_dense_rotation_special_cases():
+    """M = H/sqrt(hd) reproduces the per-head Hadamard quantizer; M = I the plain one."""
+    k, _, _ = _keys_with_outlier(T=40)
+    H = O.sylvester_hadamard(128).astype(np.float64) / math.sqrt(128)
+    for rot, rotate in ((np.stack([H, H]), True), (np.stack([np.eye(128)] * 2), False)):
+        a = O.kv4_quantize_dense(k, rot)
+        b = O.kv4_quantize(k, rotate=rotate)
+        np.testing.assert_allclose(a["scale"], b["scale"], rtol=1e-12)
+        np.testing.assert_allclose(a["offset"], b["offset"], rtol=1e-12, atol=1e-12)
+        t = b["residual"] / b["scale"][:, :, None]
+        near = np.abs(np.abs(t) - np.floor(np.abs(t)) - 0.5) < 1e-9
+        assert np.all((a["q"] == b["q"]) | near)
+
+
+def test_u3_turns_the_outlier_into_an_offset():
+    """k = n + a v: k U3 = n U3 + a e_1, and e_1 H3 / sqrt(hd) is constant, so
+    the rotated outlier is the offset a / sqrt(hd) (Eq. 5) and the residual
+    (hence scale and codes) does not depend on a."""
+    rng = np.random.default_rng(54)
+    T, hd = 32, 128
+    n = rng.standard_normal((T, 1, hd))
+    v = rng.standard_normal(hd)
+    v /= np.linalg.norm(v)
+    Hs = O.sylvester_hadamard(hd).astype(np.float64) / math.sqrt(hd)
+    M = (O.householder_to_first(v) @ Hs)[None]
+    base = O.kv4_quantize_dense(n, M)
+    a = rng.uniform(100, 1000, size=(T, 1))
+    spiked = O.kv4_quantize_dense(n + a[:, :, None] * v, M)
+    np.testing.assert_allclose(spiked["offset"] - base["offset"], a / math.sqrt(hd), rtol=1e-12)
+    np.testing.assert_allclose(spiked["scale"], base["scale"], rtol=1e-9)
+    # The plain per-head Hadamard leaves the outlier in the residual.
+    plain = O.kv4_quantize(n + a[:, :, None] * v, rotate=True)
+    assert np.all(plain["scale"] > 5 * spiked["scale"])
+
+
+def test_key_rotation_from_samples_offsets_the_outlier():
+    """M built from key samples (U3 from their top-1 PCA, then P3, then H3)
+    leaves the residual at the noise level; the outlier rides in the offset."""
+    k, dirs, a = _keys_with_outlier(T=256, mag=(30.0, 90.0))
+    perm = np.concatenate([[0], 1 + np.random.default_rng(55).permutation(127)])
+    M = O.key_rotation(k, perm)
+    with pytest.raises(ValueError):
+        O.key_rotation(k, np.roll(np.arange(128), 1))
+    rot = O.kv4_quantize_dense(k, M)
+    noise = O.kv4_quantize_dense(k - a[:, :, None] * dirs[None], M)
+    assert np.all(rot["scale"] < 1.5 * noise["scale"].max())
+    assert np.all(np.abs(rot["offset"]) > 0.5 * a / math.sqrt(128))
