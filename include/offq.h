@@ -19,6 +19,12 @@
  *   offq_weight_group_sums   offline: weight row sums per activation group
  *   offq_w4a4_linear_group   GEMM with per-group scales and zero-points
  *
+ * and, for keys with bias-induced outliers, the dense per-head rotation
+ * M = U3 P3 H3 in place of H3:
+ *
+ *   offq_kv4_quantize_rotated  key cache: rotate by M, then offset / scale / codes
+ *   offq_rotate_heads          queries: rotate by the same M
+ *
  * Conventions shared by every call
  *   - Pointers named as device buffers are device pointers allocated and owned
  *     by the caller. The library never allocates, frees, or synchronizes the
@@ -266,6 +272,48 @@ int offq_w4a4_linear_group(const uint8_t* a_codes, const float* a_scale, const f
                            int64_t T, int64_t N, int64_t K, int32_t group,
                            const uint8_t* w_codes, const float* w_scale, const float* w_groupsum,
                            void* out, int out_dtype, int64_t ldo, void* stream);
+
+/*
+ * Key cache under a dense per-head rotation -- paper Sec. 3.3 Step 2 (3):
+ * with bias-induced outliers in the keys, the per-head online Hadamard H3 is
+ * replaced by M = U3 P3 H3 (a per-head top-1 PCA rotation, a permutation and
+ * H3), applied to the RoPE-encoded outputs of W_Q and W_K, so Q K^T is
+ * unchanged for orthonormal M.
+ *
+ * offq_kv4_quantize_rotated -- for every (token, head) vector x of head_dim:
+ *   y = x M[h]  (fp32, input channels in order),
+ *   o = mean(y) with OFFQ_OFFSET (else 0), r = y - o, s = max|r| / 7,
+ *   q = clamp(round_half_even(r / s), -7, 7), stored as u = q + 8;
+ * the outputs of offq_kv4_quantize with M[h] in place of H3 / sqrt(head_dim).
+ *
+ *   kv        device, element (t, h, d) at kv[t*ld_token + h*head_dim + d];
+ *             16-byte aligned, ld_token * sizeof(elem) a multiple of 16,
+ *             ld_token >= H * head_dim.
+ *   T, H      tokens (>= 0) and heads (1..65535).
+ *   head_dim  128 in this build (OFFQ_ERR_UNSUPPORTED otherwise).
+ *   rot       device, [H][head_dim][head_dim] float32, row-major (y_j =
+ *             sum_i x_i rot[h][i][j]), 16-byte aligned. It is orthonormal
+ *             in the method; the call does not check that.
+ *   flags     0 or OFFQ_OFFSET.
+ *   codes     device, [T][H][head_dim/2] activation code format, 2-B aligned.
+ *   scale     device, [T][H] float32.
+ *   offset    device, [T][H] float32; required with OFFQ_OFFSET, else may be NULL.
+ */
+int offq_kv4_quantize_rotated(const void* kv, int dtype, int64_t T, int32_t H, int32_t head_dim,
+                              int64_t ld_token, const float* rot, int32_t flags,
+                              uint8_t* codes, float* scale, float* offset, void* stream);
+
+/*
+ * offq_rotate_heads -- the same y = x M[h] without quantization (the query
+ * side of the rotation), rounded once to out_dtype.
+ *
+ *   x, T, H, head_dim, ld_token, rot   as in offq_kv4_quantize_rotated.
+ *   out       device, element (t, h, d) at out[t*ld_out + h*head_dim + d] of
+ *             out_dtype; 16-byte aligned, ld_out * sizeof(out) a multiple of
+ *             16, ld_out >= H * head_dim.
+ */
+int offq_rotate_heads(const void* x, int dtype, int64_t T, int32_t H, int32_t head_dim, int64_t ld_token,
+                      const float* rot, void* out, int out_dtype, int64_t ld_out, void* stream);
 
 /* Bytes of a tiled activation-code buffer for T rows of K codes (-1 if K is
  * not a positive multiple of 32 or T < 0): ceil(T/32) * 32 * K / 2. */

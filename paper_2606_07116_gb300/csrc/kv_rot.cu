@@ -1,0 +1,267 @@
+// Key cache under a dense per-head rotation (offq_kv4_quantize_rotated) and the
+// same rotation alone for the queries (offq_rotate_heads).
+//
+// With bias-induced outliers in the keys, the per-head online Hadamard H3 is
+// replaced by M = U3 P3 H3 (paper Sec. 3.3 Step 2 (3)): y = x M for every
+// (token, head) vector x of head_dim = 128. Q and K take the same M, so Q K^T
+// is unchanged. The key cache is then quantized per (token, head) as with H3
+// (Sec. 4.2: the KV group is the head):
+//   o = mean(y) (with OFFQ_OFFSET), r = y - o, s = max|r| / 7,
+//   q = clamp(rne(r / s), -7, 7), stored as the nibble q + 8.
+//
+// One CTA takes one head and 64 tokens. M (64 KB) and the token tile,
+// transposed, are staged in shared memory; each lane accumulates 4 output
+// channels of 8 tokens in fp32 (32 FMAs per three 16-byte shared loads), in
+// input-channel order. Offset, scale and codes come from warp reductions
+// over the token's 128 outputs (4 per lane).
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include <mutex>
+#include <type_traits>
+
+#include "offq.h"
+#include "offq_device.cuh"
+#include "offq_host.h"
+
+namespace {
+
+using namespace offq;
+
+constexpr int kHd = 128;
+constexpr int kTokTile = 64;
+constexpr int kRotWarps = 8;
+constexpr int kTokPerWarp = kTokTile / kRotWarps;  // 8
+constexpr int kXPitch = kTokTile + 4;              // floats per transposed channel row
+constexpr int kRotSmem = (kHd * kHd + kHd * kXPitch) * 4;
+
+struct RotArgs {
+  const void* x;
+  int64_t ld_token;  // elements between consecutive tokens
+  int64_t T;
+  int H;
+  const float* rot;  // [H][128][128]
+  int quantize;      // 1: codes / scale / offset; 0: the rotated values
+  int offset;        // subtract the mean (quantize only)
+  uint8_t* codes;    // [T][H][64]
+  float* scale;      // [T][H]
+  float* off;        // [T][H] or nullptr
+  void* out;         // [T][ld_out] of out_dtype
+  int64_t ld_out;
+};
+
+template <typename Tin>
+__device__ __forceinline__ void load8(const Tin* src, float (&v)[8]) {
+  if constexpr (sizeof(Tin) == 4) {
+    const float4 a = __ldg(reinterpret_cast<const float4*>(src));
+    const float4 b = __ldg(reinterpret_cast<const float4*>(src) + 1);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  } else {
+    const uint4 u = __ldg(reinterpret_cast<const uint4*>(src));
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      if constexpr (std::is_same<Tin, __nv_bfloat16>::value) {
+        v[2 * k] = __uint_as_float(w[k] << 16);
+        v[2 * k + 1] = __uint_as_float(w[k] & 0xFFFF0000u);
+      } else {
+        const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w[k]));
+        v[2 * k] = f.x;
+        v[2 * k + 1] = f.y;
+      }
+    }
+  }
+}
+
+template <int OUT>
+__device__ __forceinline__ void store4(void* out, int64_t off, float a, float b, float c, float d) {
+  if constexpr (OUT == OFFQ_F32) {
+    *reinterpret_cast<float4*>(static_cast<float*>(out) + off) = make_float4(a, b, c, d);
+  } else if constexpr (OUT == OFFQ_BF16) {
+    const __nv_bfloat162 lo = __floats2bfloat162_rn(a, b), hi = __floats2bfloat162_rn(c, d);
+    *reinterpret_cast<uint2*>(static_cast<uint16_t*>(out) + off) =
+        make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi));
+  } else {
+    const __half2 lo = __floats2half2_rn(a, b), hi = __floats2half2_rn(c, d);
+    *reinterpret_cast<uint2*>(static_cast<uint16_t*>(out) + off) =
+        make_uint2(*reinterpret_cast<const uint32_t*>(&lo), *reinterpret_cast<const uint32_t*>(&hi));
+  }
+}
+
+template <typename Tin, int OUT>
+__global__ void __launch_bounds__(kRotWarps * 32) rotate_heads_kernel(const RotArgs a) {
+  extern __shared__ float4 smem4[];
+  float* Ms = reinterpret_cast<float*>(smem4);  // [128][128]
+  float* xs = Ms + kHd * kHd;                   // [128][kXPitch], x transposed
+  const int h = blockIdx.y;
+  const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kTokTile;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  griddep_wait();
+  griddep_launch_dependents();
+
+  const float4* Mg = reinterpret_cast<const float4*>(a.rot + static_cast<int64_t>(h) * kHd * kHd);
+  for (int i = tid; i < kHd * kHd / 4; i += kRotWarps * 32) smem4[i] = __ldg(Mg + i);
+  for (int c = tid; c < kTokTile * (kHd / 8); c += kRotWarps * 32) {
+    const int t = c / (kHd / 8), i0 = (c % (kHd / 8)) * 8;
+    const int64_t tok = t0 + t;
+    float v[8];
+    if (tok < a.T) {
+      load8(static_cast<const Tin*>(a.x) + tok * a.ld_token + static_cast<int64_t>(h) * kHd + i0, v);
+    } else {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) v[e] = 0.f;
+    }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) xs[(i0 + e) * kXPitch + t] = v[e];
+  }
+  __syncthreads();
+
+  // y[t][j] = sum_i x[t][i] M[i][j], i in order, for this warp's 8 tokens and
+  // this lane's outputs j = 4 lane .. 4 lane + 3.
+  float acc[kTokPerWarp][4];
+#pragma unroll
+  for (int t = 0; t < kTokPerWarp; ++t)
+#pragma unroll
+    for (int c = 0; c < 4; ++c) acc[t][c] = 0.f;
+  const float* xw = xs + warp * kTokPerWarp;
+#pragma unroll 4
+  for (int i = 0; i < kHd; ++i) {
+    const float4 m = *reinterpret_cast<const float4*>(Ms + i * kHd + 4 * lane);
+    const float4 xa = *reinterpret_cast<const float4*>(xw + i * kXPitch);
+    const float4 xb = *reinterpret_cast<const float4*>(xw + i * kXPitch + 4);
+    const float xv[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
+#pragma unroll
+    for (int t = 0; t < kTokPerWarp; ++t) {
+      acc[t][0] = fmaf(xv[t], m.x, acc[t][0]);
+      acc[t][1] = fmaf(xv[t], m.y, acc[t][1]);
+      acc[t][2] = fmaf(xv[t], m.z, acc[t][2]);
+      acc[t][3] = fmaf(xv[t], m.w, acc[t][3]);
+    }
+  }
+
+#pragma unroll
+  for (int t = 0; t < kTokPerWarp; ++t) {
+    const int64_t tok = t0 + warp * kTokPerWarp + t;
+    if (tok >= a.T) break;  // warp-uniform
+    const int64_t th = tok * a.H + h;
+    if (!a.quantize) {
+      store4<OUT>(a.out, tok * a.ld_out + static_cast<int64_t>(h) * kHd + 4 * lane, acc[t][0], acc[t][1],
+                  acc[t][2], acc[t][3]);
+      continue;
+    }
+    float o = 0.f;
+    if (a.offset) {
+      float sum = (acc[t][0] + acc[t][1]) + (acc[t][2] + acc[t][3]);
+#pragma unroll
+      for (int m = 16; m > 0; m >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, m);
+      o = sum * (1.0f / kHd);
+    }
+    const float r0 = acc[t][0] - o, r1 = acc[t][1] - o, r2 = acc[t][2] - o, r3 = acc[t][3] - o;
+    float amax = fmaxf(fmaxf(fabsf(r0), fabsf(r1)), fmaxf(fabsf(r2), fabsf(r3)));
+#pragma unroll
+    for (int m = 16; m > 0; m >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xFFFFFFFFu, amax, m));
+    const float inv = amax > 0.f ? __fdiv_rn(7.0f, amax) : 0.f;
+    const float rr[4] = {r0, r1, r2, r3};
+    uint32_t packed = 0;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const float q = fminf(fmaxf(rintf(rr[c] * inv), -7.f), 7.f);
+      packed |= static_cast<uint32_t>(static_cast<int>(q) + 8) << (4 * c);
+    }
+    *reinterpret_cast<uint16_t*>(a.codes + th * (kHd / 2) + 2 * lane) = static_cast<uint16_t>(packed);
+    if (lane == 0) {
+      a.scale[th] = amax * (1.0f / 7.0f);
+      if (a.off != nullptr) a.off[th] = o;
+    }
+  }
+}
+
+template <typename Tin, int OUT>
+int launch_rotate(const RotArgs& a, cudaStream_t s) {
+  auto kern = rotate_heads_kernel<Tin, OUT>;
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [&] {
+    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kRotSmem);
+  });
+  if (attr_err != cudaSuccess) return OFFQ_ERR_CUDA;
+  const dim3 grid(static_cast<unsigned>((a.T + kTokTile - 1) / kTokTile), static_cast<unsigned>(a.H));
+  return launch_pdl(kern, grid, dim3(kRotWarps * 32), kRotSmem, s, a);
+}
+
+template <int OUT>
+int dispatch_in(int dtype, const RotArgs& a, cudaStream_t s) {
+  switch (dtype) {
+    case OFFQ_F32: return launch_rotate<float, OUT>(a, s);
+    case OFFQ_BF16: return launch_rotate<__nv_bfloat16, OUT>(a, s);
+    case OFFQ_F16: return launch_rotate<__half, OUT>(a, s);
+    default: return OFFQ_ERR_INVALID_ARG;
+  }
+}
+
+int check_heads(const void* x, int dtype, int64_t T, int32_t H, int32_t head_dim, int64_t ld_token,
+                const float* rot) {
+  const int eb = elem_bytes(dtype);
+  if (eb == 0 || T < 0 || H < 1 || head_dim <= 0 || ld_token < static_cast<int64_t>(H) * head_dim)
+    return OFFQ_ERR_INVALID_ARG;
+  if (head_dim != kHd) return OFFQ_ERR_UNSUPPORTED;
+  if (T > 0x3FFFFFFF || H > 65535) return OFFQ_ERR_UNSUPPORTED;
+  if (T > 0 && (x == nullptr || rot == nullptr)) return OFFQ_ERR_INVALID_ARG;
+  if (T > 0 && (!aligned(x, 16) || (ld_token * eb) % 16 != 0 || !aligned(rot, 16))) return OFFQ_ERR_MISALIGNED;
+  return OFFQ_OK;
+}
+
+}  // namespace
+
+extern "C" int offq_kv4_quantize_rotated(const void* kv, int dtype, int64_t T, int32_t H, int32_t head_dim,
+                                         int64_t ld_token, const float* rot, int32_t flags, uint8_t* codes,
+                                         float* scale, float* offset, void* stream) {
+  if ((flags & ~OFFQ_OFFSET) != 0) return OFFQ_ERR_INVALID_ARG;
+  int st = check_heads(kv, dtype, T, H, head_dim, ld_token, rot);
+  if (st != OFFQ_OK) return st;
+  if (T == 0) return OFFQ_OK;
+  if (codes == nullptr || scale == nullptr || ((flags & OFFQ_OFFSET) && offset == nullptr))
+    return OFFQ_ERR_INVALID_ARG;
+  if (!aligned(codes, 2) || !aligned(scale, 4) || (offset != nullptr && !aligned(offset, 4)))
+    return OFFQ_ERR_MISALIGNED;
+  RotArgs a{};
+  a.x = kv;
+  a.ld_token = ld_token;
+  a.T = T;
+  a.H = H;
+  a.rot = rot;
+  a.quantize = 1;
+  a.offset = (flags & OFFQ_OFFSET) != 0;
+  a.codes = codes;
+  a.scale = scale;
+  a.off = offset;
+  return dispatch_in<OFFQ_F32>(dtype, a, static_cast<cudaStream_t>(stream));
+}
+
+extern "C" int offq_rotate_heads(const void* x, int dtype, int64_t T, int32_t H, int32_t head_dim, int64_t ld_token,
+                                 const float* rot, void* out, int out_dtype, int64_t ld_out, void* stream) {
+  const int ob = elem_bytes(out_dtype);
+  if (ob == 0 || ld_out < static_cast<int64_t>(H) * head_dim) return OFFQ_ERR_INVALID_ARG;
+  int st = check_heads(x, dtype, T, H, head_dim, ld_token, rot);
+  if (st != OFFQ_OK) return st;
+  if (T == 0) return OFFQ_OK;
+  if (out == nullptr) return OFFQ_ERR_INVALID_ARG;
+  if (!aligned(out, 16) || (ld_out * ob) % 16 != 0) return OFFQ_ERR_MISALIGNED;
+  RotArgs a{};
+  a.x = x;
+  a.ld_token = ld_token;
+  a.T = T;
+  a.H = H;
+  a.rot = rot;
+  a.quantize = 0;
+  a.out = out;
+  a.ld_out = ld_out;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  switch (out_dtype) {
+    case OFFQ_F32: return dispatch_in<OFFQ_F32>(dtype, a, s);
+    case OFFQ_BF16: return dispatch_in<OFFQ_BF16>(dtype, a, s);
+    case OFFQ_F16: return dispatch_in<OFFQ_F16>(dtype, a, s);
+    default: return OFFQ_ERR_INVALID_ARG;
+  }
+}

@@ -55,6 +55,10 @@ _SIGNATURES = {
     "offq_weight_group_sums": (_c_int, [_c_vp, _c_i64, _c_i64, _c_i32, _c_vp, _c_vp]),
     "offq_w4a4_linear_group": (_c_int, [_c_vp, _c_vp, _c_vp, _c_i64, _c_i64, _c_i64, _c_i32, _c_vp, _c_vp, _c_vp,
                                         _c_vp, _c_int, _c_i64, _c_vp]),
+    "offq_kv4_quantize_rotated": (_c_int, [_c_vp, _c_int, _c_i64, _c_i32, _c_i32, _c_i64, _c_vp, _c_i32, _c_vp,
+                                           _c_vp, _c_vp, _c_vp]),
+    "offq_rotate_heads": (_c_int, [_c_vp, _c_int, _c_i64, _c_i32, _c_i32, _c_i64, _c_vp, _c_vp, _c_int, _c_i64,
+                                   _c_vp]),
 }
 
 _lib = None
@@ -188,6 +192,21 @@ def offq_w4a4_linear_group(a_codes: torch.Tensor, a_scale: torch.Tensor, a_zero:
         _ptr(w_groupsum), _ptr(out), _dtype_code(out), ldo, _stream(stream)))
 
 
+def offq_kv4_quantize_rotated(kv: torch.Tensor, T: int, H: int, head_dim: int, ld_token: int, rot: torch.Tensor,
+                              flags: int, codes: torch.Tensor, scale: torch.Tensor, offset: Optional[torch.Tensor],
+                              stream=None) -> None:
+    _check("offq_kv4_quantize_rotated", load_library().offq_kv4_quantize_rotated(
+        _ptr(kv), _dtype_code(kv), T, H, head_dim, ld_token, _ptr(rot), flags, _ptr(codes), _ptr(scale),
+        _ptr(offset), _stream(stream)))
+
+
+def offq_rotate_heads(x: torch.Tensor, T: int, H: int, head_dim: int, ld_token: int, rot: torch.Tensor,
+                      out: torch.Tensor, ld_out: int, stream=None) -> None:
+    _check("offq_rotate_heads", load_library().offq_rotate_heads(
+        _ptr(x), _dtype_code(x), T, H, head_dim, ld_token, _ptr(rot), _ptr(out), _dtype_code(out), ld_out,
+        _stream(stream)))
+
+
 def offq_get_device_status(stream=None) -> int:
     return load_library().offq_get_device_status(_stream(stream))
 
@@ -291,4 +310,29 @@ def w4a4_linear_group(a_codes: torch.Tensor, a_scale: torch.Tensor, a_zero: torc
         out = torch.empty((T, N), dtype=out_dtype, device=a_codes.device)
     offq_w4a4_linear_group(a_codes, a_scale, a_zero, T, N, K, group, w_codes, w_scale, w_groupsum, out,
                            out.stride(0), stream)
+    return out
+
+
+def kv4_quantize_rotated(kv: torch.Tensor, rot: torch.Tensor, offset: bool = True,
+                         stream=None) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    """Key-cache codes, scales and offsets of kv [T, H, hd] under per-head rotations rot [H, hd, hd]."""
+    T, H, hd = kv.shape
+    if kv.stride(2) != 1 or kv.stride(1) != hd:
+        raise ValueError("heads of a token must be contiguous")
+    codes = torch.empty((T, H, hd // 2), dtype=torch.uint8, device=kv.device)
+    scale = torch.empty((T, H), dtype=torch.float32, device=kv.device)
+    off = torch.empty((T, H), dtype=torch.float32, device=kv.device)
+    offq_kv4_quantize_rotated(kv, T, H, hd, kv.stride(0), rot.contiguous(), OFFQ_OFFSET if offset else 0, codes,
+                              scale, off, stream)
+    return codes, scale, off
+
+
+def rotate_heads(x: torch.Tensor, rot: torch.Tensor, out_dtype: torch.dtype = torch.float32,
+                 stream=None) -> torch.Tensor:
+    """x [T, H, hd] rotated per head by rot [H, hd, hd] (y = x rot[h])."""
+    T, H, hd = x.shape
+    if x.stride(2) != 1 or x.stride(1) != hd:
+        raise ValueError("heads of a token must be contiguous")
+    out = torch.empty((T, H, hd), dtype=out_dtype, device=x.device)
+    offq_rotate_heads(x, T, H, hd, x.stride(0), rot.contiguous(), out, out.stride(0), stream)
     return out

@@ -143,3 +143,25 @@ def test_group_path_argument_checks(lib):
     assert lg(a=A8) == Q.OFFQ_ERR_MISALIGNED
     assert lg(ldo=65) == Q.OFFQ_ERR_MISALIGNED
     assert lg(T=0) == Q.OFFQ_OK
+
+
+def test_rotated_key_cache_argument_checks(lib):
+    kq = lambda kv=A16, dt=Q.OFFQ_BF16, T=4, H=8, hd=128, ld=1024, rot=A16, flags=2, c=A16, s=A16, o=A16: \
+        lib.offq_kv4_quantize_rotated(kv, dt, T, H, hd, ld, rot, flags, c, s, o, None)
+    assert kq(hd=64, ld=512) == Q.OFFQ_ERR_UNSUPPORTED     # this build rotates heads of 128
+    assert kq(H=0) == Q.OFFQ_ERR_INVALID_ARG
+    assert kq(ld=512) == Q.OFFQ_ERR_INVALID_ARG            # ld_token < H * head_dim
+    assert kq(flags=1) == Q.OFFQ_ERR_INVALID_ARG           # the rotation is M, not a flag
+    assert kq(rot=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert kq(o=None) == Q.OFFQ_ERR_INVALID_ARG            # OFFSET needs an offset buffer
+    assert kq(kv=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert kq(rot=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert kq(dt=7) == Q.OFFQ_ERR_INVALID_ARG
+    assert kq(T=0) == Q.OFFQ_OK
+    rh = lambda x=A16, T=4, H=8, hd=128, ld=1024, rot=A16, out=A16, odt=Q.OFFQ_F32, ldo=1024: \
+        lib.offq_rotate_heads(x, Q.OFFQ_BF16, T, H, hd, ld, rot, out, odt, ldo, None)
+    assert rh(ldo=512) == Q.OFFQ_ERR_INVALID_ARG
+    assert rh(odt=9) == Q.OFFQ_ERR_INVALID_ARG
+    assert rh(out=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert rh(out=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert rh(T=0) == Q.OFFQ_OK

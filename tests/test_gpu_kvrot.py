@@ -1,0 +1,146 @@
+"""GPU parity of the key cache under a dense per-head rotation M = U3 P3 H3
+(offq_kv4_quantize_rotated) and of the query-side rotation (offq_rotate_heads)
+against the oracle.
+
+Both sides use the same fp32 matrix M. Each rotated value is an fp32 chain of
+head_dim multiply-adds in input-channel order, so it differs from the float64
+value by at most (hd + 1) u sum_i |x_i| |M_ij|. The offset (a 128-term sum)
+and the scale inherit that bound, and a code may differ only where the
+oracle's r / s lies within the bound (in code units) of a rounding tie."""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2606_07116_gb300 import build as B
+from paper_2606_07116_gb300 import offq as Q
+from parity import U32
+
+pytestmark = pytest.mark.gpu
+
+HD = 128
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    B.build()
+    Q.load_library()
+
+
+def _keys(T, H, seed, outlier=True):
+    rng = np.random.default_rng(seed)
+    k = rng.standard_normal((T, H, HD))
+    if outlier:
+        dirs = rng.standard_normal((H, HD))
+        dirs /= np.linalg.norm(dirs, axis=1, keepdims=True)
+        k += rng.uniform(20, 80, size=(T, H, 1)) * dirs[None]
+    return k
+
+
+def _rotation(k, seed):
+    perm = np.concatenate([[0], 1 + np.random.default_rng(seed).permutation(HD - 1)])
+    return O.key_rotation(k, perm).astype(np.float32)
+
+
+def _bound_y(x, M):
+    return (HD + 1) * U32 * np.einsum("thi,hij->thj", np.abs(x), np.abs(M.astype(np.float64)))
+
+
+def _check_key_cache(codes, scale, off, x, M, offset=True):
+    T, H, _ = x.shape
+    ref = O.kv4_quantize_dense(x, M.astype(np.float64), offset=offset)
+    by = _bound_y(x, M).max(axis=2)                    # per (t, h)
+    y_abs = np.abs(ref["y"]).sum(axis=2)
+    bo = by + 8 * U32 * y_abs / HD if offset else np.zeros_like(by)
+    s_gpu, s_ref = scale.cpu().numpy().astype(np.float64), ref["scale"]
+    assert np.all(np.abs(s_gpu - s_ref) <= (by + bo) / 7 + 4 * U32 * s_ref), "scales out of bound"
+    if offset:
+        o_gpu = off.cpu().numpy().astype(np.float64)
+        assert np.all(np.abs(o_gpu - ref["offset"]) <= bo + 1e-30), "offsets out of bound"
+    q_gpu = O.unpack_act_codes(codes.cpu().numpy())
+    mism = q_gpu != ref["q"]
+    if mism.any():
+        assert np.all(np.abs(q_gpu - ref["q"])[mism] <= 1)
+        with np.errstate(divide="ignore", invalid="ignore"):
+            t = np.where(s_ref[..., None] > 0, ref["residual"] / s_ref[..., None], 0.0)
+            win = np.where(s_ref > 0, (by + bo) / s_ref, 0.0)[..., None] * 2 + 1e-6
+        dist = np.abs(np.abs(t) - np.floor(np.abs(t)) - 0.5)
+        assert np.all((dist < np.broadcast_to(win, dist.shape))[mism]), "code mismatch away from a rounding tie"
+        assert mism.sum() <= max(1, 1e-4 * mism.size)
+    return int(mism.sum())
+
+
+@pytest.mark.parametrize("dt", [torch.float32, torch.bfloat16, torch.float16])
+def test_rotated_key_cache_parity(dt):
+    T, H = 300, 8
+    k = _keys(T, H, seed=90)
+    M = _rotation(k, 91)
+    kt = torch.from_numpy(k).to(dt)
+    codes, scale, off = Q.kv4_quantize_rotated(kt.cuda(), torch.from_numpy(M).cuda())
+    torch.cuda.synchronize()
+    assert Q.offq_get_device_status() == Q.OFFQ_OK
+    _check_key_cache(codes, scale, off, kt.to(torch.float64).numpy(), M)
+
+
+def test_rotated_key_cache_ragged_and_strided():
+    """One token, 45 tokens (a partial tile), a token stride past the heads, no offset."""
+    for T in (1, 45):
+        H = 4
+        k = _keys(T, H, seed=92 + T)
+        M = _rotation(k, 93)
+        big = torch.zeros((T, H * HD + 64), dtype=torch.bfloat16)
+        big[:, :H * HD] = torch.from_numpy(k.reshape(T, H * HD)).to(torch.bfloat16)
+        dev = big.cuda()
+        codes = torch.empty((T, H, HD // 2), dtype=torch.uint8, device="cuda")
+        scale = torch.empty((T, H), dtype=torch.float32, device="cuda")
+        Q.offq_kv4_quantize_rotated(dev, T, H, HD, dev.stride(0), torch.from_numpy(M).cuda(), 0, codes, scale, None)
+        torch.cuda.synchronize()
+        x = big[:, :H * HD].to(torch.float64).numpy().reshape(T, H, HD)
+        _check_key_cache(codes, scale, None, x, M, offset=False)
+
+
+def test_hadamard_matrix_reproduces_h3_path():
+    """M = H / sqrt(128) gives the per-head Hadamard key cache (offq_kv4_quantize
+    with OFFQ_ROTATE | OFFQ_OFFSET) up to rounding ties."""
+    T, H = 64, 4
+    k = torch.from_numpy(_keys(T, H, seed=94, outlier=False)).to(torch.bfloat16).cuda()
+    Hm = (O.sylvester_hadamard(HD).astype(np.float64) / math.sqrt(HD)).astype(np.float32)
+    rot = torch.from_numpy(np.stack([Hm] * H)).cuda()
+    c1, s1, o1 = Q.kv4_quantize_rotated(k, rot)
+    c2, s2, o2 = Q.kv4_quantize(k, rotate=True, offset=True)
+    torch.cuda.synchronize()
+    np.testing.assert_allclose(s1.cpu().numpy(), s2.cpu().numpy(), rtol=1e-4)
+    np.testing.assert_allclose(o1.cpu().numpy(), o2.cpu().numpy(), rtol=1e-4, atol=1e-5)
+    q1, q2 = O.unpack_act_codes(c1.cpu().numpy()), O.unpack_act_codes(c2.cpu().numpy())
+    assert np.mean(q1 != q2) < 1e-3 and np.all(np.abs(q1 - q2) <= 1)
+
+
+@pytest.mark.parametrize("odt", [torch.float32, torch.bfloat16])
+def test_rotate_heads_parity_and_scores(odt):
+    T, H = 200, 8
+    k = _keys(T, H, seed=95)
+    q = np.random.default_rng(96).standard_normal((T, H, HD))
+    M = _rotation(k, 97)
+    qt = torch.from_numpy(q).to(torch.bfloat16)
+    y = Q.rotate_heads(qt.cuda(), torch.from_numpy(M).cuda(), out_dtype=odt)
+    torch.cuda.synchronize()
+    x = qt.to(torch.float64).numpy()
+    ref = O.rotate_heads(x, M.astype(np.float64))
+    tol = _bound_y(x, M) + (2.0 ** -8 * np.abs(ref) if odt == torch.bfloat16 else 0.0)
+    err = np.abs(y.float().cpu().numpy().astype(np.float64) - ref)
+    assert np.all(err <= tol + 1e-30), f"worst {np.max(err / (tol + 1e-30)):.3g}x the bound"
+
+
+def test_rotated_key_cache_full_size():
+    """The workload's key tensor: 2048 tokens x 32 heads."""
+    T, H = 2048, 32
+    k = _keys(T, H, seed=98)
+    M = _rotation(k, 99)
+    kt = torch.from_numpy(k).to(torch.bfloat16)
+    codes, scale, off = Q.kv4_quantize_rotated(kt.cuda(), torch.from_numpy(M).cuda())
+    torch.cuda.synchronize()
+    assert Q.offq_get_device_status() == Q.OFFQ_OK
+    _check_key_cache(codes, scale, off, kt.to(torch.float64).numpy(), M)
