@@ -395,6 +395,57 @@ def time_group_path(w, T, device, args, rank, flush_l2, barrier, stream, fp8_pea
     return gstep, dev_ms / steps, gemm_ms, quant_ms
 
 
+def time_key_rotation(w, T, device, args, flush_l2, stream, clk_mhz):
+    """The key cache under a dense per-head rotation M (U3 P3 H3 in place of H3)
+    and the query-side rotation, on the workload's key / query shapes."""
+    import torch
+    from paper_2606_07116_gb300 import offq as Q
+    H, hd = w.kv_heads, w.head_dim
+    g = torch.Generator(device="cpu").manual_seed(7)
+    # Any orthonormal M exercises the kernel identically: a seeded random one.
+    rot = torch.linalg.qr(torch.randn((H, hd, hd), generator=g, dtype=torch.float64))[0].to(torch.float32)
+    rot = rot.to(device).contiguous()
+    k = torch.randn((T, H, hd), generator=g).to(torch.bfloat16).to(device)
+    q = torch.randn((T, H, hd), generator=g).to(torch.bfloat16).to(device)
+    codes = torch.empty((T, H, hd // 2), dtype=torch.uint8, device=device)
+    scale = torch.empty((T, H), dtype=torch.float32, device=device)
+    off = torch.empty((T, H), dtype=torch.float32, device=device)
+    qo = torch.empty((T, H, hd), dtype=torch.bfloat16, device=device)
+    ts = {"k": [], "q": []}
+    for i in range(3 + max(1, min(args.steps, 50))):
+        flush_l2()
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        e[0].record(stream)
+        Q.offq_kv4_quantize_rotated(k, T, H, hd, k.stride(0), rot, Q.OFFQ_OFFSET, codes, scale, off, stream)
+        e[1].record(stream)
+        Q.offq_rotate_heads(q, T, H, hd, q.stride(0), rot, qo, qo.stride(0), stream)
+        e[2].record(stream)
+        torch.cuda.synchronize(device)
+        if i >= 3:
+            ts["k"].append(e[0].elapsed_time(e[1]))
+            ts["q"].append(e[1].elapsed_time(e[2]))
+    st = Q.offq_get_device_status(stream)
+    if st != Q.OFFQ_OK:
+        raise RuntimeError(f"device status after the key rotation: {Q.status_string(st)}")
+    k_ms = sum(ts["k"]) / len(ts["k"])
+    q_ms = sum(ts["q"]) / len(ts["q"])
+    flops = 2.0 * T * H * hd * hd
+    # fp32 FMA peak from unit counts and the clock: SMs x 128 FMA lanes x 2 flops x clock.
+    sms = torch.cuda.get_device_properties(device).multi_processor_count
+    peak = sms * 128 * 2 * clk_mhz * 1e6 / 1e12
+    kb = T * H * (hd * 2 + hd // 2 + 8)
+    return {
+        "what": "key cache under a dense per-head rotation M = U3 P3 H3 (offq_kv4_quantize_rotated) and the "
+                "query rotation (offq_rotate_heads), 2048 tokens x 32 heads x 128, bf16 in; per-call events",
+        "kv4_rotated_us": round(k_ms * 1e3, 2), "rotate_q_us": round(q_ms * 1e3, 2),
+        "kv4_rotated_gbs": round(kb / (k_ms * 1e-3) / 1e9, 1),
+        "roofline": {"bound": "alu", "kernel": "rotate_heads_kernel (fp32 FMA)",
+                     "achieved": round(flops / (k_ms * 1e-3) / 1e12, 2), "peak": round(peak, 1),
+                     "unit": "TFLOP/s", "frac": round(flops / (k_ms * 1e-3) / 1e12 / peak, 4),
+                     "peak_source": f"derived: {sms} SMs x 128 fp32 FMA lanes x 2 flops x {clk_mhz:.0f} MHz"},
+    }
+
+
 def _pair_times(events):
     return [events[i].elapsed_time(events[i + 1]) for i in range(0, len(events), 2)]
 
@@ -574,6 +625,10 @@ def run_gpu(args, rank, world, local_rank):
     }
     if group is not None:
         line["group_asym"] = group
+    if not args.no_group and w.kv_heads and w.head_dim == 128:
+        clocks = line["clocks"]
+        mhz = clocks.get("sm_mhz") or clocks.get("sm_max_mhz") or 2070.0
+        line["kv4_rotated"] = time_key_rotation(w, T, device, args, flush_l2, stream, mhz)
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
     return line

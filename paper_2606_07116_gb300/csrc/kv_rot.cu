@@ -9,11 +9,13 @@
 //   o = mean(y) (with OFFQ_OFFSET), r = y - o, s = max|r| / 7,
 //   q = clamp(rne(r / s), -7, 7), stored as the nibble q + 8.
 //
-// One CTA takes one head and 64 tokens. M (64 KB) and the token tile,
-// transposed, are staged in shared memory; each lane accumulates 4 output
-// channels of 8 tokens in fp32 (32 FMAs per three 16-byte shared loads), in
-// input-channel order. Offset, scale and codes come from warp reductions
-// over the token's 128 outputs (4 per lane).
+// A CTA takes one head and loops over 64-token tiles of it (tiles c, c +
+// gridDim.x, ...), so M (64 KB) is staged in shared memory once per CTA. Each
+// tile is staged transposed (a warp stores 32 consecutive tokens of one
+// channel: conflict-free); each lane accumulates 4 output channels of 8 tokens
+// in fp32 (32 FMAs per three 16-byte shared loads), in input-channel order.
+// Offset, scale and codes come from warp reductions over the token's 128
+// outputs (4 per lane).
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -50,16 +52,28 @@ struct RotArgs {
   int64_t ld_out;
 };
 
+// Raw 16-byte chunks of 8 channels (two for fp32 input), loaded ahead of use.
 template <typename Tin>
-__device__ __forceinline__ void load8(const Tin* src, float (&v)[8]) {
+struct Chunk8 {
+  uint4 u[sizeof(Tin) == 4 ? 2 : 1];
+};
+
+template <typename Tin>
+__device__ __forceinline__ void load_chunk(const Tin* src, bool ok, Chunk8<Tin>& c) {
+#pragma unroll
+  for (int k = 0; k < (sizeof(Tin) == 4 ? 2 : 1); ++k)
+    c.u[k] = ok ? __ldg(reinterpret_cast<const uint4*>(src) + k) : make_uint4(0u, 0u, 0u, 0u);
+}
+
+template <typename Tin>
+__device__ __forceinline__ void unpack_chunk(const Chunk8<Tin>& c, float (&v)[8]) {
   if constexpr (sizeof(Tin) == 4) {
-    const float4 a = __ldg(reinterpret_cast<const float4*>(src));
-    const float4 b = __ldg(reinterpret_cast<const float4*>(src) + 1);
-    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    v[0] = __uint_as_float(c.u[0].x); v[1] = __uint_as_float(c.u[0].y);
+    v[2] = __uint_as_float(c.u[0].z); v[3] = __uint_as_float(c.u[0].w);
+    v[4] = __uint_as_float(c.u[1].x); v[5] = __uint_as_float(c.u[1].y);
+    v[6] = __uint_as_float(c.u[1].z); v[7] = __uint_as_float(c.u[1].w);
   } else {
-    const uint4 u = __ldg(reinterpret_cast<const uint4*>(src));
-    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+    const uint32_t w[4] = {c.u[0].x, c.u[0].y, c.u[0].z, c.u[0].w};
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
       if constexpr (std::is_same<Tin, __nv_bfloat16>::value) {
@@ -95,86 +109,114 @@ __global__ void __launch_bounds__(kRotWarps * 32) rotate_heads_kernel(const RotA
   float* Ms = reinterpret_cast<float*>(smem4);  // [128][128]
   float* xs = Ms + kHd * kHd;                   // [128][kXPitch], x transposed
   const int h = blockIdx.y;
-  const int64_t t0 = static_cast<int64_t>(blockIdx.x) * kTokTile;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   griddep_wait();
   griddep_launch_dependents();
 
   const float4* Mg = reinterpret_cast<const float4*>(a.rot + static_cast<int64_t>(h) * kHd * kHd);
   for (int i = tid; i < kHd * kHd / 4; i += kRotWarps * 32) smem4[i] = __ldg(Mg + i);
-  for (int c = tid; c < kTokTile * (kHd / 8); c += kRotWarps * 32) {
-    const int t = c / (kHd / 8), i0 = (c % (kHd / 8)) * 8;
-    const int64_t tok = t0 + t;
-    float v[8];
-    if (tok < a.T) {
-      load8(static_cast<const Tin*>(a.x) + tok * a.ld_token + static_cast<int64_t>(h) * kHd + i0, v);
-    } else {
+  const int64_t tiles = (a.T + kTokTile - 1) / kTokTile;
+  // Thread tid owns chunks c = tid + 256 k of a tile: token c % 64, channels
+  // 8 (c / 64) .. + 7. The next tile's chunks are loaded while this one computes.
+  constexpr int kChunksPerThread = kTokTile * (kHd / 8) / (kRotWarps * 32);  // 4
+  Chunk8<Tin> pre[kChunksPerThread];
+  auto load_tile = [&](int64_t tile) {
 #pragma unroll
-      for (int e = 0; e < 8; ++e) v[e] = 0.f;
+    for (int k = 0; k < kChunksPerThread; ++k) {
+      const int c = tid + k * kRotWarps * 32;
+      const int64_t tok = tile * kTokTile + c % kTokTile;
+      const int i0 = (c / kTokTile) * 8;
+      load_chunk(static_cast<const Tin*>(a.x) + (tok < a.T ? tok : 0) * a.ld_token + static_cast<int64_t>(h) * kHd + i0,
+                 tok < a.T, pre[k]);
     }
+  };
+  if (static_cast<int64_t>(blockIdx.x) < tiles) load_tile(blockIdx.x);
+  for (int64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+    const int64_t t0 = tile * kTokTile;
+    __syncthreads();  // the previous tile's reads of xs are done (and M is staged)
 #pragma unroll
-    for (int e = 0; e < 8; ++e) xs[(i0 + e) * kXPitch + t] = v[e];
-  }
-  __syncthreads();
+    for (int k = 0; k < kChunksPerThread; ++k) {
+      const int c = tid + k * kRotWarps * 32;
+      const int t = c % kTokTile, i0 = (c / kTokTile) * 8;
+      float v[8];
+      unpack_chunk(pre[k], v);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) xs[(i0 + e) * kXPitch + t] = v[e];
+    }
+    __syncthreads();
+    if (tile + gridDim.x < tiles) load_tile(tile + gridDim.x);
 
-  // y[t][j] = sum_i x[t][i] M[i][j], i in order, for this warp's 8 tokens and
-  // this lane's outputs j = 4 lane .. 4 lane + 3.
-  float acc[kTokPerWarp][4];
+    // y[t][j] = sum_i x[t][i] M[i][j], i in order, for this warp's 8 tokens and
+    // this lane's outputs j = 4 lane .. 4 lane + 3.
+    float acc[kTokPerWarp][4];
 #pragma unroll
-  for (int t = 0; t < kTokPerWarp; ++t)
+    for (int t = 0; t < kTokPerWarp; ++t)
 #pragma unroll
-    for (int c = 0; c < 4; ++c) acc[t][c] = 0.f;
-  const float* xw = xs + warp * kTokPerWarp;
+      for (int c = 0; c < 4; ++c) acc[t][c] = 0.f;
+    const float* xw = xs + warp * kTokPerWarp;
 #pragma unroll 4
-  for (int i = 0; i < kHd; ++i) {
-    const float4 m = *reinterpret_cast<const float4*>(Ms + i * kHd + 4 * lane);
-    const float4 xa = *reinterpret_cast<const float4*>(xw + i * kXPitch);
-    const float4 xb = *reinterpret_cast<const float4*>(xw + i * kXPitch + 4);
-    const float xv[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
+    for (int i = 0; i < kHd; ++i) {
+      const float4 m = *reinterpret_cast<const float4*>(Ms + i * kHd + 4 * lane);
+      const float4 xa = *reinterpret_cast<const float4*>(xw + i * kXPitch);
+      const float4 xb = *reinterpret_cast<const float4*>(xw + i * kXPitch + 4);
+      const float xv[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
+#pragma unroll
+      for (int t = 0; t < kTokPerWarp; ++t) {
+        acc[t][0] = fmaf(xv[t], m.x, acc[t][0]);
+        acc[t][1] = fmaf(xv[t], m.y, acc[t][1]);
+        acc[t][2] = fmaf(xv[t], m.z, acc[t][2]);
+        acc[t][3] = fmaf(xv[t], m.w, acc[t][3]);
+      }
+    }
+
 #pragma unroll
     for (int t = 0; t < kTokPerWarp; ++t) {
-      acc[t][0] = fmaf(xv[t], m.x, acc[t][0]);
-      acc[t][1] = fmaf(xv[t], m.y, acc[t][1]);
-      acc[t][2] = fmaf(xv[t], m.z, acc[t][2]);
-      acc[t][3] = fmaf(xv[t], m.w, acc[t][3]);
+      const int64_t tok = t0 + warp * kTokPerWarp + t;
+      if (tok >= a.T) break;  // warp-uniform
+      const int64_t th = tok * a.H + h;
+      if (!a.quantize) {
+        store4<OUT>(a.out, tok * a.ld_out + static_cast<int64_t>(h) * kHd + 4 * lane, acc[t][0], acc[t][1],
+                    acc[t][2], acc[t][3]);
+        continue;
+      }
+      float o = 0.f;
+      if (a.offset) {
+        float sum = (acc[t][0] + acc[t][1]) + (acc[t][2] + acc[t][3]);
+#pragma unroll
+        for (int m = 16; m > 0; m >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, m);
+        o = sum * (1.0f / kHd);
+      }
+      const float r0 = acc[t][0] - o, r1 = acc[t][1] - o, r2 = acc[t][2] - o, r3 = acc[t][3] - o;
+      float amax = fmaxf(fmaxf(fabsf(r0), fabsf(r1)), fmaxf(fabsf(r2), fabsf(r3)));
+#pragma unroll
+      for (int m = 16; m > 0; m >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xFFFFFFFFu, amax, m));
+      const float inv = amax > 0.f ? __fdiv_rn(7.0f, amax) : 0.f;
+      const float rr[4] = {r0, r1, r2, r3};
+      uint32_t packed = 0;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const float q = fminf(fmaxf(rintf(rr[c] * inv), -7.f), 7.f);
+        packed |= static_cast<uint32_t>(static_cast<int>(q) + 8) << (4 * c);
+      }
+      *reinterpret_cast<uint16_t*>(a.codes + th * (kHd / 2) + 2 * lane) = static_cast<uint16_t>(packed);
+      if (lane == 0) {
+        a.scale[th] = amax * (1.0f / 7.0f);
+        if (a.off != nullptr) a.off[th] = o;
+      }
     }
   }
+}
 
-#pragma unroll
-  for (int t = 0; t < kTokPerWarp; ++t) {
-    const int64_t tok = t0 + warp * kTokPerWarp + t;
-    if (tok >= a.T) break;  // warp-uniform
-    const int64_t th = tok * a.H + h;
-    if (!a.quantize) {
-      store4<OUT>(a.out, tok * a.ld_out + static_cast<int64_t>(h) * kHd + 4 * lane, acc[t][0], acc[t][1],
-                  acc[t][2], acc[t][3]);
-      continue;
-    }
-    float o = 0.f;
-    if (a.offset) {
-      float sum = (acc[t][0] + acc[t][1]) + (acc[t][2] + acc[t][3]);
-#pragma unroll
-      for (int m = 16; m > 0; m >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, m);
-      o = sum * (1.0f / kHd);
-    }
-    const float r0 = acc[t][0] - o, r1 = acc[t][1] - o, r2 = acc[t][2] - o, r3 = acc[t][3] - o;
-    float amax = fmaxf(fmaxf(fabsf(r0), fabsf(r1)), fmaxf(fabsf(r2), fabsf(r3)));
-#pragma unroll
-    for (int m = 16; m > 0; m >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xFFFFFFFFu, amax, m));
-    const float inv = amax > 0.f ? __fdiv_rn(7.0f, amax) : 0.f;
-    const float rr[4] = {r0, r1, r2, r3};
-    uint32_t packed = 0;
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const float q = fminf(fmaxf(rintf(rr[c] * inv), -7.f), 7.f);
-      packed |= static_cast<uint32_t>(static_cast<int>(q) + 8) << (4 * c);
-    }
-    *reinterpret_cast<uint16_t*>(a.codes + th * (kHd / 2) + 2 * lane) = static_cast<uint16_t>(packed);
-    if (lane == 0) {
-      a.scale[th] = amax * (1.0f / 7.0f);
-      if (a.off != nullptr) a.off[th] = o;
-    }
+int rot_num_sms() {
+  static int sms[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (sms[dev] == 0) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    sms[dev] = v;
   }
+  return sms[dev];
 }
 
 template <typename Tin, int OUT>
@@ -186,7 +228,14 @@ int launch_rotate(const RotArgs& a, cudaStream_t s) {
     attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kRotSmem);
   });
   if (attr_err != cudaSuccess) return OFFQ_ERR_CUDA;
-  const dim3 grid(static_cast<unsigned>((a.T + kTokTile - 1) / kTokTile), static_cast<unsigned>(a.H));
+  // About two CTAs per SM (the shared-memory limit), spread over the heads;
+  // each loops over its head's token tiles.
+  const int sms = rot_num_sms();
+  if (sms < 1) return OFFQ_ERR_CUDA;
+  const int64_t tiles = (a.T + kTokTile - 1) / kTokTile;
+  int64_t per_head = (2 * sms + a.H - 1) / a.H;
+  if (per_head > tiles) per_head = tiles;
+  const dim3 grid(static_cast<unsigned>(per_head), static_cast<unsigned>(a.H));
   return launch_pdl(kern, grid, dim3(kRotWarps * 32), kRotSmem, s, a);
 }
 
