@@ -281,7 +281,9 @@ int offq_w4a4_linear_group(const uint8_t* a_codes, const float* a_scale, const f
  * unchanged for orthonormal M.
  *
  * offq_kv4_quantize_rotated -- for every (token, head) vector x of head_dim:
- *   y = x M[h]  (fp32, input channels in order),
+ *   y = x M[h]  with fp32 accumulation (bf16 keys: on the tensor cores with M
+ *               split into three bf16 parts, M = M1 + M2 + M3 to 24 bits; fp32
+ *               and fp16 keys: fp32 FMAs in input-channel order),
  *   o = mean(y) with OFFQ_OFFSET (else 0), r = y - o, s = max|r| / 7,
  *   q = clamp(round_half_even(r / s), -7, 7), stored as u = q + 8;
  * the outputs of offq_kv4_quantize with M[h] in place of H3 / sqrt(head_dim).
@@ -295,7 +297,7 @@ int offq_w4a4_linear_group(const uint8_t* a_codes, const float* a_scale, const f
  *             sum_i x_i rot[h][i][j]), 16-byte aligned. It is orthonormal
  *             in the method; the call does not check that.
  *   flags     0 or OFFQ_OFFSET.
- *   codes     device, [T][H][head_dim/2] activation code format, 2-B aligned.
+ *   codes     device, [T][H][head_dim/2] activation code format, 16-B aligned.
  *   scale     device, [T][H] float32.
  *   offset    device, [T][H] float32; required with OFFQ_OFFSET, else may be NULL.
  */

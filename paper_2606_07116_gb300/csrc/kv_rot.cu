@@ -9,7 +9,16 @@
 //   o = mean(y) (with OFFQ_OFFSET), r = y - o, s = max|r| / 7,
 //   q = clamp(rne(r / s), -7, 7), stored as the nibble q + 8.
 //
-// A CTA takes one head and loops over 64-token tiles of it (tiles c, c +
+// bf16 keys take the tensor cores: M is split into three bf16 parts,
+// M = M1 + M2 + M3 (24 significant bits, M's whole fp32 significand); bf16 x
+// bf16 products are exact, so y = x M1 + x M2 + x M3 accumulated in fp32 by
+// tcgen05.mma (kind::f16, M 128 tokens x N 128 outputs, K 3 x 128) keeps fp32
+// accuracy. A CTA takes one head, stages the three parts once (K-major, 128-byte
+// swizzle) and loops over 128-token tiles; in the epilogue each thread owns one
+// token's accumulator row in TMEM, so offset, scale and codes need no shuffles.
+//
+// Other input types (fp32, fp16) would lose bits in bf16 and take the FMA
+// kernel: a CTA takes one head and loops over 64-token tiles of it (tiles c, c +
 // gridDim.x, ...), so M (64 KB) is staged in shared memory once per CTA. Each
 // tile is staged transposed (a warp stores 32 consecutive tokens of one
 // channel: conflict-free); each lane accumulates 4 output channels of 8 tokens
@@ -50,6 +59,7 @@ struct RotArgs {
   float* off;        // [T][H] or nullptr
   void* out;         // [T][ld_out] of out_dtype
   int64_t ld_out;
+  int* status;       // device status word (bounded waits of the tensor-core kernel)
 };
 
 // Raw 16-byte chunks of 8 channels (two for fp32 input), loaded ahead of use.
@@ -207,6 +217,236 @@ __global__ void __launch_bounds__(kRotWarps * 32) rotate_heads_kernel(const RotA
   }
 }
 
+// ---------------------------------------------------------------------------
+// Tensor-core kernel (bf16 keys)
+// ---------------------------------------------------------------------------
+constexpr int kTM = 128;                    // tokens per MMA tile
+constexpr int kParts = 3;                   // bf16 parts of M
+constexpr int kAtomBytes = 128 * 128;       // 128 rows x 64 bf16 (one 128-byte swizzle atom column)
+constexpr int kOpBytes = 2 * kAtomBytes;    // 128 rows x 128 bf16
+constexpr int kMmaThreads = 128;
+constexpr int kMmaSmem = (kParts + 1) * kOpBytes + 64 + 1024;
+// kind::f16 instruction descriptor: D f32 (bits 4-5 = 1), A and B bf16 (bits
+// 7-9, 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
+constexpr uint32_t kIdescBf16 = (1u << 4) | (1u << 7) | (1u << 10) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n"
+      ".reg .pred p;\n"
+      "setp.ne.b32 p, %4, 0;\n"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n"
+      "}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void sts128v(uint32_t addr, uint4 v) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+               : "memory");
+}
+
+// Byte offset of 16-byte chunk c (8 bf16, c = 0..15) of row r in a 128-row
+// K-major operand: two 16 KB atom columns, 128-byte rows, chunk swizzle c ^ (r & 7).
+__device__ __forceinline__ uint32_t sw_off(int r, int c) {
+  return (c >> 3) * kAtomBytes + r * 128 + (((c & 7) ^ (r & 7)) << 4);
+}
+
+__device__ __forceinline__ uint32_t bf16_bits(float v) {
+  const __nv_bfloat16 b = __float2bfloat16_rn(v);
+  return static_cast<uint32_t>(*reinterpret_cast<const uint16_t*>(&b));
+}
+
+// m = hi + mid + lo + e with |e| <= 2^-24 |m| roughly: each part rounds what
+// the previous ones left (the differences are exact in fp32).
+__device__ __forceinline__ void split3(float m, uint32_t& hi, uint32_t& mid, uint32_t& lo) {
+  hi = bf16_bits(m);
+  const float r1 = m - __uint_as_float(hi << 16);
+  mid = bf16_bits(r1);
+  const float r2 = r1 - __uint_as_float(mid << 16);
+  lo = bf16_bits(r2);
+}
+
+template <int OUT>
+__global__ void __launch_bounds__(kMmaThreads, 1) rotate_heads_mma_kernel(const RotArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (base - raw);
+  const uint32_t b_base = base;                      // kParts operands B_s[n][k] = part s of M[k][n]
+  const uint32_t a_base = base + kParts * kOpBytes;  // the token tile
+  const uint32_t bar = a_base + kOpBytes;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + (kParts + 1) * kOpBytes + 16);
+  volatile int* abort = reinterpret_cast<volatile int*>(smem + (kParts + 1) * kOpBytes + 32);
+  const int h = blockIdx.y;
+  const int tid = threadIdx.x, warp = tid >> 5;
+  if (tid == 0) {
+    mbar_init(bar, 1);
+    *abort = 0;
+    mbar_fence_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(smem_u32(tmem_slot), kTM);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  griddep_wait();
+  griddep_launch_dependents();
+
+  // The three parts of M[h], transposed to K-major: thread n-major, so the
+  // reads of a row of M are coalesced and 8 consecutive n hit 8 distinct chunks.
+  // Thread n stages column n of M (k-chunks c = 0..15), four chunks' loads in
+  // flight at a time.
+  const float* Mh = a.rot + static_cast<int64_t>(h) * kHd * kHd;
+  const int n = tid;
+#pragma unroll 1
+  for (int c0 = 0; c0 < kHd / 8; c0 += 4) {
+    float m[4][8];
+#pragma unroll
+    for (int cc = 0; cc < 4; ++cc)
+#pragma unroll
+      for (int e = 0; e < 8; ++e) m[cc][e] = __ldg(Mh + (8 * (c0 + cc) + e) * kHd + n);
+#pragma unroll
+    for (int cc = 0; cc < 4; ++cc) {
+      uint32_t w[kParts][4];
+#pragma unroll
+      for (int e = 0; e < 8; e += 2) {
+        uint32_t h0, m0, l0, h1, m1, l1;
+        split3(m[cc][e], h0, m0, l0);
+        split3(m[cc][e + 1], h1, m1, l1);
+        w[0][e / 2] = h0 | (h1 << 16);
+        w[1][e / 2] = m0 | (m1 << 16);
+        w[2][e / 2] = l0 | (l1 << 16);
+      }
+#pragma unroll
+      for (int sp = 0; sp < kParts; ++sp)
+        sts128v(b_base + sp * kOpBytes + sw_off(n, c0 + cc), make_uint4(w[sp][0], w[sp][1], w[sp][2], w[sp][3]));
+    }
+  }
+
+  const int64_t tiles = (a.T + kTM - 1) / kTM;
+  uint32_t phase = 0;
+  const uint32_t row_tm = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+  // A tile's 16-byte chunks: thread tid takes chunks tid + 128 k (row >> 4,
+  // chunk & 15), all 16 loads in flight; the next tile's load overlaps this
+  // tile's MMAs and epilogue.
+  constexpr int kAChunks = kTM * 16 / kMmaThreads;  // 16
+  uint4 pre[kAChunks];
+  auto load_a = [&](int64_t tile) {
+#pragma unroll
+    for (int k = 0; k < kAChunks; ++k) {
+      const int idx = tid + k * kMmaThreads;
+      const int64_t tok = tile * kTM + (idx >> 4);
+      pre[k] = tok < a.T ? __ldg(reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(a.x) +
+                                                               tok * a.ld_token + static_cast<int64_t>(h) * kHd +
+                                                               8 * (idx & 15)))
+                         : make_uint4(0u, 0u, 0u, 0u);
+    }
+  };
+  if (static_cast<int64_t>(blockIdx.x) < tiles) load_a(blockIdx.x);
+  for (int64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+    const int64_t t0 = tile * kTM;
+#pragma unroll
+    for (int k = 0; k < kAChunks; ++k) {
+      const int idx = tid + k * kMmaThreads;
+      sts128v(a_base + sw_off(idx >> 4, idx & 15), pre[k]);
+    }
+    fence_proxy_async_smem();  // the operands, visible to the tensor core
+    tc_fence_before();         // and the previous tile's TMEM reads ordered before its MMAs
+    __syncthreads();
+    if (tid == 0) {
+      tc_fence_after();
+#pragma unroll
+      for (int sp = 0; sp < kParts; ++sp)
+#pragma unroll
+        for (int kk = 0; kk < kHd / 16; ++kk) {
+          const uint32_t koff = (kk >> 2) * kAtomBytes + (kk & 3) * 32;
+          mma_bf16(tmem, smem_desc_sw128(a_base + koff), smem_desc_sw128(b_base + sp * kOpBytes + koff), kIdescBf16,
+                   (sp | kk) != 0 ? 1u : 0u);
+        }
+      mma_commit(bar);
+    }
+    if (tile + gridDim.x < tiles) load_a(tile + gridDim.x);
+    mbar_wait(bar, phase, abort);
+    phase ^= 1;
+    __syncthreads();  // every thread has seen the MMAs finish, or the abort flag
+    if (*abort) break;
+    tc_fence_after();
+
+    // Epilogue: thread tid owns token t0 + tid (TMEM lane tid).
+    const int64_t tok = t0 + tid;
+    const bool ok = tok < a.T;
+    const int64_t th = tok * a.H + h;
+    if (a.quantize) {
+      float sum = 0.f;
+      if (a.offset) {
+#pragma unroll 1
+        for (int c = 0; c < kHd / 32; ++c) {
+          uint32_t v[32];
+          tmem_ld_32cols_waited(row_tm + c * 32, v);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) sum += __uint_as_float(v[j]);
+        }
+      }
+      const float o = sum * (1.0f / kHd);
+      float amax = 0.f;
+#pragma unroll 1
+      for (int c = 0; c < kHd / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld_32cols_waited(row_tm + c * 32, v);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) amax = fmaxf(amax, fabsf(__uint_as_float(v[j]) - o));
+      }
+      const float inv = amax > 0.f ? __fdiv_rn(7.0f, amax) : 0.f;
+#pragma unroll 1
+      for (int c = 0; c < kHd / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld_32cols_waited(row_tm + c * 32, v);
+        uint32_t pk[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const float q = fminf(fmaxf(rintf((__uint_as_float(v[j]) - o) * inv), -7.f), 7.f);
+          pk[j >> 3] |= static_cast<uint32_t>(static_cast<int>(q) + 8) << (4 * (j & 7));
+        }
+        if (ok) *reinterpret_cast<uint4*>(a.codes + th * (kHd / 2) + 16 * c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      }
+      if (ok) {
+        a.scale[th] = amax * (1.0f / 7.0f);
+        if (a.off != nullptr) a.off[th] = o;
+      }
+    } else {
+#pragma unroll 1
+      for (int c = 0; c < kHd / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld_32cols_waited(row_tm + c * 32, v);
+        if (ok) {
+#pragma unroll
+          for (int j = 0; j < 32; j += 4)
+            store4<OUT>(a.out, tok * a.ld_out + static_cast<int64_t>(h) * kHd + c * 32 + j, __uint_as_float(v[j]),
+                        __uint_as_float(v[j + 1]), __uint_as_float(v[j + 2]), __uint_as_float(v[j + 3]));
+        }
+      }
+    }
+  }
+  if (*abort && tid == 0) {
+    // Let MMAs still in flight finish (bounded) before tensor memory is released.
+    const long long t0 = clock64();
+    while (!mbar_try_wait(bar, phase ^ 1u) && clock64() - t0 < kWaitCycles) {
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTM);
+  }
+  if (tid == 0 && *abort && a.status != nullptr) atomicExch(a.status, kErrTimeout);
+}
+
 int rot_num_sms() {
   static int sms[64] = {};
   int dev = 0;
@@ -240,10 +480,30 @@ int launch_rotate(const RotArgs& a, cudaStream_t s) {
 }
 
 template <int OUT>
+int launch_rotate_mma(const RotArgs& a, cudaStream_t s) {
+  auto kern = rotate_heads_mma_kernel<OUT>;
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [&] {
+    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
+  });
+  if (attr_err != cudaSuccess) return OFFQ_ERR_CUDA;
+  // One CTA per SM (shared memory), spread over the heads; each loops over
+  // its head's 128-token tiles.
+  const int sms = rot_num_sms();
+  if (sms < 1) return OFFQ_ERR_CUDA;
+  const int64_t tiles = (a.T + kTM - 1) / kTM;
+  int64_t per_head = sms / a.H > 0 ? sms / a.H : 1;
+  if (per_head > tiles) per_head = tiles;
+  const dim3 grid(static_cast<unsigned>(per_head), static_cast<unsigned>(a.H));
+  return launch_pdl(kern, grid, dim3(kMmaThreads), kMmaSmem, s, a);
+}
+
+template <int OUT>
 int dispatch_in(int dtype, const RotArgs& a, cudaStream_t s) {
   switch (dtype) {
     case OFFQ_F32: return launch_rotate<float, OUT>(a, s);
-    case OFFQ_BF16: return launch_rotate<__nv_bfloat16, OUT>(a, s);
+    case OFFQ_BF16: return launch_rotate_mma<OUT>(a, s);
     case OFFQ_F16: return launch_rotate<__half, OUT>(a, s);
     default: return OFFQ_ERR_INVALID_ARG;
   }
@@ -272,7 +532,7 @@ extern "C" int offq_kv4_quantize_rotated(const void* kv, int dtype, int64_t T, i
   if (T == 0) return OFFQ_OK;
   if (codes == nullptr || scale == nullptr || ((flags & OFFQ_OFFSET) && offset == nullptr))
     return OFFQ_ERR_INVALID_ARG;
-  if (!aligned(codes, 2) || !aligned(scale, 4) || (offset != nullptr && !aligned(offset, 4)))
+  if (!aligned(codes, 16) || !aligned(scale, 4) || (offset != nullptr && !aligned(offset, 4)))
     return OFFQ_ERR_MISALIGNED;
   RotArgs a{};
   a.x = kv;
@@ -285,6 +545,7 @@ extern "C" int offq_kv4_quantize_rotated(const void* kv, int dtype, int64_t T, i
   a.codes = codes;
   a.scale = scale;
   a.off = offset;
+  a.status = device_status_ptr();
   return dispatch_in<OFFQ_F32>(dtype, a, static_cast<cudaStream_t>(stream));
 }
 
@@ -306,6 +567,7 @@ extern "C" int offq_rotate_heads(const void* x, int dtype, int64_t T, int32_t H,
   a.quantize = 0;
   a.out = out;
   a.ld_out = ld_out;
+  a.status = device_status_ptr();
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   switch (out_dtype) {
     case OFFQ_F32: return dispatch_in<OFFQ_F32>(dtype, a, s);

@@ -156,6 +156,7 @@ def test_rotated_key_cache_argument_checks(lib):
     assert kq(o=None) == Q.OFFQ_ERR_INVALID_ARG            # OFFSET needs an offset buffer
     assert kq(kv=A8) == Q.OFFQ_ERR_MISALIGNED
     assert kq(rot=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert kq(c=A8) == Q.OFFQ_ERR_MISALIGNED               # codes take 16-byte stores
     assert kq(dt=7) == Q.OFFQ_ERR_INVALID_ARG
     assert kq(T=0) == Q.OFFQ_OK
     rh = lambda x=A16, T=4, H=8, hd=128, ld=1024, rot=A16, out=A16, odt=Q.OFFQ_F32, ldo=1024: \

@@ -2,11 +2,17 @@
 (offq_kv4_quantize_rotated) and of the query-side rotation (offq_rotate_heads)
 against the oracle.
 
-Both sides use the same fp32 matrix M. Each rotated value is an fp32 chain of
-head_dim multiply-adds in input-channel order, so it differs from the float64
-value by at most (hd + 1) u sum_i |x_i| |M_ij|. The offset (a 128-term sum)
-and the scale inherit that bound, and a code may differ only where the
-oracle's r / s lies within the bound (in code units) of a rounding tie."""
+Both sides use the same fp32 matrix M.
+* fp32 / fp16 keys: each rotated value is an fp32 chain of head_dim
+  multiply-adds in input-channel order, at most (hd + 1) u sum_i |x_i| |M_ij|
+  from the float64 value.
+* bf16 keys (tensor cores): M is split into three bf16 parts (exact to 2^-24
+  relative), every bf16 x bf16 product is exact, and the 3 hd products are
+  summed in the tensor core's fp32 accumulator; allowing each addition a full
+  ulp (truncation), the bound is (2 * 3 hd + 8) u sum_i |x_i| |M_ij|. The
+  offset is then a sequential 128-term fp32 sum in one thread.
+The offset and the scale inherit the bound, and a code may differ only where
+the oracle's r / s lies within the bound (in code units) of a rounding tie."""
 
 import math
 
@@ -45,16 +51,17 @@ def _rotation(k, seed):
     return O.key_rotation(k, perm).astype(np.float32)
 
 
-def _bound_y(x, M):
-    return (HD + 1) * U32 * np.einsum("thi,hij->thj", np.abs(x), np.abs(M.astype(np.float64)))
+def _bound_y(x, M, tc=False):
+    factor = 2 * 3 * HD + 8 if tc else HD + 1
+    return factor * U32 * np.einsum("thi,hij->thj", np.abs(x), np.abs(M.astype(np.float64)))
 
 
-def _check_key_cache(codes, scale, off, x, M, offset=True):
+def _check_key_cache(codes, scale, off, x, M, offset=True, tc=False):
     T, H, _ = x.shape
     ref = O.kv4_quantize_dense(x, M.astype(np.float64), offset=offset)
-    by = _bound_y(x, M).max(axis=2)                    # per (t, h)
+    by = _bound_y(x, M, tc).max(axis=2)                # per (t, h)
     y_abs = np.abs(ref["y"]).sum(axis=2)
-    bo = by + 8 * U32 * y_abs / HD if offset else np.zeros_like(by)
+    bo = by + (HD + 2 if tc else 8) * U32 * y_abs / HD if offset else np.zeros_like(by)
     s_gpu, s_ref = scale.cpu().numpy().astype(np.float64), ref["scale"]
     assert np.all(np.abs(s_gpu - s_ref) <= (by + bo) / 7 + 4 * U32 * s_ref), "scales out of bound"
     if offset:
@@ -82,7 +89,7 @@ def test_rotated_key_cache_parity(dt):
     codes, scale, off = Q.kv4_quantize_rotated(kt.cuda(), torch.from_numpy(M).cuda())
     torch.cuda.synchronize()
     assert Q.offq_get_device_status() == Q.OFFQ_OK
-    _check_key_cache(codes, scale, off, kt.to(torch.float64).numpy(), M)
+    _check_key_cache(codes, scale, off, kt.to(torch.float64).numpy(), M, tc=dt == torch.bfloat16)
 
 
 def test_rotated_key_cache_ragged_and_strided():
@@ -99,7 +106,7 @@ def test_rotated_key_cache_ragged_and_strided():
         Q.offq_kv4_quantize_rotated(dev, T, H, HD, dev.stride(0), torch.from_numpy(M).cuda(), 0, codes, scale, None)
         torch.cuda.synchronize()
         x = big[:, :H * HD].to(torch.float64).numpy().reshape(T, H, HD)
-        _check_key_cache(codes, scale, None, x, M, offset=False)
+        _check_key_cache(codes, scale, None, x, M, offset=False, tc=True)
 
 
 def test_hadamard_matrix_reproduces_h3_path():
@@ -112,8 +119,15 @@ def test_hadamard_matrix_reproduces_h3_path():
     c1, s1, o1 = Q.kv4_quantize_rotated(k, rot)
     c2, s2, o2 = Q.kv4_quantize(k, rotate=True, offset=True)
     torch.cuda.synchronize()
-    np.testing.assert_allclose(s1.cpu().numpy(), s2.cpu().numpy(), rtol=1e-4)
-    np.testing.assert_allclose(o1.cpu().numpy(), o2.cpu().numpy(), rtol=1e-4, atol=1e-5)
+    # Both are within their own bounds of the float64 values: the tensor-core
+    # product here, the (log2 128 + 2)-stage butterfly there.
+    x = k.to(torch.float64).cpu().numpy()
+    b_tc = _bound_y(x, rot.cpu().numpy(), tc=True).max(axis=2)
+    b_fwht = (7 + 2) * U32 * np.abs(x).sum(axis=2) / math.sqrt(HD)
+    s1n, s2n = s1.cpu().numpy().astype(np.float64), s2.cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(s1n - s2n) <= 2 * (b_tc + b_fwht) / 7 + 8 * U32 * s2n)
+    o_tol = 2 * (b_tc + b_fwht) + (HD + 8) * U32 * np.abs(x).sum(axis=2) / HD
+    assert np.all(np.abs(o1.cpu().numpy() - o2.cpu().numpy()) <= o_tol)
     q1, q2 = O.unpack_act_codes(c1.cpu().numpy()), O.unpack_act_codes(c2.cpu().numpy())
     assert np.mean(q1 != q2) < 1e-3 and np.all(np.abs(q1 - q2) <= 1)
 
@@ -129,7 +143,7 @@ def test_rotate_heads_parity_and_scores(odt):
     torch.cuda.synchronize()
     x = qt.to(torch.float64).numpy()
     ref = O.rotate_heads(x, M.astype(np.float64))
-    tol = _bound_y(x, M) + (2.0 ** -8 * np.abs(ref) if odt == torch.bfloat16 else 0.0)
+    tol = _bound_y(x, M, tc=True) + (2.0 ** -8 * np.abs(ref) if odt == torch.bfloat16 else 0.0)
     err = np.abs(y.float().cpu().numpy().astype(np.float64) - ref)
     assert np.all(err <= tol + 1e-30), f"worst {np.max(err / (tol + 1e-30)):.3g}x the bound"
 
@@ -143,4 +157,4 @@ def test_rotated_key_cache_full_size():
     codes, scale, off = Q.kv4_quantize_rotated(kt.cuda(), torch.from_numpy(M).cuda())
     torch.cuda.synchronize()
     assert Q.offq_get_device_status() == Q.OFFQ_OK
-    _check_key_cache(codes, scale, off, kt.to(torch.float64).numpy(), M)
+    _check_key_cache(codes, scale, off, kt.to(torch.float64).numpy(), M, tc=True)
