@@ -395,7 +395,7 @@ def time_group_path(w, T, device, args, rank, flush_l2, barrier, stream, fp8_pea
     return gstep, dev_ms / steps, gemm_ms, quant_ms
 
 
-def time_key_rotation(w, T, device, args, flush_l2, stream, clk_mhz):
+def time_key_rotation(w, T, device, args, flush_l2, stream):
     """The key cache under a dense per-head rotation M (U3 P3 H3 in place of H3)
     and the query-side rotation, on the workload's key / query shapes."""
     import torch
@@ -430,19 +430,19 @@ def time_key_rotation(w, T, device, args, flush_l2, stream, clk_mhz):
     k_ms = sum(ts["k"]) / len(ts["k"])
     q_ms = sum(ts["q"]) / len(ts["q"])
     flops = 2.0 * T * H * hd * hd
-    # fp32 FMA peak from unit counts and the clock: SMs x 128 FMA lanes x 2 flops x clock.
-    sms = torch.cuda.get_device_properties(device).multi_processor_count
-    peak = sms * 128 * 2 * clk_mhz * 1e6 / 1e12
-    kb = T * H * (hd * 2 + hd // 2 + 8)
+    # Algorithmic bytes: bf16 keys in, 4-bit codes and fp32 scale / offset out, M read once.
+    kb = T * H * (hd * 2 + hd // 2 + 8) + H * hd * hd * 4
+    peaks = load_peaks()
+    gbs = kb / (k_ms * 1e-3) / 1e9
     return {
-        "what": "key cache under a dense per-head rotation M = U3 P3 H3 (offq_kv4_quantize_rotated) and the "
-                "query rotation (offq_rotate_heads), 2048 tokens x 32 heads x 128, bf16 in; per-call events",
+        "what": "key cache under a dense per-head rotation M = U3 P3 H3 (offq_kv4_quantize_rotated, bf16 keys on "
+                "the tensor cores with M in three bf16 parts) and the query rotation (offq_rotate_heads), "
+                f"{T} tokens x {H} heads x {hd}; per-call events",
         "kv4_rotated_us": round(k_ms * 1e3, 2), "rotate_q_us": round(q_ms * 1e3, 2),
-        "kv4_rotated_gbs": round(kb / (k_ms * 1e-3) / 1e9, 1),
-        "roofline": {"bound": "alu", "kernel": "rotate_heads_kernel (fp32 FMA)",
-                     "achieved": round(flops / (k_ms * 1e-3) / 1e12, 2), "peak": round(peak, 1),
-                     "unit": "TFLOP/s", "frac": round(flops / (k_ms * 1e-3) / 1e12 / peak, 4),
-                     "peak_source": f"derived: {sms} SMs x 128 fp32 FMA lanes x 2 flops x {clk_mhz:.0f} MHz"},
+        "rotation_tflops": round(flops / (k_ms * 1e-3) / 1e12, 2),
+        "roofline": {"bound": "hbm", "kernel": "rotate_heads_mma_kernel (tcgen05.mma kind::f16)",
+                     "achieved": round(gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": round(gbs / peaks["hbm_gbs"], 4), "bytes": kb},
     }
 
 
@@ -626,9 +626,7 @@ def run_gpu(args, rank, world, local_rank):
     if group is not None:
         line["group_asym"] = group
     if not args.no_group and w.kv_heads and w.head_dim == 128:
-        clocks = line["clocks"]
-        mhz = clocks.get("sm_mhz") or clocks.get("sm_max_mhz") or 2070.0
-        line["kv4_rotated"] = time_key_rotation(w, T, device, args, flush_l2, stream, mhz)
+        line["kv4_rotated"] = time_key_rotation(w, T, device, args, flush_l2, stream)
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
     return line
