@@ -452,6 +452,94 @@ def key_rotation(keys: np.ndarray, perm: Optional[np.ndarray] = None) -> np.ndar
 
 
 # ---------------------------------------------------------------------------
+# Offline transform builder  (Sec. 3.1 top-1 PCA; Sec. 3.2 group-wise
+# offsetting; Sec. 3.3 Steps 1-2)
+# ---------------------------------------------------------------------------
+#
+# From calibration activations [S sequences, L tokens, D channels]:
+#   1. per sequence, the token with the largest L-infinity norm (Sec. 3.1,
+#      "top-1"): X [S, D];
+#   2. the leading eigenvector v of C = X^T X / S (Eq. 6);
+#   3. U1: the reflection with U1 e_1 = v, so x U1 carries x . v in channel 0
+#      (the paper's full eigenvector matrix is read as any orthonormal U1
+#      whose first column is v: only the leading direction is concentrated);
+#   4. P1: sorted grouping of the channels of X U1 by their absolute maxima
+#      (Sec. 3.2): the G largest lead the G groups in descending order, the
+#      rest fill the groups in ascending order;
+#   5. the block Hadamard H1 of size g = D / G; the weights become W U1 P1 H1
+#      (Sec. 3.3 Step 2 (1)), so W x = (W M)(x M)^T for M = U1 P1 H1.
+
+
+def top1_tokens(x: np.ndarray):
+    """Per sequence of x [S, L, D], the token of largest max_d |x| (first on
+    ties). Returns (index [S] int64, rows [S, D] float64)."""
+    x = np.asarray(x, np.float64)
+    linf = np.max(np.abs(x), axis=2)
+    idx = np.argmax(linf, axis=1)
+    return idx, x[np.arange(x.shape[0]), idx]
+
+
+def top1_pca(X: np.ndarray):
+    """Leading eigenpair of C = X^T X / N by a symmetric eigensolver; the
+    eigenvector's sign makes its largest-magnitude entry positive."""
+    X = np.asarray(X, np.float64)
+    C = X.T @ X / X.shape[0]
+    lam, U = np.linalg.eigh(C)
+    v = U[:, -1]
+    if v[np.argmax(np.abs(v))] < 0:
+        v = -v
+    return v, lam[-1], lam[-2] if len(lam) > 1 else 0.0
+
+
+def sorted_grouping(mag: np.ndarray, G: int) -> np.ndarray:
+    """Permutation of D channels into G groups of D / G (Sec. 3.2): the G
+    largest |mag| lead the groups (largest first), the remaining channels fill
+    the groups in ascending order of |mag|. New channel c takes old channel
+    perm[c]; ties keep channel order."""
+    mag = np.abs(np.asarray(mag, np.float64))
+    D = len(mag)
+    if D % G:
+        raise ValueError("G must divide D")
+    order = np.argsort(-mag, kind="stable")
+    leaders, rest = order[:G], order[G:]
+    rest = rest[np.argsort(mag[rest], kind="stable")]
+    size = D // G
+    perm = np.empty(D, dtype=np.int64)
+    for gi in range(G):
+        perm[gi * size] = leaders[gi]
+        perm[gi * size + 1:(gi + 1) * size] = rest[gi * (size - 1):(gi + 1) * (size - 1)]
+    return perm
+
+
+def offset_basis(v: np.ndarray, perm: np.ndarray, g: int) -> np.ndarray:
+    """M = U1 P1 blockdiag(H_g) / sqrt(g) as a dense [D, D] matrix."""
+    D = len(v)
+    U = householder_to_first(v)
+    P = np.eye(D)[:, perm]
+    Hb = np.zeros((D, D))
+    Hs = _hadamard_f64(g) / math.sqrt(g)
+    for b in range(D // g):
+        Hb[b * g:(b + 1) * g, b * g:(b + 1) * g] = Hs
+    return U @ P @ Hb
+
+
+def build_offset_transform(x: np.ndarray, G: int) -> Dict[str, np.ndarray]:
+    """Steps 1-5 on calibration activations x [S, L, D]."""
+    idx, X = top1_tokens(x)
+    v, lam1, lam2 = top1_pca(X)
+    Xr = X @ householder_to_first(v)
+    perm = sorted_grouping(np.max(np.abs(Xr), axis=0), G)
+    D = x.shape[2]
+    return {"index": idx, "X": X, "v": v, "lam1": lam1, "lam2": lam2, "perm": perm,
+            "M": offset_basis(v, perm, D // G)}
+
+
+def fuse_rotation(w: np.ndarray, M: np.ndarray) -> np.ndarray:
+    """W M: the weight that meets activations rotated as x M (Sec. 3.3 Step 2 (1))."""
+    return np.asarray(w, np.float64) @ np.asarray(M, np.float64)
+
+
+# ---------------------------------------------------------------------------
 # Per-group asymmetric activations  (Sec. 3 Eq. 1 with its zero-point; Sec. 3.2
 # footnote at Eq. 5; Sec. 4 settings: groups of 128 activations)
 # ---------------------------------------------------------------------------

@@ -579,3 +579,86 @@ def test_key_rotation_from_samples_offsets_the_outlier():
     noise = O.kv4_quantize_dense(k - a[:, :, None] * dirs[None], M)
     assert np.all(rot["scale"] < 1.5 * noise["scale"].max())
     assert np.all(np.abs(rot["offset"]) > 0.5 * a / math.sqrt(128))
+
+
+# --------------------------------------------------------------------------
+# Offline transform builder (Sec. 3.1 top-1 PCA, Sec. 3.2 sorted grouping,
+# Sec. 3.3 Steps 1-2 fusion).
+# --------------------------------------------------------------------------
+
+def test_sorted_grouping_golden(golden_dir):
+    d = _load(golden_dir, "sorted_grouping.json")
+    vals = np.array(d["values"], dtype=np.float64)
+    perm = O.sorted_grouping(vals, d["groups"])
+    np.testing.assert_array_equal(vals[perm], d["sorted"])
+    assert list(vals[perm]) != d["zigzag_not_used"]
+
+
+def test_linf_selection_golden(golden_dir):
+    d = _load(golden_dir, "linf_sphere.json")
+    x = np.array([d["tokens"]])
+    idx, rows = O.top1_tokens(x)
+    assert idx[0] == d["selected"]
+    np.testing.assert_allclose(np.max(np.abs(x[0]), axis=1), d["linf"])
+    np.testing.assert_array_equal(rows[0], d["tokens"][d["selected"]])
+
+
+def test_top1_pca_rank_one_and_power_iteration():
+    """X = a v^T (+ tiny noise): the leading eigenvector is v (sign fixed) with
+    eigenvalue mean(a^2); an independent power iteration agrees."""
+    rng = np.random.default_rng(60)
+    v = rng.standard_normal(256)
+    v /= np.linalg.norm(v)
+    a = rng.uniform(5, 10, size=64)
+    X = np.outer(a, v)
+    vv, lam1, lam2 = O.top1_pca(X)
+    sign = 1.0 if v[np.argmax(np.abs(v))] > 0 else -1.0
+    np.testing.assert_allclose(vv, sign * v, atol=1e-12)
+    np.testing.assert_allclose(lam1, np.mean(a ** 2), rtol=1e-12)
+    assert abs(lam2) < 1e-9
+    Xn = X + 1e-3 * rng.standard_normal(X.shape)
+    vv, _, _ = O.top1_pca(Xn)
+    p = np.ones(256) / 16.0
+    for _ in range(200):
+        p = Xn.T @ (Xn @ p)
+        p /= np.linalg.norm(p)
+    assert abs(abs(p @ vv) - 1.0) < 1e-12
+
+
+def test_offset_basis_orthonormal_and_fusion_exact():
+    rng = np.random.default_rng(61)
+    D, G = 256, 4
+    v = rng.standard_normal(D)
+    perm = O.sorted_grouping(rng.standard_normal(D), G)
+    M = O.offset_basis(v, perm, D // G)
+    np.testing.assert_allclose(M @ M.T, np.eye(D), atol=1e-12)
+    x = rng.standard_normal((9, D))
+    w = rng.standard_normal((7, D))
+    np.testing.assert_allclose((x @ M) @ O.fuse_rotation(w, M).T, x @ w.T, rtol=1e-11, atol=1e-11)
+
+
+def test_builder_turns_the_outlier_into_group_offsets():
+    """Tokens n + a v (Sec. 3.1 structure): after M = U1 P1 H1 from the builder,
+    v lands in the leading channel of a group and leaves as that group's
+    constant offset a / sqrt(g) (Eq. 5); the residual no longer holds a."""
+    rng = np.random.default_rng(62)
+    S, L, D, G = 48, 16, 256, 4
+    v = rng.standard_normal(D)
+    v /= np.linalg.norm(v)
+    x = rng.standard_normal((S, L, D))
+    spikes = rng.integers(0, L, size=S)
+    a = rng.uniform(80, 120, size=S)
+    x[np.arange(S), spikes] += a[:, None] * v
+    res = O.build_offset_transform(x, G)
+    np.testing.assert_array_equal(res["index"], spikes)
+    assert abs(abs(res["v"] @ v) - 1.0) < 1e-3
+    g = D // G
+    Xr = res["X"] @ res["M"]
+    offs = Xr.reshape(S, G, g).mean(axis=2)
+    gi = int(np.argmax(np.abs(offs).mean(axis=0)))
+    np.testing.assert_allclose(np.abs(offs[:, gi]), (a + 0.0) / math.sqrt(g), rtol=0.05)
+    # Statistical consequence (the exact one is the offset above): the 4-bit
+    # step falls to the noise level.
+    q_before = O.quantize_act(res["X"], g, rotate=False, offset=False)["scale"]
+    q_after = O.quantize_act(Xr, g, rotate=False, offset=True)["scale"]
+    assert np.all(q_after < 0.5 * q_before) and q_after.mean() < 0.25 * q_before.mean()
