@@ -25,6 +25,9 @@
  *   offq_kv4_quantize_rotated  key cache: rotate by M, then offset / scale / codes
  *   offq_rotate_heads          queries: rotate by the same M
  *
+ * and the offline transform builder (top-1 tokens, top-1 PCA direction,
+ * reflection, sorted grouping, fusion into the weights).
+ *
  * Conventions shared by every call
  *   - Pointers named as device buffers are device pointers allocated and owned
  *     by the caller. The library never allocates, frees, or synchronizes the
@@ -316,6 +319,68 @@ int offq_kv4_quantize_rotated(const void* kv, int dtype, int64_t T, int32_t H, i
  */
 int offq_rotate_heads(const void* x, int dtype, int64_t T, int32_t H, int32_t head_dim, int64_t ld_token,
                       const float* rot, void* out, int out_dtype, int64_t ld_out, void* stream);
+
+/*
+ * Offline transform builder -- paper Sec. 3.1 (top-1 PCA), Sec. 3.2 (sorted
+ * grouping for group-wise offsetting), Sec. 3.3 Steps 1-2 (fusion). Run once
+ * per model on calibration activations; not on the inference path.
+ *
+ * offq_top1_tokens -- for each sequence s of x (L tokens of D channels), the
+ * token of largest L-infinity norm max_d |x| (Sec. 3.1 "top-1"; the first on
+ * ties): index[s], and that token as float32 in rows[s][0 .. D).
+ *   x         device, element (s, l, d) at x[s*ld_seq + l*ld_token + d] of dtype,
+ *             aligned to its element size; ld_token >= D, ld_seq >= L*ld_token.
+ *   S, L, D   sequences (>= 0), tokens (>= 1), channels (>= 1).
+ *   index     device, [S] int32.   rows  device, [S][D] float32.
+ */
+int offq_top1_tokens(const void* x, int dtype, int64_t S, int64_t L, int64_t D, int64_t ld_token,
+                     int64_t ld_seq, int32_t* index, float* rows, void* stream);
+
+/*
+ * offq_top1_direction -- the leading eigenvector of C = X^T X / N (Eq. 6) by
+ * `iters` steps of power iteration from v0: v <- X^T (X v), normalised. The
+ * result's largest-magnitude entry is positive; proj[n] = X[n] . v for the
+ * returned v (the tokens' top-1 scores). v and proj carry the iteration.
+ *   X     device, [N][D] float32 row-major.   v0  device, [D] float32 start vector.
+ *   v     device, [D] float32 (output).        proj device, [N] float32 (output).
+ */
+int offq_top1_direction(const float* X, int64_t N, int64_t D, int32_t iters, const float* v0, float* v,
+                        float* proj, void* stream);
+
+/*
+ * offq_reflect_rows -- out[r] = A[r] U1 with U1 = I - 2 w w^T / |w|^2,
+ * w = v/|v| - e_1: the symmetric reflection with U1 e_1 = v/|v|, so x U1
+ * carries x . v/|v| in channel 0 (the concentrated outlier channel).
+ *   A, out  device, [R][D] float32 (may not overlap).  v  device, [D] float32.
+ *   D <= 16384 in this build.
+ */
+int offq_reflect_rows(const float* A, int64_t R, int64_t D, const float* v, float* out, void* stream);
+
+/* offq_column_absmax -- mag[d] = max_r |A[r][d]| for A device [R][D] float32,
+ * mag device [D] float32. */
+int offq_column_absmax(const float* A, int64_t R, int64_t D, float* mag, void* stream);
+
+/*
+ * offq_sorted_grouping -- the sorted-grouping permutation of D channels into G
+ * groups of D/G (Sec. 3.2; Sec. 4 "Sorted versus Zigzag Grouping"): the G
+ * channels of largest |mag| lead the groups (largest first), the others fill
+ * the groups in ascending order of |mag|; equal magnitudes keep channel order.
+ * New channel c takes old channel perm[c]. HOST pointers (mag [D] float32,
+ * perm [D] int32); synchronous, no stream.
+ */
+int offq_sorted_grouping(const float* mag, int64_t D, int32_t G, int32_t* perm);
+
+/*
+ * offq_fuse_rotation -- out = W U1 P1 blockdiag(H_g)/sqrt(g): the weight that
+ * meets activations rotated as x U1 P1 H1 (Sec. 3.3 Step 2 (1)), so that
+ * W x = out (x U1 P1 H1)^T. U1 as in offq_reflect_rows; P1 from perm (new
+ * column c = old column perm[c]); H_g Sylvester.
+ *   W, out  device, [N][D] float32 (may not overlap).  v device [D] float32.
+ *   perm    device, [D] int32 permutation.   g  power of two dividing D.
+ *   D <= 16384 in this build.
+ */
+int offq_fuse_rotation(const float* W, int64_t N, int64_t D, const float* v, const int32_t* perm, int32_t g,
+                       float* out, void* stream);
 
 /* Bytes of a tiled activation-code buffer for T rows of K codes (-1 if K is
  * not a positive multiple of 32 or T < 0): ceil(T/32) * 32 * K / 2. */

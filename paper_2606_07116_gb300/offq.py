@@ -59,6 +59,12 @@ _SIGNATURES = {
                                            _c_vp, _c_vp, _c_vp]),
     "offq_rotate_heads": (_c_int, [_c_vp, _c_int, _c_i64, _c_i32, _c_i32, _c_i64, _c_vp, _c_vp, _c_int, _c_i64,
                                    _c_vp]),
+    "offq_top1_tokens": (_c_int, [_c_vp, _c_int, _c_i64, _c_i64, _c_i64, _c_i64, _c_i64, _c_vp, _c_vp, _c_vp]),
+    "offq_top1_direction": (_c_int, [_c_vp, _c_i64, _c_i64, _c_i32, _c_vp, _c_vp, _c_vp, _c_vp]),
+    "offq_reflect_rows": (_c_int, [_c_vp, _c_i64, _c_i64, _c_vp, _c_vp, _c_vp]),
+    "offq_column_absmax": (_c_int, [_c_vp, _c_i64, _c_i64, _c_vp, _c_vp]),
+    "offq_sorted_grouping": (_c_int, [_c_vp, _c_i64, _c_i32, _c_vp]),
+    "offq_fuse_rotation": (_c_int, [_c_vp, _c_i64, _c_i64, _c_vp, _c_vp, _c_i32, _c_vp, _c_vp]),
 }
 
 _lib = None
@@ -335,4 +341,68 @@ def rotate_heads(x: torch.Tensor, rot: torch.Tensor, out_dtype: torch.dtype = to
         raise ValueError("heads of a token must be contiguous")
     out = torch.empty((T, H, hd), dtype=out_dtype, device=x.device)
     offq_rotate_heads(x, T, H, hd, x.stride(0), rot.contiguous(), out, out.stride(0), stream)
+    return out
+
+
+# ---------------------------------------------------------------------------
+# Offline transform builder
+# ---------------------------------------------------------------------------
+
+def top1_tokens(x: torch.Tensor, stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """x [S, L, D] (contiguous tokens): per sequence the token of largest L-inf norm."""
+    S, L, D = x.shape
+    if x.stride(2) != 1:
+        raise ValueError("channels must be contiguous")
+    index = torch.empty((S,), dtype=torch.int32, device=x.device)
+    rows = torch.empty((S, D), dtype=torch.float32, device=x.device)
+    _check("offq_top1_tokens", load_library().offq_top1_tokens(
+        _ptr(x), _dtype_code(x), S, L, D, x.stride(1), x.stride(0), _ptr(index), _ptr(rows), _stream(stream)))
+    return index, rows
+
+
+def top1_direction(X: torch.Tensor, iters: int = 100, v0: Optional[torch.Tensor] = None,
+                   stream=None) -> Tuple[torch.Tensor, torch.Tensor]:
+    """Leading eigenvector of X^T X / N by power iteration (and X v)."""
+    N, D = X.shape
+    X = X.contiguous()
+    if v0 is None:
+        v0 = torch.ones((D,), dtype=torch.float32, device=X.device)
+    v = torch.empty((D,), dtype=torch.float32, device=X.device)
+    proj = torch.empty((N,), dtype=torch.float32, device=X.device)
+    _check("offq_top1_direction", load_library().offq_top1_direction(
+        _ptr(X), N, D, iters, _ptr(v0.contiguous()), _ptr(v), _ptr(proj), _stream(stream)))
+    return v, proj
+
+
+def reflect_rows(A: torch.Tensor, v: torch.Tensor, stream=None) -> torch.Tensor:
+    R, D = A.shape
+    out = torch.empty((R, D), dtype=torch.float32, device=A.device)
+    _check("offq_reflect_rows", load_library().offq_reflect_rows(
+        _ptr(A.contiguous()), R, D, _ptr(v), _ptr(out), _stream(stream)))
+    return out
+
+
+def column_absmax(A: torch.Tensor, stream=None) -> torch.Tensor:
+    R, D = A.shape
+    mag = torch.empty((D,), dtype=torch.float32, device=A.device)
+    _check("offq_column_absmax", load_library().offq_column_absmax(
+        _ptr(A.contiguous()), R, D, _ptr(mag), _stream(stream)))
+    return mag
+
+
+def sorted_grouping(mag: torch.Tensor, G: int) -> torch.Tensor:
+    """Host call: the sorted-grouping permutation (int32, on the host)."""
+    m = mag.detach().to("cpu", torch.float32).contiguous()
+    perm = torch.empty((m.numel(),), dtype=torch.int32)
+    _check("offq_sorted_grouping", load_library().offq_sorted_grouping(
+        ctypes.c_void_p(m.data_ptr()), m.numel(), G, ctypes.c_void_p(perm.data_ptr())))
+    return perm
+
+
+def fuse_rotation(W: torch.Tensor, v: torch.Tensor, perm: torch.Tensor, g: int, stream=None) -> torch.Tensor:
+    N, D = W.shape
+    out = torch.empty((N, D), dtype=torch.float32, device=W.device)
+    _check("offq_fuse_rotation", load_library().offq_fuse_rotation(
+        _ptr(W.contiguous()), N, D, _ptr(v), _ptr(perm.to(W.device, torch.int32).contiguous()), g, _ptr(out),
+        _stream(stream)))
     return out

@@ -166,3 +166,34 @@ def test_rotated_key_cache_argument_checks(lib):
     assert rh(out=None) == Q.OFFQ_ERR_INVALID_ARG
     assert rh(out=A8) == Q.OFFQ_ERR_MISALIGNED
     assert rh(T=0) == Q.OFFQ_OK
+
+
+def test_builder_argument_checks(lib):
+    assert lib.offq_top1_tokens(A16, Q.OFFQ_BF16, 4, 8, 64, 32, 512, A16, A16, None) == Q.OFFQ_ERR_INVALID_ARG
+    assert lib.offq_top1_tokens(A16, Q.OFFQ_BF16, 4, 8, 64, 64, 256, A16, A16, None) == Q.OFFQ_ERR_INVALID_ARG
+    assert lib.offq_top1_tokens(A16, Q.OFFQ_BF16, 0, 8, 64, 64, 512, None, None, None) == Q.OFFQ_OK
+    assert lib.offq_top1_direction(A16, 4, 64, 0, A16, A16, A16, None) == Q.OFFQ_ERR_INVALID_ARG
+    assert lib.offq_top1_direction(A16, 4, 64, 10, None, A16, A16, None) == Q.OFFQ_ERR_INVALID_ARG
+    assert lib.offq_reflect_rows(A16, 4, 32768, A16, A16, None) == Q.OFFQ_ERR_UNSUPPORTED
+    assert lib.offq_reflect_rows(A16, 0, 64, A16, A16, None) == Q.OFFQ_OK
+    assert lib.offq_fuse_rotation(A16, 4, 64, A16, A16, 48, A16, None) == Q.OFFQ_ERR_INVALID_ARG
+    assert lib.offq_fuse_rotation(A16, 4, 64, A16, None, 64, A16, None) == Q.OFFQ_ERR_INVALID_ARG
+    assert lib.offq_column_absmax(A16, 0, 64, A16, None) == Q.OFFQ_ERR_INVALID_ARG
+    assert lib.offq_sorted_grouping(None, 6, 2, None) == Q.OFFQ_ERR_INVALID_ARG
+
+
+def test_sorted_grouping_host_matches_oracle(lib):
+    """The host grouping is plain C++: exact against the oracle, including the
+    paper's example and ties."""
+    import numpy as np
+    import torch
+    import oracle as O
+    vals = torch.tensor([1, 2, 3, 4, 50, 60], dtype=torch.float32)
+    perm = Q.sorted_grouping(vals, 2).numpy()
+    assert list(vals.numpy()[perm]) == [60, 1, 2, 50, 3, 4]
+    rng = np.random.default_rng(70)
+    for D, G in [(256, 4), (4096, 32), (64, 1), (12, 3)]:
+        m = rng.standard_normal(D).astype(np.float32)
+        m[rng.integers(0, D, size=D // 8)] = 0.5  # ties
+        np.testing.assert_array_equal(Q.sorted_grouping(torch.from_numpy(m), G).numpy(),
+                                      O.sorted_grouping(m.astype(np.float64), G))
