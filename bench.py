@@ -446,6 +446,55 @@ def time_key_rotation(w, T, device, args, flush_l2, stream):
     }
 
 
+def time_builder(device, args, flush_l2, stream):
+    """The offline transform builder on a calibration set of 64 sequences x 512
+    tokens x 4096 channels (bf16), fusing a 11008 x 4096 weight."""
+    import torch
+    from paper_2606_07116_gb300 import offq as Q
+    S, L, D, N, G, iters = 64, 512, 4096, 11008, 1, 100
+    g = torch.Generator(device="cpu").manual_seed(11)
+    x = torch.randn((S, L, D), generator=g).to(torch.bfloat16).to(device)
+    W = (torch.randn((N, D), generator=g) * 0.02).to(device)
+    peaks = load_peaks()
+
+    def timed(fn, reps):
+        ts = []
+        for i in range(2 + reps):
+            flush_l2()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            out = fn()
+            e1.record(stream)
+            torch.cuda.synchronize(device)
+            if i >= 2:
+                ts.append(e0.elapsed_time(e1))
+        return sum(ts) / len(ts), out
+
+    reps = max(1, min(args.steps, 20))
+    tok_ms, (_, rows) = timed(lambda: Q.top1_tokens(x, stream), reps)
+    dir_ms, (v, _) = timed(lambda: Q.top1_direction(rows, iters=iters, stream=stream), max(1, reps // 4))
+    mag = Q.column_absmax(Q.reflect_rows(rows, v, stream), stream)
+    perm = Q.sorted_grouping(mag, G)
+    fuse_ms, _ = timed(lambda: Q.fuse_rotation(W, v, perm, D // G, stream), reps)
+    st = Q.offq_get_device_status(stream)
+    if st != Q.OFFQ_OK:
+        raise RuntimeError(f"device status after the builder: {Q.status_string(st)}")
+    tok_bytes = S * L * D * 2 + S * D * 4
+    fuse_bytes = 2 * N * D * 4
+    tok_gbs = tok_bytes / (tok_ms * 1e-3) / 1e9
+    return {
+        "what": f"offline transform builder: top-1 L-inf tokens of {S} x {L} x {D} bf16, {iters} power-iteration "
+                f"steps on the {S} x {D} selection, fusion of U1 P1 H1 (g = {D // G}) into a {N} x {D} fp32 weight; "
+                "per-call events",
+        "top1_tokens_us": round(tok_ms * 1e3, 2), "top1_tokens_gbs": round(tok_gbs, 1),
+        "direction_us": round(dir_ms * 1e3, 2),
+        "fuse_us": round(fuse_ms * 1e3, 2), "fuse_gbs": round(fuse_bytes / (fuse_ms * 1e-3) / 1e9, 1),
+        "roofline": {"bound": "hbm", "kernel": "top1_scan_kernel", "achieved": round(tok_gbs, 1),
+                     "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": round(tok_gbs / peaks["hbm_gbs"], 4)},
+    }
+
+
 def _pair_times(events):
     return [events[i].elapsed_time(events[i + 1]) for i in range(0, len(events), 2)]
 
@@ -627,6 +676,8 @@ def run_gpu(args, rank, world, local_rank):
         line["group_asym"] = group
     if not args.no_group and w.kv_heads and w.head_dim == 128:
         line["kv4_rotated"] = time_key_rotation(w, T, device, args, flush_l2, stream)
+    if not args.no_group:
+        line["builder"] = time_builder(device, args, flush_l2, stream)
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
     return line

@@ -34,32 +34,61 @@ __device__ __forceinline__ float to_f(Tin v) {
   else return __half2float(v);
 }
 
-constexpr int kTopThreads = 512;
+constexpr int kTopThreads = 256;
+constexpr int kTopChunks = 16;  // CTAs per sequence in the scan
 
-// One CTA per sequence: warps take tokens round-robin, each token's L-inf norm
-// is a warp max; the CTA keeps the largest (first on ties) and copies that row.
 template <typename Tin>
-__global__ void __launch_bounds__(kTopThreads) top1_tokens_kernel(const Tin* __restrict__ x, int64_t L, int64_t D,
-                                                                  int64_t ld_token, int64_t ld_seq,
-                                                                  int32_t* __restrict__ index,
-                                                                  float* __restrict__ rows) {
+__device__ __forceinline__ float absmax16b(const Tin* p) {
+  const uint4 u = __ldg(reinterpret_cast<const uint4*>(p));
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+  float m = 0.f;
+  if constexpr (sizeof(Tin) == 4) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) m = fmaxf(m, fabsf(__uint_as_float(w[k])));
+  } else {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      if constexpr (std::is_same<Tin, __nv_bfloat16>::value) {
+        m = fmaxf(m, fmaxf(fabsf(__uint_as_float(w[k] << 16)), fabsf(__uint_as_float(w[k] & 0xFFFF0000u))));
+      } else {
+        const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&w[k]));
+        m = fmaxf(m, fmaxf(fabsf(f.x), fabsf(f.y)));
+      }
+    }
+  }
+  return m;
+}
+
+// Pass 1: CTA (c, s) scans tokens c, c + kTopChunks, ... of sequence s, a warp
+// per token (16-byte loads when the rows allow them), and leaves its largest
+// L-inf norm and first token index in rows[s][2c], rows[s][2c + 1] (the output
+// rows hold the partials until pass 2 overwrites them).
+template <typename Tin>
+__global__ void __launch_bounds__(kTopThreads) top1_scan_kernel(const Tin* __restrict__ x, int64_t L, int64_t D,
+                                                                int64_t ld_token, int64_t ld_seq, int vec,
+                                                                float* __restrict__ rows) {
   __shared__ float best_v[kTopThreads / 32];
   __shared__ int64_t best_i[kTopThreads / 32];
-  __shared__ int64_t sel;
   griddep_wait();
   griddep_launch_dependents();
-  const int64_t s = blockIdx.x;
+  const int64_t s = blockIdx.y;
+  const int c = blockIdx.x;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const Tin* xs = x + s * ld_seq;
+  constexpr int kPer16 = 16 / sizeof(Tin);
   float bv = -1.f;
   int64_t bi = 0;
-  for (int64_t l = warp; l < L; l += kTopThreads / 32) {
+  for (int64_t l = c + static_cast<int64_t>(warp) * kTopChunks; l < L; l += static_cast<int64_t>(kTopChunks) * (kTopThreads / 32)) {
     const Tin* row = xs + l * ld_token;
     float m = 0.f;
-    for (int64_t d = lane; d < D; d += 32) m = fmaxf(m, fabsf(to_f(row[d])));
+    if (vec) {
+      for (int64_t d = static_cast<int64_t>(lane) * kPer16; d < D; d += 32 * kPer16) m = fmaxf(m, absmax16b(row + d));
+    } else {
+      for (int64_t d = lane; d < D; d += 32) m = fmaxf(m, fabsf(to_f(row[d])));
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, o));
-    if (m > bv) {  // tokens visited in increasing order per warp: first on ties
+    if (m > bv) {  // a warp visits its tokens in increasing order: first on ties
       bv = m;
       bi = l;
     }
@@ -77,11 +106,38 @@ __global__ void __launch_bounds__(kTopThreads) top1_tokens_kernel(const Tin* __r
         v = best_v[w];
         i = best_i[w];
       }
+    rows[s * D + 2 * c] = v;
+    rows[s * D + 2 * c + 1] = __int_as_float(static_cast<int>(i));
+  }
+}
+
+// Pass 2: per sequence, the best of the partials (first index on ties), then
+// that token copied into rows[s].
+template <typename Tin>
+__global__ void __launch_bounds__(kTopThreads) top1_pick_kernel(const Tin* __restrict__ x, int64_t L, int64_t D,
+                                                                int64_t ld_token, int64_t ld_seq,
+                                                                int32_t* __restrict__ index,
+                                                                float* __restrict__ rows) {
+  __shared__ int64_t sel;
+  griddep_wait();
+  griddep_launch_dependents();
+  const int64_t s = blockIdx.x;
+  if (threadIdx.x == 0) {
+    float v = -2.f;
+    int64_t i = 0;
+    for (int c = 0; c < kTopChunks && c < L; ++c) {
+      const float pv = rows[s * D + 2 * c];
+      const int64_t pi = __float_as_int(rows[s * D + 2 * c + 1]);
+      if (pv > v || (pv == v && pi < i)) {
+        v = pv;
+        i = pi;
+      }
+    }
     sel = i;
     index[s] = static_cast<int32_t>(i);
   }
   __syncthreads();
-  const Tin* row = xs + sel * ld_token;
+  const Tin* row = x + s * ld_seq + sel * ld_token;
   for (int64_t d = threadIdx.x; d < D; d += kTopThreads) rows[s * D + d] = to_f(row[d]);
 }
 
@@ -251,24 +307,36 @@ constexpr int64_t kMaxRowD = 16384;  // two rows of floats in shared memory
 
 extern "C" int offq_top1_tokens(const void* x, int dtype, int64_t S, int64_t L, int64_t D, int64_t ld_token,
                                 int64_t ld_seq, int32_t* index, float* rows, void* stream) {
-  if (elem_bytes(dtype) == 0 || S < 0 || L < 1 || D < 1 || ld_token < D || ld_seq < L * ld_token)
-    return OFFQ_ERR_INVALID_ARG;
-  if (L > 0x7FFFFFFF || S > 0x7FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
+  const int eb = elem_bytes(dtype);
+  if (eb == 0 || S < 0 || L < 1 || D < 1 || ld_token < D || ld_seq < L * ld_token) return OFFQ_ERR_INVALID_ARG;
+  if (D < 2 * kTopChunks) return OFFQ_ERR_UNSUPPORTED;  // the partials live in rows[s]
+  if (L > 0x7FFFFFFF || S > 65535) return OFFQ_ERR_UNSUPPORTED;
   if (S == 0) return OFFQ_OK;
   if (x == nullptr || index == nullptr || rows == nullptr) return OFFQ_ERR_INVALID_ARG;
-  if (!aligned(x, elem_bytes(dtype)) || !aligned(index, 4) || !aligned(rows, 4)) return OFFQ_ERR_MISALIGNED;
+  if (!aligned(x, eb) || !aligned(index, 4) || !aligned(rows, 4)) return OFFQ_ERR_MISALIGNED;
+  const int vec = aligned(x, 16) && (ld_token * eb) % 16 == 0 && (ld_seq * eb) % 16 == 0 && (D * eb) % 16 == 0;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  const dim3 grid(static_cast<unsigned>(S)), block(kTopThreads);
+  const dim3 scan_grid(kTopChunks, static_cast<unsigned>(S)), pick_grid(static_cast<unsigned>(S)), block(kTopThreads);
+  int rc;
   switch (dtype) {
-    case OFFQ_F32:
-      return launch_pdl(top1_tokens_kernel<float>, grid, block, 0, s, static_cast<const float*>(x), L, D, ld_token,
-                        ld_seq, index, rows);
-    case OFFQ_BF16:
-      return launch_pdl(top1_tokens_kernel<__nv_bfloat16>, grid, block, 0, s, static_cast<const __nv_bfloat16*>(x),
-                        L, D, ld_token, ld_seq, index, rows);
-    case OFFQ_F16:
-      return launch_pdl(top1_tokens_kernel<__half>, grid, block, 0, s, static_cast<const __half*>(x), L, D, ld_token,
-                        ld_seq, index, rows);
+    case OFFQ_F32: {
+      const float* p = static_cast<const float*>(x);
+      rc = launch_pdl(top1_scan_kernel<float>, scan_grid, block, 0, s, p, L, D, ld_token, ld_seq, vec, rows);
+      return rc != OFFQ_OK ? rc : launch_pdl(top1_pick_kernel<float>, pick_grid, block, 0, s, p, L, D, ld_token,
+                                             ld_seq, index, rows);
+    }
+    case OFFQ_BF16: {
+      const __nv_bfloat16* p = static_cast<const __nv_bfloat16*>(x);
+      rc = launch_pdl(top1_scan_kernel<__nv_bfloat16>, scan_grid, block, 0, s, p, L, D, ld_token, ld_seq, vec, rows);
+      return rc != OFFQ_OK ? rc : launch_pdl(top1_pick_kernel<__nv_bfloat16>, pick_grid, block, 0, s, p, L, D,
+                                             ld_token, ld_seq, index, rows);
+    }
+    case OFFQ_F16: {
+      const __half* p = static_cast<const __half*>(x);
+      rc = launch_pdl(top1_scan_kernel<__half>, scan_grid, block, 0, s, p, L, D, ld_token, ld_seq, vec, rows);
+      return rc != OFFQ_OK ? rc : launch_pdl(top1_pick_kernel<__half>, pick_grid, block, 0, s, p, L, D, ld_token,
+                                             ld_seq, index, rows);
+    }
     default: return OFFQ_ERR_INVALID_ARG;
   }
 }
