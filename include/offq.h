@@ -24,6 +24,9 @@
  *
  *   offq_kv4_quantize_rotated  key cache: rotate by M, then offset / scale / codes
  *   offq_rotate_heads          queries: rotate by the same M
+ *   offq_prepare_key_rotation  offline: M in three bf16 parts, tensor-core order
+ *   offq_kv4_quantize_prepared, offq_rotate_heads_prepared
+ *                              the two above from the prepared parts (bf16)
  *
  * and the offline transform builder (top-1 tokens, top-1 PCA direction,
  * reflection, sorted grouping, fusion into the weights).
@@ -79,6 +82,9 @@ extern "C" {
 #endif
 
 #define OFFQ_ABI_VERSION 1
+
+/* Bytes of one head's prepared rotation (offq_prepare_key_rotation). */
+#define OFFQ_KEY_ROTATION_BYTES 98304
 
 typedef enum {
   OFFQ_OK = 0,
@@ -319,6 +325,41 @@ int offq_kv4_quantize_rotated(const void* kv, int dtype, int64_t T, int32_t H, i
  */
 int offq_rotate_heads(const void* x, int dtype, int64_t T, int32_t H, int32_t head_dim, int64_t ld_token,
                       const float* rot, void* out, int out_dtype, int64_t ld_out, void* stream);
+
+/*
+ * offq_prepare_key_rotation -- offline, once per model: each M[h] split into
+ * three bf16 parts, M = M1 + M2 + M3 (M1 = bf16(M), M2 = bf16(M - M1),
+ * M3 = bf16(M - M1 - M2), differences exact in float32: the parts carry M's
+ * 24-bit significand), written in the operand order of the tensor-core
+ * kernel, which then copies a head's parts into shared memory as they are
+ * instead of splitting M in every CTA.
+ *
+ *   rot       device, as in offq_kv4_quantize_rotated.
+ *   H         heads (1..65535).   head_dim  128 in this build.
+ *   prepared  device, H * OFFQ_KEY_ROTATION_BYTES bytes, 16-byte aligned,
+ *             written. An opaque image: head h's bytes start at
+ *             h * OFFQ_KEY_ROTATION_BYTES; part s (0..2) of it is 128 rows
+ *             n of 128 bf16 M_s[k][n] (k-major), 16-byte chunks swizzled
+ *             within 128-byte rows.
+ */
+int offq_prepare_key_rotation(const float* rot, int32_t H, int32_t head_dim, void* prepared, void* stream);
+
+/*
+ * offq_kv4_quantize_prepared / offq_rotate_heads_prepared --
+ * offq_kv4_quantize_rotated and offq_rotate_heads for bf16 inputs, with M
+ * given as offq_prepare_key_rotation's image. Same arithmetic and results
+ * (the tensor-core path with M in three bf16 parts).
+ *
+ *   dtype     OFFQ_BF16 (OFFQ_ERR_UNSUPPORTED otherwise).
+ *   prepared  device, offq_prepare_key_rotation's output for the same H.
+ *   other arguments as in offq_kv4_quantize_rotated / offq_rotate_heads.
+ */
+int offq_kv4_quantize_prepared(const void* kv, int dtype, int64_t T, int32_t H, int32_t head_dim,
+                               int64_t ld_token, const void* prepared, int32_t flags,
+                               uint8_t* codes, float* scale, float* offset, void* stream);
+int offq_rotate_heads_prepared(const void* x, int dtype, int64_t T, int32_t H, int32_t head_dim,
+                               int64_t ld_token, const void* prepared, void* out, int out_dtype,
+                               int64_t ld_out, void* stream);
 
 /*
  * Offline transform builder -- paper Sec. 3.1 (top-1 PCA), Sec. 3.2 (sorted

@@ -52,6 +52,7 @@ struct RotArgs {
   int64_t T;
   int H;
   const float* rot;  // [H][128][128]
+  const void* prep;  // the prepared image (tensor-core kernel), or nullptr: split rot in the kernel
   int quantize;      // 1: codes / scale / offset; 0: the rotated values
   int offset;        // subtract the mean (quantize only)
   uint8_t* codes;    // [T][H][64]
@@ -220,12 +221,18 @@ __global__ void __launch_bounds__(kRotWarps * 32) rotate_heads_kernel(const RotA
 // ---------------------------------------------------------------------------
 // Tensor-core kernel (bf16 keys)
 // ---------------------------------------------------------------------------
-constexpr int kTM = 128;                    // tokens per MMA tile
-constexpr int kParts = 3;                   // bf16 parts of M
-constexpr int kAtomBytes = 128 * 128;       // 128 rows x 64 bf16 (one 128-byte swizzle atom column)
-constexpr int kOpBytes = 2 * kAtomBytes;    // 128 rows x 128 bf16
-constexpr int kMmaThreads = 128;
-constexpr int kMmaSmem = (kParts + 1) * kOpBytes + 64 + 1024;
+constexpr int kTM = 128;                       // tokens per MMA tile
+constexpr int kParts = 3;                      // bf16 parts of M
+constexpr int kAtomBytes = 128 * 128;          // 128 rows x 64 bf16 (one 128-byte swizzle atom column)
+constexpr int kOpBytes = 2 * kAtomBytes;       // 128 rows x 128 bf16
+constexpr int kPrepBytes = kParts * kOpBytes;  // one head's three parts
+constexpr int kWG = 4;                         // warpgroups, each with its own tile, accumulator and barrier
+constexpr int kMmaThreads = 128 * kWG;
+constexpr int kCtrlOff = kPrepBytes + kWG * kOpBytes;  // barriers, TMEM address, abort flag
+constexpr int kMmaSmem = kCtrlOff + 128 + 1024;
+static_assert(kPrepBytes == OFFQ_KEY_ROTATION_BYTES, "prepared image size");
+static_assert(kWG * 4 == kHd / 8, "each warpgroup splits four k-chunks of M");
+static_assert(kMmaSmem <= 232448, "one CTA per SM");
 // kind::f16 instruction descriptor: D f32 (bits 4-5 = 1), A and B bf16 (bits
 // 7-9, 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
 constexpr uint32_t kIdescBf16 = (1u << 4) | (1u << 7) | (1u << 10) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
@@ -245,6 +252,54 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint6
 __device__ __forceinline__ void sts128v(uint32_t addr, uint4 v) {
   asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
                : "memory");
+}
+
+// 1.5 * 2^23 + 8 and the bits of 1.5 * 2^23: fl(x + kRoundMagic) for |x| < 2^21
+// is 1.5 * 2^23 + 8 + round_half_even(x), whose bits are kRoundMagicBits + that.
+constexpr float kRoundMagic = 12582920.0f;
+constexpr uint32_t kRoundMagicBits = 0x4B400000u;
+
+__device__ __forceinline__ uint64_t add2v(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ uint64_t sub2v(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+
+// Global -> shared bulk copy (async proxy), completing `bytes` on an mbarrier.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "l"(src), "r"(bytes), "r"(bar)
+               : "memory");
+}
+
+// 16-byte global -> shared copy; src_bytes = 0 writes 16 zero bytes instead.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
+// Barrier over the 128 threads of one warpgroup (named barrier `id`).
+__device__ __forceinline__ void wg_sync(int id) { asm volatile("bar.sync %0, 128;" ::"r"(id) : "memory"); }
+
+// The same barrier, returning whether `pred` held for any of the 128 threads.
+__device__ __forceinline__ bool wg_any(int id, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n"
+      ".reg .pred p, q;\n"
+      "setp.ne.b32 p, %1, 0;\n"
+      "bar.red.or.pred q, %2, 128, p;\n"
+      "selp.u32 %0, 1, 0, q;\n"
+      "}\n"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(pred)), "r"(id)
+      : "memory");
+  return r != 0;
 }
 
 // Byte offset of 16-byte chunk c (8 bf16, c = 0..15) of row r in a 128-row
@@ -268,26 +323,79 @@ __device__ __forceinline__ void split3(float m, uint32_t& hi, uint32_t& mid, uin
   lo = bf16_bits(r2);
 }
 
+// Column n of M, k-chunks c0 .. c0 + 3 (k = 8 c0 .. 8 c0 + 31): w[cc][s] holds
+// part s of M[8 (c0 + cc) .. + 7][n] as 8 bf16. The 32 loads of a thread are
+// in flight together; across threads (consecutive n) they are coalesced.
+__device__ __forceinline__ void split_column(const float* Mh, int n, int c0, uint4 (&w)[4][kParts]) {
+  float m[4][8];
+#pragma unroll
+  for (int cc = 0; cc < 4; ++cc)
+#pragma unroll
+    for (int e = 0; e < 8; ++e) m[cc][e] = __ldg(Mh + (8 * (c0 + cc) + e) * kHd + n);
+#pragma unroll
+  for (int cc = 0; cc < 4; ++cc) {
+    uint32_t p[kParts][4];
+#pragma unroll
+    for (int e = 0; e < 8; e += 2) {
+      uint32_t h0, m0, l0, h1, m1, l1;
+      split3(m[cc][e], h0, m0, l0);
+      split3(m[cc][e + 1], h1, m1, l1);
+      p[0][e / 2] = h0 | (h1 << 16);
+      p[1][e / 2] = m0 | (m1 << 16);
+      p[2][e / 2] = l0 | (l1 << 16);
+    }
+#pragma unroll
+    for (int s = 0; s < kParts; ++s) w[cc][s] = make_uint4(p[s][0], p[s][1], p[s][2], p[s][3]);
+  }
+}
+
+// The prepared image: head h's part s at prep[h][s], B_s[n][k] = part s of
+// M[k][n] in the shared-memory operand layout (sw_off), so the tensor-core
+// kernel copies it as is. Grid (4, H) x 128 threads: thread n, k-chunks 4 bx .. + 3.
+__global__ void __launch_bounds__(128) prepare_rotation_kernel(const float* __restrict__ rot,
+                                                               uint8_t* __restrict__ prep) {
+  const int h = blockIdx.y, n = threadIdx.x, c0 = 4 * blockIdx.x;
+  griddep_wait();
+  griddep_launch_dependents();
+  uint4 w[4][kParts];
+  split_column(rot + static_cast<int64_t>(h) * kHd * kHd, n, c0, w);
+  uint8_t* dst = prep + static_cast<int64_t>(h) * kPrepBytes;
+#pragma unroll
+  for (int cc = 0; cc < 4; ++cc)
+#pragma unroll
+    for (int s = 0; s < kParts; ++s) *reinterpret_cast<uint4*>(dst + s * kOpBytes + sw_off(n, c0 + cc)) = w[cc][s];
+}
+
+// One CTA per (head, share of its tiles); four warpgroups each take every
+// fourth of the CTA's 128-token tiles with their own tile buffer, TMEM
+// accumulator (128 columns) and completion barrier, so one warpgroup's loads
+// and epilogue overlap the others' MMAs. M's three parts are staged once per
+// CTA: copied from the prepared image (one bulk copy per part) or split here.
 template <int OUT>
 __global__ void __launch_bounds__(kMmaThreads, 1) rotate_heads_mma_kernel(const RotArgs a) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* smem = smem_raw + (base - raw);
-  const uint32_t b_base = base;                      // kParts operands B_s[n][k] = part s of M[k][n]
-  const uint32_t a_base = base + kParts * kOpBytes;  // the token tile
-  const uint32_t bar = a_base + kOpBytes;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + (kParts + 1) * kOpBytes + 16);
-  volatile int* abort = reinterpret_cast<volatile int*>(smem + (kParts + 1) * kOpBytes + 32);
+  const uint32_t b_base = base;  // kParts operands B_s[n][k] = part s of M[k][n]
+  const uint32_t ctrl = base + kCtrlOff;
+  const uint32_t bar_b = ctrl;  // the prepared parts have landed
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kCtrlOff + 48);
+  volatile int* abort = reinterpret_cast<volatile int*>(smem + kCtrlOff + 56);
   const int h = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5;
+  const int wg = warp >> 2, wt = tid & 127;
+  const uint32_t a_tile = base + kPrepBytes + wg * kOpBytes;  // this warpgroup's token tile
+  const uint32_t bar = ctrl + 8 + 8 * wg;                     // its MMAs have completed
   if (tid == 0) {
-    mbar_init(bar, 1);
+    mbar_init(bar_b, 1);
+#pragma unroll
+    for (int g = 0; g < kWG; ++g) mbar_init(ctrl + 8 + 8 * g, 1);
     *abort = 0;
     mbar_fence_init();
   }
   if (warp == 0) {
-    tmem_alloc(smem_u32(tmem_slot), kTM);
+    tmem_alloc(smem_u32(tmem_slot), kWG * kTM);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -297,120 +405,132 @@ __global__ void __launch_bounds__(kMmaThreads, 1) rotate_heads_mma_kernel(const 
   griddep_wait();
   griddep_launch_dependents();
 
-  // The three parts of M[h], transposed to K-major: thread n-major, so the
-  // reads of a row of M are coalesced and 8 consecutive n hit 8 distinct chunks.
-  // Thread n stages column n of M (k-chunks c = 0..15), four chunks' loads in
-  // flight at a time.
-  const float* Mh = a.rot + static_cast<int64_t>(h) * kHd * kHd;
-  const int n = tid;
-#pragma unroll 1
-  for (int c0 = 0; c0 < kHd / 8; c0 += 4) {
-    float m[4][8];
+  const uint8_t* prep = static_cast<const uint8_t*>(a.prep);
+  if (prep != nullptr && tid == 0) {
+    mbar_arrive_expect_tx(bar_b, kPrepBytes);
 #pragma unroll
-    for (int cc = 0; cc < 4; ++cc)
-#pragma unroll
-      for (int e = 0; e < 8; ++e) m[cc][e] = __ldg(Mh + (8 * (c0 + cc) + e) * kHd + n);
-#pragma unroll
-    for (int cc = 0; cc < 4; ++cc) {
-      uint32_t w[kParts][4];
-#pragma unroll
-      for (int e = 0; e < 8; e += 2) {
-        uint32_t h0, m0, l0, h1, m1, l1;
-        split3(m[cc][e], h0, m0, l0);
-        split3(m[cc][e + 1], h1, m1, l1);
-        w[0][e / 2] = h0 | (h1 << 16);
-        w[1][e / 2] = m0 | (m1 << 16);
-        w[2][e / 2] = l0 | (l1 << 16);
-      }
-#pragma unroll
-      for (int sp = 0; sp < kParts; ++sp)
-        sts128v(b_base + sp * kOpBytes + sw_off(n, c0 + cc), make_uint4(w[sp][0], w[sp][1], w[sp][2], w[sp][3]));
-    }
+    for (int s = 0; s < kParts; ++s)
+      bulk_load(b_base + s * kOpBytes, prep + static_cast<int64_t>(h) * kPrepBytes + s * kOpBytes, kOpBytes, bar_b);
   }
 
   const int64_t tiles = (a.T + kTM - 1) / kTM;
-  uint32_t phase = 0;
-  const uint32_t row_tm = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-  // A tile's 16-byte chunks: thread tid takes chunks tid + 128 k (row >> 4,
-  // chunk & 15), all 16 loads in flight; the next tile's load overlaps this
-  // tile's MMAs and epilogue.
-  constexpr int kAChunks = kTM * 16 / kMmaThreads;  // 16
-  uint4 pre[kAChunks];
-  auto load_a = [&](int64_t tile) {
+  const int64_t stride = static_cast<int64_t>(kWG) * gridDim.x;
+  // Token tile `tile` into this warpgroup's buffer: thread wt copies 16-byte
+  // chunks wt + 128 k (row >> 4, chunk & 15); rows past T are zero-filled.
+  const __nv_bfloat16* xh = static_cast<const __nv_bfloat16*>(a.x) + static_cast<int64_t>(h) * kHd;
+  auto load_tile = [&](int64_t tile) {
 #pragma unroll
-    for (int k = 0; k < kAChunks; ++k) {
-      const int idx = tid + k * kMmaThreads;
+    for (int k = 0; k < kTM * 16 / 128; ++k) {
+      const int idx = wt + k * 128;
       const int64_t tok = tile * kTM + (idx >> 4);
-      pre[k] = tok < a.T ? __ldg(reinterpret_cast<const uint4*>(static_cast<const __nv_bfloat16*>(a.x) +
-                                                               tok * a.ld_token + static_cast<int64_t>(h) * kHd +
-                                                               8 * (idx & 15)))
-                         : make_uint4(0u, 0u, 0u, 0u);
+      const bool ok = tok < a.T;
+      const void* src = ok ? static_cast<const void*>(xh + tok * a.ld_token + 8 * (idx & 15)) : a.x;
+      cp_async16(a_tile + sw_off(idx >> 4, idx & 15), src, ok ? 16u : 0u);
     }
   };
-  if (static_cast<int64_t>(blockIdx.x) < tiles) load_a(blockIdx.x);
-  for (int64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
-    const int64_t t0 = tile * kTM;
-#pragma unroll
-    for (int k = 0; k < kAChunks; ++k) {
-      const int idx = tid + k * kMmaThreads;
-      sts128v(a_base + sw_off(idx >> 4, idx & 15), pre[k]);
-    }
-    fence_proxy_async_smem();  // the operands, visible to the tensor core
-    tc_fence_before();         // and the previous tile's TMEM reads ordered before its MMAs
-    __syncthreads();
-    if (tid == 0) {
-      tc_fence_after();
-#pragma unroll
-      for (int sp = 0; sp < kParts; ++sp)
-#pragma unroll
-        for (int kk = 0; kk < kHd / 16; ++kk) {
-          const uint32_t koff = (kk >> 2) * kAtomBytes + (kk & 3) * 32;
-          mma_bf16(tmem, smem_desc_sw128(a_base + koff), smem_desc_sw128(b_base + sp * kOpBytes + koff), kIdescBf16,
-                   (sp | kk) != 0 ? 1u : 0u);
-        }
-      mma_commit(bar);
-    }
-    if (tile + gridDim.x < tiles) load_a(tile + gridDim.x);
-    mbar_wait(bar, phase, abort);
-    phase ^= 1;
-    __syncthreads();  // every thread has seen the MMAs finish, or the abort flag
-    if (*abort) break;
-    tc_fence_after();
+  int64_t tile = blockIdx.x + static_cast<int64_t>(wg) * gridDim.x;
+  if (tile < tiles) load_tile(tile);
 
-    // Epilogue: thread tid owns token t0 + tid (TMEM lane tid).
-    const int64_t tok = t0 + tid;
+  if (prep == nullptr) {
+    // Split M[h] here while the first tiles load: thread (n = wt, warpgroup
+    // wg) stages k-chunks 4 wg .. 4 wg + 3 of column n.
+    uint4 w[4][kParts];
+    split_column(a.rot + static_cast<int64_t>(h) * kHd * kHd, wt, 4 * wg, w);
+#pragma unroll
+    for (int cc = 0; cc < 4; ++cc)
+#pragma unroll
+      for (int s = 0; s < kParts; ++s) sts128v(b_base + s * kOpBytes + sw_off(wt, 4 * wg + cc), w[cc][s]);
+    fence_proxy_async_smem();
+    __syncthreads();
+  }
+
+  bool b_ready = prep == nullptr;  // (issuing thread) the parts are in shared memory
+  bool pending = false;            // (issuing thread) MMAs committed, completion not yet seen
+  uint32_t phase = 0;
+  const uint32_t acc = tmem + wg * kTM;                                                // accumulator columns
+  const uint32_t row_tm = acc + (static_cast<uint32_t>((warp & 3) * 32) << 16);  // this warp's TMEM lanes
+  for (; tile < tiles; tile += stride) {
+    cp_async_wait_all();
+    fence_proxy_async_smem();  // the tile, visible to the tensor core
+    tc_fence_before();         // and this warpgroup's previous TMEM reads ordered before its MMAs
+    wg_sync(1 + wg);
+    if (wt == 0) {
+      if (!b_ready) b_ready = mbar_wait(bar_b, 0, abort);
+      if (b_ready) {
+        tc_fence_after();
+#pragma unroll
+        for (int sp = 0; sp < kParts; ++sp)
+#pragma unroll
+          for (int kk = 0; kk < kHd / 16; ++kk) {
+            const uint32_t koff = (kk >> 2) * kAtomBytes + (kk & 3) * 32;
+            mma_bf16(acc, smem_desc_sw128(a_tile + koff), smem_desc_sw128(b_base + sp * kOpBytes + koff), kIdescBf16,
+                     (sp | kk) != 0 ? 1u : 0u);
+          }
+        mma_commit(bar);
+        pending = true;
+      }
+    }
+    const bool done = mbar_wait(bar, phase, abort);
+    if (wt == 0 && done) pending = false;
+    if (wg_any(1 + wg, !done)) break;  // the whole warpgroup leaves together
+    phase ^= 1;
+    tc_fence_after();
+    // The MMAs have read the tile buffer: the next tile's copies overlap this epilogue.
+    if (tile + stride < tiles) load_tile(tile + stride);
+
+    // Epilogue: thread wt owns token t0 + wt (TMEM lane wt of the accumulator).
+    const int64_t tok = tile * kTM + wt;
     const bool ok = tok < a.T;
     const int64_t th = tok * a.H + h;
     if (a.quantize) {
-      float sum = 0.f;
-      if (a.offset) {
+      // Pass 1: the offset (two fp32 partial sums, lanes of one f32x2 add)
+      // and the extremes of y.
+      uint64_t sum2 = pack2(0.f, 0.f);
+      float ymax0 = -INFINITY, ymax1 = -INFINITY, ymin0 = INFINITY, ymin1 = INFINITY;
 #pragma unroll 1
-        for (int c = 0; c < kHd / 32; ++c) {
-          uint32_t v[32];
-          tmem_ld_32cols_waited(row_tm + c * 32, v);
+      for (int c = 0; c < kHd / 32; ++c) {
+        uint32_t v[32];
+        tmem_ld_32cols_waited(row_tm + c * 32, v);
 #pragma unroll
-          for (int j = 0; j < 32; ++j) sum += __uint_as_float(v[j]);
+        for (int j = 0; j < 32; j += 2) {
+          const float y0 = __uint_as_float(v[j]), y1 = __uint_as_float(v[j + 1]);
+          sum2 = add2v(sum2, pack2(y0, y1));
+          ymax0 = fmaxf(ymax0, y0);
+          ymax1 = fmaxf(ymax1, y1);
+          ymin0 = fminf(ymin0, y0);
+          ymin1 = fminf(ymin1, y1);
         }
       }
-      const float o = sum * (1.0f / kHd);
-      float amax = 0.f;
-#pragma unroll 1
-      for (int c = 0; c < kHd / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld_32cols_waited(row_tm + c * 32, v);
-#pragma unroll
-        for (int j = 0; j < 32; ++j) amax = fmaxf(amax, fabsf(__uint_as_float(v[j]) - o));
-      }
+      float s0, s1;
+      unpack2(sum2, s0, s1);
+      const float o = a.offset ? (s0 + s1) * (1.0f / kHd) : 0.f;
+      // max_j |fl(y_j - o)| from the extremes: rounding is monotone and
+      // fl(o - y) = -fl(y - o), so the largest are fl(ymax - o) and fl(o - ymin).
+      const float amax = fmaxf(fmaxf(ymax0, ymax1) - o, o - fminf(ymin0, ymin1));
       const float inv = amax > 0.f ? __fdiv_rn(7.0f, amax) : 0.f;
+      // Pass 2: q = rne(fl(fl(y - o) * inv)). |fl(y - o)| <= amax and
+      // inv <= (7 / amax)(1 + 2^-24), so |q| <= 7 and the clamp to [-7, 7]
+      // never binds. Adding 1.5 * 2^23 + 8 rounds to the nearest even integer
+      // (the float spacing there is 1) and leaves u = q + 8 in the low bits of
+      // the sum; eight of them are packed with shifts and one bias subtraction.
+      const uint64_t o2 = pack2(o, o), inv2 = pack2(inv, inv), magic2 = pack2(kRoundMagic, kRoundMagic);
 #pragma unroll 1
       for (int c = 0; c < kHd / 32; ++c) {
         uint32_t v[32];
         tmem_ld_32cols_waited(row_tm + c * 32, v);
-        uint32_t pk[4] = {0u, 0u, 0u, 0u};
+        uint32_t pk[4];
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const float q = fminf(fmaxf(rintf((__uint_as_float(v[j]) - o) * inv), -7.f), 7.f);
-          pk[j >> 3] |= static_cast<uint32_t>(static_cast<int>(q) + 8) << (4 * (j & 7));
+        for (int w8 = 0; w8 < 4; ++w8) {
+          uint32_t word = 0u;
+#pragma unroll
+          for (int j = 8 * w8 + 6; j >= 8 * w8; j -= 2) {
+            const uint64_t r2 = sub2v(pack2(__uint_as_float(v[j]), __uint_as_float(v[j + 1])), o2);
+            float f0, f1;
+            unpack2(add2v(mul2v(r2, inv2), magic2), f0, f1);
+            word = (word << 4) + __float_as_uint(f1);
+            word = (word << 4) + __float_as_uint(f0);
+          }
+          pk[w8] = word - kRoundMagicBits * 0x11111111u;
         }
         if (ok) *reinterpret_cast<uint4*>(a.codes + th * (kHd / 2) + 16 * c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
       }
@@ -432,17 +552,25 @@ __global__ void __launch_bounds__(kMmaThreads, 1) rotate_heads_mma_kernel(const 
       }
     }
   }
-  if (*abort && tid == 0) {
-    // Let MMAs still in flight finish (bounded) before tensor memory is released.
-    const long long t0 = clock64();
-    while (!mbar_try_wait(bar, phase ^ 1u) && clock64() - t0 < kWaitCycles) {
+  cp_async_wait_all();  // no copy into shared memory outlives the CTA
+  if (wt == 0 && pending) {
+    // A wait ran out with MMAs in flight: let them finish (bounded) before
+    // tensor memory is released.
+    const long long c0 = clock64();
+    while (!mbar_try_wait(bar, phase) && clock64() - c0 < kWaitCycles) {
+    }
+  }
+  if (tid == 0 && !b_ready) {
+    // Likewise the bulk copy of the prepared parts.
+    const long long c0 = clock64();
+    while (!mbar_try_wait(bar_b, 0) && clock64() - c0 < kWaitCycles) {
     }
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
     tc_fence_after();
-    tmem_dealloc(tmem, kTM);
+    tmem_dealloc(tmem, kWG * kTM);
   }
   if (tid == 0 && *abort && a.status != nullptr) atomicExch(a.status, kErrTimeout);
 }
@@ -488,8 +616,8 @@ int launch_rotate_mma(const RotArgs& a, cudaStream_t s) {
     attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
   });
   if (attr_err != cudaSuccess) return OFFQ_ERR_CUDA;
-  // One CTA per SM (shared memory), spread over the heads; each loops over
-  // its head's 128-token tiles.
+  // One CTA per SM (shared memory), spread over the heads; each takes every
+  // gridDim.x-th of its head's 128-token tiles.
   const int sms = rot_num_sms();
   if (sms < 1) return OFFQ_ERR_CUDA;
   const int64_t tiles = (a.T + kTM - 1) / kTM;
@@ -510,7 +638,7 @@ int dispatch_in(int dtype, const RotArgs& a, cudaStream_t s) {
 }
 
 int check_heads(const void* x, int dtype, int64_t T, int32_t H, int32_t head_dim, int64_t ld_token,
-                const float* rot) {
+                const void* rot) {
   const int eb = elem_bytes(dtype);
   if (eb == 0 || T < 0 || H < 1 || head_dim <= 0 || ld_token < static_cast<int64_t>(H) * head_dim)
     return OFFQ_ERR_INVALID_ARG;
@@ -573,6 +701,74 @@ extern "C" int offq_rotate_heads(const void* x, int dtype, int64_t T, int32_t H,
     case OFFQ_F32: return dispatch_in<OFFQ_F32>(dtype, a, s);
     case OFFQ_BF16: return dispatch_in<OFFQ_BF16>(dtype, a, s);
     case OFFQ_F16: return dispatch_in<OFFQ_F16>(dtype, a, s);
+    default: return OFFQ_ERR_INVALID_ARG;
+  }
+}
+
+extern "C" int offq_prepare_key_rotation(const float* rot, int32_t H, int32_t head_dim, void* prepared,
+                                         void* stream) {
+  if (H < 1 || head_dim <= 0) return OFFQ_ERR_INVALID_ARG;
+  if (head_dim != kHd) return OFFQ_ERR_UNSUPPORTED;
+  if (H > 65535) return OFFQ_ERR_UNSUPPORTED;
+  if (rot == nullptr || prepared == nullptr) return OFFQ_ERR_INVALID_ARG;
+  if (!aligned(rot, 16) || !aligned(prepared, 16)) return OFFQ_ERR_MISALIGNED;
+  return launch_pdl(prepare_rotation_kernel, dim3(kHd / 32, static_cast<unsigned>(H)), dim3(kHd),
+                    0, static_cast<cudaStream_t>(stream), rot, static_cast<uint8_t*>(prepared));
+}
+
+extern "C" int offq_kv4_quantize_prepared(const void* kv, int dtype, int64_t T, int32_t H, int32_t head_dim,
+                                          int64_t ld_token, const void* prepared, int32_t flags, uint8_t* codes,
+                                          float* scale, float* offset, void* stream) {
+  if ((flags & ~OFFQ_OFFSET) != 0) return OFFQ_ERR_INVALID_ARG;
+  int st = check_heads(kv, dtype, T, H, head_dim, ld_token, prepared);
+  if (st != OFFQ_OK) return st;
+  if (dtype != OFFQ_BF16) return OFFQ_ERR_UNSUPPORTED;
+  if (T == 0) return OFFQ_OK;
+  if (codes == nullptr || scale == nullptr || ((flags & OFFQ_OFFSET) && offset == nullptr))
+    return OFFQ_ERR_INVALID_ARG;
+  if (!aligned(codes, 16) || !aligned(scale, 4) || (offset != nullptr && !aligned(offset, 4)))
+    return OFFQ_ERR_MISALIGNED;
+  RotArgs a{};
+  a.x = kv;
+  a.ld_token = ld_token;
+  a.T = T;
+  a.H = H;
+  a.prep = prepared;
+  a.quantize = 1;
+  a.offset = (flags & OFFQ_OFFSET) != 0;
+  a.codes = codes;
+  a.scale = scale;
+  a.off = offset;
+  a.status = device_status_ptr();
+  return launch_rotate_mma<OFFQ_F32>(a, static_cast<cudaStream_t>(stream));
+}
+
+extern "C" int offq_rotate_heads_prepared(const void* x, int dtype, int64_t T, int32_t H, int32_t head_dim,
+                                          int64_t ld_token, const void* prepared, void* out, int out_dtype,
+                                          int64_t ld_out, void* stream) {
+  const int ob = elem_bytes(out_dtype);
+  if (ob == 0 || ld_out < static_cast<int64_t>(H) * head_dim) return OFFQ_ERR_INVALID_ARG;
+  int st = check_heads(x, dtype, T, H, head_dim, ld_token, prepared);
+  if (st != OFFQ_OK) return st;
+  if (dtype != OFFQ_BF16) return OFFQ_ERR_UNSUPPORTED;
+  if (T == 0) return OFFQ_OK;
+  if (out == nullptr) return OFFQ_ERR_INVALID_ARG;
+  if (!aligned(out, 16) || (ld_out * ob) % 16 != 0) return OFFQ_ERR_MISALIGNED;
+  RotArgs a{};
+  a.x = x;
+  a.ld_token = ld_token;
+  a.T = T;
+  a.H = H;
+  a.prep = prepared;
+  a.quantize = 0;
+  a.out = out;
+  a.ld_out = ld_out;
+  a.status = device_status_ptr();
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  switch (out_dtype) {
+    case OFFQ_F32: return launch_rotate_mma<OFFQ_F32>(a, s);
+    case OFFQ_BF16: return launch_rotate_mma<OFFQ_BF16>(a, s);
+    case OFFQ_F16: return launch_rotate_mma<OFFQ_F16>(a, s);
     default: return OFFQ_ERR_INVALID_ARG;
   }
 }

@@ -59,6 +59,11 @@ _SIGNATURES = {
                                            _c_vp, _c_vp, _c_vp]),
     "offq_rotate_heads": (_c_int, [_c_vp, _c_int, _c_i64, _c_i32, _c_i32, _c_i64, _c_vp, _c_vp, _c_int, _c_i64,
                                    _c_vp]),
+    "offq_prepare_key_rotation": (_c_int, [_c_vp, _c_i32, _c_i32, _c_vp, _c_vp]),
+    "offq_kv4_quantize_prepared": (_c_int, [_c_vp, _c_int, _c_i64, _c_i32, _c_i32, _c_i64, _c_vp, _c_i32, _c_vp,
+                                            _c_vp, _c_vp, _c_vp]),
+    "offq_rotate_heads_prepared": (_c_int, [_c_vp, _c_int, _c_i64, _c_i32, _c_i32, _c_i64, _c_vp, _c_vp, _c_int,
+                                            _c_i64, _c_vp]),
     "offq_top1_tokens": (_c_int, [_c_vp, _c_int, _c_i64, _c_i64, _c_i64, _c_i64, _c_i64, _c_vp, _c_vp, _c_vp]),
     "offq_top1_direction": (_c_int, [_c_vp, _c_i64, _c_i64, _c_i32, _c_vp, _c_vp, _c_vp, _c_vp]),
     "offq_reflect_rows": (_c_int, [_c_vp, _c_i64, _c_i64, _c_vp, _c_vp, _c_vp]),
@@ -213,6 +218,27 @@ def offq_rotate_heads(x: torch.Tensor, T: int, H: int, head_dim: int, ld_token: 
         _stream(stream)))
 
 
+def offq_prepare_key_rotation(rot: torch.Tensor, H: int, head_dim: int, prepared: torch.Tensor,
+                              stream=None) -> None:
+    _check("offq_prepare_key_rotation", load_library().offq_prepare_key_rotation(
+        _ptr(rot), H, head_dim, _ptr(prepared), _stream(stream)))
+
+
+def offq_kv4_quantize_prepared(kv: torch.Tensor, T: int, H: int, head_dim: int, ld_token: int,
+                               prepared: torch.Tensor, flags: int, codes: torch.Tensor, scale: torch.Tensor,
+                               offset: Optional[torch.Tensor], stream=None) -> None:
+    _check("offq_kv4_quantize_prepared", load_library().offq_kv4_quantize_prepared(
+        _ptr(kv), _dtype_code(kv), T, H, head_dim, ld_token, _ptr(prepared), flags, _ptr(codes), _ptr(scale),
+        _ptr(offset), _stream(stream)))
+
+
+def offq_rotate_heads_prepared(x: torch.Tensor, T: int, H: int, head_dim: int, ld_token: int,
+                               prepared: torch.Tensor, out: torch.Tensor, ld_out: int, stream=None) -> None:
+    _check("offq_rotate_heads_prepared", load_library().offq_rotate_heads_prepared(
+        _ptr(x), _dtype_code(x), T, H, head_dim, ld_token, _ptr(prepared), _ptr(out), _dtype_code(out), ld_out,
+        _stream(stream)))
+
+
 def offq_get_device_status(stream=None) -> int:
     return load_library().offq_get_device_status(_stream(stream))
 
@@ -341,6 +367,42 @@ def rotate_heads(x: torch.Tensor, rot: torch.Tensor, out_dtype: torch.dtype = to
         raise ValueError("heads of a token must be contiguous")
     out = torch.empty((T, H, hd), dtype=out_dtype, device=x.device)
     offq_rotate_heads(x, T, H, hd, x.stride(0), rot.contiguous(), out, out.stride(0), stream)
+    return out
+
+
+KEY_ROTATION_BYTES = 98304  # OFFQ_KEY_ROTATION_BYTES: one head's prepared rotation
+
+
+def prepare_key_rotation(rot: torch.Tensor, stream=None) -> torch.Tensor:
+    """rot [H, hd, hd] float32 -> the prepared image [H, KEY_ROTATION_BYTES] (uint8)."""
+    H, hd, _ = rot.shape
+    prep = torch.empty((H, KEY_ROTATION_BYTES), dtype=torch.uint8, device=rot.device)
+    offq_prepare_key_rotation(rot.contiguous(), H, hd, prep, stream)
+    return prep
+
+
+def kv4_quantize_prepared(kv: torch.Tensor, prepared: torch.Tensor, offset: bool = True,
+                          stream=None) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    """kv4_quantize_rotated for bf16 kv [T, H, hd] with M given as prepare_key_rotation's image."""
+    T, H, hd = kv.shape
+    if kv.stride(2) != 1 or kv.stride(1) != hd:
+        raise ValueError("heads of a token must be contiguous")
+    codes = torch.empty((T, H, hd // 2), dtype=torch.uint8, device=kv.device)
+    scale = torch.empty((T, H), dtype=torch.float32, device=kv.device)
+    off = torch.empty((T, H), dtype=torch.float32, device=kv.device)
+    offq_kv4_quantize_prepared(kv, T, H, hd, kv.stride(0), prepared, OFFQ_OFFSET if offset else 0, codes, scale,
+                               off, stream)
+    return codes, scale, off
+
+
+def rotate_heads_prepared(x: torch.Tensor, prepared: torch.Tensor, out_dtype: torch.dtype = torch.float32,
+                          stream=None) -> torch.Tensor:
+    """rotate_heads for bf16 x [T, H, hd] with M given as prepare_key_rotation's image."""
+    T, H, hd = x.shape
+    if x.stride(2) != 1 or x.stride(1) != hd:
+        raise ValueError("heads of a token must be contiguous")
+    out = torch.empty((T, H, hd), dtype=out_dtype, device=x.device)
+    offq_rotate_heads_prepared(x, T, H, hd, x.stride(0), prepared, out, out.stride(0), stream)
     return out
 
 

@@ -168,6 +168,36 @@ def test_rotated_key_cache_argument_checks(lib):
     assert rh(T=0) == Q.OFFQ_OK
 
 
+def test_prepared_key_rotation_argument_checks(lib):
+    pr = lambda rot=A16, H=8, hd=128, prep=A16: lib.offq_prepare_key_rotation(rot, H, hd, prep, None)
+    assert pr(hd=64) == Q.OFFQ_ERR_UNSUPPORTED
+    assert pr(H=0) == Q.OFFQ_ERR_INVALID_ARG
+    assert pr(H=70000) == Q.OFFQ_ERR_UNSUPPORTED
+    assert pr(rot=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert pr(prep=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert pr(rot=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert pr(prep=A8) == Q.OFFQ_ERR_MISALIGNED
+    kp = lambda kv=A16, dt=Q.OFFQ_BF16, T=4, H=8, hd=128, ld=1024, prep=A16, flags=2, c=A16, s=A16, o=A16: \
+        lib.offq_kv4_quantize_prepared(kv, dt, T, H, hd, ld, prep, flags, c, s, o, None)
+    assert kp(dt=Q.OFFQ_F32) == Q.OFFQ_ERR_UNSUPPORTED     # the prepared parts serve bf16 inputs
+    assert kp(dt=Q.OFFQ_F16) == Q.OFFQ_ERR_UNSUPPORTED
+    assert kp(hd=64, ld=512) == Q.OFFQ_ERR_UNSUPPORTED
+    assert kp(prep=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert kp(prep=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert kp(flags=1) == Q.OFFQ_ERR_INVALID_ARG
+    assert kp(o=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert kp(c=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert kp(T=0) == Q.OFFQ_OK
+    rp = lambda x=A16, dt=Q.OFFQ_BF16, T=4, prep=A16, out=A16, odt=Q.OFFQ_F32, ldo=1024: \
+        lib.offq_rotate_heads_prepared(x, dt, T, 8, 128, 1024, prep, out, odt, ldo, None)
+    assert rp(dt=Q.OFFQ_F32) == Q.OFFQ_ERR_UNSUPPORTED
+    assert rp(prep=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert rp(ldo=512) == Q.OFFQ_ERR_INVALID_ARG
+    assert rp(out=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert rp(out=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert rp(T=0) == Q.OFFQ_OK
+
+
 def test_builder_argument_checks(lib):
     assert lib.offq_top1_tokens(A16, Q.OFFQ_BF16, 4, 8, 64, 32, 512, A16, A16, None) == Q.OFFQ_ERR_INVALID_ARG
     assert lib.offq_top1_tokens(A16, Q.OFFQ_BF16, 4, 8, 64, 64, 256, A16, A16, None) == Q.OFFQ_ERR_INVALID_ARG

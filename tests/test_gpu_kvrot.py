@@ -158,3 +158,89 @@ def test_rotated_key_cache_full_size():
     torch.cuda.synchronize()
     assert Q.offq_get_device_status() == Q.OFFQ_OK
     _check_key_cache(codes, scale, off, kt.to(torch.float64).numpy(), M, tc=True)
+
+
+def _bf16_rne(a):
+    """float32 -> bf16 (round to nearest even) -> float32, on the host."""
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(torch.bfloat16).float().numpy()
+
+
+def _decode_prepared(prep, H):
+    """The prepared image back to the parts [H][3][k][n] as float32, undoing
+    the chunk swizzle: chunk c (k = 8c .. 8c+7) of row n sits in atom column
+    c // 8, slot (c % 8) ^ (n % 8) of the row's 128 bytes."""
+    u = prep.cpu().numpy().view(np.uint16).reshape(H, 3, 2, HD, 8, 8)
+    n = np.arange(HD)[:, None]
+    c = np.arange(16)[None, :]
+    g = u[:, :, c >> 3, n, (c & 7) ^ (n & 7), :]          # [H, 3, n, c, e]
+    parts = g.reshape(H, 3, HD, HD).transpose(0, 1, 3, 2)  # [H, 3, k = 8c + e, n]
+    return (parts.astype(np.uint32) << 16).view(np.float32)
+
+
+def test_prepared_image_is_the_three_part_split():
+    H = 3
+    k = _keys(16, H, seed=100)
+    M = _rotation(k, 101)
+    M[2] = (O.sylvester_hadamard(HD) / math.sqrt(HD)).astype(np.float32)
+    prep = Q.prepare_key_rotation(torch.from_numpy(M).cuda())
+    torch.cuda.synchronize()
+    parts = _decode_prepared(prep, H)
+    hi = _bf16_rne(M)
+    r1 = (M - hi).astype(np.float32)
+    mid = _bf16_rne(r1)
+    lo = _bf16_rne((r1 - mid).astype(np.float32))
+    assert np.array_equal(parts[:, 0], hi) and np.array_equal(parts[:, 1], mid) and np.array_equal(parts[:, 2], lo)
+    rebuilt = parts[:, 0].astype(np.float64) + parts[:, 1] + parts[:, 2]
+    assert np.all(np.abs(rebuilt - M) <= 2.0 ** -26 * np.abs(M))
+
+
+@pytest.mark.parametrize("T,H", [(1, 4), (45, 4), (300, 8), (600, 160)])
+def test_prepared_key_cache_parity(T, H):
+    """The prepared parts give the in-kernel split's outputs bit for bit and
+    stay within the tensor-core bound of the oracle. With 160 heads each CTA
+    takes all of its head's tiles, so every warpgroup loops over several."""
+    k = _keys(T, H, seed=102 + T)
+    M = _rotation(k, 103)
+    kt = torch.from_numpy(k).to(torch.bfloat16).cuda()
+    rot = torch.from_numpy(M).cuda()
+    prep = Q.prepare_key_rotation(rot)
+    for offset in (True, False):
+        c1, s1, o1 = Q.kv4_quantize_prepared(kt, prep, offset=offset)
+        c2, s2, o2 = Q.kv4_quantize_rotated(kt, rot, offset=offset)
+        torch.cuda.synchronize()
+        assert Q.offq_get_device_status() == Q.OFFQ_OK
+        assert torch.equal(c1, c2) and torch.equal(s1, s2)
+        if offset:
+            assert torch.equal(o1, o2)
+        _check_key_cache(c1, s1, o1 if offset else None, kt.to(torch.float64).cpu().numpy(), M, offset=offset,
+                         tc=True)
+
+
+@pytest.mark.parametrize("odt", [torch.float32, torch.bfloat16, torch.float16])
+def test_rotate_heads_prepared(odt):
+    T, H = 333, 160
+    q = np.random.default_rng(104).standard_normal((T, H, HD))
+    M = _rotation(_keys(8, H, seed=105), 106)
+    qt = torch.from_numpy(q).to(torch.bfloat16)
+    rot = torch.from_numpy(M).cuda()
+    y1 = Q.rotate_heads_prepared(qt.cuda(), Q.prepare_key_rotation(rot), out_dtype=odt)
+    y2 = Q.rotate_heads(qt.cuda(), rot, out_dtype=odt)
+    torch.cuda.synchronize()
+    assert torch.equal(y1, y2)
+    if odt == torch.float32:
+        x = qt.to(torch.float64).numpy()
+        err = np.abs(y1.cpu().numpy().astype(np.float64) - O.rotate_heads(x, M.astype(np.float64)))
+        assert np.all(err <= _bound_y(x, M, tc=True) + 1e-30)
+
+
+def test_prepared_key_cache_full_size():
+    """The workload's key tensor, 2048 tokens x 32 heads, through the prepared call."""
+    T, H = 2048, 32
+    k = _keys(T, H, seed=107)
+    M = _rotation(k, 108)
+    kt = torch.from_numpy(k).to(torch.bfloat16)
+    prep = Q.prepare_key_rotation(torch.from_numpy(M).cuda())
+    codes, scale, off = Q.kv4_quantize_prepared(kt.cuda(), prep)
+    torch.cuda.synchronize()
+    assert Q.offq_get_device_status() == Q.OFFQ_OK
+    _check_key_cache(codes, scale, off, kt.to(torch.float64).numpy(), M, tc=True)
