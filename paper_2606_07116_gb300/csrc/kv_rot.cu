@@ -26,6 +26,7 @@
 // Offset, scale and codes come from warp reductions over the token's 128
 // outputs (4 per lane).
 #include <cuda_bf16.h>
+#include <cudaTypedefs.h>
 #include <cuda_fp16.h>
 
 #include <mutex>
@@ -226,12 +227,16 @@ constexpr int kParts = 3;                      // bf16 parts of M
 constexpr int kAtomBytes = 128 * 128;          // 128 rows x 64 bf16 (one 128-byte swizzle atom column)
 constexpr int kOpBytes = 2 * kAtomBytes;       // 128 rows x 128 bf16
 constexpr int kPrepBytes = kParts * kOpBytes;  // one head's three parts
-constexpr int kWG = 4;                         // warpgroups, each with its own tile, accumulator and barrier
-constexpr int kMmaThreads = 128 * kWG;
-constexpr int kCtrlOff = kPrepBytes + kWG * kOpBytes;  // barriers, TMEM address, abort flag
-constexpr int kMmaSmem = kCtrlOff + 128 + 1024;
+constexpr int kSlots = 4;                      // token-tile ring
+constexpr int kAcc = 3;                        // TMEM accumulators, 128 columns each
+constexpr int kEpi = 3;                        // epilogue warpgroups, group e reading accumulator e
+constexpr int kMmaThreads = 64 + 128 * kEpi;   // TMA warp, MMA warp, epilogue
+constexpr int kCtrlOff = kPrepBytes + kSlots * kOpBytes;  // barriers, TMEM address, abort flag
+constexpr int kCtrlBars = 8 * (1 + 2 * kSlots + 2 * kAcc);
+constexpr int kMmaSmem = kCtrlOff + kCtrlBars + 8 + 1024;
 static_assert(kPrepBytes == OFFQ_KEY_ROTATION_BYTES, "prepared image size");
-static_assert(kWG * 4 == kHd / 8, "each warpgroup splits four k-chunks of M");
+static_assert(kEpi == kAcc, "each epilogue group owns one accumulator and takes its phases in order");
+static_assert(kAcc * kTM <= 512, "TMEM columns");
 static_assert(kMmaSmem <= 232448, "one CTA per SM");
 // kind::f16 instruction descriptor: D f32 (bits 4-5 = 1), A and B bf16 (bits
 // 7-9, 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
@@ -275,31 +280,6 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
   asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
                "l"(src), "r"(bytes), "r"(bar)
                : "memory");
-}
-
-// 16-byte global -> shared copy; src_bytes = 0 writes 16 zero bytes instead.
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, uint32_t src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
-}
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
-
-// Barrier over the 128 threads of one warpgroup (named barrier `id`).
-__device__ __forceinline__ void wg_sync(int id) { asm volatile("bar.sync %0, 128;" ::"r"(id) : "memory"); }
-
-// The same barrier, returning whether `pred` held for any of the 128 threads.
-__device__ __forceinline__ bool wg_any(int id, bool pred) {
-  uint32_t r;
-  asm volatile(
-      "{\n"
-      ".reg .pred p, q;\n"
-      "setp.ne.b32 p, %1, 0;\n"
-      "bar.red.or.pred q, %2, 128, p;\n"
-      "selp.u32 %0, 1, 0, q;\n"
-      "}\n"
-      : "=r"(r)
-      : "r"(static_cast<uint32_t>(pred)), "r"(id)
-      : "memory");
-  return r != 0;
 }
 
 // Byte offset of 16-byte chunk c (8 bf16, c = 0..15) of row r in a 128-row
@@ -366,36 +346,53 @@ __global__ void __launch_bounds__(128) prepare_rotation_kernel(const float* __re
     for (int s = 0; s < kParts; ++s) *reinterpret_cast<uint4*>(dst + s * kOpBytes + sw_off(n, c0 + cc)) = w[cc][s];
 }
 
-// One CTA per (head, share of its tiles); four warpgroups each take every
-// fourth of the CTA's 128-token tiles with their own tile buffer, TMEM
-// accumulator (128 columns) and completion barrier, so one warpgroup's loads
-// and epilogue overlap the others' MMAs. M's three parts are staged once per
-// CTA: copied from the prepared image (one bulk copy per part) or split here.
+// One CTA per (head, share of its tiles), warp-specialised:
+//   warp 0    loads the CTA's 128-token tiles by TMA into a ring of kSlots
+//             buffers (two 64-channel boxes per tile, 128-byte swizzle) and,
+//             with a prepared image, M's three parts by one bulk copy each;
+//   warp 1    allocates the accumulators and issues each tile's 3 x 8 MMAs;
+//   warps 2.. (kEpi groups of four) read an accumulator, write the codes and
+//             free it: group e takes the CTA's tiles e, e + kEpi, ... in
+//             accumulator e.
+// Without a prepared image the epilogue warps split M into the three parts
+// before their first tile.
 template <int OUT>
-__global__ void __launch_bounds__(kMmaThreads, 1) rotate_heads_mma_kernel(const RotArgs a) {
+__global__ void __launch_bounds__(kMmaThreads, 1)
+    rotate_heads_mma_kernel(const __grid_constant__ CUtensorMap xmap, const RotArgs a) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* smem = smem_raw + (base - raw);
-  const uint32_t b_base = base;  // kParts operands B_s[n][k] = part s of M[k][n]
+  const uint32_t b_base = base;                     // kParts operands B_s[n][k] = part s of M[k][n]
+  const uint32_t ring = base + kPrepBytes;          // kSlots token tiles
   const uint32_t ctrl = base + kCtrlOff;
-  const uint32_t bar_b = ctrl;  // the prepared parts have landed
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kCtrlOff + 48);
-  volatile int* abort = reinterpret_cast<volatile int*>(smem + kCtrlOff + 56);
+  const uint32_t bar_b = ctrl;                      // the three parts are in shared memory
+  const uint32_t full0 = ctrl + 8;                  // [kSlots] a tile has landed
+  const uint32_t empty0 = full0 + 8 * kSlots;       // [kSlots] its MMAs have read it
+  const uint32_t tfull0 = empty0 + 8 * kSlots;      // [kAcc] an accumulator holds a tile's y
+  const uint32_t tempty0 = tfull0 + 8 * kAcc;       // [kAcc] its four epilogue warps have read it
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kCtrlOff + kCtrlBars);
+  volatile int* abort = reinterpret_cast<volatile int*>(smem + kCtrlOff + kCtrlBars + 4);
   const int h = blockIdx.y;
-  const int tid = threadIdx.x, warp = tid >> 5;
-  const int wg = warp >> 2, wt = tid & 127;
-  const uint32_t a_tile = base + kPrepBytes + wg * kOpBytes;  // this warpgroup's token tile
-  const uint32_t bar = ctrl + 8 + 8 * wg;                     // its MMAs have completed
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const bool prepared = a.prep != nullptr;
   if (tid == 0) {
-    mbar_init(bar_b, 1);
+    mbar_init(bar_b, prepared ? 1 : 128 * kEpi);
 #pragma unroll
-    for (int g = 0; g < kWG; ++g) mbar_init(ctrl + 8 + 8 * g, 1);
+    for (int s = 0; s < kSlots; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+#pragma unroll
+    for (int x = 0; x < kAcc; ++x) {
+      mbar_init(tfull0 + 8 * x, 1);
+      mbar_init(tempty0 + 8 * x, 4);
+    }
     *abort = 0;
     mbar_fence_init();
   }
-  if (warp == 0) {
-    tmem_alloc(smem_u32(tmem_slot), kWG * kTM);
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), 512);
     tmem_relinquish();
   }
   tc_fence_before();
@@ -405,172 +402,189 @@ __global__ void __launch_bounds__(kMmaThreads, 1) rotate_heads_mma_kernel(const 
   griddep_wait();
   griddep_launch_dependents();
 
-  const uint8_t* prep = static_cast<const uint8_t*>(a.prep);
-  if (prep != nullptr && tid == 0) {
-    mbar_arrive_expect_tx(bar_b, kPrepBytes);
-#pragma unroll
-    for (int s = 0; s < kParts; ++s)
-      bulk_load(b_base + s * kOpBytes, prep + static_cast<int64_t>(h) * kPrepBytes + s * kOpBytes, kOpBytes, bar_b);
-  }
-
   const int64_t tiles = (a.T + kTM - 1) / kTM;
-  const int64_t stride = static_cast<int64_t>(kWG) * gridDim.x;
-  // Token tile `tile` into this warpgroup's buffer: thread wt copies 16-byte
-  // chunks wt + 128 k (row >> 4, chunk & 15); rows past T are zero-filled.
-  const __nv_bfloat16* xh = static_cast<const __nv_bfloat16*>(a.x) + static_cast<int64_t>(h) * kHd;
-  auto load_tile = [&](int64_t tile) {
+  const int n_local = static_cast<int>((tiles - blockIdx.x + gridDim.x - 1) / gridDim.x);  // >= 1
+
+  if (warp == 0) {
+    if (lane == 0) {
+      if (prepared) {
+        const uint8_t* src = static_cast<const uint8_t*>(a.prep) + static_cast<int64_t>(h) * kPrepBytes;
+        mbar_arrive_expect_tx(bar_b, kPrepBytes);
 #pragma unroll
-    for (int k = 0; k < kTM * 16 / 128; ++k) {
-      const int idx = wt + k * 128;
-      const int64_t tok = tile * kTM + (idx >> 4);
+        for (int s = 0; s < kParts; ++s) bulk_load(b_base + s * kOpBytes, src + s * kOpBytes, kOpBytes, bar_b);
+      }
+      tma_prefetch_desc(&xmap);
+      int i = 0;
+      for (; i < n_local; ++i) {
+        const int s = i % kSlots;
+        if (i >= kSlots && !mbar_wait(empty0 + 8 * s, ((i / kSlots) - 1) & 1, abort)) break;
+        const int y = static_cast<int>((blockIdx.x + static_cast<int64_t>(i) * gridDim.x) * kTM);
+        const uint32_t dst = ring + s * kOpBytes;
+        mbar_arrive_expect_tx(full0 + 8 * s, kOpBytes);
+        tma_load_2d(dst, &xmap, full0 + 8 * s, h * kHd, y);
+        tma_load_2d(dst + kAtomBytes, &xmap, full0 + 8 * s, h * kHd + 64, y);
+      }
+      if (*abort) {
+        // Copies still in flight land (bounded) before shared memory is released.
+        const long long c0 = clock64();
+        for (int j = i - 1; j >= 0 && j >= i - kSlots; --j)
+          while (!mbar_try_wait(full0 + 8 * (j % kSlots), (j / kSlots) & 1) && clock64() - c0 < kWaitCycles) {
+          }
+        if (prepared)
+          while (!mbar_try_wait(bar_b, 0) && clock64() - c0 < kWaitCycles) {
+          }
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0) {
+      int committed = -1;
+      if (mbar_wait(bar_b, 0, abort)) {
+        for (int i = 0; i < n_local; ++i) {
+          const int s = i % kSlots, x = i % kAcc;
+          if (!mbar_wait(full0 + 8 * s, (i / kSlots) & 1, abort)) break;
+          if (i >= kAcc && !mbar_wait(tempty0 + 8 * x, ((i / kAcc) - 1) & 1, abort)) break;
+          tc_fence_after();
+          const uint32_t at = ring + s * kOpBytes, acc = tmem + x * kTM;
+#pragma unroll
+          for (int sp = 0; sp < kParts; ++sp)
+#pragma unroll
+            for (int kk = 0; kk < kHd / 16; ++kk) {
+              const uint32_t koff = (kk >> 2) * kAtomBytes + (kk & 3) * 32;
+              mma_bf16(acc, smem_desc_sw128(at + koff), smem_desc_sw128(b_base + sp * kOpBytes + koff), kIdescBf16,
+                       (sp | kk) != 0 ? 1u : 0u);
+            }
+          mma_commit(empty0 + 8 * s);  // the tile buffer is free once these MMAs are done
+          mma_commit(tfull0 + 8 * x);
+          committed = i;
+        }
+      }
+      if (*abort && committed >= 0) {
+        // MMAs complete in issue order: wait (bounded) for the last commit
+        // before tensor memory is released.
+        const long long c0 = clock64();
+        while (!mbar_try_wait(tfull0 + 8 * (committed % kAcc), (committed / kAcc) & 1) &&
+               clock64() - c0 < kWaitCycles) {
+        }
+      }
+    }
+    __syncwarp();
+  } else {
+    const int e = (warp - 2) >> 2;  // epilogue group
+    const int q = warp & 3;         // the TMEM lane quadrant this warp may read
+    const int et = tid - 64;
+    if (!prepared) {
+      // Units u = (column n = u % 128, k-chunks 4 (u / 128) .. + 3) of M[h].
+      for (int u = et; u < 4 * kHd; u += 128 * kEpi) {
+        uint4 w[4][kParts];
+        const int n = u & (kHd - 1), c0 = 4 * (u >> 7);
+        split_column(a.rot + static_cast<int64_t>(h) * kHd * kHd, n, c0, w);
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc)
+#pragma unroll
+          for (int s = 0; s < kParts; ++s) sts128v(b_base + s * kOpBytes + sw_off(n, c0 + cc), w[cc][s]);
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(bar_b);
+    }
+    for (int i = e; i < n_local; i += kEpi) {
+      const int x = i % kAcc;
+      const bool waited = mbar_wait(tfull0 + 8 * x, (i / kAcc) & 1, abort);
+      if (__any_sync(0xFFFFFFFFu, !waited)) break;  // the warp leaves together
+      tc_fence_after();
+      const uint32_t row_tm = tmem + x * kTM + (static_cast<uint32_t>(q * 32) << 16);
+      // Thread (q, lane) owns token tile * 128 + 32 q + lane (TMEM lane 32 q + lane).
+      const int64_t tok = (blockIdx.x + static_cast<int64_t>(i) * gridDim.x) * kTM + q * 32 + lane;
       const bool ok = tok < a.T;
-      const void* src = ok ? static_cast<const void*>(xh + tok * a.ld_token + 8 * (idx & 15)) : a.x;
-      cp_async16(a_tile + sw_off(idx >> 4, idx & 15), src, ok ? 16u : 0u);
-    }
-  };
-  int64_t tile = blockIdx.x + static_cast<int64_t>(wg) * gridDim.x;
-  if (tile < tiles) load_tile(tile);
-
-  if (prep == nullptr) {
-    // Split M[h] here while the first tiles load: thread (n = wt, warpgroup
-    // wg) stages k-chunks 4 wg .. 4 wg + 3 of column n.
-    uint4 w[4][kParts];
-    split_column(a.rot + static_cast<int64_t>(h) * kHd * kHd, wt, 4 * wg, w);
+      const int64_t th = tok * a.H + h;
+      if (a.quantize) {
+        // Pass 1: the offset (two fp32 partial sums, lanes of one f32x2 add)
+        // and the extremes of y.
+        uint64_t sum2 = pack2(0.f, 0.f);
+        float ymax0 = -INFINITY, ymax1 = -INFINITY, ymin0 = INFINITY, ymin1 = INFINITY;
+#pragma unroll 1
+        for (int c = 0; c < kHd / 32; ++c) {
+          uint32_t v[32];
+          tmem_ld_32cols_waited(row_tm + c * 32, v);
 #pragma unroll
-    for (int cc = 0; cc < 4; ++cc)
-#pragma unroll
-      for (int s = 0; s < kParts; ++s) sts128v(b_base + s * kOpBytes + sw_off(wt, 4 * wg + cc), w[cc][s]);
-    fence_proxy_async_smem();
-    __syncthreads();
-  }
-
-  bool b_ready = prep == nullptr;  // (issuing thread) the parts are in shared memory
-  bool pending = false;            // (issuing thread) MMAs committed, completion not yet seen
-  uint32_t phase = 0;
-  const uint32_t acc = tmem + wg * kTM;                                                // accumulator columns
-  const uint32_t row_tm = acc + (static_cast<uint32_t>((warp & 3) * 32) << 16);  // this warp's TMEM lanes
-  for (; tile < tiles; tile += stride) {
-    cp_async_wait_all();
-    fence_proxy_async_smem();  // the tile, visible to the tensor core
-    tc_fence_before();         // and this warpgroup's previous TMEM reads ordered before its MMAs
-    wg_sync(1 + wg);
-    if (wt == 0) {
-      if (!b_ready) b_ready = mbar_wait(bar_b, 0, abort);
-      if (b_ready) {
-        tc_fence_after();
-#pragma unroll
-        for (int sp = 0; sp < kParts; ++sp)
-#pragma unroll
-          for (int kk = 0; kk < kHd / 16; ++kk) {
-            const uint32_t koff = (kk >> 2) * kAtomBytes + (kk & 3) * 32;
-            mma_bf16(acc, smem_desc_sw128(a_tile + koff), smem_desc_sw128(b_base + sp * kOpBytes + koff), kIdescBf16,
-                     (sp | kk) != 0 ? 1u : 0u);
+          for (int j = 0; j < 32; j += 2) {
+            const float y0 = __uint_as_float(v[j]), y1 = __uint_as_float(v[j + 1]);
+            sum2 = add2v(sum2, pack2(y0, y1));
+            ymax0 = fmaxf(ymax0, y0);
+            ymax1 = fmaxf(ymax1, y1);
+            ymin0 = fminf(ymin0, y0);
+            ymin1 = fminf(ymin1, y1);
           }
-        mma_commit(bar);
-        pending = true;
-      }
-    }
-    const bool done = mbar_wait(bar, phase, abort);
-    if (wt == 0 && done) pending = false;
-    if (wg_any(1 + wg, !done)) break;  // the whole warpgroup leaves together
-    phase ^= 1;
-    tc_fence_after();
-    // The MMAs have read the tile buffer: the next tile's copies overlap this epilogue.
-    if (tile + stride < tiles) load_tile(tile + stride);
-
-    // Epilogue: thread wt owns token t0 + wt (TMEM lane wt of the accumulator).
-    const int64_t tok = tile * kTM + wt;
-    const bool ok = tok < a.T;
-    const int64_t th = tok * a.H + h;
-    if (a.quantize) {
-      // Pass 1: the offset (two fp32 partial sums, lanes of one f32x2 add)
-      // and the extremes of y.
-      uint64_t sum2 = pack2(0.f, 0.f);
-      float ymax0 = -INFINITY, ymax1 = -INFINITY, ymin0 = INFINITY, ymin1 = INFINITY;
-#pragma unroll 1
-      for (int c = 0; c < kHd / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld_32cols_waited(row_tm + c * 32, v);
-#pragma unroll
-        for (int j = 0; j < 32; j += 2) {
-          const float y0 = __uint_as_float(v[j]), y1 = __uint_as_float(v[j + 1]);
-          sum2 = add2v(sum2, pack2(y0, y1));
-          ymax0 = fmaxf(ymax0, y0);
-          ymax1 = fmaxf(ymax1, y1);
-          ymin0 = fminf(ymin0, y0);
-          ymin1 = fminf(ymin1, y1);
         }
-      }
-      float s0, s1;
-      unpack2(sum2, s0, s1);
-      const float o = a.offset ? (s0 + s1) * (1.0f / kHd) : 0.f;
-      // max_j |fl(y_j - o)| from the extremes: rounding is monotone and
-      // fl(o - y) = -fl(y - o), so the largest are fl(ymax - o) and fl(o - ymin).
-      const float amax = fmaxf(fmaxf(ymax0, ymax1) - o, o - fminf(ymin0, ymin1));
-      const float inv = amax > 0.f ? __fdiv_rn(7.0f, amax) : 0.f;
-      // Pass 2: q = rne(fl(fl(y - o) * inv)). |fl(y - o)| <= amax and
-      // inv <= (7 / amax)(1 + 2^-24), so |q| <= 7 and the clamp to [-7, 7]
-      // never binds. Adding 1.5 * 2^23 + 8 rounds to the nearest even integer
-      // (the float spacing there is 1) and leaves u = q + 8 in the low bits of
-      // the sum; eight of them are packed with shifts and one bias subtraction.
-      const uint64_t o2 = pack2(o, o), inv2 = pack2(inv, inv), magic2 = pack2(kRoundMagic, kRoundMagic);
+        float s0, s1;
+        unpack2(sum2, s0, s1);
+        const float o = a.offset ? (s0 + s1) * (1.0f / kHd) : 0.f;
+        // max_j |fl(y_j - o)| from the extremes: rounding is monotone and
+        // fl(o - y) = -fl(y - o), so the largest are fl(ymax - o) and fl(o - ymin).
+        const float amax = fmaxf(fmaxf(ymax0, ymax1) - o, o - fminf(ymin0, ymin1));
+        const float inv = amax > 0.f ? __fdiv_rn(7.0f, amax) : 0.f;
+        // Pass 2: q = rne(fl(fl(y - o) * inv)). |fl(y - o)| <= amax and
+        // inv <= (7 / amax)(1 + 2^-24), so |q| <= 7 and the clamp to [-7, 7]
+        // never binds. Adding 1.5 * 2^23 + 8 rounds to the nearest even integer
+        // (the float spacing there is 1) and leaves u = q + 8 in the low bits of
+        // the sum; eight of them are packed with shifts and one bias subtraction.
+        const uint64_t o2 = pack2(o, o), inv2 = pack2(inv, inv), magic2 = pack2(kRoundMagic, kRoundMagic);
 #pragma unroll 1
-      for (int c = 0; c < kHd / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld_32cols_waited(row_tm + c * 32, v);
-        uint32_t pk[4];
-#pragma unroll
-        for (int w8 = 0; w8 < 4; ++w8) {
-          uint32_t word = 0u;
-#pragma unroll
-          for (int j = 8 * w8 + 6; j >= 8 * w8; j -= 2) {
-            const uint64_t r2 = sub2v(pack2(__uint_as_float(v[j]), __uint_as_float(v[j + 1])), o2);
-            float f0, f1;
-            unpack2(add2v(mul2v(r2, inv2), magic2), f0, f1);
-            word = (word << 4) + __float_as_uint(f1);
-            word = (word << 4) + __float_as_uint(f0);
+        for (int c = 0; c < kHd / 32; ++c) {
+          uint32_t v[32];
+          tmem_ld_32cols_waited(row_tm + c * 32, v);
+          if (c == kHd / 32 - 1) {
+            // The accumulator's last read: hand it back to the MMA warp.
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(tempty0 + 8 * x);
           }
-          pk[w8] = word - kRoundMagicBits * 0x11111111u;
+          uint32_t pk[4];
+#pragma unroll
+          for (int w8 = 0; w8 < 4; ++w8) {
+            uint32_t word = 0u;
+#pragma unroll
+            for (int j = 8 * w8 + 6; j >= 8 * w8; j -= 2) {
+              const uint64_t r2 = sub2v(pack2(__uint_as_float(v[j]), __uint_as_float(v[j + 1])), o2);
+              float f0, f1;
+              unpack2(add2v(mul2v(r2, inv2), magic2), f0, f1);
+              word = (word << 4) + __float_as_uint(f1);
+              word = (word << 4) + __float_as_uint(f0);
+            }
+            pk[w8] = word - kRoundMagicBits * 0x11111111u;
+          }
+          if (ok)
+            *reinterpret_cast<uint4*>(a.codes + th * (kHd / 2) + 16 * c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
         }
-        if (ok) *reinterpret_cast<uint4*>(a.codes + th * (kHd / 2) + 16 * c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-      }
-      if (ok) {
-        a.scale[th] = amax * (1.0f / 7.0f);
-        if (a.off != nullptr) a.off[th] = o;
-      }
-    } else {
-#pragma unroll 1
-      for (int c = 0; c < kHd / 32; ++c) {
-        uint32_t v[32];
-        tmem_ld_32cols_waited(row_tm + c * 32, v);
         if (ok) {
+          a.scale[th] = amax * (1.0f / 7.0f);
+          if (a.off != nullptr) a.off[th] = o;
+        }
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < kHd / 32; ++c) {
+          uint32_t v[32];
+          tmem_ld_32cols_waited(row_tm + c * 32, v);
+          if (c == kHd / 32 - 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(tempty0 + 8 * x);
+          }
+          if (ok) {
 #pragma unroll
-          for (int j = 0; j < 32; j += 4)
-            store4<OUT>(a.out, tok * a.ld_out + static_cast<int64_t>(h) * kHd + c * 32 + j, __uint_as_float(v[j]),
-                        __uint_as_float(v[j + 1]), __uint_as_float(v[j + 2]), __uint_as_float(v[j + 3]));
+            for (int j = 0; j < 32; j += 4)
+              store4<OUT>(a.out, tok * a.ld_out + static_cast<int64_t>(h) * kHd + c * 32 + j, __uint_as_float(v[j]),
+                          __uint_as_float(v[j + 1]), __uint_as_float(v[j + 2]), __uint_as_float(v[j + 3]));
+          }
         }
       }
-    }
-  }
-  cp_async_wait_all();  // no copy into shared memory outlives the CTA
-  if (wt == 0 && pending) {
-    // A wait ran out with MMAs in flight: let them finish (bounded) before
-    // tensor memory is released.
-    const long long c0 = clock64();
-    while (!mbar_try_wait(bar, phase) && clock64() - c0 < kWaitCycles) {
-    }
-  }
-  if (tid == 0 && !b_ready) {
-    // Likewise the bulk copy of the prepared parts.
-    const long long c0 = clock64();
-    while (!mbar_try_wait(bar_b, 0) && clock64() - c0 < kWaitCycles) {
     }
   }
   tc_fence_before();
   __syncthreads();
-  if (warp == 0) {
+  if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, kWG * kTM);
+    tmem_dealloc(tmem, 512);
   }
   if (tid == 0 && *abort && a.status != nullptr) atomicExch(a.status, kErrTimeout);
 }
@@ -607,6 +621,36 @@ int launch_rotate(const RotArgs& a, cudaStream_t s) {
   return launch_pdl(kern, grid, dim3(kRotWarps * 32), kRotSmem, s, a);
 }
 
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// The bf16 keys as a 2-D tensor of T rows of H * 128 channels (row pitch
+// ld_token elements), read in boxes of 64 channels x 128 tokens with the
+// 128-byte swizzle of the MMA operand; rows past T read as zeros.
+int encode_keys_map(CUtensorMap* map, const void* x, int64_t T, int H, int64_t ld_token) {
+  const auto enc = tensor_map_encoder();
+  if (enc == nullptr) return OFFQ_ERR_CUDA;
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(H) * kHd, static_cast<cuuint64_t>(T)};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld_token) * 2};
+  const cuuint32_t box[2] = {64, kTM};
+  const cuuint32_t elem_strides[2] = {1, 1};
+  const CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(x), dims, strides, box,
+                         elem_strides, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? OFFQ_OK : OFFQ_ERR_CUDA;
+}
+
 template <int OUT>
 int launch_rotate_mma(const RotArgs& a, cudaStream_t s) {
   auto kern = rotate_heads_mma_kernel<OUT>;
@@ -616,6 +660,8 @@ int launch_rotate_mma(const RotArgs& a, cudaStream_t s) {
     attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
   });
   if (attr_err != cudaSuccess) return OFFQ_ERR_CUDA;
+  CUtensorMap xmap;
+  if (encode_keys_map(&xmap, a.x, a.T, a.H, a.ld_token) != OFFQ_OK) return OFFQ_ERR_CUDA;
   // One CTA per SM (shared memory), spread over the heads; each takes every
   // gridDim.x-th of its head's 128-token tiles.
   const int sms = rot_num_sms();
@@ -624,7 +670,7 @@ int launch_rotate_mma(const RotArgs& a, cudaStream_t s) {
   int64_t per_head = sms / a.H > 0 ? sms / a.H : 1;
   if (per_head > tiles) per_head = tiles;
   const dim3 grid(static_cast<unsigned>(per_head), static_cast<unsigned>(a.H));
-  return launch_pdl(kern, grid, dim3(kMmaThreads), kMmaSmem, s, a);
+  return launch_pdl(kern, grid, dim3(kMmaThreads), kMmaSmem, s, xmap, a);
 }
 
 template <int OUT>
