@@ -414,9 +414,15 @@ def time_key_rotation(w, T, device, args, flush_l2, stream):
     # M is fixed per model: its three bf16 parts are prepared once, offline.
     prep = torch.empty((H, Q.KEY_ROTATION_BYTES), dtype=torch.uint8, device=device)
     Q.offq_prepare_key_rotation(rot, H, hd, prep, stream)
-    ts = {"k": [], "q": [], "k_split": []}
+    # The structured form of the method's M = U3 P3 H3: a seeded top-1 direction
+    # and a permutation keeping channel 0 first per head.
+    v = torch.randn((H, hd), generator=g)
+    perm = torch.stack([torch.cat([torch.zeros(1, dtype=torch.int64), 1 + torch.randperm(hd - 1, generator=g)])
+                        for _ in range(H)]).to(torch.int32)
+    refl = Q.prepare_key_reflection(v, perm, device=device)
+    ts = {"k": [], "q": [], "k_split": [], "k_refl": []}
     for i in range(3 + max(1, min(args.steps, 50))):
-        e = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(8)]
         flush_l2()
         e[0].record(stream)
         Q.offq_kv4_quantize_prepared(k, T, H, hd, k.stride(0), prep, Q.OFFQ_OFFSET, codes, scale, off, stream)
@@ -429,17 +435,23 @@ def time_key_rotation(w, T, device, args, flush_l2, stream):
         e[4].record(stream)
         Q.offq_kv4_quantize_rotated(k, T, H, hd, k.stride(0), rot, Q.OFFQ_OFFSET, codes, scale, off, stream)
         e[5].record(stream)
+        flush_l2()
+        e[6].record(stream)
+        Q.offq_kv4_quantize_reflected(k, T, H, hd, k.stride(0), refl, Q.OFFQ_OFFSET, codes, scale, off, stream)
+        e[7].record(stream)
         torch.cuda.synchronize(device)
         if i >= 3:
             ts["k"].append(e[0].elapsed_time(e[1]))
             ts["q"].append(e[2].elapsed_time(e[3]))
             ts["k_split"].append(e[4].elapsed_time(e[5]))
+            ts["k_refl"].append(e[6].elapsed_time(e[7]))
     st = Q.offq_get_device_status(stream)
     if st != Q.OFFQ_OK:
         raise RuntimeError(f"device status after the key rotation: {Q.status_string(st)}")
     k_ms = sum(ts["k"]) / len(ts["k"])
     q_ms = sum(ts["q"]) / len(ts["q"])
     ks_ms = sum(ts["k_split"]) / len(ts["k_split"])
+    kr_ms = sum(ts["k_refl"]) / len(ts["k_refl"])
     flops = 2.0 * T * H * hd * hd
     # Algorithmic bytes: bf16 keys in, 4-bit codes and fp32 scale / offset out, M read once.
     kb = T * H * (hd * 2 + hd // 2 + 8) + H * hd * hd * 4
@@ -450,9 +462,10 @@ def time_key_rotation(w, T, device, args, flush_l2, stream):
                 "the tensor cores, M's three bf16 parts prepared offline) and the query rotation "
                 "(offq_rotate_heads_prepared), "
                 f"{T} tokens x {H} heads x {hd}; per-call events, L2 flushed before each call; "
-                "kv4_rotated_split_us: offq_kv4_quantize_rotated, which splits M in every CTA",
+                "kv4_rotated_split_us: offq_kv4_quantize_rotated, which splits M in every CTA; "
+                "kv4_reflected_us: offq_kv4_quantize_reflected, M in structured form (one +-1 product of N = 144)",
         "kv4_rotated_us": round(k_ms * 1e3, 2), "rotate_q_us": round(q_ms * 1e3, 2),
-        "kv4_rotated_split_us": round(ks_ms * 1e3, 2),
+        "kv4_rotated_split_us": round(ks_ms * 1e3, 2), "kv4_reflected_us": round(kr_ms * 1e3, 2),
         "rotation_tflops": round(flops / (k_ms * 1e-3) / 1e12, 2),
         "roofline": {"bound": "hbm", "kernel": "rotate_heads_mma_kernel (tcgen05.mma kind::f16)",
                      "achieved": round(gbs, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",

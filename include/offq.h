@@ -27,6 +27,10 @@
  *   offq_prepare_key_rotation  offline: M in three bf16 parts, tensor-core order
  *   offq_kv4_quantize_prepared, offq_rotate_heads_prepared
  *                              the two above from the prepared parts (bf16)
+ *   offq_prepare_key_reflection  offline (host): M = U3 P3 H3 from U3's
+ *                              direction and P3, in structured form
+ *   offq_kv4_quantize_reflected, offq_rotate_heads_reflected
+ *                              key cache / queries with the structured M (bf16)
  *
  * and the offline transform builder (top-1 tokens, top-1 PCA direction,
  * reflection, sorted grouping, fusion into the weights).
@@ -85,6 +89,8 @@ extern "C" {
 
 /* Bytes of one head's prepared rotation (offq_prepare_key_rotation). */
 #define OFFQ_KEY_ROTATION_BYTES 98304
+/* Bytes of one head's prepared structured rotation (offq_prepare_key_reflection). */
+#define OFFQ_KEY_REFLECTION_BYTES 37376
 
 typedef enum {
   OFFQ_OK = 0,
@@ -360,6 +366,50 @@ int offq_kv4_quantize_prepared(const void* kv, int dtype, int64_t T, int32_t H, 
 int offq_rotate_heads_prepared(const void* x, int dtype, int64_t T, int32_t H, int32_t head_dim,
                                int64_t ld_token, const void* prepared, void* out, int out_dtype,
                                int64_t ld_out, void* stream);
+
+/*
+ * The structured form of M = U3 P3 H3 -- paper Sec. 3.3 Step 2 (3) with Step 1
+ * (2)'s top-1 PCA rotation taken as the reflection U3 = I - 2 w w^T that maps
+ * channel 0 to the head's top-1 direction v (w = (v/|v| - e_0) normalised;
+ * U3 = I when v/|v| = e_0), P3 the channel permutation ((x P3)_c = x_perm[c])
+ * and H3 = H / sqrt(128) the normalised Sylvester Hadamard. Then
+ *   y = x M = u - 2 (x . w) w'',  u = x P3 H3,  w'' = (P3 H3)^T w,
+ * and x P3 H3 has +-1 coefficients (exact in bf16): one tensor-core product
+ * of N = 144 per tile gives u * sqrt(128) and x . w (w in three bf16 parts),
+ * instead of the three-part product with a general M.
+ *
+ * offq_prepare_key_reflection -- HOST function, offline: the per-head image.
+ *   v         host, [H][head_dim] float32, head h's top-1 direction (any
+ *             nonzero length; OFFQ_ERR_INVALID_ARG for a zero or non-finite v).
+ *   perm      host, [H][head_dim] int32, each row a permutation of
+ *             0..head_dim-1 (OFFQ_ERR_INVALID_ARG otherwise). The method keeps
+ *             perm[h][0] = 0 (the concentrated channel stays first); the call
+ *             does not require it.
+ *   H, head_dim  heads (1..65535), 128.
+ *   prepared  host, H * OFFQ_KEY_REFLECTION_BYTES bytes, written: for each
+ *             head, 144 rows n x 128 bf16 (k-major, 16-byte chunks swizzled
+ *             within 128-byte rows, the 64-channel halves 18432 bytes apart):
+ *             rows n < 128 are sqrt(128) (P3 H3)[k][n] = +-1, rows 128..130
+ *             the bf16 parts of fp32(w), rows 131..143 zero; then w'' as 128
+ *             float32 (computed in float64, rounded once). Copy it to the
+ *             device as is.
+ *
+ * offq_kv4_quantize_reflected / offq_rotate_heads_reflected --
+ * offq_kv4_quantize_rotated and offq_rotate_heads for bf16 inputs with M in
+ * this form: y_j = fma(acc_j, fp32(1/sqrt(128)), fl(-2 d w''_j)), where acc =
+ * sqrt(128) x P3 H3 and d = x . w are fp32 tensor-core sums of exact products.
+ *   dtype     OFFQ_BF16 (OFFQ_ERR_UNSUPPORTED otherwise).
+ *   prepared  device, 16-byte aligned, offq_prepare_key_reflection's image.
+ *   other arguments as in offq_kv4_quantize_rotated / offq_rotate_heads.
+ */
+int offq_prepare_key_reflection(const float* v, const int32_t* perm, int32_t H, int32_t head_dim,
+                                void* prepared);
+int offq_kv4_quantize_reflected(const void* kv, int dtype, int64_t T, int32_t H, int32_t head_dim,
+                                int64_t ld_token, const void* prepared, int32_t flags,
+                                uint8_t* codes, float* scale, float* offset, void* stream);
+int offq_rotate_heads_reflected(const void* x, int dtype, int64_t T, int32_t H, int32_t head_dim,
+                                int64_t ld_token, const void* prepared, void* out, int out_dtype,
+                                int64_t ld_out, void* stream);
 
 /*
  * Offline transform builder -- paper Sec. 3.1 (top-1 PCA), Sec. 3.2 (sorted

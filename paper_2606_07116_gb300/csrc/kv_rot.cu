@@ -29,6 +29,8 @@
 #include <cudaTypedefs.h>
 #include <cuda_fp16.h>
 
+#include <cmath>
+#include <cstring>
 #include <mutex>
 #include <type_traits>
 
@@ -227,20 +229,43 @@ constexpr int kParts = 3;                      // bf16 parts of M
 constexpr int kAtomBytes = 128 * 128;          // 128 rows x 64 bf16 (one 128-byte swizzle atom column)
 constexpr int kOpBytes = 2 * kAtomBytes;       // 128 rows x 128 bf16
 constexpr int kPrepBytes = kParts * kOpBytes;  // one head's three parts
-constexpr int kSlots = 4;                      // token-tile ring
-constexpr int kAcc = 3;                        // TMEM accumulators, 128 columns each
+constexpr int kAcc = 3;                        // TMEM accumulators
 constexpr int kEpi = 3;                        // epilogue warpgroups, group e reading accumulator e
 constexpr int kMmaThreads = 64 + 128 * kEpi;   // TMA warp, MMA warp, epilogue
-constexpr int kCtrlOff = kPrepBytes + kSlots * kOpBytes;  // barriers, TMEM address, abort flag
-constexpr int kCtrlBars = 8 * (1 + 2 * kSlots + 2 * kAcc);
-constexpr int kMmaSmem = kCtrlOff + kCtrlBars + 8 + 1024;
 static_assert(kPrepBytes == OFFQ_KEY_ROTATION_BYTES, "prepared image size");
 static_assert(kEpi == kAcc, "each epilogue group owns one accumulator and takes its phases in order");
-static_assert(kAcc * kTM <= 512, "TMEM columns");
-static_assert(kMmaSmem <= 232448, "one CTA per SM");
-// kind::f16 instruction descriptor: D f32 (bits 4-5 = 1), A and B bf16 (bits
-// 7-9, 10-12 = 1), both K-major, N >> 3 at bit 17, M >> 4 at bit 24.
-constexpr uint32_t kIdescBf16 = (1u << 4) | (1u << 7) | (1u << 10) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
+
+// The structured rotation M = U3 P3 H3 with U3 = I - 2 w w^T (a reflection):
+// x M = u - 2 (x . w) w'' with u = x P3 H3 and w'' = (P3 H3)^T w. B holds
+// rows n < 128 of sqrt(128) (P3 H)^T (entries +-1, exact in bf16), then the
+// three bf16 parts of w (so one MMA also gives x . w), then zero rows to N = 144.
+constexpr int kRefRows = 144;
+constexpr int kRefAtom = kRefRows * 128;          // one 64-channel atom column of B
+constexpr int kRefBBytes = 2 * kRefAtom;
+constexpr int kRefImgBytes = kRefBBytes + kHd * 4;  // B, then w'' (fp32)
+constexpr float kInvSqrtHd = 0.08838834764831844055f;  // 1 / sqrt(128), rounded to fp32
+static_assert(kRefImgBytes == OFFQ_KEY_REFLECTION_BYTES, "prepared reflection size");
+
+// Shared and tensor memory of the two variants: the dense one keeps M's
+// three parts (96 KB) and four tile slots, the structured one its 36 KB
+// image and five.
+template <bool REFLECT>
+struct RotLayout {
+  static constexpr int kImg = REFLECT ? kRefImgBytes : kPrepBytes;     // bytes copied per head
+  static constexpr int kBSmem = (kImg + 1023) / 1024 * 1024;          // ring stays 1024-aligned
+  static constexpr int kSlots = REFLECT ? 5 : 4;
+  static constexpr int kN = REFLECT ? kRefRows : kHd;                 // MMA N
+  static constexpr int kAccCols = REFLECT ? 160 : kHd;               // accumulator stride in TMEM
+  static constexpr int kCtrlOff = kBSmem + kSlots * kOpBytes;       // barriers, TMEM address, abort flag
+  static constexpr int kCtrlBars = 8 * (1 + 2 * kSlots + 2 * kAcc);
+  static constexpr int kSmem = kCtrlOff + kCtrlBars + 8 + 1024;
+  // kind::f16: D f32 (bits 4-5 = 1), A and B bf16 (7-9, 10-12 = 1), both
+  // K-major, N >> 3 at bit 17, M >> 4 at bit 24.
+  static constexpr uint32_t kIdesc =
+      (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(kN >> 3) << 17) | ((128u >> 4) << 24);
+  static_assert(kSmem <= 232448, "one CTA per SM");
+  static_assert(kAcc * kAccCols <= 512, "TMEM columns");
+};
 
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
                                          uint32_t accumulate) {
@@ -280,6 +305,39 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
   asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
                "l"(src), "r"(bytes), "r"(bar)
                : "memory");
+}
+
+// Waits for this thread's TMEM loads; the registers they fill are operands, so
+// no use of them moves above the wait.
+__device__ __forceinline__ void tmem_wait_into(uint32_t (&r)[32]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                 "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]),
+                 "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
+                 "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]),
+                 "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+               :
+               : "memory");
+}
+
+// The four 32-column chunks of this thread's 128-column TMEM row: f(v, c) on
+// chunk c while chunk c + 1 is loading; last() once all four are loaded.
+template <typename F, typename G>
+__device__ __forceinline__ void tmem_row_pass(uint32_t row_tm, F&& f, G&& last) {
+  uint32_t va[32], vb[32];
+  tmem_ld_32cols(row_tm, va);
+  tmem_wait_into(va);
+  tmem_ld_32cols(row_tm + 32, vb);
+  f(va, 0);
+  tmem_wait_into(vb);
+  tmem_ld_32cols(row_tm + 64, va);
+  f(vb, 1);
+  tmem_wait_into(va);
+  tmem_ld_32cols(row_tm + 96, vb);
+  f(va, 2);
+  tmem_wait_into(vb);
+  last();
+  f(vb, 3);
 }
 
 // Byte offset of 16-byte chunk c (8 bf16, c = 0..15) of row r in a 128-row
@@ -355,31 +413,34 @@ __global__ void __launch_bounds__(128) prepare_rotation_kernel(const float* __re
 //             free it: group e takes the CTA's tiles e, e + kEpi, ... in
 //             accumulator e.
 // Without a prepared image the epilogue warps split M into the three parts
-// before their first tile.
-template <int OUT>
+// before their first tile. REFLECT: the structured image instead (one MMA of
+// N = 144 per 16 channels; the epilogue forms y = u - 2 (x . w) w'').
+template <int OUT, bool REFLECT>
 __global__ void __launch_bounds__(kMmaThreads, 1)
     rotate_heads_mma_kernel(const __grid_constant__ CUtensorMap xmap, const RotArgs a) {
+  using L = RotLayout<REFLECT>;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* smem = smem_raw + (base - raw);
-  const uint32_t b_base = base;                     // kParts operands B_s[n][k] = part s of M[k][n]
-  const uint32_t ring = base + kPrepBytes;          // kSlots token tiles
-  const uint32_t ctrl = base + kCtrlOff;
-  const uint32_t bar_b = ctrl;                      // the three parts are in shared memory
+  // B: kParts operands B_s[n][k] = part s of M[k][n], or the structured image.
+  const uint32_t b_base = base;
+  const uint32_t ring = base + L::kBSmem;           // L::kSlots token tiles
+  const uint32_t ctrl = base + L::kCtrlOff;
+  const uint32_t bar_b = ctrl;                      // B is in shared memory
   const uint32_t full0 = ctrl + 8;                  // [kSlots] a tile has landed
-  const uint32_t empty0 = full0 + 8 * kSlots;       // [kSlots] its MMAs have read it
-  const uint32_t tfull0 = empty0 + 8 * kSlots;      // [kAcc] an accumulator holds a tile's y
+  const uint32_t empty0 = full0 + 8 * L::kSlots;    // [kSlots] its MMAs have read it
+  const uint32_t tfull0 = empty0 + 8 * L::kSlots;   // [kAcc] an accumulator holds a tile's product
   const uint32_t tempty0 = tfull0 + 8 * kAcc;       // [kAcc] its four epilogue warps have read it
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kCtrlOff + kCtrlBars);
-  volatile int* abort = reinterpret_cast<volatile int*>(smem + kCtrlOff + kCtrlBars + 4);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::kCtrlOff + L::kCtrlBars);
+  volatile int* abort = reinterpret_cast<volatile int*>(smem + L::kCtrlOff + L::kCtrlBars + 4);
   const int h = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const bool prepared = a.prep != nullptr;
   if (tid == 0) {
     mbar_init(bar_b, prepared ? 1 : 128 * kEpi);
 #pragma unroll
-    for (int s = 0; s < kSlots; ++s) {
+    for (int s = 0; s < L::kSlots; ++s) {
       mbar_init(full0 + 8 * s, 1);
       mbar_init(empty0 + 8 * s, 1);
     }
@@ -408,16 +469,20 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       if (prepared) {
-        const uint8_t* src = static_cast<const uint8_t*>(a.prep) + static_cast<int64_t>(h) * kPrepBytes;
-        mbar_arrive_expect_tx(bar_b, kPrepBytes);
+        const uint8_t* src = static_cast<const uint8_t*>(a.prep) + static_cast<int64_t>(h) * L::kImg;
+        mbar_arrive_expect_tx(bar_b, L::kImg);
+        if constexpr (REFLECT) {
+          bulk_load(b_base, src, L::kImg, bar_b);
+        } else {
 #pragma unroll
-        for (int s = 0; s < kParts; ++s) bulk_load(b_base + s * kOpBytes, src + s * kOpBytes, kOpBytes, bar_b);
+          for (int s = 0; s < kParts; ++s) bulk_load(b_base + s * kOpBytes, src + s * kOpBytes, kOpBytes, bar_b);
+        }
       }
       tma_prefetch_desc(&xmap);
       int i = 0;
       for (; i < n_local; ++i) {
-        const int s = i % kSlots;
-        if (i >= kSlots && !mbar_wait(empty0 + 8 * s, ((i / kSlots) - 1) & 1, abort)) break;
+        const int s = i % L::kSlots;
+        if (i >= L::kSlots && !mbar_wait(empty0 + 8 * s, ((i / L::kSlots) - 1) & 1, abort)) break;
         const int y = static_cast<int>((blockIdx.x + static_cast<int64_t>(i) * gridDim.x) * kTM);
         const uint32_t dst = ring + s * kOpBytes;
         mbar_arrive_expect_tx(full0 + 8 * s, kOpBytes);
@@ -427,8 +492,8 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
       if (*abort) {
         // Copies still in flight land (bounded) before shared memory is released.
         const long long c0 = clock64();
-        for (int j = i - 1; j >= 0 && j >= i - kSlots; --j)
-          while (!mbar_try_wait(full0 + 8 * (j % kSlots), (j / kSlots) & 1) && clock64() - c0 < kWaitCycles) {
+        for (int j = i - 1; j >= 0 && j >= i - L::kSlots; --j)
+          while (!mbar_try_wait(full0 + 8 * (j % L::kSlots), (j / L::kSlots) & 1) && clock64() - c0 < kWaitCycles) {
           }
         if (prepared)
           while (!mbar_try_wait(bar_b, 0) && clock64() - c0 < kWaitCycles) {
@@ -441,19 +506,28 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
       int committed = -1;
       if (mbar_wait(bar_b, 0, abort)) {
         for (int i = 0; i < n_local; ++i) {
-          const int s = i % kSlots, x = i % kAcc;
-          if (!mbar_wait(full0 + 8 * s, (i / kSlots) & 1, abort)) break;
+          const int s = i % L::kSlots, x = i % kAcc;
+          if (!mbar_wait(full0 + 8 * s, (i / L::kSlots) & 1, abort)) break;
           if (i >= kAcc && !mbar_wait(tempty0 + 8 * x, ((i / kAcc) - 1) & 1, abort)) break;
           tc_fence_after();
-          const uint32_t at = ring + s * kOpBytes, acc = tmem + x * kTM;
-#pragma unroll
-          for (int sp = 0; sp < kParts; ++sp)
+          const uint32_t at = ring + s * kOpBytes, acc = tmem + x * L::kAccCols;
+          if constexpr (REFLECT) {
 #pragma unroll
             for (int kk = 0; kk < kHd / 16; ++kk) {
-              const uint32_t koff = (kk >> 2) * kAtomBytes + (kk & 3) * 32;
-              mma_bf16(acc, smem_desc_sw128(at + koff), smem_desc_sw128(b_base + sp * kOpBytes + koff), kIdescBf16,
-                       (sp | kk) != 0 ? 1u : 0u);
+              const uint32_t koff = (kk & 3) * 32;
+              mma_bf16(acc, smem_desc_sw128(at + (kk >> 2) * kAtomBytes + koff),
+                       smem_desc_sw128(b_base + (kk >> 2) * kRefAtom + koff), L::kIdesc, kk != 0 ? 1u : 0u);
             }
+          } else {
+#pragma unroll
+            for (int sp = 0; sp < kParts; ++sp)
+#pragma unroll
+              for (int kk = 0; kk < kHd / 16; ++kk) {
+                const uint32_t koff = (kk >> 2) * kAtomBytes + (kk & 3) * 32;
+                mma_bf16(acc, smem_desc_sw128(at + koff), smem_desc_sw128(b_base + sp * kOpBytes + koff), L::kIdesc,
+                         (sp | kk) != 0 ? 1u : 0u);
+              }
+          }
           mma_commit(empty0 + 8 * s);  // the tile buffer is free once these MMAs are done
           mma_commit(tfull0 + 8 * x);
           committed = i;
@@ -473,7 +547,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
     const int e = (warp - 2) >> 2;  // epilogue group
     const int q = warp & 3;         // the TMEM lane quadrant this warp may read
     const int et = tid - 64;
-    if (!prepared) {
+    if (!REFLECT && !prepared) {
       // Units u = (column n = u % 128, k-chunks 4 (u / 128) .. + 3) of M[h].
       for (int u = et; u < 4 * kHd; u += 128 * kEpi) {
         uint4 w[4][kParts];
@@ -492,7 +566,26 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
       const bool waited = mbar_wait(tfull0 + 8 * x, (i / kAcc) & 1, abort);
       if (__any_sync(0xFFFFFFFFu, !waited)) break;  // the warp leaves together
       tc_fence_after();
-      const uint32_t row_tm = tmem + x * kTM + (static_cast<uint32_t>(q * 32) << 16);
+      const uint32_t row_tm = tmem + x * L::kAccCols + (static_cast<uint32_t>(q * 32) << 16);
+      // y for columns (j, j + 1) of a 32-column chunk c: the accumulator, or
+      // (structured) fma(acc, 1/sqrt(128), fl(-2 d w''_j)) with d = x . w.
+      uint64_t nd2 = 0;
+      if constexpr (REFLECT) {
+        uint32_t dv[16];
+        tmem_ld_16cols(row_tm + kHd, dv);
+        tmem_ld_wait();
+        const float d = (__uint_as_float(dv[0]) + __uint_as_float(dv[1])) + __uint_as_float(dv[2]);  // x . w
+        nd2 = pack2(-2.f * d, -2.f * d);
+      }
+      const uint64_t* w2 = reinterpret_cast<const uint64_t*>(smem + kRefBBytes);  // w'' pairs (structured)
+      auto ypair = [&](const uint32_t (&v)[32], int c, int j) -> uint64_t {
+        const uint64_t acc2 = pack2(__uint_as_float(v[j]), __uint_as_float(v[j + 1]));
+        if constexpr (REFLECT) {
+          return fma2v(acc2, pack2(kInvSqrtHd, kInvSqrtHd), mul2v(nd2, w2[(c * 32 + j) >> 1]));
+        } else {
+          return acc2;
+        }
+      };
       // Thread (q, lane) owns token tile * 128 + 32 q + lane (TMEM lane 32 q + lane).
       const int64_t tok = (blockIdx.x + static_cast<int64_t>(i) * gridDim.x) * kTM + q * 32 + lane;
       const bool ok = tok < a.T;
@@ -502,20 +595,22 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
         // and the extremes of y.
         uint64_t sum2 = pack2(0.f, 0.f);
         float ymax0 = -INFINITY, ymax1 = -INFINITY, ymin0 = INFINITY, ymin1 = INFINITY;
-#pragma unroll 1
-        for (int c = 0; c < kHd / 32; ++c) {
-          uint32_t v[32];
-          tmem_ld_32cols_waited(row_tm + c * 32, v);
+        tmem_row_pass(
+            row_tm,
+            [&](const uint32_t (&v)[32], int c) {
 #pragma unroll
-          for (int j = 0; j < 32; j += 2) {
-            const float y0 = __uint_as_float(v[j]), y1 = __uint_as_float(v[j + 1]);
-            sum2 = add2v(sum2, pack2(y0, y1));
-            ymax0 = fmaxf(ymax0, y0);
-            ymax1 = fmaxf(ymax1, y1);
-            ymin0 = fminf(ymin0, y0);
-            ymin1 = fminf(ymin1, y1);
-          }
-        }
+              for (int j = 0; j < 32; j += 2) {
+                const uint64_t y2 = ypair(v, c, j);
+                float y0, y1;
+                unpack2(y2, y0, y1);
+                sum2 = add2v(sum2, y2);
+                ymax0 = fmaxf(ymax0, y0);
+                ymax1 = fmaxf(ymax1, y1);
+                ymin0 = fminf(ymin0, y0);
+                ymin1 = fminf(ymin1, y1);
+              }
+            },
+            [] {});
         float s0, s1;
         unpack2(sum2, s0, s1);
         const float o = a.offset ? (s0 + s1) * (1.0f / kHd) : 0.f;
@@ -529,54 +624,56 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
         // (the float spacing there is 1) and leaves u = q + 8 in the low bits of
         // the sum; eight of them are packed with shifts and one bias subtraction.
         const uint64_t o2 = pack2(o, o), inv2 = pack2(inv, inv), magic2 = pack2(kRoundMagic, kRoundMagic);
-#pragma unroll 1
-        for (int c = 0; c < kHd / 32; ++c) {
-          uint32_t v[32];
-          tmem_ld_32cols_waited(row_tm + c * 32, v);
-          if (c == kHd / 32 - 1) {
-            // The accumulator's last read: hand it back to the MMA warp.
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(tempty0 + 8 * x);
-          }
-          uint32_t pk[4];
+        tmem_row_pass(
+            row_tm,
+            [&](const uint32_t (&v)[32], int c) {
+              uint32_t pk[4];
 #pragma unroll
-          for (int w8 = 0; w8 < 4; ++w8) {
-            uint32_t word = 0u;
+              for (int w8 = 0; w8 < 4; ++w8) {
+                uint32_t word = 0u;
 #pragma unroll
-            for (int j = 8 * w8 + 6; j >= 8 * w8; j -= 2) {
-              const uint64_t r2 = sub2v(pack2(__uint_as_float(v[j]), __uint_as_float(v[j + 1])), o2);
-              float f0, f1;
-              unpack2(add2v(mul2v(r2, inv2), magic2), f0, f1);
-              word = (word << 4) + __float_as_uint(f1);
-              word = (word << 4) + __float_as_uint(f0);
-            }
-            pk[w8] = word - kRoundMagicBits * 0x11111111u;
-          }
-          if (ok)
-            *reinterpret_cast<uint4*>(a.codes + th * (kHd / 2) + 16 * c) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-        }
+                for (int j = 8 * w8 + 6; j >= 8 * w8; j -= 2) {
+                  const uint64_t r2 = sub2v(ypair(v, c, j), o2);
+                  float f0, f1;
+                  unpack2(add2v(mul2v(r2, inv2), magic2), f0, f1);
+                  word = (word << 4) + __float_as_uint(f1);
+                  word = (word << 4) + __float_as_uint(f0);
+                }
+                pk[w8] = word - kRoundMagicBits * 0x11111111u;
+              }
+              if (ok)
+                *reinterpret_cast<uint4*>(a.codes + th * (kHd / 2) + 16 * c) =
+                    make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            },
+            [&] {
+              // The accumulator's last read: hand it back to the MMA warp.
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(tempty0 + 8 * x);
+            });
         if (ok) {
           a.scale[th] = amax * (1.0f / 7.0f);
           if (a.off != nullptr) a.off[th] = o;
         }
       } else {
-#pragma unroll 1
-        for (int c = 0; c < kHd / 32; ++c) {
-          uint32_t v[32];
-          tmem_ld_32cols_waited(row_tm + c * 32, v);
-          if (c == kHd / 32 - 1) {
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(tempty0 + 8 * x);
-          }
-          if (ok) {
+        tmem_row_pass(
+            row_tm,
+            [&](const uint32_t (&v)[32], int c) {
+              if (ok) {
 #pragma unroll
-            for (int j = 0; j < 32; j += 4)
-              store4<OUT>(a.out, tok * a.ld_out + static_cast<int64_t>(h) * kHd + c * 32 + j, __uint_as_float(v[j]),
-                          __uint_as_float(v[j + 1]), __uint_as_float(v[j + 2]), __uint_as_float(v[j + 3]));
-          }
-        }
+                for (int j = 0; j < 32; j += 4) {
+                  float y0, y1, y2, y3;
+                  unpack2(ypair(v, c, j), y0, y1);
+                  unpack2(ypair(v, c, j + 2), y2, y3);
+                  store4<OUT>(a.out, tok * a.ld_out + static_cast<int64_t>(h) * kHd + c * 32 + j, y0, y1, y2, y3);
+                }
+              }
+            },
+            [&] {
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(tempty0 + 8 * x);
+            });
       }
     }
   }
@@ -651,13 +748,14 @@ int encode_keys_map(CUtensorMap* map, const void* x, int64_t T, int H, int64_t l
   return r == CUDA_SUCCESS ? OFFQ_OK : OFFQ_ERR_CUDA;
 }
 
-template <int OUT>
+template <int OUT, bool REFLECT = false>
 int launch_rotate_mma(const RotArgs& a, cudaStream_t s) {
-  auto kern = rotate_heads_mma_kernel<OUT>;
+  using L = RotLayout<REFLECT>;
+  auto kern = rotate_heads_mma_kernel<OUT, REFLECT>;
   static std::once_flag once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [&] {
-    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kMmaSmem);
+    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kSmem);
   });
   if (attr_err != cudaSuccess) return OFFQ_ERR_CUDA;
   CUtensorMap xmap;
@@ -670,7 +768,7 @@ int launch_rotate_mma(const RotArgs& a, cudaStream_t s) {
   int64_t per_head = sms / a.H > 0 ? sms / a.H : 1;
   if (per_head > tiles) per_head = tiles;
   const dim3 grid(static_cast<unsigned>(per_head), static_cast<unsigned>(a.H));
-  return launch_pdl(kern, grid, dim3(kMmaThreads), kMmaSmem, s, xmap, a);
+  return launch_pdl(kern, grid, dim3(kMmaThreads), L::kSmem, s, xmap, a);
 }
 
 template <int OUT>
@@ -815,6 +913,159 @@ extern "C" int offq_rotate_heads_prepared(const void* x, int dtype, int64_t T, i
     case OFFQ_F32: return launch_rotate_mma<OFFQ_F32>(a, s);
     case OFFQ_BF16: return launch_rotate_mma<OFFQ_BF16>(a, s);
     case OFFQ_F16: return launch_rotate_mma<OFFQ_F16>(a, s);
+    default: return OFFQ_ERR_INVALID_ARG;
+  }
+}
+
+namespace {
+
+// Host round-to-nearest-even of a finite float to bf16 bits.
+uint16_t host_bf16(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  return static_cast<uint16_t>((u + 0x7FFFu + ((u >> 16) & 1u)) >> 16);
+}
+
+float host_bf16_value(uint16_t b) {
+  const uint32_t u = static_cast<uint32_t>(b) << 16;
+  float f;
+  std::memcpy(&f, &u, 4);
+  return f;
+}
+
+}  // namespace
+
+extern "C" int offq_prepare_key_reflection(const float* v, const int32_t* perm, int32_t H, int32_t head_dim,
+                                           void* prepared) {
+  if (H < 1 || head_dim <= 0) return OFFQ_ERR_INVALID_ARG;
+  if (head_dim != kHd) return OFFQ_ERR_UNSUPPORTED;
+  if (H > 65535) return OFFQ_ERR_UNSUPPORTED;
+  if (v == nullptr || perm == nullptr || prepared == nullptr) return OFFQ_ERR_INVALID_ARG;
+  for (int32_t h = 0; h < H; ++h) {
+    bool seen[kHd] = {};
+    double nv = 0.0;
+    for (int c = 0; c < kHd; ++c) {
+      const int32_t p = perm[static_cast<int64_t>(h) * kHd + c];
+      if (p < 0 || p >= kHd || seen[p]) return OFFQ_ERR_INVALID_ARG;
+      seen[p] = true;
+      const double vc = v[static_cast<int64_t>(h) * kHd + c];
+      if (!std::isfinite(vc)) return OFFQ_ERR_INVALID_ARG;
+      nv += vc * vc;
+    }
+    if (!(nv > 0.0)) return OFFQ_ERR_INVALID_ARG;
+  }
+  uint8_t* out = static_cast<uint8_t*>(prepared);
+  for (int32_t h = 0; h < H; ++h) {
+    const float* vh = v + static_cast<int64_t>(h) * kHd;
+    const int32_t* ph = perm + static_cast<int64_t>(h) * kHd;
+    // The reflection taking e_0 to v / |v|: U3 = I - 2 w w^T, w = (v/|v| - e_0)
+    // normalised (U3 = I when v / |v| = e_0), in float64.
+    double nv = 0.0;
+    for (int c = 0; c < kHd; ++c) nv += static_cast<double>(vh[c]) * vh[c];
+    nv = std::sqrt(nv);
+    double w[kHd];
+    double nw = 0.0;
+    for (int c = 0; c < kHd; ++c) {
+      w[c] = vh[c] / nv - (c == 0 ? 1.0 : 0.0);
+      nw += w[c] * w[c];
+    }
+    if (nw < 1e-30) {
+      for (int c = 0; c < kHd; ++c) w[c] = 0.0;
+    } else {
+      nw = std::sqrt(nw);
+      for (int c = 0; c < kHd; ++c) w[c] /= nw;
+    }
+    // (x P3)_c = x_perm[c], so (P3 H)[k][n] = H[inv[k]][n] with inv = perm^-1,
+    // and H[i][n] = (-1)^popcount(i & n) (Sylvester).
+    int inv[kHd];
+    for (int c = 0; c < kHd; ++c) inv[ph[c]] = c;
+    auto ph_entry = [&](int k, int n) { return (__builtin_popcount(static_cast<unsigned>(inv[k] & n)) & 1) ? -1 : 1; };
+    uint8_t* img = out + static_cast<int64_t>(h) * kRefImgBytes;
+    std::memset(img, 0, kRefImgBytes);
+    // Rows 128..130: the three bf16 parts of fp32(w).
+    uint16_t wp[3][kHd];
+    for (int k = 0; k < kHd; ++k) {
+      const float wf = static_cast<float>(w[k]);
+      wp[0][k] = host_bf16(wf);
+      const float r1 = wf - host_bf16_value(wp[0][k]);
+      wp[1][k] = host_bf16(r1);
+      const float r2 = r1 - host_bf16_value(wp[1][k]);
+      wp[2][k] = host_bf16(r2);
+    }
+    for (int r = 0; r < kRefRows; ++r)
+      for (int c = 0; c < kHd / 8; ++c) {
+        uint16_t chunk[8] = {};
+        for (int e = 0; e < 8; ++e) {
+          const int k = 8 * c + e;
+          if (r < kHd) chunk[e] = ph_entry(k, r) > 0 ? 0x3F80u : 0xBF80u;
+          else if (r < kHd + 3) chunk[e] = wp[r - kHd][k];
+        }
+        std::memcpy(img + (c >> 3) * kRefAtom + r * 128 + (((c & 7) ^ (r & 7)) << 4), chunk, 16);
+      }
+    // w'' = (P3 H3)^T w, H3 = H / sqrt(128).
+    float* wpp = reinterpret_cast<float*>(img + kRefBBytes);
+    for (int n = 0; n < kHd; ++n) {
+      double acc = 0.0;
+      for (int k = 0; k < kHd; ++k) acc += ph_entry(k, n) * w[k];
+      wpp[n] = static_cast<float>(acc / std::sqrt(static_cast<double>(kHd)));
+    }
+  }
+  return OFFQ_OK;
+}
+
+extern "C" int offq_kv4_quantize_reflected(const void* kv, int dtype, int64_t T, int32_t H, int32_t head_dim,
+                                           int64_t ld_token, const void* prepared, int32_t flags, uint8_t* codes,
+                                           float* scale, float* offset, void* stream) {
+  if ((flags & ~OFFQ_OFFSET) != 0) return OFFQ_ERR_INVALID_ARG;
+  int st = check_heads(kv, dtype, T, H, head_dim, ld_token, prepared);
+  if (st != OFFQ_OK) return st;
+  if (dtype != OFFQ_BF16) return OFFQ_ERR_UNSUPPORTED;
+  if (T == 0) return OFFQ_OK;
+  if (codes == nullptr || scale == nullptr || ((flags & OFFQ_OFFSET) && offset == nullptr))
+    return OFFQ_ERR_INVALID_ARG;
+  if (!aligned(codes, 16) || !aligned(scale, 4) || (offset != nullptr && !aligned(offset, 4)))
+    return OFFQ_ERR_MISALIGNED;
+  RotArgs a{};
+  a.x = kv;
+  a.ld_token = ld_token;
+  a.T = T;
+  a.H = H;
+  a.prep = prepared;
+  a.quantize = 1;
+  a.offset = (flags & OFFQ_OFFSET) != 0;
+  a.codes = codes;
+  a.scale = scale;
+  a.off = offset;
+  a.status = device_status_ptr();
+  return launch_rotate_mma<OFFQ_F32, true>(a, static_cast<cudaStream_t>(stream));
+}
+
+extern "C" int offq_rotate_heads_reflected(const void* x, int dtype, int64_t T, int32_t H, int32_t head_dim,
+                                           int64_t ld_token, const void* prepared, void* out, int out_dtype,
+                                           int64_t ld_out, void* stream) {
+  const int ob = elem_bytes(out_dtype);
+  if (ob == 0 || ld_out < static_cast<int64_t>(H) * head_dim) return OFFQ_ERR_INVALID_ARG;
+  int st = check_heads(x, dtype, T, H, head_dim, ld_token, prepared);
+  if (st != OFFQ_OK) return st;
+  if (dtype != OFFQ_BF16) return OFFQ_ERR_UNSUPPORTED;
+  if (T == 0) return OFFQ_OK;
+  if (out == nullptr) return OFFQ_ERR_INVALID_ARG;
+  if (!aligned(out, 16) || (ld_out * ob) % 16 != 0) return OFFQ_ERR_MISALIGNED;
+  RotArgs a{};
+  a.x = x;
+  a.ld_token = ld_token;
+  a.T = T;
+  a.H = H;
+  a.prep = prepared;
+  a.quantize = 0;
+  a.out = out;
+  a.ld_out = ld_out;
+  a.status = device_status_ptr();
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  switch (out_dtype) {
+    case OFFQ_F32: return launch_rotate_mma<OFFQ_F32, true>(a, s);
+    case OFFQ_BF16: return launch_rotate_mma<OFFQ_BF16, true>(a, s);
+    case OFFQ_F16: return launch_rotate_mma<OFFQ_F16, true>(a, s);
     default: return OFFQ_ERR_INVALID_ARG;
   }
 }

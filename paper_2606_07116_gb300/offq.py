@@ -64,6 +64,11 @@ _SIGNATURES = {
                                             _c_vp, _c_vp, _c_vp]),
     "offq_rotate_heads_prepared": (_c_int, [_c_vp, _c_int, _c_i64, _c_i32, _c_i32, _c_i64, _c_vp, _c_vp, _c_int,
                                             _c_i64, _c_vp]),
+    "offq_prepare_key_reflection": (_c_int, [_c_vp, _c_vp, _c_i32, _c_i32, _c_vp]),
+    "offq_kv4_quantize_reflected": (_c_int, [_c_vp, _c_int, _c_i64, _c_i32, _c_i32, _c_i64, _c_vp, _c_i32, _c_vp,
+                                             _c_vp, _c_vp, _c_vp]),
+    "offq_rotate_heads_reflected": (_c_int, [_c_vp, _c_int, _c_i64, _c_i32, _c_i32, _c_i64, _c_vp, _c_vp, _c_int,
+                                             _c_i64, _c_vp]),
     "offq_top1_tokens": (_c_int, [_c_vp, _c_int, _c_i64, _c_i64, _c_i64, _c_i64, _c_i64, _c_vp, _c_vp, _c_vp]),
     "offq_top1_direction": (_c_int, [_c_vp, _c_i64, _c_i64, _c_i32, _c_vp, _c_vp, _c_vp, _c_vp]),
     "offq_reflect_rows": (_c_int, [_c_vp, _c_i64, _c_i64, _c_vp, _c_vp, _c_vp]),
@@ -239,6 +244,32 @@ def offq_rotate_heads_prepared(x: torch.Tensor, T: int, H: int, head_dim: int, l
         _stream(stream)))
 
 
+def offq_prepare_key_reflection(v: torch.Tensor, perm: torch.Tensor, H: int, head_dim: int,
+                                prepared: torch.Tensor) -> None:
+    """Host call: v [H, hd] float32, perm [H, hd] int32 and prepared (uint8) all in host memory."""
+    for t in (v, perm, prepared):
+        if t.device.type != "cpu" or not t.is_contiguous():
+            raise ValueError("offq_prepare_key_reflection takes contiguous host tensors")
+    _check("offq_prepare_key_reflection", load_library().offq_prepare_key_reflection(
+        ctypes.c_void_p(v.data_ptr()), ctypes.c_void_p(perm.data_ptr()), H, head_dim,
+        ctypes.c_void_p(prepared.data_ptr())))
+
+
+def offq_kv4_quantize_reflected(kv: torch.Tensor, T: int, H: int, head_dim: int, ld_token: int,
+                                prepared: torch.Tensor, flags: int, codes: torch.Tensor, scale: torch.Tensor,
+                                offset: Optional[torch.Tensor], stream=None) -> None:
+    _check("offq_kv4_quantize_reflected", load_library().offq_kv4_quantize_reflected(
+        _ptr(kv), _dtype_code(kv), T, H, head_dim, ld_token, _ptr(prepared), flags, _ptr(codes), _ptr(scale),
+        _ptr(offset), _stream(stream)))
+
+
+def offq_rotate_heads_reflected(x: torch.Tensor, T: int, H: int, head_dim: int, ld_token: int,
+                                prepared: torch.Tensor, out: torch.Tensor, ld_out: int, stream=None) -> None:
+    _check("offq_rotate_heads_reflected", load_library().offq_rotate_heads_reflected(
+        _ptr(x), _dtype_code(x), T, H, head_dim, ld_token, _ptr(prepared), _ptr(out), _dtype_code(out), ld_out,
+        _stream(stream)))
+
+
 def offq_get_device_status(stream=None) -> int:
     return load_library().offq_get_device_status(_stream(stream))
 
@@ -403,6 +434,45 @@ def rotate_heads_prepared(x: torch.Tensor, prepared: torch.Tensor, out_dtype: to
         raise ValueError("heads of a token must be contiguous")
     out = torch.empty((T, H, hd), dtype=out_dtype, device=x.device)
     offq_rotate_heads_prepared(x, T, H, hd, x.stride(0), prepared, out, out.stride(0), stream)
+    return out
+
+
+KEY_REFLECTION_BYTES = 37376  # OFFQ_KEY_REFLECTION_BYTES: one head's structured rotation
+
+
+def prepare_key_reflection(v: torch.Tensor, perm: torch.Tensor, device=None) -> torch.Tensor:
+    """Top-1 directions v [H, hd] and permutations perm [H, hd] -> the structured
+    image [H, KEY_REFLECTION_BYTES] (uint8), built on the host and copied to `device`."""
+    H, hd = v.shape
+    vh = v.detach().to("cpu", torch.float32).contiguous()
+    ph = perm.detach().to("cpu", torch.int32).contiguous()
+    img = torch.empty((H, KEY_REFLECTION_BYTES), dtype=torch.uint8)
+    offq_prepare_key_reflection(vh, ph, H, hd, img)
+    return img.to(device) if device is not None else img
+
+
+def kv4_quantize_reflected(kv: torch.Tensor, prepared: torch.Tensor, offset: bool = True,
+                           stream=None) -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    """Key-cache codes, scales and offsets of bf16 kv [T, H, hd] under the structured M = U3 P3 H3."""
+    T, H, hd = kv.shape
+    if kv.stride(2) != 1 or kv.stride(1) != hd:
+        raise ValueError("heads of a token must be contiguous")
+    codes = torch.empty((T, H, hd // 2), dtype=torch.uint8, device=kv.device)
+    scale = torch.empty((T, H), dtype=torch.float32, device=kv.device)
+    off = torch.empty((T, H), dtype=torch.float32, device=kv.device)
+    offq_kv4_quantize_reflected(kv, T, H, hd, kv.stride(0), prepared, OFFQ_OFFSET if offset else 0, codes, scale,
+                                off, stream)
+    return codes, scale, off
+
+
+def rotate_heads_reflected(x: torch.Tensor, prepared: torch.Tensor, out_dtype: torch.dtype = torch.float32,
+                           stream=None) -> torch.Tensor:
+    """bf16 x [T, H, hd] rotated per head by the structured M = U3 P3 H3."""
+    T, H, hd = x.shape
+    if x.stride(2) != 1 or x.stride(1) != hd:
+        raise ValueError("heads of a token must be contiguous")
+    out = torch.empty((T, H, hd), dtype=out_dtype, device=x.device)
+    offq_rotate_heads_reflected(x, T, H, hd, x.stride(0), prepared, out, out.stride(0), stream)
     return out
 
 

@@ -3,8 +3,11 @@ rejects bad arguments on the host (no GPU needed: no call here reaches a
 CUDA runtime function)."""
 
 import ctypes
+import math
 
+import numpy as np
 import pytest
+import torch
 
 from paper_2606_07116_gb300 import build as B
 from paper_2606_07116_gb300 import offq as Q
@@ -227,3 +230,75 @@ def test_sorted_grouping_host_matches_oracle(lib):
         m[rng.integers(0, D, size=D // 8)] = 0.5  # ties
         np.testing.assert_array_equal(Q.sorted_grouping(torch.from_numpy(m), G).numpy(),
                                       O.sorted_grouping(m.astype(np.float64), G))
+
+
+def _decode_reflection(img, H):
+    """The structured image back to B [H][144][128] (float64) and w'' [H][128]."""
+    u = np.frombuffer(img.numpy().tobytes(), dtype=np.uint8).reshape(H, -1)
+    b = u[:, :36864].copy().view(np.uint16).reshape(H, 2, 144, 8, 8)   # [h][half][row][slot][e]
+    n = np.arange(144)[:, None]
+    c = np.arange(16)[None, :]
+    g = b[:, c >> 3, n, (c & 7) ^ (n & 7), :]                           # [H, 144, 16, 8]
+    B = ((g.reshape(H, 144, 128).astype(np.uint32) << 16).view(np.float32)).astype(np.float64)
+    wpp = u[:, 36864:].copy().view(np.float32).astype(np.float64)
+    return B, wpp
+
+
+def test_key_reflection_image_matches_the_oracle_rotation(lib):
+    """Host prepare of M = U3 P3 H3: the +-1 rows are sqrt(128) (P3 H3)^T, the
+    three parts of w rebuild the reflection, and w'' = (P3 H3)^T w, so the image
+    gives the oracle's M back (Sec. 3.3 Step 2 (3))."""
+    import oracle as O
+    H, hd = 3, 128
+    rng = np.random.default_rng(5)
+    keys = rng.standard_normal((64, H, hd))
+    keys[:, :, 5] += 30.0                            # a concentrated channel per head
+    keys[:, 2, :] = 0.01 * rng.standard_normal((64, hd))
+    keys[:, 2, 0] += 40.0                            # head 2: direction ~ e_0 (U3 close to I)
+    perm = np.stack([np.concatenate([[0], 1 + rng.permutation(hd - 1)]) for _ in range(H)]).astype(np.int32)
+    v = np.stack([O.top1_pca_direction(keys[:, h, :]) for h in range(H)]).astype(np.float32)
+    img = Q.prepare_key_reflection(torch.from_numpy(v), torch.from_numpy(perm))
+    B, wpp = _decode_reflection(img, H)
+    Hs = O.sylvester_hadamard(hd).astype(np.float64) / math.sqrt(hd)
+    for h in range(H):
+        PH = np.eye(hd)[:, perm[h]] @ Hs
+        assert np.array_equal(B[h, :hd], np.sign(PH.T))  # sqrt(128) (P3 H3)[k][n] = +-1 at row n
+        assert np.all(B[h, hd + 3:] == 0)
+        w = B[h, hd] + B[h, hd + 1] + B[h, hd + 2]
+        U = np.eye(hd) - 2.0 * np.outer(w, w)
+        M_img = U @ PH
+        M_ref = O.householder_to_first(v[h].astype(np.float64)) @ PH
+        assert np.max(np.abs(M_img - M_ref)) < 1e-6
+        # w'' from the float64 w, rounded once; w here is fp32(w) (its parts'
+        # sum), at most 2^-24 |w_k| from the float64 w in each entry.
+        tol = 2.0 ** -24 * (np.abs(PH.T @ w) + np.abs(PH.T) @ np.abs(w)) * 2
+        assert np.all(np.abs(wpp[h] - PH.T @ w) <= tol)
+
+
+def test_key_reflection_argument_checks(lib):
+    hd = 128
+    v = torch.ones((2, hd), dtype=torch.float32)
+    perm = torch.arange(hd, dtype=torch.int32).repeat(2, 1)
+    out = torch.empty((2, Q.KEY_REFLECTION_BYTES), dtype=torch.uint8)
+    call = lambda v=v, perm=perm, H=2, hd=hd: lib.offq_prepare_key_reflection(
+        ctypes.c_void_p(v.data_ptr()), ctypes.c_void_p(perm.data_ptr()), H, hd, ctypes.c_void_p(out.data_ptr()))
+    assert call() == Q.OFFQ_OK
+    assert call(hd=64) == Q.OFFQ_ERR_UNSUPPORTED
+    assert call(H=0) == Q.OFFQ_ERR_INVALID_ARG
+    bad = perm.clone(); bad[1, 7] = 3                # not a permutation
+    assert call(perm=bad) == Q.OFFQ_ERR_INVALID_ARG
+    zero = v.clone(); zero[1] = 0.0                   # no direction
+    assert call(v=zero) == Q.OFFQ_ERR_INVALID_ARG
+    assert lib.offq_prepare_key_reflection(None, None, 2, hd, None) == Q.OFFQ_ERR_INVALID_ARG
+    kr = lambda dt=Q.OFFQ_BF16, prep=A16, flags=2, T=4: \
+        lib.offq_kv4_quantize_reflected(A16, dt, T, 8, 128, 1024, prep, flags, A16, A16, A16, None)
+    assert kr(dt=Q.OFFQ_F32) == Q.OFFQ_ERR_UNSUPPORTED
+    assert kr(prep=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert kr(prep=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert kr(flags=1) == Q.OFFQ_ERR_INVALID_ARG
+    assert kr(T=0) == Q.OFFQ_OK
+    rr = lambda dt=Q.OFFQ_BF16, out=A16, T=4: \
+        lib.offq_rotate_heads_reflected(A16, dt, T, 8, 128, 1024, A16, out, Q.OFFQ_F32, 1024, None)
+    assert rr(dt=Q.OFFQ_F16) == Q.OFFQ_ERR_UNSUPPORTED
+    assert rr(out=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert rr(T=0) == Q.OFFQ_OK

@@ -56,10 +56,11 @@ def _bound_y(x, M, tc=False):
     return factor * U32 * np.einsum("thi,hij->thj", np.abs(x), np.abs(M.astype(np.float64)))
 
 
-def _check_key_cache(codes, scale, off, x, M, offset=True, tc=False):
+def _check_key_cache(codes, scale, off, x, M, offset=True, tc=False, by=None):
     T, H, _ = x.shape
     ref = O.kv4_quantize_dense(x, M.astype(np.float64), offset=offset)
-    by = _bound_y(x, M, tc).max(axis=2)                # per (t, h)
+    if by is None:
+        by = _bound_y(x, M, tc).max(axis=2)            # per (t, h)
     y_abs = np.abs(ref["y"]).sum(axis=2)
     bo = by + (HD + 2 if tc else 8) * U32 * y_abs / HD if offset else np.zeros_like(by)
     s_gpu, s_ref = scale.cpu().numpy().astype(np.float64), ref["scale"]
@@ -244,3 +245,90 @@ def test_prepared_key_cache_full_size():
     torch.cuda.synchronize()
     assert Q.offq_get_device_status() == Q.OFFQ_OK
     _check_key_cache(codes, scale, off, kt.to(torch.float64).numpy(), M, tc=True)
+
+
+# ---------------------------------------------------------------------------
+# The structured form M = U3 P3 H3 (offq_prepare_key_reflection and the
+# *_reflected calls): y = fma(acc, fp32(1/sqrt(128)), fl(-2 d w'')) with
+# acc = sqrt(128) x P3 H3 (exact +-1 products, fp32 sum over 128 terms) and
+# d = x . w (exact products with w's three bf16 parts, fp32 sums). With A =
+# sum |x_i|, Bw = sum |x_i w_i|, u = x P3 H3, each y_j is within
+#   u32 [ (2 hd + 8) A / sqrt(hd) + 2 |u_j| + 2 |w''_j| (2 hd + 12) Bw + 4 |d| |w''_j| + |y_j| ]
+# of its float64 value: the accumulations (a full ulp per addition), fp32(1/sqrt(128)),
+# fp32(w) and fp32(w''), the product -2 d w''_j and the final fma.
+# ---------------------------------------------------------------------------
+def _reflection_case(T, H, seed, e0_head=False):
+    k = _keys(T, H, seed)
+    rng = np.random.default_rng(seed + 1)
+    perm = np.stack([np.concatenate([[0], 1 + rng.permutation(HD - 1)]) for _ in range(H)]).astype(np.int32)
+    v = np.stack([O.top1_pca_direction(k[:, h, :]) for h in range(H)]).astype(np.float32)
+    if e0_head:
+        v[0] = 0.0
+        v[0, 0] = 1.0                                  # U3 = I for head 0
+    Hs = O.sylvester_hadamard(HD).astype(np.float64) / math.sqrt(HD)
+    PH = np.stack([np.eye(HD)[:, perm[h]] @ Hs for h in range(H)])
+    U = np.stack([O.householder_to_first(v[h].astype(np.float64)) for h in range(H)])
+    M = np.einsum("hij,hjk->hik", U, PH)
+    return k, v, perm, M, U, PH
+
+
+def _bound_reflected(x, U, PH):
+    T, H, _ = x.shape
+    W = np.zeros((H, HD))
+    for h in range(H):
+        lam, vec = np.linalg.eigh(U[h])               # U = I - 2 w w^T: w is the eigenvector of eigenvalue -1
+        if lam[0] < 0:
+            W[h] = vec[:, 0]
+    w2 = np.einsum("hkn,hk->hn", PH, W)
+    A = np.abs(x).sum(axis=2)
+    Bw = np.einsum("thi,hi->th", np.abs(x), np.abs(W))
+    d = np.einsum("thi,hi->th", x, W)
+    u = np.einsum("thi,hij->thj", x, PH)
+    y = u - 2 * d[..., None] * w2[None]
+    return U32 * ((2 * HD + 8) * A[..., None] / math.sqrt(HD) + 2 * np.abs(u)
+                  + 2 * np.abs(w2)[None] * (2 * HD + 12) * Bw[..., None]
+                  + 4 * np.abs(d)[..., None] * np.abs(w2)[None] + np.abs(y))
+
+
+@pytest.mark.parametrize("T,H,e0", [(1, 4, False), (45, 4, True), (300, 8, False), (600, 160, True)])
+def test_reflected_key_cache_parity(T, H, e0):
+    k, v, perm, M, U, PH = _reflection_case(T, H, seed=110 + T, e0_head=e0)
+    kt = torch.from_numpy(k).to(torch.bfloat16)
+    x = kt.to(torch.float64).numpy()
+    prep = Q.prepare_key_reflection(torch.from_numpy(v), torch.from_numpy(perm), device="cuda")
+    by = _bound_reflected(x, U, PH).max(axis=2)
+    for offset in (True, False):
+        codes, scale, off = Q.kv4_quantize_reflected(kt.cuda(), prep, offset=offset)
+        torch.cuda.synchronize()
+        assert Q.offq_get_device_status() == Q.OFFQ_OK
+        _check_key_cache(codes, scale, off if offset else None, x, M, offset=offset, by=by)
+
+
+@pytest.mark.parametrize("odt", [torch.float32, torch.bfloat16, torch.float16])
+def test_rotate_heads_reflected_parity(odt):
+    T, H = 333, 8
+    k, v, perm, M, U, PH = _reflection_case(64, H, seed=120)
+    q = np.random.default_rng(121).standard_normal((T, H, HD)) * 3.0
+    qt = torch.from_numpy(q).to(torch.bfloat16)
+    x = qt.to(torch.float64).numpy()
+    prep = Q.prepare_key_reflection(torch.from_numpy(v), torch.from_numpy(perm), device="cuda")
+    y = Q.rotate_heads_reflected(qt.cuda(), prep, out_dtype=odt)
+    torch.cuda.synchronize()
+    ref = O.rotate_heads(x, M)
+    rnd = {torch.float32: 0.0, torch.bfloat16: 2.0 ** -8, torch.float16: 2.0 ** -11}[odt]
+    tol = _bound_reflected(x, U, PH) * (1 + rnd) + rnd * np.abs(ref)
+    err = np.abs(y.float().cpu().numpy().astype(np.float64) - ref)
+    assert np.all(err <= tol + 1e-30), f"worst {np.max(err / (tol + 1e-30)):.3g}x the bound"
+
+
+def test_reflected_key_cache_full_size():
+    """The workload's key tensor, 2048 tokens x 32 heads, with the structured M."""
+    T, H = 2048, 32
+    k, v, perm, M, U, PH = _reflection_case(T, H, seed=130)
+    kt = torch.from_numpy(k).to(torch.bfloat16)
+    x = kt.to(torch.float64).numpy()
+    prep = Q.prepare_key_reflection(torch.from_numpy(v), torch.from_numpy(perm), device="cuda")
+    codes, scale, off = Q.kv4_quantize_reflected(kt.cuda(), prep)
+    torch.cuda.synchronize()
+    assert Q.offq_get_device_status() == Q.OFFQ_OK
+    _check_key_cache(codes, scale, off, x, M, by=_bound_reflected(x, U, PH).max(axis=2))
