@@ -816,9 +816,26 @@ def main():
     ap.add_argument("--no-group", action="store_true", help="skip the per-group asymmetric path's timing")
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work for cpu_baseline")
     ap.add_argument("--ref-budget", type=float, default=120.0, help="seconds of oracle work for --impl reference")
+    ap.add_argument("--key-rotation-tokens", type=int, default=0,
+                    help="time only the key-cache rotation calls, at this many tokens, and print that object "
+                         "(a side measurement for profiling, not the bench line)")
     args = ap.parse_args()
     if args.warmup < 3:
         raise SystemExit("--warmup must be at least 3")
+    if args.key_rotation_tokens > 0:
+        import torch
+        device = torch.device("cuda", 0)
+        torch.cuda.set_device(device)
+        w = workload_by_name(args.workload)
+        flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
+
+        def flush_l2():
+            flush.zero_()
+            flush[:L2_FLUSH_BYTES // 2].view(torch.int32).amax()
+
+        print(json.dumps(time_key_rotation(w, args.key_rotation_tokens, device, args, flush_l2,
+                                           torch.cuda.current_stream(device))), flush=True)
+        return
 
     world = _env_int("WORLD_SIZE", 1)
     rank = _env_int("RANK", 0)
