@@ -300,6 +300,50 @@ __device__ __forceinline__ uint64_t sub2v(uint64_t a, uint64_t b) {
   return r;
 }
 
+// Shared -> global TMA store of one box (tensor coordinates x, y), tracked in
+// this thread's bulk groups; rows past the tensor are not written.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, uint32_t src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(map),
+               "r"(src), "r"(x), "r"(y)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// This thread's bulk stores have read their shared-memory source.
+__device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// This thread's bulk stores are complete.
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+// Barrier over the 128 threads of named barrier `id`.
+__device__ __forceinline__ void wg_sync(int id) { asm volatile("bar.sync %0, 128;" ::"r"(id) : "memory"); }
+
+// The same barrier, returning whether `pred` held for any of the 128 threads.
+__device__ __forceinline__ bool wg_any(int id, bool pred) {
+  uint32_t r;
+  asm volatile(
+      "{\n"
+      ".reg .pred p, q;\n"
+      "setp.ne.b32 p, %1, 0;\n"
+      "bar.red.or.pred q, %2, 128, p;\n"
+      "selp.u32 %0, 1, 0, q;\n"
+      "}\n"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(pred)), "r"(id)
+      : "memory");
+  return r != 0;
+}
+
+// Two floats as one 32-bit word of 16-bit values (round to nearest even).
+template <int OUT>
+__device__ __forceinline__ uint32_t pack16(float a, float b) {
+  if constexpr (OUT == OFFQ_BF16) {
+    const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<const uint32_t*>(&v);
+  } else {
+    const __half2 v = __floats2half2_rn(a, b);
+    return *reinterpret_cast<const uint32_t*>(&v);
+  }
+}
+
 // Global -> shared bulk copy (async proxy), completing `bytes` on an mbarrier.
 __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
   asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
@@ -417,8 +461,12 @@ __global__ void __launch_bounds__(128) prepare_rotation_kernel(const float* __re
 // N = 144 per 16 channels; the epilogue forms y = u - 2 (x . w) w'').
 template <int OUT, bool REFLECT>
 __global__ void __launch_bounds__(kMmaThreads, 1)
-    rotate_heads_mma_kernel(const __grid_constant__ CUtensorMap xmap, const RotArgs a) {
+    rotate_heads_mma_kernel(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap omap,
+                            const RotArgs a) {
   using L = RotLayout<REFLECT>;
+  // 16-bit rotated outputs (the query side) are staged in the tile's own ring
+  // slot and leave by TMA stores; the slot is freed after the store has read it.
+  constexpr bool kStage = OUT != OFFQ_F32;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -528,7 +576,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
                          (sp | kk) != 0 ? 1u : 0u);
               }
           }
-          mma_commit(empty0 + 8 * s);  // the tile buffer is free once these MMAs are done
+          if constexpr (!kStage) mma_commit(empty0 + 8 * s);  // the tile buffer is free once these MMAs are done
           mma_commit(tfull0 + 8 * x);
           committed = i;
         }
@@ -564,7 +612,9 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
     for (int i = e; i < n_local; i += kEpi) {
       const int x = i % kAcc;
       const bool waited = mbar_wait(tfull0 + 8 * x, (i / kAcc) & 1, abort);
-      if (__any_sync(0xFFFFFFFFu, !waited)) break;  // the warp leaves together
+      // The warp leaves together; with staged outputs (a group barrier per
+      // tile) the whole group does.
+      if (kStage ? wg_any(1 + e, !waited) : __any_sync(0xFFFFFFFFu, !waited)) break;
       tc_fence_after();
       const uint32_t row_tm = tmem + x * L::kAccCols + (static_cast<uint32_t>(q * 32) << 16);
       // y for columns (j, j + 1) of a 32-column chunk c: the accumulator, or
@@ -655,6 +705,41 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
           a.scale[th] = amax * (1.0f / 7.0f);
           if (a.off != nullptr) a.off[th] = o;
         }
+      } else if constexpr (kStage) {
+        // Row q * 32 + lane of the slot, in the swizzled layout of the
+        // output tensor map's two 64-channel boxes.
+        const int s = i % L::kSlots;
+        const uint32_t st = ring + s * kOpBytes;
+        tmem_row_pass(
+            row_tm,
+            [&](const uint32_t (&v)[32], int c) {
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                uint32_t pk[4];
+#pragma unroll
+                for (int p = 0; p < 4; ++p) {
+                  float y0, y1;
+                  unpack2(ypair(v, c, 8 * k + 2 * p), y0, y1);
+                  pk[p] = pack16<OUT>(y0, y1);
+                }
+                sts128v(st + sw_off(q * 32 + lane, 4 * c + k), make_uint4(pk[0], pk[1], pk[2], pk[3]));
+              }
+            },
+            [&] {
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(tempty0 + 8 * x);
+            });
+        fence_proxy_async_smem();  // the staged rows, visible to the TMA unit
+        wg_sync(1 + e);
+        if (warp == 2 + 4 * e && lane == 0) {
+          const int y0 = static_cast<int>((blockIdx.x + static_cast<int64_t>(i) * gridDim.x) * kTM);
+          tma_store_2d(&omap, st, h * kHd, y0);
+          tma_store_2d(&omap, st + kAtomBytes, h * kHd + 64, y0);
+          bulk_commit();
+          bulk_wait_read_all();
+          mbar_arrive(empty0 + 8 * s);
+        }
       } else {
         tmem_row_pass(
             row_tm,
@@ -675,6 +760,9 @@ __global__ void __launch_bounds__(kMmaThreads, 1)
               if (lane == 0) mbar_arrive(tempty0 + 8 * x);
             });
       }
+    }
+    if constexpr (kStage) {
+      if (warp == 2 + 4 * e && lane == 0) bulk_wait_all();  // the stores are complete before the CTA exits
     }
   }
   tc_fence_before();
@@ -732,17 +820,19 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   return fn;
 }
 
-// The bf16 keys as a 2-D tensor of T rows of H * 128 channels (row pitch
-// ld_token elements), read in boxes of 64 channels x 128 tokens with the
-// 128-byte swizzle of the MMA operand; rows past T read as zeros.
-int encode_keys_map(CUtensorMap* map, const void* x, int64_t T, int H, int64_t ld_token) {
+// A [T][H * 128] tensor of 16-bit elements (row pitch ld elements) in boxes
+// of 64 channels x 128 tokens with the 128-byte swizzle of the MMA operand:
+// the bf16 keys read (rows past T read as zeros), or the 16-bit rotated
+// outputs written (rows past T are not written).
+int encode_heads_map(CUtensorMap* map, const void* x, int dtype, int64_t T, int H, int64_t ld) {
   const auto enc = tensor_map_encoder();
   if (enc == nullptr) return OFFQ_ERR_CUDA;
   const cuuint64_t dims[2] = {static_cast<cuuint64_t>(H) * kHd, static_cast<cuuint64_t>(T)};
-  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld_token) * 2};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
   const cuuint32_t box[2] = {64, kTM};
   const cuuint32_t elem_strides[2] = {1, 1};
-  const CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(x), dims, strides, box,
+  const CUresult r = enc(map, dtype == OFFQ_F16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                         const_cast<void*>(x), dims, strides, box,
                          elem_strides, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS ? OFFQ_OK : OFFQ_ERR_CUDA;
@@ -758,8 +848,13 @@ int launch_rotate_mma(const RotArgs& a, cudaStream_t s) {
     attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kSmem);
   });
   if (attr_err != cudaSuccess) return OFFQ_ERR_CUDA;
-  CUtensorMap xmap;
-  if (encode_keys_map(&xmap, a.x, a.T, a.H, a.ld_token) != OFFQ_OK) return OFFQ_ERR_CUDA;
+  CUtensorMap xmap, omap;
+  if (encode_heads_map(&xmap, a.x, OFFQ_BF16, a.T, a.H, a.ld_token) != OFFQ_OK) return OFFQ_ERR_CUDA;
+  if constexpr (OUT != OFFQ_F32) {
+    if (encode_heads_map(&omap, a.out, OUT, a.T, a.H, a.ld_out) != OFFQ_OK) return OFFQ_ERR_CUDA;
+  } else {
+    omap = xmap;  // not used
+  }
   // One CTA per SM (shared memory), spread over the heads; each takes every
   // gridDim.x-th of its head's 128-token tiles.
   const int sms = rot_num_sms();
@@ -768,7 +863,7 @@ int launch_rotate_mma(const RotArgs& a, cudaStream_t s) {
   int64_t per_head = sms / a.H > 0 ? sms / a.H : 1;
   if (per_head > tiles) per_head = tiles;
   const dim3 grid(static_cast<unsigned>(per_head), static_cast<unsigned>(a.H));
-  return launch_pdl(kern, grid, dim3(kMmaThreads), L::kSmem, s, xmap, a);
+  return launch_pdl(kern, grid, dim3(kMmaThreads), L::kSmem, s, xmap, omap, a);
 }
 
 template <int OUT>

@@ -332,3 +332,27 @@ def test_reflected_key_cache_full_size():
     torch.cuda.synchronize()
     assert Q.offq_get_device_status() == Q.OFFQ_OK
     _check_key_cache(codes, scale, off, x, M, by=_bound_reflected(x, U, PH).max(axis=2))
+
+
+@pytest.mark.parametrize("odt", [torch.bfloat16, torch.float16])
+def test_rotate_heads_staged_store_ragged_and_padded(odt):
+    """16-bit outputs leave by TMA stores of 128-token boxes: one token and 45
+    tokens (partial boxes), an output row pitch past the heads whose padding
+    must stay untouched, and the same values as the fp32 output rounded once."""
+    for T in (1, 45):
+        H = 4
+        k, v, perm, M, U, PH = _reflection_case(16, H, seed=140 + T)
+        x = torch.from_numpy(np.random.default_rng(141 + T).standard_normal((T, H, HD))).to(torch.bfloat16).cuda()
+        rot = torch.from_numpy(M.astype(np.float32)).cuda()
+        prep = Q.prepare_key_rotation(rot)
+        refl = Q.prepare_key_reflection(torch.from_numpy(v), torch.from_numpy(perm), device="cuda")
+        ld = H * HD + 72
+        for call, img in ((Q.offq_rotate_heads_prepared, prep), (Q.offq_rotate_heads_reflected, refl)):
+            out = torch.full((T, ld), 7.0, dtype=odt, device="cuda")
+            call(x, T, H, HD, x.stride(0), img, out, ld)
+            ref = torch.empty((T, H, HD), dtype=torch.float32, device="cuda")
+            call(x, T, H, HD, x.stride(0), img, ref, H * HD)
+            torch.cuda.synchronize()
+            assert Q.offq_get_device_status() == Q.OFFQ_OK
+            assert torch.all(out[:, H * HD:] == 7.0), "padding written"
+            assert torch.equal(out[:, :H * HD], ref.reshape(T, H * HD).to(odt))
