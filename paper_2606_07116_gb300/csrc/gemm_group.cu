@@ -12,13 +12,18 @@
 // times 2^-18 below 2^24 * 2^-18, is exact in the fp32 accumulator.
 //
 // One 128-code k-tile is one group, so the per-(token, group) scale cannot sit
-// in the operands: the pair MMA (M 256, N 128) writes each group's P_j into one
-// of two TMEM partial buffers, and eight scaler warps fold it into a running
-// fp32 sum held in their registers,
-//   d = fma(-z, R, P)   (exact while |z R| < 2^24),   S = fma(s, d, S),
-// (on the accumulator's P * 2^-18, with -z * 2^-18 and s * 2^18),
+// in the operands, but the zero-point can: P_j - z R_j = sum (u - z) q_w. The A
+// converters widen u - zc with zc = clamp(z, 0, 15) (|u - zc| <= 15 is exact
+// in E4M3), the pair MMA (M 256, N 128) writes each group's P_j - zc R_j into
+// one of two TMEM partial buffers, and eight scaler warps fold it into a
+// running fp32 sum held in their registers,
+//   d = fma(-(z - zc), R, acc)   (only in a warp with a row whose group does
+//                                 not straddle zero; exact while |z R| < 2^24),
+//   S = fma(s, d, S),
+// (on the accumulator's values * 2^-18, with the factors scaled to match),
 // while the MMA fills the other buffer. After a tile's last group the scalers
-// multiply by s_w and store y, rounding once to the output type.
+// multiply by s_w and store y, rounding once to the output type. d equals
+// P_j - z R_j exactly either way, so the result does not depend on zc.
 //
 // TMEM (512 columns per CTA): P0 [0, 128), P1 [128, 256), 6 A stages of 32
 // columns [256, 448). The N = 128 pair tile keeps both partials next to the
@@ -115,6 +120,17 @@ __device__ __forceinline__ void load_group_kt(const uint8_t* blk, int kchunks, i
     else
       v[j] = make_uint4(0u, 0u, 0u, 0u);
   }
+}
+
+// Eight activation codes u (nibbles) minus a zero-point zc in [0, 15], as eight
+// E4M3 bytes of (u - zc) * 2^-9 in widen_act's order: sign at bit 7, |u - zc|
+// in bits 0-3 (exact, like the plain codes). c4 = 0x80808080 - zc * 0x01010101,
+// z4 = zc * 0x01010101. Byte-wise, u + c4 = 0x80 + u - zc never borrows from
+// the next byte, and its bit 7 is clear exactly when u < zc.
+__device__ __forceinline__ void widen_act_zp(uint32_t w, uint32_t c4, uint32_t z4, uint32_t& lo, uint32_t& hi) {
+  const uint32_t u0 = w & 0x0F0F0F0Fu, u1 = (w >> 4) & 0x0F0F0F0Fu;
+  lo = (~(u0 + c4) & 0x80808080u) | __vabsdiffu4(u0, z4);
+  hi = (~(u1 + c4) & 0x80808080u) | __vabsdiffu4(u1, z4);
 }
 
 // Two 64-bit shared-memory words (four floats as two packed pairs).
@@ -246,18 +262,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGThreads, 1)
         tile += clusters;
       }
     };
+    // A warps: this lane's row's zero-point of each loaded k-tile (group),
+    // clamped to [0, 15], to subtract in the operand.
+    auto load_zc = [&](int tile, int kt) -> uint32_t {
+      const int t = (tile / p.n_tiles) * 2 * GBM + static_cast<int>(rank) * GBM + quarter * 32 + lane;
+      const float z = t < p.T ? __ldg(p.a_zero + static_cast<int64_t>(t) * p.Gq + kt) : 0.f;
+      return static_cast<uint32_t>(fminf(fmaxf(z, 0.f), 15.f));
+    };
     uint4 ring[kGRing][kGChunks];
+    uint32_t zring[kGRing];
     int ld_tile = cluster, ld_kt = 0;
     int blk_tile = ld_tile;
     const uint8_t* blk = block_ptr(ld_tile);
 #pragma unroll
     for (int r = 0; r < kGRing; ++r) {
+      zring[r] = 0u;
       if (ld_tile < num_tiles) {
         if (ld_tile != blk_tile) {
           blk_tile = ld_tile;
           blk = block_ptr(ld_tile);
         }
         load_group_kt(blk, p.kchunks, ld_kt, ring[r]);
+        if (is_a) zring[r] = load_zc(ld_tile, ld_kt);
       }
       advance(ld_tile, ld_kt);
     }
@@ -276,13 +302,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGThreads, 1)
         }
         if (is_a) {
           tc_fence_after();
+          const uint32_t z4 = zring[r] * 0x01010101u, c4 = 0x80808080u - z4;
           uint32_t f8[32];
 #pragma unroll
           for (int c = 0; c < kGChunks; ++c) {
-            widen_act(ring[r][c].x, f8[8 * c + 0], f8[8 * c + 1]);
-            widen_act(ring[r][c].y, f8[8 * c + 2], f8[8 * c + 3]);
-            widen_act(ring[r][c].z, f8[8 * c + 4], f8[8 * c + 5]);
-            widen_act(ring[r][c].w, f8[8 * c + 6], f8[8 * c + 7]);
+            widen_act_zp(ring[r][c].x, c4, z4, f8[8 * c + 0], f8[8 * c + 1]);
+            widen_act_zp(ring[r][c].y, c4, z4, f8[8 * c + 2], f8[8 * c + 3]);
+            widen_act_zp(ring[r][c].z, c4, z4, f8[8 * c + 4], f8[8 * c + 5]);
+            widen_act_zp(ring[r][c].w, c4, z4, f8[8 * c + 6], f8[8 * c + 7]);
           }
           tmem_st_32cols(tmem + (static_cast<uint32_t>(quarter * 32) << 16) + kGACol0 + s * kGAColsPerStage, f8);
           tmem_st_wait();
@@ -311,6 +338,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGThreads, 1)
             blk = block_ptr(ld_tile);
           }
           load_group_kt(blk, p.kchunks, ld_kt, ring[r]);
+          if (is_a) zring[r] = load_zc(ld_tile, ld_kt);
         }
         advance(ld_tile, ld_kt);
         advance(tile, kt);
@@ -363,10 +391,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGThreads, 1)
       for (int kt = 0; kt < nk; ++kt, ++j) {
         const uint32_t b = j & 1u, use = j >> 1;
         const bool last = kt == nk - 1;
-        // The accumulator holds P * 2^-18 (each E4M3 operand carries 2^-9):
-        // d' = P 2^-18 - z R 2^-18 and s 2^18 d' = s (P - z R), all exact scalings.
+        // The accumulator holds (P - zc R) * 2^-18: the A operand already carries
+        // u - zc with zc = clamp(z, 0, 15), and each E4M3 operand 2^-9. What is
+        // left of the zero-point, (z - zc) R, is nonzero only for a group that
+        // does not straddle zero; a warp with such a row adds it here:
+        // d' = acc - (z - zc) R 2^-18 and s 2^18 d' = s (P - z R), all exact.
         const float sg = s_next * 262144.0f;
-        const float nz = z_next * -3.814697265625e-06f;
+        const float dz = z_next - fminf(fmaxf(z_next, 0.f), 15.f);
+        const float nz = dz * -3.814697265625e-06f;
+        const bool fix = __any_sync(0xFFFFFFFFu, dz != 0.f);
         if (row_ok && kt + 1 < nk) {
           s_next = __ldg(srow + kt + 1);
           z_next = __ldg(zrow + kt + 1);
@@ -395,12 +428,25 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGThreads, 1)
             __syncwarp();
             if (lane == 0) arrive_cluster(pempty_l + 8u * b);
           }
+          if (fix) {
+            // The zero-point's remainder, in place: d = fma(-(z - zc) 2^-18, R, acc).
+#pragma unroll
+            for (int q4 = 0; q4 < 8; ++q4) {
+              uint64_t r01, r23;
+              lds_2x64(rrow + (c * 32 + 4 * q4) * 4, r01, r23);
+              float f0, f1, f2, f3;
+              unpack2(fma2v(NZ, r01, pack2(__uint_as_float(pv[4 * q4]), __uint_as_float(pv[4 * q4 + 1]))), f0, f1);
+              unpack2(fma2v(NZ, r23, pack2(__uint_as_float(pv[4 * q4 + 2]), __uint_as_float(pv[4 * q4 + 3]))), f2, f3);
+              pv[4 * q4] = __float_as_uint(f0);
+              pv[4 * q4 + 1] = __float_as_uint(f1);
+              pv[4 * q4 + 2] = __float_as_uint(f2);
+              pv[4 * q4 + 3] = __float_as_uint(f3);
+            }
+          }
 #pragma unroll
           for (int q4 = 0; q4 < 8; ++q4) {
-            uint64_t r01, r23;
-            lds_2x64(rrow + (c * 32 + 4 * q4) * 4, r01, r23);
-            const uint64_t d0 = fma2v(NZ, r01, pack2(__uint_as_float(pv[4 * q4]), __uint_as_float(pv[4 * q4 + 1])));
-            const uint64_t d1 = fma2v(NZ, r23, pack2(__uint_as_float(pv[4 * q4 + 2]), __uint_as_float(pv[4 * q4 + 3])));
+            const uint64_t d0 = pack2(__uint_as_float(pv[4 * q4]), __uint_as_float(pv[4 * q4 + 1]));
+            const uint64_t d1 = pack2(__uint_as_float(pv[4 * q4 + 2]), __uint_as_float(pv[4 * q4 + 3]));
             uint64_t& a0 = S2[c * 16 + 2 * q4];
             uint64_t& a1 = S2[c * 16 + 2 * q4 + 1];
             if (kt == 0) {

@@ -95,8 +95,9 @@ def test_weight_group_sums_exact(N, K, g):
     np.testing.assert_array_equal(sums.cpu().numpy(), O.weight_group_sums(qw, 128).astype(np.float32))
 
 
-def _check_group_layer(T, K, N, g, out_dt, rotate, seed=0, rows=None, ldo=None, mult=60.0):
-    x = W.activations(T, K, seed=seed, n_out=3, mult=mult)
+def _check_group_layer(T, K, N, g, out_dt, rotate, seed=0, rows=None, ldo=None, mult=60.0, x=None):
+    if x is None:
+        x = W.activations(T, K, seed=seed, n_out=3, mult=mult)
     w = W.weights(N, K, seed=seed + 1)
     xt = torch.from_numpy(x).to(torch.bfloat16).cuda()
     a_codes, a_scale, a_zero = Q.quantize_act_group(xt, g, rotate=rotate)
@@ -177,3 +178,24 @@ def test_group_gemm_is_repeatable():
     y2 = Q.w4a4_linear_group(*a, wc, ws, gs)
     torch.cuda.synchronize()
     assert torch.equal(y1, y2)
+
+
+def test_group_gemm_zero_points_outside_the_code_range():
+    """Groups that do not straddle zero have z = -rne(min/s) outside [0, 15]:
+    the kernel subtracts clamp(z, 0, 15) in the operand and the rest through
+    the weight group sums. Shifted groups are mixed with ordinary ones within
+    each warp's 32 rows."""
+    T, K, N = 300, 1024, 640
+    x = W.activations(T, K, seed=90, n_out=3, mult=60.0)
+    rng = np.random.default_rng(91)
+    for t in range(T):
+        if t % 3 == 0:
+            j = rng.integers(0, K // 128)
+            x[t, 128 * j:128 * (j + 1)] += rng.choice([-1.0, 1.0]) * rng.uniform(20.0, 200.0)
+    x[7] = np.abs(x[7]) + 1.0                          # every group of a row positive
+    x[8] = -np.abs(x[8]) - 1.0                         # every group negative
+    xt = torch.from_numpy(x).to(torch.bfloat16).cuda()
+    _, _, zero = Q.quantize_act_group(xt, 1024, rotate=False)
+    z = zero.cpu().numpy()
+    assert (z < 0).any() and (z > 15).any() and ((z >= 0) & (z <= 15)).any()
+    _check_group_layer(T, K, N, 1024, "f32", False, x=x)
