@@ -522,6 +522,81 @@ def time_builder(device, args, flush_l2, stream):
     }
 
 
+def device_activations(T: int, K: int, w: W.Workload, seed: int, device):
+    """The workload's activation recipe drawn on the device (seeded): N(0, 1) or
+    Student-t(3) entries, plus the outlier channels with per-token jitter, in bf16.
+    For timing only: rows this large take too long to draw on the host."""
+    import torch
+    gen = torch.Generator(device=device).manual_seed(seed)
+    x = torch.randn((T, K), generator=gen, device=device)
+    if w.dist == "student_t3":
+        chi2 = sum(torch.randn((T, K), generator=gen, device=device) ** 2 for _ in range(3))
+        x /= torch.sqrt(chi2 / 3.0)
+    if w.n_out > 0 and w.mult != 0.0:
+        amp = w.mult * (1.0 + 0.1 * torch.randn((T,), generator=gen, device=device))
+        for c in W.outlier_channels(K, w.n_out):
+            x[:, c] = amp
+    return x.to(torch.bfloat16)
+
+
+def time_quant_sites(device, args, flush_l2, stream):
+    """The activation quantizer alone on the prefill inputs of the larger Llama
+    shapes (Llama-3-8B MLP at 4096 tokens, Llama-2-70B at 8192 tokens): rows
+    long enough that the launch cost no longer hides the kernel's streaming
+    rate. Per-call events, L2 flushed before each call."""
+    import torch
+    from paper_2606_07116_gb300 import offq as Q
+    peaks = load_peaks()
+    out = {"what": "offq_quantize_act alone on the prefill layer inputs of the Llama-3-8B MLP and Llama-2-70B "
+                   "shapes (bf16 in; offsets on; the block Hadamard on the down-proj inputs); per-call events, "
+                   "L2 flushed before each call", "sites": []}
+    best = None
+    reps = max(1, min(args.steps, 20))
+    for wname in ("llama3_8b_mlp", "llama2_70b"):
+        w = workload_by_name(wname)
+        T = w.T
+        shapes = set()
+        for i, (name, K, rotate, _) in enumerate(sites(w)):
+            if (K, rotate) in shapes:
+                continue  # a site of the same shape was timed already
+            shapes.add((K, rotate))
+            g = W.block_for(K)
+            x = device_activations(T, K, w, seed=1000 + i, device=device)
+            codes = torch.empty((Q.padded_rows(T), K // 2), dtype=torch.uint8, device=device)
+            scale = torch.empty((T,), dtype=torch.float32, device=device)
+            off = torch.empty((T, K // g), dtype=torch.float32, device=device)
+            flags = (Q.OFFQ_ROTATE if rotate else 0) | Q.OFFQ_OFFSET
+            ts = []
+            for r in range(2 + reps):
+                flush_l2()
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                Q.offq_quantize_act(x, T, K, x.stride(0), g, flags, codes, scale, off, stream)
+                e1.record(stream)
+                torch.cuda.synchronize(device)
+                if r >= 2:
+                    ts.append(e0.elapsed_time(e1))
+            ms = sum(ts) / len(ts)
+            nbytes = T * K * 2 + T * K // 2 + 4 * T + 4 * T * (K // g)
+            gbs = nbytes / (ms * 1e-3) / 1e9
+            site = {"workload": wname, "site": name, "T": T, "K": K, "g": g, "rotate": bool(rotate),
+                    "us": round(ms * 1e3, 2), "bytes": nbytes, "gbs": round(gbs, 1),
+                    "frac": round(gbs / peaks["hbm_gbs"], 4)}
+            out["sites"].append(site)
+            if best is None or nbytes > best["bytes"]:
+                best = site
+            del x, codes, scale, off
+    st = Q.offq_get_device_status(stream)
+    if st != Q.OFFQ_OK:
+        raise RuntimeError(f"device status after the quantizer sites: {Q.status_string(st)}")
+    torch.cuda.empty_cache()
+    out["roofline"] = {"bound": "hbm", "kernel": "offq_quantize_act on the largest site "
+                                                 f"({best['workload']} {best['site']}, {best['T']} x {best['K']})",
+                       "achieved": best["gbs"], "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": best["frac"]}
+    return out
+
+
 def _pair_times(events):
     return [events[i].elapsed_time(events[i + 1]) for i in range(0, len(events), 2)]
 
@@ -705,6 +780,8 @@ def run_gpu(args, rank, world, local_rank):
         line["kv4_rotated"] = time_key_rotation(w, T, device, args, flush_l2, stream)
     if not args.no_group:
         line["builder"] = time_builder(device, args, flush_l2, stream)
+    if not args.no_group and world == 1:
+        line["act_quant_prefill"] = time_quant_sites(device, args, flush_l2, stream)
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
     return line
