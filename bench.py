@@ -896,9 +896,26 @@ def main():
     ap.add_argument("--key-rotation-tokens", type=int, default=0,
                     help="time only the key-cache rotation calls, at this many tokens, and print that object "
                          "(a side measurement for profiling, not the bench line)")
+    ap.add_argument("--quant-sites", action="store_true",
+                    help="time only the activation quantizer on the larger prefill inputs and print that object "
+                         "(a side measurement for profiling, not the bench line)")
     args = ap.parse_args()
     if args.warmup < 3:
         raise SystemExit("--warmup must be at least 3")
+    if args.quant_sites:
+        import torch
+        import __graft_entry__ as G
+        G.build()
+        device = torch.device("cuda", 0)
+        torch.cuda.set_device(device)
+        flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
+
+        def flush_l2():
+            flush.zero_()
+            flush[:L2_FLUSH_BYTES // 2].view(torch.int32).amax()
+
+        print(json.dumps(time_quant_sites(device, args, flush_l2, torch.cuda.current_stream(device))), flush=True)
+        return
     if args.key_rotation_tokens > 0:
         import torch
         device = torch.device("cuda", 0)

@@ -61,6 +61,7 @@ struct QuantArgs {
   int tpr;          // threads per row (a power of two <= 32 or a multiple of 32)
   int rows_per_cta;
   int tiled;        // codes in the 32-row tiled operand layout (else row-major)
+  int* status;      // device status word (bounded waits that run out write here)
 };
 
 template <int L>
@@ -564,6 +565,14 @@ struct RawChunk {
       w[4] = b.x; w[5] = b.y; w[6] = b.z; w[7] = b.w;
     }
   }
+  __device__ __forceinline__ void load_smem(const uint8_t* p) {
+    const uint4 a = *reinterpret_cast<const uint4*>(p);
+    w[0] = a.x; w[1] = a.y; w[2] = a.z; w[3] = a.w;
+    if constexpr (kWords == 8) {
+      const uint4 b = *reinterpret_cast<const uint4*>(p + 16);
+      w[4] = b.x; w[5] = b.y; w[6] = b.z; w[7] = b.w;
+    }
+  }
   __device__ __forceinline__ void unpack(float (&v)[8]) const {
     if constexpr (kWords == 8) {
 #pragma unroll
@@ -725,6 +734,159 @@ __global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantAr
   }
 }
 
+// The same rows (no rotation, one offset block g == K) when a row fits a
+// shared-memory slot: a persistent kernel whose warps each own a ring of S row
+// slots. Lane 0 fills the slots with bulk asynchronous copies (cp.async.bulk,
+// completion counted in bytes on the slot's mbarrier) up to S - 1 rows ahead of
+// the row the warp quantizes, so HBM keeps streaming later rows while the
+// warp runs both sweeps of the current one out of shared memory. Rows are
+// dealt to the grid's warps round-robin.
+constexpr int kBulkRingBytes = 192 * 1024;  // ring bytes per CTA at most
+
+__device__ __forceinline__ void bulk_load_row(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "l"(src), "r"(bytes), "r"(bar)
+               : "memory");
+}
+
+template <typename Tin>
+__global__ void __launch_bounds__(256) quantize_rows_bulk_kernel(const QuantArgs a, int S) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  __shared__ int abort_flag;
+  constexpr int kChunkBytes = 8 * static_cast<int>(sizeof(Tin));
+  const int W = static_cast<int>(blockDim.x >> 5);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int K = a.K;
+  const uint32_t rb = static_cast<uint32_t>(K) * static_cast<uint32_t>(sizeof(Tin));  // a multiple of 64
+  const int cpl = K / 256;                                                            // chunks per lane
+  uint8_t* ring = smem + static_cast<size_t>(warp) * S * rb;
+  const uint32_t bar0 = smem_u32(smem + static_cast<size_t>(W) * S * rb) + 8u * static_cast<uint32_t>(warp * S);
+  if (threadIdx.x == 0) abort_flag = 0;
+  if (lane < S) mbar_init(bar0 + 8u * lane, 1);
+  mbar_fence_init();
+  __syncthreads();
+  griddep_wait();
+  griddep_launch_dependents();
+
+  const bool offs = (a.flags & OFFQ_OFFSET) != 0;
+  const int64_t TW = static_cast<int64_t>(gridDim.x) * W;
+  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * W + warp;
+  const Tin* x = static_cast<const Tin*>(a.x);
+  auto row_src = [&](int64_t r) {
+    const int64_t t = r / a.H;
+    return x + t * a.ld_t + (r - t * a.H) * a.ld_h;
+  };
+
+  // Prologue: the first S rows of this warp in flight.
+  int64_t issued = 0;
+  for (int s = 0; s < S; ++s) {
+    const int64_t r = r0 + s * TW;
+    if (r >= a.rows) break;
+    if (lane == 0) {
+      mbar_arrive_expect_tx(bar0 + 8u * s, rb);
+      bulk_load_row(smem_u32(ring + static_cast<size_t>(s) * rb), row_src(r), rb, bar0 + 8u * s);
+    }
+    ++issued;
+  }
+
+  const int cpr = K / 32;  // 16-byte code chunks per row
+  int slot = 0;
+  uint32_t phase = 0;
+  int64_t done = 0;
+  bool ok = true;
+  for (int64_t r = r0; r < a.rows; r += TW) {
+    const uint32_t bar = bar0 + 8u * slot;
+    if (!mbar_wait(bar, phase, &abort_flag)) {
+      ok = false;
+      break;
+    }
+    const uint8_t* rowp = ring + static_cast<size_t>(slot) * rb;
+
+    // Sweep 1: packed min / max of the raw values and the fp32 row sum.
+    RowMinMax<Tin> mm;
+    float s0 = 0.f, s1 = 0.f;
+#pragma unroll 4
+    for (int j = 0; j < cpl; ++j) {
+      RawChunk<Tin> c;
+      c.load_smem(rowp + (lane + 32 * j) * kChunkBytes);
+#pragma unroll
+      for (int e = 0; e < RawChunk<Tin>::kWords; ++e) mm.add_word(c.w[e]);
+      float v[8];
+      c.unpack(v);
+      add2(v[0], v[1], v[2], v[3]);
+      add2(v[4], v[5], v[6], v[7]);
+      add2(v[0], v[1], v[4], v[5]);
+      add2(s0, s1, v[0], v[1]);
+    }
+    float sum = s0 + s1, mn, mx;
+    mm.result(mn, mx);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+      mn = fminf(mn, __shfl_xor_sync(0xFFFFFFFFu, mn, o));
+      mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, o));
+    }
+    const float off = offs ? sum * (1.0f / static_cast<float>(K)) : 0.f;  // K is a power of two
+    const float m = fmaxf(fmaxf(mx - off, off - mn), 0.f);
+    const float inv = m > 0.f ? __fdiv_rn(7.0f, m) : 0.f;
+
+    // Sweep 2: codes, one 4-byte word per 8-channel chunk.
+    uint8_t* tile_row = a.tiled ? a.codes + (r >> 5) * cpr * 512 + (r & 31) * 16 : a.codes + r * (K / 2);
+#pragma unroll 4
+    for (int j = 0; j < cpl; ++j) {
+      const int c = lane + 32 * j;
+      RawChunk<Tin> ch;
+      ch.load_smem(rowp + c * kChunkBytes);
+      float v[8];
+      ch.unpack(v);
+#pragma unroll
+      for (int e = 0; e < 8; e += 2) {
+        sub2(v[e], v[e + 1], off);
+        fma2(v[e], v[e + 1], inv, kMagic8);
+      }
+      const uint32_t w = pack_codes8(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]),
+                                     __float_as_uint(v[3]), __float_as_uint(v[4]), __float_as_uint(v[5]),
+                                     __float_as_uint(v[6]), __float_as_uint(v[7]));
+      const int bo = 4 * c;  // byte of the row-major row
+      uint8_t* dst = a.tiled ? tile_row + (bo >> 4) * 512 + (bo & 15) : tile_row + bo;
+      *reinterpret_cast<uint32_t*>(dst) = w;
+    }
+    if (lane == 0) {
+      a.scale[r] = m * a.scale_mul;
+      if (a.offset != nullptr) a.offset[r] = off;
+    }
+    ++done;
+
+    // Every lane has read the slot: refill it with the row S turns ahead.
+    __syncwarp();
+    const int64_t rn = r + S * TW;
+    if (rn < a.rows) {
+      if (lane == 0) {
+        mbar_arrive_expect_tx(bar, rb);
+        bulk_load_row(smem_u32(ring + static_cast<size_t>(slot) * rb), row_src(rn), rb, bar);
+      }
+      ++issued;
+    }
+    if (++slot == S) {
+      slot = 0;
+      phase ^= 1u;
+    }
+  }
+  if (!ok && lane == 0) {
+    // A wait ran out: let this warp's copies still in flight land (bounded),
+    // then report the timeout.
+    for (int64_t j = done; j < issued; ++j) {
+      const uint32_t b = bar0 + 8u * static_cast<uint32_t>(j % S);
+      const uint32_t p = static_cast<uint32_t>((j / S) & 1);
+      const long long t0 = clock64();
+      while (!mbar_try_wait(b, p) && clock64() - t0 < kWaitCycles) {
+      }
+    }
+    if (a.status != nullptr) atomicExch(a.status, kErrTimeout);
+  }
+}
+
 // Asks for the largest shared-memory carveout for a kernel, once per device,
 // so that the CTAs' shared memory does not cap residency below the register
 // limit.
@@ -808,9 +970,52 @@ int launch_stream(const QuantArgs& a, cudaStream_t stream) {
   return launch_pdl(quantize_rows_stream_kernel<Tin, CB>, dim3(static_cast<unsigned>(grid)), dim3(256), 0, stream, a);
 }
 
+// Streaming multiprocessors of the current device (queried once per device).
+int sm_count() {
+  static int cache[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (dev < 64 && cache[dev] > 0) return cache[dev];
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  if (dev < 64) cache[dev] = n;
+  return n;
+}
+
+constexpr int kNoFit = 1;  // launch_bulk: the row does not fit the ring; use the register kernel
+
+// The ring geometry: the most warps (8 down to 4) whose rings of 2 to 4 row
+// slots fit kBulkRingBytes.
+template <typename Tin>
+int launch_bulk(const QuantArgs& a, cudaStream_t stream) {
+  if (a.H != 1) return kNoFit;
+  const int64_t rb = static_cast<int64_t>(a.K) * static_cast<int64_t>(sizeof(Tin));
+  int W = 8, S = 0;
+  for (; W >= 4; --W) {
+    S = static_cast<int>(std::min<int64_t>(4, kBulkRingBytes / (W * rb)));
+    if (S >= 2) break;
+  }
+  if (S < 2) return kNoFit;
+  const size_t smem = static_cast<size_t>(W) * S * rb + static_cast<size_t>(W) * S * 8;
+  auto kern = quantize_rows_bulk_kernel<Tin>;
+  if (smem > 48 * 1024 &&
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) != cudaSuccess)
+    return OFFQ_ERR_CUDA;
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, W * 32, smem) != cudaSuccess || per_sm < 1)
+    return OFFQ_ERR_CUDA;
+  const int sms = sm_count();
+  if (sms <= 0) return OFFQ_ERR_CUDA;
+  const int64_t grid = std::min<int64_t>((a.rows + W - 1) / W, static_cast<int64_t>(sms) * per_sm);
+  return launch_pdl(kern, dim3(static_cast<unsigned>(grid)), dim3(W * 32), smem, stream, a, S);
+}
+
 template <typename Tin>
 int dispatch_g(const QuantArgs& a, int g, cudaStream_t s) {
-  if ((a.flags & OFFQ_ROTATE) == 0 && a.G == 1 && g >= 1024) return launch_stream<Tin>(a, s);
+  if ((a.flags & OFFQ_ROTATE) == 0 && a.G == 1 && g >= 1024) {
+    const int st = launch_bulk<Tin>(a, s);
+    return st == kNoFit ? launch_stream<Tin>(a, s) : st;
+  }
   switch (g) {
     case 32: return launch_narrow<5, Tin>(a, s);
     case 64: return launch_narrow<6, Tin>(a, s);
@@ -829,6 +1034,7 @@ int run_quant(QuantArgs a, int dtype, int g, cudaStream_t s) {
   const double isg = (a.flags & OFFQ_ROTATE) ? 1.0 / std::sqrt(static_cast<double>(g)) : 1.0;
   a.inv_sqrt_g = static_cast<float>(isg);
   a.scale_mul = static_cast<float>(isg / 7.0);
+  a.status = device_status_ptr();
   switch (dtype) {
     case OFFQ_BF16: return dispatch_g<__nv_bfloat16>(a, g, s);
     case OFFQ_F16: return dispatch_g<__half>(a, g, s);

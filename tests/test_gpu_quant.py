@@ -81,13 +81,25 @@ def test_quantize_workload_shapes(T, K, g, dist):
     _quant_and_check(_host(x, "bf16"), g, True, True)
 
 
-@pytest.mark.parametrize("K,dt", [(1024, "bf16"), (4096, "bf16"), (4096, "f16"), (4096, "f32"), (8192, "bf16")])
+@pytest.mark.parametrize("K,dt", [(1024, "bf16"), (4096, "bf16"), (4096, "f16"), (4096, "f32"), (8192, "bf16"),
+                                  (8192, "f32")])
 @pytest.mark.parametrize("offset", [True, False])
 def test_quantize_whole_row_block_without_rotation(K, dt, offset):
-    """One offset block per row and no rotation (the q/k/v, o and gate/up sites); 45 rows leave a
-    ragged last CTA, and K = 8192 bf16 / 4096 fp32 rows take the two-sweep path."""
+    """One offset block per row and no rotation (the q/k/v, o and gate/up sites); 45 rows leave
+    warps without a row. Rows up to 24 KB take the shared-memory ring kernel; K = 8192 fp32 rows
+    take the register kernel's two-sweep path."""
     x = W.activations(45, K, seed=31 + K, n_out=4, mult=100.0)
     _quant_and_check(_host(x, dt), K, False, offset)
+
+
+@pytest.mark.parametrize("T,K,dt", [(40000, 1024, "bf16"), (5003, 8192, "bf16"), (4099, 4096, "f32")])
+def test_quantize_whole_row_many_rows_per_warp(T, K, dt):
+    """Enough rows that every warp of the persistent ring kernel quantizes several, so each slot
+    is refilled and its barrier phase flips more than once; checked on sampled rows including
+    the first and the last."""
+    x = W.activations(T, K, seed=57 + K, n_out=4, mult=100.0)
+    rows = np.unique(np.concatenate([W.unit_index_sample(T, 384, seed=5), [0, 1, T - 2, T - 1]]))
+    _quant_and_check(_host(x, dt), K, False, True, rows=rows)
 
 
 def test_quantize_toy_fp32():
