@@ -243,6 +243,69 @@ __device__ __forceinline__ float tree_sum(const float* v) {
   }
 }
 
+// ---------------------------------------------------------------------------
+// Row rings of the persistent kernels: shared-memory slots filled by bulk
+// asynchronous copies (cp.async.bulk) whose bytes complete on an mbarrier.
+// ---------------------------------------------------------------------------
+constexpr size_t kMaxDynSmem = 226 * 1024;  // dynamic bytes; the static flag needs a few more
+
+__device__ __forceinline__ void bulk_load_row(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "l"(src), "r"(bytes), "r"(bar)
+               : "memory");
+}
+
+// Rows [grp*R, grp*R + R) of a one-head input (those below a.rows) into the
+// slot, row l at byte l * K * sizeof(Tin); one copy when the rows are
+// contiguous. Called by one thread.
+template <typename Tin>
+__device__ __forceinline__ void ring_issue(const QuantArgs& a, int64_t grp, int R, uint8_t* slot, uint32_t bar) {
+  const int64_t r0 = grp * R;
+  const int n = static_cast<int>(a.rows - r0 < R ? a.rows - r0 : R);
+  const uint32_t rb = static_cast<uint32_t>(a.K) * static_cast<uint32_t>(sizeof(Tin));
+  const Tin* x = static_cast<const Tin*>(a.x);
+  mbar_arrive_expect_tx(bar, static_cast<uint32_t>(n) * rb);
+  if (a.ld_t == a.K) {
+    bulk_load_row(smem_u32(slot), x + r0 * a.K, static_cast<uint32_t>(n) * rb, bar);
+  } else {
+    for (int l = 0; l < n; ++l) bulk_load_row(smem_u32(slot + static_cast<size_t>(l) * rb), x + (r0 + l) * a.ld_t, rb, bar);
+  }
+}
+
+// A slot wait ran out somewhere in the CTA: thread 0 lets the copy land
+// (bounded) and reports the timeout.
+__device__ __forceinline__ void ring_fail(uint32_t bar, uint32_t parity, int* status) {
+  if (threadIdx.x != 0) return;
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity) && clock64() - t0 < kWaitCycles) {
+  }
+  if (status != nullptr) atomicExch(status, kErrTimeout);
+}
+
+// One 8-element chunk of a staged row (shared memory) as fp32.
+__device__ __forceinline__ void load_chunk8_smem(const __nv_bfloat16* p, float* v) {
+  const uint4 w = *reinterpret_cast<const uint4*>(p);
+  bf16x2_to_f32(w.x, v[0], v[1]);
+  bf16x2_to_f32(w.y, v[2], v[3]);
+  bf16x2_to_f32(w.z, v[4], v[5]);
+  bf16x2_to_f32(w.w, v[6], v[7]);
+}
+
+__device__ __forceinline__ void load_chunk8_smem(const __half* p, float* v) {
+  const uint4 w = *reinterpret_cast<const uint4*>(p);
+  f16x2_to_f32(w.x, v[0], v[1]);
+  f16x2_to_f32(w.y, v[2], v[3]);
+  f16x2_to_f32(w.z, v[4], v[5]);
+  f16x2_to_f32(w.w, v[6], v[7]);
+}
+
+__device__ __forceinline__ void load_chunk8_smem(const float* p, float* v) {
+  const float4 a = *reinterpret_cast<const float4*>(p);
+  const float4 b = *reinterpret_cast<const float4*>(p + 4);
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+  v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+
 // Geometry of quantize_rows_kernel (g = 2^L <= 512). E >= 2^(3+P) puts a
 // thread's in-block position (pass-1 index bits 3..3+P-1) below the bits it
 // holds in registers, so a pass-2 thread owns E contiguous channels.
@@ -272,41 +335,83 @@ __device__ __forceinline__ int swz_narrow(int idx) {
   }
 }
 
-template <int L, typename Tin>
+// kRing: persistent form for one-head inputs. The CTA's rows_per_cta rows of
+// group grp (rows grp*R ..) are staged in a shared-memory slot by bulk copies;
+// once pass 1 has read them, the copy of the CTA's next group is issued, so
+// its HBM reads overlap this group's arithmetic.
+template <int L, typename Tin, bool kRing>
 __global__ void __launch_bounds__(NarrowGeo<L>::kMaxThreads) quantize_rows_kernel(const QuantArgs a) {
   using GG = NarrowGeo<L>;
   constexpr int E = GG::kE, P = GG::kP, TPB = GG::kTPB, NC = GG::kNC, LOGE = GG::kLogE;
   constexpr int g = 1 << L;
-  griddep_wait();
-  griddep_launch_dependents();
 
   extern __shared__ __align__(16) uint8_t smem[];
+  __shared__ int abort_flag;
   float* red = reinterpret_cast<float*>(smem);          // 32 floats for group_reduce
   float* buf = reinterpret_cast<float*>(smem + 128);    // [rows_per_cta][K] fp32 transpose
   const bool rotate = (a.flags & OFFQ_ROTATE) != 0;
   const bool offs = (a.flags & OFFQ_OFFSET) != 0;
   const int K = a.K;
+  const int R = a.rows_per_cta;
+  uint8_t* slot = smem + 128 + static_cast<size_t>(R) * K * 4;  // kRing: [R][K] inputs
+  const uint32_t bar = smem_u32(slot + static_cast<size_t>(R) * K * sizeof(Tin));
 
   const int tid = threadIdx.x;
   const int lrow = tid / a.tpr;
   const int j = tid - lrow * a.tpr;
-  const int64_t row = static_cast<int64_t>(blockIdx.x) * a.rows_per_cta + lrow;
-  const bool row_ok = row < a.rows;
-  const bool active = row_ok && (j < a.G * TPB);
   const int b = j >> P;
   const int t = j & (TPB - 1);
+  const int64_t ngroups = (a.rows + R - 1) / R;
+  int64_t grp = blockIdx.x;
+  uint32_t phase = 0;
+  if constexpr (kRing) {
+    if (tid == 0) {
+      abort_flag = 0;
+      mbar_init(bar, 1);
+      mbar_fence_init();
+    }
+    __syncthreads();
+  }
+  griddep_wait();
+  griddep_launch_dependents();
+  if constexpr (kRing) {
+    if (tid == 0 && grp < ngroups) ring_issue<Tin>(a, grp, R, slot, bar);
+  }
+
+  while (true) {
+  const int64_t row = grp * R + lrow;
+  const bool row_ok = row < a.rows;
+  const bool active = row_ok && (j < a.G * TPB);
 
   // Pass 1: register 8i + c holds channel 8t + 8 TPB i + c of block b.
   float v[E];
-  if (active) {
-    const int64_t tok = row / a.H;
-    const int64_t h = row - tok * a.H;
-    const Tin* p = static_cast<const Tin*>(a.x) + tok * a.ld_t + h * a.ld_h + static_cast<int64_t>(b) * g + 8 * t;
+  if constexpr (kRing) {
+    const bool ok = mbar_wait(bar, phase, &abort_flag);
+    phase ^= 1u;
+    if (ok && active) {
+      const Tin* p = reinterpret_cast<const Tin*>(slot) + static_cast<size_t>(lrow) * K + b * g + 8 * t;
 #pragma unroll
-    for (int i = 0; i < NC; ++i) load_chunk8(p + i * 8 * TPB, &v[8 * i]);
+      for (int i = 0; i < NC; ++i) load_chunk8_smem(p + i * 8 * TPB, &v[8 * i]);
+    } else {
+#pragma unroll
+      for (int r = 0; r < E; ++r) v[r] = 0.f;
+    }
+    if (!__syncthreads_and(ok)) {
+      ring_fail(bar, phase ^ 1u, a.status);
+      return;
+    }
+    if (tid == 0 && grp + gridDim.x < ngroups) ring_issue<Tin>(a, grp + gridDim.x, R, slot, bar);
   } else {
+    if (active) {
+      const int64_t tok = row / a.H;
+      const int64_t h = row - tok * a.H;
+      const Tin* p = static_cast<const Tin*>(a.x) + tok * a.ld_t + h * a.ld_h + static_cast<int64_t>(b) * g + 8 * t;
 #pragma unroll
-    for (int r = 0; r < E; ++r) v[r] = 0.f;
+      for (int i = 0; i < NC; ++i) load_chunk8(p + i * 8 * TPB, &v[8 * i]);
+    } else {
+#pragma unroll
+      for (int r = 0; r < E; ++r) v[r] = 0.f;
+    }
   }
 
   float off = 0.f;
@@ -398,17 +503,22 @@ __global__ void __launch_bounds__(NarrowGeo<L>::kMaxThreads) quantize_rows_kerne
   if (active && t == 0 && a.offset != nullptr) {
     a.offset[row * a.G + b] = offs ? (rotate ? off * a.inv_sqrt_g : off) : 0.f;
   }
+  if constexpr (!kRing) break;
+  grp += gridDim.x;
+  if (grp >= ngroups) break;
+  }
 }
 
-template <int L, typename Tin>
+// kRing: persistent form for one-head inputs, as in quantize_rows_kernel (the
+// slot follows the reduction scratch in shared memory).
+template <int L, typename Tin, bool kRing>
 __global__ void __launch_bounds__(WideGeo<L>::kMaxThreads) quantize_rows_wide_kernel(const QuantArgs a) {
   using GG = WideGeo<L>;
   constexpr int E = GG::kE, P = GG::kP, TPB = GG::kTPB, Q = GG::kQ, NC = GG::kNC, LOGE = GG::kLogE;
   constexpr int g = 1 << L;
-  griddep_wait();
-  griddep_launch_dependents();
 
   extern __shared__ __align__(16) uint8_t smem[];
+  __shared__ int abort_flag;
   const bool rotate = (a.flags & OFFQ_ROTATE) != 0;
   const bool offs = (a.flags & OFFQ_OFFSET) != 0;
   const int R = a.rows_per_cta;
@@ -416,26 +526,64 @@ __global__ void __launch_bounds__(WideGeo<L>::kMaxThreads) quantize_rows_wide_ke
   float* buf = reinterpret_cast<float*>(smem);                                  // [R][K] fp32 (rotate)
   uint8_t* cbuf = smem + (rotate ? static_cast<size_t>(R) * K * 4 : 0);         // [R][K/2] codes
   float* red = reinterpret_cast<float*>(cbuf + static_cast<size_t>(R) * (K / 2));
+  uint8_t* slot = reinterpret_cast<uint8_t*>(red + 32);                         // kRing: [R][K] inputs
+  const uint32_t bar = smem_u32(slot + static_cast<size_t>(R) * K * sizeof(Tin));
 
   const int tid = threadIdx.x;
   const int lrow = tid / a.tpr;
   const int j = tid - lrow * a.tpr;
-  const int64_t row = static_cast<int64_t>(blockIdx.x) * R + lrow;
-  const bool row_ok = row < a.rows;
-  const bool active = row_ok && (j < a.G * TPB);
   const int b = j / TPB;
   const int t1 = j % TPB;
+  const int64_t ngroups = (a.rows + R - 1) / R;
+  int64_t grp = blockIdx.x;
+  uint32_t phase = 0;
+  if constexpr (kRing) {
+    if (tid == 0) {
+      abort_flag = 0;
+      mbar_init(bar, 1);
+      mbar_fence_init();
+    }
+    __syncthreads();
+  }
+  griddep_wait();
+  griddep_launch_dependents();
+  if constexpr (kRing) {
+    if (tid == 0 && grp < ngroups) ring_issue<Tin>(a, grp, R, slot, bar);
+  }
+
+  while (true) {
+  const int64_t row = grp * R + lrow;
+  const bool row_ok = row < a.rows;
+  const bool active = row_ok && (j < a.G * TPB);
 
   float v[E];
-  if (active) {
-    const int64_t t = row / a.H;
-    const int64_t h = row - t * a.H;
-    const Tin* p = static_cast<const Tin*>(a.x) + t * a.ld_t + h * a.ld_h + static_cast<int64_t>(b) * g + 8 * t1;
+  if constexpr (kRing) {
+    const bool ok = mbar_wait(bar, phase, &abort_flag);
+    phase ^= 1u;
+    if (ok && active) {
+      const Tin* p = reinterpret_cast<const Tin*>(slot) + static_cast<size_t>(lrow) * K + b * g + 8 * t1;
 #pragma unroll
-    for (int i = 0; i < NC; ++i) load_chunk8(p + i * 8 * TPB, &v[8 * i]);
+      for (int i = 0; i < NC; ++i) load_chunk8_smem(p + i * 8 * TPB, &v[8 * i]);
+    } else {
+#pragma unroll
+      for (int r = 0; r < E; ++r) v[r] = 0.f;
+    }
+    if (!__syncthreads_and(ok)) {
+      ring_fail(bar, phase ^ 1u, a.status);
+      return;
+    }
+    if (tid == 0 && grp + gridDim.x < ngroups) ring_issue<Tin>(a, grp + gridDim.x, R, slot, bar);
   } else {
+    if (active) {
+      const int64_t t = row / a.H;
+      const int64_t h = row - t * a.H;
+      const Tin* p = static_cast<const Tin*>(a.x) + t * a.ld_t + h * a.ld_h + static_cast<int64_t>(b) * g + 8 * t1;
 #pragma unroll
-    for (int r = 0; r < E; ++r) v[r] = 0.f;
+      for (int i = 0; i < NC; ++i) load_chunk8(p + i * 8 * TPB, &v[8 * i]);
+    } else {
+#pragma unroll
+      for (int r = 0; r < E; ++r) v[r] = 0.f;
+    }
   }
 
   float off = 0.f;
@@ -445,7 +593,15 @@ __global__ void __launch_bounds__(WideGeo<L>::kMaxThreads) quantize_rows_wide_ke
       off = v[0];
       v[0] = 0.f;
     }
-    fwht_bits<E, 0, LOGE>(v);  // index bits {0,1,2} and {3+P, .., L-1}
+    // Index bits {0,1,2} and {3+P, .., L-1}: bit 0 on scalar adds, the others
+    // packed on the (even, odd) register pairs the loads produced.
+#pragma unroll
+    for (int r = 0; r < E; r += 2) {
+      const float x0 = v[r], x1 = v[r + 1];
+      v[r] = x0 + x1;
+      v[r + 1] = x0 - x1;
+    }
+    fwht_reg_stages<E, 1, LOGE>(v);
     float* rb = buf + static_cast<size_t>(lrow) * K + static_cast<size_t>(b) * g;
     if (active) {
 #pragma unroll
@@ -502,14 +658,14 @@ __global__ void __launch_bounds__(WideGeo<L>::kMaxThreads) quantize_rows_wide_ke
 #pragma unroll
       for (int hi = 0; hi < (1 << P); ++hi) {
         const int e = ((t1 & ((1 << (3 - Q)) - 1)) << Q) | (hi << 3) | ((t1 >> (3 - Q)) << (3 + P));
+        // Bits 4-21 of a rounded value are zero, so (u1 << 4) + u0 carries the
+        // byte of two codes in its low 8 bits.
         if constexpr (Q == 2) {
-          const uint32_t u0 = __float_as_uint(v[4 * hi]) & 0xFu, u1 = __float_as_uint(v[4 * hi + 1]) & 0xFu;
-          const uint32_t u2 = __float_as_uint(v[4 * hi + 2]) & 0xFu, u3 = __float_as_uint(v[4 * hi + 3]) & 0xFu;
-          *reinterpret_cast<uint16_t*>(crow + e / 2) =
-              static_cast<uint16_t>(u0 | (u1 << 4) | (u2 << 8) | (u3 << 12));
+          const uint32_t b0 = (__float_as_uint(v[4 * hi + 1]) << 4) + __float_as_uint(v[4 * hi]);
+          const uint32_t b1 = (__float_as_uint(v[4 * hi + 3]) << 4) + __float_as_uint(v[4 * hi + 2]);
+          *reinterpret_cast<uint16_t*>(crow + e / 2) = static_cast<uint16_t>(__byte_perm(b0, b1, 0x0040));
         } else {
-          const uint32_t u0 = __float_as_uint(v[2 * hi]) & 0xFu, u1 = __float_as_uint(v[2 * hi + 1]) & 0xFu;
-          crow[e / 2] = static_cast<uint8_t>(u0 | (u1 << 4));
+          crow[e / 2] = static_cast<uint8_t>((__float_as_uint(v[2 * hi + 1]) << 4) + __float_as_uint(v[2 * hi]));
         }
       }
     } else {
@@ -543,6 +699,10 @@ __global__ void __launch_bounds__(WideGeo<L>::kMaxThreads) quantize_rows_wide_ke
   if (row_ok && j == 0) a.scale[row] = m * a.scale_mul;
   if (active && t1 == 0 && a.offset != nullptr) {
     a.offset[row * a.G + b] = offs ? (rotate ? off * a.inv_sqrt_g : off) : 0.f;
+  }
+  if constexpr (!kRing) break;
+  grp += gridDim.x;
+  if (grp >= ngroups) break;
   }
 }
 
@@ -743,12 +903,6 @@ __global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantAr
 // dealt to the grid's warps round-robin.
 constexpr int kBulkRingBytes = 192 * 1024;  // ring bytes per CTA at most
 
-__device__ __forceinline__ void bulk_load_row(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
-  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
-               "l"(src), "r"(bytes), "r"(bar)
-               : "memory");
-}
-
 template <typename Tin>
 __global__ void __launch_bounds__(256) quantize_rows_bulk_kernel(const QuantArgs a, int S) {
   extern __shared__ __align__(128) uint8_t smem[];
@@ -903,6 +1057,40 @@ int prefer_max_shared(F* kern) {
   return OFFQ_OK;
 }
 
+// Streaming multiprocessors of the current device (queried once per device).
+int sm_count() {
+  static int cache[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (dev < 64 && cache[dev] > 0) return cache[dev];
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  if (dev < 64) cache[dev] = n;
+  return n;
+}
+
+constexpr int kNoRing = 1;  // launch_ring: use the one-shot kernel instead
+
+// Launches the persistent (ring) form of a row kernel when the input has one
+// head, there are more row groups than SMs, and the slot fits: one CTA per
+// resident slot, each looping over the groups grid-stride.
+template <typename F>
+int launch_ring(F* kern, const QuantArgs& a, int threads, size_t smem, cudaStream_t stream) {
+  if (a.H != 1 || smem > kMaxDynSmem) return kNoRing;
+  const int sms = sm_count();
+  const int64_t groups = (a.rows + a.rows_per_cta - 1) / a.rows_per_cta;
+  if (sms <= 0 || groups <= sms) return kNoRing;
+  if (prefer_max_shared(kern) != OFFQ_OK) return OFFQ_ERR_CUDA;
+  if (smem > 48 * 1024 &&
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) != cudaSuccess)
+    return OFFQ_ERR_CUDA;
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem) != cudaSuccess) return OFFQ_ERR_CUDA;
+  if (per_sm < 1) return kNoRing;
+  const int64_t grid = std::min<int64_t>(groups, static_cast<int64_t>(sms) * per_sm);
+  return launch_pdl(kern, dim3(static_cast<unsigned>(grid)), dim3(threads), smem, stream, a);
+}
+
 template <int L, typename Tin>
 int launch_narrow(QuantArgs a, cudaStream_t stream) {
   using GG = NarrowGeo<L>;
@@ -920,7 +1108,10 @@ int launch_narrow(QuantArgs a, cudaStream_t stream) {
   a.tpr = tpr;
   a.rows_per_cta = R;
   const size_t smem = 128 + static_cast<size_t>(R) * row_smem;
-  auto kern = quantize_rows_kernel<L, Tin>;
+  const int rs = launch_ring(quantize_rows_kernel<L, Tin, true>, a, R * tpr,
+                             smem + static_cast<size_t>(R) * a.K * sizeof(Tin) + 8, stream);
+  if (rs != kNoRing) return rs;
+  auto kern = quantize_rows_kernel<L, Tin, false>;
   if (prefer_max_shared(kern) != OFFQ_OK) return OFFQ_ERR_CUDA;
   if (smem > 48 * 1024) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
@@ -950,7 +1141,10 @@ int launch_wide(QuantArgs a, cudaStream_t stream) {
   a.tpr = tpr;
   a.rows_per_cta = R;
   const size_t smem = static_cast<size_t>(R) * row_smem + 32 * sizeof(float);
-  auto kern = quantize_rows_wide_kernel<L, Tin>;
+  const int rs = launch_ring(quantize_rows_wide_kernel<L, Tin, true>, a, R * tpr,
+                             smem + static_cast<size_t>(R) * a.K * sizeof(Tin) + 8, stream);
+  if (rs != kNoRing) return rs;
+  auto kern = quantize_rows_wide_kernel<L, Tin, false>;
   if (smem > 48 * 1024) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
         cudaSuccess)
@@ -968,18 +1162,6 @@ int launch_stream(const QuantArgs& a, cudaStream_t stream) {
   // Up to 16 chunks (64 registers of bf16) per lane stay resident.
   constexpr int CB = sizeof(Tin) == 4 ? 8 : 16;
   return launch_pdl(quantize_rows_stream_kernel<Tin, CB>, dim3(static_cast<unsigned>(grid)), dim3(256), 0, stream, a);
-}
-
-// Streaming multiprocessors of the current device (queried once per device).
-int sm_count() {
-  static int cache[64] = {};
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-  if (dev < 64 && cache[dev] > 0) return cache[dev];
-  int n = 0;
-  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-  if (dev < 64) cache[dev] = n;
-  return n;
 }
 
 constexpr int kNoFit = 1;  // launch_bulk: the row does not fit the ring; use the register kernel

@@ -102,6 +102,29 @@ def test_quantize_whole_row_many_rows_per_warp(T, K, dt):
     _quant_and_check(_host(x, dt), K, False, True, rows=rows)
 
 
+@pytest.mark.parametrize("g", [32, 64, 128, 256, 512, 1024, 2048, 4096, 8192])
+@pytest.mark.parametrize("G", [1, 3])
+def test_quantize_persistent_ring(g, G):
+    """Enough rows (about 2^24 channels) that the row groups outnumber the SMs, so the
+    persistent form stages each CTA's groups through its shared-memory slot; sampled rows,
+    including the first and the last, against the oracle."""
+    K = g * G
+    T = max(700, 2 ** 24 // K)
+    x = W.activations(T, K, seed=300 + g + G, n_out=3, mult=80.0)
+    rows = np.unique(np.concatenate([W.unit_index_sample(T, 160, seed=9), [0, 1, T - 2, T - 1]]))
+    _quant_and_check(_host(x, "bf16"), g, True, True, rows=rows)
+
+
+@pytest.mark.parametrize("dt,ld_pad", [("f32", 0), ("bf16", 64), ("f16", 0)])
+def test_quantize_persistent_ring_dtypes_and_stride(dt, ld_pad):
+    """The persistent form on the down-proj shape (43 blocks of 256) with fp32 / fp16 rows, and
+    with padded rows that take one bulk copy per row."""
+    T, K, g = 1600, 11008, 256
+    x = W.activations(T, K, seed=41, n_out=4, mult=100.0)
+    rows = np.unique(np.concatenate([W.unit_index_sample(T, 160, seed=10), [0, T - 1]]))
+    _quant_and_check(_host(x, dt), g, True, True, rows=rows, ldx=(K + ld_pad) if ld_pad else None)
+
+
 def test_quantize_toy_fp32():
     w = W.WORKLOADS["toy"]
     x = W.layer_inputs(w, w.layers[0])
