@@ -62,6 +62,7 @@ struct QuantArgs {
   int rows_per_cta;
   int tiled;        // codes in the 32-row tiled operand layout (else row-major)
   int* status;      // device status word (bounded waits that run out write here)
+  int ring_slots;   // persistent forms: slots of rows_per_cta rows each (1 to 3)
 };
 
 template <int L>
@@ -272,12 +273,48 @@ __device__ __forceinline__ void ring_issue(const QuantArgs& a, int64_t grp, int 
   }
 }
 
-// A slot wait ran out somewhere in the CTA: thread 0 lets the copy land
-// (bounded) and reports the timeout.
-__device__ __forceinline__ void ring_fail(uint32_t bar, uint32_t parity, int* status) {
+// The ring of a persistent row kernel: S slots of R rows, slot k at
+// base + k * slot_bytes with its mbarrier at bar0 + 8 k. The CTA's i-th group
+// (blockIdx.x + i * gridDim.x) lands in slot i mod S; s and phase name the slot
+// of the group being consumed and the parity of its completion.
+struct RowRing {
+  uint8_t* base;
+  uint32_t bar0;
+  uint32_t slot_bytes;
+  int S;
+  int s;
+  uint32_t phase;
+  __device__ __forceinline__ uint8_t* slot() const { return base + static_cast<size_t>(s) * slot_bytes; }
+  __device__ __forceinline__ uint32_t bar() const { return bar0 + 8u * static_cast<uint32_t>(s); }
+  __device__ __forceinline__ void advance() {
+    if (++s == S) {
+      s = 0;
+      phase ^= 1u;
+    }
+  }
+};
+
+// Thread 0 initialises the slots' barriers and issues the CTA's first S groups.
+template <typename Tin>
+__device__ __forceinline__ void ring_start(const QuantArgs& a, const RowRing& ring, int R, int64_t ngroups) {
   if (threadIdx.x != 0) return;
-  const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity) && clock64() - t0 < kWaitCycles) {
+  for (int k = 0; k < ring.S; ++k) {
+    const int64_t grp = blockIdx.x + static_cast<int64_t>(k) * gridDim.x;
+    if (grp < ngroups) ring_issue<Tin>(a, grp, R, ring.base + static_cast<size_t>(k) * ring.slot_bytes, ring.bar0 + 8u * k);
+  }
+}
+
+// A slot wait ran out somewhere in the CTA while consuming group grp: thread 0
+// lets every copy still in flight land (bounded waits) and reports the timeout.
+__device__ __forceinline__ void ring_fail(const RowRing& ring, int64_t grp, int64_t ngroups, int* status) {
+  if (threadIdx.x != 0) return;
+  for (int d = 0; d < ring.S; ++d) {
+    if (grp + static_cast<int64_t>(d) * gridDim.x >= ngroups) break;
+    const int k = (ring.s + d) % ring.S;
+    const uint32_t parity = ring.s + d < ring.S ? ring.phase : (ring.phase ^ 1u);
+    const long long t0 = clock64();
+    while (!mbar_try_wait(ring.bar0 + 8u * k, parity) && clock64() - t0 < kWaitCycles) {
+    }
   }
   if (status != nullptr) atomicExch(status, kErrTimeout);
 }
@@ -316,7 +353,9 @@ struct NarrowGeo {
   static constexpr int kP = L - kLogE;        // log2 threads per block
   static constexpr int kTPB = 1 << kP;
   static constexpr int kNC = kE / 8;          // 8-channel loads per thread
-  static constexpr int kMaxThreads = 512;     // 128 blocks of g = 256 or 64 of g = 512
+  // 128 blocks of g = 256 or 64 of g = 512; 128 registers of data per thread
+  // (g = 1024) need the 255-register limit of 256-thread CTAs.
+  static constexpr int kMaxThreads = kE >= 128 ? 256 : 512;
   static_assert(3 + kP <= kLogE && kP >= 1 && kE >= 16, "narrow geometry");
 };
 
@@ -353,8 +392,14 @@ __global__ void __launch_bounds__(NarrowGeo<L>::kMaxThreads) quantize_rows_kerne
   const bool offs = (a.flags & OFFQ_OFFSET) != 0;
   const int K = a.K;
   const int R = a.rows_per_cta;
-  uint8_t* slot = smem + 128 + static_cast<size_t>(R) * K * 4;  // kRing: [R][K] inputs
-  const uint32_t bar = smem_u32(slot + static_cast<size_t>(R) * K * sizeof(Tin));
+  // kRing: ring_slots slots of [R][K] inputs after the transpose buffer, then their barriers.
+  RowRing ring;
+  ring.base = smem + 128 + static_cast<size_t>(R) * K * 4;
+  ring.slot_bytes = static_cast<uint32_t>(R) * K * sizeof(Tin);
+  ring.S = a.ring_slots;
+  ring.bar0 = smem_u32(ring.base + static_cast<size_t>(ring.S) * ring.slot_bytes);
+  ring.s = 0;
+  ring.phase = 0;
 
   const int tid = threadIdx.x;
   const int lrow = tid / a.tpr;
@@ -363,149 +408,148 @@ __global__ void __launch_bounds__(NarrowGeo<L>::kMaxThreads) quantize_rows_kerne
   const int t = j & (TPB - 1);
   const int64_t ngroups = (a.rows + R - 1) / R;
   int64_t grp = blockIdx.x;
-  uint32_t phase = 0;
   if constexpr (kRing) {
     if (tid == 0) {
       abort_flag = 0;
-      mbar_init(bar, 1);
+      for (int k = 0; k < ring.S; ++k) mbar_init(ring.bar0 + 8u * k, 1);
       mbar_fence_init();
     }
     __syncthreads();
   }
   griddep_wait();
   griddep_launch_dependents();
-  if constexpr (kRing) {
-    if (tid == 0 && grp < ngroups) ring_issue<Tin>(a, grp, R, slot, bar);
-  }
+  if constexpr (kRing) ring_start<Tin>(a, ring, R, ngroups);
 
   while (true) {
-  const int64_t row = grp * R + lrow;
-  const bool row_ok = row < a.rows;
-  const bool active = row_ok && (j < a.G * TPB);
+    const int64_t row = grp * R + lrow;
+    const bool row_ok = row < a.rows;
+    const bool active = row_ok && (j < a.G * TPB);
 
-  // Pass 1: register 8i + c holds channel 8t + 8 TPB i + c of block b.
-  float v[E];
-  if constexpr (kRing) {
-    const bool ok = mbar_wait(bar, phase, &abort_flag);
-    phase ^= 1u;
-    if (ok && active) {
-      const Tin* p = reinterpret_cast<const Tin*>(slot) + static_cast<size_t>(lrow) * K + b * g + 8 * t;
+    // Pass 1: register 8i + c holds channel 8t + 8 TPB i + c of block b.
+    float v[E];
+    if constexpr (kRing) {
+      const bool ok = mbar_wait(ring.bar(), ring.phase, &abort_flag);
+      if (ok && active) {
+        const Tin* p = reinterpret_cast<const Tin*>(ring.slot()) + static_cast<size_t>(lrow) * K + b * g + 8 * t;
 #pragma unroll
-      for (int i = 0; i < NC; ++i) load_chunk8_smem(p + i * 8 * TPB, &v[8 * i]);
-    } else {
+        for (int i = 0; i < NC; ++i) load_chunk8_smem(p + i * 8 * TPB, &v[8 * i]);
+      } else {
 #pragma unroll
-      for (int r = 0; r < E; ++r) v[r] = 0.f;
-    }
-    if (!__syncthreads_and(ok)) {
-      ring_fail(bar, phase ^ 1u, a.status);
-      return;
-    }
-    if (tid == 0 && grp + gridDim.x < ngroups) ring_issue<Tin>(a, grp + gridDim.x, R, slot, bar);
-  } else {
-    if (active) {
-      const int64_t tok = row / a.H;
-      const int64_t h = row - tok * a.H;
-      const Tin* p = static_cast<const Tin*>(a.x) + tok * a.ld_t + h * a.ld_h + static_cast<int64_t>(b) * g + 8 * t;
-#pragma unroll
-      for (int i = 0; i < NC; ++i) load_chunk8(p + i * 8 * TPB, &v[8 * i]);
-    } else {
-#pragma unroll
-      for (int r = 0; r < E; ++r) v[r] = 0.f;
-    }
-  }
-
-  float off = 0.f;
-  if (rotate) {
-    // Offset = x[block start] / sqrt(g); removing it first leaves the residual.
-    if (offs && t == 0) {
-      off = v[0];
-      v[0] = 0.f;
-    }
-    fwht_reg_stages<E, 1, LOGE>(v);   // channel bits 1, 2 and 3+P .. L-1
-  } else if (offs) {
-    // Block mean by a pairwise tree (depth log2(E) in the thread, P across threads).
-    off = group_reduce<false>(tree_sum<E>(v), TPB, red) * (1.0f / static_cast<float>(g));
-  }
-
-  const int base = lrow * K + b * g;
-  if (active) {
-#pragma unroll
-    for (int i = 0; i < NC; ++i) {
-      const int e0 = base + 8 * t + 8 * TPB * i;
-      *reinterpret_cast<float4*>(buf + swz_narrow<L, LOGE>(e0)) =
-          make_float4(v[8 * i], v[8 * i + 1], v[8 * i + 2], v[8 * i + 3]);
-      *reinterpret_cast<float4*>(buf + swz_narrow<L, LOGE>(e0 + 4)) =
-          make_float4(v[8 * i + 4], v[8 * i + 5], v[8 * i + 6], v[8 * i + 7]);
-    }
-  }
-  __syncwarp();  // a block's TPB <= 8 threads share one warp
-  // Pass 2: register r holds channel E t + r of block b.
-  if (active) {
-#pragma unroll
-    for (int m = 0; m < E / 4; ++m) {
-      const float4 f = *reinterpret_cast<const float4*>(buf + swz_narrow<L, LOGE>(base + E * t + 4 * m));
-      v[4 * m] = f.x;
-      v[4 * m + 1] = f.y;
-      v[4 * m + 2] = f.z;
-      v[4 * m + 3] = f.w;
-    }
-  }
-  if (rotate) {
-#pragma unroll
-    for (int r = 0; r < E; r += 2) {   // channel bit 0
-      const float x0 = v[r], x1 = v[r + 1];
-      v[r] = x0 + x1;
-      v[r + 1] = x0 - x1;
-    }
-    fwht_reg_stages<E, 3, 3 + P>(v);   // channel bits 3 .. 3+P-1
-  } else if (offs) {
-#pragma unroll
-    for (int r = 0; r < E; r += 2) sub2(v[r], v[r + 1], off);
-  }
-
-  // Per-row absmax of the residual.
-  float mx[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-  for (int r = 0; r < E; ++r) mx[r & 3] = fmaxf(mx[r & 3], fabsf(v[r]));
-  float m = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
-  m = group_reduce<true>(m, a.tpr, red);
-  const float inv = m > 0.f ? __fdiv_rn(7.0f, m) : 0.f;
-
-#pragma unroll
-  for (int r = 0; r < E; r += 2) fma2(v[r], v[r + 1], inv, kMagic8);
-
-  if (active) {
-    uint32_t wd[E / 8];
-#pragma unroll
-    for (int w = 0; w < E / 8; ++w) {
-      const float* q = &v[8 * w];
-      wd[w] = pack_codes8(__float_as_uint(q[0]), __float_as_uint(q[1]), __float_as_uint(q[2]),
-                          __float_as_uint(q[3]), __float_as_uint(q[4]), __float_as_uint(q[5]),
-                          __float_as_uint(q[6]), __float_as_uint(q[7]));
-    }
-    const int es = b * g + E * t;              // first channel of the thread's run
-    const int cpr = K / 32;                    // 16-byte chunks per row
-    uint8_t* rdst = a.tiled ? a.codes + (row >> 5) * cpr * 512 + (row & 31) * 16
-                            : a.codes + row * (K / 2);
-    const int cstride = a.tiled ? 512 : 16;    // bytes between consecutive chunks of a row
-    if constexpr (E >= 32) {
-#pragma unroll
-      for (int q = 0; q < E / 32; ++q) {
-        *reinterpret_cast<uint4*>(rdst + ((es >> 5) + q) * cstride) =
-            make_uint4(wd[4 * q], wd[4 * q + 1], wd[4 * q + 2], wd[4 * q + 3]);
+        for (int r = 0; r < E; ++r) v[r] = 0.f;
       }
+      if (!__syncthreads_and(ok)) {
+        ring_fail(ring, grp, ngroups, a.status);
+        return;
+      }
+      // Every thread has read the slot: it takes the group S turns ahead.
+      const int64_t next = grp + static_cast<int64_t>(ring.S) * gridDim.x;
+      if (tid == 0 && next < ngroups) ring_issue<Tin>(a, next, R, ring.slot(), ring.bar());
+      ring.advance();
     } else {
-      *reinterpret_cast<uint2*>(rdst + (es >> 5) * cstride + (es & 31) / 2) = make_uint2(wd[0], wd[1]);
+      if (active) {
+        const int64_t tok = row / a.H;
+        const int64_t h = row - tok * a.H;
+        const Tin* p = static_cast<const Tin*>(a.x) + tok * a.ld_t + h * a.ld_h + static_cast<int64_t>(b) * g + 8 * t;
+#pragma unroll
+        for (int i = 0; i < NC; ++i) load_chunk8(p + i * 8 * TPB, &v[8 * i]);
+      } else {
+#pragma unroll
+        for (int r = 0; r < E; ++r) v[r] = 0.f;
+      }
     }
-  }
 
-  if (row_ok && j == 0) a.scale[row] = m * a.scale_mul;
-  if (active && t == 0 && a.offset != nullptr) {
-    a.offset[row * a.G + b] = offs ? (rotate ? off * a.inv_sqrt_g : off) : 0.f;
-  }
-  if constexpr (!kRing) break;
-  grp += gridDim.x;
-  if (grp >= ngroups) break;
+    float off = 0.f;
+    if (rotate) {
+      // Offset = x[block start] / sqrt(g); removing it first leaves the residual.
+      if (offs && t == 0) {
+        off = v[0];
+        v[0] = 0.f;
+      }
+      fwht_reg_stages<E, 1, LOGE>(v);   // channel bits 1, 2 and 3+P .. L-1
+    } else if (offs) {
+      // Block mean by a pairwise tree (depth log2(E) in the thread, P across threads).
+      off = group_reduce<false>(tree_sum<E>(v), TPB, red) * (1.0f / static_cast<float>(g));
+    }
+
+    const int base = lrow * K + b * g;
+    if (active) {
+#pragma unroll
+      for (int i = 0; i < NC; ++i) {
+        const int e0 = base + 8 * t + 8 * TPB * i;
+        *reinterpret_cast<float4*>(buf + swz_narrow<L, LOGE>(e0)) =
+            make_float4(v[8 * i], v[8 * i + 1], v[8 * i + 2], v[8 * i + 3]);
+        *reinterpret_cast<float4*>(buf + swz_narrow<L, LOGE>(e0 + 4)) =
+            make_float4(v[8 * i + 4], v[8 * i + 5], v[8 * i + 6], v[8 * i + 7]);
+      }
+    }
+    __syncwarp();  // a block's TPB <= 8 threads share one warp
+    // Pass 2: register r holds channel E t + r of block b.
+    if (active) {
+#pragma unroll
+      for (int m = 0; m < E / 4; ++m) {
+        const float4 f = *reinterpret_cast<const float4*>(buf + swz_narrow<L, LOGE>(base + E * t + 4 * m));
+        v[4 * m] = f.x;
+        v[4 * m + 1] = f.y;
+        v[4 * m + 2] = f.z;
+        v[4 * m + 3] = f.w;
+      }
+    }
+    if (rotate) {
+#pragma unroll
+      for (int r = 0; r < E; r += 2) {   // channel bit 0
+        const float x0 = v[r], x1 = v[r + 1];
+        v[r] = x0 + x1;
+        v[r + 1] = x0 - x1;
+      }
+      fwht_reg_stages<E, 3, 3 + P>(v);   // channel bits 3 .. 3+P-1
+    } else if (offs) {
+#pragma unroll
+      for (int r = 0; r < E; r += 2) sub2(v[r], v[r + 1], off);
+    }
+
+    // Per-row absmax of the residual.
+    float mx[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int r = 0; r < E; ++r) mx[r & 3] = fmaxf(mx[r & 3], fabsf(v[r]));
+    float m = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
+    m = group_reduce<true>(m, a.tpr, red);
+    const float inv = m > 0.f ? __fdiv_rn(7.0f, m) : 0.f;
+
+#pragma unroll
+    for (int r = 0; r < E; r += 2) fma2(v[r], v[r + 1], inv, kMagic8);
+
+    if (active) {
+      uint32_t wd[E / 8];
+#pragma unroll
+      for (int w = 0; w < E / 8; ++w) {
+        const float* q = &v[8 * w];
+        wd[w] = pack_codes8(__float_as_uint(q[0]), __float_as_uint(q[1]), __float_as_uint(q[2]),
+                            __float_as_uint(q[3]), __float_as_uint(q[4]), __float_as_uint(q[5]),
+                            __float_as_uint(q[6]), __float_as_uint(q[7]));
+      }
+      const int es = b * g + E * t;              // first channel of the thread's run
+      const int cpr = K / 32;                    // 16-byte chunks per row
+      uint8_t* rdst = a.tiled ? a.codes + (row >> 5) * cpr * 512 + (row & 31) * 16
+                              : a.codes + row * (K / 2);
+      const int cstride = a.tiled ? 512 : 16;    // bytes between consecutive chunks of a row
+      if constexpr (E >= 32) {
+#pragma unroll
+        for (int q = 0; q < E / 32; ++q) {
+          *reinterpret_cast<uint4*>(rdst + ((es >> 5) + q) * cstride) =
+              make_uint4(wd[4 * q], wd[4 * q + 1], wd[4 * q + 2], wd[4 * q + 3]);
+        }
+      } else {
+        *reinterpret_cast<uint2*>(rdst + (es >> 5) * cstride + (es & 31) / 2) = make_uint2(wd[0], wd[1]);
+      }
+    }
+
+    if (row_ok && j == 0) a.scale[row] = m * a.scale_mul;
+    if (active && t == 0 && a.offset != nullptr) {
+      a.offset[row * a.G + b] = offs ? (rotate ? off * a.inv_sqrt_g : off) : 0.f;
+    }
+    if constexpr (!kRing) break;
+    grp += gridDim.x;
+    if (grp >= ngroups) break;
   }
 }
 
@@ -526,8 +570,14 @@ __global__ void __launch_bounds__(WideGeo<L>::kMaxThreads) quantize_rows_wide_ke
   float* buf = reinterpret_cast<float*>(smem);                                  // [R][K] fp32 (rotate)
   uint8_t* cbuf = smem + (rotate ? static_cast<size_t>(R) * K * 4 : 0);         // [R][K/2] codes
   float* red = reinterpret_cast<float*>(cbuf + static_cast<size_t>(R) * (K / 2));
-  uint8_t* slot = reinterpret_cast<uint8_t*>(red + 32);                         // kRing: [R][K] inputs
-  const uint32_t bar = smem_u32(slot + static_cast<size_t>(R) * K * sizeof(Tin));
+  // kRing: ring_slots slots of [R][K] inputs after the reduction scratch, then their barriers.
+  RowRing ring;
+  ring.base = reinterpret_cast<uint8_t*>(red + 32);
+  ring.slot_bytes = static_cast<uint32_t>(R) * K * sizeof(Tin);
+  ring.S = a.ring_slots;
+  ring.bar0 = smem_u32(ring.base + static_cast<size_t>(ring.S) * ring.slot_bytes);
+  ring.s = 0;
+  ring.phase = 0;
 
   const int tid = threadIdx.x;
   const int lrow = tid / a.tpr;
@@ -536,173 +586,172 @@ __global__ void __launch_bounds__(WideGeo<L>::kMaxThreads) quantize_rows_wide_ke
   const int t1 = j % TPB;
   const int64_t ngroups = (a.rows + R - 1) / R;
   int64_t grp = blockIdx.x;
-  uint32_t phase = 0;
   if constexpr (kRing) {
     if (tid == 0) {
       abort_flag = 0;
-      mbar_init(bar, 1);
+      for (int k = 0; k < ring.S; ++k) mbar_init(ring.bar0 + 8u * k, 1);
       mbar_fence_init();
     }
     __syncthreads();
   }
   griddep_wait();
   griddep_launch_dependents();
-  if constexpr (kRing) {
-    if (tid == 0 && grp < ngroups) ring_issue<Tin>(a, grp, R, slot, bar);
-  }
+  if constexpr (kRing) ring_start<Tin>(a, ring, R, ngroups);
 
   while (true) {
-  const int64_t row = grp * R + lrow;
-  const bool row_ok = row < a.rows;
-  const bool active = row_ok && (j < a.G * TPB);
+    const int64_t row = grp * R + lrow;
+    const bool row_ok = row < a.rows;
+    const bool active = row_ok && (j < a.G * TPB);
 
-  float v[E];
-  if constexpr (kRing) {
-    const bool ok = mbar_wait(bar, phase, &abort_flag);
-    phase ^= 1u;
-    if (ok && active) {
-      const Tin* p = reinterpret_cast<const Tin*>(slot) + static_cast<size_t>(lrow) * K + b * g + 8 * t1;
+    float v[E];
+    if constexpr (kRing) {
+      const bool ok = mbar_wait(ring.bar(), ring.phase, &abort_flag);
+      if (ok && active) {
+        const Tin* p = reinterpret_cast<const Tin*>(ring.slot()) + static_cast<size_t>(lrow) * K + b * g + 8 * t1;
 #pragma unroll
-      for (int i = 0; i < NC; ++i) load_chunk8_smem(p + i * 8 * TPB, &v[8 * i]);
+        for (int i = 0; i < NC; ++i) load_chunk8_smem(p + i * 8 * TPB, &v[8 * i]);
+      } else {
+#pragma unroll
+        for (int r = 0; r < E; ++r) v[r] = 0.f;
+      }
+      if (!__syncthreads_and(ok)) {
+        ring_fail(ring, grp, ngroups, a.status);
+        return;
+      }
+      // Every thread has read the slot: it takes the group S turns ahead.
+      const int64_t next = grp + static_cast<int64_t>(ring.S) * gridDim.x;
+      if (tid == 0 && next < ngroups) ring_issue<Tin>(a, next, R, ring.slot(), ring.bar());
+      ring.advance();
     } else {
+      if (active) {
+        const int64_t t = row / a.H;
+        const int64_t h = row - t * a.H;
+        const Tin* p = static_cast<const Tin*>(a.x) + t * a.ld_t + h * a.ld_h + static_cast<int64_t>(b) * g + 8 * t1;
 #pragma unroll
-      for (int r = 0; r < E; ++r) v[r] = 0.f;
-    }
-    if (!__syncthreads_and(ok)) {
-      ring_fail(bar, phase ^ 1u, a.status);
-      return;
-    }
-    if (tid == 0 && grp + gridDim.x < ngroups) ring_issue<Tin>(a, grp + gridDim.x, R, slot, bar);
-  } else {
-    if (active) {
-      const int64_t t = row / a.H;
-      const int64_t h = row - t * a.H;
-      const Tin* p = static_cast<const Tin*>(a.x) + t * a.ld_t + h * a.ld_h + static_cast<int64_t>(b) * g + 8 * t1;
+        for (int i = 0; i < NC; ++i) load_chunk8(p + i * 8 * TPB, &v[8 * i]);
+      } else {
 #pragma unroll
-      for (int i = 0; i < NC; ++i) load_chunk8(p + i * 8 * TPB, &v[8 * i]);
-    } else {
-#pragma unroll
-      for (int r = 0; r < E; ++r) v[r] = 0.f;
-    }
-  }
-
-  float off = 0.f;
-  if (rotate) {
-    // Offset = x[block start] / sqrt(g); removing it first leaves the residual.
-    if (offs && t1 == 0) {
-      off = v[0];
-      v[0] = 0.f;
-    }
-    // Index bits {0,1,2} and {3+P, .., L-1}: bit 0 on scalar adds, the others
-    // packed on the (even, odd) register pairs the loads produced.
-#pragma unroll
-    for (int r = 0; r < E; r += 2) {
-      const float x0 = v[r], x1 = v[r + 1];
-      v[r] = x0 + x1;
-      v[r + 1] = x0 - x1;
-    }
-    fwht_reg_stages<E, 1, LOGE>(v);
-    float* rb = buf + static_cast<size_t>(lrow) * K + static_cast<size_t>(b) * g;
-    if (active) {
-#pragma unroll
-      for (int i = 0; i < NC; ++i) {
-        const int e0 = 8 * t1 + 8 * TPB * i;
-        *reinterpret_cast<float4*>(rb + swz<P>(e0)) = make_float4(v[8 * i], v[8 * i + 1], v[8 * i + 2], v[8 * i + 3]);
-        *reinterpret_cast<float4*>(rb + swz<P>(e0 + 4)) =
-            make_float4(v[8 * i + 4], v[8 * i + 5], v[8 * i + 6], v[8 * i + 7]);
+        for (int r = 0; r < E; ++r) v[r] = 0.f;
       }
     }
-    // A block's TPB threads share one warp (TPB <= 32) except for g = 8192.
+
+    float off = 0.f;
+    if (rotate) {
+      // Offset = x[block start] / sqrt(g); removing it first leaves the residual.
+      if (offs && t1 == 0) {
+        off = v[0];
+        v[0] = 0.f;
+      }
+      // Index bits {0,1,2} and {3+P, .., L-1}: bit 0 on scalar adds, the others
+      // packed on the (even, odd) register pairs the loads produced.
+#pragma unroll
+      for (int r = 0; r < E; r += 2) {
+        const float x0 = v[r], x1 = v[r + 1];
+        v[r] = x0 + x1;
+        v[r + 1] = x0 - x1;
+      }
+      fwht_reg_stages<E, 1, LOGE>(v);
+      float* rb = buf + static_cast<size_t>(lrow) * K + static_cast<size_t>(b) * g;
+      if (active) {
+#pragma unroll
+        for (int i = 0; i < NC; ++i) {
+          const int e0 = 8 * t1 + 8 * TPB * i;
+          *reinterpret_cast<float4*>(rb + swz<P>(e0)) = make_float4(v[8 * i], v[8 * i + 1], v[8 * i + 2], v[8 * i + 3]);
+          *reinterpret_cast<float4*>(rb + swz<P>(e0 + 4)) =
+              make_float4(v[8 * i + 4], v[8 * i + 5], v[8 * i + 6], v[8 * i + 7]);
+        }
+      }
+      // A block's TPB threads share one warp (TPB <= 32) except for g = 8192.
+      if constexpr (TPB <= 32) {
+        __syncwarp();
+      } else {
+        __syncthreads();
+      }
+      if (active) {
+#pragma unroll
+        for (int hi = 0; hi < (1 << P); ++hi) {
+          const int e = ((t1 & ((1 << (3 - Q)) - 1)) << Q) | (hi << 3) | ((t1 >> (3 - Q)) << (3 + P));
+          if constexpr (Q == 2) {
+            const float4 f = *reinterpret_cast<const float4*>(rb + swz<P>(e));
+            v[4 * hi] = f.x; v[4 * hi + 1] = f.y; v[4 * hi + 2] = f.z; v[4 * hi + 3] = f.w;
+          } else {
+            const float2 f = *reinterpret_cast<const float2*>(rb + swz<P>(e));
+            v[2 * hi] = f.x; v[2 * hi + 1] = f.y;
+          }
+        }
+      }
+      fwht_bits<E, Q, LOGE>(v);  // index bits {3, .., 3+P-1}
+    } else if (offs) {
+      float s = 0.f;
+#pragma unroll
+      for (int r = 0; r < E; ++r) s += v[r];
+      s = group_reduce<false>(s, TPB, red);
+      off = s * (1.0f / static_cast<float>(g));
+#pragma unroll
+      for (int r = 0; r < E; ++r) v[r] -= off;
+    }
+
+    // Per-row absmax of the residual.
+    float m = 0.f;
+#pragma unroll
+    for (int r = 0; r < E; ++r) m = fmaxf(m, fabsf(v[r]));
+    m = group_reduce<true>(m, a.tpr, red);
+    const float inv = m > 0.f ? __fdiv_rn(7.0f, m) : 0.f;
+
+#pragma unroll
+    for (int r = 0; r < E; r += 2) fma2(v[r], v[r + 1], inv, kMagic8);
+
+    uint8_t* crow = cbuf + static_cast<size_t>(lrow) * (K / 2) + static_cast<size_t>(b) * (g / 2);
+    if (active) {
+      if (rotate) {
+#pragma unroll
+        for (int hi = 0; hi < (1 << P); ++hi) {
+          const int e = ((t1 & ((1 << (3 - Q)) - 1)) << Q) | (hi << 3) | ((t1 >> (3 - Q)) << (3 + P));
+          // Bits 4-21 of a rounded value are zero, so (u1 << 4) + u0 carries the
+          // byte of two codes in its low 8 bits.
+          if constexpr (Q == 2) {
+            const uint32_t b0 = (__float_as_uint(v[4 * hi + 1]) << 4) + __float_as_uint(v[4 * hi]);
+            const uint32_t b1 = (__float_as_uint(v[4 * hi + 3]) << 4) + __float_as_uint(v[4 * hi + 2]);
+            *reinterpret_cast<uint16_t*>(crow + e / 2) = static_cast<uint16_t>(__byte_perm(b0, b1, 0x0040));
+          } else {
+            crow[e / 2] = static_cast<uint8_t>((__float_as_uint(v[2 * hi + 1]) << 4) + __float_as_uint(v[2 * hi]));
+          }
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < NC; ++i) {
+          uint32_t w = 0;
+#pragma unroll
+          for (int e = 0; e < 8; ++e) w |= (__float_as_uint(v[8 * i + e]) & 0xFu) << (4 * e);
+          *reinterpret_cast<uint32_t*>(crow + 4 * t1 + 4 * TPB * i) = w;
+        }
+      }
+    }
+    // Each block's TPB threads write the block's g/2 code bytes as 16-byte chunks.
     if constexpr (TPB <= 32) {
       __syncwarp();
     } else {
       __syncthreads();
     }
     if (active) {
-#pragma unroll
-      for (int hi = 0; hi < (1 << P); ++hi) {
-        const int e = ((t1 & ((1 << (3 - Q)) - 1)) << Q) | (hi << 3) | ((t1 >> (3 - Q)) << (3 + P));
-        if constexpr (Q == 2) {
-          const float4 f = *reinterpret_cast<const float4*>(rb + swz<P>(e));
-          v[4 * hi] = f.x; v[4 * hi + 1] = f.y; v[4 * hi + 2] = f.z; v[4 * hi + 3] = f.w;
-        } else {
-          const float2 f = *reinterpret_cast<const float2*>(rb + swz<P>(e));
-          v[2 * hi] = f.x; v[2 * hi + 1] = f.y;
-        }
+      const int cpr = K / 32;       // 16-byte chunks per row
+      const int cpb = g / 32;       // 16-byte chunks per block
+      for (int c = t1; c < cpb; c += TPB) {
+        const int cc = b * cpb + c;
+        const uint4 w = *reinterpret_cast<const uint4*>(crow + c * 16);
+        uint8_t* dst = a.tiled ? a.codes + ((row >> 5) * cpr + cc) * 512 + (row & 31) * 16
+                               : a.codes + row * (K / 2) + cc * 16;
+        *reinterpret_cast<uint4*>(dst) = w;
       }
     }
-    fwht_bits<E, Q, LOGE>(v);  // index bits {3, .., 3+P-1}
-  } else if (offs) {
-    float s = 0.f;
-#pragma unroll
-    for (int r = 0; r < E; ++r) s += v[r];
-    s = group_reduce<false>(s, TPB, red);
-    off = s * (1.0f / static_cast<float>(g));
-#pragma unroll
-    for (int r = 0; r < E; ++r) v[r] -= off;
-  }
 
-  // Per-row absmax of the residual.
-  float m = 0.f;
-#pragma unroll
-  for (int r = 0; r < E; ++r) m = fmaxf(m, fabsf(v[r]));
-  m = group_reduce<true>(m, a.tpr, red);
-  const float inv = m > 0.f ? __fdiv_rn(7.0f, m) : 0.f;
-
-#pragma unroll
-  for (int r = 0; r < E; r += 2) fma2(v[r], v[r + 1], inv, kMagic8);
-
-  uint8_t* crow = cbuf + static_cast<size_t>(lrow) * (K / 2) + static_cast<size_t>(b) * (g / 2);
-  if (active) {
-    if (rotate) {
-#pragma unroll
-      for (int hi = 0; hi < (1 << P); ++hi) {
-        const int e = ((t1 & ((1 << (3 - Q)) - 1)) << Q) | (hi << 3) | ((t1 >> (3 - Q)) << (3 + P));
-        // Bits 4-21 of a rounded value are zero, so (u1 << 4) + u0 carries the
-        // byte of two codes in its low 8 bits.
-        if constexpr (Q == 2) {
-          const uint32_t b0 = (__float_as_uint(v[4 * hi + 1]) << 4) + __float_as_uint(v[4 * hi]);
-          const uint32_t b1 = (__float_as_uint(v[4 * hi + 3]) << 4) + __float_as_uint(v[4 * hi + 2]);
-          *reinterpret_cast<uint16_t*>(crow + e / 2) = static_cast<uint16_t>(__byte_perm(b0, b1, 0x0040));
-        } else {
-          crow[e / 2] = static_cast<uint8_t>((__float_as_uint(v[2 * hi + 1]) << 4) + __float_as_uint(v[2 * hi]));
-        }
-      }
-    } else {
-#pragma unroll
-      for (int i = 0; i < NC; ++i) {
-        uint32_t w = 0;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) w |= (__float_as_uint(v[8 * i + e]) & 0xFu) << (4 * e);
-        *reinterpret_cast<uint32_t*>(crow + 4 * t1 + 4 * TPB * i) = w;
-      }
+    if (row_ok && j == 0) a.scale[row] = m * a.scale_mul;
+    if (active && t1 == 0 && a.offset != nullptr) {
+      a.offset[row * a.G + b] = offs ? (rotate ? off * a.inv_sqrt_g : off) : 0.f;
     }
-  }
-  // Each block's TPB threads write the block's g/2 code bytes as 16-byte chunks.
-  if constexpr (TPB <= 32) {
-    __syncwarp();
-  } else {
-    __syncthreads();
-  }
-  if (active) {
-    const int cpr = K / 32;       // 16-byte chunks per row
-    const int cpb = g / 32;       // 16-byte chunks per block
-    for (int c = t1; c < cpb; c += TPB) {
-      const int cc = b * cpb + c;
-      const uint4 w = *reinterpret_cast<const uint4*>(crow + c * 16);
-      uint8_t* dst = a.tiled ? a.codes + ((row >> 5) * cpr + cc) * 512 + (row & 31) * 16
-                             : a.codes + row * (K / 2) + cc * 16;
-      *reinterpret_cast<uint4*>(dst) = w;
-    }
-  }
-
-  if (row_ok && j == 0) a.scale[row] = m * a.scale_mul;
-  if (active && t1 == 0 && a.offset != nullptr) {
-    a.offset[row * a.G + b] = offs ? (rotate ? off * a.inv_sqrt_g : off) : 0.f;
-  }
-  if constexpr (!kRing) break;
-  grp += gridDim.x;
-  if (grp >= ngroups) break;
+    if constexpr (!kRing) break;
+    grp += gridDim.x;
+    if (grp >= ngroups) break;
   }
 }
 
@@ -1074,20 +1123,35 @@ constexpr int kNoRing = 1;  // launch_ring: use the one-shot kernel instead
 // Launches the persistent (ring) form of a row kernel when the input has one
 // head, there are more row groups than SMs, and the slot fits: one CTA per
 // resident slot, each looping over the groups grid-stride.
+// base_smem is the kernel's shared memory without the ring, slot_bytes one
+// slot (rows_per_cta rows of input). The slot count (1 to 3) is the one with
+// the most slots per SM, so the most rows in flight; ties take more slots.
 template <typename F>
-int launch_ring(F* kern, const QuantArgs& a, int threads, size_t smem, cudaStream_t stream) {
-  if (a.H != 1 || smem > kMaxDynSmem) return kNoRing;
+int launch_ring(F* kern, QuantArgs a, int threads, size_t base_smem, size_t slot_bytes, cudaStream_t stream) {
+  if (a.H != 1) return kNoRing;
   const int sms = sm_count();
   const int64_t groups = (a.rows + a.rows_per_cta - 1) / a.rows_per_cta;
   if (sms <= 0 || groups <= sms) return kNoRing;
   if (prefer_max_shared(kern) != OFFQ_OK) return OFFQ_ERR_CUDA;
-  if (smem > 48 * 1024 &&
-      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) != cudaSuccess)
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kMaxDynSmem)) !=
+      cudaSuccess)
     return OFFQ_ERR_CUDA;
-  int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem) != cudaSuccess) return OFFQ_ERR_CUDA;
-  if (per_sm < 1) return kNoRing;
-  const int64_t grid = std::min<int64_t>(groups, static_cast<int64_t>(sms) * per_sm);
+  int best_s = 0, best_per_sm = 0;
+  for (int S = 1; S <= 3; ++S) {
+    const size_t smem = base_smem + S * (slot_bytes + 8);
+    if (smem > kMaxDynSmem) break;
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem) != cudaSuccess)
+      return OFFQ_ERR_CUDA;
+    if (per_sm >= 1 && per_sm * S >= best_per_sm * best_s) {
+      best_s = S;
+      best_per_sm = per_sm;
+    }
+  }
+  if (best_s == 0) return kNoRing;
+  a.ring_slots = best_s;
+  const size_t smem = base_smem + best_s * (slot_bytes + 8);
+  const int64_t grid = std::min<int64_t>(groups, static_cast<int64_t>(sms) * best_per_sm);
   return launch_pdl(kern, dim3(static_cast<unsigned>(grid)), dim3(threads), smem, stream, a);
 }
 
@@ -1108,8 +1172,8 @@ int launch_narrow(QuantArgs a, cudaStream_t stream) {
   a.tpr = tpr;
   a.rows_per_cta = R;
   const size_t smem = 128 + static_cast<size_t>(R) * row_smem;
-  const int rs = launch_ring(quantize_rows_kernel<L, Tin, true>, a, R * tpr,
-                             smem + static_cast<size_t>(R) * a.K * sizeof(Tin) + 8, stream);
+  const int rs = launch_ring(quantize_rows_kernel<L, Tin, true>, a, R * tpr, smem,
+                             static_cast<size_t>(R) * a.K * sizeof(Tin), stream);
   if (rs != kNoRing) return rs;
   auto kern = quantize_rows_kernel<L, Tin, false>;
   if (prefer_max_shared(kern) != OFFQ_OK) return OFFQ_ERR_CUDA;
@@ -1141,8 +1205,8 @@ int launch_wide(QuantArgs a, cudaStream_t stream) {
   a.tpr = tpr;
   a.rows_per_cta = R;
   const size_t smem = static_cast<size_t>(R) * row_smem + 32 * sizeof(float);
-  const int rs = launch_ring(quantize_rows_wide_kernel<L, Tin, true>, a, R * tpr,
-                             smem + static_cast<size_t>(R) * a.K * sizeof(Tin) + 8, stream);
+  const int rs = launch_ring(quantize_rows_wide_kernel<L, Tin, true>, a, R * tpr, smem,
+                             static_cast<size_t>(R) * a.K * sizeof(Tin), stream);
   if (rs != kNoRing) return rs;
   auto kern = quantize_rows_wide_kernel<L, Tin, false>;
   if (smem > 48 * 1024) {
@@ -1204,7 +1268,7 @@ int dispatch_g(const QuantArgs& a, int g, cudaStream_t s) {
     case 128: return launch_narrow<7, Tin>(a, s);
     case 256: return launch_narrow<8, Tin>(a, s);
     case 512: return launch_narrow<9, Tin>(a, s);
-    case 1024: return launch_wide<10, Tin>(a, s);
+    case 1024: return launch_narrow<10, Tin>(a, s);
     case 2048: return launch_wide<11, Tin>(a, s);
     case 4096: return launch_wide<12, Tin>(a, s);
     case 8192: return launch_wide<13, Tin>(a, s);
