@@ -14,7 +14,7 @@
 //
 // Kernel layouts (per g = 2^L; the Hadamard is a Kronecker product of 2x2
 // stages, so the stages may run in any order):
-//  * g <= 512 (quantize_rows_kernel): a thread owns E = 2^ceil((L+3)/2)
+//  * g <= 1024 (quantize_rows_kernel): a thread owns E = 2^ceil((L+3)/2)
 //    elements and TPB = g / E threads share a block. Pass 1 loads 16-byte
 //    vectors (8 channels, coalesced across the block's threads) and runs the
 //    stages of every index bit it holds except bit 0; one swizzled transpose
@@ -23,12 +23,18 @@
 //    thread packs its E codes into whole 16-byte chunks of the code buffer.
 //    Packed fp32x2 instructions take register pairs that differ in index bit 0,
 //    so the bit-0 stage alone runs on scalar adds.
-//  * g >= 1024 (quantize_rows_wide_kernel): E = 2^ceil((L+1)/2) elements per
+//  * g >= 2048 (quantize_rows_wide_kernel): E = 2^ceil((L+1)/2) elements per
 //    thread, the same two passes with pass 2 keeping the lowest one or two
 //    index bits, and codes staged in shared memory before the 16-byte writes.
+//  * Both come in a one-shot form (a CTA per group of rows) and, for one-head
+//    inputs with more row groups than SMs, a persistent form whose CTAs stage
+//    their next groups in shared memory by bulk async copies (cp.async.bulk,
+//    mbarrier completion) while they compute the current one.
 //  * No rotation and one block of g >= 1024 per row
-//    (quantize_rows_stream_kernel): a warp per row, offset and absmax from one
-//    sweep, codes from a second.
+//    (quantize_rows_bulk_kernel): a persistent kernel whose warps stream rows
+//    through their own rings of shared-memory slots; offset and absmax from one
+//    sweep of the slot, codes from a second. Rows too long for the ring take
+//    quantize_rows_stream_kernel (a warp per row, the row in registers).
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
