@@ -597,6 +597,75 @@ def time_quant_sites(device, args, flush_l2, stream):
     return out
 
 
+def time_decode(device, args, flush_l2, stream):
+    """The decode sweep on Llama-2-7B shapes: T = 1, 8, 32, 64 tokens through the
+    activation quantizer, one 4096 -> 11008 W4A4 linear and the KV4 quantizer of
+    32 heads x 128 per token (keys with the per-head Hadamard, values offset
+    only). Per-call events, L2 flushed before each call, so every GEMM streams
+    its 22.5 MB of weight codes from HBM."""
+    import torch
+    from paper_2606_07116_gb300 import offq as Q
+    peaks = load_peaks()
+    K, N, H, hd = 4096, 11008, 32, 128
+    g = W.block_for(K)
+    wt = torch.from_numpy(W.weights(N, K, seed=501)).to(device)
+    wc, ws, wr = Q.prepare_weight(wt, g, rotate=False)
+    del wt
+    w_bytes = wc.numel() + 4 * N + 4 * N * (K // g)
+    reps = max(1, min(args.steps, 50))
+    out = {"what": "decode on Llama-2-7B shapes: offq_quantize_act + offq_w4a4_linear 4096 -> 11008 + "
+                   "offq_kv4_quantize of the keys (rotated) and values, per-call events, L2 flushed before "
+                   "each call; weight_gbs = weight codes, scales and row sums read by the GEMM / its time",
+           "points": []}
+    best = None
+    for T in W.DECODE_BATCHES:
+        x = W.to_bf16(W.activations(T, K, seed=600 + T, n_out=4, mult=100.0)).to(device)
+        kv = W.to_bf16(W.kv_heads(T, H, hd, seed=700 + T)).to(device).reshape(T, H * hd)
+        codes = torch.empty((Q.padded_rows(T), K // 2), dtype=torch.uint8, device=device)
+        scale = torch.empty((T,), dtype=torch.float32, device=device)
+        off = torch.empty((T, K // g), dtype=torch.float32, device=device)
+        y = torch.empty((T, N), dtype=torch.bfloat16, device=device)
+        kc = torch.empty((T, H, hd // 2), dtype=torch.uint8, device=device)
+        ks = torch.empty((T, H), dtype=torch.float32, device=device)
+        ko = torch.empty((T, H), dtype=torch.float32, device=device)
+        ts = {"quant": [], "gemm": [], "kv4": []}
+        for r in range(3 + reps):
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
+            flush_l2()
+            ev[0].record(stream)
+            Q.offq_quantize_act(x, T, K, x.stride(0), g, Q.OFFQ_OFFSET, codes, scale, off, stream)
+            ev[1].record(stream)
+            flush_l2()
+            ev[2].record(stream)
+            Q.offq_w4a4_linear(codes, scale, off, T, N, K, g, wc, ws, wr, y, y.stride(0), None, stream)
+            ev[3].record(stream)
+            flush_l2()
+            ev[4].record(stream)
+            Q.offq_kv4_quantize(kv, T, H, hd, kv.stride(0), Q.OFFQ_ROTATE | Q.OFFQ_OFFSET, kc, ks, ko, stream)
+            Q.offq_kv4_quantize(kv, T, H, hd, kv.stride(0), Q.OFFQ_OFFSET, kc, ks, ko, stream)
+            ev[5].record(stream)
+            torch.cuda.synchronize(device)
+            if r >= 3:
+                ts["quant"].append(ev[0].elapsed_time(ev[1]))
+                ts["gemm"].append(ev[2].elapsed_time(ev[3]))
+                ts["kv4"].append(ev[4].elapsed_time(ev[5]))
+        qm, gm, km = (sum(ts[k]) / len(ts[k]) for k in ("quant", "gemm", "kv4"))
+        gbs = w_bytes / (gm * 1e-3) / 1e9
+        pt = {"T": T, "quant_us": round(qm * 1e3, 2), "gemm_us": round(gm * 1e3, 2), "kv4_us": round(km * 1e3, 2),
+              "gemm_tops": round(2.0 * T * N * K / (gm * 1e-3) / 1e12, 3), "weight_gbs": round(gbs, 1),
+              "weight_frac": round(gbs / peaks["hbm_gbs"], 4)}
+        out["points"].append(pt)
+        if best is None or pt["weight_gbs"] > best["weight_gbs"]:
+            best = pt
+    st = Q.offq_get_device_status(stream)
+    if st != Q.OFFQ_OK:
+        raise RuntimeError(f"device status after the decode sweep: {Q.status_string(st)}")
+    out["roofline"] = {"bound": "hbm", "kernel": f"w4a4_gemm_kernel weight stream (T = {best['T']})",
+                       "achieved": best["weight_gbs"], "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                       "frac": best["weight_frac"], "bytes": w_bytes}
+    return out
+
+
 def _pair_times(events):
     return [events[i].elapsed_time(events[i + 1]) for i in range(0, len(events), 2)]
 
@@ -782,6 +851,7 @@ def run_gpu(args, rank, world, local_rank):
         line["builder"] = time_builder(device, args, flush_l2, stream)
     if not args.no_group and world == 1:
         line["act_quant_prefill"] = time_quant_sites(device, args, flush_l2, stream)
+        line["decode"] = time_decode(device, args, flush_l2, stream)
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w, budget_s=args.cpu_budget)
     return line
@@ -896,12 +966,28 @@ def main():
     ap.add_argument("--key-rotation-tokens", type=int, default=0,
                     help="time only the key-cache rotation calls, at this many tokens, and print that object "
                          "(a side measurement for profiling, not the bench line)")
+    ap.add_argument("--decode", action="store_true",
+                    help="time only the decode sweep (1/8/32/64 tokens) and print that object")
     ap.add_argument("--quant-sites", action="store_true",
                     help="time only the activation quantizer on the larger prefill inputs and print that object "
                          "(a side measurement for profiling, not the bench line)")
     args = ap.parse_args()
     if args.warmup < 3:
         raise SystemExit("--warmup must be at least 3")
+    if args.decode:
+        import torch
+        import __graft_entry__ as G
+        G.build()
+        device = torch.device("cuda", 0)
+        torch.cuda.set_device(device)
+        flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
+
+        def flush_l2():
+            flush.zero_()
+            flush[:L2_FLUSH_BYTES // 2].view(torch.int32).amax()
+
+        print(json.dumps(time_decode(device, args, flush_l2, torch.cuda.current_stream(device))), flush=True)
+        return
     if args.quant_sites:
         import torch
         import __graft_entry__ as G

@@ -116,6 +116,7 @@ def test_oracle_codes_through_gemm():
     (40, 4096, 512, 32, "f32", None),      # 128 offset blocks of 32 channels
     (300, 1024, 800, 128, "bf16", None),   # the paper's group size, 8 blocks; several tiles per CTA
     (50, 1024, 258, 256, "bf16", 264),     # N % 4 != 0 with 4 offset blocks (scalar epilogue loads)
+    (5, 96, 200, 32, "f32", None),         # K = 96: a k-tile of three 32-channel chunks
     # 2 x 40 pair tiles: on 76 clusters the 4 tiles past the first wave are cut
     # along N into 64-column pieces (ragged N at the end), with 4 and 1 offset blocks.
     (512, 1024, 10200, 256, "bf16", None),
