@@ -64,3 +64,18 @@ def test_reference_arm_runs_on_rank_zero_only():
     class Args:
         workload, steps, warmup, ref_budget = "toy", 1, 0, 0.1
     assert bench.run_reference(Args, rank=1, world=2) is None
+
+
+def test_reference_arm_line_on_rank_zero():
+    """The reference arm times the float64 oracle on a bounded token sample and prints the
+    base contract's keys, with an end-to-end figure that copies nothing."""
+    class Args:
+        workload, steps, warmup, ref_budget = "toy", 2, 1, 0.5
+    line = bench.run_reference(Args, rank=0, world=1)
+    assert line["impl"] == "reference" and line["metric"] == bench.METRIC and line["unit"] == bench.UNIT
+    assert line["value"] > 0 and line["higher_is_better"] is True and line["steps"] == 2
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["value"] == line["value"]
+    assert line["cpu_baseline"]["cores"] >= 1
+    assert line["e2e"] == {"value": line["value"], "unit": bench.UNIT, "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
+    assert 4 <= line["config"]["tokens_per_step"] <= 16
