@@ -129,7 +129,7 @@ class ClockSampler:
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(
-                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "50",
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "20",
                  "-i", str(self.dev)], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.first = threading.Event()
             self.thread = threading.Thread(target=self._read, daemon=True)
@@ -143,7 +143,7 @@ class ClockSampler:
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.perf_counter(), line.strip()))
             self.first.set()
 
     def __exit__(self, *exc):
@@ -155,13 +155,16 @@ class ClockSampler:
                 self.proc.kill()
             self.thread.join(timeout=5)
 
-    def summary(self):
-        if self.error or not self.lines:
+    def summary(self, t0=None, t1=None):
+        """Median SM clock, maximum clock, power and throttle reasons of the
+        samples taken between host times t0 and t1 (all samples by default)."""
+        lines = [ln for t, ln in self.lines if (t0 is None or t >= t0) and (t1 is None or t <= t1)]
+        if self.error or not lines:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0,
                     "note": self.error or "no nvidia-smi samples"}
         sm, smax, power, reasons = [], [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for ln in self.lines:
+        for ln in lines:
             parts = [p.strip() for p in ln.split(",")]
             if len(parts) < 9:
                 continue
@@ -194,10 +197,9 @@ class GpuStep:
         dt = torch.bfloat16 if w.x_dtype == "bf16" else torch.float32
         self.sites = []
         for i, (name, K, rotate, layers) in enumerate(sites(w)):
-            x = W.activations(T, K, seed=seed_base + 10 + i, dist=w.dist, n_out=w.n_out, mult=w.mult)
-            host = torch.from_numpy(x).to(dt).pin_memory()
-            dev = host.to(device)
-            dev_alt = host.to(device)  # end-to-end steps alternate between two input buffers
+            dev = device_activations(T, K, w, seed=seed_base + 10 + i, device=device).to(dt)
+            host = dev.cpu().pin_memory()
+            dev_alt = dev.clone()  # end-to-end steps alternate between two input buffers
             g = W.block_for(K)
             codes = torch.empty((Q.padded_rows(T), K // 2), dtype=torch.uint8, device=device)
             scale = torch.empty((T,), dtype=torch.float32, device=device)
@@ -205,8 +207,9 @@ class GpuStep:
             flags = (Q.OFFQ_ROTATE if rotate else 0) | Q.OFFQ_OFFSET
             gemms = []
             for l in layers:
-                wt = torch.from_numpy(W.weights(l.N, l.K, seed=seed_base + 100 + len(self.sites) * 10 + len(gemms)))
-                wc, ws, wr = Q.prepare_weight(wt.to(device), g, rotate=l.rotate)
+                wt = device_weights(l.N, l.K, seed=seed_base + 100 + len(self.sites) * 10 + len(gemms), device=device)
+                wc, ws, wr = Q.prepare_weight(wt, g, rotate=l.rotate)
+                del wt
                 out = torch.empty((T, l.N), dtype=torch.bfloat16, device=device)
                 gemms.append({"layer": l, "codes": wc, "scale": ws, "rowsum": wr, "out": out})
             self.sites.append({"name": name, "K": K, "g": g, "flags": flags, "host": host, "dev": dev,
@@ -314,14 +317,14 @@ class GroupStep:
         dt = torch.bfloat16 if w.x_dtype == "bf16" else torch.float32
         self.sites = []
         for i, (name, K, rotate, layers) in enumerate(sites(w)):
-            x = torch.from_numpy(W.activations(T, K, seed=seed_base + 10 + i, dist=w.dist, n_out=w.n_out,
-                                               mult=w.mult)).to(dt).to(device)
+            x = device_activations(T, K, w, seed=seed_base + 10 + i, device=device).to(dt)
             g = W.block_for(K)
             G = K // Q.GROUP
             gemms = []
             for l in layers:
-                wt = torch.from_numpy(W.weights(l.N, l.K, seed=seed_base + 100 + len(self.sites) * 10 + len(gemms)))
-                wc, ws, _ = Q.prepare_weight(wt.to(device), g, rotate=l.rotate)
+                wt = device_weights(l.N, l.K, seed=seed_base + 100 + len(self.sites) * 10 + len(gemms), device=device)
+                wc, ws, _ = Q.prepare_weight(wt, g, rotate=l.rotate)
+                del wt
                 gemms.append({"layer": l, "codes": wc, "scale": ws, "gsum": Q.weight_group_sums(wc, l.N, l.K),
                               "out": torch.empty((T, l.N), dtype=torch.bfloat16, device=device)})
             self.sites.append({"K": K, "g": g, "flags": Q.OFFQ_ROTATE if rotate else 0, "x": x,
@@ -520,6 +523,14 @@ def time_builder(device, args, flush_l2, stream):
         "roofline": {"bound": "hbm", "kernel": "top1_scan_kernel", "achieved": round(tok_gbs, 1),
                      "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": round(tok_gbs / peaks["hbm_gbs"], 4)},
     }
+
+
+def device_weights(N: int, K: int, seed: int, device, std: float = 0.02):
+    """Weights W [N, K] ~ N(0, std^2) in fp32, drawn on the device (seeded): the
+    recipe of workloads.weights, for timing (the 70B layers hold 0.86 G weights)."""
+    import torch
+    gen = torch.Generator(device=device).manual_seed(seed)
+    return torch.randn((N, K), generator=gen, device=device) * std
 
 
 def device_activations(T: int, K: int, w: W.Workload, seed: int, device):
@@ -735,15 +746,17 @@ def run_gpu(args, rank, world, local_rank):
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     barrier()
     torch.cuda.synchronize(device)
-    with ClockSampler(device.index if device.index is not None else 0) as clk:
-        wall0 = time.perf_counter()
-        for i in range(args.steps):
-            flush_l2()
-            starts[i].record(stream)
-            step.run(stream)
-            ends[i].record(stream)
-        torch.cuda.synchronize(device)
-        wall1 = time.perf_counter()
+    # The sampler runs through the timed region and the per-call phase that the
+    # roofline's kernel times come from; each window is summarised on its own.
+    clk = ClockSampler(device.index if device.index is not None else 0).__enter__()
+    wall0 = time.perf_counter()
+    for i in range(args.steps):
+        flush_l2()
+        starts[i].record(stream)
+        step.run(stream)
+        ends[i].record(stream)
+    torch.cuda.synchronize(device)
+    wall1 = time.perf_counter()
     barrier()
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     dev_ms = sum(step_ms)
@@ -751,10 +764,13 @@ def run_gpu(args, rank, world, local_rank):
     # ---- per-kernel durations: the same steps again, an event pair around every call ----
     timers = {}
     kb = max(1, min(args.steps, 50))
+    wall2 = time.perf_counter()
     for _ in range(kb):
         flush_l2()
         step.run(stream, timers=timers)
     torch.cuda.synchronize(device)
+    wall3 = time.perf_counter()
+    clk.__exit__(None, None, None)
     gemm_ms = sum(_pair_times(timers["gemm"])) * args.steps / kb
     quant_ms = sum(_pair_times(timers["quant"])) * args.steps / kb
     kv_ms = sum(_pair_times(timers.get("kv4", []))) * args.steps / kb if timers.get("kv4") else 0.0
@@ -783,7 +799,9 @@ def run_gpu(args, rank, world, local_rank):
     e2e_value = job_tops(ops, world, e2e_ms)
 
     peaks = load_peaks()
-    fp8_peak = peaks["bf16_tflops_sustained"] * FP8_PER_BF16
+    # The GEMMs are timed per call (an event pair around each launch), so the
+    # burst rate is their denominator.
+    fp8_peak = peaks["bf16_tflops"] * FP8_PER_BF16
     group = None
     if not args.no_group:
         gstep, g_ms, g_gemm_ms, g_quant_ms = time_group_path(w, T, device, args, rank, flush_l2, barrier, stream,
@@ -824,8 +842,8 @@ def run_gpu(args, rank, world, local_rank):
         "roofline": {"bound": "tensor", "kernel": "w4a4_gemm_kernel (tcgen05.mma kind::f8f6f4)",
                      "achieved": round(gemm_tflops, 2), "peak": round(fp8_peak, 1), "unit": "TFLOP/s",
                      "frac": round(gemm_tflops / fp8_peak, 4),
-                     "peak_source": f"{peaks['source']}: bf16 sustained {peaks['bf16_tflops_sustained']} "
-                                    f"x nominal fp8/bf16 ratio {FP8_PER_BF16}",
+                     "peak_source": f"{peaks['source']}: bf16 burst {peaks['bf16_tflops']} "
+                                    f"x nominal fp8/bf16 ratio {FP8_PER_BF16} (the GEMMs are timed per call)",
                      "traffic": traffic["bytes_per_launch"] if traffic else None,
                      "traffic_note": traffic.get("note") if traffic else "no ncu record for this gemm.cu",
                      "gemm_ms_per_step": round(gemm_ms / args.steps, 4)},
@@ -841,7 +859,8 @@ def run_gpu(args, rank, world, local_rank):
         "gpu_launches": step.launches_per_step() * args.steps,
         "kernel_timing": f"per-launch durations from {kb} more flushed steps with an event pair around every call",
         "wall_s_timed_region": round(wall1 - wall0, 4),
-        "clocks": clk.summary(),
+        "clocks": clk.summary(wall0, wall1),
+        "clocks_kernel_timing": clk.summary(wall2, wall3),
     }
     if group is not None:
         line["group_asym"] = group
@@ -955,9 +974,9 @@ def run_reference(args, rank, world):
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=10)
-    ap.add_argument("--workload", default="llama2_7b")
+    ap.add_argument("--workload", default="llama2_70b")
     ap.add_argument("--impl", default="offq", choices=["offq", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-group", action="store_true", help="skip the per-group asymmetric path's timing")

@@ -153,6 +153,10 @@ int offq_quantize_act(const void* x, int x_dtype, int64_t T, int64_t K, int64_t 
  * and rounded once to the output type.
  *
  *   a_codes   device, tiled activation codes of T rows (offq_quantize_act), 16-B aligned.
+ *             The buffer holds ceil(T/32)*32 rows. Rows T .. ceil(T/32)*32-1 may
+ *             hold anything: they are read as operands (every nibble is a
+ *             finite fp8 value), but the output rows they feed are never
+ *             written, nor do they reach acc_debug.
  *   a_scale   device, [T] float32.
  *   a_offset  device, [T][K/g] float32, or NULL for all-zero offsets.
  *   T, N, K   tokens, output channels, input channels; T >= 0, N >= 1,

@@ -565,32 +565,18 @@ GROUP = 128  # activation group size of the evaluated setting (Sec. 4)
 UMAX = 15    # largest code of Eq. 1's unsigned grid for b = 4
 
 
-def quantize_groups_asym(y: np.ndarray, group: int, fp32: bool = False):
+def quantize_groups_asym(y: np.ndarray, group: int):
     """Eq. 1 with a zero-point for every group of ``group`` channels of each row.
 
     Returns q (int64 [T, K], in [0, 15]), s (float64 [T, K/group]) and z
-    (float64, integer-valued, [T, K/group]).
-
-    With ``fp32`` the same formula is evaluated in IEEE single precision, the
-    precision the kernels decide codes in (the paper fixes none): y rounded to
-    fp32, s = fl(fl(max - min) / 15), z = -rne(fl(min / s)), and
-    q = clamp(rne(fl(y * fl(1 / s))) + z, 0, 15).
+    (float64, integer-valued, [T, K/group]). The decisions are taken in
+    float64: z = -rne(min / s) and q = clamp(rne(y / s) + z, 0, 15), with the
+    division Eq. 1 writes.
     """
     y = np.asarray(y, dtype=np.float64)
     T, K = y.shape
     if K % group != 0:
         raise ValueError("group must divide K")
-    if fp32:
-        yg = y.astype(np.float32).reshape(T, K // group, group)
-        mn, mx = yg.min(axis=2), yg.max(axis=2)
-        s = (mx - mn) / np.float32(UMAX)
-        z = np.zeros_like(s)
-        q = np.zeros(yg.shape, dtype=np.int64)
-        nz = s > 0
-        inv = np.float32(1.0) / s[nz]
-        z[nz] = -np.rint(mn[nz] / s[nz])
-        q[nz] = np.clip(np.rint(yg[nz] * inv[:, None]) + z[nz][:, None], 0, UMAX).astype(np.int64)
-        return q.reshape(T, K), s.astype(np.float64), z.astype(np.float64)
     yg = y.reshape(T, K // group, group)
     mn, mx = yg.min(axis=2), yg.max(axis=2)
     s = (mx - mn) / UMAX
@@ -613,8 +599,7 @@ def pack_unsigned_codes(q: np.ndarray) -> np.ndarray:
     return (u[..., 0::2] | (u[..., 1::2] << 4)).astype(np.uint8)
 
 
-def quantize_act_group(x: np.ndarray, g: int, group: int = GROUP, rotate: bool = True,
-                       fp32: bool = False) -> Dict[str, np.ndarray]:
+def quantize_act_group(x: np.ndarray, g: int, group: int = GROUP, rotate: bool = True) -> Dict[str, np.ndarray]:
     """Rotate -> per-group asymmetric quantize -> pack one batch of token rows X [T, K].
 
     Steps, in the paper's order:
@@ -624,8 +609,7 @@ def quantize_act_group(x: np.ndarray, g: int, group: int = GROUP, rotate: bool =
 
     As in :func:`quantize_act`, the codes are taken from the unnormalised
     product X H (y / s is the same ratio), so the decisions see no 1/sqrt(g)
-    rounding. ``fp32`` takes the decisions in single precision
-    (:func:`quantize_groups_asym`); the transform stays float64.
+    rounding.
     """
     x = np.asarray(x, dtype=np.float64)
     T, K = x.shape
@@ -641,7 +625,7 @@ def quantize_act_group(x: np.ndarray, g: int, group: int = GROUP, rotate: bool =
     else:
         yu = x.copy()
         norm = 1.0
-    q, su, z = quantize_groups_asym(yu, group, fp32=fp32)
+    q, su, z = quantize_groups_asym(yu, group)
     return {"y": yu / norm, "q": q, "scale": su / norm, "zero": z, "codes": pack_unsigned_codes(q)}
 
 

@@ -10,9 +10,8 @@ namespace {
 // bounded wait runs out; offq_get_device_status reads and clears it.
 __device__ int g_device_status = 0;
 
-constexpr int kMaxDevices = 64;
 std::mutex g_mu;
-int* g_status_ptr[kMaxDevices] = {};
+int* g_status_ptr[offq::kMaxDevices] = {};
 
 }  // namespace
 

@@ -642,12 +642,7 @@ int launch_gemm(const GemmParams& p, cudaStream_t s) {
   auto kern = w4a4_gemm_kernel<OUT, kOneBlock>;
   constexpr int kThreads = Roles<kOneBlock>::kThreads;
   constexpr int kSmemBytes = Smem<kOneBlock>::kBytes;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [&] {
-    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-  });
-  if (attr_err != cudaSuccess) return OFFQ_ERR_CUDA;
+  if (!smem_optin<w4a4_gemm_kernel<OUT, kOneBlock>>(kSmemBytes)) return OFFQ_ERR_CUDA;
   const int sms = num_sms();
   if (sms < 2) return OFFQ_ERR_CUDA;
   const int tiles = p.m_pairs * p.n_tiles;

@@ -508,12 +508,7 @@ int group_num_sms() {
 template <int OUT>
 int launch_group_gemm(const GroupParams& p, cudaStream_t s) {
   auto kern = w4a4_group_gemm_kernel<OUT>;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [&] {
-    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kGBytes);
-  });
-  if (attr_err != cudaSuccess) return OFFQ_ERR_CUDA;
+  if (!smem_optin<w4a4_group_gemm_kernel<OUT>>(kGBytes)) return OFFQ_ERR_CUDA;
   const int sms = group_num_sms();
   if (sms < 2) return OFFQ_ERR_CUDA;
   const int tiles = p.m_pairs * p.n_tiles;

@@ -789,12 +789,7 @@ int rot_num_sms() {
 template <typename Tin, int OUT>
 int launch_rotate(const RotArgs& a, cudaStream_t s) {
   auto kern = rotate_heads_kernel<Tin, OUT>;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [&] {
-    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kRotSmem);
-  });
-  if (attr_err != cudaSuccess) return OFFQ_ERR_CUDA;
+  if (!smem_optin<rotate_heads_kernel<Tin, OUT>>(kRotSmem)) return OFFQ_ERR_CUDA;
   // About two CTAs per SM (the shared-memory limit), spread over the heads;
   // each loops over its head's token tiles.
   const int sms = rot_num_sms();
@@ -842,12 +837,7 @@ template <int OUT, bool REFLECT = false>
 int launch_rotate_mma(const RotArgs& a, cudaStream_t s) {
   using L = RotLayout<REFLECT>;
   auto kern = rotate_heads_mma_kernel<OUT, REFLECT>;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [&] {
-    attr_err = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, L::kSmem);
-  });
-  if (attr_err != cudaSuccess) return OFFQ_ERR_CUDA;
+  if (!smem_optin<rotate_heads_mma_kernel<OUT, REFLECT>>(L::kSmem)) return OFFQ_ERR_CUDA;
   CUtensorMap xmap, omap;
   if (encode_heads_map(&xmap, a.x, OFFQ_BF16, a.T, a.H, a.ld_token) != OFFQ_OK) return OFFQ_ERR_CUDA;
   if constexpr (OUT != OFFQ_F32) {

@@ -1,7 +1,9 @@
 // Host-side helpers shared by the OffQ translation units (not part of the ABI).
 #pragma once
 
+#include <atomic>
 #include <cstdint>
+#include <mutex>
 #include <utility>
 #include <cuda_runtime.h>
 
@@ -49,6 +51,28 @@ inline int launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...) == cudaSuccess ? OFFQ_OK : OFFQ_ERR_CUDA;
+}
+
+constexpr int kMaxDevices = 64;
+
+// Opts kKernel in to `bytes` of dynamic shared memory on the current device.
+// The attribute belongs to the device's context, so it is set once per device
+// (not once per process): a process that launches on a second GPU sets it
+// there too. Returns false if the device query or the attribute call failed.
+template <auto kKernel>
+inline bool smem_optin(int bytes) {
+  static std::atomic<bool> done[kMaxDevices] = {};
+  static std::mutex mu;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return false;
+  if (done[dev].load(std::memory_order_acquire)) return true;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!done[dev].load(std::memory_order_relaxed)) {
+    if (cudaFuncSetAttribute(kKernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) != cudaSuccess)
+      return false;
+    done[dev].store(true, std::memory_order_release);
+  }
+  return true;
 }
 
 // Largest input dimension the row quantizer stages in shared memory.

@@ -193,3 +193,46 @@ def test_llama2_70b_down_shape_sampled():
     """K = 28672 in 28 offset blocks of 1024, 6 outliers at 200x (1024 tokens, 1024 outputs)."""
     rows = W.unit_index_sample(1024, 64, seed=7)
     _check_layer(1024, 28672, 1024, 1024, "bf16", rows=rows, n_out=6, mult=200.0)
+
+
+def _check_config_layer(T, K, N, g, rows, dist, n_out, mult, seed):
+    """A launch at a configuration's own shape (the bench's q/k/v/o/gate/up sites:
+    codes made without the online rotation), checked on sampled token rows
+    against all N outputs; only the sampled rows leave the device."""
+    x = W.activations(T, K, seed=seed, dist=dist, n_out=n_out, mult=mult)
+    gen = torch.Generator(device="cuda").manual_seed(seed + 1)
+    w = torch.randn((N, K), generator=gen, device="cuda") * 0.02
+    a_codes, a_scale, a_off = Q.quantize_act(torch.from_numpy(x).to(torch.bfloat16).cuda(), g, rotate=False,
+                                             offset=True)
+    w_codes, w_scale, rowsum = Q.prepare_weight(w, g, rotate=False)
+    del w
+    out = torch.full((T, N), float("nan"), dtype=torch.bfloat16, device="cuda")
+    acc = torch.zeros((T, N), dtype=torch.int32, device="cuda")
+    Q.offq_w4a4_linear(a_codes, a_scale, a_off, T, N, K, g, w_codes, w_scale, rowsum, out, N, acc)
+    torch.cuda.synchronize()
+    assert Q.offq_get_device_status() == Q.OFFQ_OK
+    sel = torch.from_numpy(rows).cuda()
+    y = out.index_select(0, sel).float().cpu().numpy().astype(np.float64)
+    acc_s = acc.index_select(0, sel).cpu().numpy()
+    del out, acc
+    qa = act_q(a_codes, T, K)[rows]
+    qw = weight_q(w_codes, N, K)
+    sa = a_scale.cpu().numpy().astype(np.float64)[rows]
+    oa = a_off.cpu().numpy().astype(np.float64)[rows]
+    sw = w_scale.cpu().numpy().astype(np.float64)
+    R = rowsum.cpu().numpy().astype(np.float64)
+    acc_ref = O.int_gemm(qa + 8, qw)
+    np.testing.assert_array_equal(acc_s, acc_ref)
+    y_ref = O.epilogue(O.int_gemm(qa, qw), sa, oa, sw, R)
+    check_outputs(y, y_ref, epilogue_terms(acc_ref, sa, oa, sw, R), K // g, "bf16")
+
+
+@pytest.mark.parametrize("T,K,N,g,nrows,dist,n_out,mult", [
+    (2048, 8192, 8192, 8192, 48, "normal", 6, 200.0),       # Llama-2-70B q / o: one offset block of 8192
+    (8192, 8192, 1024, 8192, 96, "normal", 6, 200.0),       # Llama-2-70B k / v (8 KV heads x 128), full prefill
+    (2048, 8192, 28672, 8192, 32, "normal", 6, 200.0),      # Llama-2-70B gate / up: 112 output tiles
+    (4096, 4096, 14336, 4096, 48, "student_t3", 3, 100.0),  # Llama-3-8B gate / up
+])
+def test_config_gemm_shapes_sampled(T, K, N, g, nrows, dist, n_out, mult):
+    rows = np.unique(np.concatenate([W.unit_index_sample(T, nrows, seed=N % 97), [0, T - 1]]))
+    _check_config_layer(T, K, N, g, rows, dist, n_out, mult, seed=K + N)

@@ -81,6 +81,22 @@ def test_quantize_workload_shapes(T, K, g, dist):
     _quant_and_check(_host(x, "bf16"), g, True, True)
 
 
+def _device_rows(T, K, dist, n_out, mult, seed):
+    """A full prefill input drawn on the host from the workload recipe, bf16."""
+    return _host(W.activations(T, K, seed=seed, dist=dist, n_out=n_out, mult=mult), "bf16")
+
+
+@pytest.mark.parametrize("T,K,g,rotate,dist,n_out,mult", [
+    (8192, 8192, 8192, False, "normal", 6, 200.0),       # Llama-2-70B attention / MLP input
+    (8192, 28672, 1024, True, "normal", 6, 200.0),       # Llama-2-70B down-proj input, 28 blocks
+    (4096, 14336, 1024, True, "student_t3", 3, 100.0),   # Llama-3-8B down-proj input, 14 blocks
+])
+def test_quantize_config_sites_sampled(T, K, g, rotate, dist, n_out, mult):
+    """The bench's prefill launches at full size, checked on sampled rows (first and last included)."""
+    rows = np.unique(np.concatenate([W.unit_index_sample(T, 96, seed=K % 89), [0, T - 1]]))
+    _quant_and_check(_device_rows(T, K, dist, n_out, mult, seed=K + 3), g, rotate, True, rows=rows)
+
+
 @pytest.mark.parametrize("K,dt", [(1024, "bf16"), (4096, "bf16"), (4096, "f16"), (4096, "f32"), (8192, "bf16"),
                                   (8192, "f32")])
 @pytest.mark.parametrize("offset", [True, False])
@@ -203,6 +219,26 @@ def test_kv4_against_oracle(T, H, flags):
     x64 = kvh.to(torch.float64).numpy().reshape(T * H, hd)
     check_scales(scale.cpu().numpy().reshape(-1), ref["scale"].reshape(-1), x64, hd, rotate)
     check_offsets(off.cpu().numpy().reshape(-1, 1), ref["offset"].reshape(-1, 1), x64, hd, rotate)
+
+
+def test_kv4_llama2_70b_prefill():
+    """KV4 of the Llama-2-70B keys and values at prefill size: 8192 tokens x 8 heads x 128, every
+    (token, head) checked, with and without the per-head Hadamard."""
+    T, H, hd = 8192, 8, 128
+    kv = W.kv_heads(T, H, hd, seed=81)
+    kvh = _host(kv.reshape(T, H * hd), "bf16").reshape(T, H, hd)
+    x64 = kvh.to(torch.float64).numpy()
+    for rotate in (True, False):
+        codes, scale, off = Q.kv4_quantize(kvh.cuda(), rotate=rotate, offset=True)
+        torch.cuda.synchronize()
+        assert Q.offq_get_device_status() == Q.OFFQ_OK
+        ref = O.kv4_quantize(x64, rotate=rotate, offset=True)
+        q = O.unpack_act_codes(codes.cpu().numpy())
+        check_codes(q.reshape(T * H, hd), ref["q"].reshape(T * H, hd), ref["residual"].reshape(T * H, hd),
+                    ref["scale"].reshape(T * H))
+        check_scales(scale.cpu().numpy().reshape(-1), ref["scale"].reshape(-1), x64.reshape(T * H, hd), hd, rotate)
+        check_offsets(off.cpu().numpy().reshape(-1, 1), ref["offset"].reshape(-1, 1), x64.reshape(T * H, hd), hd,
+                      rotate)
 
 
 def test_kv4_padded_token_stride():
