@@ -233,16 +233,17 @@ int offq_prepare_weight(const void* w, int dtype, int64_t N, int64_t K, int32_t 
  * then for each group j of `group` channels of y:
  *   s[j] = (max - min) / 15,  z[j] = -round_half_even(min / s[j])  (any integer),
  *   u = clamp(round_half_even(y / s[j]) + z[j], 0, 15);
- * a constant group gets s = z = u = 0. y ~ s (u - z).
+ * a constant group gets s = z = u = 0. y ~ s (u - z). The ratios y / s and
+ * min / s are taken as 15 y / (max - min) and 15 min / (max - min) in fp32 (s
+ * is not rounded first), so exact half-integer ratios round half to even.
  *
  *   x       device, [T][ldx] elements of x_dtype, row-major; 16-byte aligned,
  *           ldx * sizeof(elem) a multiple of 16, ldx >= K.
  *   T       token rows, >= 0 (T = 0 launches nothing).
  *   K       channels, a multiple of `group` (and of g with the rotation),
  *           K <= 65536.
- *   g       rotation block (power of two in [32, 8192]; this build rotates
- *           blocks of at most 512 and returns OFFQ_ERR_UNSUPPORTED above);
- *           ignored without OFFQ_ROTATE.
+ *   g       rotation block, power of two in [32, 8192]; ignored without
+ *           OFFQ_ROTATE.
  *   group   channels per quantization group; this build supports 128
  *           (OFFQ_ERR_UNSUPPORTED for other positive values).
  *   flags   0 or OFFQ_ROTATE.

@@ -570,8 +570,15 @@ def quantize_groups_asym(y: np.ndarray, group: int):
 
     Returns q (int64 [T, K], in [0, 15]), s (float64 [T, K/group]) and z
     (float64, integer-valued, [T, K/group]). The decisions are taken in
-    float64: z = -rne(min / s) and q = clamp(rne(y / s) + z, 0, 15), with the
-    division Eq. 1 writes.
+    float64: z = -rne(min / s) and q = clamp(rne(y / s) + z, 0, 15).
+
+    The ratio y / s of Eq. 1, with s = (max - min) / 15, is the real number
+    15 y / (max - min); it is evaluated in that form, so s is not rounded
+    before the division. For values of bf16, f16 or f32 inputs (and their
+    float64 Hadamard transforms) 15 y and max - min are exact in float64, so a
+    ratio that is exactly a half-integer is seen as one and rounds half to
+    even. Such ties are frequent: on a bf16 grid max - min and y share few
+    significant bits.
     """
     y = np.asarray(y, dtype=np.float64)
     T, K = y.shape
@@ -579,12 +586,13 @@ def quantize_groups_asym(y: np.ndarray, group: int):
         raise ValueError("group must divide K")
     yg = y.reshape(T, K // group, group)
     mn, mx = yg.min(axis=2), yg.max(axis=2)
-    s = (mx - mn) / UMAX
+    rng = mx - mn
+    s = rng / UMAX
     z = np.zeros_like(s)
     q = np.zeros(yg.shape, dtype=np.int64)
-    nz = s > 0
-    z[nz] = -np.rint(mn[nz] / s[nz])
-    q[nz] = np.clip(np.rint(yg[nz] / s[nz][:, None]) + z[nz][:, None], 0, UMAX).astype(np.int64)
+    nz = rng > 0
+    z[nz] = -np.rint(UMAX * mn[nz] / rng[nz])
+    q[nz] = np.clip(np.rint(UMAX * yg[nz] / rng[nz][:, None]) + z[nz][:, None], 0, UMAX).astype(np.int64)
     return q.reshape(T, K), s, z
 
 

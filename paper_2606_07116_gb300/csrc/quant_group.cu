@@ -9,11 +9,17 @@
 // group gets s = 0, z = 0, u = 0.
 //
 // One warp takes one 512-channel chunk of a row: lane l holds 16 consecutive
-// channels, a group is 8 lanes. With the rotation on (block g <= 512, a power
-// of two) the Sylvester transform runs in place: index bits 0-3 inside the
-// lane, bits 4.. across lanes (shuffle partner l ^ 2^(b-4)); the codes are
-// decided on the unnormalised transform (y / s is the same ratio) and only the
-// stored scale carries the 1/sqrt(g).
+// channels, a group is 8 lanes. With the rotation on (block g a power of two)
+// the Sylvester transform runs in place: index bits 0-3 inside the lane, bits
+// 4-8 across lanes (shuffle partner l ^ 2^(b-4)), and for g >= 1024 bits 9..
+// across the warps of the CTA, which holds whole blocks (a shared-memory
+// exchange per bit). The codes are decided on the unnormalised transform
+// (y / s is the same ratio) and only the stored scale carries the 1/sqrt(g).
+//
+// Eq. 1's y / s is evaluated as 15 y / (max - min), the same real number
+// without s rounded first: for bf16 / f16 inputs 15 y and max - min are exact
+// in fp32, so a ratio that is exactly a half-integer (frequent on those
+// grids) stays one and rounds half to even; so does -min / s for z.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -30,7 +36,8 @@ using namespace offq;
 constexpr int kQGroup = 128;
 constexpr int kChunk = 512;          // channels per warp
 constexpr int kPerLane = kChunk / 32;  // 16
-constexpr int kQWarps = 8;
+constexpr int kQWarps = 8;           // warps per CTA for blocks up to 4096 (16 for 8192)
+constexpr int kMaxQWarps = 16;
 
 struct GroupQuantArgs {
   const void* x;
@@ -78,17 +85,26 @@ __device__ __forceinline__ void load16(const Tin* src, float (&v)[kPerLane]) {
 }
 
 template <typename Tin>
-__global__ void __launch_bounds__(kQWarps * 32) quantize_group_kernel(const GroupQuantArgs a) {
+__global__ void __launch_bounds__(kMaxQWarps * 32) quantize_group_kernel(const GroupQuantArgs a) {
+  extern __shared__ float xchg[];  // cross-warp stages: [warps][512]
   griddep_wait();
   griddep_launch_dependents();
   const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  const int warps = blockDim.x >> 5;
   const int chunks = (a.K + kChunk - 1) / kChunk;
-  const int64_t item = static_cast<int64_t>(blockIdx.x) * kQWarps + (threadIdx.x >> 5);
-  if (item >= a.T * chunks) return;  // warp-uniform
-  const int64_t row = item / chunks;
-  const int ch = static_cast<int>(item - row * chunks);
+  const int64_t item = static_cast<int64_t>(blockIdx.x) * warps + warp;
+  // Blocks of g >= 1024 span g / 512 warps of one CTA: every warp takes part in
+  // the exchange barriers, so none returns early then. (A CTA's first item and
+  // a row's chunk count are multiples of g / 512, so a block never straddles
+  // CTAs, and an item past the end lies in a block with no valid item.)
+  const bool cross = a.log2g > 9;
+  const bool valid = item < a.T * chunks;
+  if (!valid && !cross) return;  // warp-uniform
+  const int64_t row = valid ? item / chunks : 0;
+  const int ch = valid ? static_cast<int>(item - row * chunks) : 0;
   const int c0 = ch * kChunk + lane * kPerLane;
-  const bool active = c0 < a.K;  // uniform over each 8-lane group (K % 128 == 0)
+  const bool active = valid && c0 < a.K;  // uniform over each 8-lane group (K % 128 == 0)
 
   float v[kPerLane];
   if (active) {
@@ -114,7 +130,8 @@ __global__ void __launch_bounds__(kQWarps * 32) quantize_group_kernel(const Grou
         }
       }
     }
-    for (int b = 4; b < a.log2g; ++b) {
+    const int lane_bits = a.log2g < 9 ? a.log2g : 9;
+    for (int b = 4; b < lane_bits; ++b) {
       const int m = 1 << (b - 4);
       const bool upper = (lane & m) != 0;
 #pragma unroll
@@ -122,6 +139,23 @@ __global__ void __launch_bounds__(kQWarps * 32) quantize_group_kernel(const Grou
         const float o = __shfl_xor_sync(0xFFFFFFFFu, v[i], m);
         v[i] = upper ? o - v[i] : v[i] + o;
       }
+    }
+    // Bits 9.. of the block index: the partner warp is warp ^ 2^(b-9), through
+    // shared memory (element i of lane l of warp w at w*512 + i*32 + l).
+    for (int b = 9; b < a.log2g; ++b) {
+      const int m = 1 << (b - 9);
+      const bool upper = (warp & m) != 0;
+      float* mine = xchg + warp * kChunk + lane;
+      const float* theirs = xchg + (warp ^ m) * kChunk + lane;
+#pragma unroll
+      for (int i = 0; i < kPerLane; ++i) mine[i * 32] = v[i];
+      __syncthreads();
+#pragma unroll
+      for (int i = 0; i < kPerLane; ++i) {
+        const float o = theirs[i * 32];
+        v[i] = upper ? o - v[i] : v[i] + o;
+      }
+      __syncthreads();
     }
   }
 
@@ -137,16 +171,15 @@ __global__ void __launch_bounds__(kQWarps * 32) quantize_group_kernel(const Grou
     mn = fminf(mn, __shfl_xor_sync(0xFFFFFFFFu, mn, m));
     mx = fmaxf(mx, __shfl_xor_sync(0xFFFFFFFFu, mx, m));
   }
-  const float su = __fdiv_rn(mx - mn, 15.0f);
-  float inv = 0.f, z = 0.f;
-  if (su > 0.f) {
-    inv = __frcp_rn(su);
-    z = -rintf(__fdiv_rn(mn, su));
-  }
+  // s = range / 15; the decisions take y / s as 15 y / range (one rounding).
+  const float range = mx - mn;
+  const float su = __fdiv_rn(range, 15.0f);
+  float z = 0.f;
+  if (su > 0.f) z = -rintf(__fdiv_rn(15.0f * mn, range));
   uint32_t packed[2] = {0u, 0u};
 #pragma unroll
   for (int i = 0; i < kPerLane; ++i) {
-    const float q = su > 0.f ? fminf(fmaxf(rintf(v[i] * inv) + z, 0.f), 15.f) : 0.f;
+    const float q = su > 0.f ? fminf(fmaxf(rintf(__fdiv_rn(15.0f * v[i], range)) + z, 0.f), 15.f) : 0.f;
     packed[i >> 3] |= static_cast<uint32_t>(q) << (4 * (i & 7));
   }
   if (!active) return;
@@ -209,7 +242,6 @@ extern "C" int offq_quantize_act_group(const void* x, int x_dtype, int64_t T, in
   const bool rotate = (flags & OFFQ_ROTATE) != 0;
   if (rotate) {
     if (!is_pow2(g) || g < 32 || g > 8192 || K % g != 0) return OFFQ_ERR_INVALID_ARG;
-    if (g > kChunk) return OFFQ_ERR_UNSUPPORTED;
   }
   if (K > kMaxGemmK || T > 0x3FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
   if (T == 0) return OFFQ_OK;
@@ -228,12 +260,16 @@ extern "C" int offq_quantize_act_group(const void* x, int x_dtype, int64_t T, in
   a.scale = scale;
   a.zero = zero;
   const int64_t items = T * ((K + kChunk - 1) / kChunk);
-  const dim3 grid(static_cast<unsigned>((items + kQWarps - 1) / kQWarps));
+  // g >= 1024: a CTA holds whole blocks (g / 512 warps each); 16 warps for g = 8192.
+  const int warps = rotate && g > kQWarps * kChunk ? static_cast<int>(g / kChunk) : kQWarps;
+  const size_t smem = rotate && g > kChunk ? static_cast<size_t>(warps) * kChunk * sizeof(float) : 0;
+  const dim3 grid(static_cast<unsigned>((items + warps - 1) / warps));
+  const dim3 block(static_cast<unsigned>(warps * 32));
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   switch (x_dtype) {
-    case OFFQ_F32: return launch_pdl(quantize_group_kernel<float>, grid, dim3(kQWarps * 32), 0, s, a);
-    case OFFQ_BF16: return launch_pdl(quantize_group_kernel<__nv_bfloat16>, grid, dim3(kQWarps * 32), 0, s, a);
-    case OFFQ_F16: return launch_pdl(quantize_group_kernel<__half>, grid, dim3(kQWarps * 32), 0, s, a);
+    case OFFQ_F32: return launch_pdl(quantize_group_kernel<float>, grid, block, smem, s, a);
+    case OFFQ_BF16: return launch_pdl(quantize_group_kernel<__nv_bfloat16>, grid, block, smem, s, a);
+    case OFFQ_F16: return launch_pdl(quantize_group_kernel<__half>, grid, block, smem, s, a);
     default: return OFFQ_ERR_INVALID_ARG;
   }
 }

@@ -121,7 +121,7 @@ def test_group_path_argument_checks(lib):
     assert qg(group=0) == Q.OFFQ_ERR_INVALID_ARG
     assert qg(K=1000, ldx=1000) == Q.OFFQ_ERR_INVALID_ARG  # group does not divide K
     assert qg(g=100) == Q.OFFQ_ERR_INVALID_ARG             # rotation block not a power of two
-    assert qg(g=1024) == Q.OFFQ_ERR_UNSUPPORTED            # rotation blocks above 512
+    assert qg(g=2048) == Q.OFFQ_ERR_INVALID_ARG            # rotation block does not divide K
     assert qg(flags=2) == Q.OFFQ_ERR_INVALID_ARG           # no explicit offset on this path
     assert qg(ldx=1000) == Q.OFFQ_ERR_INVALID_ARG
     assert qg(z=None) == Q.OFFQ_ERR_INVALID_ARG

@@ -53,6 +53,18 @@ def test_group_quantizer_parity(in_dt, rotate, g):
     check_group_quant(q, scale.cpu().numpy(), zero.cpu().numpy(), ref, xe, g, rotate)
 
 
+@pytest.mark.parametrize("g", [1024, 2048, 4096, 8192])
+def test_group_quantizer_rotation_across_warps(g):
+    """Rotation blocks of g >= 1024 span g / 512 warps of a CTA (index bits 9.. go through shared
+    memory); 37 rows leave the last CTA with items past the end, and K = 3 g blocks for g <= 4096."""
+    T = 37
+    K = 3 * g if g <= 4096 else g
+    x = W.activations(T, K, seed=64 + g, n_out=3, mult=120.0)
+    xe, codes, scale, zero, q = _quant(x, g, True)
+    ref = O.quantize_act_group(xe, g, 128, rotate=True)
+    check_group_quant(q, scale.cpu().numpy(), zero.cpu().numpy(), ref, xe, g, True)
+
+
 def test_group_quantizer_ragged_chunk_and_offsets():
     """K = 11008 (21.5 chunks of 512) with the g = 256 rotation of the
     down-projection input, and rows with large common offsets."""

@@ -369,6 +369,28 @@ def test_group_affine_grid_is_exact():
         np.testing.assert_array_equal(O.dequantize_act_group(q, s, z, group)[0], y)
 
 
+def test_group_exact_ties_round_half_even():
+    """Values exactly half-way between two grid points of Eq. 1 round to the
+    even quotient: y / s = k + 1/2 - z0 goes to the even one of k - z0 and
+    k + 1 - z0, for every k and for steps and zero-points that are powers of
+    two, bf16-sized grids and shifted ranges alike."""
+    for s0 in (2.0 ** -3, 0.75, 1.0, 3.0, 2.0 ** 5):
+        for z0 in (-9, -1, 0, 3, 8, 21):
+            ks = np.arange(15)
+            y = s0 * np.concatenate([[0 - z0, 15 - z0], ks + 0.5 - z0])
+            q, s, z = O.quantize_groups_asym(y[None, :], y.size)
+            assert s[0, 0] == s0 and z[0, 0] == z0
+            even = (ks - z0) % 2 == 0
+            np.testing.assert_array_equal(q[0, 2:], np.where(even, ks, ks + 1))
+            assert q[0, 0] == 0 and q[0, 1] == 15
+    # A tie on the zero-point itself: min / s = -(z + 1/2) takes the even z.
+    for zt in (2.5, 3.5, -4.5):
+        mn = -zt
+        y = np.array([mn, mn + 15.0, mn + 0.25])
+        q, s, z = O.quantize_groups_asym(y[None, :], 3)
+        assert s[0, 0] == 1.0 and z[0, 0] == (np.floor(zt) if np.floor(zt) % 2 == 0 else np.ceil(zt))
+
+
 def test_group_eq5_two_channel_example(golden_dir):
     """Eq. 5's two-channel token: after H/sqrt(2) the outlier x1 is a common
     offset, so with one group of 2 the step is 2|x2| / (15 sqrt 2) whatever x1
