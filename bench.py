@@ -677,6 +677,43 @@ def time_decode(device, args, flush_l2, stream):
     return out
 
 
+def time_gemm_shape(device, args, flush_l2, stream):
+    """One offq_w4a4_linear shape alone (T, K -> N, block g; codes made without
+    the rotation unless g < K), per-call events after an L2 flush: a side
+    measurement for profiling, not the bench line."""
+    import torch
+    from paper_2606_07116_gb300 import offq as Q
+    T, K, N = (int(v) for v in args.gemm.split(",")[:3])
+    g = W.block_for(K)
+    w = workload_by_name(args.workload)
+    x = device_activations(T, K, w, seed=900, device=device)
+    codes, scale, off = Q.quantize_act(x, g, rotate=g < K, offset=True)
+    del x
+    wc, ws, wr = Q.prepare_weight(device_weights(N, K, seed=901, device=device), g, rotate=g < K)
+    y = torch.empty((T, N), dtype=torch.bfloat16, device=device)
+    reps = max(1, min(args.steps, 50))
+    ts = []
+    for r in range(args.warmup + reps):
+        flush_l2()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        Q.offq_w4a4_linear(codes, scale, off, T, N, K, g, wc, ws, wr, y, N, None, stream)
+        e1.record(stream)
+        torch.cuda.synchronize(device)
+        if r >= args.warmup:
+            ts.append(e0.elapsed_time(e1))
+    st = Q.offq_get_device_status(stream)
+    if st != Q.OFFQ_OK:
+        raise RuntimeError(f"device status after the GEMM: {Q.status_string(st)}")
+    ms = sum(ts) / len(ts)
+    peaks = load_peaks()
+    tflops = 2.0 * T * N * K / (ms * 1e-3) / 1e12
+    peak = peaks["bf16_tflops"] * FP8_PER_BF16
+    return {"gemm": {"T": T, "K": K, "N": N, "g": g}, "us": round(ms * 1e3, 2), "tflops": round(tflops, 1),
+            "peak": peak, "frac": round(tflops / peak, 4), "reps": reps}
+
+
 def _pair_times(events):
     return [events[i].elapsed_time(events[i + 1]) for i in range(0, len(events), 2)]
 
@@ -928,6 +965,7 @@ def _cores():
 def cpu_baseline(w: W.Workload, budget_s: float = 15.0):
     ostep = OracleStep(w, w.T)
     rows = W.unit_index_sample(w.T, 8, seed=1)
+    ostep.run(rows)  # the first pass warms BLAS threads and the Hadamard cache
     t0 = time.perf_counter()
     ostep.run(rows)
     per_tok = (time.perf_counter() - t0) / len(rows)
@@ -952,6 +990,9 @@ def run_reference(args, rank, world):
     t0 = time.perf_counter()
     ostep.run(probe)
     per_tok = (time.perf_counter() - t0) / len(probe)
+    t0 = time.perf_counter()
+    ostep.run(probe)  # a second probe, with BLAS threads and the Hadamard cache warm
+    per_tok = min(per_tok, (time.perf_counter() - t0) / len(probe))
     per_step_budget = max(1.0, args.ref_budget / max(1, args.steps + args.warmup))
     n = int(max(4, min(w.T, per_step_budget / max(per_tok, 1e-9))))
     rows = W.unit_index_sample(w.T, n, seed=2)
@@ -987,6 +1028,9 @@ def main():
                          "(a side measurement for profiling, not the bench line)")
     ap.add_argument("--decode", action="store_true",
                     help="time only the decode sweep (1/8/32/64 tokens) and print that object")
+    ap.add_argument("--gemm", default="",
+                    help="T,K,N: time only offq_w4a4_linear at this shape (bf16 out) and print that object "
+                         "(a side measurement for profiling, not the bench line)")
     ap.add_argument("--quant-sites", action="store_true",
                     help="time only the activation quantizer on the larger prefill inputs and print that object "
                          "(a side measurement for profiling, not the bench line)")
@@ -1006,6 +1050,20 @@ def main():
             flush[:L2_FLUSH_BYTES // 2].view(torch.int32).amax()
 
         print(json.dumps(time_decode(device, args, flush_l2, torch.cuda.current_stream(device))), flush=True)
+        return
+    if args.gemm:
+        import torch
+        import __graft_entry__ as G
+        G.build()
+        device = torch.device("cuda", 0)
+        torch.cuda.set_device(device)
+        flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=device)
+
+        def flush_l2():
+            flush.zero_()
+            flush[:L2_FLUSH_BYTES // 2].view(torch.int32).amax()
+
+        print(json.dumps(time_gemm_shape(device, args, flush_l2, torch.cuda.current_stream(device))), flush=True)
         return
     if args.quant_sites:
         import torch

@@ -1,8 +1,8 @@
 // W4A4 GEMM of the OffQ path (offq_w4a4_linear) on the 5th-generation tensor
 // cores of sm_103a, with the dequant + offset epilogue fused.
 //
-//   y[t][n] = s_w[n] * ( s_a[t] * acc'[t][n] + sum_b (o[t][b] - 8 s_a[t]) * R[b][n] )
-//   acc'[t][n] = sum_k (q_a[t][k] + 8) * q_w[n][k]
+//   y[t][n] = s_w[n] * ( s_a[t] * (acc'[t][n] - 8 Rt[n]) + sum_b o[t][b] * R[b][n] )
+//   acc'[t][n] = sum_k (q_a[t][k] + 8) * q_w[n][k],   Rt[n] = sum_b R[b][n]
 //
 // acc' is what the tensor cores accumulate: activation codes are stored as
 // u = q + 8 (1..15) and weight codes as sign-magnitude q (-7..7). Both widen to
@@ -10,8 +10,10 @@
 // the values 0..15 * 2^-9 (subnormals and the first binade share one step), and
 // the sign bit negates. Every product and partial sum is then an integer times
 // 2^-18 below 2^24 * 2^-18 for K <= 65536, exact in the fp32 accumulator. The
-// "+8" is removed in the epilogue with the weight block row sums R, together
-// with the offsets: sum_b 8 s_a R[b][n] = 8 s_a sum_k q_w[n][k].
+// "+8" is removed in the epilogue, still exactly: acc' - 8 Rt[n] is the integer
+// dot product times 2^-18, with the weight row sum Rt = sum_k q_w[n][k] (the
+// block row sums R added up). Only then is it scaled, so an output near zero
+// is not the small difference of two large rounded terms.
 //
 // Design. Widening 4-bit codes to fp8 operands costs shared-memory bandwidth,
 // which the tensor core's operand reads share. So:
@@ -114,7 +116,8 @@ struct Smem {
   static constexpr int kOffW = kOffR + kMaxG * BN * 4;
   static constexpr int kOffO = kOffW + BN * 4;
   static constexpr int kOffSa = kOffO + BM * kGp * 4;
-  static constexpr int kOffOut = kOffSa + BM * 4;  // one block: staged output rows; several: the correction half
+  static constexpr int kOffRt = kOffSa + BM * 4;    // several blocks: -8 Rt[n] 2^-18 per column
+  static constexpr int kOffOut = kOffRt + BN * 4;   // one block: staged output rows; several: the correction half
   static constexpr int kOffBars = kOffOut + (kOneBlock ? BM * kOutPitch : BM * kCorrPitch);
   static constexpr int kOffMisc = kOffBars + kNumBars * 8;
   static constexpr int kBytes = kOffMisc + 64 + 1024;  // + slack to align the base to 1024
@@ -137,6 +140,7 @@ struct GemmParams {
   int* status;
   int T, N, K, G;
   int m_pairs, n_tiles;    // pair tiles: m_pairs x n_tiles
+  int raster_m;            // m-pairs per raster group (see tile_mn)
   int t_blocks, n_blocks;  // 32-row tiles present in the code buffers
   int kchunks;             // K / 32
   int vec_ok;              // rowsum and w_scale rows are 16-byte aligned
@@ -158,22 +162,43 @@ __device__ __forceinline__ void load_kt(const uint8_t* blk, int kchunks, int kt,
   }
 }
 
+// Pair tile index -> (m-pair, n-tile). Tiles are taken in groups of raster_m
+// m-pairs; within a group the m-pair runs fastest. The clusters running at one
+// time then share a few weight tiles across all m-pairs of the group, so each
+// weight tile comes from DRAM about once per group while the group's
+// activation rows (at most ~32 MB, chosen on the host) stay in L2.
+__device__ __forceinline__ void tile_mn(const GemmParams& p, int tile, int& mp, int& nt) {
+  const int per_group = p.raster_m * p.n_tiles;
+  const int grp = tile / per_group;
+  const int local = tile - grp * per_group;
+  const int m_left = p.m_pairs - grp * p.raster_m;
+  const int gm = m_left < p.raster_m ? m_left : p.raster_m;
+  nt = local / gm;
+  mp = grp * p.raster_m + (local - nt * gm);
+}
+
 // Row block (of 32 rows) of this CTA's A rows / B rows for a pair tile.
 __device__ __forceinline__ int a_block(const GemmParams& p, int tile, uint32_t rank, int quarter) {
-  return ((tile / p.n_tiles) * 2 * BM + static_cast<int>(rank) * BM + quarter * 32) >> 5;
+  int mp, nt;
+  tile_mn(p, tile, mp, nt);
+  return (mp * 2 * BM + static_cast<int>(rank) * BM + quarter * 32) >> 5;
 }
 
 __device__ __forceinline__ int b_block(const GemmParams& p, int tile, uint32_t rank, int wb) {
-  return ((tile % p.n_tiles) * BN + static_cast<int>(rank) * BNH + wb * 32) >> 5;
+  int mp, nt;
+  tile_mn(p, tile, mp, nt);
+  return (nt * BN + static_cast<int>(rank) * BNH + wb * 32) >> 5;
 }
 
 // Persistent pair kernel: cluster c processes pair tiles c, c + clusters, ...
-// (pair tile index = m_pair * n_tiles + n_tile). The k-tile counter g runs
+// (pair tile index mapped to (m-pair, n-tile) by tile_mn). The k-tile counter g runs
 // across tiles so the stage ring never drains between tiles.
-// kOneBlock: the offsets span the whole row (G == 1). Layers with several
+// kOneBlock: the offsets span the whole row (G == 1). kUnstaged: more than
+// kMaxStageG offset blocks, whose constants are read from global memory at the
+// tile end. Layers with several
 // offset blocks run a separate instantiation, so the register allocation of
 // the common one-block kernel does not carry the G-term epilogue loop.
-template <int OUT, bool kOneBlock>
+template <int OUT, bool kOneBlock, bool kUnstaged>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kThreads, 1)
     w4a4_gemm_kernel(const GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -369,11 +394,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
     const int half = (warp - kFirstEpi) / 4;   // which kEpiCols accumulator columns
     const int et = threadIdx.x - kFirstEpi * 32;
     const int G = kOneBlock ? 1 : p.G;
-    const bool staged = kOneBlock || G <= kMaxStageG;
+    // More offset blocks than the staging area holds take their own
+    // instantiation, so its register needs stay out of the staged kernels.
+    constexpr bool staged = !kUnstaged;
     float* Rs = reinterpret_cast<float*>(smem + kOffR);
     float* Ws = reinterpret_cast<float*>(smem + kOffW);
     float* Os = reinterpret_cast<float*>(smem + kOffO);
     float* Sa = reinterpret_cast<float*>(smem + kOffSa);
+    float* Rt = reinterpret_cast<float*>(smem + SL::kOffRt);
     const uint32_t acc_empty_l = leader_addr(acc_empty);
     // Loop exit decided only from a flag the epilogue warps write before their
     // own barrier, so all eight warps leave together (bar.sync has no timeout).
@@ -382,8 +410,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
     epi_sync<kEpiWarps>();
     int lt = 0;
     for (int tile = cluster; tile < num_tiles; tile += clusters, ++lt) {
-      const int m0 = (tile / p.n_tiles) * 2 * BM + static_cast<int>(rank) * BM;
-      const int nt0 = (tile % p.n_tiles) * BN;
+      int mp, nt;
+      tile_mn(p, tile, mp, nt);
+      const int m0 = mp * 2 * BM + static_cast<int>(rank) * BM;
+      const int nt0 = nt * BN;
       // Stage this tile's constants while the main loop runs.
       if (staged) {
         for (int i = et; i < G * BN; i += kEpiWarps * 32) {
@@ -395,14 +425,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
         for (int i = et; i < BM * G; i += kEpiWarps * 32) {
           const int r = i / G, b = i - r * G, t = m0 + r;
           float v = 0.f;
-          if (t < p.T) {
-            const float o = p.a_offset != nullptr ? __ldg(p.a_offset + static_cast<int64_t>(t) * G + b) : 0.f;
-            v = o - 8.0f * __ldg(p.a_scale + t);
-          }
+          if (t < p.T && p.a_offset != nullptr) v = __ldg(p.a_offset + static_cast<int64_t>(t) * G + b);
           Os[r * kStageGp + b] = v;
         }
       }
       epi_sync<kEpiWarps>();
+      if (!kOneBlock && staged) {
+        // Rt[n] * 8 * 2^-18 = sum_b R[b][n] * 2^-15: integers, exact in fp32.
+        for (int i = et; i < BN; i += kEpiWarps * 32) {
+          float r = 0.f;
+          for (int b = 0; b < G; ++b) r += Rs[b * BN + i];
+          Rt[i] = r * -0x1p-15f;
+        }
+        epi_sync<kEpiWarps>();
+      }
       if constexpr (!kOneBlock) {
         if (staged) {
           // While this tile's MMAs run: its offset correction, per element the same
@@ -488,7 +524,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
           float z[CW];
 #pragma unroll
           for (int jj = 0; jj < CW; ++jj) {
-            const float accf = __uint_as_float(acc[jj]) * 262144.0f;  // exact: * 2^18
+            // (acc' - 8 Rt) 2^-18, then * 2^18: both steps exact.
+            const float accf = (__uint_as_float(acc[jj]) + Rt[jc + jj]) * 262144.0f;
             z[jj] = Ws[jc + jj] * fmaf(sa, accf, __uint_as_float(cr[jj]));
           }
           store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, z, nvalid);
@@ -501,12 +538,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
         }
       } else if (kOneBlock) {
         // Packed fp32 pairs; each lane rounds as y = s_w * fma(s_a, acc * 2^18, o R)
-        // does (s_a * 2^18 and its product with acc are exact). 16-bit rows go to
-        // shared memory and leave by one bulk copy per row once the accumulator is
-        // read, so the tile's output write overlaps the next tile's MMAs.
+        // does, with acc = (acc' - 8 R) 2^-18 formed exactly first (s_a * 2^18 and
+        // its product with acc are exact). 16-bit rows go to shared memory and
+        // leave by one bulk copy per row once the accumulator is read, so the
+        // tile's output write overlaps the next tile's MMAs.
         const float sa2 = Sa[rl] * 262144.0f;
         const float ob = Os[rl * kStageGp];
         const uint64_t SA2 = pack2(sa2, sa2), OB = pack2(ob, ob);
+        const uint64_t M8 = pack2(-0x1p-15f, -0x1p-15f);  // -8 * 2^-18
         const bool async_out = OUT != OFFQ_F32 && p.async_out != 0;
         const uint32_t orow_s = base + SL::kOffOut + rl * kOutPitch;
         if (async_out) bulk_wait_read_all();  // this row's previous copy has read the buffer
@@ -526,12 +565,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
 #pragma unroll
             for (int q4 = 0; q4 < CW / 4; ++q4) {
               const float4 rv = r4[q4], wv = w4[q4];
-              const uint64_t A0 = pack2(__uint_as_float(acc[4 * q4]), __uint_as_float(acc[4 * q4 + 1]));
-              const uint64_t A1 = pack2(__uint_as_float(acc[4 * q4 + 2]), __uint_as_float(acc[4 * q4 + 3]));
-              unpack2(mul2v(pack2(wv.x, wv.y), fma2v(SA2, A0, mul2v(OB, pack2(rv.x, rv.y)))), y[4 * q4],
-                      y[4 * q4 + 1]);
-              unpack2(mul2v(pack2(wv.z, wv.w), fma2v(SA2, A1, mul2v(OB, pack2(rv.z, rv.w)))), y[4 * q4 + 2],
-                      y[4 * q4 + 3]);
+              const uint64_t R0 = pack2(rv.x, rv.y), R1 = pack2(rv.z, rv.w);
+              const uint64_t A0 =
+                  fma2v(R0, M8, pack2(__uint_as_float(acc[4 * q4]), __uint_as_float(acc[4 * q4 + 1])));
+              const uint64_t A1 =
+                  fma2v(R1, M8, pack2(__uint_as_float(acc[4 * q4 + 2]), __uint_as_float(acc[4 * q4 + 3])));
+              unpack2(mul2v(pack2(wv.x, wv.y), fma2v(SA2, A0, mul2v(OB, R0))), y[4 * q4], y[4 * q4 + 1]);
+              unpack2(mul2v(pack2(wv.z, wv.w), fma2v(SA2, A1, mul2v(OB, R1))), y[4 * q4 + 2], y[4 * q4 + 3]);
             }
             if (async_out) {
               uint32_t hv[CW / 2];
@@ -577,19 +617,26 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
           const int nb = n0 + c * CW;
           if (!row_ok || nb >= p.N) continue;
           const int nvalid = p.N - nb < CW ? p.N - nb : CW;
-          float y[CW];
+          float y[CW], a[CW];
 #pragma unroll
-          for (int jj = 0; jj < CW; ++jj) y[jj] = 0.f;
+          for (int jj = 0; jj < CW; ++jj) {
+            y[jj] = 0.f;
+            a[jj] = __uint_as_float(acc[jj]);
+          }
           for (int b = 0; b < G; ++b) {
-            const float ob = (has_off ? __ldg(orow + b) : 0.f) - 8.0f * sa;
+            const float ob = has_off ? __ldg(orow + b) : 0.f;
             const float* rb = p.rowsum + static_cast<int64_t>(b) * p.N + nb;
 #pragma unroll
             for (int jj = 0; jj < CW; ++jj)
-              if (jj < nvalid) y[jj] = fmaf(ob, __ldg(rb + jj), y[jj]);
+              if (jj < nvalid) {
+                const float r = __ldg(rb + jj);
+                y[jj] = fmaf(ob, r, y[jj]);
+                a[jj] = fmaf(r, -0x1p-15f, a[jj]);  // acc' - 8 R, in units of 2^-18: exact
+              }
           }
 #pragma unroll
           for (int jj = 0; jj < CW; ++jj) {
-            const float accf = __uint_as_float(acc[jj]) * 262144.0f;
+            const float accf = a[jj] * 262144.0f;
             y[jj] = jj < nvalid ? __ldg(p.w_scale + nb + jj) * fmaf(sa, accf, y[jj]) : 0.f;
           }
           store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, y, nvalid);
@@ -637,12 +684,12 @@ int num_sms() {
   return sms[dev];
 }
 
-template <int OUT, bool kOneBlock>
+template <int OUT, bool kOneBlock, bool kUnstaged = false>
 int launch_gemm(const GemmParams& p, cudaStream_t s) {
-  auto kern = w4a4_gemm_kernel<OUT, kOneBlock>;
+  auto kern = w4a4_gemm_kernel<OUT, kOneBlock, kUnstaged>;
   constexpr int kThreads = Roles<kOneBlock>::kThreads;
   constexpr int kSmemBytes = Smem<kOneBlock>::kBytes;
-  if (!smem_optin<w4a4_gemm_kernel<OUT, kOneBlock>>(kSmemBytes)) return OFFQ_ERR_CUDA;
+  if (!smem_optin<w4a4_gemm_kernel<OUT, kOneBlock, kUnstaged>>(kSmemBytes)) return OFFQ_ERR_CUDA;
   const int sms = num_sms();
   if (sms < 2) return OFFQ_ERR_CUDA;
   const int tiles = p.m_pairs * p.n_tiles;
@@ -686,16 +733,28 @@ extern "C" int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, co
   p.G = static_cast<int>(K / g);
   p.m_pairs = static_cast<int>((T + 2 * BM - 1) / (2 * BM));
   p.n_tiles = static_cast<int>((N + BN - 1) / BN);
+  // Raster groups of m-pairs whose activation codes total at most ~32 MB.
+  const int64_t pair_bytes = 2 * BM * (K / 2);
+  int64_t rm = (int64_t{32} << 20) / pair_bytes;
+  if (rm < 1) rm = 1;
+  p.raster_m = static_cast<int>(rm < p.m_pairs ? rm : p.m_pairs);
   p.t_blocks = static_cast<int>((T + 31) / 32);
   p.n_blocks = static_cast<int>((N + 31) / 32);
   p.kchunks = static_cast<int>(K / 32);
   p.vec_ok = aligned(w_offsum, 16) && aligned(w_scale, 16) && (N % 4 == 0);
   p.async_out = out_dtype != OFFQ_F32 && N % 8 == 0;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const bool unstaged = p.G > kMaxStageG;
   switch (out_dtype) {
-    case OFFQ_F32: return p.G == 1 ? launch_gemm<OFFQ_F32, true>(p, s) : launch_gemm<OFFQ_F32, false>(p, s);
-    case OFFQ_BF16: return p.G == 1 ? launch_gemm<OFFQ_BF16, true>(p, s) : launch_gemm<OFFQ_BF16, false>(p, s);
-    case OFFQ_F16: return p.G == 1 ? launch_gemm<OFFQ_F16, true>(p, s) : launch_gemm<OFFQ_F16, false>(p, s);
+    case OFFQ_F32:
+      return p.G == 1 ? launch_gemm<OFFQ_F32, true>(p, s)
+                      : unstaged ? launch_gemm<OFFQ_F32, false, true>(p, s) : launch_gemm<OFFQ_F32, false>(p, s);
+    case OFFQ_BF16:
+      return p.G == 1 ? launch_gemm<OFFQ_BF16, true>(p, s)
+                      : unstaged ? launch_gemm<OFFQ_BF16, false, true>(p, s) : launch_gemm<OFFQ_BF16, false>(p, s);
+    case OFFQ_F16:
+      return p.G == 1 ? launch_gemm<OFFQ_F16, true>(p, s)
+                      : unstaged ? launch_gemm<OFFQ_F16, false, true>(p, s) : launch_gemm<OFFQ_F16, false>(p, s);
     default: return OFFQ_ERR_INVALID_ARG;
   }
 }

@@ -12,10 +12,11 @@ u = 2^-24), never from observed differences:
   at most L u sum|x| over its block; the scale inherits that relative to max|r|.
   Without the rotation the offset is an fp32 block sum whose summation depth
   is at most g/8 + 16.
-* GEMM outputs. Integer accumulators are exact. The epilogue is a chain of G+2
-  fp32 multiply-adds whose error is bounded by (G + 4) u times the sum of the
-  magnitudes of its terms; a bf16 / fp16 result adds half an ulp of its own
-  format (relative 2^-8 / 2^-11).
+* GEMM outputs. Integer accumulators are exact, and so is the removal of the
+  activation codes' +8 from them (an integer below 2^24). The epilogue is then
+  a chain of G+2 fp32 multiply-adds over s_a acc and the offset terms o_b R_b,
+  whose error is bounded by (G + 4) u times the sum of their magnitudes; a
+  bf16 / fp16 result adds half an ulp of its own format (relative 2^-8 / 2^-11).
 """
 
 from __future__ import annotations
@@ -87,13 +88,13 @@ def check_offsets(o_gpu, o_ref, x, g, rotate, what="offset"):
     assert not np.any(bad), f"{what}: {bad.sum()} offsets out of tolerance"
 
 
-def epilogue_terms(acc_raw, s_a, o, s_w, R):
-    """Magnitudes the fp32 epilogue adds up (float64), for its error bound."""
+def epilogue_terms(acc, s_a, o, s_w, R):
+    """Magnitudes the fp32 epilogue adds up (float64), for its error bound:
+    s_w (|s_a acc| + sum_b |o_b| |R_b|), acc the integer dot product of the codes."""
     s_a = np.asarray(s_a, np.float64)
     s_w = np.abs(np.asarray(s_w, np.float64))
-    o = np.asarray(o, np.float64)
-    o_shift = np.abs(o - 8.0 * s_a[:, None])
-    return s_w[None, :] * (np.abs(s_a[:, None] * np.asarray(acc_raw, np.float64)) + o_shift @ np.abs(R))
+    o = np.abs(np.asarray(o, np.float64))
+    return s_w[None, :] * (np.abs(s_a[:, None] * np.asarray(acc, np.float64)) + o @ np.abs(R))
 
 
 def check_outputs(y_gpu, y_ref, terms, G, out_dtype: str, what="y"):

@@ -56,8 +56,9 @@ def _check_layer(T, K, N, g, out_dt, rotate=True, seed=0, ldo=None, rows=None, n
     # The accumulator the tensor cores hold: sum_k (q_a + 8) q_w, exact.
     acc_ref = O.int_gemm(qa + 8, qw)
     np.testing.assert_array_equal(acc[sel], acc_ref)
-    y_ref = O.epilogue(O.int_gemm(qa, qw), sa, oa, sw, R)
-    terms = epilogue_terms(acc_ref, sa, oa, sw, R)
+    dot = O.int_gemm(qa, qw)
+    y_ref = O.epilogue(dot, sa, oa, sw, R)
+    terms = epilogue_terms(dot, sa, oa, sw, R)
     check_outputs(y[sel], y_ref, terms, K // g, out_dt)
     return y[sel], y_ref, x[sel], w
 
@@ -77,7 +78,7 @@ def test_toy_layer(out_dt):
     sa, oa = a_scale.cpu().numpy().astype(np.float64), a_off.cpu().numpy().astype(np.float64)
     sw, R = w_scale.cpu().numpy().astype(np.float64), rowsum.cpu().numpy().astype(np.float64)
     y_ref = O.epilogue(O.int_gemm(qa, qw), sa, oa, sw, R)
-    check_outputs(y, y_ref, epilogue_terms(O.int_gemm(qa + 8, qw), sa, oa, sw, R), 1, out_dt)
+    check_outputs(y, y_ref, epilogue_terms(O.int_gemm(qa, qw), sa, oa, sw, R), 1, out_dt)
     if out_dt == "f16":
         assert max_rel_err_floored(y, y_ref) <= 2e-3
     # Quality sanity against the unquantized layer (not parity).
@@ -102,7 +103,7 @@ def test_oracle_codes_through_gemm():
     oa = a["offset"].astype(np.float32).astype(np.float64)
     sw = wp["scale"].astype(np.float32).astype(np.float64)
     y_ref = O.epilogue(O.int_gemm(a["q"], wp["q"]), sa, oa, sw, wp["offsum"])
-    check_outputs(y, y_ref, epilogue_terms(O.int_gemm(a["q"] + 8, wp["q"]), sa, oa, sw, wp["offsum"]), K // g, "f32")
+    check_outputs(y, y_ref, epilogue_terms(O.int_gemm(a["q"], wp["q"]), sa, oa, sw, wp["offsum"]), K // g, "f32")
 
 
 @pytest.mark.parametrize("T,K,N,g,out_dt,ldo", [
@@ -143,7 +144,7 @@ def test_null_offset_means_zero():
     R = rowsum.cpu().numpy().astype(np.float64)
     zero = np.zeros((T, 1))
     y_ref = O.epilogue(O.int_gemm(qa, qw), sa, zero, sw, R)
-    check_outputs(y, y_ref, epilogue_terms(acc, sa, zero, sw, R), 1, "f32")
+    check_outputs(y, y_ref, epilogue_terms(O.int_gemm(qa, qw), sa, zero, sw, R), 1, "f32")
 
 
 def test_accumulator_exact_at_largest_k():
@@ -223,8 +224,9 @@ def _check_config_layer(T, K, N, g, rows, dist, n_out, mult, seed):
     R = rowsum.cpu().numpy().astype(np.float64)
     acc_ref = O.int_gemm(qa + 8, qw)
     np.testing.assert_array_equal(acc_s, acc_ref)
-    y_ref = O.epilogue(O.int_gemm(qa, qw), sa, oa, sw, R)
-    check_outputs(y, y_ref, epilogue_terms(acc_ref, sa, oa, sw, R), K // g, "bf16")
+    dot = O.int_gemm(qa, qw)
+    y_ref = O.epilogue(dot, sa, oa, sw, R)
+    check_outputs(y, y_ref, epilogue_terms(dot, sa, oa, sw, R), K // g, "bf16")
 
 
 @pytest.mark.parametrize("T,K,N,g,nrows,dist,n_out,mult", [
@@ -236,3 +238,43 @@ def _check_config_layer(T, K, N, g, rows, dist, n_out, mult, seed):
 def test_config_gemm_shapes_sampled(T, K, N, g, nrows, dist, n_out, mult):
     rows = np.unique(np.concatenate([W.unit_index_sample(T, nrows, seed=N % 97), [0, T - 1]]))
     _check_config_layer(T, K, N, g, rows, dist, n_out, mult, seed=K + N)
+
+
+@pytest.mark.parametrize("K,g", [(4096, 4096), (11008, 256), (4096, 32)])
+def test_outputs_near_zero_against_large_row_sums(K, g):
+    """Weight rows of all +7 (row sums 7K) against activation rows whose codes add up to
+    0, +-1, +-2, ...: every output is a small multiple of s_a s_w next to the 8 s_a R that the
+    tensor cores carry in acc'. Removing that term in the integer domain leaves each fp32 output
+    within a few rounding errors of the float64 result (max relative error 2e-3 with no floor,
+    f32 out), for one block, 43 blocks, and the unstaged 128-block epilogue."""
+    T, N = 64, 512
+    rng = np.random.default_rng(K + g)
+    qa = rng.integers(-7, 8, size=(T, K))
+    # Make each row's code sum a small integer: move the excess onto channels with room.
+    for t in range(T):
+        target = t % 9 - 4
+        excess = int(qa[t].sum()) - target
+        while excess != 0:
+            k = int(rng.integers(0, K))
+            step = max(-7 - qa[t, k], min(7 - qa[t, k], -excess))
+            qa[t, k] += step
+            excess += step
+    qw = rng.integers(-7, 8, size=(N, K))
+    qw[::2] = 7                                            # every other weight row all +7
+    sa = rng.uniform(0.5, 2.0, size=T).astype(np.float32)
+    sw = rng.uniform(0.5, 2.0, size=N).astype(np.float32)
+    R = qw.reshape(N, K // g, g).sum(axis=2).T.astype(np.float32)
+    dev = lambda arr, dt: torch.from_numpy(np.ascontiguousarray(arr)).to(dt).cuda()
+    y, acc = _run_gemm(dev(O.tile_codes(O.pack_act_codes(qa)).reshape(-1, K // 2), torch.uint8),
+                       dev(sa, torch.float32), None,
+                       dev(O.tile_codes(O.pack_weight_codes(qw)).reshape(-1, K // 2), torch.uint8),
+                       dev(sw, torch.float32), dev(R, torch.float32), g, "f32")
+    np.testing.assert_array_equal(acc, O.int_gemm(qa + 8, qw))
+    dot = O.int_gemm(qa, qw)
+    zero = np.zeros((T, K // g))
+    y_ref = O.epilogue(dot, sa.astype(np.float64), zero, sw.astype(np.float64), R.astype(np.float64))
+    np.testing.assert_array_equal(dot[:, ::2], np.repeat(7 * (np.arange(T) % 9 - 4)[:, None], N // 2, axis=1))
+    check_outputs(y, y_ref, epilogue_terms(dot, sa, zero, sw, R), K // g, "f32")
+    nz = y_ref != 0
+    assert np.all(y[~nz] == 0)
+    assert np.max(np.abs(y[nz] - y_ref[nz]) / np.abs(y_ref[nz])) <= 2e-3
