@@ -493,6 +493,24 @@ int64_t offq_weight_codes_bytes(int64_t N, int64_t K);
  */
 int offq_get_device_status(void* stream);
 
+/*
+ * offq_set_wait_cycles -- test hook for the failure path (no counterpart in
+ * the paper). Sets, for the calls that follow in this process, the budget in
+ * SM clock cycles of the bounded waits with which the persistent row
+ * quantizers (offq_quantize_act and offq_kv4_quantize on inputs with more row
+ * groups than SMs, and the shared-memory ring kernel of rotation-free
+ * single-block rows) wait for the rows they stage by bulk copies. A budget
+ * shorter than the default makes those waits behave as waits for a flag that
+ * nothing sets: they do not look at their barrier and give up after about
+ * that many cycles. The kernel then lets every copy already in flight land
+ * (waiting for it with the full budget), returns without writing the rest of
+ * its outputs, and records OFFQ_ERR_TIMEOUT for offq_get_device_status.
+ * 0 restores the default (about 2 s), and with it the normal waits. Returns
+ * OFFQ_ERR_INVALID_ARG for a negative value. The setting is process-wide and
+ * is read when a call launches; meant for tests only.
+ */
+int offq_set_wait_cycles(int64_t cycles);
+
 /* Human-readable name of a status code (static string, never NULL). */
 const char* offq_status_string(int status);
 

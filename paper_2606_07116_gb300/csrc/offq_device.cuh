@@ -83,6 +83,23 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
   }
 }
 
+// As mbar_wait, with a budget of `budget` cycles. A budget below kWaitCycles
+// is a test setting of the failure path: the wait then does not look at its
+// barrier, as if it waited for a flag that nothing sets, and gives up after
+// that many cycles (setting *abort). Whatever the barrier tracks (a copy in
+// flight) still completes, and the caller's teardown waits for it.
+__device__ __forceinline__ bool mbar_wait_for(uint32_t bar, uint32_t parity, volatile int* abort, long long budget) {
+  if (budget >= kWaitCycles) return mbar_wait(bar, parity, abort);
+  const long long t0 = clock64();
+  while (!*abort) {
+    if (clock64() - t0 > budget) {
+      *abort = 1;
+      break;
+    }
+  }
+  return false;
+}
+
 // ---------------------------------------------------------------------------
 // TMA (bulk tensor copies, global -> shared, completion on an mbarrier)
 // ---------------------------------------------------------------------------

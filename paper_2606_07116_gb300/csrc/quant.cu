@@ -39,6 +39,7 @@
 #include <cuda_fp16.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <type_traits>
 
@@ -69,6 +70,7 @@ struct QuantArgs {
   int tiled;        // codes in the 32-row tiled operand layout (else row-major)
   int* status;      // device status word (bounded waits that run out write here)
   int ring_slots;   // persistent forms: slots of rows_per_cta rows each (1 to 3)
+  long long wait_cycles;  // persistent forms: budget of a wait for a staged row (kWaitCycles unless a test sets it)
 };
 
 template <int L>
@@ -434,7 +436,7 @@ __global__ void __launch_bounds__(NarrowGeo<L>::kMaxThreads) quantize_rows_kerne
     // Pass 1: register 8i + c holds channel 8t + 8 TPB i + c of block b.
     float v[E];
     if constexpr (kRing) {
-      const bool ok = mbar_wait(ring.bar(), ring.phase, &abort_flag);
+      const bool ok = mbar_wait_for(ring.bar(), ring.phase, &abort_flag, a.wait_cycles);
       if (ok && active) {
         const Tin* p = reinterpret_cast<const Tin*>(ring.slot()) + static_cast<size_t>(lrow) * K + b * g + 8 * t;
 #pragma unroll
@@ -611,7 +613,7 @@ __global__ void __launch_bounds__(WideGeo<L>::kMaxThreads) quantize_rows_wide_ke
 
     float v[E];
     if constexpr (kRing) {
-      const bool ok = mbar_wait(ring.bar(), ring.phase, &abort_flag);
+      const bool ok = mbar_wait_for(ring.bar(), ring.phase, &abort_flag, a.wait_cycles);
       if (ok && active) {
         const Tin* p = reinterpret_cast<const Tin*>(ring.slot()) + static_cast<size_t>(lrow) * K + b * g + 8 * t1;
 #pragma unroll
@@ -1006,7 +1008,8 @@ __global__ void __launch_bounds__(256) quantize_rows_bulk_kernel(const QuantArgs
   bool ok = true;
   for (int64_t r = r0; r < a.rows; r += TW) {
     const uint32_t bar = bar0 + 8u * slot;
-    if (!mbar_wait(bar, phase, &abort_flag)) {
+    // Warp-uniform outcome: the sweeps below shuffle across the whole warp.
+    if (!__all_sync(0xFFFFFFFFu, mbar_wait_for(bar, phase, &abort_flag, a.wait_cycles))) {
       ok = false;
       break;
     }
@@ -1282,11 +1285,16 @@ int dispatch_g(const QuantArgs& a, int g, cudaStream_t s) {
   }
 }
 
+// Budget of the persistent kernels' waits for a staged row, in SM cycles
+// (offq_set_wait_cycles; kWaitCycles unless a test shortens it).
+std::atomic<long long> g_row_wait_cycles{kWaitCycles};
+
 int run_quant(QuantArgs a, int dtype, int g, cudaStream_t s) {
   const double isg = (a.flags & OFFQ_ROTATE) ? 1.0 / std::sqrt(static_cast<double>(g)) : 1.0;
   a.inv_sqrt_g = static_cast<float>(isg);
   a.scale_mul = static_cast<float>(isg / 7.0);
   a.status = device_status_ptr();
+  a.wait_cycles = g_row_wait_cycles.load(std::memory_order_relaxed);
   switch (dtype) {
     case OFFQ_BF16: return dispatch_g<__nv_bfloat16>(a, g, s);
     case OFFQ_F16: return dispatch_g<__half>(a, g, s);
@@ -1447,4 +1455,10 @@ extern "C" int64_t offq_act_codes_bytes(int64_t T, int64_t K) {
 extern "C" int64_t offq_weight_codes_bytes(int64_t N, int64_t K) {
   if (N < 1 || K <= 0 || K % 32 != 0) return -1;
   return (N + 31) / 32 * 32 * (K / 2);
+}
+
+extern "C" int offq_set_wait_cycles(int64_t cycles) {
+  if (cycles < 0) return OFFQ_ERR_INVALID_ARG;
+  g_row_wait_cycles.store(cycles == 0 || cycles > kWaitCycles ? kWaitCycles : cycles, std::memory_order_relaxed);
+  return OFFQ_OK;
 }

@@ -46,6 +46,7 @@ _SIGNATURES = {
     "offq_kv4_quantize": (_c_int, [_c_vp, _c_int, _c_i64, _c_i32, _c_i32, _c_i64, _c_i32, _c_vp, _c_vp, _c_vp, _c_vp]),
     "offq_prepare_weight": (_c_int, [_c_vp, _c_int, _c_i64, _c_i64, _c_i32, _c_i32, _c_vp, _c_vp, _c_vp, _c_vp]),
     "offq_get_device_status": (_c_int, [_c_vp]),
+    "offq_set_wait_cycles": (_c_int, [_c_i64]),
     "offq_status_string": (ctypes.c_char_p, [_c_int]),
     "offq_abi_version": (_c_int, []),
     "offq_act_codes_bytes": (_c_i64, [_c_i64, _c_i64]),
@@ -272,6 +273,12 @@ def offq_rotate_heads_reflected(x: torch.Tensor, T: int, H: int, head_dim: int, 
 
 def offq_get_device_status(stream=None) -> int:
     return load_library().offq_get_device_status(_stream(stream))
+
+
+def offq_set_wait_cycles(cycles: int) -> None:
+    """Test hook: budget of the persistent quantizers' waits for staged rows
+    (0 restores the default)."""
+    _check("offq_set_wait_cycles", load_library().offq_set_wait_cycles(cycles))
 
 
 def offq_act_codes_bytes(T: int, K: int) -> int:

@@ -27,6 +27,11 @@ def test_exports_every_declared_symbol(lib):
         assert hasattr(lib, name), name
 
 
+def test_wait_budget_hook_arguments(lib):
+    assert lib.offq_set_wait_cycles(-1) == Q.OFFQ_ERR_INVALID_ARG
+    assert lib.offq_set_wait_cycles(0) == Q.OFFQ_OK
+
+
 def test_status_strings_and_version(lib):
     assert Q.abi_version() == 1
     for code, name in [(0, "OFFQ_OK"), (-1, "OFFQ_ERR_INVALID_ARG"), (-2, "OFFQ_ERR_UNSUPPORTED"),
