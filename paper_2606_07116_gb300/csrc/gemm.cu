@@ -716,6 +716,11 @@ extern "C" int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, co
       (a_offset != nullptr && !aligned(a_offset, 4)) || (acc_debug != nullptr && !aligned(acc_debug, 4)))
     return OFFQ_ERR_MISALIGNED;
 
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (T <= decode_max_tokens())
+    return w4a4_linear_decode(a_codes, a_scale, a_offset, T, N, K, g, w_codes, w_scale, w_offsum, out, out_dtype, ldo,
+                              acc_debug, s);
+
   GemmParams p{};
   p.a_codes = a_codes;
   p.w_codes = w_codes;
@@ -743,7 +748,6 @@ extern "C" int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, co
   p.kchunks = static_cast<int>(K / 32);
   p.vec_ok = aligned(w_offsum, 16) && aligned(w_scale, 16) && (N % 4 == 0);
   p.async_out = out_dtype != OFFQ_F32 && N % 8 == 0;
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
   const bool unstaged = p.G > kMaxStageG;
   switch (out_dtype) {
     case OFFQ_F32:

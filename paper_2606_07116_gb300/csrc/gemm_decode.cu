@@ -1,0 +1,461 @@
+// W4A4 GEMM of the OffQ path for few tokens (decode, T <= 64): the same
+// product and epilogue as w4a4_gemm_kernel (paper Sec. 1: all matrix
+// multiplications in uniform 4-bit execution; Eq. 5: the offsets meet the
+// weight block row sums),
+//
+//   y[t][n] = s_w[n] * ( s_a[t] * (acc'[n][t] - 8 Rt[n]) + sum_b o[t][b] * R[b][n] ),
+//   acc'[n][t] = sum_k q_w[n][k] * (q_a[t][k] + 8),   Rt[n] = sum_b R[b][n],
+//
+// laid out for the regime where the weights dominate the bytes: each weight
+// code is read once and used by at most 64 tokens, so the time is the HBM
+// stream of the weight codes.
+//
+// Design:
+//  * The MMA's M side is the weights: a CTA owns whole 32-row blocks of the
+//    weight codes (block counts differ by at most one between CTAs) over the
+//    whole K, so every SM streams an equal share of the weight bytes with no
+//    reduction across CTAs; up to 4 blocks (128 rows, one TMEM lane quarter
+//    each) make one pass of the accumulator. The N side is the tokens, padded
+//    to a multiple of 16 (tcgen05.mma.cta_group::1.kind::f8f6f4, M = 128,
+//    N = 16..64, K = 32), both operands in shared memory: with N this small,
+//    reading the 4 KB A operand of each instruction dominates the MMA, and the
+//    shared-memory path reads it faster than tensor memory.
+//  * In the tiled code layout a block's codes are contiguous along K (16-byte
+//    chunk c of row r at ((block * K/32 + c) * 32 + r) * 16), so one plain bulk
+//    copy (cp.async.bulk) moves 4 k-tiles of a block, 8 KB. The copies land in
+//    a ring of packed slots (one slot: 4 k-tiles of the pass's blocks and of
+//    the tokens), as many as shared memory holds; the converters release a slot
+//    as soon as they have read it.
+//  * Converter warps (four per 32-row quarter, taking turns by k-tile) widen
+//    the weights (sign-magnitude nibbles -> E4M3) and the activation codes
+//    (u = q + 8 -> E4M3 u * 2^-9) into the 128-byte-swizzled K-major operands,
+//    through a ring of 4 operand stages that the MMAs release. The products are integers
+//    times 2^-18, exact in the fp32 accumulator.
+//  * Epilogue warps compute each row's offset correction sum_b o[t][b] R[b][n]
+//    while the pass's MMAs run (into tensor memory), then drain the
+//    accumulator: lane = weight row n, column = token t, so a warp writes 32
+//    consecutive outputs of one token at a time.
+// Warps: 0 bulk-copy producer (and TMEM allocation), 1-16 converters, 17 MMA
+// issuer, 18-21 epilogue. Every wait is bounded; a wait that runs out aborts
+// the CTA, which lets its copies and MMAs in flight finish before it exits and
+// records OFFQ_ERR_TIMEOUT in the device status word.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include "offq.h"
+#include "offq_device.cuh"
+#include "offq_host.h"
+#include "pair_common.cuh"
+
+namespace {
+
+using namespace offq;
+
+constexpr int kDecMaxT = 64;           // tokens handled (MMA N <= 64)
+constexpr int kDecBK = 128;            // codes per k-tile
+constexpr int kDecKtBytes = 32 * kDecBK / 2;  // 2 KB: one block's (or 32 tokens') codes of one k-tile
+constexpr int kDecSlotKt = 4;          // k-tiles per packed slot (one bulk copy of 8 KB per block)
+constexpr int kDecOpStages = 4;        // operand stages (A and B in shared memory)
+constexpr int kDecAStage = 128 * kDecBK;  // 16 KB: E4M3 A operand, 128 weight rows x 128 B
+constexpr int kDecMaxPk = 16;          // packed slots at most
+constexpr int kDecPhases = 4;          // converter warps per TMEM lane quarter
+constexpr int kDecConv0 = 1, kDecMma = kDecConv0 + 4 * kDecPhases, kDecEpi0 = kDecMma + 1;
+constexpr int kDecThreads = (kDecEpi0 + 4) * 32;
+// Tensor memory: accumulator (64 columns), offset correction (64).
+constexpr int kDecAcc = 0, kDecCorr = 64, kDecTmemCols = 128;
+constexpr int kDecSmemMax = 224 * 1024;  // dynamic shared memory of the kernel (opt-in)
+constexpr int kDecNumBars = 2 * kDecMaxPk + 2 * kDecOpStages + 2;
+
+// Shared memory, laid out at launch from the block and token counts:
+//   [op stages x A operand (16 KB)] [op stages x B operand (n_mma rows x 128 B, 1024-aligned)]
+//   [pk slots x (blocks x 4 k-tiles, token blocks x 4 k-tiles)] [s_a] [barriers] [misc]
+struct DecLayout {
+  int off_b;     // first B operand stage (after the A stages)
+  int b_stage;   // bytes of one B operand stage
+  int w_bytes;   // weight part of a packed slot: max blocks per pass x 4 k-tiles x 2 KB
+  int pk_slot;   // bytes of one packed slot
+  int n_pk;      // packed slots
+  int off_pk, off_sa, off_bars, off_misc;
+};
+
+struct DecodeParams {
+  DecLayout L;
+  const uint8_t* a_codes;
+  const uint8_t* w_codes;
+  const float* a_scale;
+  const float* a_offset;   // [T][G] or nullptr
+  const float* w_scale;
+  const float* rowsum;     // [G][N]
+  void* out;
+  int64_t ldo;
+  int32_t* acc_debug;
+  int* status;
+  int T, N, K, G;
+  int n_mma;               // tokens padded to a multiple of 16
+  int nk;                  // k-tiles
+  int kchunks;             // K / 32
+  int a_blocks;            // 32-token blocks of the activation codes
+  int blk_q, blk_r;        // blocks per CTA: blk_q, plus one for the first blk_r CTAs
+};
+
+__device__ __forceinline__ void mbar_arrive_n(uint32_t bar, uint32_t n) {
+  asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(n) : "memory");
+}
+
+template <int OUT>
+__global__ void __launch_bounds__(kDecThreads, 1) w4a4_decode_kernel(const DecodeParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* smem = smem_raw + (base - raw);
+  const DecLayout& L = p.L;
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int c = blockIdx.x;
+  const int nblocks = p.blk_q + (c < p.blk_r ? 1 : 0);               // weight row blocks of this CTA
+  const int first = c * p.blk_q + (c < p.blk_r ? c : p.blk_r);       // its first block
+  const int passes = (nblocks + 3) / 4;
+  const int groups = (p.nk + kDecSlotKt - 1) / kDecSlotKt;           // packed slots per pass
+  const int npk = L.n_pk;
+  const uint32_t bar0 = base + L.off_bars;
+  auto pk_full = [&](int i) { return bar0 + 8u * i; };                               // copies landed
+  auto pk_empty = [&](int i) { return bar0 + 8u * (kDecMaxPk + i); };                // converters read the slot
+  auto op_full = [&](int s) { return bar0 + 8u * (2 * kDecMaxPk + s); };             // operands converted
+  auto op_empty = [&](int s) { return bar0 + 8u * (2 * kDecMaxPk + kDecOpStages + s); };  // MMAs done
+  const uint32_t acc_full = bar0 + 8u * (2 * kDecMaxPk + 2 * kDecOpStages);          // a pass's MMAs done
+  const uint32_t acc_empty = acc_full + 8u;                                          // its accumulator read
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L.off_misc);
+  volatile int* abort = reinterpret_cast<volatile int*>(smem + L.off_misc + 16);
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < npk; ++i) {
+      mbar_init(pk_full(i), 1);
+      mbar_init(pk_empty(i), 4 * kDecSlotKt);  // four warps per k-tile of the slot
+    }
+    for (int s = 0; s < kDecOpStages; ++s) {
+      mbar_init(op_full(s), 4);
+      mbar_init(op_empty(s), 1);
+    }
+    mbar_init(acc_full, 1);
+    mbar_init(acc_empty, 4);
+    *abort = 0;
+    mbar_fence_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(smem_u32(tmem_slot), kDecTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  griddep_wait();
+  griddep_launch_dependents();
+
+  int steps_issued = 0;  // producer: packed slots filled
+  int commits = 0;       // MMA issuer: passes committed to acc_full
+
+  if (warp == 0) {
+    // ---------------- bulk-copy producer ----------------
+    if (lane == 0) {
+      int st = 0;
+      bool ok = true;
+      for (int j = 0; j < passes && ok; ++j) {
+        const int nbp = nblocks - 4 * j < 4 ? nblocks - 4 * j : 4;
+        const int blk0 = first + 4 * j;
+        for (int g = 0; g < groups; ++g, ++st) {
+          const int i = st % npk;
+          if (!mbar_wait(pk_empty(i), ((st / npk) & 1) ^ 1, abort)) {
+            ok = false;
+            break;
+          }
+          const int c0 = 4 * kDecSlotKt * g;  // first chunk of the slot
+          const int nch = p.kchunks - c0 < 4 * kDecSlotKt ? p.kchunks - c0 : 4 * kDecSlotKt;
+          const uint32_t bytes = static_cast<uint32_t>(nch) * 512u;
+          mbar_arrive_expect_tx(pk_full(i), bytes * static_cast<uint32_t>(nbp + p.a_blocks));
+          const uint32_t slot = base + L.off_pk + i * L.pk_slot;
+          for (int jb = 0; jb < nbp; ++jb)
+            bulk_load(slot + jb * kDecSlotKt * kDecKtBytes,
+                      p.w_codes + (static_cast<int64_t>(blk0 + jb) * p.kchunks + c0) * 512, bytes, pk_full(i));
+          for (int ab = 0; ab < p.a_blocks; ++ab)
+            bulk_load(slot + L.w_bytes + ab * kDecSlotKt * kDecKtBytes,
+                      p.a_codes + (static_cast<int64_t>(ab) * p.kchunks + c0) * 512, bytes, pk_full(i));
+          steps_issued = st + 1;
+        }
+      }
+    }
+  } else if (warp < kDecMma) {
+    // ---------------- converters ----------------
+    const int q = warp & 3;                     // TMEM lane quarter = block within the pass
+    const int phase = (warp - kDecConv0) / 4;   // this warp's k-tiles: u == phase mod kDecPhases
+    const int t = 32 * q + lane;                // this lane's token row of B
+    const bool b_row = t < p.n_mma;
+    const int total = passes * p.nk;
+    for (int u = phase; u < total; u += kDecPhases) {
+      const int j = u / p.nk, kt = u - j * p.nk;
+      const int g = kt / kDecSlotKt, i = kt - g * kDecSlotKt;
+      const int st = j * groups + g;
+      const int slot_i = st % npk;
+      const int s = u % kDecOpStages;
+      const int nbp = nblocks - 4 * j < 4 ? nblocks - 4 * j : 4;
+      if (!__all_sync(0xFFFFFFFFu, mbar_wait(pk_full(slot_i), (st / npk) & 1, abort))) break;
+      const uint32_t slot = base + L.off_pk + slot_i * L.pk_slot;
+      uint4 wv[4], av[4];
+#pragma unroll
+      for (int cc = 0; cc < 4; ++cc) {
+        const bool chunk_ok = 4 * kt + cc < p.kchunks;
+        wv[cc] = q < nbp && chunk_ok ? lds128(slot + (q * kDecSlotKt + i) * kDecKtBytes + cc * 512 + lane * 16)
+                                     : make_uint4(0u, 0u, 0u, 0u);
+        av[cc] = b_row && chunk_ok
+                     ? lds128(slot + L.w_bytes + ((t >> 5) * kDecSlotKt + i) * kDecKtBytes + cc * 512 + (t & 31) * 16)
+                     : make_uint4(0u, 0u, 0u, 0u);
+      }
+      __syncwarp();
+      if (lane == 0) {
+        // The last k-tile of a short last slot also arrives for the k-tiles it lacks.
+        const int in_slot = p.nk - g * kDecSlotKt < kDecSlotKt ? p.nk - g * kDecSlotKt : kDecSlotKt;
+        mbar_arrive_n(pk_empty(slot_i), i == in_slot - 1 ? 1 + kDecSlotKt - in_slot : 1);
+      }
+      if (!__all_sync(0xFFFFFFFFu, mbar_wait(op_empty(s), ((u / kDecOpStages) & 1) ^ 1, abort))) break;
+      {
+        // A: this weight row's 128 codes -> one 128-byte row of the swizzled operand.
+        const int jr = 32 * q + lane;
+        const uint32_t dst = base + s * kDecAStage + (jr >> 3) * 1024 + (jr & 7) * 128;
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) {
+          uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
+          widen_weight(wv[cc].x, a0, a1);
+          widen_weight(wv[cc].y, a2, a3);
+          widen_weight(wv[cc].z, b0, b1);
+          widen_weight(wv[cc].w, b2, b3);
+          sts128(dst + (((2 * cc) ^ (jr & 7)) << 4), a0, a1, a2, a3);
+          sts128(dst + (((2 * cc + 1) ^ (jr & 7)) << 4), b0, b1, b2, b3);
+        }
+      }
+      if (b_row) {
+        const uint32_t dst = base + L.off_b + s * L.b_stage + (t >> 3) * 1024 + (t & 7) * 128;
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) {
+          uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
+          widen_act(av[cc].x, a0, a1);
+          widen_act(av[cc].y, a2, a3);
+          widen_act(av[cc].z, b0, b1);
+          widen_act(av[cc].w, b2, b3);
+          sts128(dst + (((2 * cc) ^ (t & 7)) << 4), a0, a1, a2, a3);
+          sts128(dst + (((2 * cc + 1) ^ (t & 7)) << 4), b0, b1, b2, b3);
+        }
+      }
+      fence_proxy_async_smem();  // the operand rows, visible to the MMA's reads
+      __syncwarp();
+      if (lane == 0) mbar_arrive(op_full(s));
+    }
+  } else if (warp == kDecMma) {
+    // ---------------- MMA issuer ----------------
+    if (lane == 0) {
+      const uint32_t idesc = idesc_e4m3_f32(128, p.n_mma);
+      bool ok = true;
+      for (int j = 0; j < passes && ok; ++j) {
+        ok = mbar_wait(acc_empty, (j & 1) ^ 1, abort);  // the previous pass has been read out
+        tc_fence_after();
+        for (int kt = 0; kt < p.nk && ok; ++kt) {
+          const int u = j * p.nk + kt;
+          const int s = u % kDecOpStages;
+          if (!mbar_wait(op_full(s), (u / kDecOpStages) & 1, abort)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_addr = base + s * kDecAStage;
+          const uint32_t b_addr = base + L.off_b + s * L.b_stage;
+#pragma unroll
+          for (int kk = 0; kk < kDecBK / 32; ++kk)
+            mma_f8f6f4(tmem + kDecAcc, smem_desc_sw128(a_addr + 32 * kk), smem_desc_sw128(b_addr + 32 * kk), idesc,
+                       (kt | kk) != 0 ? 1u : 0u);
+          mma_commit(op_empty(s));
+        }
+        mma_commit(acc_full);  // also after an abort: its arrival tells teardown the MMAs are done
+        ++commits;
+      }
+    }
+  } else {
+    // ---------------- epilogue ----------------
+    const int q = warp & 3;
+    float* Sa = reinterpret_cast<float*>(smem + L.off_sa);
+    const int et = threadIdx.x - kDecEpi0 * 32;
+    for (int i = et; i < kDecMaxT; i += 4 * 32) Sa[i] = i < p.T ? __ldg(p.a_scale + i) : 0.f;
+    asm volatile("bar.sync 1, 128;" ::: "memory");  // Sa staged by the four epilogue warps
+    const uint32_t lane_base = static_cast<uint32_t>(32 * q) << 16;
+    for (int j = 0; j < passes; ++j) {
+      const int n = (first + 4 * j + q) * 32 + lane;
+      const bool row_ok = q < (nblocks - 4 * j < 4 ? nblocks - 4 * j : 4) && n < p.N;
+      // Offset correction corr[t] = sum_b o[t][b] R[b][n] while the pass's MMAs run.
+      for (int t0 = 0; t0 < p.n_mma; t0 += 16) {
+        uint32_t cr[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) cr[i] = 0u;
+        if (row_ok && p.a_offset != nullptr) {
+          float cv[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) cv[i] = 0.f;
+          for (int b = 0; b < p.G; ++b) {
+            const float rv = __ldg(p.rowsum + static_cast<int64_t>(b) * p.N + n);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              const int tt = t0 + i;
+              const float o = tt < p.T ? __ldg(p.a_offset + static_cast<int64_t>(tt) * p.G + b) : 0.f;
+              cv[i] = b == 0 ? o * rv : fmaf(o, rv, cv[i]);
+            }
+          }
+#pragma unroll
+          for (int i = 0; i < 16; ++i) cr[i] = __float_as_uint(cv[i]);
+        }
+        tmem_st_16cols(tmem + lane_base + kDecCorr + t0, cr);
+      }
+      tmem_st_wait();
+      // -8 Rt[n] 2^-18: integers, exact in fp32.
+      float rt = 0.f, sw = 0.f;
+      if (row_ok) {
+        for (int b = 0; b < p.G; ++b) rt += __ldg(p.rowsum + static_cast<int64_t>(b) * p.N + n);
+        sw = __ldg(p.w_scale + n);
+      }
+      const float m8r = rt * -0x1p-15f;
+      const bool ok = __all_sync(0xFFFFFFFFu, mbar_wait(acc_full, j & 1, abort)) && !*abort;
+      tc_fence_after();
+      if (!ok) break;
+      for (int t0 = 0; t0 < p.n_mma; t0 += 16) {
+        uint32_t acc[16], cr[16];
+        tmem_ld_16cols(tmem + lane_base + kDecAcc + t0, acc);
+        tmem_ld_16cols(tmem + lane_base + kDecCorr + t0, cr);
+        tmem_ld_wait();
+        if (!row_ok) continue;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const int tt = t0 + i;
+          if (tt >= p.T) break;
+          const float a = (__uint_as_float(acc[i]) + m8r) * 262144.0f;  // exact: the integer dot product
+          const float y = sw * fmaf(Sa[tt], a, __uint_as_float(cr[i]));
+          const int64_t off = static_cast<int64_t>(tt) * p.ldo + n;
+          if (OUT == OFFQ_F32) {
+            static_cast<float*>(p.out)[off] = y;
+          } else if (OUT == OFFQ_BF16) {
+            static_cast<__nv_bfloat16*>(p.out)[off] = __float2bfloat16_rn(y);
+          } else {
+            static_cast<__half*>(p.out)[off] = __float2half_rn(y);
+          }
+          if (p.acc_debug != nullptr)
+            p.acc_debug[static_cast<int64_t>(tt) * p.N + n] = __float2int_rn(__uint_as_float(acc[i]) * 262144.0f);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acc_empty);
+    }
+  }
+
+  // ---------------- teardown ----------------
+  if (warp == 0 && lane == 0 && *abort) {
+    // Copies of slots nobody consumed land before the CTA ends: the last use of
+    // each slot (earlier uses of a slot completed before its reuse).
+    for (int st = steps_issued > npk ? steps_issued - npk : 0; st < steps_issued; ++st)
+      mbar_wait_teardown(pk_full(st % npk), (st / npk) & 1);
+  }
+  if (warp == kDecMma && lane == 0 && commits > 0)
+    mbar_wait_teardown(acc_full, (commits - 1) & 1);  // the MMAs are done before TMEM is released
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kDecTmemCols);
+  }
+  if (threadIdx.x == 0 && *abort && p.status != nullptr) atomicExch(p.status, kErrTimeout);
+}
+
+int decode_num_sms() {
+  static int sms[kMaxDevices] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return 0;
+  if (sms[dev] == 0) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    sms[dev] = v;
+  }
+  return sms[dev];
+}
+
+// Shared-memory layout for passes of up to `max_blocks` weight blocks and T
+// tokens: the operand stages, then as many packed slots as fit.
+DecLayout decode_layout(int max_blocks, int T) {
+  DecLayout L{};
+  const int n_mma = (T + 15) / 16 * 16;
+  const int a_blocks = (T + 31) / 32;
+  L.b_stage = (n_mma * kDecBK + 1023) / 1024 * 1024;
+  L.off_b = kDecOpStages * kDecAStage;
+  L.w_bytes = max_blocks * kDecSlotKt * kDecKtBytes;
+  L.pk_slot = L.w_bytes + a_blocks * kDecSlotKt * kDecKtBytes;
+  const int fixed = L.off_b + kDecOpStages * L.b_stage + kDecMaxT * 4 + kDecNumBars * 8 + 64 + 1024;
+  const int n = (kDecSmemMax - fixed) / L.pk_slot;
+  L.n_pk = n < kDecMaxPk ? n : kDecMaxPk;
+  L.off_pk = L.off_b + kDecOpStages * L.b_stage;
+  L.off_sa = L.off_pk + L.n_pk * L.pk_slot;
+  L.off_bars = L.off_sa + kDecMaxT * 4;
+  L.off_misc = L.off_bars + kDecNumBars * 8;
+  return L;
+}
+
+template <int OUT>
+int launch_decode(const DecodeParams& p, int grid, cudaStream_t s) {
+  if (!smem_optin<w4a4_decode_kernel<OUT>>(kDecSmemMax)) return OFFQ_ERR_CUDA;
+  const size_t bytes = static_cast<size_t>(p.L.off_misc) + 64 + 1024;
+  return launch_pdl(w4a4_decode_kernel<OUT>, dim3(grid), dim3(kDecThreads), bytes, s, p);
+}
+
+}  // namespace
+
+namespace offq {
+
+int decode_max_tokens() { return kDecMaxT; }
+
+// The decode form of offq_w4a4_linear (arguments checked by the caller; T in 1..64).
+int w4a4_linear_decode(const uint8_t* a_codes, const float* a_scale, const float* a_offset, int64_t T, int64_t N,
+                       int64_t K, int32_t g, const uint8_t* w_codes, const float* w_scale, const float* w_offsum,
+                       void* out, int out_dtype, int64_t ldo, int32_t* acc_debug, cudaStream_t stream) {
+  const int sms = decode_num_sms();
+  if (sms < 1) return OFFQ_ERR_CUDA;
+  const int64_t nblk = (N + 31) / 32;
+  const int64_t grid = nblk < sms ? nblk : sms;
+  DecodeParams p{};
+  p.a_codes = a_codes;
+  p.w_codes = w_codes;
+  p.a_scale = a_scale;
+  p.a_offset = a_offset;
+  p.w_scale = w_scale;
+  p.rowsum = w_offsum;
+  p.out = out;
+  p.ldo = ldo;
+  p.acc_debug = acc_debug;
+  p.status = device_status_ptr();
+  p.T = static_cast<int>(T);
+  p.N = static_cast<int>(N);
+  p.K = static_cast<int>(K);
+  p.G = static_cast<int>(K / g);
+  p.n_mma = static_cast<int>((T + 15) / 16 * 16);
+  p.nk = static_cast<int>((K + kDecBK - 1) / kDecBK);
+  p.kchunks = static_cast<int>(K / 32);
+  p.a_blocks = static_cast<int>((T + 31) / 32);
+  p.blk_q = static_cast<int>(nblk / grid);
+  p.blk_r = static_cast<int>(nblk % grid);
+  const int max_blocks = p.blk_q + (p.blk_r > 0 ? 1 : 0);
+  p.L = decode_layout(max_blocks < 4 ? max_blocks : 4, p.T);
+  if (p.L.n_pk < 2) return OFFQ_ERR_UNSUPPORTED;
+  const int gr = static_cast<int>(grid);
+  switch (out_dtype) {
+    case OFFQ_F32: return launch_decode<OFFQ_F32>(p, gr, stream);
+    case OFFQ_BF16: return launch_decode<OFFQ_BF16>(p, gr, stream);
+    case OFFQ_F16: return launch_decode<OFFQ_F16>(p, gr, stream);
+    default: return OFFQ_ERR_INVALID_ARG;
+  }
+}
+
+}  // namespace offq

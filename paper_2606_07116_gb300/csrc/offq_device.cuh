@@ -83,6 +83,16 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
   }
 }
 
+// Waits (bounded, ignoring any abort flag) for the phase with the given parity
+// of a barrier of this CTA: used at teardown, for copies or MMAs in flight.
+__device__ __forceinline__ bool mbar_wait_teardown(uint32_t bar, uint32_t parity) {
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity)) {
+    if (clock64() - t0 > kWaitCycles) return false;
+  }
+  return true;
+}
+
 // As mbar_wait, with a budget of `budget` cycles. A budget below kWaitCycles
 // is a test setting of the failure path: the wait then does not look at its
 // barrier, as if it waited for a flag that nothing sets, and gives up after

@@ -75,6 +75,14 @@ inline bool smem_optin(int bytes) {
   return true;
 }
 
+// Decode form of offq_w4a4_linear (csrc/gemm_decode.cu): tokens it takes at
+// most, and the launch for 1 <= T <= decode_max_tokens() with arguments
+// already checked by offq_w4a4_linear.
+int decode_max_tokens();
+int w4a4_linear_decode(const uint8_t* a_codes, const float* a_scale, const float* a_offset, int64_t T, int64_t N,
+                       int64_t K, int32_t g, const uint8_t* w_codes, const float* w_scale, const float* w_offsum,
+                       void* out, int out_dtype, int64_t ldo, int32_t* acc_debug, cudaStream_t stream);
+
 // Largest input dimension the row quantizer stages in shared memory.
 constexpr int64_t kMaxQuantK = 32768;
 // Largest K of the GEMM: every partial sum stays an integer below 2^24.

@@ -148,6 +148,15 @@ __device__ __forceinline__ uint4 ldg_stream(const uint8_t* p) {
   return r;
 }
 
+// Bulk copy global -> this CTA's shared memory, completing `bytes` on the
+// mbarrier at `bar` (both addresses 16-byte aligned, bytes a multiple of 16).
+__device__ __forceinline__ void bulk_load(uint32_t sdst, const void* gsrc, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   sdst),
+               "l"(gsrc), "r"(bytes), "r"(bar)
+               : "memory");
+}
+
 // Bulk copy shared -> global (async proxy), tracked per thread in bulk groups.
 __device__ __forceinline__ void bulk_store(void* gdst, uint32_t ssrc, uint32_t bytes) {
   asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(gdst), "r"(ssrc), "r"(bytes)

@@ -122,6 +122,10 @@ def test_oracle_codes_through_gemm():
     # along N into 64-column pieces (ragged N at the end), with 4 and 1 offset blocks.
     (512, 1024, 10200, 256, "bf16", None),
     (512, 1024, 10200, 1024, "f32", 10208),
+    # Decode form (T <= 64): more weight blocks than 4 per SM, so each CTA makes two passes of its
+    # accumulator; and a K that is not a multiple of the 4-k-tile bulk copies.
+    (8, 1024, 28672, 1024, "bf16", None),
+    (17, 1920, 640, 128, "f16", None),
 ])
 def test_layers(T, K, N, g, out_dt, ldo):
     _check_layer(T, K, N, g, out_dt, ldo=ldo, seed=T + K)
