@@ -684,3 +684,170 @@ def effective_bits(group: int, code_bits: int = 4, param_bits: int = 16, n_param
 def effective_bits_per_token_offset(K: int, g: int, code_bits: int = 4, param_bits: int = 32) -> float:
     """Bits per activation of this path's layout: one scale per token and one offset per block."""
     return (code_bits * K + param_bits * (1 + K // g)) / K
+
+
+# ---------------------------------------------------------------------------
+# MXFP4 activations and weights with the offset as zero-point
+# (Sec. 3.4 "Generality on Data Formats": micro-scaling formats extended with
+# a zero-point absorb the outlier the same way; the paper leaves it to future
+# work, so the readings below are this build's)
+# ---------------------------------------------------------------------------
+#
+# Element format: MXFP4's E2M1 (OCP Microscaling Formats v1.0): sign, 2-bit
+# exponent, 1-bit mantissa; magnitudes 0, 0.5, 1, 1.5, 2, 3, 4, 6 for the
+# 3-bit codes 0..7, the sign in bit 3 of the nibble.
+# Readings:
+# * Zero-point: the offsetting block's offset (Eq. 5), one per block of g
+#   channels as in the main path, subtracted before the micro-scaled residual is
+#   quantized; it leaves through the weights' dequantized block sums.
+# * Scale: one power of two 2^X per 32 consecutive channels of a row (MXFP4's
+#   shared exponent), X = floor(log2(amax)) - 2, so that amax / 2^X lies in
+#   [4, 8); values round to the nearest E2M1 magnitude, ties to the even
+#   mantissa, and saturate at 6.
+# * Span: within a row no block exponent is more than 6 below the row's
+#   largest one (X = max(X, Xmax - 6); an all-zero block takes Xmax - 6). Every
+#   code times its block's power of two relative to 2^(Xmax - 6) is then an exact
+#   E4M3 value (at most 6 * 2^6 = 384), the form the GEMM multiplies in.
+
+MX_BLOCK = 32
+MX_SPAN = 6
+E2M1_MAG = np.array([0.0, 0.5, 1.0, 1.5, 2.0, 3.0, 4.0, 6.0])
+
+
+def e2m1_value(code: np.ndarray) -> np.ndarray:
+    """Value of 4-bit E2M1 codes (sign in bit 3, magnitude code in bits 0-2)."""
+    code = np.asarray(code, dtype=np.int64)
+    return np.where(code & 8, -1.0, 1.0) * E2M1_MAG[code & 7]
+
+
+def rne_e2m1(v: np.ndarray) -> np.ndarray:
+    """Nearest E2M1 code of each value, ties to the even mantissa (magnitude code
+    with bit 0 clear), magnitudes above 6 saturating to 6. Returns int64 codes."""
+    v = np.asarray(v, dtype=np.float64)
+    a = np.abs(v)
+    d = np.abs(a[..., None] - E2M1_MAG)              # distance to each magnitude
+    best = d.min(axis=-1, keepdims=True)
+    cand = d <= best                                 # nearest magnitudes (two at a tie)
+    even = cand & (np.arange(8) % 2 == 0)
+    pick = np.where(even.any(axis=-1), np.argmax(even, axis=-1), np.argmax(cand, axis=-1))
+    pick = np.where(a >= 6.0, 7, pick)
+    return np.where((v < 0) & (pick > 0), pick | 8, pick).astype(np.int64)
+
+
+def mx_block_exponents(r: np.ndarray, block: int = MX_BLOCK, span: int = MX_SPAN):
+    """Shared exponents X [T, K/block] of the readings above and the row's Xmax [T]."""
+    T, K = r.shape
+    amax = np.abs(r.reshape(T, K // block, block)).max(axis=2)
+    with np.errstate(divide="ignore"):
+        X = np.where(amax > 0, np.floor(np.log2(np.where(amax > 0, amax, 1.0))) - 2, -np.inf)
+    xmax = X.max(axis=1)
+    xmax = np.where(np.isfinite(xmax), xmax, 0.0)     # an all-zero row: any exponent
+    X = np.maximum(X, xmax[:, None] - span)
+    return X.astype(np.int64), xmax.astype(np.int64)
+
+
+def quantize_mx_rows(r: np.ndarray, block: int = MX_BLOCK, span: int = MX_SPAN) -> Dict[str, np.ndarray]:
+    """MXFP4 codes of rows r [T, K] (float64): per block 2^X and E2M1 codes."""
+    T, K = r.shape
+    X, xmax = mx_block_exponents(r, block, span)
+    scale = np.repeat(np.ldexp(1.0, X), block, axis=1)
+    codes = rne_e2m1(r / scale)
+    return {"code": codes, "X": X, "xmax": xmax, "value": e2m1_value(codes) * scale,
+            "shift": X - (xmax[:, None] - span), "row_scale": np.ldexp(1.0, xmax - span)}
+
+
+def quantize_act_mx(x: np.ndarray, g: int, rotate: bool = True, offset: bool = True) -> Dict[str, np.ndarray]:
+    """Rotate -> offset -> MXFP4 residual for token rows X [T, K].
+
+      1. Y = X H / sqrt(g) block-wise when ``rotate`` (Eq. 4).
+      2. o[t, b] = mean of block b of Y when ``offset`` (Eq. 5).
+      3. R = Y - o, quantized per 32 channels (quantize_mx_rows).
+    X_hat = R_hat + o is what the activation stands for.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    T, K = x.shape
+    if K % g != 0 or K % MX_BLOCK != 0:
+        raise ValueError("g and 32 must divide K")
+    G = K // g
+    if rotate:
+        H = _hadamard_f64(g)
+        yu = np.empty_like(x)
+        for b in range(G):
+            sl = slice(b * g, (b + 1) * g)
+            yu[:, sl] = x[:, sl] @ H
+        norm = math.sqrt(g)
+    else:
+        yu = x.copy()
+        norm = 1.0
+    ou = block_offsets(yu, g) if offset else np.zeros((T, G))
+    r = subtract_offsets(yu, ou, g) / norm
+    res = quantize_mx_rows(r)
+    res.update({"y": yu / norm, "offset": ou / norm, "residual": r})
+    return res
+
+
+def prepare_weight_mx(w: np.ndarray, g: int, rotate: bool = True) -> Dict[str, np.ndarray]:
+    """MXFP4 weights W [N, K] per output row (no offset): W_eff = W blockdiag(H_g) / sqrt(g)
+    when the input takes the online rotation, then quantize_mx_rows. ``offsum[b, n]`` is the
+    block sum of the operand values code * 2^shift (the dequantized weights over the row's
+    2^(Xmax - 6)), which the offsets meet in the GEMM."""
+    res = quantize_act_mx(w, g, rotate=rotate, offset=False)
+    N, K = res["code"].shape
+    opv = e2m1_value(res["code"]) * np.repeat(np.ldexp(1.0, res["shift"]), MX_BLOCK, axis=1)
+    res["operand"] = opv
+    res["offsum"] = opv.reshape(N, K // g, g).sum(axis=2).T
+    return res
+
+
+def mx_linear(a: Dict[str, np.ndarray], w: Dict[str, np.ndarray], g: int) -> Dict[str, np.ndarray]:
+    """y = (R_hat + o) W_hat^T in float64, from the codes of quantize_act_mx and
+    prepare_weight_mx: the residual product plus the offsets' block-sum term."""
+    K = a["code"].shape[1]
+    ra = a["value"]
+    wv = w["value"]
+    T = ra.shape[0]
+    o = np.repeat(a["offset"], g, axis=1)
+    y = ra @ wv.T + o @ wv.T
+    # The same value in the factored form the kernels use.
+    opa = e2m1_value(a["code"]) * np.repeat(np.ldexp(1.0, a["shift"]), MX_BLOCK, axis=1)
+    acc = opa @ w["operand"].T
+    y2 = np.outer(a["row_scale"], w["row_scale"]) * acc + w["row_scale"][None, :] * (a["offset"] @ w["offsum"])
+    return {"y": y, "y_factored": y2, "acc": acc}
+
+
+def pack_mx_codes(code: np.ndarray) -> np.ndarray:
+    """E2M1 codes [.., K] (int 0..15) -> bytes [.., K/2], even channel in the low nibble."""
+    code = np.asarray(code, dtype=np.int64)
+    if np.any((code < 0) | (code > 15)):
+        raise ValueError("code out of range")
+    u = code.astype(np.uint8)
+    return (u[..., 0::2] | (u[..., 1::2] << 4)).astype(np.uint8)
+
+
+def unpack_mx_codes(packed: np.ndarray) -> np.ndarray:
+    p = np.asarray(packed, dtype=np.uint8).astype(np.int64)
+    out = np.empty(p.shape[:-1] + (2 * p.shape[-1],), dtype=np.int64)
+    out[..., 0::2] = p & 0xF
+    out[..., 1::2] = p >> 4
+    return out
+
+
+def tile_mx_shifts(shift: np.ndarray) -> np.ndarray:
+    """Block shifts [R, K/32] (0..6) -> the tiled byte layout the GEMM reads: rows padded
+    to 32, for 32-row block rb and k-tile kt (4 blocks of 32 channels) the 4 shifts of
+    row r at ((rb * (K/128) + kt) * 32 + r % 32) * 4 + (block % 4)."""
+    s = np.asarray(shift, dtype=np.int64)
+    R, B = s.shape
+    if B % 4:
+        raise ValueError("K must be a multiple of 128")
+    Rp = -(-R // TILE_ROWS) * TILE_ROWS
+    t = np.zeros((Rp, B), dtype=np.uint8)
+    t[:R] = s.astype(np.uint8)
+    return t.reshape(Rp // TILE_ROWS, TILE_ROWS, B // 4, 4).transpose(0, 2, 1, 3).reshape(-1).copy()
+
+
+def untile_mx_shifts(tiled: np.ndarray, R: int, K: int) -> np.ndarray:
+    t = np.asarray(tiled, dtype=np.uint8).reshape(-1)
+    Rp = -(-R // TILE_ROWS) * TILE_ROWS
+    B = K // MX_BLOCK
+    return t[:Rp * B].reshape(Rp // TILE_ROWS, B // 4, TILE_ROWS, 4).transpose(0, 2, 1, 3).reshape(Rp, B)[:R].astype(np.int64)

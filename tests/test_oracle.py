@@ -667,3 +667,111 @@ def test_builder_turns_the_outlier_into_group_offsets():
     q_before = O.quantize_act(res["X"], g, rotate=False, offset=False)["scale"]
     q_after = O.quantize_act(Xr, g, rotate=False, offset=True)["scale"]
     assert np.all(q_after < 0.5 * q_before) and q_after.mean() < 0.25 * q_before.mean()
+
+
+# --------------------------------------------------------------------------
+# MXFP4 residuals with the offset as zero-point (Sec. 3.4, "Generality on
+# Data Formats"; readings with quantize_mx_rows).
+# --------------------------------------------------------------------------
+
+def test_mx_rounding_fixture(golden_dir):
+    d = _load(golden_dir, "mxfp4_blocks.json")
+    v = np.array([e["v"] for e in d["rounding"]])
+    np.testing.assert_array_equal(O.rne_e2m1(v), [e["code"] for e in d["rounding"]])
+    for blk in d["blocks"]:
+        res = O.quantize_mx_rows(np.array([blk["x"]]))
+        assert res["X"][0, 0] == blk["X"]
+        np.testing.assert_array_equal(res["code"][0], blk["code"])
+
+
+def test_mx_grid_points_round_trip_and_error_bound():
+    # Every E2M1 value comes back as its own code (-0 as +0).
+    codes = np.arange(16)
+    back = O.rne_e2m1(O.e2m1_value(codes))
+    np.testing.assert_array_equal(back, np.where(codes == 8, 0, codes))
+    # Monotone, and within half the local grid gap of the value (saturated values aside).
+    v = np.linspace(-8, 8, 20001)
+    q = O.e2m1_value(O.rne_e2m1(v))
+    assert np.all(np.diff(q) >= 0)
+    grid = np.concatenate([-O.E2M1_MAG[::-1], O.E2M1_MAG[1:]])
+    inside = np.abs(v) <= 6
+    gaps = np.diff(grid)
+    idx = np.clip(np.searchsorted(grid, v[inside]) - 1, 0, len(gaps) - 1)
+    assert np.all(np.abs(v[inside] - q[inside]) <= gaps[idx] / 2 + 1e-15)
+
+
+def test_mx_block_exponent_places_the_largest_value_on_the_top_binades():
+    rng = np.random.default_rng(45)
+    r = rng.standard_normal((64, 256)) * np.exp(rng.uniform(-8, 8, size=(64, 1)))
+    res = O.quantize_mx_rows(r)
+    blk = np.abs(r.reshape(64, 8, 32)).max(axis=2)
+    ratio = blk / np.ldexp(1.0, res["X"])
+    unclamped = res["X"] > res["xmax"][:, None] - O.MX_SPAN
+    assert np.all((ratio[unclamped] >= 4) & (ratio[unclamped] < 8))
+    # The block maximum codes to magnitude 4 or 6 (or saturates at 6).
+    mags = np.abs(O.e2m1_value(res["code"])).reshape(64, 8, 32).max(axis=2)
+    assert np.all(np.isin(mags[unclamped], [4.0, 6.0]))
+    # Reconstruction error: half a grid gap (at most 2^X) below saturation, 2 * 2^X at it.
+    err = np.abs(res["value"] - r).reshape(64, 8, 32).max(axis=2)
+    assert np.all(err <= 2 * np.ldexp(1.0, res["X"]) + 1e-300)
+
+
+def test_mx_span_clamp_and_zero_blocks():
+    r = np.zeros((1, 128))
+    r[0, :32] = 1000.0 * np.linspace(-1, 1, 32)   # X = floor(log2 1000) - 2 = 7
+    r[0, 32:64] = 1e-3                            # would be X = -12; clamped to 7 - 6 = 1
+    res = O.quantize_mx_rows(r)
+    np.testing.assert_array_equal(res["X"][0], [7, 1, 1, 1])
+    np.testing.assert_array_equal(res["shift"][0], [6, 0, 0, 0])
+    assert np.all(res["code"][0, 32:] == 0)       # 1e-3 / 2 rounds to 0
+    assert res["row_scale"][0] == 2.0
+
+
+def test_mx_offset_absorbs_the_outlier():
+    """Eq. 5 through the MX residual: pairs [x1, x2] rotated by H_2 leave the constant
+    offset x1 / sqrt 2 and residuals +-x2 / sqrt 2, so the codes and exponents do not
+    depend on the outlier x1."""
+    x2 = np.array([0.3, -1.7, 2.5, 0.9] * 8)
+    base = np.stack([np.zeros(32), x2], axis=1).reshape(1, 64)
+    for x1 in (0.0, 50.0, -400.0, 1e4):
+        x = base.copy()
+        x[0, 0::2] = x1
+        res = O.quantize_act_mx(x, 2, rotate=True, offset=True)
+        np.testing.assert_allclose(res["offset"][0], x1 / math.sqrt(2), rtol=1e-14)
+        ref = O.quantize_act_mx(base, 2, rotate=True, offset=True)
+        np.testing.assert_array_equal(res["code"], ref["code"])
+        np.testing.assert_array_equal(res["X"], ref["X"])
+
+
+def test_mx_linear_equals_the_dequantized_product():
+    rng = np.random.default_rng(46)
+    T, K, N, g = 12, 512, 40, 256
+    x = rng.standard_normal((T, K))
+    x[:, ::g] += 80.0
+    w = rng.standard_normal((N, K)) * 0.02
+    a = O.quantize_act_mx(x, g)
+    wp = O.prepare_weight_mx(w, g)
+    res = O.mx_linear(a, wp, g)
+    xh = a["value"] + np.repeat(a["offset"], g, axis=1)
+    ref = xh @ wp["value"].T
+    np.testing.assert_allclose(res["y"], ref, rtol=1e-12, atol=1e-12 * np.abs(ref).max())
+    np.testing.assert_allclose(res["y_factored"], ref, rtol=1e-12, atol=1e-12 * np.abs(ref).max())
+    # The operand values are exact E4M3 numbers: multiples of 2^-1 up to 384.
+    opv = np.abs(wp["operand"])
+    assert opv.max() <= 384 and np.all(opv * 2 == np.round(opv * 2))
+    # And the layer approximates the unquantized one (the rotation cancels).
+    y32 = O.linear_reference(x, w)
+    assert np.linalg.norm(res["y"] - y32) < 0.3 * np.linalg.norm(y32)
+
+
+def test_mx_pack_and_shift_layouts():
+    rng = np.random.default_rng(47)
+    code = rng.integers(0, 16, size=(37, 256))
+    p = O.pack_mx_codes(code)
+    assert p[0, 0] == (code[0, 0] | (code[0, 1] << 4))
+    np.testing.assert_array_equal(O.unpack_mx_codes(p), code)
+    sh = rng.integers(0, 7, size=(37, 8))
+    t = O.tile_mx_shifts(sh)
+    # Row 33 (second 32-row block, row 1), block 5 (k-tile 1, position 1).
+    assert t[((1 * 2 + 1) * 32 + 1) * 4 + 1] == sh[33, 5]
+    np.testing.assert_array_equal(O.untile_mx_shifts(t, 37, 256), sh)
