@@ -364,11 +364,71 @@ class GroupStep:
                 rec("gemm")
 
 
-def time_group_path(w, T, device, args, rank, flush_l2, barrier, stream, fp8_peak, peaks):
-    """Step time and per-kernel rates of the per-group path (same protocol as the main step)."""
+class MxStep:
+    """The same layers in MXFP4 with the offsets as zero-points (Sec. 3.4's
+    extension to micro-scaled formats): per site the MX quantizer (rotation and
+    offsets as the main path), then its layers' MX GEMMs (E2M1 codes widened to
+    exact E4M3 with their 32-channel shifts, the offsets' rank-G epilogue)."""
+
+    def __init__(self, w: W.Workload, T: int, device, seed_base: int = 0):
+        import torch
+        from paper_2606_07116_gb300 import offq as Q
+        self.torch, self.Q, self.T = torch, Q, T
+        dt = torch.bfloat16 if w.x_dtype == "bf16" else torch.float32
+        self.sites = []
+        for i, (name, K, rotate, layers) in enumerate(sites(w)):
+            x = device_activations(T, K, w, seed=seed_base + 10 + i, device=device).to(dt)
+            g = W.block_for(K)
+            gemms = []
+            for l in layers:
+                wt = device_weights(l.N, l.K, seed=seed_base + 100 + len(self.sites) * 10 + len(gemms), device=device)
+                wc, wsh, wsc, wsum = Q.prepare_weight_mx(wt, g, rotate=l.rotate)
+                del wt
+                gemms.append({"layer": l, "codes": wc, "shifts": wsh, "scale": wsc, "offsum": wsum,
+                              "out": torch.empty((T, l.N), dtype=torch.bfloat16, device=device)})
+            self.sites.append({"K": K, "g": g, "flags": (Q.OFFQ_ROTATE if rotate else 0) | Q.OFFQ_OFFSET, "x": x,
+                               "codes": torch.empty((Q.padded_rows(T), K // 2), dtype=torch.uint8, device=device),
+                               "shifts": torch.empty((Q.mx_shift_bytes(T, K),), dtype=torch.uint8, device=device),
+                               "scale": torch.empty((T,), dtype=torch.float32, device=device),
+                               "off": torch.empty((T, K // g), dtype=torch.float32, device=device),
+                               "gemms": gemms})
+        torch.cuda.synchronize(device)
+
+    def launches_per_step(self):
+        return len(self.sites) + sum(len(s["gemms"]) for s in self.sites)
+
+    def quant_bytes(self):
+        T = self.T
+        return sum(T * s["K"] * s["x"].element_size() + T * s["K"] // 2 + T * s["K"] // 32 + 4 * T
+                   + 4 * T * (s["K"] // s["g"]) for s in self.sites)
+
+    def run(self, stream, timers=None):
+        Q, torch, T = self.Q, self.torch, self.T
+
+        def rec(kind):
+            if timers is not None:
+                e = torch.cuda.Event(enable_timing=True)
+                e.record(stream)
+                timers.setdefault(kind, []).append(e)
+
+        for s in self.sites:
+            rec("quant")
+            Q.offq_quantize_act_mx(s["x"], T, s["K"], s["x"].stride(0), s["g"], s["flags"], s["codes"],
+                                   s["shifts"], s["scale"], s["off"], stream)
+            rec("quant")
+            for gm in s["gemms"]:
+                l = gm["layer"]
+                rec("gemm")
+                Q.offq_mx_linear(s["codes"], s["shifts"], s["scale"], s["off"], T, l.N, l.K, s["g"], gm["codes"],
+                                 gm["shifts"], gm["scale"], gm["offsum"], gm["out"], gm["out"].stride(0), stream)
+                rec("gemm")
+
+
+def time_variant_path(step_cls, w, T, device, args, rank, flush_l2, barrier, stream):
+    """Step time and per-kernel rates of a variant path (same protocol as the main step)."""
     import torch
     from paper_2606_07116_gb300 import offq as Q
-    gstep = GroupStep(w, T, device, seed_base=rank_seed_base(rank))
+    gstep = step_cls(w, T, device, seed_base=rank_seed_base(rank))
     for _ in range(args.warmup):
         flush_l2()
         gstep.run(stream)
@@ -392,7 +452,7 @@ def time_group_path(w, T, device, args, rank, flush_l2, barrier, stream, fp8_pea
     torch.cuda.synchronize(device)
     st = Q.offq_get_device_status(stream)
     if st != Q.OFFQ_OK:
-        raise RuntimeError(f"device status after the group path: {Q.status_string(st)}")
+        raise RuntimeError(f"device status after {step_cls.__name__}: {Q.status_string(st)}")
     gemm_ms = sum(_pair_times(timers["gemm"])) / kb
     quant_ms = sum(_pair_times(timers["quant"])) / kb
     return gstep, dev_ms / steps, gemm_ms, quant_ms
@@ -859,10 +919,10 @@ def run_gpu(args, rank, world, local_rank):
     # The GEMMs are timed per call (an event pair around each launch), so the
     # burst rate is their denominator.
     fp8_peak = peaks["bf16_tflops"] * FP8_PER_BF16
-    group = None
+    group = mxfp4 = None
     if not args.no_group:
-        gstep, g_ms, g_gemm_ms, g_quant_ms = time_group_path(w, T, device, args, rank, flush_l2, barrier, stream,
-                                                             fp8_peak, peaks)
+        gstep, g_ms, g_gemm_ms, g_quant_ms = time_variant_path(GroupStep, w, T, device, args, rank, flush_l2,
+                                                               barrier, stream)
         (g_ms,) = reduce_over_ranks([g_ms], dist, device)
         g_gemm_tflops = ops / (g_gemm_ms * 1e-3) / 1e12
         g_quant_gbs = gstep.quant_bytes() / (g_quant_ms * 1e-3) / 1e9
@@ -879,6 +939,26 @@ def run_gpu(args, rank, world, local_rank):
                           "bytes_per_step": gstep.quant_bytes()},
             "gpu_launches": gstep.launches_per_step() * args.steps,
         }
+        del gstep
+        mstep, m_ms, m_gemm_ms, m_quant_ms = time_variant_path(MxStep, w, T, device, args, rank, flush_l2,
+                                                               barrier, stream)
+        (m_ms,) = reduce_over_ranks([m_ms], dist, device)
+        m_gemm_tflops = ops / (m_gemm_ms * 1e-3) / 1e12
+        m_quant_gbs = mstep.quant_bytes() / (m_quant_ms * 1e-3) / 1e9
+        mxfp4 = {
+            "what": "the same layers in MXFP4 (E2M1 codes, a power-of-two scale per 32 channels) with the offsets "
+                    "as zero-points: offq_quantize_act_mx + offq_mx_linear, no KV4",
+            "value": round(job_tops(ops, world, m_ms), 3), "unit": UNIT, "ms_per_step": round(m_ms, 4),
+            "roofline": {"bound": "tensor", "kernel": "w4a4_gemm_kernel<MX> (tcgen05.mma kind::f8f6f4, codes "
+                                                      "widened with their block shifts in the converter warps)",
+                         "achieved": round(m_gemm_tflops, 2), "peak": round(fp8_peak, 1), "unit": "TFLOP/s",
+                         "frac": round(m_gemm_tflops / fp8_peak, 4), "gemm_ms_per_step": round(m_gemm_ms, 4)},
+            "act_quant": {"value": round(m_quant_gbs, 1), "unit": "GB/s", "peak": peaks["hbm_gbs"],
+                          "frac": round(m_quant_gbs / peaks["hbm_gbs"], 4), "ms_per_step": round(m_quant_ms, 4),
+                          "bytes_per_step": mstep.quant_bytes()},
+            "gpu_launches": mstep.launches_per_step() * args.steps,
+        }
+        del mstep
     gemm_tflops = ops * args.steps / (gemm_ms * 1e-3) / 1e12
     quant_gbs = step.quant_bytes() * args.steps / (quant_ms * 1e-3) / 1e9
     kv_gbs = step.kv_bytes() * args.steps / (kv_ms * 1e-3) / 1e9 if kv_ms > 0 else None
@@ -921,6 +1001,8 @@ def run_gpu(args, rank, world, local_rank):
     }
     if group is not None:
         line["group_asym"] = group
+    if mxfp4 is not None:
+        line["mxfp4"] = mxfp4
     if not args.no_group and w.kv_heads and w.head_dim == 128:
         line["kv4_rotated"] = time_key_rotation(w, T, device, args, flush_l2, stream)
     if not args.no_group:

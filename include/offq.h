@@ -478,6 +478,64 @@ int offq_sorted_grouping(const float* mag, int64_t D, int32_t G, int32_t* perm);
 int offq_fuse_rotation(const float* W, int64_t N, int64_t D, const float* v, const int32_t* perm, int32_t g,
                        float* out, void* stream);
 
+/*
+ * MXFP4 residuals with the offset as zero-point (paper Sec. 3.4 "Generality
+ * on Data Formats": micro-scaling formats extended with a zero-point per block
+ * absorb the outlier offset; the paper leaves the extension to future work).
+ *
+ * offq_quantize_act_mx -- for each token row x (K channels):
+ *   y = x_b H_g / sqrt(g) per block b of g channels   if OFFQ_ROTATE (else y = x)
+ *   o[b] = mean(y_b) if OFFQ_OFFSET (else 0),  r = y - o
+ * then per 32 channels j of r (MXFP4's shared exponent and E2M1 elements):
+ *   X_j = floor(log2(max |r_j|)) - 2, raised to at least Xmax - 6 (Xmax the
+ *         row's largest; an all-zero block takes Xmax - 6),
+ *   e = E2M1 code of r / 2^X_j: nearest of the magnitudes 0, 0.5, 1, 1.5, 2, 3,
+ *       4, 6 (codes 0..7), ties to the even code, saturating at 6; sign in bit 3.
+ * r ~ value(e) * 2^X_j, so x ~ value(e) * 2^X_j + o.
+ *
+ *   x, T, K, ldx  as offq_quantize_act; K a multiple of g and of 128, K <= 32768.
+ *   g         block of the rotation and of the offsets, power of two in [32, 8192].
+ *   codes     device, offq_act_codes_bytes(T, K) bytes: e as nibbles, two per byte
+ *             (even channel low), in the tiled operand layout, 16-B aligned.
+ *   shifts    device, offq_mx_shift_bytes(T, K) bytes, 4-B aligned: sh_j = X_j -
+ *             (Xmax - 6) in 0..6, byte ((r/32 * K/128 + j/4) * 32 + r%32) * 4 + j%4
+ *             for row r and block j (the four shifts of a row's 128-code k-tile
+ *             are one 32-bit word).
+ *   row_scale device, [T] float32: 2^(Xmax - 6).
+ *   offset    device, [T][K/g] float32; required with OFFQ_OFFSET.
+ * Rows of the last 32-row group beyond T are left as they are.
+ */
+int offq_quantize_act_mx(const void* x, int x_dtype, int64_t T, int64_t K, int64_t ldx, int32_t g, int32_t flags,
+                         uint8_t* codes, uint8_t* shifts, float* row_scale, float* offset, void* stream);
+
+/*
+ * offq_prepare_weight_mx -- offline: MXFP4 weights W [N][K] (row-major, dtype
+ * OFFQ_F32/BF16/F16), per output row as offq_quantize_act_mx without offsets,
+ * after the rotation fused into W when `rotate` (W_eff = W blockdiag(H_g)/sqrt(g)).
+ *   w_codes, w_shifts, w_scale  as codes, shifts, row_scale above (N rows); the
+ *             padding rows of the last 32-row group are zero codes and shifts.
+ *   w_offsum  device, [K/g][N] float32: R[b][n] = sum over block b of
+ *             value(e) * 2^sh (the operand values; exact, multiples of 1/2).
+ */
+int offq_prepare_weight_mx(const void* w, int dtype, int64_t N, int64_t K, int32_t g, int32_t rotate,
+                           uint8_t* w_codes, uint8_t* w_shifts, float* w_scale, float* w_offsum, void* stream);
+
+/*
+ * offq_mx_linear -- the W4A4 linear of MXFP4 operands:
+ *   y[t][n] = s_w[n] * ( s_a[t] * sum_k A[t][k] W[n][k] + sum_b o[t][b] R[b][n] ),
+ * A = value(e_a) * 2^sh_a and W = value(e_w) * 2^sh_w, each an exact E4M3 value,
+ * multiplied on the tensor cores (kind::f8f6f4) with fp32 accumulation,
+ * s_a / s_w the row scales. Arguments as offq_w4a4_linear (no acc_debug), plus
+ * the shift buffers; K a multiple of 128 and of g.
+ */
+int offq_mx_linear(const uint8_t* a_codes, const uint8_t* a_shifts, const float* a_scale, const float* a_offset,
+                   int64_t T, int64_t N, int64_t K, int32_t g, const uint8_t* w_codes, const uint8_t* w_shifts,
+                   const float* w_scale, const float* w_offsum, void* out, int out_dtype, int64_t ldo, void* stream);
+
+/* Bytes of a tiled MXFP4 shift buffer for R rows of K channels (-1 unless K is
+ * a positive multiple of 128 and R >= 0): ceil(R/32) * 32 * K / 32. */
+int64_t offq_mx_shift_bytes(int64_t R, int64_t K);
+
 /* Bytes of a tiled activation-code buffer for T rows of K codes (-1 if K is
  * not a positive multiple of 32 or T < 0): ceil(T/32) * 32 * K / 2. */
 int64_t offq_act_codes_bytes(int64_t T, int64_t K);

@@ -145,7 +145,17 @@ struct GemmParams {
   int kchunks;             // K / 32
   int vec_ok;              // rowsum and w_scale rows are 16-byte aligned
   int async_out;           // 16-bit output and N % 8 == 0: one-block rows leave by bulk copy
+  // MXFP4 operands (kFmtMx): per row and 32-channel block a shift 0..6, tiled as
+  // ((row/32 * K/128 + k-tile) * 32 + row%32) * 4 + block%4.
+  const uint8_t* a_shifts;
+  const uint8_t* w_shifts;
+  int nkt;                 // K / 128
 };
+
+// Operand formats of the pair kernel: 4-bit integers (activations u = q + 8,
+// weights sign-magnitude), or MXFP4 E2M1 codes whose block shifts place each
+// code times its block's power of two on the E4M3 grid.
+constexpr int kFmtInt4 = 0, kFmtMx = 1;
 
 // Loads the four 16-byte chunks of k-tile kt of one row of a tiled code matrix
 // (zeros where the row block or the chunk does not exist).
@@ -198,9 +208,13 @@ __device__ __forceinline__ int b_block(const GemmParams& p, int tile, uint32_t r
 // tile end. Layers with several
 // offset blocks run a separate instantiation, so the register allocation of
 // the common one-block kernel does not carry the G-term epilogue loop.
-template <int OUT, bool kOneBlock, bool kUnstaged>
+template <int OUT, bool kOneBlock, bool kUnstaged, int FMT>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kThreads, 1)
     w4a4_gemm_kernel(const GemmParams p) {
+  // Integer operands are integers times 2^-9 (the accumulator carries 2^-18) and
+  // the activations carry +8; MXFP4 operands are the values themselves.
+  constexpr bool kPlus8 = FMT == kFmtInt4;
+  constexpr float kAccScale = FMT == kFmtInt4 ? 262144.0f : 1.0f;
   extern __shared__ uint8_t smem_raw[];
   using SL = Smem<kOneBlock>;
   using RL = Roles<kOneBlock>;
@@ -300,11 +314,32 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
     const int rb_count = is_a ? p.t_blocks : p.n_blocks;
     // This lane's first byte of the row block a tile needs (nullptr: the block
     // lies past the buffer's rows). Computed once per tile, not per load.
+    const uint8_t* shifts = is_a ? p.a_shifts : p.w_shifts;
     auto block_ptr = [&](int tile) -> const uint8_t* {
       const int rb = is_a ? a_block(p, tile, rank, quarter) : b_block(p, tile, rank, wb);
       return rb < rb_count ? codes + static_cast<int64_t>(rb) * p.kchunks * 512 + lane * 16 : nullptr;
     };
+    // MXFP4: this lane's shift words of the row block a tile needs (nullptr as above).
+    auto shift_ptr = [&](int tile) -> const uint8_t* {
+      if constexpr (FMT == kFmtMx) {
+        const int rb = is_a ? a_block(p, tile, rank, quarter) : b_block(p, tile, rank, wb);
+        return rb < rb_count ? shifts + (static_cast<int64_t>(rb) * p.nkt * 32 + lane) * 4 : nullptr;
+      } else {
+        (void)tile;
+        return nullptr;
+      }
+    };
+    auto load_shift = [&](const uint8_t* sblk, int kt) -> uint32_t {
+      if constexpr (FMT == kFmtMx) {
+        return sblk != nullptr ? __ldg(reinterpret_cast<const uint32_t*>(sblk + kt * 128)) : 0u;
+      } else {
+        (void)sblk;
+        (void)kt;
+        return 0u;
+      }
+    };
     uint4 ring[kPrefetch][kChunksPerKt];
+    uint32_t sring[kPrefetch];
     int ld_tile = cluster, ld_kt = 0;  // next k-tile to load
     auto advance1 = [&](int& tile, int& kt) {
       if (++kt == nk) {
@@ -322,13 +357,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
     const int start_tile = ld_tile, start_kt = ld_kt;
 #pragma unroll
     for (int i = 0; i < kPrefetch; ++i) {
-      if (ld_tile < num_tiles) load_kt(block_ptr(ld_tile), p.kchunks, ld_kt, ring[i]);
+      sring[i] = 0u;
+      if (ld_tile < num_tiles) {
+        load_kt(block_ptr(ld_tile), p.kchunks, ld_kt, ring[i]);
+        sring[i] = load_shift(shift_ptr(ld_tile), ld_kt);
+      }
       advance(ld_tile, ld_kt);
     }
     int tile = start_tile, kt = start_kt;
     int s = part, phase = 0;  // stage and phase parity of this warp's k-tile g (g == part mod split)
-    int blk_tile = ld_tile;  // the tile whose row block blk points into
+    int blk_tile = ld_tile;  // the tile whose row block blk (and sblk) points into
     const uint8_t* blk = ld_tile < num_tiles ? block_ptr(ld_tile) : nullptr;
+    const uint8_t* sblk = ld_tile < num_tiles ? shift_ptr(ld_tile) : nullptr;
     bool run = tile < num_tiles;
     while (run) {
 #pragma unroll
@@ -345,10 +385,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
           uint32_t f8[32];
 #pragma unroll
           for (int j = 0; j < kChunksPerKt; ++j) {
-            widen_act(ring[slot][j].x, f8[8 * j + 0], f8[8 * j + 1]);
-            widen_act(ring[slot][j].y, f8[8 * j + 2], f8[8 * j + 3]);
-            widen_act(ring[slot][j].z, f8[8 * j + 4], f8[8 * j + 5]);
-            widen_act(ring[slot][j].w, f8[8 * j + 6], f8[8 * j + 7]);
+            if constexpr (FMT == kFmtMx) {
+              uint32_t llo, lhi;
+              mx_lut((sring[slot] >> (8 * j)) & 0xFFu, llo, lhi);
+              widen_mx(ring[slot][j].x, llo, lhi, f8[8 * j + 0], f8[8 * j + 1]);
+              widen_mx(ring[slot][j].y, llo, lhi, f8[8 * j + 2], f8[8 * j + 3]);
+              widen_mx(ring[slot][j].z, llo, lhi, f8[8 * j + 4], f8[8 * j + 5]);
+              widen_mx(ring[slot][j].w, llo, lhi, f8[8 * j + 6], f8[8 * j + 7]);
+            } else {
+              widen_act(ring[slot][j].x, f8[8 * j + 0], f8[8 * j + 1]);
+              widen_act(ring[slot][j].y, f8[8 * j + 2], f8[8 * j + 3]);
+              widen_act(ring[slot][j].z, f8[8 * j + 4], f8[8 * j + 5]);
+              widen_act(ring[slot][j].w, f8[8 * j + 6], f8[8 * j + 7]);
+            }
           }
           tmem_st_32cols(tmem + (static_cast<uint32_t>(quarter * 32) << 16) + kACol0 + s * kAColsPerStage, f8);
           tmem_st_wait();
@@ -359,10 +408,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
 #pragma unroll
           for (int j = 0; j < kChunksPerKt; ++j) {
             uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
-            widen_weight(ring[slot][j].x, a0, a1);
-            widen_weight(ring[slot][j].y, a2, a3);
-            widen_weight(ring[slot][j].z, b0, b1);
-            widen_weight(ring[slot][j].w, b2, b3);
+            if constexpr (FMT == kFmtMx) {
+              uint32_t llo, lhi;
+              mx_lut((sring[slot] >> (8 * j)) & 0xFFu, llo, lhi);
+              widen_mx(ring[slot][j].x, llo, lhi, a0, a1);
+              widen_mx(ring[slot][j].y, llo, lhi, a2, a3);
+              widen_mx(ring[slot][j].z, llo, lhi, b0, b1);
+              widen_mx(ring[slot][j].w, llo, lhi, b2, b3);
+            } else {
+              widen_weight(ring[slot][j].x, a0, a1);
+              widen_weight(ring[slot][j].y, a2, a3);
+              widen_weight(ring[slot][j].z, b0, b1);
+              widen_weight(ring[slot][j].w, b2, b3);
+            }
             sts128(st + (((2 * j) ^ (r & 7)) << 4), a0, a1, a2, a3);
             sts128(st + (((2 * j + 1) ^ (r & 7)) << 4), b0, b1, b2, b3);
           }
@@ -375,8 +433,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
           if (ld_tile != blk_tile) {
             blk_tile = ld_tile;
             blk = block_ptr(ld_tile);
+            sblk = shift_ptr(ld_tile);
           }
           load_kt(blk, p.kchunks, ld_kt, ring[slot]);
+          sring[slot] = load_shift(sblk, ld_kt);
         }
         advance(ld_tile, ld_kt);
         advance(tile, kt);
@@ -430,7 +490,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
         }
       }
       epi_sync<kEpiWarps>();
-      if (!kOneBlock && staged) {
+      if (!kOneBlock && staged && kPlus8) {
         // Rt[n] * 8 * 2^-18 = sum_b R[b][n] * 2^-15: integers, exact in fp32.
         for (int i = et; i < BN; i += kEpiWarps * 32) {
           float r = 0.f;
@@ -525,7 +585,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
 #pragma unroll
           for (int jj = 0; jj < CW; ++jj) {
             // (acc' - 8 Rt) 2^-18, then * 2^18: both steps exact.
-            const float accf = (__uint_as_float(acc[jj]) + Rt[jc + jj]) * 262144.0f;
+            const float accf = kPlus8 ? (__uint_as_float(acc[jj]) + Rt[jc + jj]) * kAccScale : __uint_as_float(acc[jj]);
             z[jj] = Ws[jc + jj] * fmaf(sa, accf, __uint_as_float(cr[jj]));
           }
           store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, z, nvalid);
@@ -542,7 +602,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
         // its product with acc are exact). 16-bit rows go to shared memory and
         // leave by one bulk copy per row once the accumulator is read, so the
         // tile's output write overlaps the next tile's MMAs.
-        const float sa2 = Sa[rl] * 262144.0f;
+        const float sa2 = Sa[rl] * kAccScale;
         const float ob = Os[rl * kStageGp];
         const uint64_t SA2 = pack2(sa2, sa2), OB = pack2(ob, ob);
         const uint64_t M8 = pack2(-0x1p-15f, -0x1p-15f);  // -8 * 2^-18
@@ -566,10 +626,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
             for (int q4 = 0; q4 < CW / 4; ++q4) {
               const float4 rv = r4[q4], wv = w4[q4];
               const uint64_t R0 = pack2(rv.x, rv.y), R1 = pack2(rv.z, rv.w);
-              const uint64_t A0 =
-                  fma2v(R0, M8, pack2(__uint_as_float(acc[4 * q4]), __uint_as_float(acc[4 * q4 + 1])));
-              const uint64_t A1 =
-                  fma2v(R1, M8, pack2(__uint_as_float(acc[4 * q4 + 2]), __uint_as_float(acc[4 * q4 + 3])));
+              uint64_t A0 = pack2(__uint_as_float(acc[4 * q4]), __uint_as_float(acc[4 * q4 + 1]));
+              uint64_t A1 = pack2(__uint_as_float(acc[4 * q4 + 2]), __uint_as_float(acc[4 * q4 + 3]));
+              if constexpr (kPlus8) {
+                A0 = fma2v(R0, M8, A0);
+                A1 = fma2v(R1, M8, A1);
+              }
               unpack2(mul2v(pack2(wv.x, wv.y), fma2v(SA2, A0, mul2v(OB, R0))), y[4 * q4], y[4 * q4 + 1]);
               unpack2(mul2v(pack2(wv.z, wv.w), fma2v(SA2, A1, mul2v(OB, R1))), y[4 * q4 + 2], y[4 * q4 + 3]);
             }
@@ -631,12 +693,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
               if (jj < nvalid) {
                 const float r = __ldg(rb + jj);
                 y[jj] = fmaf(ob, r, y[jj]);
-                a[jj] = fmaf(r, -0x1p-15f, a[jj]);  // acc' - 8 R, in units of 2^-18: exact
+                if (kPlus8) a[jj] = fmaf(r, -0x1p-15f, a[jj]);  // acc' - 8 R, in units of 2^-18: exact
               }
           }
 #pragma unroll
           for (int jj = 0; jj < CW; ++jj) {
-            const float accf = a[jj] * 262144.0f;
+            const float accf = a[jj] * kAccScale;
             y[jj] = jj < nvalid ? __ldg(p.w_scale + nb + jj) * fmaf(sa, accf, y[jj]) : 0.f;
           }
           store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, y, nvalid);
@@ -684,12 +746,12 @@ int num_sms() {
   return sms[dev];
 }
 
-template <int OUT, bool kOneBlock, bool kUnstaged = false>
+template <int OUT, bool kOneBlock, bool kUnstaged, int FMT>
 int launch_gemm(const GemmParams& p, cudaStream_t s) {
-  auto kern = w4a4_gemm_kernel<OUT, kOneBlock, kUnstaged>;
+  auto kern = w4a4_gemm_kernel<OUT, kOneBlock, kUnstaged, FMT>;
   constexpr int kThreads = Roles<kOneBlock>::kThreads;
   constexpr int kSmemBytes = Smem<kOneBlock>::kBytes;
-  if (!smem_optin<w4a4_gemm_kernel<OUT, kOneBlock, kUnstaged>>(kSmemBytes)) return OFFQ_ERR_CUDA;
+  if (!smem_optin<w4a4_gemm_kernel<OUT, kOneBlock, kUnstaged, FMT>>(kSmemBytes)) return OFFQ_ERR_CUDA;
   const int sms = num_sms();
   if (sms < 2) return OFFQ_ERR_CUDA;
   const int tiles = p.m_pairs * p.n_tiles;
@@ -697,30 +759,30 @@ int launch_gemm(const GemmParams& p, cudaStream_t s) {
   return launch_pdl(kern, dim3(2 * clusters), dim3(kThreads), kSmemBytes, s, p);
 }
 
-}  // namespace
+template <int FMT>
+int dispatch_gemm(const GemmParams& p, int out_dtype, cudaStream_t s) {
+  const bool unstaged = p.G > kMaxStageG;
+  switch (out_dtype) {
+    case OFFQ_F32:
+      return p.G == 1 ? launch_gemm<OFFQ_F32, true, false, FMT>(p, s)
+                      : unstaged ? launch_gemm<OFFQ_F32, false, true, FMT>(p, s)
+                                 : launch_gemm<OFFQ_F32, false, false, FMT>(p, s);
+    case OFFQ_BF16:
+      return p.G == 1 ? launch_gemm<OFFQ_BF16, true, false, FMT>(p, s)
+                      : unstaged ? launch_gemm<OFFQ_BF16, false, true, FMT>(p, s)
+                                 : launch_gemm<OFFQ_BF16, false, false, FMT>(p, s);
+    case OFFQ_F16:
+      return p.G == 1 ? launch_gemm<OFFQ_F16, true, false, FMT>(p, s)
+                      : unstaged ? launch_gemm<OFFQ_F16, false, true, FMT>(p, s)
+                                 : launch_gemm<OFFQ_F16, false, false, FMT>(p, s);
+    default: return OFFQ_ERR_INVALID_ARG;
+  }
+}
 
-extern "C" int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, const float* a_offset, int64_t T,
-                                int64_t N, int64_t K, int32_t g, const uint8_t* w_codes, const float* w_scale,
-                                const float* w_offsum, void* out, int out_dtype, int64_t ldo, int32_t* acc_debug,
-                                void* stream) {
-  const int ob = elem_bytes(out_dtype);
-  if (ob == 0 || T < 0 || N < 1 || !is_pow2(g) || g < 32 || g > 8192) return OFFQ_ERR_INVALID_ARG;
-  if (K <= 0 || K % g != 0 || K % 32 != 0 || ldo < N) return OFFQ_ERR_INVALID_ARG;
-  if (K > kMaxGemmK || T > 0x3FFFFFFF || N > 0x3FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
-  if (T == 0) return OFFQ_OK;
-  if (a_codes == nullptr || a_scale == nullptr || w_codes == nullptr || w_scale == nullptr || w_offsum == nullptr ||
-      out == nullptr)
-    return OFFQ_ERR_INVALID_ARG;
-  if (!aligned(a_codes, 16) || !aligned(w_codes, 16) || !aligned(out, 16) || (ldo * ob) % 16 != 0 ||
-      !aligned(a_scale, 4) || !aligned(w_scale, 4) || !aligned(w_offsum, 4) ||
-      (a_offset != nullptr && !aligned(a_offset, 4)) || (acc_debug != nullptr && !aligned(acc_debug, 4)))
-    return OFFQ_ERR_MISALIGNED;
-
-  cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (T <= decode_max_tokens())
-    return w4a4_linear_decode(a_codes, a_scale, a_offset, T, N, K, g, w_codes, w_scale, w_offsum, out, out_dtype, ldo,
-                              acc_debug, s);
-
+// The shapes, tile counts and raster of one launch (arguments already checked).
+GemmParams gemm_params(const uint8_t* a_codes, const float* a_scale, const float* a_offset, int64_t T, int64_t N,
+                       int64_t K, int32_t g, const uint8_t* w_codes, const float* w_scale, const float* w_offsum,
+                       void* out, int out_dtype, int64_t ldo, int32_t* acc_debug) {
   GemmParams p{};
   p.a_codes = a_codes;
   p.w_codes = w_codes;
@@ -746,19 +808,59 @@ extern "C" int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, co
   p.t_blocks = static_cast<int>((T + 31) / 32);
   p.n_blocks = static_cast<int>((N + 31) / 32);
   p.kchunks = static_cast<int>(K / 32);
+  p.nkt = static_cast<int>(K / 128);
   p.vec_ok = aligned(w_offsum, 16) && aligned(w_scale, 16) && (N % 4 == 0);
   p.async_out = out_dtype != OFFQ_F32 && N % 8 == 0;
-  const bool unstaged = p.G > kMaxStageG;
-  switch (out_dtype) {
-    case OFFQ_F32:
-      return p.G == 1 ? launch_gemm<OFFQ_F32, true>(p, s)
-                      : unstaged ? launch_gemm<OFFQ_F32, false, true>(p, s) : launch_gemm<OFFQ_F32, false>(p, s);
-    case OFFQ_BF16:
-      return p.G == 1 ? launch_gemm<OFFQ_BF16, true>(p, s)
-                      : unstaged ? launch_gemm<OFFQ_BF16, false, true>(p, s) : launch_gemm<OFFQ_BF16, false>(p, s);
-    case OFFQ_F16:
-      return p.G == 1 ? launch_gemm<OFFQ_F16, true>(p, s)
-                      : unstaged ? launch_gemm<OFFQ_F16, false, true>(p, s) : launch_gemm<OFFQ_F16, false>(p, s);
-    default: return OFFQ_ERR_INVALID_ARG;
-  }
+  return p;
+}
+
+}  // namespace
+
+extern "C" int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, const float* a_offset, int64_t T,
+                                int64_t N, int64_t K, int32_t g, const uint8_t* w_codes, const float* w_scale,
+                                const float* w_offsum, void* out, int out_dtype, int64_t ldo, int32_t* acc_debug,
+                                void* stream) {
+  const int ob = elem_bytes(out_dtype);
+  if (ob == 0 || T < 0 || N < 1 || !is_pow2(g) || g < 32 || g > 8192) return OFFQ_ERR_INVALID_ARG;
+  if (K <= 0 || K % g != 0 || K % 32 != 0 || ldo < N) return OFFQ_ERR_INVALID_ARG;
+  if (K > kMaxGemmK || T > 0x3FFFFFFF || N > 0x3FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
+  if (T == 0) return OFFQ_OK;
+  if (a_codes == nullptr || a_scale == nullptr || w_codes == nullptr || w_scale == nullptr || w_offsum == nullptr ||
+      out == nullptr)
+    return OFFQ_ERR_INVALID_ARG;
+  if (!aligned(a_codes, 16) || !aligned(w_codes, 16) || !aligned(out, 16) || (ldo * ob) % 16 != 0 ||
+      !aligned(a_scale, 4) || !aligned(w_scale, 4) || !aligned(w_offsum, 4) ||
+      (a_offset != nullptr && !aligned(a_offset, 4)) || (acc_debug != nullptr && !aligned(acc_debug, 4)))
+    return OFFQ_ERR_MISALIGNED;
+
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (T <= decode_max_tokens())
+    return w4a4_linear_decode(a_codes, a_scale, a_offset, T, N, K, g, w_codes, w_scale, w_offsum, out, out_dtype, ldo,
+                              acc_debug, s);
+  const GemmParams p = gemm_params(a_codes, a_scale, a_offset, T, N, K, g, w_codes, w_scale, w_offsum, out, out_dtype,
+                                   ldo, acc_debug);
+  return dispatch_gemm<kFmtInt4>(p, out_dtype, s);
+}
+
+extern "C" int offq_mx_linear(const uint8_t* a_codes, const uint8_t* a_shifts, const float* a_scale,
+                              const float* a_offset, int64_t T, int64_t N, int64_t K, int32_t g,
+                              const uint8_t* w_codes, const uint8_t* w_shifts, const float* w_scale,
+                              const float* w_offsum, void* out, int out_dtype, int64_t ldo, void* stream) {
+  const int ob = elem_bytes(out_dtype);
+  if (ob == 0 || T < 0 || N < 1 || !is_pow2(g) || g < 32 || g > 8192) return OFFQ_ERR_INVALID_ARG;
+  if (K <= 0 || K % g != 0 || K % 128 != 0 || ldo < N) return OFFQ_ERR_INVALID_ARG;
+  if (K > kMaxGemmK || T > 0x3FFFFFFF || N > 0x3FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
+  if (T == 0) return OFFQ_OK;
+  if (a_codes == nullptr || a_shifts == nullptr || a_scale == nullptr || w_codes == nullptr || w_shifts == nullptr ||
+      w_scale == nullptr || w_offsum == nullptr || out == nullptr)
+    return OFFQ_ERR_INVALID_ARG;
+  if (!aligned(a_codes, 16) || !aligned(w_codes, 16) || !aligned(out, 16) || (ldo * ob) % 16 != 0 ||
+      !aligned(a_shifts, 4) || !aligned(w_shifts, 4) || !aligned(a_scale, 4) || !aligned(w_scale, 4) ||
+      !aligned(w_offsum, 4) || (a_offset != nullptr && !aligned(a_offset, 4)))
+    return OFFQ_ERR_MISALIGNED;
+  GemmParams p = gemm_params(a_codes, a_scale, a_offset, T, N, K, g, w_codes, w_scale, w_offsum, out, out_dtype, ldo,
+                             nullptr);
+  p.a_shifts = a_shifts;
+  p.w_shifts = w_shifts;
+  return dispatch_gemm<kFmtMx>(p, out_dtype, static_cast<cudaStream_t>(stream));
 }

@@ -193,6 +193,30 @@ __device__ __forceinline__ void widen_weight(uint32_t w, uint32_t& lo, uint32_t&
   hi = __funnelshift_r(w, w, 4) & 0x87878787u;
 }
 
+// E4M3 bytes of four E2M1 codes, one per byte of x (sign in bit 3, magnitude
+// code in bits 0-2), with the byte table lut_lo:lut_hi (magnitude code -> E4M3
+// byte of the magnitude times the block's power of two).
+__device__ __forceinline__ uint32_t mx_bytes(uint32_t x, uint32_t lut_lo, uint32_t lut_hi) {
+  const uint32_t m = x & 0x07070707u;
+  const uint32_t t = m | (m >> 4);                  // byte 0: m0 | m1 << 4, byte 2: m2 | m3 << 4
+  const uint32_t sel = __byte_perm(t, 0u, 0x0020);  // the four magnitude codes as byte selectors
+  return __byte_perm(lut_lo, lut_hi, sel) | ((x & 0x08080808u) << 4);
+}
+
+// Byte table of the E2M1 magnitudes 0, .5, 1, 1.5, 2, 3, 4, 6 times 2^sh as E4M3
+// (exponent field 6 + sh .. 9 + sh, sh in 0..6; zero stays zero).
+__device__ __forceinline__ void mx_lut(uint32_t sh, uint32_t& lut_lo, uint32_t& lut_hi) {
+  lut_lo = 0x3C383000u + sh * 0x08080800u;
+  lut_hi = 0x4C484440u + sh * 0x08080808u;
+}
+
+// Eight MXFP4 codes (two per byte, even channel low) -> eight E4M3 bytes in the
+// channel order of widen_act / widen_weight: [c0 c2 c4 c6 | c1 c3 c5 c7].
+__device__ __forceinline__ void widen_mx(uint32_t w, uint32_t lut_lo, uint32_t lut_hi, uint32_t& lo, uint32_t& hi) {
+  lo = mx_bytes(w & 0x0F0F0F0Fu, lut_lo, lut_hi);
+  hi = mx_bytes((w >> 4) & 0x0F0F0F0Fu, lut_lo, lut_hi);
+}
+
 template <int OUT, int CW>
 __device__ __forceinline__ void store_out(void* out, int64_t off, const float* y, int nvalid) {
   if (OUT == OFFQ_F32) {

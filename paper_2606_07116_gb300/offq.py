@@ -47,6 +47,13 @@ _SIGNATURES = {
     "offq_prepare_weight": (_c_int, [_c_vp, _c_int, _c_i64, _c_i64, _c_i32, _c_i32, _c_vp, _c_vp, _c_vp, _c_vp]),
     "offq_get_device_status": (_c_int, [_c_vp]),
     "offq_set_wait_cycles": (_c_int, [_c_i64]),
+    "offq_quantize_act_mx": (_c_int, [_c_vp, _c_int, _c_i64, _c_i64, _c_i64, _c_i32, _c_i32, _c_vp, _c_vp, _c_vp,
+                                      _c_vp, _c_vp]),
+    "offq_prepare_weight_mx": (_c_int, [_c_vp, _c_int, _c_i64, _c_i64, _c_i32, _c_i32, _c_vp, _c_vp, _c_vp, _c_vp,
+                                        _c_vp]),
+    "offq_mx_linear": (_c_int, [_c_vp, _c_vp, _c_vp, _c_vp, _c_i64, _c_i64, _c_i64, _c_i32, _c_vp, _c_vp, _c_vp,
+                                _c_vp, _c_vp, _c_int, _c_i64, _c_vp]),
+    "offq_mx_shift_bytes": (_c_i64, [_c_i64, _c_i64]),
     "offq_status_string": (ctypes.c_char_p, [_c_int]),
     "offq_abi_version": (_c_int, []),
     "offq_act_codes_bytes": (_c_i64, [_c_i64, _c_i64]),
@@ -545,3 +552,59 @@ def fuse_rotation(W: torch.Tensor, v: torch.Tensor, perm: torch.Tensor, g: int, 
         _ptr(W.contiguous()), N, D, _ptr(v), _ptr(perm.to(W.device, torch.int32).contiguous()), g, _ptr(out),
         _stream(stream)))
     return out
+
+
+# ---------------------------------------------------------------------------
+# MXFP4 residuals with the offset as zero-point
+# ---------------------------------------------------------------------------
+
+def offq_quantize_act_mx(x: torch.Tensor, T: int, K: int, ldx: int, g: int, flags: int, codes: torch.Tensor,
+                         shifts: torch.Tensor, row_scale: torch.Tensor, offset: Optional[torch.Tensor],
+                         stream=None) -> None:
+    _check("offq_quantize_act_mx", load_library().offq_quantize_act_mx(
+        _ptr(x), _dtype_code(x), T, K, ldx, g, flags, _ptr(codes), _ptr(shifts), _ptr(row_scale), _ptr(offset),
+        _stream(stream)))
+
+
+def offq_prepare_weight_mx(w: torch.Tensor, N: int, K: int, g: int, rotate: int, w_codes: torch.Tensor,
+                           w_shifts: torch.Tensor, w_scale: torch.Tensor, w_offsum: torch.Tensor,
+                           stream=None) -> None:
+    _check("offq_prepare_weight_mx", load_library().offq_prepare_weight_mx(
+        _ptr(w), _dtype_code(w), N, K, g, rotate, _ptr(w_codes), _ptr(w_shifts), _ptr(w_scale), _ptr(w_offsum),
+        _stream(stream)))
+
+
+def offq_mx_linear(a_codes, a_shifts, a_scale, a_offset, T: int, N: int, K: int, g: int, w_codes, w_shifts,
+                   w_scale, w_offsum, out: torch.Tensor, ldo: int, stream=None) -> None:
+    _check("offq_mx_linear", load_library().offq_mx_linear(
+        _ptr(a_codes), _ptr(a_shifts), _ptr(a_scale), _ptr(a_offset), T, N, K, g, _ptr(w_codes), _ptr(w_shifts),
+        _ptr(w_scale), _ptr(w_offsum), _ptr(out), _dtype_code(out), ldo, _stream(stream)))
+
+
+def mx_shift_bytes(R: int, K: int) -> int:
+    return load_library().offq_mx_shift_bytes(R, K)
+
+
+def quantize_act_mx(x: torch.Tensor, g: int, rotate: bool = True, offset: bool = True):
+    """Allocating wrapper: (codes, shifts, row_scale, offset) for rows x [T, K]."""
+    T, K = x.shape
+    dev = x.device
+    codes = torch.empty((padded_rows(T), K // 2), dtype=torch.uint8, device=dev)
+    shifts = torch.empty((mx_shift_bytes(T, K),), dtype=torch.uint8, device=dev)
+    scale = torch.empty((T,), dtype=torch.float32, device=dev)
+    off = torch.empty((T, K // g), dtype=torch.float32, device=dev)
+    flags = (OFFQ_ROTATE if rotate else 0) | (OFFQ_OFFSET if offset else 0)
+    offq_quantize_act_mx(x, T, K, x.stride(0), g, flags, codes, shifts, scale, off)
+    return codes, shifts, scale, off
+
+
+def prepare_weight_mx(w: torch.Tensor, g: int, rotate: bool = True):
+    """Allocating wrapper: (codes, shifts, scale, offsum) for weights w [N, K]."""
+    N, K = w.shape
+    dev = w.device
+    codes = torch.empty((padded_rows(N), K // 2), dtype=torch.uint8, device=dev)
+    shifts = torch.empty((mx_shift_bytes(N, K),), dtype=torch.uint8, device=dev)
+    scale = torch.empty((N,), dtype=torch.float32, device=dev)
+    offsum = torch.empty((K // g, N), dtype=torch.float32, device=dev)
+    offq_prepare_weight_mx(w.contiguous(), N, K, g, 1 if rotate else 0, codes, shifts, scale, offsum)
+    return codes, shifts, scale, offsum

@@ -119,6 +119,41 @@ def test_code_buffer_sizes(lib):
     assert Q.offq_weight_codes_bytes(0, 1024) == -1
 
 
+def test_mx_argument_checks(lib):
+    def qm(x=A16, dt=Q.OFFQ_BF16, T=8, K=1024, ldx=1024, g=256, flags=3, c=A16, sh=A16, s=A16, o=A16):
+        return lib.offq_quantize_act_mx(x, dt, T, K, ldx, g, flags, c, sh, s, o, None)
+    assert qm(g=100) == Q.OFFQ_ERR_INVALID_ARG
+    assert qm(g=16) == Q.OFFQ_ERR_INVALID_ARG
+    assert qm(K=1000, ldx=1000) == Q.OFFQ_ERR_INVALID_ARG      # g does not divide K
+    assert qm(K=1088, ldx=1088, g=64) == Q.OFFQ_ERR_INVALID_ARG  # K not a multiple of 128
+    assert qm(K=65536, ldx=65536, g=4096) == Q.OFFQ_ERR_UNSUPPORTED
+    assert qm(ldx=512) == Q.OFFQ_ERR_INVALID_ARG
+    assert qm(flags=4) == Q.OFFQ_ERR_INVALID_ARG
+    assert qm(o=None) == Q.OFFQ_ERR_INVALID_ARG                # OFFSET needs an offset buffer
+    assert qm(sh=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert qm(x=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert qm(T=0) == Q.OFFQ_OK
+    pm = lib.offq_prepare_weight_mx
+    assert pm(A16, Q.OFFQ_F32, 0, 1024, 256, 1, A16, A16, A16, A16, None) == Q.OFFQ_ERR_INVALID_ARG  # N = 0
+    assert pm(A16, Q.OFFQ_F32, 8, 1024, 256, 1, A16, A16, A16, None, None) == Q.OFFQ_ERR_INVALID_ARG
+    assert pm(A16, Q.OFFQ_F32, 8, 1000, 200, 1, A16, A16, A16, A16, None) == Q.OFFQ_ERR_INVALID_ARG
+
+    def lm(T=8, N=64, K=1024, g=256, a=A16, sh=A16, w=A16, out=A16, dt=Q.OFFQ_BF16, ldo=64):
+        return lib.offq_mx_linear(a, sh, A16, A16, T, N, K, g, w, A16, A16, A16, out, dt, ldo, None)
+    assert lm(K=1000) == Q.OFFQ_ERR_INVALID_ARG
+    assert lm(K=1088, g=64) == Q.OFFQ_ERR_INVALID_ARG
+    assert lm(N=0) == Q.OFFQ_ERR_INVALID_ARG
+    assert lm(ldo=32) == Q.OFFQ_ERR_INVALID_ARG
+    assert lm(dt=9) == Q.OFFQ_ERR_INVALID_ARG
+    assert lm(K=131072, g=4096) == Q.OFFQ_ERR_UNSUPPORTED
+    assert lm(sh=None) == Q.OFFQ_ERR_INVALID_ARG
+    assert lm(a=A8) == Q.OFFQ_ERR_MISALIGNED
+    assert lm(T=0) == Q.OFFQ_OK
+    assert Q.mx_shift_bytes(1, 4096) == 32 * 128
+    assert Q.mx_shift_bytes(33, 128) == 64 * 4
+    assert Q.mx_shift_bytes(4, 96) == -1
+
+
 def test_group_path_argument_checks(lib):
     qg = lambda x=A16, dt=Q.OFFQ_BF16, T=4, K=1024, ldx=1024, g=256, group=128, flags=1, c=A16, s=A16, z=A16: \
         lib.offq_quantize_act_group(x, dt, T, K, ldx, g, group, flags, c, s, z, None)
