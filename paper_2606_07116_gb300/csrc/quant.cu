@@ -763,6 +763,210 @@ __global__ void __launch_bounds__(WideGeo<L>::kMaxThreads) quantize_rows_wide_ke
   }
 }
 
+// g = 1024 with the rotation, persistent: a warp per block of 1024 channels,
+// 32 channels per lane, so a CTA of up to 28 warps holds whole rows in
+// registers at 32 data registers a thread (the register file holds two rows
+// of 28672 channels). Rows arrive in a ring of shared-memory slots filled by
+// bulk copies. Channel e of a block has index bits e0..e9. Pass 1: lane l,
+// register j holds e = l + 32 j (conflict-free 2- or 4-byte loads from the
+// slot) and runs the stages of e5..e9; a transpose through the warp's 4 KB of
+// shared memory gives lane l the channels e = 32 l + j, whose stages (e0..e4)
+// pass 2 runs; the lane then owns one whole 16-byte code chunk. The row's
+// absmax crosses warps through shared memory (one barrier per row group).
+constexpr int k1kMaxWarps = 28;
+
+template <typename Tin>
+__device__ __forceinline__ float smem_elem(const Tin* p) {
+  if constexpr (sizeof(Tin) == 4) {
+    return *reinterpret_cast<const float*>(p);
+  } else if constexpr (std::is_same<Tin, __nv_bfloat16>::value) {
+    return __uint_as_float(static_cast<uint32_t>(*reinterpret_cast<const uint16_t*>(p)) << 16);
+  } else {
+    return __half2float(*p);
+  }
+}
+
+// max(a, b, c) in one instruction.
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
+// Shared-memory accesses by 32-bit address.
+__device__ __forceinline__ void sts_f32(uint32_t addr, float v) {
+  asm volatile("st.shared.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
+}
+__device__ __forceinline__ float4 lds_f32x4(uint32_t addr) {
+  float4 r;
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(r.x), "=f"(r.y), "=f"(r.z), "=f"(r.w) : "r"(addr) : "memory");
+  return r;
+}
+
+// Transpose swizzle (float index within a warp's 1024): the 16-byte chunk index
+// (bits 2-4) takes bits 5-7 as well. Pass-1 stores (fixed j, 32 lanes) stay
+// within one 128-byte row; the pass-2 float4 loads of a quarter-warp hit eight
+// distinct chunks.
+__device__ __forceinline__ int swz1k(int e) { return e ^ (((e >> 5) & 7) << 2); }
+
+// Butterflies of register bit M of quantize_rows_1k_kernel, whose 32 values sit
+// in 16 float2 pairs (register 2i in .x, 2i + 1 in .y): bit 0 within each pair,
+// bit M >= 1 between pairs i and i + 2^(M-1), two lanes per packed add.
+template <int M>
+__device__ __forceinline__ void fwht1k_stage(float2 (&v)[16]) {
+  if constexpr (M == 0) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = make_float2(v[i].x + v[i].y, v[i].x - v[i].y);
+  } else {
+    constexpr int d = 1 << (M - 1);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      if ((i & d) == 0) {
+        const float2 p = v[i], q = v[i + d];
+        v[i] = __fadd2_rn(p, q);
+        v[i + d] = __ffma2_rn(q, make_float2(-1.0f, -1.0f), p);  // p - q, one rounding
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ void fwht1k_pass(float2 (&v)[16]) {
+  fwht1k_stage<0>(v);
+  fwht1k_stage<1>(v);
+  fwht1k_stage<2>(v);
+  fwht1k_stage<3>(v);
+  fwht1k_stage<4>(v);
+}
+
+template <typename Tin>
+__global__ void __launch_bounds__(k1kMaxWarps * 32, 1) quantize_rows_1k_kernel(const QuantArgs a) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  __shared__ int abort_flag;
+  __shared__ float wmax[k1kMaxWarps];
+  const int K = a.K, G = a.G, R = a.rows_per_cta;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int lrow = warp / G;
+  const int b = warp - lrow * G;
+  const bool offs = (a.flags & OFFQ_OFFSET) != 0;
+  const uint32_t scr32 = smem_u32(smem) + 4096u * warp;  // the warp's transpose scratch
+  RowRing ring;
+  ring.base = smem + static_cast<size_t>(R) * G * 4096;
+  ring.slot_bytes = static_cast<uint32_t>(R) * K * sizeof(Tin);
+  ring.S = a.ring_slots;
+  ring.bar0 = smem_u32(ring.base + static_cast<size_t>(ring.S) * ring.slot_bytes);
+  ring.s = 0;
+  ring.phase = 0;
+  // Rows fit an int here (the launcher checks), so group and row indices are 32-bit.
+  const int ngroups = static_cast<int>((a.rows + R - 1) / R);
+  int grp = blockIdx.x;
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    for (int k = 0; k < ring.S; ++k) mbar_init(ring.bar0 + 8u * k, 1);
+    mbar_fence_init();
+  }
+  __syncthreads();
+  griddep_wait();
+  griddep_launch_dependents();
+  ring_start<Tin>(a, ring, R, ngroups);
+
+  const int cpr = K / 32;
+  const int cstride = a.tiled ? 512 : 16;
+  const int blk_off = lrow * K + b * 1024 + lane;
+  while (true) {
+    const int row = grp * R + lrow;
+    const bool row_ok = row < a.rows;
+    // v[i].x: channel lane + 64 i, v[i].y: channel lane + 64 i + 32 (register j = 2i, 2i + 1).
+    float2 v[16];
+    const bool ok = mbar_wait_for(ring.bar(), ring.phase, &abort_flag, a.wait_cycles);
+    if (ok && row_ok) {
+      const Tin* p = reinterpret_cast<const Tin*>(ring.slot()) + blk_off;
+#pragma unroll
+      for (int i = 0; i < 16; ++i) v[i] = make_float2(smem_elem(p + 64 * i), smem_elem(p + 64 * i + 32));
+    } else {
+#pragma unroll
+      for (int i = 0; i < 16; ++i) v[i] = make_float2(0.f, 0.f);
+    }
+    // Offset = x[block start] / sqrt(g); removing it first leaves the residual.
+    float off = 0.f;
+    if (offs && lane == 0) {
+      off = v[0].x;
+      v[0].x = 0.f;
+    }
+    fwht1k_pass(v);  // channel bits 5..9
+    // Transpose through the warp's scratch: channel e at byte 4 swz1k(e). Register j of
+    // lane l (e = l + 32 j) lands at 128 j + (4 l ^ 16 (j & 7)): eight lane bases, the
+    // rest immediate offsets. Lane l then reads its row's float4 k at 128 l + (16 k ^ 16 (l & 7)).
+    {
+      uint32_t wb[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) wb[q] = scr32 + ((4u * lane) ^ (16u * q));
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        sts_f32(wb[(2 * i) & 7] + 128u * (2 * i), v[i].x);
+        sts_f32(wb[(2 * i + 1) & 7] + 128u * (2 * i + 1), v[i].y);
+      }
+    }
+    __syncwarp();
+    // Now register j = 4k + c holds channel 32 lane + j.
+    {
+      const uint32_t rb = scr32 + 128u * lane;
+      const uint32_t rx = 16u * (lane & 7);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const float4 f = lds_f32x4(rb + ((16u * k) ^ rx));
+        v[2 * k] = make_float2(f.x, f.y);
+        v[2 * k + 1] = make_float2(f.z, f.w);
+      }
+    }
+    fwht1k_pass(v);  // channel bits 0..4
+
+    // Row absmax: the lane's, the warp's (non-negative floats order as their
+    // bit patterns), then over the row's G warps.
+    float mx0 = 0.f, mx1 = 0.f;
+#pragma unroll
+    for (int i = 0; i < 16; i += 2) {
+      mx0 = fmax3(mx0, fabsf(v[i].x), fabsf(v[i].y));
+      mx1 = fmax3(mx1, fabsf(v[i + 1].x), fabsf(v[i + 1].y));
+    }
+    const uint32_t wm = __reduce_max_sync(0xFFFFFFFFu, __float_as_uint(fmaxf(mx0, mx1)));
+    if (lane == 0) wmax[warp] = __uint_as_float(wm);
+    // One barrier per row group: the warps' maxima are visible, every thread has read
+    // the slot (so it takes the group S turns ahead), and a wait that ran out anywhere
+    // in the CTA is seen by all.
+    if (!__syncthreads_and(ok)) {
+      ring_fail(ring, grp, ngroups, a.status);
+      return;
+    }
+    const int next = grp + ring.S * static_cast<int>(gridDim.x);
+    if (threadIdx.x == 0 && next < ngroups) ring_issue<Tin>(a, next, R, ring.slot(), ring.bar());
+    ring.advance();
+    const float m = __uint_as_float(
+        __reduce_max_sync(0xFFFFFFFFu, lane < G ? __float_as_uint(wmax[lrow * G + lane]) : 0u));
+    const float inv = m > 0.f ? __fdiv_rn(7.0f, m) : 0.f;
+
+    const float2 inv2 = make_float2(inv, inv), mag2 = make_float2(kMagic8, kMagic8);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __ffma2_rn(v[i], inv2, mag2);
+    uint32_t wd[4];
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      const float2* q = &v[4 * w];
+      wd[w] = pack_codes8(__float_as_uint(q[0].x), __float_as_uint(q[0].y), __float_as_uint(q[1].x),
+                          __float_as_uint(q[1].y), __float_as_uint(q[2].x), __float_as_uint(q[2].y),
+                          __float_as_uint(q[3].x), __float_as_uint(q[3].y));
+    }
+    if (row_ok) {
+      uint8_t* rdst = a.tiled ? a.codes + static_cast<int64_t>(row >> 5) * cpr * 512 + (row & 31) * 16
+                              : a.codes + static_cast<int64_t>(row) * (K / 2);
+      *reinterpret_cast<uint4*>(rdst + (b * 32 + lane) * cstride) = make_uint4(wd[0], wd[1], wd[2], wd[3]);
+      if (b == 0 && lane == 0) a.scale[row] = m * a.scale_mul;
+      if (lane == 0 && a.offset != nullptr) a.offset[static_cast<int64_t>(row) * G + b] = offs ? off * a.inv_sqrt_g : 0.f;
+    }
+    grp += gridDim.x;
+    if (grp >= ngroups) break;
+  }
+}
+
 // Rows without the rotation whose offset block is the whole row (g == K): one
 // warp per row. Each lane issues the loads of up to CB 8-element chunks at once
 // and keeps them (raw) in registers, so a row of up to 256*CB elements costs one
@@ -1228,6 +1432,51 @@ int launch_wide(QuantArgs a, cudaStream_t stream) {
   return launch_pdl(kern, dim3(static_cast<unsigned>(grid)), dim3(R * tpr), smem, stream, a);
 }
 
+// quantize_rows_1k_kernel: R rows of G warps per CTA. One row per CTA unless a
+// CTA would have fewer than 4 warps: CTAs of G <= 14 warps share an SM and
+// drift apart, so one CTA's barrier waits overlap another's arithmetic. The
+// ring takes 2 or 3 slots, whichever gives more CTAs per SM (ties: more
+// slots); 1 slot only when 2 do not fit. kNoRing when the one-shot kernels
+// serve better (one head required, more row groups than SMs).
+template <typename Tin>
+int launch_1k(QuantArgs a, cudaStream_t stream) {
+  if (a.H != 1 || (a.flags & OFFQ_ROTATE) == 0 || a.G > k1kMaxWarps) return kNoRing;
+  const int sms = sm_count();
+  if (sms <= 0) return OFFQ_ERR_CUDA;
+  const int R = std::max(1, 4 / a.G);
+  const int64_t groups = (a.rows + R - 1) / R;
+  if (groups <= sms || a.rows + R > 0x7FFFFFFF) return kNoRing;
+  auto kern = quantize_rows_1k_kernel<Tin>;
+  if (prefer_max_shared(kern) != OFFQ_OK) return OFFQ_ERR_CUDA;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kMaxDynSmem)) !=
+      cudaSuccess)
+    return OFFQ_ERR_CUDA;
+  const int threads = R * a.G * 32;
+  const size_t fixed = static_cast<size_t>(R) * a.G * 4096;
+  const size_t slot = static_cast<size_t>(R) * a.K * sizeof(Tin) + 8;
+  int best_s = 0, best_per_sm = 0;
+  for (int S = 1; S <= 3; ++S) {
+    const size_t smem = fixed + S * slot;
+    if (smem > kMaxDynSmem) break;
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem) != cudaSuccess)
+      return OFFQ_ERR_CUDA;
+    if (per_sm < 1) break;
+    const bool better = best_s == 0 || (best_s == 1 && S >= 2) || (S >= 2 && per_sm >= best_per_sm);
+    if (better) {
+      best_s = S;
+      best_per_sm = per_sm;
+    }
+  }
+  if (best_s == 0) return kNoRing;
+  a.rows_per_cta = R;
+  a.ring_slots = best_s;
+  a.tpr = a.G * 32;
+  const size_t smem = fixed + best_s * slot;
+  const int64_t grid = std::min<int64_t>(groups, static_cast<int64_t>(sms) * best_per_sm);
+  return launch_pdl(kern, dim3(static_cast<unsigned>(grid)), dim3(threads), smem, stream, a);
+}
+
 template <typename Tin>
 int launch_stream(const QuantArgs& a, cudaStream_t stream) {
   const int64_t grid = (a.rows + 7) / 8;
@@ -1277,7 +1526,10 @@ int dispatch_g(const QuantArgs& a, int g, cudaStream_t s) {
     case 128: return launch_narrow<7, Tin>(a, s);
     case 256: return launch_narrow<8, Tin>(a, s);
     case 512: return launch_narrow<9, Tin>(a, s);
-    case 1024: return launch_narrow<10, Tin>(a, s);
+    case 1024: {
+      const int st = launch_1k<Tin>(a, s);
+      return st == kNoRing ? launch_narrow<10, Tin>(a, s) : st;
+    }
     case 2048: return launch_wide<11, Tin>(a, s);
     case 4096: return launch_wide<12, Tin>(a, s);
     case 8192: return launch_wide<13, Tin>(a, s);

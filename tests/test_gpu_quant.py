@@ -141,6 +141,22 @@ def test_quantize_persistent_ring_dtypes_and_stride(dt, ld_pad):
     _quant_and_check(_host(x, dt), g, True, True, rows=rows, ldx=(K + ld_pad) if ld_pad else None)
 
 
+@pytest.mark.parametrize("T,K,dt,ld_pad,offset", [
+    (1700, 5120, "f32", 0, True),      # 5 blocks, one row per CTA and one slot of fp32 rows
+    (900, 14336, "f16", 0, True),      # Llama-3-8B down-proj width: two rows of 14 warps per CTA
+    (3001, 2048, "bf16", 64, True),    # padded rows (one bulk copy per row), a ragged last group
+    (4500, 1024, "bf16", 0, False),    # 28 rows of one block per CTA, no offsets
+    (760, 28672, "bf16", 0, False),    # Llama-2-70B down-proj width, no offsets
+])
+def test_quantize_warp_per_block_kernel(T, K, dt, ld_pad, offset):
+    """The persistent g = 1024 kernel (a warp per block, rows held in registers) across dtypes,
+    row counts per CTA, padded rows and the offset flag; sampled rows including the first and
+    the last."""
+    x = W.activations(T, K, seed=61 + K, n_out=4, mult=100.0)
+    rows = np.unique(np.concatenate([W.unit_index_sample(T, 160, seed=12), [0, 1, T - 2, T - 1]]))
+    _quant_and_check(_host(x, dt), 1024, True, offset, rows=rows, ldx=(K + ld_pad) if ld_pad else None)
+
+
 def test_quantize_toy_fp32():
     w = W.WORKLOADS["toy"]
     x = W.layer_inputs(w, w.layers[0])

@@ -28,7 +28,8 @@ def _lib():
 
 
 @pytest.mark.parametrize("T,K,g,rotate", [
-    (4096, 2048, 1024, True),    # the ring form of the block-Hadamard kernel (g <= 1024)
+    (4096, 2048, 1024, True),    # the warp-per-block kernel of g = 1024 with the rotation
+    (8192, 2048, 512, True),     # the ring form of the block-Hadamard kernel (g <= 1024)
     (2048, 8192, 4096, True),    # the ring form of the wide kernel (g >= 2048)
     (8192, 4096, 4096, False),   # the shared-memory ring kernel of rotation-free rows (per-warp rings)
 ])
