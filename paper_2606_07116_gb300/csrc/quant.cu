@@ -690,9 +690,8 @@ __global__ void __launch_bounds__(WideGeo<L>::kMaxThreads) quantize_rows_wide_ke
       }
       fwht_bits<E, Q, LOGE>(v);  // index bits {3, .., 3+P-1}
     } else if (offs) {
-      float s = 0.f;
-#pragma unroll
-      for (int r = 0; r < E; ++r) s += v[r];
+      // Block mean by a pairwise tree (depth log2(E) in the thread, P across threads).
+      float s = tree_sum<E>(v);
       s = group_reduce<false>(s, TPB, red);
       off = s * (1.0f / static_cast<float>(g));
 #pragma unroll
@@ -1067,6 +1066,44 @@ __device__ __forceinline__ void add2(float& a0, float& a1, float b0, float b1) {
   unpack2(R, a0, a1);
 }
 
+// Pairwise summation over a stream of values whose count is a power of two
+// (at most 2^L): level k holds the sum of the last complete run of 2^k values,
+// so each value joins a balanced tree and the total, read at level
+// log2(count), has depth log2(count).
+template <int L>
+struct PairwiseSum {
+  float lvl[L + 1];
+  int n = 0;
+  __device__ __forceinline__ void add(float c) {
+    bool carry = true;
+#pragma unroll
+    for (int k = 0; k <= L; ++k) {
+      const bool full = (n >> k) & 1;
+      if (carry && full) c = lvl[k] + c;
+      if (carry && !full) lvl[k] = c;
+      carry = carry && full;
+    }
+    ++n;
+  }
+  // The total once n is a power of two.
+  __device__ __forceinline__ float total() const {
+    float t = 0.f;
+#pragma unroll
+    for (int k = 0; k <= L; ++k) {
+      if (n == (1 << k)) t = lvl[k];
+    }
+    return t;
+  }
+};
+
+// Sum of the 8 values of a chunk by a tree of depth 3.
+__device__ __forceinline__ float chunk_sum8(float (&v)[8]) {
+  add2(v[0], v[1], v[2], v[3]);
+  add2(v[4], v[5], v[6], v[7]);
+  add2(v[0], v[1], v[4], v[5]);
+  return v[0] + v[1];
+}
+
 template <typename Tin, int CB>
 __global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantArgs a) {
   griddep_wait();
@@ -1085,29 +1122,32 @@ __global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantAr
 
   RawChunk<Tin> raw[CB];
   RowMinMax<Tin> mm;
-  float s0 = 0.f, s1 = 0.f;
+  PairwiseSum<6> ps;  // the batches' sums (a power of two of them)
   for (int c0 = 0; c0 < nch; c0 += 32 * CB) {
 #pragma unroll
     for (int i = 0; i < CB; ++i) {
       const int c = c0 + lane + 32 * i;
       if (c < nch) raw[i].load(xr + 8 * c);
     }
+    float cs[CB];
 #pragma unroll
     for (int i = 0; i < CB; ++i) {
       const int c = c0 + lane + 32 * i;
+      cs[i] = 0.f;
       if (c < nch) {
 #pragma unroll
         for (int e = 0; e < RawChunk<Tin>::kWords; ++e) mm.add_word(raw[i].w[e]);
         float v[8];
         raw[i].unpack(v);
-        add2(v[0], v[1], v[2], v[3]);
-        add2(v[4], v[5], v[6], v[7]);
-        add2(v[0], v[1], v[4], v[5]);
-        add2(s0, s1, v[0], v[1]);
+        cs[i] = chunk_sum8(v);
       }
     }
+    // The batch's chunks present are its first min(CB, nch/32) (a power of two): the
+    // zeros after them add exactly, so the tree's depth over real terms is log2 of that.
+    ps.add(tree_sum<CB>(cs));
   }
-  float sum = s0 + s1, mn, mx;
+  // Row sum: depth 3 in the chunk, log2 over the lane's chunks, 5 over the warp.
+  float sum = ps.total(), mn, mx;
   mm.result(mn, mx);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -1164,7 +1204,8 @@ __global__ void __launch_bounds__(256) quantize_rows_stream_kernel(const QuantAr
 // dealt to the grid's warps round-robin.
 constexpr int kBulkRingBytes = 192 * 1024;  // ring bytes per CTA at most
 
-template <typename Tin>
+// CPL = K / 256: the 8-channel chunks each lane sweeps (a power of two, 4 to 32).
+template <typename Tin, int CPL>
 __global__ void __launch_bounds__(256) quantize_rows_bulk_kernel(const QuantArgs a, int S) {
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ int abort_flag;
@@ -1174,7 +1215,7 @@ __global__ void __launch_bounds__(256) quantize_rows_bulk_kernel(const QuantArgs
   const int lane = threadIdx.x & 31;
   const int K = a.K;
   const uint32_t rb = static_cast<uint32_t>(K) * static_cast<uint32_t>(sizeof(Tin));  // a multiple of 64
-  const int cpl = K / 256;                                                            // chunks per lane
+  constexpr int cpl = CPL;                                                            // chunks per lane
   uint8_t* ring = smem + static_cast<size_t>(warp) * S * rb;
   const uint32_t bar0 = smem_u32(smem + static_cast<size_t>(W) * S * rb) + 8u * static_cast<uint32_t>(warp * S);
   if (threadIdx.x == 0) abort_flag = 0;
@@ -1221,8 +1262,10 @@ __global__ void __launch_bounds__(256) quantize_rows_bulk_kernel(const QuantArgs
 
     // Sweep 1: packed min / max of the raw values and the fp32 row sum.
     RowMinMax<Tin> mm;
-    float s0 = 0.f, s1 = 0.f;
-#pragma unroll 4
+    // Chunk sums as packed pairs (even and odd channels), combined pairwise; fully
+    // unrolled, so the carries resolve at compile time and log2(cpl) + 1 pairs stay live.
+    float2 lvl[6];
+#pragma unroll
     for (int j = 0; j < cpl; ++j) {
       RawChunk<Tin> c;
       c.load_smem(rowp + (lane + 32 * j) * kChunkBytes);
@@ -1233,9 +1276,25 @@ __global__ void __launch_bounds__(256) quantize_rows_bulk_kernel(const QuantArgs
       add2(v[0], v[1], v[2], v[3]);
       add2(v[4], v[5], v[6], v[7]);
       add2(v[0], v[1], v[4], v[5]);
-      add2(s0, s1, v[0], v[1]);
+      float2 p = make_float2(v[0], v[1]);
+#pragma unroll
+      for (int k = 0; k < 6; ++k) {
+        if ((j >> k) & 1) {
+          p = __fadd2_rn(lvl[k], p);
+        } else {
+          lvl[k] = p;
+          break;
+        }
+      }
     }
-    float sum = s0 + s1, mn, mx;
+    // Row sum: depth 3 in the chunk, log2(cpl) over the lane's chunks, 1 for the pair,
+    // 5 over the warp.
+    float2 tot = lvl[0];
+#pragma unroll
+    for (int k = 1; k < 6; ++k) {
+      if (cpl == (1 << k)) tot = lvl[k];
+    }
+    float sum = tot.x + tot.y, mn, mx;
     mm.result(mn, mx);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -1501,7 +1560,14 @@ int launch_bulk(const QuantArgs& a, cudaStream_t stream) {
   }
   if (S < 2) return kNoFit;
   const size_t smem = static_cast<size_t>(W) * S * rb + static_cast<size_t>(W) * S * 8;
-  auto kern = quantize_rows_bulk_kernel<Tin>;
+  decltype(&quantize_rows_bulk_kernel<Tin, 4>) kern = nullptr;
+  switch (a.K / 256) {
+    case 4: kern = quantize_rows_bulk_kernel<Tin, 4>; break;
+    case 8: kern = quantize_rows_bulk_kernel<Tin, 8>; break;
+    case 16: kern = quantize_rows_bulk_kernel<Tin, 16>; break;
+    case 32: kern = quantize_rows_bulk_kernel<Tin, 32>; break;
+    default: return kNoFit;
+  }
   if (smem > 48 * 1024 &&
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) != cudaSuccess)
     return OFFQ_ERR_CUDA;

@@ -123,10 +123,28 @@ __global__ void __launch_bounds__(kMxThreads) quantize_mx_kernel(const MxArgs a)
     for (int i = tid; i < K; i += kMxThreads) row[i] *= a.inv_sqrt_g;
     __syncthreads();
   } else if (offs) {
-    // Block sums: a warp per block, lanes in sequence, then a shuffle tree.
+    // Block sums: a warp per block, each lane's g/32 values by a pairwise tree
+    // (a power of two of them), then a shuffle tree: depth log2(g).
     for (int b = warp; b < a.G; b += kMxWarps) {
+      float lvl[9];
+      int n = 0;
+      for (int i = lane; i < g; i += 32) {
+        float c = row[b * g + i];
+        bool carry = true;
+#pragma unroll
+        for (int k = 0; k < 9; ++k) {
+          const bool full = (n >> k) & 1;
+          if (carry && full) c = lvl[k] + c;
+          if (carry && !full) lvl[k] = c;
+          carry = carry && full;
+        }
+        ++n;
+      }
       float s = 0.f;
-      for (int i = lane; i < g; i += 32) s += row[b * g + i];
+#pragma unroll
+      for (int k = 0; k < 9; ++k) {
+        if (n == (1 << k)) s = lvl[k];
+      }
 #pragma unroll
       for (int m = 16; m > 0; m >>= 1) s += __shfl_xor_sync(0xFFFFFFFFu, s, m);
       const float o = s * (1.0f / static_cast<float>(g));

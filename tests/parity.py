@@ -80,9 +80,10 @@ def check_offsets(o_gpu, o_ref, x, g, rotate, what="offset"):
     if rotate:
         tol = 4 * U32 * np.abs(o_ref)   # x[0] * fl(1/sqrt(g)): two roundings
     else:
-        # A block sum in fp32: the kernels add at most g/8 + 16 terms in sequence
-        # along any path of their summation trees.
-        depth = g // 8 + 16
+        # A block sum in fp32 by balanced trees: every kernel adds the g values of a
+        # block along paths of log2(g) additions (the 1/g is exact); one extra level
+        # of slack.
+        depth = int(math.log2(g)) + 1
         tol = depth * U32 * x.reshape(T, K // g, g).sum(axis=2) / g + 2 * U32 * np.abs(o_ref)
     bad = np.abs(o_gpu - o_ref) > tol
     assert not np.any(bad), f"{what}: {bad.sum()} offsets out of tolerance"
