@@ -161,12 +161,14 @@ constexpr int kFmtInt4 = 0, kFmtMx = 1;
 // (zeros where the row block or the chunk does not exist).
 // blk: this lane's first byte of the row block (nullptr if the block does not
 // exist); the block's chunk c starts 512 * c bytes further.
-__device__ __forceinline__ void load_kt(const uint8_t* blk, int kchunks, int kt, uint4 (&v)[kChunksPerKt]) {
+// pol: the L2 policy of the loads.
+__device__ __forceinline__ void load_kt(const uint8_t* blk, int kchunks, int kt, uint4 (&v)[kChunksPerKt],
+                                        uint64_t pol) {
 #pragma unroll
   for (int j = 0; j < kChunksPerKt; ++j) {
     const int c = kt * kChunksPerKt + j;
     if (blk != nullptr && c < kchunks)
-      v[j] = ldg_stream(blk + c * 512);
+      v[j] = ldg_stream_hint(blk + c * 512, pol);
     else
       v[j] = make_uint4(0u, 0u, 0u, 0u);
   }
@@ -311,6 +313,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
     constexpr int split = RL::kSplitA;
     const uint32_t full_l = leader_addr(full(0));
     const uint8_t* codes = is_a ? p.a_codes : p.w_codes;
+    // The raster keeps a group of m-pairs' activation codes for every n-tile, so
+    // they are kept in L2 ahead of the weight tiles streaming past them.
+    const uint64_t pol = is_a ? l2_evict_last() : l2_evict_normal();
     const int rb_count = is_a ? p.t_blocks : p.n_blocks;
     // This lane's first byte of the row block a tile needs (nullptr: the block
     // lies past the buffer's rows). Computed once per tile, not per load.
@@ -359,7 +364,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
     for (int i = 0; i < kPrefetch; ++i) {
       sring[i] = 0u;
       if (ld_tile < num_tiles) {
-        load_kt(block_ptr(ld_tile), p.kchunks, ld_kt, ring[i]);
+        load_kt(block_ptr(ld_tile), p.kchunks, ld_kt, ring[i], pol);
         sring[i] = load_shift(shift_ptr(ld_tile), ld_kt);
       }
       advance(ld_tile, ld_kt);
@@ -435,7 +440,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
             blk = block_ptr(ld_tile);
             sblk = shift_ptr(ld_tile);
           }
-          load_kt(blk, p.kchunks, ld_kt, ring[slot]);
+          load_kt(blk, p.kchunks, ld_kt, ring[slot], pol);
           sring[slot] = load_shift(sblk, ld_kt);
         }
         advance(ld_tile, ld_kt);
@@ -450,6 +455,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
     }
   } else {
     // ---------------- epilogue ----------------
+    const uint64_t out_pol = l2_evict_first();  // outputs: nothing here reads them again
     const int quarter = warp & 3;              // TMEM lanes this warp may read
     const int half = (warp - kFirstEpi) / 4;   // which kEpiCols accumulator columns
     const int et = threadIdx.x - kFirstEpi * 32;
@@ -588,7 +594,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
             const float accf = kPlus8 ? (__uint_as_float(acc[jj]) + Rt[jc + jj]) * kAccScale : __uint_as_float(acc[jj]);
             z[jj] = Ws[jc + jj] * fmaf(sa, accf, __uint_as_float(cr[jj]));
           }
-          store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, z, nvalid);
+          store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, z, nvalid, out_pol);
           if (p.acc_debug != nullptr) {
             int32_t* d = p.acc_debug + static_cast<int64_t>(t) * p.N + nb;
 #pragma unroll
@@ -650,7 +656,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
               sts128(orow_s + (c + h) * CW * 2, hv[0], hv[1], hv[2], hv[3]);
               sts128(orow_s + (c + h) * CW * 2 + 16, hv[4], hv[5], hv[6], hv[7]);
             } else {
-              store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, y, nvalid);
+              store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, y, nvalid, out_pol);
             }
             if (p.acc_debug != nullptr) {
               int32_t* d = p.acc_debug + static_cast<int64_t>(t) * p.N + nb;
@@ -664,7 +670,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
           const int ncols = p.N - n0 < kEpiCols ? p.N - n0 : kEpiCols;
           fence_proxy_async_smem();  // the row's shared stores, visible to the bulk copy
           bulk_store(static_cast<uint16_t*>(p.out) + static_cast<int64_t>(t) * p.ldo + n0, orow_s,
-                     static_cast<uint32_t>(ncols) * 2);
+                     static_cast<uint32_t>(ncols) * 2, out_pol);
           bulk_commit();
         }
       } else {
@@ -701,7 +707,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(Roles<kOneBlock>::kT
             const float accf = a[jj] * kAccScale;
             y[jj] = jj < nvalid ? __ldg(p.w_scale + nb + jj) * fmaf(sa, accf, y[jj]) : 0.f;
           }
-          store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, y, nvalid);
+          store_out<OUT, CW>(p.out, static_cast<int64_t>(t) * p.ldo + nb, y, nvalid, out_pol);
           if (p.acc_debug != nullptr) {
             int32_t* d = p.acc_debug + static_cast<int64_t>(t) * p.N + nb;
 #pragma unroll

@@ -148,6 +148,40 @@ __device__ __forceinline__ uint4 ldg_stream(const uint8_t* p) {
   return r;
 }
 
+// L2 eviction policies (createpolicy): evict_last for operand codes that later
+// tiles read again, evict_first for outputs, which nothing in the kernel reads.
+__device__ __forceinline__ uint64_t l2_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t l2_evict_normal() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t l2_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+// ldg_stream with an L2 eviction policy.
+__device__ __forceinline__ uint4 ldg_stream_hint(const uint8_t* p, uint64_t pol) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.L2::cache_hint.v4.u32 {%0,%1,%2,%3}, [%4], %5;"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p), "l"(pol));
+  return r;
+}
+
+// A 16-byte global store with an L2 eviction policy.
+__device__ __forceinline__ void stg_hint(void* p, uint4 v, uint64_t pol) {
+  asm volatile("st.global.L2::cache_hint.v4.b32 [%0], {%1,%2,%3,%4}, %5;" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z),
+               "r"(v.w), "l"(pol)
+               : "memory");
+}
+
 // Bulk copy global -> this CTA's shared memory, completing `bytes` on the
 // mbarrier at `bar` (both addresses 16-byte aligned, bytes a multiple of 16).
 __device__ __forceinline__ void bulk_load(uint32_t sdst, const void* gsrc, uint32_t bytes, uint32_t bar) {
@@ -157,9 +191,11 @@ __device__ __forceinline__ void bulk_load(uint32_t sdst, const void* gsrc, uint3
                : "memory");
 }
 
-// Bulk copy shared -> global (async proxy), tracked per thread in bulk groups.
-__device__ __forceinline__ void bulk_store(void* gdst, uint32_t ssrc, uint32_t bytes) {
-  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(gdst), "r"(ssrc), "r"(bytes)
+// Bulk copy shared -> global (async proxy), tracked per thread in bulk groups,
+// with an L2 eviction policy for the written lines.
+__device__ __forceinline__ void bulk_store(void* gdst, uint32_t ssrc, uint32_t bytes, uint64_t pol) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group.L2::cache_hint [%0], [%1], %2, %3;" ::"l"(gdst),
+               "r"(ssrc), "r"(bytes), "l"(pol)
                : "memory");
 }
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
@@ -217,14 +253,26 @@ __device__ __forceinline__ void widen_mx(uint32_t w, uint32_t lut_lo, uint32_t l
   hi = mx_bytes((w >> 4) & 0x0F0F0F0Fu, lut_lo, lut_hi);
 }
 
+// A 16-byte store, with the L2 policy pol unless pol is 0.
+__device__ __forceinline__ void stg_maybe_hint(void* p, uint4 v, uint64_t pol) {
+  if (pol != 0)
+    stg_hint(p, v, pol);
+  else
+    *reinterpret_cast<uint4*>(p) = v;
+}
+
+// Outputs of CW consecutive columns (nvalid of them inside the matrix); whole
+// runs leave by 16-byte stores, with the L2 policy pol unless pol is 0.
 template <int OUT, int CW>
-__device__ __forceinline__ void store_out(void* out, int64_t off, const float* y, int nvalid) {
+__device__ __forceinline__ void store_out(void* out, int64_t off, const float* y, int nvalid, uint64_t pol = 0) {
   if (OUT == OFFQ_F32) {
     float* o = static_cast<float*>(out) + off;
     if (nvalid == CW) {
 #pragma unroll
       for (int i = 0; i < CW / 4; ++i)
-        *reinterpret_cast<float4*>(o + 4 * i) = make_float4(y[4 * i], y[4 * i + 1], y[4 * i + 2], y[4 * i + 3]);
+        stg_maybe_hint(o + 4 * i, make_uint4(__float_as_uint(y[4 * i]), __float_as_uint(y[4 * i + 1]),
+                                             __float_as_uint(y[4 * i + 2]), __float_as_uint(y[4 * i + 3])),
+                       pol);
     } else {
 #pragma unroll
       for (int i = 0; i < CW; ++i)
@@ -246,7 +294,7 @@ __device__ __forceinline__ void store_out(void* out, int64_t off, const float* y
     if (nvalid == CW) {
 #pragma unroll
       for (int i = 0; i < CW / 8; ++i)
-        *reinterpret_cast<uint4*>(o + 8 * i) = make_uint4(p[4 * i], p[4 * i + 1], p[4 * i + 2], p[4 * i + 3]);
+        stg_maybe_hint(o + 8 * i, make_uint4(p[4 * i], p[4 * i + 1], p[4 * i + 2], p[4 * i + 3]), pol);
     } else {
 #pragma unroll
       for (int i = 0; i < CW; ++i)
