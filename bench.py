@@ -751,7 +751,8 @@ def time_decode(device, args, flush_l2, stream):
     if st != Q.OFFQ_OK:
         raise RuntimeError(f"device status after the decode sweep: {Q.status_string(st)}")
     del sets
-    out["roofline"] = {"bound": "hbm", "kernel": f"w4a4_decode_kernel weight stream (T = {best['T']})",
+    kern = "w4a4_gemv_kernel (dp4a, T <= 4)" if best["T"] <= 4 else "w4a4_decode_kernel (tcgen05, 4 < T <= 64)"
+    out["roofline"] = {"bound": "hbm", "kernel": f"{kern} weight stream (T = {best['T']})",
                        "achieved": best["weight_gbs"], "peak": peaks["hbm_gbs"], "unit": "GB/s",
                        "frac": best["weight_frac"], "bytes": w_bytes}
     return out

@@ -411,6 +411,179 @@ int launch_decode(const DecodeParams& p, int grid, cudaStream_t s) {
   return launch_pdl(w4a4_decode_kernel<OUT>, dim3(grid), dim3(kDecThreads), bytes, s, p);
 }
 
+// ---------------------------------------------------------------------------
+// Few-token form (T <= 4): integer dot products on the CUDA cores.
+//
+// At T <= 4 every weight code meets at most 4 activations, so widening it for
+// the tensor cores costs more than the products: the weights stream from HBM
+// straight into registers and meet the activations in dp4a (four int8
+// products per instruction, exact int32 sums). (Measured on 4096 -> 11008:
+// 10.3 us at one token, 16.4 us at eight, where the tensor-core form takes
+// 14.9; the sign-magnitude unpacking and one dp4a per 4 codes and token make
+// the cost grow with T.) A CTA owns one 32-row weight block: lane l of each of
+// its 8 warps takes row l, warp w a contiguous eighth of the K chunks, 8
+// chunks (128 B of codes per lane) in flight;
+// the warps' partial sums meet in shared memory. The activation codes
+// (u = q + 8 nibbles) are unpacked once per CTA into shared memory as the byte
+// vectors dp4a takes, so the accumulator is acc' = sum (q_a + 8) q_w and the
+// epilogue is the decode kernel's, term for term.
+// ---------------------------------------------------------------------------
+constexpr int kGemvWarps = 8;
+constexpr int kGemvBatch = 8;  // chunks of weight codes in flight per lane (128 B)
+constexpr int kGemvMaxT = 4;
+constexpr int kGemvMaxActBytes = 96 * 1024;  // NT * K bytes of unpacked activations
+
+struct GemvParams {
+  const uint8_t* a_codes;
+  const uint8_t* w_codes;
+  const float* a_scale;
+  const float* a_offset;
+  const float* w_scale;
+  const float* rowsum;   // [G][N]
+  void* out;
+  int64_t ldo;
+  int32_t* acc_debug;
+  int T, N, G, kchunks;
+};
+
+// Eight interleaved sign-magnitude weight codes (one 32-bit word, channels
+// c0..c7) as two vectors of signed bytes: even = (c0, c2, c4, c6),
+// odd = (c1, c3, c5, c7). Byte j holds |q(c2j)| in bits 0-2 and its sign in
+// bit 7, |q(c2j+1)| in bits 4-6, and in bit 3 the sign of c(2j-1 mod 8), so
+// the odd signs sit one byte up (rotate by 8). Negation is (m ^ 0xFF) + 1 per
+// byte, with no carry out of a byte since a code of magnitude 0 has sign 0.
+__device__ __forceinline__ void weight_bytes(uint32_t w, int& even, int& odd) {
+  const uint32_t me = w & 0x07070707u;
+  const uint32_t se = (w >> 7) & 0x01010101u;
+  even = static_cast<int>((me ^ (se * 0xFFu)) + se);
+  const uint32_t mo = (w >> 4) & 0x07070707u;
+  const uint32_t so = (__funnelshift_r(w, w, 8) >> 3) & 0x01010101u;
+  odd = static_cast<int>((mo ^ (so * 0xFFu)) + so);
+}
+
+template <int OUT, int NT>
+__global__ void __launch_bounds__(kGemvWarps * 32, 3) w4a4_gemv_kernel(const GemvParams p) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  // act: [NT][kchunks][8] words (E0 O0 E1 O1 E2 O2 E3 O3 of a 32-code chunk);
+  // red: [kGemvWarps][NT][32] partial sums.
+  uint32_t* act = reinterpret_cast<uint32_t*>(smem);
+  int* red = reinterpret_cast<int*>(smem + static_cast<size_t>(NT) * p.kchunks * 32);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int rb = blockIdx.x;  // weight row block
+  const int kc = p.kchunks;
+  // This warp's K chunks and the first batch of weight loads. They are issued
+  // before the wait for the kernel ahead in the stream (programmatic dependent
+  // launch), which produces the activations, not the weights: no kernel of this
+  // library that writes weight codes releases its dependents early.
+  const int per = (kc + kGemvWarps - 1) / kGemvWarps;
+  const int c0 = warp * per;
+  const int c1 = c0 + per < kc ? c0 + per : kc;
+  const uint8_t* wrow = p.w_codes + (static_cast<int64_t>(rb) * kc) * 512 + lane * 16;
+  uint4 wv[kGemvBatch];
+#pragma unroll
+  for (int i = 0; i < kGemvBatch; ++i)
+    wv[i] = c0 + i < c1 ? ldg_stream(wrow + static_cast<int64_t>(c0 + i) * 512) : make_uint4(0u, 0u, 0u, 0u);
+  griddep_wait();
+  griddep_launch_dependents();
+
+  // Unpack the activation codes: token t, chunk c -> 8 words of byte vectors.
+  for (int i = threadIdx.x; i < NT * kc; i += kGemvWarps * 32) {
+    const int t = i / kc, c = i - t * kc;
+    uint4 a = make_uint4(0u, 0u, 0u, 0u);
+    if (t < p.T) a = __ldg(reinterpret_cast<const uint4*>(p.a_codes + ((t >> 5) * kc + c) * 512 + (t & 31) * 16));
+    uint4* dst = reinterpret_cast<uint4*>(act + static_cast<size_t>(i) * 8);
+    dst[0] = make_uint4(a.x & 0x0F0F0F0Fu, (a.x >> 4) & 0x0F0F0F0Fu, a.y & 0x0F0F0F0Fu, (a.y >> 4) & 0x0F0F0F0Fu);
+    dst[1] = make_uint4(a.z & 0x0F0F0F0Fu, (a.z >> 4) & 0x0F0F0F0Fu, a.w & 0x0F0F0F0Fu, (a.w >> 4) & 0x0F0F0F0Fu);
+  }
+  __syncthreads();
+
+  int acc[NT];
+#pragma unroll
+  for (int t = 0; t < NT; ++t) acc[t] = 0;
+  for (int cb = c0; cb < c1; cb += kGemvBatch) {
+#pragma unroll
+    for (int i = 0; i < kGemvBatch; ++i) {
+      const int c = cb + i;
+      if (c >= c1) break;
+      const uint4 w = wv[i];
+      // The load kGemvBatch chunks ahead takes this register.
+      const int cn = c + kGemvBatch;
+      wv[i] = cn < c1 ? ldg_stream(wrow + static_cast<int64_t>(cn) * 512) : make_uint4(0u, 0u, 0u, 0u);
+      int e0, o0, e1, o1, e2, o2, e3, o3;
+      weight_bytes(w.x, e0, o0);
+      weight_bytes(w.y, e1, o1);
+      weight_bytes(w.z, e2, o2);
+      weight_bytes(w.w, e3, o3);
+#pragma unroll
+      for (int t = 0; t < NT; ++t) {
+        const uint4* av = reinterpret_cast<const uint4*>(act + (static_cast<size_t>(t) * kc + c) * 8);
+        const uint4 a0 = av[0], a1 = av[1];
+        int s = acc[t];
+        s = __dp4a(e0, static_cast<int>(a0.x), s);
+        s = __dp4a(o0, static_cast<int>(a0.y), s);
+        s = __dp4a(e1, static_cast<int>(a0.z), s);
+        s = __dp4a(o1, static_cast<int>(a0.w), s);
+        s = __dp4a(e2, static_cast<int>(a1.x), s);
+        s = __dp4a(o2, static_cast<int>(a1.y), s);
+        s = __dp4a(e3, static_cast<int>(a1.z), s);
+        s = __dp4a(o3, static_cast<int>(a1.w), s);
+        acc[t] = s;
+      }
+    }
+  }
+#pragma unroll
+  for (int t = 0; t < NT; ++t) red[(warp * NT + t) * 32 + lane] = acc[t];
+  __syncthreads();
+
+  // Epilogue: thread (t, lane) for row n = 32 rb + lane, as the decode kernel's:
+  // corr = sum_b o[t][b] R[b][n] (block 0 multiplied, then FMAs in block order),
+  // a = acc' - 8 Rt[n] (exact), y = s_w * fma(s_a, a, corr).
+  const int t = threadIdx.x >> 5;
+  const int n = rb * 32 + lane;
+  if (t < NT && t < p.T && n < p.N) {
+    int accp = 0;
+#pragma unroll
+    for (int w = 0; w < kGemvWarps; ++w) accp += red[(w * NT + t) * 32 + lane];
+    float rt = 0.f, corr = 0.f;
+    for (int b = 0; b < p.G; ++b) {
+      const float rv = __ldg(p.rowsum + static_cast<int64_t>(b) * p.N + n);
+      rt += rv;
+      if (p.a_offset != nullptr) {
+        const float o = __ldg(p.a_offset + static_cast<int64_t>(t) * p.G + b);
+        corr = b == 0 ? o * rv : fmaf(o, rv, corr);
+      }
+    }
+    const float a = static_cast<float>(accp - 8 * static_cast<int>(rt));
+    const float y = __ldg(p.w_scale + n) * fmaf(__ldg(p.a_scale + t), a, corr);
+    const int64_t off = static_cast<int64_t>(t) * p.ldo + n;
+    if (OUT == OFFQ_F32) {
+      static_cast<float*>(p.out)[off] = y;
+    } else if (OUT == OFFQ_BF16) {
+      static_cast<__nv_bfloat16*>(p.out)[off] = __float2bfloat16_rn(y);
+    } else {
+      static_cast<__half*>(p.out)[off] = __float2half_rn(y);
+    }
+    if (p.acc_debug != nullptr) p.acc_debug[static_cast<int64_t>(t) * p.N + n] = accp;
+  }
+}
+
+template <int OUT, int NT>
+int launch_gemv(const GemvParams& p, int blocks, cudaStream_t s) {
+  const size_t bytes = static_cast<size_t>(NT) * p.kchunks * 32 + static_cast<size_t>(kGemvWarps) * NT * 32 * 4;
+  if (bytes > 48 * 1024 && !smem_optin<w4a4_gemv_kernel<OUT, NT>>(kGemvMaxActBytes + kGemvWarps * kGemvMaxT * 32 * 4))
+    return OFFQ_ERR_CUDA;
+  return launch_pdl(w4a4_gemv_kernel<OUT, NT>, dim3(blocks), dim3(kGemvWarps * 32), bytes, s, p);
+}
+
+template <int OUT>
+int dispatch_gemv(const GemvParams& p, int nt, int blocks, cudaStream_t s) {
+  switch (nt) {
+    case 1: return launch_gemv<OUT, 1>(p, blocks, s);
+    case 2: return launch_gemv<OUT, 2>(p, blocks, s);
+    default: return launch_gemv<OUT, 4>(p, blocks, s);
+  }
+}
+
 }  // namespace
 
 namespace offq {
@@ -421,6 +594,31 @@ int decode_max_tokens() { return kDecMaxT; }
 int w4a4_linear_decode(const uint8_t* a_codes, const float* a_scale, const float* a_offset, int64_t T, int64_t N,
                        int64_t K, int32_t g, const uint8_t* w_codes, const float* w_scale, const float* w_offsum,
                        void* out, int out_dtype, int64_t ldo, int32_t* acc_debug, cudaStream_t stream) {
+  const int nt = T <= 1 ? 1 : (T <= 2 ? 2 : 4);
+  if (T <= kGemvMaxT && static_cast<int64_t>(nt) * K <= kGemvMaxActBytes) {
+    GemvParams q{};
+    q.a_codes = a_codes;
+    q.w_codes = w_codes;
+    q.a_scale = a_scale;
+    q.a_offset = a_offset;
+    q.w_scale = w_scale;
+    q.rowsum = w_offsum;
+    q.out = out;
+    q.ldo = ldo;
+    q.acc_debug = acc_debug;
+    q.T = static_cast<int>(T);
+    q.N = static_cast<int>(N);
+    q.G = static_cast<int>(K / g);
+    q.kchunks = static_cast<int>(K / 32);
+    const int64_t blocks = (N + 31) / 32;
+    if (blocks > 0x7FFFFFFF) return OFFQ_ERR_UNSUPPORTED;
+    switch (out_dtype) {
+      case OFFQ_F32: return dispatch_gemv<OFFQ_F32>(q, nt, static_cast<int>(blocks), stream);
+      case OFFQ_BF16: return dispatch_gemv<OFFQ_BF16>(q, nt, static_cast<int>(blocks), stream);
+      case OFFQ_F16: return dispatch_gemv<OFFQ_F16>(q, nt, static_cast<int>(blocks), stream);
+      default: return OFFQ_ERR_INVALID_ARG;
+    }
+  }
   const int sms = decode_num_sms();
   if (sms < 1) return OFFQ_ERR_CUDA;
   const int64_t nblk = (N + 31) / 32;

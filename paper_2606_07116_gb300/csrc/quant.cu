@@ -1632,10 +1632,11 @@ int check_row_shape(int64_t K, int32_t g) {
 // Offline: activation-format codes (q + 8) -> weight format, in place, plus the
 // integer block row sums R[b][n]; the padding rows of the last 32-row tile are
 // zeroed. Codes are in the tiled operand layout. One thread per (row, block).
+// It does not release its dependents early: the few-token GEMM starts reading
+// weight codes and row sums before it waits for the kernel ahead of it.
 __global__ void weight_repack_kernel(uint8_t* __restrict__ codes, float* __restrict__ rowsum, int64_t N,
                                      int64_t N_pad, int K, int g) {
   griddep_wait();
-  griddep_launch_dependents();
   const int G = K / g;
   const int64_t id = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (id >= N_pad * G) return;
