@@ -149,7 +149,8 @@ int offq_quantize_act(const void* x, int x_dtype, int64_t T, int64_t K, int64_t 
  *           + s_w[n] * sum_b o[t][b] * R[b][n]
  *
  * accumulated exactly in integers (the tensor cores see both codes as exact
- * fp8 values; every partial sum is an integer below 2^24), dequantized in fp32
+ * fp8 values; at T <= 4 the CUDA cores use dp4a; every partial sum is an
+ * integer below 2^24), dequantized in fp32
  * and rounded once to the output type.
  *
  *   a_codes   device, tiled activation codes of T rows (offq_quantize_act), 16-B aligned.
@@ -171,6 +172,15 @@ int offq_quantize_act(const void* x, int x_dtype, int64_t T, int64_t K, int64_t 
  *   acc_debug device, [T][N] int32 or NULL. When given, also receives the
  *             integer the tensor cores accumulate, sum_k (q_a + 8) * q_w
  *             (equal to the true dot product plus 8 * sum_k q_w[n][k]).
+ * Forms: T > 64 the pair-tile tensor-core kernel; 5 <= T <= 64 the decode
+ * kernel (weights on the MMA's M side); T <= 4 (with T' * K <= 96 KB, T'
+ * the token count rounded up to 1, 2 or 4) the CUDA-core form. All give the
+ * same accumulator and apply the same epilogue.
+ * Ordering: the T <= 4 form starts reading w_codes before the kernel ahead of
+ * it in the stream has finished (programmatic dependent launch), so the
+ * weight codes must not be written by a kernel that releases its dependents
+ * early (ordinary kernels never do; no kernel of this library that writes
+ * weight codes does).
  */
 int offq_w4a4_linear(const uint8_t* a_codes, const float* a_scale, const float* a_offset,
                      int64_t T, int64_t N, int64_t K, int32_t g,
