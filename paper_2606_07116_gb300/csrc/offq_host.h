@@ -79,6 +79,10 @@ inline bool smem_optin(int bytes) {
 // most, and the launch for 1 <= T <= decode_max_tokens() with arguments
 // already checked by offq_w4a4_linear.
 int decode_max_tokens();
+// MXFP4 activation rows on the persistent warp-per-1024-channel layout; 1 when
+// the shape or row count does not suit it (csrc/quant.cu).
+int quantize_mx_rows_fast(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx, int32_t g, int32_t flags,
+                          uint8_t* codes, uint8_t* shifts, float* row_scale, float* offset, cudaStream_t s);
 int w4a4_linear_decode(const uint8_t* a_codes, const float* a_scale, const float* a_offset, int64_t T, int64_t N,
                        int64_t K, int32_t g, const uint8_t* w_codes, const float* w_scale, const float* w_offsum,
                        void* out, int out_dtype, int64_t ldo, int32_t* acc_debug, cudaStream_t stream);

@@ -71,6 +71,8 @@ struct QuantArgs {
   int* status;      // device status word (bounded waits that run out write here)
   int ring_slots;   // persistent forms: slots of rows_per_cta rows each (1 to 3)
   long long wait_cycles;  // persistent forms: budget of a wait for a staged row (kWaitCycles unless a test sets it)
+  uint8_t* shifts;  // MXFP4 form: tiled block shifts (else nullptr)
+  int g;            // MXFP4 form: the offset block
 };
 
 template <int L>
@@ -966,6 +968,220 @@ __global__ void __launch_bounds__(k1kMaxWarps * 32, 1) quantize_rows_1k_kernel(c
   }
 }
 
+// MXFP4 rows (the Sec. 3.4 extension), persistent, on the layout of
+// quantize_rows_1k_kernel: a warp per 1024 channels, so after the rotation (or,
+// without it, straight from the staged row) lane l holds the 32 consecutive
+// channels 32 l + j of its warp's span, one whole MX block. Per row: offsets
+// (the block-leading channel over sqrt(1024) with the rotation; without it the
+// mean over g = 1024 m channels by a balanced tree, across the m warps of the
+// block through shared memory), the residual, the lane's block exponent
+// X = floor(log2 amax) - 2, the row's largest through shared memory (one
+// barrier), X kept within 6 of it, then the codes by the E2M1 conversion
+// instruction (round to nearest even, saturating at 6; a code of magnitude 0
+// keeps sign 0), one 16-byte store of the block's codes and its shift byte.
+// With the rotation the values are 32 r (unnormalised by sqrt(1024) = 2^5,
+// exact), so their exponents are offset by 5.
+
+// floor(log2(a)) for a normal positive fp32 a, from its exponent field.
+__device__ __forceinline__ int floor_log2(float a) { return static_cast<int>((__float_as_uint(a) >> 23) & 0xFF) - 127; }
+
+// 2^e as fp32 for -126 <= e <= 127.
+__device__ __forceinline__ float pow2f(int e) { return __uint_as_float(static_cast<uint32_t>(e + 127) << 23); }
+
+// Two fp32 values -> one byte of E2M1 codes (hi in bits 4-7, lo in bits 0-3).
+__device__ __forceinline__ uint32_t e2m1x2(float hi, float lo) {
+  uint16_t r;
+  asm("{\n.reg .b8 t;\ncvt.rn.satfinite.e2m1x2.f32 t, %1, %2;\nmov.b16 %0, {t, 0};\n}" : "=h"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// Clears the sign bit of every nibble whose magnitude bits are 0 (E2M1 -0 -> +0).
+__device__ __forceinline__ uint32_t e2m1_clear_neg_zero(uint32_t w) {
+  const uint32_t mag = w & 0x77777777u;
+  const uint32_t nonzero = (mag + 0x77777777u) & 0x88888888u;  // bit 3 of each nibble: magnitude >= 1
+  return mag | (w & nonzero);
+}
+
+template <typename Tin, bool kRot>
+__global__ void __launch_bounds__(k1kMaxWarps * 32, 1) quantize_mx_1k_kernel(const QuantArgs a) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  __shared__ int abort_flag;
+  __shared__ float wpart[k1kMaxWarps];  // per-warp block sums (no rotation, g > 1024)
+  __shared__ int wmaxx[k1kMaxWarps];    // per-warp largest block exponent (+ 1024)
+  const int K = a.K, R = a.rows_per_cta;
+  const int nbw = K / 1024;  // warps per row
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int lrow = warp / nbw;
+  const int b = warp - lrow * nbw;          // 1024-channel span of this warp
+  const int m = a.g / 1024;                 // warps per offset block (no rotation)
+  const int G = a.G;
+  const bool offs = (a.flags & OFFQ_OFFSET) != 0;
+  const uint32_t scr32 = smem_u32(smem) + 4096u * warp;  // the warp's transpose scratch (rotation)
+  RowRing ring;
+  ring.base = smem + (kRot ? static_cast<size_t>(R) * nbw * 4096 : 0);
+  ring.slot_bytes = static_cast<uint32_t>(R) * K * sizeof(Tin);
+  ring.S = a.ring_slots;
+  ring.bar0 = smem_u32(ring.base + static_cast<size_t>(ring.S) * ring.slot_bytes);
+  ring.s = 0;
+  ring.phase = 0;
+  const int ngroups = static_cast<int>((a.rows + R - 1) / R);
+  int grp = blockIdx.x;
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    for (int k = 0; k < ring.S; ++k) mbar_init(ring.bar0 + 8u * k, 1);
+    mbar_fence_init();
+  }
+  __syncthreads();
+  griddep_wait();
+  griddep_launch_dependents();
+  ring_start<Tin>(a, ring, R, ngroups);
+
+  const int cpr = K / 32;
+  const int nkt = K / 128;
+  while (true) {
+    const int row = grp * R + lrow;
+    const bool row_ok = row < a.rows;
+    float2 v[16];  // v[i] = channels (32 lane + 2i, 32 lane + 2i + 1) of the span, after pass 2
+    const bool ok = mbar_wait_for(ring.bar(), ring.phase, &abort_flag, a.wait_cycles);
+    float off = 0.f;
+    if constexpr (kRot) {
+      if (ok && row_ok) {
+        const Tin* p = reinterpret_cast<const Tin*>(ring.slot()) + static_cast<size_t>(lrow) * K + b * 1024 + lane;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = make_float2(smem_elem(p + 64 * i), smem_elem(p + 64 * i + 32));
+      } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = make_float2(0.f, 0.f);
+      }
+      if (offs && lane == 0) {
+        off = v[0].x;
+        v[0].x = 0.f;
+      }
+      fwht1k_pass(v);  // channel bits 5..9
+      {
+        uint32_t wb[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) wb[q] = scr32 + ((4u * lane) ^ (16u * q));
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          sts_f32(wb[(2 * i) & 7] + 128u * (2 * i), v[i].x);
+          sts_f32(wb[(2 * i + 1) & 7] + 128u * (2 * i + 1), v[i].y);
+        }
+      }
+      __syncwarp();
+      {
+        const uint32_t rb = scr32 + 128u * lane;
+        const uint32_t rx = 16u * (lane & 7);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const float4 f = lds_f32x4(rb + ((16u * k) ^ rx));
+          v[2 * k] = make_float2(f.x, f.y);
+          v[2 * k + 1] = make_float2(f.z, f.w);
+        }
+      }
+      fwht1k_pass(v);  // channel bits 0..4
+    } else {
+      if (ok && row_ok) {
+        const Tin* p = reinterpret_cast<const Tin*>(ring.slot()) + static_cast<size_t>(lrow) * K + b * 1024 + 32 * lane;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          float f[8];
+          load_chunk8_smem(p + 8 * c, f);
+#pragma unroll
+          for (int e = 0; e < 4; ++e) v[4 * c + e] = make_float2(f[2 * e], f[2 * e + 1]);
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = make_float2(0.f, 0.f);
+      }
+      if (offs) {
+        // Block mean over g = 1024 m channels: a tree over the lane's 32, the warp's
+        // 32 lanes, then the m warps of the block.
+        float2 t8[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) t8[i] = __fadd2_rn(v[i], v[i + 8]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) t8[i] = __fadd2_rn(t8[i], t8[i + 4]);
+#pragma unroll
+        for (int i = 0; i < 2; ++i) t8[i] = __fadd2_rn(t8[i], t8[i + 2]);
+        t8[0] = __fadd2_rn(t8[0], t8[1]);
+        float sum = t8[0].x + t8[0].y;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xFFFFFFFFu, sum, o);
+        if (m > 1) {
+          if (lane == 0) wpart[warp] = sum;
+          __syncthreads();
+          const int w0 = lrow * nbw + (b / m) * m;  // first warp of this offset block
+          float part[8];
+          for (int i = 0; i < 8; ++i) part[i] = i < m ? wpart[w0 + i] : 0.f;
+          // m is a power of two <= 8: pairwise
+          for (int h = 4; h > 0; h >>= 1)
+            for (int i = 0; i < h; ++i) part[i] += part[i + h];
+          sum = part[0];
+          __syncthreads();  // wpart is read before the next row writes it
+        }
+        off = sum * (1.0f / static_cast<float>(a.g));
+        const float2 o2 = make_float2(off, off);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = __fadd2_rn(v[i], make_float2(-o2.x, -o2.y));
+      }
+    }
+
+    // The lane's block exponent, then the row's largest.
+    float mx0 = 0.f, mx1 = 0.f;
+#pragma unroll
+    for (int i = 0; i < 16; i += 2) {
+      mx0 = fmax3(mx0, fabsf(v[i].x), fabsf(v[i].y));
+      mx1 = fmax3(mx1, fabsf(v[i + 1].x), fabsf(v[i + 1].y));
+    }
+    const float amax = fmaxf(mx0, mx1);
+    constexpr int kUnnorm = kRot ? 5 : 0;  // values are 2^5 r with the rotation
+    const int xl = amax > 0.f ? floor_log2(amax) - 2 - kUnnorm : -1000;
+    const uint32_t wx = __reduce_max_sync(0xFFFFFFFFu, static_cast<uint32_t>(xl + 1024));
+    if (lane == 0) wmaxx[warp] = static_cast<int>(wx);
+    if (!__syncthreads_and(ok)) {
+      ring_fail(ring, grp, ngroups, a.status);
+      return;
+    }
+    const int next = grp + ring.S * static_cast<int>(gridDim.x);
+    if (threadIdx.x == 0 && next < ngroups) ring_issue<Tin>(a, next, R, ring.slot(), ring.bar());
+    ring.advance();
+    int xmax = static_cast<int>(__reduce_max_sync(0xFFFFFFFFu, lane < nbw ? static_cast<uint32_t>(wmaxx[lrow * nbw + lane]) : 0u)) - 1024;
+    if (xmax < -900) xmax = 0;  // an all-zero row: any exponent
+    const int xlo = xmax - 6;
+    const int X = xl > xlo ? xl : xlo;
+    const float sc = pow2f(-(X + kUnnorm));
+    uint32_t wd[4];
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      uint32_t bytes[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float2 f = v[4 * w + q];
+        bytes[q] = e2m1x2(f.y * sc, f.x * sc);
+      }
+      wd[w] = e2m1_clear_neg_zero(bytes[0] | (bytes[1] << 8) | (bytes[2] << 16) | (bytes[3] << 24));
+    }
+    if (row_ok) {
+      const int mb = b * 32 + lane;  // the row's MX block
+      uint8_t* rdst = a.codes + static_cast<int64_t>(row >> 5) * cpr * 512 + (row & 31) * 16;
+      *reinterpret_cast<uint4*>(rdst + static_cast<int64_t>(mb) * 512) = make_uint4(wd[0], wd[1], wd[2], wd[3]);
+      a.shifts[((static_cast<int64_t>(row >> 5) * nkt + (mb >> 2)) * 32 + (row & 31)) * 4 + (mb & 3)] =
+          static_cast<uint8_t>(X - xlo);
+      if (b == 0 && lane == 0) a.scale[row] = pow2f(xlo);
+      if (lane == 0 && a.offset != nullptr) {
+        if constexpr (kRot) {
+          a.offset[static_cast<int64_t>(row) * G + b] = offs ? off * 0.03125f : 0.f;
+        } else {
+          if (b % m == 0) a.offset[static_cast<int64_t>(row) * G + b / m] = offs ? off : 0.f;
+        }
+      }
+    }
+    grp += gridDim.x;
+    if (grp >= ngroups) break;
+  }
+}
+
 // Rows without the rotation whose offset block is the whole row (g == K): one
 // warp per row. Each lane issues the loads of up to CB 8-element chunks at once
 // and keeps them (raw) in registers, so a row of up to 256*CB elements costs one
@@ -1536,6 +1752,50 @@ int launch_1k(QuantArgs a, cudaStream_t stream) {
   return launch_pdl(kern, dim3(static_cast<unsigned>(grid)), dim3(threads), smem, stream, a);
 }
 
+// quantize_mx_1k_kernel: one row of K/1024 warps per CTA (rows per CTA grow
+// while a CTA has fewer than 4 warps), the ring as launch_1k's. kNoRing when the
+// shape does not fit it (the generic MX kernel serves those).
+template <typename Tin, bool kRot>
+int launch_mx_1k(QuantArgs a, cudaStream_t stream) {
+  const int nbw = a.K / 1024;
+  if (a.H != 1 || a.K % 1024 != 0 || nbw > k1kMaxWarps) return kNoRing;
+  if (kRot ? a.g != 1024 : (a.g % 1024 != 0 || a.g / 1024 > 8)) return kNoRing;
+  const int sms = sm_count();
+  if (sms <= 0) return OFFQ_ERR_CUDA;
+  const int R = std::max(1, 4 / nbw);
+  const int64_t groups = (a.rows + R - 1) / R;
+  if (groups <= sms || a.rows + R > 0x7FFFFFFF) return kNoRing;
+  auto kern = quantize_mx_1k_kernel<Tin, kRot>;
+  if (prefer_max_shared(kern) != OFFQ_OK) return OFFQ_ERR_CUDA;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kMaxDynSmem)) !=
+      cudaSuccess)
+    return OFFQ_ERR_CUDA;
+  const int threads = R * nbw * 32;
+  const size_t fixed = kRot ? static_cast<size_t>(R) * nbw * 4096 : 0;
+  const size_t slot = static_cast<size_t>(R) * a.K * sizeof(Tin) + 8;
+  int best_s = 0, best_per_sm = 0;
+  for (int S = 1; S <= 3; ++S) {
+    const size_t smem = fixed + S * slot;
+    if (smem > kMaxDynSmem) break;
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem) != cudaSuccess)
+      return OFFQ_ERR_CUDA;
+    if (per_sm < 1) break;
+    const bool better = best_s == 0 || (best_s == 1 && S >= 2) || (S >= 2 && per_sm >= best_per_sm);
+    if (better) {
+      best_s = S;
+      best_per_sm = per_sm;
+    }
+  }
+  if (best_s == 0) return kNoRing;
+  a.rows_per_cta = R;
+  a.ring_slots = best_s;
+  a.tpr = nbw * 32;
+  const size_t smem = fixed + best_s * slot;
+  const int64_t grid = std::min<int64_t>(groups, static_cast<int64_t>(sms) * best_per_sm);
+  return launch_pdl(kern, dim3(static_cast<unsigned>(grid)), dim3(threads), smem, stream, a);
+}
+
 template <typename Tin>
 int launch_stream(const QuantArgs& a, cudaStream_t stream) {
   const int64_t grid = (a.rows + 7) / 8;
@@ -1673,6 +1933,42 @@ __global__ void weight_repack_kernel(uint8_t* __restrict__ codes, float* __restr
 }
 
 }  // namespace
+
+namespace offq {
+
+// The MXFP4 row quantizer on the warp-per-1024-channel layout (arguments checked
+// by the caller). Returns 1 when the shape or the row count does not suit it.
+int quantize_mx_rows_fast(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx, int32_t g, int32_t flags,
+                          uint8_t* codes, uint8_t* shifts, float* row_scale, float* offset, cudaStream_t s) {
+  QuantArgs a{};
+  a.x = x;
+  a.ld_t = ldx;
+  a.ld_h = 0;
+  a.rows = rows;
+  a.H = 1;
+  a.K = static_cast<int>(K);
+  a.G = static_cast<int>(K / g);
+  a.flags = flags;
+  a.codes = codes;
+  a.scale = row_scale;
+  a.offset = offset;
+  a.tiled = 1;
+  a.status = device_status_ptr();
+  a.wait_cycles = g_row_wait_cycles.load(std::memory_order_relaxed);
+  a.shifts = shifts;
+  a.g = g;
+  const bool rot = (flags & OFFQ_ROTATE) != 0;
+  int st = kNoRing;
+  switch (dtype) {
+    case OFFQ_BF16: st = rot ? launch_mx_1k<__nv_bfloat16, true>(a, s) : launch_mx_1k<__nv_bfloat16, false>(a, s); break;
+    case OFFQ_F16: st = rot ? launch_mx_1k<__half, true>(a, s) : launch_mx_1k<__half, false>(a, s); break;
+    case OFFQ_F32: st = rot ? launch_mx_1k<float, true>(a, s) : launch_mx_1k<float, false>(a, s); break;
+    default: return OFFQ_ERR_INVALID_ARG;
+  }
+  return st == kNoRing ? 1 : st;
+}
+
+}  // namespace offq
 
 extern "C" int offq_quantize_act(const void* x, int x_dtype, int64_t T, int64_t K, int64_t ldx, int32_t g,
                                  int32_t flags, uint8_t* codes, float* scale, float* offset, void* stream) {

@@ -272,8 +272,18 @@ int run_mx(const void* x, int dtype, int64_t rows, int64_t K, int64_t ldx, int32
 extern "C" int offq_quantize_act_mx(const void* x, int x_dtype, int64_t T, int64_t K, int64_t ldx, int32_t g,
                                     int32_t flags, uint8_t* codes, uint8_t* shifts, float* row_scale, float* offset,
                                     void* stream) {
-  return run_mx(x, x_dtype, T, K, ldx, g, flags, codes, shifts, row_scale, offset, nullptr, false,
-                static_cast<cudaStream_t>(stream));
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // Prefill-sized inputs of 1024-multiple widths take the persistent form; the
+  // arguments are checked by run_mx's rules first (a dry check with zero rows).
+  const int chk = run_mx(x, x_dtype, 0, K, ldx, g, flags, codes, shifts, row_scale, offset, nullptr, false, s);
+  if (chk != OFFQ_OK) return chk;
+  if (T > 0 && x != nullptr && codes != nullptr && shifts != nullptr && row_scale != nullptr &&
+      ((flags & OFFQ_OFFSET) == 0 || offset != nullptr) && aligned(x, 16) && (ldx * elem_bytes(x_dtype)) % 16 == 0 &&
+      aligned(codes, 16) && aligned(row_scale, 4) && (offset == nullptr || aligned(offset, 4))) {
+    const int st = quantize_mx_rows_fast(x, x_dtype, T, K, ldx, g, flags, codes, shifts, row_scale, offset, s);
+    if (st != 1) return st;
+  }
+  return run_mx(x, x_dtype, T, K, ldx, g, flags, codes, shifts, row_scale, offset, nullptr, false, s);
 }
 
 extern "C" int offq_prepare_weight_mx(const void* w, int dtype, int64_t N, int64_t K, int32_t g, int32_t rotate,

@@ -89,6 +89,26 @@ def test_mx_quantizer_parity(dt, T, K, g, rotate):
     assert np.all((sh >= 0) & (sh <= O.MX_SPAN))
 
 
+@pytest.mark.parametrize("T,K,g,rotate,dt", [
+    (700, 28672, 1024, True, "bf16"),     # Llama-2-70B down-proj width: one row of 28 warps per CTA
+    (1200, 8192, 8192, False, "bf16"),    # one offset block over the 8 warps of a row
+    (2000, 4096, 2048, False, "f16"),     # offset blocks of two warps
+    (1500, 2048, 1024, True, "f32"),      # two rows per CTA, fp32 rows
+    (5003, 1024, 1024, False, "bf16"),    # four rows of one warp per CTA, a ragged last group
+])
+def test_mx_quantizer_persistent_form(T, K, g, rotate, dt):
+    """Prefill-sized inputs take the persistent warp-per-1024-channel MX kernel: sampled rows
+    (first and last included) against the oracle."""
+    x = W.activations(T, K, seed=T + K + g, n_out=4, mult=100.0)
+    xe, codes, shifts, scale, off = _quant(x, g, rotate, dt)
+    rows = np.unique(np.concatenate([W.unit_index_sample(T, 96, seed=13), [0, 1, T - 2, T - 1]]))
+    ref = O.quantize_act_mx(xe[rows], g, rotate=rotate, offset=True)
+    code, sh, X = _decode(codes, shifts, scale, T, K)
+    check_mx(code[rows], X[rows], ref, xe[rows], g, rotate)
+    check_offsets(off.cpu().numpy()[rows], ref["offset"], xe[rows], g, rotate)
+    assert np.all((sh >= 0) & (sh <= O.MX_SPAN))
+
+
 def test_mx_weight_prep_and_block_sums():
     N, K, g = 300, 1024, 256
     w = W.weights(N, K, seed=91)
