@@ -465,7 +465,7 @@ template <int OUT, int NT>
 __global__ void __launch_bounds__(kGemvWarps * 32, 3) w4a4_gemv_kernel(const GemvParams p) {
   extern __shared__ __align__(16) uint8_t smem[];
   // act: [NT][kchunks][8] words (E0 O0 E1 O1 E2 O2 E3 O3 of a 32-code chunk);
-  // red: [kGemvWarps][NT][32] partial sums.
+  // red: [kGemvWarps][NT][32] partial sums; then the epilogue constants.
   uint32_t* act = reinterpret_cast<uint32_t*>(smem);
   int* red = reinterpret_cast<int*>(smem + static_cast<size_t>(NT) * p.kchunks * 32);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -483,19 +483,52 @@ __global__ void __launch_bounds__(kGemvWarps * 32, 3) w4a4_gemv_kernel(const Gem
 #pragma unroll
   for (int i = 0; i < kGemvBatch; ++i)
     wv[i] = c0 + i < c1 ? ldg_stream(wrow + static_cast<int64_t>(c0 + i) * 512) : make_uint4(0u, 0u, 0u, 0u);
+  // The epilogue's weight-side constants (thread (t, lane) of warps t < NT), also
+  // ahead of the wait: s_w[n] and Rt[n] = sum_b R[b][n].
+  // They wait in shared memory (ec: [4][NT][32] = s_w, Rt, s_a, corr), not in
+  // registers, which the loads in flight need.
+  float* ec = reinterpret_cast<float*>(red + kGemvWarps * NT * 32);
+  {
+    const int et = warp, n = rb * 32 + lane;
+    if (et < NT && n < p.N) {
+      float rt = 0.f;
+      for (int b = 0; b < p.G; ++b) rt += __ldg(p.rowsum + static_cast<int64_t>(b) * p.N + n);
+      ec[(0 * NT + et) * 32 + lane] = __ldg(p.w_scale + n);
+      ec[(1 * NT + et) * 32 + lane] = rt;
+    }
+  }
   griddep_wait();
   griddep_launch_dependents();
 
-  // Unpack the activation codes: token t, chunk c -> 8 words of byte vectors.
-  for (int i = threadIdx.x; i < NT * kc; i += kGemvWarps * 32) {
-    const int t = i / kc, c = i - t * kc;
+  // This warp unpacks the activation codes of its own chunks: token t, chunk c ->
+  // 8 words of byte vectors (no CTA barrier; the warp reads only what it wrote).
+  const int nw = c1 > c0 ? c1 - c0 : 0;
+  for (int i = lane; i < NT * nw; i += 32) {
+    const int t = i / nw, c = c0 + (i - t * nw);
     uint4 a = make_uint4(0u, 0u, 0u, 0u);
     if (t < p.T) a = __ldg(reinterpret_cast<const uint4*>(p.a_codes + ((t >> 5) * kc + c) * 512 + (t & 31) * 16));
-    uint4* dst = reinterpret_cast<uint4*>(act + static_cast<size_t>(i) * 8);
+    uint4* dst = reinterpret_cast<uint4*>(act + (static_cast<size_t>(t) * kc + c) * 8);
     dst[0] = make_uint4(a.x & 0x0F0F0F0Fu, (a.x >> 4) & 0x0F0F0F0Fu, a.y & 0x0F0F0F0Fu, (a.y >> 4) & 0x0F0F0F0Fu);
     dst[1] = make_uint4(a.z & 0x0F0F0F0Fu, (a.z >> 4) & 0x0F0F0F0Fu, a.w & 0x0F0F0F0Fu, (a.w >> 4) & 0x0F0F0F0Fu);
   }
-  __syncthreads();
+  // The activation-side constants of the epilogue: s_a[t] and the offset term
+  // corr = sum_b o[t][b] R[b][n] (block 0 multiplied, then FMAs in block order).
+  {
+    const int et = warp, n = rb * 32 + lane;
+    if (et < NT && et < p.T && n < p.N) {
+      float corr = 0.f;
+      if (p.a_offset != nullptr) {
+        for (int b = 0; b < p.G; ++b) {
+          const float rv = __ldg(p.rowsum + static_cast<int64_t>(b) * p.N + n);
+          const float o = __ldg(p.a_offset + static_cast<int64_t>(et) * p.G + b);
+          corr = b == 0 ? o * rv : fmaf(o, rv, corr);
+        }
+      }
+      ec[(2 * NT + et) * 32 + lane] = __ldg(p.a_scale + et);
+      ec[(3 * NT + et) * 32 + lane] = corr;
+    }
+  }
+  __syncwarp();
 
   int acc[NT];
 #pragma unroll
@@ -536,26 +569,16 @@ __global__ void __launch_bounds__(kGemvWarps * 32, 3) w4a4_gemv_kernel(const Gem
   __syncthreads();
 
   // Epilogue: thread (t, lane) for row n = 32 rb + lane, as the decode kernel's:
-  // corr = sum_b o[t][b] R[b][n] (block 0 multiplied, then FMAs in block order),
   // a = acc' - 8 Rt[n] (exact), y = s_w * fma(s_a, a, corr).
-  const int t = threadIdx.x >> 5;
-  const int n = rb * 32 + lane;
-  if (t < NT && t < p.T && n < p.N) {
+  const int et = warp, n = rb * 32 + lane;
+  if (et < NT && et < p.T && n < p.N) {
     int accp = 0;
 #pragma unroll
-    for (int w = 0; w < kGemvWarps; ++w) accp += red[(w * NT + t) * 32 + lane];
-    float rt = 0.f, corr = 0.f;
-    for (int b = 0; b < p.G; ++b) {
-      const float rv = __ldg(p.rowsum + static_cast<int64_t>(b) * p.N + n);
-      rt += rv;
-      if (p.a_offset != nullptr) {
-        const float o = __ldg(p.a_offset + static_cast<int64_t>(t) * p.G + b);
-        corr = b == 0 ? o * rv : fmaf(o, rv, corr);
-      }
-    }
+    for (int w = 0; w < kGemvWarps; ++w) accp += red[(w * NT + et) * 32 + lane];
+    const float rt = ec[(1 * NT + et) * 32 + lane];
     const float a = static_cast<float>(accp - 8 * static_cast<int>(rt));
-    const float y = __ldg(p.w_scale + n) * fmaf(__ldg(p.a_scale + t), a, corr);
-    const int64_t off = static_cast<int64_t>(t) * p.ldo + n;
+    const float y = ec[(0 * NT + et) * 32 + lane] * fmaf(ec[(2 * NT + et) * 32 + lane], a, ec[(3 * NT + et) * 32 + lane]);
+    const int64_t off = static_cast<int64_t>(et) * p.ldo + n;
     if (OUT == OFFQ_F32) {
       static_cast<float*>(p.out)[off] = y;
     } else if (OUT == OFFQ_BF16) {
@@ -563,14 +586,16 @@ __global__ void __launch_bounds__(kGemvWarps * 32, 3) w4a4_gemv_kernel(const Gem
     } else {
       static_cast<__half*>(p.out)[off] = __float2half_rn(y);
     }
-    if (p.acc_debug != nullptr) p.acc_debug[static_cast<int64_t>(t) * p.N + n] = accp;
+    if (p.acc_debug != nullptr) p.acc_debug[static_cast<int64_t>(et) * p.N + n] = accp;
   }
 }
 
 template <int OUT, int NT>
 int launch_gemv(const GemvParams& p, int blocks, cudaStream_t s) {
-  const size_t bytes = static_cast<size_t>(NT) * p.kchunks * 32 + static_cast<size_t>(kGemvWarps) * NT * 32 * 4;
-  if (bytes > 48 * 1024 && !smem_optin<w4a4_gemv_kernel<OUT, NT>>(kGemvMaxActBytes + kGemvWarps * kGemvMaxT * 32 * 4))
+  const size_t bytes =
+      static_cast<size_t>(NT) * p.kchunks * 32 + static_cast<size_t>(kGemvWarps + 4) * NT * 32 * 4;
+  if (bytes > 48 * 1024 &&
+      !smem_optin<w4a4_gemv_kernel<OUT, NT>>(kGemvMaxActBytes + (kGemvWarps + 4) * kGemvMaxT * 32 * 4))
     return OFFQ_ERR_CUDA;
   return launch_pdl(w4a4_gemv_kernel<OUT, NT>, dim3(blocks), dim3(kGemvWarps * 32), bytes, s, p);
 }
