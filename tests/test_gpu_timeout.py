@@ -64,3 +64,28 @@ def test_wait_budget_argument_checks():
     lib = Q.load_library()
     assert lib.offq_set_wait_cycles(-1) == Q.OFFQ_ERR_INVALID_ARG
     assert lib.offq_set_wait_cycles(0) == Q.OFFQ_OK
+
+
+def test_shortened_wait_times_out_in_the_mx_quantizer():
+    """The persistent MXFP4 quantizer (warp per 1024 channels) under the same test budget."""
+    T, K, g = 4096, 2048, 1024
+    x = torch.from_numpy(W.activations(T, K, seed=77, n_out=3, mult=80.0)).to(torch.bfloat16)
+    xd = x.cuda()
+    assert Q.offq_get_device_status() == Q.OFFQ_OK
+    Q.offq_set_wait_cycles(1)
+    try:
+        codes, shifts, scale, off = Q.quantize_act_mx(xd, g, rotate=True, offset=True)
+        torch.cuda.synchronize()
+    finally:
+        Q.offq_set_wait_cycles(0)
+    assert Q.offq_get_device_status() == Q.OFFQ_ERR_TIMEOUT
+    assert Q.offq_get_device_status() == Q.OFFQ_OK
+    codes, shifts, scale, off = Q.quantize_act_mx(xd, g, rotate=True, offset=True)
+    torch.cuda.synchronize()
+    assert Q.offq_get_device_status() == Q.OFFQ_OK
+    rows = np.unique(np.concatenate([W.unit_index_sample(T, 32, seed=4), [0, T - 1]]))
+    ref = O.quantize_act_mx(x.to(torch.float64).numpy()[rows], g, rotate=True, offset=True)
+    np.testing.assert_allclose(off.cpu().numpy()[rows], ref["offset"], rtol=1e-6)
+    xlo = np.round(np.log2(scale.cpu().numpy()[rows].astype(np.float64)))
+    assert np.all(np.abs(xlo - (ref["xmax"] - O.MX_SPAN)) <= 1)
+
