@@ -804,12 +804,6 @@ __device__ __forceinline__ float4 lds_f32x4(uint32_t addr) {
   return r;
 }
 
-// Transpose swizzle (float index within a warp's 1024): the 16-byte chunk index
-// (bits 2-4) takes bits 5-7 as well. Pass-1 stores (fixed j, 32 lanes) stay
-// within one 128-byte row; the pass-2 float4 loads of a quarter-warp hit eight
-// distinct chunks.
-__device__ __forceinline__ int swz1k(int e) { return e ^ (((e >> 5) & 7) << 2); }
-
 // Butterflies of register bit M of quantize_rows_1k_kernel, whose 32 values sit
 // in 16 float2 pairs (register 2i in .x, 2i + 1 in .y): bit 0 within each pair,
 // bit M >= 1 between pairs i and i + 2^(M-1), two lanes per packed add.
@@ -894,9 +888,12 @@ __global__ void __launch_bounds__(k1kMaxWarps * 32, 1) quantize_rows_1k_kernel(c
       v[0].x = 0.f;
     }
     fwht1k_pass(v);  // channel bits 5..9
-    // Transpose through the warp's scratch: channel e at byte 4 swz1k(e). Register j of
-    // lane l (e = l + 32 j) lands at 128 j + (4 l ^ 16 (j & 7)): eight lane bases, the
-    // rest immediate offsets. Lane l then reads its row's float4 k at 128 l + (16 k ^ 16 (l & 7)).
+    // Transpose through the warp's scratch: channel e at float e ^ (((e >> 5) & 7) << 2)
+    // (the 16-byte chunk index takes bits 5-7 as well, so the stores of one register
+    // hit 32 banks and the float4 loads of a quarter-warp 8 distinct chunks). Register j
+    // of lane l (e = l + 32 j) lands at byte 128 j + (4 l ^ 16 (j & 7)): eight lane bases,
+    // the rest immediate offsets. Lane l then reads its row's float4 k at
+    // 128 l + (16 k ^ 16 (l & 7)).
     {
       uint32_t wb[8];
 #pragma unroll
