@@ -181,6 +181,31 @@ def test_accumulator_exact_at_largest_k():
     np.testing.assert_array_equal(y, O.int_gemm(qa, qw).astype(np.float64))
 
 
+@pytest.mark.parametrize("T", [1, 8, 96])
+def test_accumulator_exact_at_maximum_k(T):
+    """K = 65536, the largest the ABI takes, with every code at +-7, through each form of the
+    linear (CUDA-core at 1 token, the decode kernel at 8, the pair kernel at 96): the largest
+    sum, 15 * 7 * 65536 < 2^24, stays exact."""
+    N, K, g = 256, 65536, 8192
+    qa = np.full((T, K), 7, dtype=np.int64)
+    qa[1::2] = -7
+    qa[:, ::5] = 3
+    qw = np.full((N, K), 7, dtype=np.int64)
+    qw[::3] = -7
+    qw[:, ::7] = 0
+    dev = lambda arr, dt: torch.from_numpy(np.ascontiguousarray(arr)).to(dt).cuda()
+    sa = np.full(T, 0.5, dtype=np.float32)
+    sw = np.full(N, 0.25, dtype=np.float32)
+    R = qw.reshape(N, K // g, g).sum(axis=2).T.astype(np.float32)
+    y, acc = _run_gemm(dev(O.tile_codes(O.pack_act_codes(qa)).reshape(-1, K // 2), torch.uint8),
+                       dev(sa, torch.float32), None,
+                       dev(O.tile_codes(O.pack_weight_codes(qw)).reshape(-1, K // 2), torch.uint8), dev(sw, torch.float32),
+                       dev(R, torch.float32),
+                       g, "f32")
+    np.testing.assert_array_equal(acc, O.int_gemm(qa + 8, qw))
+    np.testing.assert_array_equal(y, 0.125 * O.int_gemm(qa, qw).astype(np.float64))
+
+
 def test_full_llama2_7b_gate_sampled():
     """Full 2048 x 4096 -> 11008 launch, checked on 128 sampled token rows."""
     rows = W.unit_index_sample(2048, 128, seed=4)

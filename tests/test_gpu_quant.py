@@ -157,6 +157,17 @@ def test_quantize_warp_per_block_kernel(T, K, dt, ld_pad, offset):
     _quant_and_check(_host(x, dt), 1024, True, offset, rows=rows, ldx=(K + ld_pad) if ld_pad else None)
 
 
+@pytest.mark.parametrize("T,K,g,rotate", [
+    (300, 32768, 1024, True),    # the largest K, 32 blocks of 1024: past the warp-per-block kernel's 28
+    (40, 32768, 32768 // 4, False),  # the largest K without rotation, 4 offset blocks
+    (33, 32768, 32768 // 4, True),   # the largest K with the widest rotation block (8192)
+])
+def test_quantize_maximum_k(T, K, g, rotate):
+    x = W.activations(T, K, seed=83 + T, n_out=4, mult=100.0)
+    rows = np.unique(np.concatenate([W.unit_index_sample(T, 48, seed=14), [0, T - 1]]))
+    _quant_and_check(_host(x, "bf16"), g, rotate, True, rows=rows)
+
+
 def test_quantize_toy_fp32():
     w = W.WORKLOADS["toy"]
     x = W.layer_inputs(w, w.layers[0])
