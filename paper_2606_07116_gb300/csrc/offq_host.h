@@ -6,6 +6,7 @@
 #include <mutex>
 #include <utility>
 #include <cuda_runtime.h>
+#include <cudaTypedefs.h>
 
 #include "offq.h"
 
@@ -86,6 +87,29 @@ int quantize_mx_rows_fast(const void* x, int dtype, int64_t rows, int64_t K, int
 int w4a4_linear_decode(const uint8_t* a_codes, const float* a_scale, const float* a_offset, int64_t T, int64_t N,
                        int64_t K, int32_t g, const uint8_t* w_codes, const float* w_scale, const float* w_offsum,
                        void* out, int out_dtype, int64_t ldo, int32_t* acc_debug, cudaStream_t stream);
+
+// Rows of the g = 1024 rotating quantizer on the tensor cores (bf16 input, one
+// head; csrc/quant_mma.cu). Returns 1 when the shape, alignment or row count
+// does not suit it, else the launch status.
+struct MmaQuantRows {
+  const void* x;       // bf16 [rows][ld_t]
+  int64_t ld_t;
+  int64_t rows;
+  int K;
+  int flags;           // OFFQ_OFFSET (OFFQ_ROTATE implied)
+  uint8_t* codes;
+  float* scale;
+  float* offset;       // [rows][K / 1024] or nullptr
+  int tiled;
+  float inv_sqrt_g;
+  float scale_mul;
+  int* status;
+  long long wait_cycles;
+};
+int quantize_rows_mma(const MmaQuantRows& p, cudaStream_t s);
+
+// cuTensorMapEncodeTiled from the driver (nullptr if unavailable; csrc/kv_rot.cu).
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder();
 
 // Largest input dimension the row quantizer stages in shared memory.
 constexpr int64_t kMaxQuantK = 32768;

@@ -1850,6 +1850,26 @@ int dispatch_g(const QuantArgs& a, int g, cudaStream_t s) {
     case 256: return launch_narrow<8, Tin>(a, s);
     case 512: return launch_narrow<9, Tin>(a, s);
     case 1024: {
+      if constexpr (std::is_same<Tin, __nv_bfloat16>::value) {
+        if (a.H == 1 && (a.flags & OFFQ_ROTATE) != 0) {
+          MmaQuantRows p{};
+          p.x = a.x;
+          p.ld_t = a.ld_t;
+          p.rows = a.rows;
+          p.K = a.K;
+          p.flags = a.flags;
+          p.codes = a.codes;
+          p.scale = a.scale;
+          p.offset = a.offset;
+          p.tiled = a.tiled;
+          p.inv_sqrt_g = a.inv_sqrt_g;
+          p.scale_mul = a.scale_mul;
+          p.status = a.status;
+          p.wait_cycles = a.wait_cycles;
+          const int st = quantize_rows_mma(p, s);
+          if (st != 1) return st;
+        }
+      }
       const int st = launch_1k<Tin>(a, s);
       return st == kNoRing ? launch_narrow<10, Tin>(a, s) : st;
     }

@@ -10,6 +10,11 @@ u = 2^-24), never from observed differences:
 * Scales and offsets. The kernel's transform is a radix-2 tree of L = log2(g)
   fp32 additions per output, so each rotated value carries an absolute error of
   at most L u sum|x| over its block; the scale inherits that relative to max|r|.
+  The tensor-core form of g = 1024 (bf16 rows) sums the first 32 terms of each
+  output in the MMA's fp32 accumulator: its products are exact, and allowing
+  each of the 32 additions a full ulp (truncation), plus the removal of x[0]
+  and the 5 register stages, the bound is TC_FACTOR u sum|x| over the block.
+  There a code may also differ within that bound (in code units) of a tie.
   Without the rotation the offset is an fp32 block sum whose summation depth
   is at most g/8 + 16.
 * GEMM outputs. Integer accumulators are exact, and so is the removal of the
@@ -26,12 +31,15 @@ import math
 import numpy as np
 
 U32 = 2.0 ** -24
+TC_FACTOR = 2 * 32 + 8 + 1 + 5 + 4
 TIE_WINDOW = 1e-3
 MAX_MISMATCH_FRACTION = 1e-4
 
 
-def check_codes(q_gpu: np.ndarray, q_ref: np.ndarray, r_ref: np.ndarray, s_ref: np.ndarray, what: str = "codes"):
-    """q_* int codes [rows, K]; r_ref residual [rows, K]; s_ref scale [rows] (oracle, float64)."""
+def check_codes(q_gpu: np.ndarray, q_ref: np.ndarray, r_ref: np.ndarray, s_ref: np.ndarray, what: str = "codes",
+                window=None):
+    """q_* int codes [rows, K]; r_ref residual [rows, K]; s_ref scale [rows] (oracle, float64).
+    window: per-row tie window in code units (at least TIE_WINDOW) where the kernel's bound is wider."""
     q_gpu = np.asarray(q_gpu, dtype=np.int64)
     q_ref = np.asarray(q_ref, dtype=np.int64)
     assert q_gpu.shape == q_ref.shape, (q_gpu.shape, q_ref.shape)
@@ -46,26 +54,53 @@ def check_codes(q_gpu: np.ndarray, q_ref: np.ndarray, r_ref: np.ndarray, s_ref: 
         z = np.where(s > 0, np.asarray(r_ref, np.float64) / s, 0.0)
     zm = np.abs(z[mism])
     dist = np.abs(zm - np.floor(zm) - 0.5)
-    assert np.all(dist < TIE_WINDOW), f"{what}: mismatch away from a rounding tie (min dist {dist.max():.3g})"
+    win = TIE_WINDOW
+    if window is not None:
+        w = np.broadcast_to(np.asarray(window, np.float64).reshape(-1, *([1] * (q_ref.ndim - 1))), q_ref.shape)
+        win = np.maximum(TIE_WINDOW, w[mism])
+    assert np.all(dist < win), f"{what}: mismatch away from a rounding tie (min dist {dist.max():.3g})"
     frac = n / q_ref.size
     assert frac <= MAX_MISMATCH_FRACTION, f"{what}: {n} codes differ ({frac:.2e} > {MAX_MISMATCH_FRACTION})"
     return n
 
 
-def rotation_abs_error(x: np.ndarray, g: int, rotate: bool) -> np.ndarray:
-    """Per-row bound on the absolute fp32 error of an unnormalised rotated value."""
+def rotation_abs_error(x: np.ndarray, g: int, rotate: bool, tc: bool = False) -> np.ndarray:
+    """Per-row bound on the absolute fp32 error of an unnormalised rotated value
+    (tc: the tensor-core form of g = 1024)."""
     x = np.abs(np.asarray(x, np.float64))
     T, K = x.shape
     blk = x.reshape(T, K // g, g).sum(axis=2).max(axis=1)
     L = int(math.log2(g)) if rotate else 0
-    return (L + 2) * U32 * blk
+    return (TC_FACTOR if tc else L + 2) * U32 * blk
 
 
-def check_scales(s_gpu, s_ref, x, g, rotate, what="scale"):
+def code_window(s_ref, x, g, tc: bool = False):
+    """Per-row tie window in code units: r / s moves by at most the residual's bound
+    over s plus the scale's relative error times 7."""
+    s_ref = np.asarray(s_ref, np.float64)
+    err = rotation_abs_error(x, g, True, tc) / math.sqrt(g)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        return np.where(s_ref > 0, 2.0 * err / s_ref, 0.0) + 1e-6
+
+
+def tensor_core_form(x, g: int, rotate: bool, ldx=None) -> bool:
+    """Whether offq_quantize_act takes the tensor-core form of g = 1024 for the torch
+    tensor x: bf16 rows of 1024 G channels (G <= 64) with the rotation, a row pitch of a
+    multiple of 8 elements, and at least as many tiles of 64 // G rows as SMs."""
+    import torch
+    T, K = x.shape
+    ld = K if ldx is None else ldx
+    if x.dtype != torch.bfloat16 or g != 1024 or not rotate or K % 1024 or K // 1024 > 64 or ld % 8:
+        return False
+    P = 64 // (K // 1024)
+    return -(-T // P) >= torch.cuda.get_device_properties(0).multi_processor_count
+
+
+def check_scales(s_gpu, s_ref, x, g, rotate, what="scale", tc=False):
     s_gpu = np.asarray(s_gpu, np.float64)
     s_ref = np.asarray(s_ref, np.float64)
     norm = math.sqrt(g) if rotate else 1.0
-    err_u = rotation_abs_error(x, g, rotate)          # on the unnormalised residual
+    err_u = rotation_abs_error(x, g, rotate, tc)      # on the unnormalised residual
     tol = err_u / (7.0 * norm) + 4 * U32 * np.abs(s_ref)
     bad = np.abs(s_gpu - s_ref) > tol
     assert not np.any(bad), f"{what}: {bad.sum()} rows out of tolerance; worst " \

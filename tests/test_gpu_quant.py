@@ -11,7 +11,7 @@ import oracle as O
 import workloads as W
 from paper_2606_07116_gb300 import build as B
 from paper_2606_07116_gb300 import offq as Q
-from parity import act_q, check_codes, check_offsets, check_scales, weight_q
+from parity import act_q, check_codes, check_offsets, check_scales, code_window, tensor_core_form, weight_q
 
 pytestmark = pytest.mark.gpu
 
@@ -31,6 +31,7 @@ def _host(x32: np.ndarray, dt: str) -> torch.Tensor:
 
 def _quant_and_check(x_host: torch.Tensor, g: int, rotate: bool, offset: bool, rows=None, ldx=None):
     T, K = x_host.shape
+    tc = tensor_core_form(x_host, g, rotate, ldx)
     if ldx is None:
         xd = x_host.cuda()
     else:
@@ -44,8 +45,9 @@ def _quant_and_check(x_host: torch.Tensor, g: int, rotate: bool, offset: bool, r
     sel = np.arange(T) if rows is None else rows
     ref = O.quantize_act(x64[sel], g, rotate=rotate, offset=offset)
     q_gpu = act_q(codes, T, K)[sel]
-    nmis = check_codes(q_gpu, ref["q"], ref["residual"], ref["scale"])
-    check_scales(scale.cpu().numpy()[sel], ref["scale"], x64[sel], g, rotate)
+    window = code_window(ref["scale"], x64[sel], g, tc) if tc else None
+    nmis = check_codes(q_gpu, ref["q"], ref["residual"], ref["scale"], window=window)
+    check_scales(scale.cpu().numpy()[sel], ref["scale"], x64[sel], g, rotate, tc=tc)
     o = off.cpu().numpy()[sel]
     if offset:
         check_offsets(o, ref["offset"], x64[sel], g, rotate)
@@ -184,6 +186,61 @@ def test_quantize_full_llama2_7b_sampled():
 def test_quantize_strided_rows():
     x = W.activations(21, 1024, seed=12, n_out=1, mult=20.0)
     _quant_and_check(_host(x, "bf16"), 1024, True, True, ldx=1024 + 64)
+
+
+@pytest.mark.parametrize("G,extra,offset,ld_pad", [
+    (1, 37, True, 0),      # 64 tokens of one block per tile, a ragged last tile
+    (2, 5, True, 64),      # padded rows
+    (3, 0, True, 0),       # 21 tokens x 3 blocks: 63 of a half's 64 rows
+    (5, 11, False, 0),     # no offsets
+    (14, 3, True, 0),      # Llama-3-8B down-proj width
+    (28, 1, False, 8),     # Llama-2-70B down-proj width, pitch K + 8
+    (32, 1, True, 0),      # the largest K (32768): 2 tokens per tile
+])
+def test_quantize_tensor_core_form(G, extra, offset, ld_pad):
+    """The tensor-core form of g = 1024 (bf16 rows, at least one tile per SM) across block
+    counts per row, tile fill, ragged last tiles, padded rows and the offset flag; sampled
+    rows plus every row of the first and the last tile."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    P = 64 // G
+    T, K = sms * P + extra, 1024 * G
+    x = _host(W.activations(T, K, seed=90 + G, n_out=4, mult=100.0), "bf16")
+    ldx = K + ld_pad if ld_pad else None
+    assert tensor_core_form(x, 1024, True, ldx)
+    last0 = (T - 1) // P * P
+    rows = np.unique(np.concatenate([W.unit_index_sample(T, 96, seed=G), np.arange(P), np.arange(last0, T)]))
+    _quant_and_check(x, 1024, True, offset, rows=rows, ldx=ldx)
+
+
+def test_quantize_tensor_core_form_degenerate_rows():
+    """Zero rows, rows whose only nonzero channels lead their blocks (zero residual), a unit
+    channel, a constant row and one large value, inside a launch that takes the tensor cores."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    G = 4
+    T, K = sms * 16, 4096
+    x = W.activations(T, K, seed=17, n_out=2, mult=40.0).astype(np.float32)
+    x[0] = 0.0
+    x[1] = 0.0
+    x[1, ::1024] = [3.0, -250.0, 0.5, 8192.0]
+    x[2] = 0.0
+    x[2, 1024 + 77] = 1.0
+    x[3] = 2.5
+    x[T - 1, 4000] = 3e4
+    xh = _host(x, "bf16")
+    assert tensor_core_form(xh, 1024, True)
+    codes, scale, off = Q.quantize_act(xh.cuda(), 1024)
+    torch.cuda.synchronize()
+    q = act_q(codes, T, K)
+    assert np.all(q[0] == 0) and scale[0].item() == 0.0 and np.all(off[0].cpu().numpy() == 0.0)
+    assert np.all(q[1] == 0) and scale[1].item() == 0.0
+    np.testing.assert_array_equal(off[1].cpu().numpy(), np.array([3.0, -250.0, 0.5, 8192.0]) / 32.0)
+    H = O.sylvester_hadamard(1024)
+    np.testing.assert_array_equal(q[2, 1024:2048], 7 * H[77])
+    assert np.all(q[2, :1024] == 0) and np.all(q[2, 2048:] == 0)
+    # A constant block c rotates to (32 c, 0, ..., 0): residual 32 c - c / 32 at channel 0.
+    assert np.all(q[3, ::1024] == 7) and np.count_nonzero(q[3]) == 4
+    rows = np.unique(np.concatenate([np.arange(8), W.unit_index_sample(T, 32, seed=5), [T - 1]]))
+    _quant_and_check(xh, 1024, True, True, rows=rows)
 
 
 def test_quantize_degenerate_rows():

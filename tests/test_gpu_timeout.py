@@ -16,7 +16,7 @@ import oracle as O
 import workloads as W
 from paper_2606_07116_gb300 import build as B
 from paper_2606_07116_gb300 import offq as Q
-from parity import act_q, check_codes, check_scales
+from parity import act_q, check_codes, check_scales, code_window, tensor_core_form
 
 pytestmark = pytest.mark.gpu
 
@@ -32,6 +32,7 @@ def _lib():
     (8192, 2048, 512, True),     # the ring form of the block-Hadamard kernel (g <= 1024)
     (2048, 8192, 4096, True),    # the ring form of the wide kernel (g >= 2048)
     (8192, 4096, 4096, False),   # the shared-memory ring kernel of rotation-free rows (per-warp rings)
+    (2048, 14336, 1024, True),   # the tensor-core form of g = 1024 (its register warps' wait for the MMAs)
 ])
 def test_shortened_wait_times_out_and_the_device_recovers(T, K, g, rotate):
     x = torch.from_numpy(W.activations(T, K, seed=T + K, n_out=3, mult=80.0)).to(torch.bfloat16)
@@ -56,8 +57,10 @@ def test_shortened_wait_times_out_and_the_device_recovers(T, K, g, rotate):
     rows = np.unique(np.concatenate([W.unit_index_sample(T, 64, seed=3), [0, T - 1]]))
     x64 = x.to(torch.float64).numpy()[rows]
     ref = O.quantize_act(x64, g, rotate=rotate, offset=True)
-    check_codes(act_q(codes, T, K)[rows], ref["q"], ref["residual"], ref["scale"])
-    check_scales(scale.cpu().numpy()[rows], ref["scale"], x64, g, rotate)
+    tc = tensor_core_form(x, g, rotate)
+    window = code_window(ref["scale"], x64, g, tc) if tc else None
+    check_codes(act_q(codes, T, K)[rows], ref["q"], ref["residual"], ref["scale"], window=window)
+    check_scales(scale.cpu().numpy()[rows], ref["scale"], x64, g, rotate, tc=tc)
 
 
 def test_wait_budget_argument_checks():
