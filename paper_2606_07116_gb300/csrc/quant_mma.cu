@@ -169,6 +169,81 @@ __device__ __forceinline__ void tmem_ld_groups(uint32_t col0, uint32_t (&r)[64])
       : "memory");
 }
 
+// tmem_ld_groups with the warp pair's barrier between the loads and their
+// wait: the barrier's wait overlaps the loads' latency.
+__device__ __forceinline__ void tmem_ld_groups_pair_sync(uint32_t col0, int pair_bar, uint32_t (&r)[64]) {
+  asm volatile(
+      "{\n"
+      ".reg .b32 ta;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%64];\n"
+      "add.u32 ta, %64, 32;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%4,%5,%6,%7}, [ta];\n"
+      "add.u32 ta, %64, 64;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%8,%9,%10,%11}, [ta];\n"
+      "add.u32 ta, %64, 96;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%12,%13,%14,%15}, [ta];\n"
+      "add.u32 ta, %64, 128;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%16,%17,%18,%19}, [ta];\n"
+      "add.u32 ta, %64, 160;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%20,%21,%22,%23}, [ta];\n"
+      "add.u32 ta, %64, 192;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%24,%25,%26,%27}, [ta];\n"
+      "add.u32 ta, %64, 224;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%28,%29,%30,%31}, [ta];\n"
+      "add.u32 ta, %64, 256;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%32,%33,%34,%35}, [ta];\n"
+      "add.u32 ta, %64, 288;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%36,%37,%38,%39}, [ta];\n"
+      "add.u32 ta, %64, 320;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%40,%41,%42,%43}, [ta];\n"
+      "add.u32 ta, %64, 352;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%44,%45,%46,%47}, [ta];\n"
+      "add.u32 ta, %64, 384;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%48,%49,%50,%51}, [ta];\n"
+      "add.u32 ta, %64, 416;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%52,%53,%54,%55}, [ta];\n"
+      "add.u32 ta, %64, 448;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%56,%57,%58,%59}, [ta];\n"
+      "add.u32 ta, %64, 480;\n"
+      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%60,%61,%62,%63}, [ta];\n"
+      "bar.sync %65, 64;\n"
+      "tcgen05.wait::ld.sync.aligned;\n"
+      "}\n"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]),
+        "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]),
+        "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]),
+        "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]),
+        "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+      : "r"(col0), "r"(pair_bar)
+      : "memory");
+}
+
+// Columns col0 .. col0 + 31 and col1 .. col1 + 31 of the thread's TMEM lane,
+// waited in the same statement.
+__device__ __forceinline__ void tmem_ld_2x32_waited(uint32_t col0, uint32_t col1, uint32_t (&r)[64]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%64];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,"
+      "%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%65];\n"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]),
+        "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]),
+        "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]),
+        "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]),
+        "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+      : "r"(col0), "r"(col1)
+      : "memory");
+}
+
 // Four consecutive columns of the thread's TMEM lane from two fp32 pairs.
 __device__ __forceinline__ void tmem_st4(uint32_t taddr, uint64_t lo, uint64_t hi) {
   asm volatile(
@@ -243,59 +318,69 @@ __device__ __forceinline__ uint32_t pack8(const uint32_t* u) {
   return __byte_perm(__byte_perm(b0, b1, 0x0040), __byte_perm(b2, b3, 0x0040), 0x5410);
 }
 
-// One first-sweep pass of a thread of half H: output channels a' = a0 .. a0 + 3
-// of the 16 groups of its TMEM lane (columns col + 32 b), the H_16 stages, the
-// H_2 stage with the partner thread (through xw / xr), and the results back in
-// place: the thread keeps groups 8 H .. 8 H + 7, output bit h = e of group
-// 8 H + k lands in column slot 8 (e ^ H) + k.
+// The first sweep of a thread of half H, in 4 passes of 4 output channels a'
+// (columns col + 4 c + 32 b of its TMEM lane for the 16 groups b): per pass
+// the H_16 stages, the H_2 stage with the partner thread (through xw / xr, two
+// buffers alternating), and the results back in place: the thread keeps
+// groups 8 H .. 8 H + 7, output bit h = e of group 8 H + k lands in column slot
+// 8 (e ^ H) + k. The next pass's TMEM loads are issued before the pair barrier.
 template <int H>
-__device__ __forceinline__ void first_pass(uint32_t col, uint32_t xw, uint32_t xr, int pair_bar, uint64_t x0x0,
-                                           Extremes& ex) {
+__device__ __forceinline__ void first_sweep(uint32_t col, uint32_t xw, uint32_t xr, int pair_bar, uint64_t x0x0,
+                                            Extremes& ex) {
   uint32_t r[64];
   tmem_ld_groups(col, r);
-  uint64_t p[16][2];
-#pragma unroll
-  for (int b = 0; b < 16; ++b) {
-    p[b][0] = pack2(__uint_as_float(r[4 * b]), __uint_as_float(r[4 * b + 1]));
-    p[b][1] = pack2(__uint_as_float(r[4 * b + 2]), __uint_as_float(r[4 * b + 3]));
-  }
-  if (H == 0) {
-    // Group 0 of the first half holds the block's leading channel: every
-    // output of its H_32 includes x[0] once. Removing it is removing the offset
-    // (x0x0 is zero without OFFQ_OFFSET).
-    p[0][0] = sub2(p[0][0], x0x0);
-    p[0][1] = sub2(p[0][1], x0x0);
-  }
-#pragma unroll
-  for (int d = 1; d < 16; d <<= 1) {
+#pragma unroll 1
+  for (int c = 0; c < 4; ++c) {
+    const uint32_t buf = (c & 1) * kXBufBytes;
+    uint64_t p[16][2];
 #pragma unroll
     for (int b = 0; b < 16; ++b) {
-      if ((b & d) == 0) {
+      p[b][0] = pack2(__uint_as_float(r[4 * b]), __uint_as_float(r[4 * b + 1]));
+      p[b][1] = pack2(__uint_as_float(r[4 * b + 2]), __uint_as_float(r[4 * b + 3]));
+    }
+    if (H == 0) {
+      // Group 0 of the first half holds the block's leading channel: every
+      // output of its H_32 includes x[0] once. Removing it is removing the
+      // offset (x0x0 is zero without OFFQ_OFFSET).
+      p[0][0] = sub2(p[0][0], x0x0);
+      p[0][1] = sub2(p[0][1], x0x0);
+    }
 #pragma unroll
-        for (int k = 0; k < 2; ++k) {
-          const uint64_t u = p[b][k], v = p[b + d][k];
-          p[b][k] = add2(u, v);
-          p[b + d][k] = sub2(u, v);
+    for (int d = 1; d < 16; d <<= 1) {
+#pragma unroll
+      for (int b = 0; b < 16; ++b) {
+        if ((b & d) == 0) {
+#pragma unroll
+          for (int k = 0; k < 2; ++k) {
+            const uint64_t u = p[b][k], v = p[b + d][k];
+            p[b][k] = add2(u, v);
+            p[b + d][k] = sub2(u, v);
+          }
         }
       }
     }
-  }
 #pragma unroll
-  for (int k = 0; k < 8; ++k) sts_pair(xw + k * 512, p[8 * (1 - H) + k][0], p[8 * (1 - H) + k][1]);
-  bar_sync(pair_bar, 64);
+    for (int k = 0; k < 8; ++k) sts_pair(xw + buf + k * 512, p[8 * (1 - H) + k][0], p[8 * (1 - H) + k][1]);
+    if (c < 3) {
+      tmem_ld_groups_pair_sync(col + 4 * (c + 1), pair_bar, r);
+    } else {
+      bar_sync(pair_bar, 64);
+    }
+    const uint32_t cc = col + 4 * c;
 #pragma unroll
-  for (int k = 0; k < 8; ++k) {
-    uint64_t t0, t1;
-    lds_pair(xr + k * 512, t0, t1);
-    const uint64_t u0 = p[8 * H + k][0], u1 = p[8 * H + k][1];
-    // Output bit 0 is (half 0) + (half 1), bit 1 is (half 0) - (half 1).
-    const uint64_t s0 = add2(u0, t0), s1 = add2(u1, t1);
-    const uint64_t d0 = H == 0 ? sub2(u0, t0) : sub2(t0, u0);
-    const uint64_t d1 = H == 0 ? sub2(u1, t1) : sub2(t1, u1);
-    tmem_st4(col + 32 * (8 * H + k), s0, s1);
-    tmem_st4(col + 32 * (8 * (1 - H) + k), d0, d1);
-    ex.add(s0, s1);
-    ex.add(d0, d1);
+    for (int k = 0; k < 8; ++k) {
+      uint64_t t0, t1;
+      lds_pair(xr + buf + k * 512, t0, t1);
+      const uint64_t u0 = p[8 * H + k][0], u1 = p[8 * H + k][1];
+      // Output bit 0 is (half 0) + (half 1), bit 1 is (half 0) - (half 1).
+      const uint64_t s0 = add2(u0, t0), s1 = add2(u1, t1);
+      const uint64_t d0 = H == 0 ? sub2(u0, t0) : sub2(t0, u0);
+      const uint64_t d1 = H == 0 ? sub2(u1, t1) : sub2(t1, u1);
+      tmem_st4(cc + 32 * (8 * H + k), s0, s1);
+      tmem_st4(cc + 32 * (8 * (1 - H) + k), d0, d1);
+      ex.add(s0, s1);
+      ex.add(d0, d1);
+    }
   }
 }
 
@@ -447,13 +532,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t x0x0 = pack2(x0, x0);
       Extremes ex;
       const uint32_t col = tl + 16 * wg;  // output channels a' = 16 wg .. 16 wg + 15
-      uint32_t buf = 0;
       if (h == 0) {
-#pragma unroll 1
-        for (int c = 0; c < 4; ++c, buf ^= kXBufBytes) first_pass<0>(col + 4 * c, xw + buf, xr + buf, pair_bar, x0x0, ex);
+        first_sweep<0>(col, xw, xr, pair_bar, x0x0, ex);
       } else {
-#pragma unroll 1
-        for (int c = 0; c < 4; ++c, buf ^= kXBufBytes) first_pass<1>(col + 4 * c, xw + buf, xr + buf, pair_bar, x0x0, ex);
+        first_sweep<1>(col, xw, xr, pair_bar, x0x0, ex);
       }
       const float m = ex.absmax();
       tmem_st_wait();
@@ -476,24 +558,34 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int kt0 = 32 * j + 16 * (wg ^ h) + 8 * h;
       uint8_t* dst0 = a.codes + ((row >> 5) * cpr + kt0) * 512 + (row & 31) * 16;  // the 32-row tiled layout
 #pragma unroll 1
-      for (int k = 0; k < 8; ++k) {
-        uint32_t v[32];
-        tmem_ld_32cols_waited(tl + 32 * (8 * wg + k), v);
-        // Slot 8 wg + k is read in this lane quarter: the next tile's MMAs may
-        // overwrite it once the four quarters have.
+      for (int k = 0; k < 8; k += 2) {
+        uint32_t v[64];
+        const uint32_t q = 8 * wg + k;
+        tmem_ld_2x32_waited(tl + 32 * q, tl + 32 * (q + 1), v);
+        // Slots q and q + 1 are read in this lane quarter: the next tile's MMAs
+        // may overwrite them once the four quarters have.
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(tempty0 + 8 * (8 * wg + k));
-        uint32_t u[32];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          float f0, f1;
-          unpack2(fma2v(pack2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])), inv2, mag2), f0, f1);
-          u[2 * i] = __float_as_uint(f0);
-          u[2 * i + 1] = __float_as_uint(f1);
+        if (lane == 0) {
+          mbar_arrive(tempty0 + 8 * q);
+          mbar_arrive(tempty0 + 8 * (q + 1));
         }
-        if (ok)
-          *reinterpret_cast<uint4*>(dst0 + k * 512) = make_uint4(pack8(u), pack8(u + 8), pack8(u + 16), pack8(u + 24));
+#pragma unroll
+        for (int hk = 0; hk < 2; ++hk) {
+          uint32_t u[32];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            float f0, f1;
+            unpack2(fma2v(pack2(__uint_as_float(v[32 * hk + 2 * i]), __uint_as_float(v[32 * hk + 2 * i + 1])), inv2,
+                          mag2),
+                    f0, f1);
+            u[2 * i] = __float_as_uint(f0);
+            u[2 * i + 1] = __float_as_uint(f1);
+          }
+          if (ok)
+            *reinterpret_cast<uint4*>(dst0 + (k + hk) * 512) =
+                make_uint4(pack8(u), pack8(u + 8), pack8(u + 16), pack8(u + 24));
+        }
       }
       if (wg == 0 && h == 0 && ok) {
         if (a.offset != nullptr) a.offset[row * G + j] = x0 * a.inv_sqrt_g;
