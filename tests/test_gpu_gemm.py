@@ -129,13 +129,17 @@ def test_oracle_codes_through_gemm():
     # Few-token form (T <= 4, dp4a on the CUDA cores): every token count class (1, 2, 4 with
     # 3 padded), K = 1056 (33 chunks: the eighths of K are uneven and the last warp has none),
     # K = 11008 at 4 tokens (43 KB of unpacked activations, 43 offset blocks), and a K whose
-    # unpacked activations exceed its budget (4 x 32768 bytes: the tensor-core form).
+    # unpacked activations exceed its budget (4 x 32768 bytes: the tensor-core form). Then the
+    # decode kernel at its smallest token counts (5 to 8: 11 to 14 padded MMA columns).
     (1, 1024, 300, 256, "f32", None),
     (2, 4096, 1000, 4096, "f16", 1000),
     (3, 1056, 520, 32, "bf16", None),
     (4, 11008, 264, 256, "bf16", 272),
-    (5, 11008, 4096, 256, "f32", None),
     (4, 32768, 512, 1024, "bf16", None),
+    (5, 11008, 4096, 256, "f32", None),
+    (6, 1056, 700, 32, "f16", 704),
+    (7, 4096, 1000, 1024, "bf16", 1008),
+    (8, 11008, 520, 256, "f32", None),
 ])
 def test_layers(T, K, N, g, out_dt, ldo):
     _check_layer(T, K, N, g, out_dt, ldo=ldo, seed=T + K)
@@ -320,17 +324,18 @@ def test_outputs_near_zero_against_large_row_sums(K, g):
 
 
 def test_few_token_forms_agree():
-    """4 tokens take the CUDA-core form, 5 the tensor-core decode kernel: on the same 4 rows
+    """4 tokens take the CUDA-core form, 5 to 9 the tensor-core decode kernel: on the same rows
     both give the same integer accumulators and, with the same epilogue chain, the same
     output bits."""
-    T, K, N, g = 5, 4096, 11008, 4096
+    T, K, N, g = 9, 4096, 11008, 4096
     x = W.activations(T, K, seed=71, n_out=4, mult=100.0)
     w = W.weights(N, K, seed=72)
     a_codes, a_scale, a_off = Q.quantize_act(torch.from_numpy(x).to(torch.bfloat16).cuda(), g, rotate=False)
     w_codes, w_scale, rowsum = Q.prepare_weight(torch.from_numpy(w).cuda(), g, rotate=False)
     for dt in ("bf16", "f32"):
-        y5, acc5 = _run_gemm(a_codes, a_scale, a_off, w_codes, w_scale, rowsum, g, dt, T=5)
-        y4, acc4 = _run_gemm(a_codes, a_scale[:4], a_off[:4], w_codes, w_scale, rowsum, g, dt, T=4)
-        np.testing.assert_array_equal(acc4, acc5[:4])
-        np.testing.assert_array_equal(y4, y5[:4])
+        y9, acc9 = _run_gemm(a_codes, a_scale, a_off, w_codes, w_scale, rowsum, g, dt, T=9)
+        for t in (8, 5, 4):
+            yt, acct = _run_gemm(a_codes, a_scale[:t], a_off[:t], w_codes, w_scale, rowsum, g, dt, T=t)
+            np.testing.assert_array_equal(acct, acc9[:t])
+            np.testing.assert_array_equal(yt, y9[:t])
 
