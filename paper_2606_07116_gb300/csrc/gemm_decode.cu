@@ -418,9 +418,9 @@ int launch_decode(const DecodeParams& p, int grid, cudaStream_t s) {
 // the tensor cores costs more than the products: the weights stream from HBM
 // straight into registers and meet the activations in dp4a (four int8
 // products per instruction, exact int32 sums). (Measured on 4096 -> 11008:
-// 10.3 us at one token, 16.4 us at eight, where the tensor-core form takes
-// 14.9; the sign-magnitude unpacking and one dp4a per 4 codes and token make
-// the cost grow with T.) A CTA owns one 32-row weight block: lane l of each of
+// 8.3 us at one token; at eight tokens 14.85 us, level with the tensor-core
+// form's 14.9, so the tensor cores take T >= 5: the sign-magnitude unpacking
+// and one dp4a per 4 codes and token make the cost grow with T.) A CTA owns one 32-row weight block: lane l of each of
 // its 8 warps takes row l, warp w a contiguous eighth of the K chunks, 8
 // chunks (128 B of codes per lane) in flight;
 // the warps' partial sums meet in shared memory. The activation codes
