@@ -60,7 +60,8 @@ constexpr int kSlabs = 8;                            // 64-channel slabs of a ha
 constexpr int kHalfRows = 64;                        // (token, block) rows per half
 constexpr int kSlabBytes = 2 * kHalfRows * 128;      // both halves of one slab
 constexpr int kABytes = kSlabs * kSlabBytes;         // 128 KB
-constexpr int kBBytes = 32 * 128;                    // H_32, 128-byte swizzled rows
+constexpr int kBSlab = 128 * 128;                    // H_128, channels 64 k .. 64 k + 63 of its 128 rows
+constexpr int kBBytes = 2 * kBSlab;
 constexpr int kRegWarps = 8;                         // two per TMEM lane quarter
 constexpr int kXWarpBytes = 8 * 32 * 16;             // a warp's exchange area: 8 groups x 32 lanes x 16 B
 constexpr int kXBufBytes = kRegWarps * kXWarpBytes;
@@ -73,8 +74,8 @@ constexpr int kProducerWarp = kRegWarps, kMmaWarp = kRegWarps + 1;
 constexpr int kThreads = 32 * (kRegWarps + 2);
 static_assert(kSmem <= 232448, "one CTA per SM");
 // kind::f16: D f32 (bits 4-5 = 1), A and B bf16 (7-9, 10-12 = 1), both
-// K-major, N = 32 (N >> 3 at bit 17), M = 128 (M >> 4 at bit 24).
-constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((32u >> 3) << 17) | ((128u >> 4) << 24);
+// K-major, N = 128 (N >> 3 at bit 17), M = 128 (M >> 4 at bit 24).
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((128u >> 3) << 17) | ((128u >> 4) << 24);
 
 // Named barriers: 0 is __syncthreads; 1-4 the four warp pairs (w, w ^ 2) of
 // the register warps; 5 all register warps; 6 their per-tile vote.
@@ -117,44 +118,20 @@ __device__ __forceinline__ bool bar_any(int id, int count, bool pred) {
   return r != 0;
 }
 
-// Columns col0 + 32 b + (0..3) of the thread's TMEM lane into r[4 b .. 4 b + 3],
-// b = 0..15, with the wait in the same statement (no register is read before
-// its data has arrived).
-__device__ __forceinline__ void tmem_ld_groups(uint32_t col0, uint32_t (&r)[64]) {
+// Columns col0 + 128 c + (0..15) of the thread's TMEM lane into
+// r[16 c .. 16 c + 15], c = 0..3, with the wait in the same statement (no
+// register is read before its data has arrived).
+__device__ __forceinline__ void tmem_ld_chunks(uint32_t col0, uint32_t (&r)[64]) {
   asm volatile(
       "{\n"
       ".reg .b32 ta;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%64];\n"
-      "add.u32 ta, %64, 32;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%4,%5,%6,%7}, [ta];\n"
-      "add.u32 ta, %64, 64;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%8,%9,%10,%11}, [ta];\n"
-      "add.u32 ta, %64, 96;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%12,%13,%14,%15}, [ta];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%64];\n"
       "add.u32 ta, %64, 128;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%16,%17,%18,%19}, [ta];\n"
-      "add.u32 ta, %64, 160;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%20,%21,%22,%23}, [ta];\n"
-      "add.u32 ta, %64, 192;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%24,%25,%26,%27}, [ta];\n"
-      "add.u32 ta, %64, 224;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%28,%29,%30,%31}, [ta];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [ta];\n"
       "add.u32 ta, %64, 256;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%32,%33,%34,%35}, [ta];\n"
-      "add.u32 ta, %64, 288;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%36,%37,%38,%39}, [ta];\n"
-      "add.u32 ta, %64, 320;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%40,%41,%42,%43}, [ta];\n"
-      "add.u32 ta, %64, 352;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%44,%45,%46,%47}, [ta];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47}, [ta];\n"
       "add.u32 ta, %64, 384;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%48,%49,%50,%51}, [ta];\n"
-      "add.u32 ta, %64, 416;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%52,%53,%54,%55}, [ta];\n"
-      "add.u32 ta, %64, 448;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%56,%57,%58,%59}, [ta];\n"
-      "add.u32 ta, %64, 480;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%60,%61,%62,%63}, [ta];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [ta];\n"
       "tcgen05.wait::ld.sync.aligned;\n"
       "}\n"
       : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
@@ -169,43 +146,19 @@ __device__ __forceinline__ void tmem_ld_groups(uint32_t col0, uint32_t (&r)[64])
       : "memory");
 }
 
-// tmem_ld_groups with the warp pair's barrier between the loads and their
+// tmem_ld_chunks with the warp pair's barrier between the loads and their
 // wait: the barrier's wait overlaps the loads' latency.
-__device__ __forceinline__ void tmem_ld_groups_pair_sync(uint32_t col0, int pair_bar, uint32_t (&r)[64]) {
+__device__ __forceinline__ void tmem_ld_chunks_pair_sync(uint32_t col0, int pair_bar, uint32_t (&r)[64]) {
   asm volatile(
       "{\n"
       ".reg .b32 ta;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%64];\n"
-      "add.u32 ta, %64, 32;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%4,%5,%6,%7}, [ta];\n"
-      "add.u32 ta, %64, 64;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%8,%9,%10,%11}, [ta];\n"
-      "add.u32 ta, %64, 96;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%12,%13,%14,%15}, [ta];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%64];\n"
       "add.u32 ta, %64, 128;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%16,%17,%18,%19}, [ta];\n"
-      "add.u32 ta, %64, 160;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%20,%21,%22,%23}, [ta];\n"
-      "add.u32 ta, %64, 192;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%24,%25,%26,%27}, [ta];\n"
-      "add.u32 ta, %64, 224;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%28,%29,%30,%31}, [ta];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [ta];\n"
       "add.u32 ta, %64, 256;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%32,%33,%34,%35}, [ta];\n"
-      "add.u32 ta, %64, 288;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%36,%37,%38,%39}, [ta];\n"
-      "add.u32 ta, %64, 320;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%40,%41,%42,%43}, [ta];\n"
-      "add.u32 ta, %64, 352;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%44,%45,%46,%47}, [ta];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47}, [ta];\n"
       "add.u32 ta, %64, 384;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%48,%49,%50,%51}, [ta];\n"
-      "add.u32 ta, %64, 416;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%52,%53,%54,%55}, [ta];\n"
-      "add.u32 ta, %64, 448;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%56,%57,%58,%59}, [ta];\n"
-      "add.u32 ta, %64, 480;\n"
-      "tcgen05.ld.sync.aligned.32x32b.x4.b32 {%60,%61,%62,%63}, [ta];\n"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [ta];\n"
       "bar.sync %65, 64;\n"
       "tcgen05.wait::ld.sync.aligned;\n"
       "}\n"
@@ -244,16 +197,23 @@ __device__ __forceinline__ void tmem_ld_2x32_waited(uint32_t col0, uint32_t col1
       : "memory");
 }
 
-// Four consecutive columns of the thread's TMEM lane from two fp32 pairs.
-__device__ __forceinline__ void tmem_st4(uint32_t taddr, uint64_t lo, uint64_t hi) {
+// Sixteen consecutive columns of the thread's TMEM lane from eight fp32 pairs.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint64_t (&v)[8]) {
   asm volatile(
       "{\n"
-      ".reg .b32 a0, a1, a2, a3;\n"
+      ".reg .b32 a<16>;\n"
       "mov.b64 {a0, a1}, %1;\n"
       "mov.b64 {a2, a3}, %2;\n"
-      "tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {a0, a1, a2, a3};\n"
+      "mov.b64 {a4, a5}, %3;\n"
+      "mov.b64 {a6, a7}, %4;\n"
+      "mov.b64 {a8, a9}, %5;\n"
+      "mov.b64 {a10, a11}, %6;\n"
+      "mov.b64 {a12, a13}, %7;\n"
+      "mov.b64 {a14, a15}, %8;\n"
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {a0, a1, a2, a3, a4, a5, a6, a7, a8, a9, a10, a11, a12, a13, "
+      "a14, a15};\n"
       "}\n" ::"r"(taddr),
-      "l"(lo), "l"(hi)
+      "l"(v[0]), "l"(v[1]), "l"(v[2]), "l"(v[3]), "l"(v[4]), "l"(v[5]), "l"(v[6]), "l"(v[7])
       : "memory");
 }
 
@@ -318,68 +278,77 @@ __device__ __forceinline__ uint32_t pack8(const uint32_t* u) {
   return __byte_perm(__byte_perm(b0, b1, 0x0040), __byte_perm(b2, b3, 0x0040), 0x5410);
 }
 
-// The first sweep of a thread of half H, in 4 passes of 4 output channels a'
-// (columns col + 4 c + 32 b of its TMEM lane for the 16 groups b): per pass
-// the H_16 stages, the H_2 stage with the partner thread (through xw / xr, two
-// buffers alternating), and the results back in place: the thread keeps
-// groups 8 H .. 8 H + 7, output bit h = e of group 8 H + k lands in column slot
-// 8 (e ^ H) + k. The next pass's TMEM loads are issued before the pair barrier.
+// The first sweep of a thread of half H, in 4 passes of 16 output channels n
+// of the 4 chunks (columns col + 16 i + 128 c of its TMEM lane, pass i): per
+// pass the H_4 stages over the chunks, the H_2 stage with the partner thread
+// (through xw / xr, two buffers alternating), and the results back in place:
+// the thread keeps output chunks 2 H and 2 H + 1; output bit h = e of chunk
+// c' lands in chunk position c' for e = 0 and c' ^ 2 for e = 1. The next
+// pass's TMEM loads are issued before the pair barrier.
 template <int H>
 __device__ __forceinline__ void first_sweep(uint32_t col, uint32_t xw, uint32_t xr, int pair_bar, uint64_t x0x0,
                                             Extremes& ex) {
   uint32_t r[64];
-  tmem_ld_groups(col, r);
+  tmem_ld_chunks(col, r);
 #pragma unroll 1
-  for (int c = 0; c < 4; ++c) {
-    const uint32_t buf = (c & 1) * kXBufBytes;
-    uint64_t p[16][2];
+  for (int i = 0; i < 4; ++i) {
+    const uint32_t buf = (i & 1) * kXBufBytes;
+    uint64_t p[4][8];
 #pragma unroll
-    for (int b = 0; b < 16; ++b) {
-      p[b][0] = pack2(__uint_as_float(r[4 * b]), __uint_as_float(r[4 * b + 1]));
-      p[b][1] = pack2(__uint_as_float(r[4 * b + 2]), __uint_as_float(r[4 * b + 3]));
-    }
+    for (int c = 0; c < 4; ++c)
+#pragma unroll
+      for (int k = 0; k < 8; ++k) p[c][k] = pack2(__uint_as_float(r[16 * c + 2 * k]), __uint_as_float(r[16 * c + 2 * k + 1]));
     if (H == 0) {
-      // Group 0 of the first half holds the block's leading channel: every
-      // output of its H_32 includes x[0] once. Removing it is removing the
+      // Chunk 0 of the first half holds the block's leading channel: every
+      // output of its H_128 includes x[0] once. Removing it is removing the
       // offset (x0x0 is zero without OFFQ_OFFSET).
-      p[0][0] = sub2(p[0][0], x0x0);
-      p[0][1] = sub2(p[0][1], x0x0);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) p[0][k] = sub2(p[0][k], x0x0);
     }
 #pragma unroll
-    for (int d = 1; d < 16; d <<= 1) {
+    for (int d = 1; d < 4; d <<= 1) {
 #pragma unroll
-      for (int b = 0; b < 16; ++b) {
-        if ((b & d) == 0) {
+      for (int c = 0; c < 4; ++c) {
+        if ((c & d) == 0) {
 #pragma unroll
-          for (int k = 0; k < 2; ++k) {
-            const uint64_t u = p[b][k], v = p[b + d][k];
-            p[b][k] = add2(u, v);
-            p[b + d][k] = sub2(u, v);
+          for (int k = 0; k < 8; ++k) {
+            const uint64_t u = p[c][k], v = p[c + d][k];
+            p[c][k] = add2(u, v);
+            p[c + d][k] = sub2(u, v);
           }
         }
       }
     }
+    // Send chunks 2 (1 - H), 2 (1 - H) + 1: entry k of the buffer is chunk
+    // 2 (1 - H) + (k >> 2), pairs 2 (k & 3), 2 (k & 3) + 1.
 #pragma unroll
-    for (int k = 0; k < 8; ++k) sts_pair(xw + buf + k * 512, p[8 * (1 - H) + k][0], p[8 * (1 - H) + k][1]);
-    if (c < 3) {
-      tmem_ld_groups_pair_sync(col + 4 * (c + 1), pair_bar, r);
+    for (int k = 0; k < 8; ++k)
+      sts_pair(xw + buf + k * 512, p[2 * (1 - H) + (k >> 2)][2 * (k & 3)], p[2 * (1 - H) + (k >> 2)][2 * (k & 3) + 1]);
+    if (i < 3) {
+      tmem_ld_chunks_pair_sync(col + 16 * (i + 1), pair_bar, r);
     } else {
       bar_sync(pair_bar, 64);
     }
-    const uint32_t cc = col + 4 * c;
+    uint64_t sum[2][8], dif[2][8];
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
       uint64_t t0, t1;
       lds_pair(xr + buf + k * 512, t0, t1);
-      const uint64_t u0 = p[8 * H + k][0], u1 = p[8 * H + k][1];
+      const int c = 2 * H + (k >> 2), j = 2 * (k & 3);
+      const uint64_t u0 = p[c][j], u1 = p[c][j + 1];
       // Output bit 0 is (half 0) + (half 1), bit 1 is (half 0) - (half 1).
-      const uint64_t s0 = add2(u0, t0), s1 = add2(u1, t1);
-      const uint64_t d0 = H == 0 ? sub2(u0, t0) : sub2(t0, u0);
-      const uint64_t d1 = H == 0 ? sub2(u1, t1) : sub2(t1, u1);
-      tmem_st4(cc + 32 * (8 * H + k), s0, s1);
-      tmem_st4(cc + 32 * (8 * (1 - H) + k), d0, d1);
-      ex.add(s0, s1);
-      ex.add(d0, d1);
+      sum[k >> 2][j] = add2(u0, t0);
+      sum[k >> 2][j + 1] = add2(u1, t1);
+      dif[k >> 2][j] = H == 0 ? sub2(u0, t0) : sub2(t0, u0);
+      dif[k >> 2][j + 1] = H == 0 ? sub2(u1, t1) : sub2(t1, u1);
+      ex.add(sum[k >> 2][j], sum[k >> 2][j + 1]);
+      ex.add(dif[k >> 2][j], dif[k >> 2][j + 1]);
+    }
+    const uint32_t cc = col + 16 * i;
+#pragma unroll
+    for (int kk = 0; kk < 2; ++kk) {
+      tmem_st16(cc + 128 * (2 * H + kk), sum[kk]);
+      tmem_st16(cc + 128 * (2 * (1 - H) + kk), dif[kk]);
     }
   }
 }
@@ -414,21 +383,25 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (tid < kHalfRows) keys[tid] = 0ull;
   if (tid < 256) {
-    // B = H_32 (B[n][k] = (-1)^popcount(n & k)), K-major: row n is 128 bytes,
-    // 16-byte chunk c (channels 8c .. 8c + 7) at chunk c ^ (n & 7); chunks 4-7
-    // (channels 32-63) are zero and never read.
-    const int n = tid >> 3, pc = tid & 7, c = pc ^ (n & 7);
-    uint32_t w[4];
+    // B = H_128 (B[n][k] = (-1)^popcount(n & k)), K-major in two slabs of 64
+    // channels: row n of slab bs is 128 bytes, 16-byte chunk c (channels
+    // 64 bs + 8 c .. + 7) at chunk c ^ (n & 7).
+    const int n = tid >> 1, bs = tid & 1;
+#pragma unroll 1
+    for (int pc = 0; pc < 8; ++pc) {
+      const int c = pc ^ (n & 7);
+      uint32_t w[4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int k = 8 * c + 2 * i;
-      const uint32_t lo = (__popc(n & k) & 1) ? 0xBF80u : 0x3F80u;
-      const uint32_t hi = (__popc(n & (k + 1)) & 1) ? 0xBF80u : 0x3F80u;
-      w[i] = c < 4 ? (lo | (hi << 16)) : 0u;
+      for (int i = 0; i < 4; ++i) {
+        const int k = 64 * bs + 8 * c + 2 * i;
+        const uint32_t lo = (__popc(n & k) & 1) ? 0xBF80u : 0x3F80u;
+        const uint32_t hi = (__popc(n & (k + 1)) & 1) ? 0xBF80u : 0x3F80u;
+        w[i] = lo | (hi << 16);
+      }
+      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(b_s + bs * kBSlab + n * 128 + pc * 16),
+                   "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3])
+                   : "memory");
     }
-    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(b_s + n * 128 + pc * 16), "r"(w[0]), "r"(w[1]),
-                 "r"(w[2]), "r"(w[3])
-                 : "memory");
     fence_proxy_async_smem();
   }
   if (warp == kMmaWarp) {
@@ -479,24 +452,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool issued = false;
       for (int n = 0; n < n_local; ++n) {
         bool ok = true;
-        for (int s = 0; s < kSlabs; ++s) {
-          // Slab s writes column slots 2 s and 2 s + 1: each must have been read
-          // by the previous tile's second sweep.
-          if (!mbar_wait(full0 + 8 * s, n & 1, abort) ||
-              (n > 0 && (!mbar_wait(tempty0 + 16 * s, (n - 1) & 1, abort) ||
-                         !mbar_wait(tempty0 + 16 * s + 8, (n - 1) & 1, abort)))) {
-            ok = false;
-            break;
-          }
+        for (int c = 0; c < 4; ++c) {
+          // Chunk c (slabs 2 c, 2 c + 1) writes column slots 4 c .. 4 c + 3: each
+          // must have been read by the previous tile's second sweep.
+          ok = mbar_wait(full0 + 16 * c, n & 1, abort) && mbar_wait(full0 + 16 * c + 8, n & 1, abort);
+          for (int q = 4 * c; ok && n > 0 && q < 4 * c + 4; ++q) ok = mbar_wait(tempty0 + 8 * q, (n - 1) & 1, abort);
+          if (!ok) break;
           tc_fence_after();
 #pragma unroll
-          for (int g2 = 0; g2 < 2; ++g2)
-#pragma unroll
-            for (int kk = 0; kk < 2; ++kk)
-              mma_bf16(tmem + 32 * (2 * s + g2), smem_desc_sw128(a_s + s * kSlabBytes + 64 * g2 + 32 * kk),
-                       smem_desc_sw128(b_s + 32 * kk), kIdesc, kk);
+          for (int kk = 0; kk < 8; ++kk)
+            mma_bf16(tmem + 128 * c, smem_desc_sw128(a_s + (2 * c + (kk >> 2)) * kSlabBytes + 32 * (kk & 3)),
+                     smem_desc_sw128(b_s + (kk >> 2) * kBSlab + 32 * (kk & 3)), kIdesc, kk);
           issued = true;
-          mma_commit(empty0 + 8 * s);  // slab s may take the next tile
+          mma_commit(empty0 + 16 * c);  // slabs 2 c and 2 c + 1 may take the next tile
+          mma_commit(empty0 + 16 * c + 8);
         }
         if (!ok) break;
         mma_commit(tfull);
@@ -531,7 +500,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const uint64_t x0x0 = pack2(x0, x0);
       Extremes ex;
-      const uint32_t col = tl + 16 * wg;  // output channels a' = 16 wg .. 16 wg + 15
+      const uint32_t col = tl + 64 * wg;  // output channels n = 64 wg .. 64 wg + 63 of each chunk
       if (h == 0) {
         first_sweep<0>(col, xw, xr, pair_bar, x0x0, ex);
       } else {

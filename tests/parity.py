@@ -10,10 +10,11 @@ u = 2^-24), never from observed differences:
 * Scales and offsets. The kernel's transform is a radix-2 tree of L = log2(g)
   fp32 additions per output, so each rotated value carries an absolute error of
   at most L u sum|x| over its block; the scale inherits that relative to max|r|.
-  The tensor-core form of g = 1024 (bf16 rows) sums the first 32 terms of each
-  output in the MMA's fp32 accumulator: its products are exact, and allowing
-  each of the 32 additions a full ulp (truncation), plus the removal of x[0]
-  and the 5 register stages, the bound is TC_FACTOR u sum|x| over the block.
+  The tensor-core form of g = 1024 (bf16 rows) sums the first 128 terms of each
+  output (the H_128 factor) in the MMA's fp32 accumulator: its products are
+  exact, and allowing each of the 128 additions two ulps (truncation), plus the
+  removal of x[0] and the 3 register stages, the bound is TC_FACTOR u sum|x|
+  over the block.
   There a code may also differ within that bound (in code units) of a tie.
   Without the rotation the offset is an fp32 block sum whose summation depth
   is at most g/8 + 16.
@@ -31,7 +32,7 @@ import math
 import numpy as np
 
 U32 = 2.0 ** -24
-TC_FACTOR = 2 * 32 + 8 + 1 + 5 + 4
+TC_FACTOR = 2 * 128 + 8 + 1 + 3 + 4
 TIE_WINDOW = 1e-3
 MAX_MISMATCH_FRACTION = 1e-4
 
