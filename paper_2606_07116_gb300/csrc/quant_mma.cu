@@ -245,26 +245,24 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
   return r;
 }
 
-__device__ __forceinline__ float min3(float a, float b, float c) {
-  float r;
-  asm("min.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
-  return r;
-}
-
-// Running extremes of a thread's values, two independent chains each; the
-// absmax is max(hi, -lo) at the end.
-struct Extremes {
-  float hi0 = 0.f, hi1 = 0.f, lo0 = 0.f, lo1 = 0.f;
-  __device__ __forceinline__ void add(uint64_t u, uint64_t v) {
+// Running absmax of a thread's outputs, two independent chains. The outputs
+// come in pairs fl(u + t), fl(u - t) (the H_2 stage); rounding is symmetric
+// and monotone, so the larger magnitude of the two is exactly fl(|u| + |t|).
+struct AbsMax {
+  float m0 = 0.f, m1 = 0.f;
+  __device__ __forceinline__ void add_a(uint64_t u, uint64_t t) {
     float a, b, c, d;
     unpack2(u, a, b);
-    unpack2(v, c, d);
-    hi0 = max3(hi0, a, b);
-    lo0 = min3(lo0, a, b);
-    hi1 = max3(hi1, c, d);
-    lo1 = min3(lo1, c, d);
+    unpack2(t, c, d);
+    m0 = max3(m0, fabsf(a) + fabsf(c), fabsf(b) + fabsf(d));
   }
-  __device__ __forceinline__ float absmax() const { return fmaxf(fmaxf(hi0, hi1), -fminf(lo0, lo1)); }
+  __device__ __forceinline__ void add_b(uint64_t u, uint64_t t) {
+    float a, b, c, d;
+    unpack2(u, a, b);
+    unpack2(t, c, d);
+    m1 = max3(m1, fabsf(a) + fabsf(c), fabsf(b) + fabsf(d));
+  }
+  __device__ __forceinline__ float value() const { return fmaxf(m0, m1); }
 };
 
 // fl(x * inv + 1.5 * 2^23 + 8) has rne(x * inv) + 8 in its low mantissa bits
@@ -287,7 +285,7 @@ __device__ __forceinline__ uint32_t pack8(const uint32_t* u) {
 // pass's TMEM loads are issued before the pair barrier.
 template <int H>
 __device__ __forceinline__ void first_sweep(uint32_t col, uint32_t xw, uint32_t xr, int pair_bar, uint64_t x0x0,
-                                            Extremes& ex) {
+                                            AbsMax& am) {
   uint32_t r[64];
   tmem_ld_chunks(col, r);
 #pragma unroll 1
@@ -341,8 +339,8 @@ __device__ __forceinline__ void first_sweep(uint32_t col, uint32_t xw, uint32_t 
       sum[k >> 2][j + 1] = add2(u1, t1);
       dif[k >> 2][j] = H == 0 ? sub2(u0, t0) : sub2(t0, u0);
       dif[k >> 2][j + 1] = H == 0 ? sub2(u1, t1) : sub2(t1, u1);
-      ex.add(sum[k >> 2][j], sum[k >> 2][j + 1]);
-      ex.add(dif[k >> 2][j], dif[k >> 2][j + 1]);
+      am.add_a(u0, t0);
+      am.add_b(u1, t1);
     }
     const uint32_t cc = col + 16 * i;
 #pragma unroll
@@ -499,14 +497,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (bar_any(kBarVote, 32 * kRegWarps, !waited)) break;
       tc_fence_after();
       const uint64_t x0x0 = pack2(x0, x0);
-      Extremes ex;
+      AbsMax am;
       const uint32_t col = tl + 64 * wg;  // output channels n = 64 wg .. 64 wg + 63 of each chunk
       if (h == 0) {
-        first_sweep<0>(col, xw, xr, pair_bar, x0x0, ex);
+        first_sweep<0>(col, xw, xr, pair_bar, x0x0, am);
       } else {
-        first_sweep<1>(col, xw, xr, pair_bar, x0x0, ex);
+        first_sweep<1>(col, xw, xr, pair_bar, x0x0, am);
       }
-      const float m = ex.absmax();
+      const float m = am.value();
       tmem_st_wait();
       // Row absmax: per row of this warp a warp maximum (non-negative floats
       // order as their bits), then a 64-bit atomic max keyed by the tile
