@@ -134,6 +134,15 @@ enum {
  *   scale   device, [T] float32.
  *   offset  device, [T][K/g] float32; required with OFFQ_OFFSET; when given
  *           without OFFQ_OFFSET it is filled with zeros; may be NULL otherwise.
+ *
+ * Arithmetic: fp32 throughout; the rounding decisions are taken in fp32. The
+ * rotation is a radix-2 tree of fp32 additions, except for bf16 rows with
+ * g = 1024 and OFFQ_ROTATE when ceil(T / floor(65536 / K)) (tiles of up to
+ * 64 blocks of whole tokens) is at least the SM count: those take the tensor cores
+ * for a 128-point factor of the Hadamard (exact bf16 x +-1 products summed in
+ * the MMA's fp32 accumulator), with the remaining three factors in fp32. The
+ * two forms agree within their fp32 error bounds, not bit for bit, so a code
+ * near a rounding tie may differ between them.
  */
 int offq_quantize_act(const void* x, int x_dtype, int64_t T, int64_t K, int64_t ldx,
                       int32_t g, int32_t flags,
