@@ -1,5 +1,5 @@
 // The g = 1024 rotating activation quantizer (offq_quantize_act, bf16 rows of
-// one head) with the first half of the transform on the tensor cores.
+// one head) with a 128-point factor of the transform on the tensor cores.
 //
 // Per row and block of 1024 channels (paper Sec. 3.2, Eq. 4-5; Sec. 3 Eq. 1):
 // R = x H_1024 / 32 - o with o = x[0] / 32, s = max|R| / 7 over the row,
@@ -8,38 +8,40 @@
 // from the transform's input removes the offset) and 1/32 goes only into the
 // stored scale and offset.
 //
-// The Sylvester matrix factors over channel bits, H_1024 = H_2 (x) H_16 (x) H_32
-// for channel c = 512 h + 32 b + a (h: half block, b: 32-channel group of the
-// half, a: channel in the group):
-//  * bits a (H_32) on the tensor cores: tcgen05.mma kind::f16, A = the bf16
-//    rows, B = H_32 (entries +-1, exact in bf16), so every product is exact
-//    and the accumulator holds the fp32 sum of 32 of them. The A tile has
+// The Sylvester matrix factors over channel bits, H_1024 = H_2 (x) H_4 (x) H_128
+// for channel c = 512 h + 128 c + a (h: half block, c: 128-channel chunk of
+// the half, a: channel in the chunk):
+//  * bits a (H_128) on the tensor cores: tcgen05.mma kind::f16, A = the bf16
+//    rows, B = H_128 (entries +-1, exact in bf16), so every product is exact
+//    and the accumulator holds the fp32 sum of 128 of them. The A tile has
 //    128 rows, (h, token, block) for 64 (token, block) pairs: row
 //    64 h + t G + j holds channels 512 h .. 512 h + 511 of block j of the
 //    tile's token t, loaded by TMA from a 4-D view [T][G][2][512] of the
-//    activations (128-byte swizzle, 64-channel slabs). One MMA of N = 32 per
-//    group b and 16 channels of K writes columns 32 b .. 32 b + 31 of TMEM
-//    lane (h, t, j): all 512 columns hold the tile.
-//  * bits b (H_16) in registers: a thread owns one TMEM lane and, per pass,
-//    2 output channels a' of all 16 groups (16 loads of 2 columns), and runs
-//    4 butterfly stages on fp32x2 pairs.
+//    activations (128-byte swizzle, 64-channel slabs). Per chunk c, MMAs of
+//    N = 128 write columns 128 c .. 128 c + 127 of TMEM lane (h, t, j): the
+//    tile fills all 512 columns.
+//  * bits c (H_4) in registers: a thread owns one TMEM lane and, per pass,
+//    16 output channels n of the 4 chunks (4 loads of 16 columns), and runs
+//    2 butterfly stages on fp32x2 pairs.
 //  * bit h (H_2) between the two lanes of a (token, block): threads h = 0 and
 //    1 (warps w and w ^ 2, same lane) swap half their values through shared
-//    memory; each forms both outputs of 8 groups and writes them back to its
-//    TMEM columns.
-// The row's absmax goes through shared memory (a per-warp maximum per row,
-// then a 64-bit atomic max keyed by the tile), and a second sweep reads 32
-// output channels per TMEM load, rounds them (magic-number rounding) and
-// writes one 16-byte chunk of codes.
+//    memory; each forms both outputs of 2 chunks and writes them back to its
+//    TMEM columns. The larger magnitude of each output pair is fl(|u| + |t|)
+//    of its inputs, which gives the row's absmax.
+// The absmax goes through shared memory (a per-warp maximum per row, then a
+// 64-bit atomic max keyed by the tile), and a second sweep reads 32 output
+// channels per TMEM load, rounds them (magic-number rounding) and writes one
+// 16-byte chunk of codes. Each 32-column slot is handed to the next tile's
+// MMAs as soon as it has been read.
 //
-// Roles (576 threads, one CTA per SM, persistent over tiles):
-//   warp 16    TMA producer: per tile, 8 slabs of both halves; slab s of the
-//              next tile is loaded as soon as the MMAs have read slab s;
-//   warp 17    allocates TMEM (512 columns) and issues the MMAs;
-//   warps 0-15 the register work, four warps per TMEM lane quarter (warps
-//              w, w + 4, w + 8, w + 12): warp w takes output channels a' in
-//              8 (w / 4) .. 8 (w / 4) + 7 in the first sweep and column slots
-//              4 (w / 4) .. 4 (w / 4) + 3 in the second.
+// Roles (320 threads, one CTA per SM, persistent over tiles):
+//   warp 8    TMA producer: per tile, 8 slabs of both halves; slab s of the
+//             next tile is loaded as soon as the MMAs have read slab s;
+//   warp 9    allocates TMEM (512 columns) and issues the MMAs;
+//   warps 0-7 the register work, two warps per TMEM lane quarter (warps w and
+//             w + 4): warp w takes output channels n in 64 (w / 4) ..
+//             64 (w / 4) + 63 of every chunk in the first sweep and column
+//             slots 8 (w / 4) .. 8 (w / 4) + 7 in the second.
 // Every wait is bounded; a wait that runs out marks the CTA aborted, the
 // copies and MMAs in flight are waited for (bounded) and TMEM is released.
 #include <cuda_bf16.h>
@@ -63,7 +65,7 @@ constexpr int kABytes = kSlabs * kSlabBytes;         // 128 KB
 constexpr int kBSlab = 128 * 128;                    // H_128, channels 64 k .. 64 k + 63 of its 128 rows
 constexpr int kBBytes = 2 * kBSlab;
 constexpr int kRegWarps = 8;                         // two per TMEM lane quarter
-constexpr int kXWarpBytes = 8 * 32 * 16;             // a warp's exchange area: 8 groups x 32 lanes x 16 B
+constexpr int kXWarpBytes = 8 * 32 * 16;             // a warp's exchange area: 8 entries x 32 lanes x 16 B
 constexpr int kXBufBytes = kRegWarps * kXWarpBytes;
 constexpr int kXBytes = 2 * kXBufBytes;              // two buffers, alternating passes
 constexpr int kCtrlOff = kABytes + kBBytes + kXBytes;
