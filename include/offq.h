@@ -576,11 +576,13 @@ int offq_get_device_status(void* stream);
  * SM clock cycles of the bounded waits with which the persistent row
  * quantizers (offq_quantize_act and offq_kv4_quantize on inputs with more row
  * groups than SMs, and the shared-memory ring kernel of rotation-free
- * single-block rows) wait for the rows they stage by bulk copies. A budget
- * shorter than the default makes those waits behave as waits for a flag that
- * nothing sets: they do not look at their barrier and give up after about
- * that many cycles. The kernel then lets every copy already in flight land
- * (waiting for it with the full budget), returns without writing the rest of
+ * single-block rows) wait for the rows they stage by bulk copies, and with
+ * which the tensor-core form of offq_quantize_act (bf16, g = 1024) waits for
+ * each tile's MMAs. A budget shorter than the default makes those waits
+ * behave as waits for a flag that nothing sets: they do not look at their
+ * barrier and give up after about that many cycles. The kernel then lets
+ * every copy and MMA already in flight complete (waiting for it with the full
+ * budget), releases its tensor memory, returns without writing the rest of
  * its outputs, and records OFFQ_ERR_TIMEOUT for offq_get_device_status.
  * 0 restores the default (about 2 s), and with it the normal waits. Returns
  * OFFQ_ERR_INVALID_ARG for a negative value. The setting is process-wide and
