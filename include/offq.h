@@ -95,7 +95,7 @@ extern "C" {
 typedef enum {
   OFFQ_OK = 0,
   OFFQ_ERR_INVALID_ARG = -1,  /* shape, flag or NULL pointer not allowed   */
-  OFFQ_ERR_UNSUPPORTED = -2,  /* valid request this build does not handle  */
+  OFFQ_ERR_UNSUPPORTED = -2,  /* valid request the library does not handle */
   OFFQ_ERR_MISALIGNED = -3,   /* pointer / leading dimension alignment     */
   OFFQ_ERR_CUDA = -4,         /* a CUDA runtime call failed                */
   OFFQ_ERR_TIMEOUT = -5       /* a device-side bounded wait ran out        */
@@ -263,7 +263,7 @@ int offq_prepare_weight(const void* w, int dtype, int64_t N, int64_t K, int32_t 
  *           K <= 65536.
  *   g       rotation block, power of two in [32, 8192]; ignored without
  *           OFFQ_ROTATE.
- *   group   channels per quantization group; this build supports 128
+ *   group   channels per quantization group; this library supports 128
  *           (OFFQ_ERR_UNSUPPORTED for other positive values).
  *   flags   0 or OFFQ_ROTATE.
  *   codes   device, offq_act_codes_bytes(T, K) bytes: u as the nibble, two per
@@ -301,7 +301,7 @@ int offq_weight_group_sums(const uint8_t* w_codes, int64_t N, int64_t K, int32_t
  *
  *   a_codes, a_scale, a_zero  from offq_quantize_act_group (T rows, K channels).
  *   T, N, K     T >= 0, N >= 1, K a multiple of group, K <= 65536.
- *   group       128 in this build (OFFQ_ERR_UNSUPPORTED otherwise).
+ *   group       128 in this library (OFFQ_ERR_UNSUPPORTED otherwise).
  *   w_codes, w_scale          from offq_prepare_weight (any rotation block).
  *   w_groupsum  from offq_weight_group_sums with the same group.
  *   out         device, [T][ldo] of out_dtype, ldo >= N, 16-byte aligned with
@@ -331,7 +331,7 @@ int offq_w4a4_linear_group(const uint8_t* a_codes, const float* a_scale, const f
  *             16-byte aligned, ld_token * sizeof(elem) a multiple of 16,
  *             ld_token >= H * head_dim.
  *   T, H      tokens (>= 0) and heads (1..65535).
- *   head_dim  128 in this build (OFFQ_ERR_UNSUPPORTED otherwise).
+ *   head_dim  128 in this library (OFFQ_ERR_UNSUPPORTED otherwise).
  *   rot       device, [H][head_dim][head_dim] float32, row-major (y_j =
  *             sum_i x_i rot[h][i][j]), 16-byte aligned. It is orthonormal
  *             in the method; the call does not check that.
@@ -365,7 +365,7 @@ int offq_rotate_heads(const void* x, int dtype, int64_t T, int32_t H, int32_t he
  * instead of splitting M in every CTA.
  *
  *   rot       device, as in offq_kv4_quantize_rotated.
- *   H         heads (1..65535).   head_dim  128 in this build.
+ *   H         heads (1..65535).   head_dim  128 in this library.
  *   prepared  device, H * OFFQ_KEY_ROTATION_BYTES bytes, 16-byte aligned,
  *             written. An opaque image: head h's bytes start at
  *             h * OFFQ_KEY_ROTATION_BYTES; part s (0..2) of it is 128 rows
@@ -467,7 +467,7 @@ int offq_top1_direction(const float* X, int64_t N, int64_t D, int32_t iters, con
  * w = v/|v| - e_1: the symmetric reflection with U1 e_1 = v/|v|, so x U1
  * carries x . v/|v| in channel 0 (the concentrated outlier channel).
  *   A, out  device, [R][D] float32 (may not overlap).  v  device, [D] float32.
- *   D <= 16384 in this build.
+ *   D <= 16384 in this library.
  */
 int offq_reflect_rows(const float* A, int64_t R, int64_t D, const float* v, float* out, void* stream);
 
@@ -492,7 +492,7 @@ int offq_sorted_grouping(const float* mag, int64_t D, int32_t G, int32_t* perm);
  * column c = old column perm[c]); H_g Sylvester.
  *   W, out  device, [N][D] float32 (may not overlap).  v device [D] float32.
  *   perm    device, [D] int32 permutation.   g  power of two dividing D.
- *   D <= 16384 in this build.
+ *   D <= 16384 in this library.
  */
 int offq_fuse_rotation(const float* W, int64_t N, int64_t D, const float* v, const int32_t* perm, int32_t g,
                        float* out, void* stream);

@@ -690,7 +690,7 @@ def effective_bits_per_token_offset(K: int, g: int, code_bits: int = 4, param_bi
 # MXFP4 activations and weights with the offset as zero-point
 # (Sec. 3.4 "Generality on Data Formats": micro-scaling formats extended with
 # a zero-point absorb the outlier the same way; the paper leaves it to future
-# work, so the readings below are this build's)
+# work, so the readings below are this implementation's own)
 # ---------------------------------------------------------------------------
 #
 # Element format: MXFP4's E2M1 (OCP Microscaling Formats v1.0): sign, 2-bit

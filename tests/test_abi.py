@@ -157,7 +157,7 @@ def test_mx_argument_checks(lib):
 def test_group_path_argument_checks(lib):
     qg = lambda x=A16, dt=Q.OFFQ_BF16, T=4, K=1024, ldx=1024, g=256, group=128, flags=1, c=A16, s=A16, z=A16: \
         lib.offq_quantize_act_group(x, dt, T, K, ldx, g, group, flags, c, s, z, None)
-    assert qg(group=64) == Q.OFFQ_ERR_UNSUPPORTED          # this build quantizes groups of 128
+    assert qg(group=64) == Q.OFFQ_ERR_UNSUPPORTED          # the library quantizes groups of 128
     assert qg(group=0) == Q.OFFQ_ERR_INVALID_ARG
     assert qg(K=1000, ldx=1000) == Q.OFFQ_ERR_INVALID_ARG  # group does not divide K
     assert qg(g=100) == Q.OFFQ_ERR_INVALID_ARG             # rotation block not a power of two
@@ -191,7 +191,7 @@ def test_group_path_argument_checks(lib):
 def test_rotated_key_cache_argument_checks(lib):
     kq = lambda kv=A16, dt=Q.OFFQ_BF16, T=4, H=8, hd=128, ld=1024, rot=A16, flags=2, c=A16, s=A16, o=A16: \
         lib.offq_kv4_quantize_rotated(kv, dt, T, H, hd, ld, rot, flags, c, s, o, None)
-    assert kq(hd=64, ld=512) == Q.OFFQ_ERR_UNSUPPORTED     # this build rotates heads of 128
+    assert kq(hd=64, ld=512) == Q.OFFQ_ERR_UNSUPPORTED     # the library rotates heads of 128
     assert kq(H=0) == Q.OFFQ_ERR_INVALID_ARG
     assert kq(ld=512) == Q.OFFQ_ERR_INVALID_ARG            # ld_token < H * head_dim
     assert kq(flags=1) == Q.OFFQ_ERR_INVALID_ARG           # the rotation is M, not a flag
