@@ -12,6 +12,8 @@ them.
   and bits 4-21 of its pattern are zero.
 * The 4-bit integer operands of the GEMM: the bytes 0x00..0x0F read as E4M3
   are exactly 0, 1, ..., 15 times 2^-9 (subnormals up to 7, then exponent 1).
+* The tensor-core quantizer's derived error bound stays a tight tie window on
+  the inputs it serves.
 """
 
 import numpy as np
@@ -74,3 +76,19 @@ def test_small_integers_are_exact_e4m3_subnormals():
         # The weights' sign-magnitude bytes: bit 7 is the sign of the same value.
         if k < 8:
             assert e4m3(0x80 | k) == -k * 2.0 ** -9
+
+
+def test_tensor_core_bound_keeps_the_tie_window_tight():
+    """The tensor-core quantizer's error bound (TC_FACTOR u sum|x| per block) in code
+    units, on the prefill recipes it serves (Llama-2-70B and Llama-3-8B down-proj
+    inputs): a code may differ from the oracle's only within that window of a
+    rounding tie, so the bound must stay far below half a code step."""
+    import oracle as O
+    import workloads as W
+    from parity import code_window
+
+    for K, dist, n_out, mult in [(28672, "normal", 6, 200.0), (14336, "student_t3", 3, 100.0)]:
+        x = W.activations(16, K, seed=5, dist=dist, n_out=n_out, mult=mult).astype(np.float64)
+        ref = O.quantize_act(x, 1024, rotate=True, offset=True)
+        w = code_window(ref["scale"], x, 1024, tc=True)
+        assert np.all(w < 2e-3), (K, float(w.max()))
